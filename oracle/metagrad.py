@@ -1,0 +1,172 @@
+"""Oracle meta-gradient: Algorithm 1 (standard Truncated-BPTT) in float64 on the CPU.
+
+Test infrastructure only (see ``oracle/__init__.py``).
+
+Inner loop (Eq. 2 with the momentum state as the optimiser state upsilon):
+    m_{t+1}     = mu * m_t + grad L_t(theta_t),      m_0 = 0
+    theta_{t+1} = theta_t - lr (*) m_{t+1}
+with lr = alpha, or exp(eta_lr) per parameter, or exp(eta_s) for a scalar log-lr, and
+L_t = (1/B) sum_b sigmoid(eta_{t,b}) l_b when per-example weight logits are meta-parameters.
+Outer loss V(theta_T) is the unweighted mean loss on the held-out batch.
+
+``meta_grad`` differentiates V through the unrolled loop by reverse mode at both levels
+(Algorithm 1): the inner gradient is recorded with ``create_graph`` so that the outer
+backward pass runs reverse-over-reverse through it.  Per-inner-step checkpointing
+(Section 4): the rollout keeps (theta_t, m_t); the backward sweep rebuilds the tape of one
+step at a time and pulls the cotangent (theta_bar_{t+1}, m_bar_{t+1}) through it.
+
+Index convention (the algorithm listings mix 0- and 1-based ranges): steps t = 0..T-1, and
+the weight logits eta_{t,.} act at step t.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import model
+
+F64 = torch.float64
+EXAMPLE_WEIGHTS, PARAM_LOGLR, SCALAR_LOGLR = 1, 2, 4
+
+
+def t64(a) -> torch.Tensor:
+    if isinstance(a, torch.Tensor):
+        return a.detach().to(F64) if a.is_floating_point() else a.detach()
+    a = np.asarray(a)
+    if a.dtype.kind in "iu":
+        return torch.from_numpy(a.astype(np.int64))
+    return torch.from_numpy(a.astype(np.float64))
+
+
+def split_eta(w, eta: torch.Tensor):
+    """Split the flat meta-parameter vector: [T*B example logits][P log-lrs][1 scalar log-lr]."""
+    o, ex, plr, slr = 0, None, None, None
+    if w.meta_kind & EXAMPLE_WEIGHTS:
+        ex = eta[o:o + w.T * w.B].reshape(w.T, w.B)
+        o += w.T * w.B
+    if w.meta_kind & PARAM_LOGLR:
+        plr = eta[o:o + w.n_params]
+        o += w.n_params
+    if w.meta_kind & SCALAR_LOGLR:
+        slr = eta[o]
+        o += 1
+    return ex, plr, slr
+
+
+def learning_rate(w, eta: torch.Tensor):
+    _, plr, slr = split_eta(w, eta)
+    if plr is not None:
+        return torch.exp(plr)
+    if slr is not None:
+        return torch.exp(slr)
+    return torch.tensor(w.alpha, dtype=F64)
+
+
+def example_weights(w, eta: torch.Tensor, t: int):
+    ex, _, _ = split_eta(w, eta)
+    if ex is None:
+        return torch.ones(w.B, dtype=F64)
+    return torch.sigmoid(ex[t])
+
+
+def _step(w, theta, m, eta, x, y, t, create_graph):
+    """One inner update Phi(theta_t, m_t, eta, x_t) -> (theta_{t+1}, m_{t+1})."""
+    L = model.weighted_inner_loss(w, theta, x, y, example_weights(w, eta, t))
+    (g,) = torch.autograd.grad(L, theta, create_graph=create_graph)
+    m_next = w.momentum * m + g
+    theta_next = theta - learning_rate(w, eta) * m_next
+    return theta_next, m_next
+
+
+def rollout(w, inp, eta=None):
+    """Inner rollout storing every (theta_t, m_t), t = 0..T.  Returns (thetas, ms)."""
+    eta = t64(inp.eta if eta is None else eta)
+    X, Y = t64(inp.inner_x), t64(inp.inner_y)
+    theta = t64(inp.theta0)
+    m = torch.zeros_like(theta)
+    thetas, ms = [theta], [m]
+    for t in range(w.T):
+        th = theta.clone().requires_grad_(True)
+        with torch.enable_grad():
+            tn, mn = _step(w, th, m, eta, X[t], Y[t], t, create_graph=False)
+        theta, m = tn.detach(), mn.detach()
+        thetas.append(theta)
+        ms.append(m)
+    return thetas, ms
+
+
+def value(w, inp, eta=None) -> float:
+    """V(theta_T(eta)): the outer loss after the unrolled inner loop (first-order only)."""
+    thetas, _ = rollout(w, inp, eta)
+    return float(model.outer_loss(w, thetas[-1], t64(inp.outer_x), t64(inp.outer_y)))
+
+
+def meta_grad(w, inp, eta=None):
+    """dV/d eta, dV/d theta_0 and V by Algorithm 1 with per-step checkpointing.
+
+    Returns a dict with numpy float64 arrays 'd_eta' [n_eta], 'd_theta0' [P] and float 'V'.
+    """
+    eta0 = t64(inp.eta if eta is None else eta)
+    X, Y = t64(inp.inner_x), t64(inp.inner_y)
+    thetas, ms = rollout(w, inp, eta0)
+    # Outer gradient (Eq. 4): cotangent (dV/d theta_T, 0) on (theta_T, m_T).
+    thT = thetas[-1].clone().requires_grad_(True)
+    with torch.enable_grad():
+        V = model.outer_loss(w, thT, t64(inp.outer_x), t64(inp.outer_y))
+        (theta_bar,) = torch.autograd.grad(V, thT)
+    m_bar = torch.zeros_like(theta_bar)
+    d_eta = torch.zeros_like(eta0)
+    for t in range(w.T - 1, -1, -1):
+        th = thetas[t].clone().requires_grad_(True)
+        m = ms[t].clone().requires_grad_(True)
+        et = eta0.clone().requires_grad_(True)
+        with torch.enable_grad():
+            tn, mn = _step(w, th, m, et, X[t], Y[t], t, create_graph=True)
+            gt, gm, ge = torch.autograd.grad((tn, mn), (th, m, et), (theta_bar, m_bar),
+                                             allow_unused=True)
+        theta_bar = gt
+        m_bar = gm if gm is not None else torch.zeros_like(m_bar)
+        if ge is not None:
+            d_eta = d_eta + ge
+    return {"d_eta": d_eta.numpy(), "d_theta0": theta_bar.numpy(), "V": float(V.detach())}
+
+
+def grad(w, theta, x, y, weights=None):
+    """grad_theta L with L = (1/B) sum_b weights_b l_b (weights default to 1)."""
+    th = t64(theta).clone().requires_grad_(True)
+    x, y = t64(x), t64(y)
+    wt = torch.ones(x.shape[0], dtype=F64) if weights is None else t64(weights)
+    with torch.enable_grad():
+        L = model.weighted_inner_loss(w, th, x, y, wt)
+        (g,) = torch.autograd.grad(L, th)
+    return g.numpy()
+
+
+def hvp(w, theta, x, y, v, weights=None):
+    """H v with H = d^2 L / d theta^2, by reverse-over-reverse (grad of <grad L, v>)."""
+    th = t64(theta).clone().requires_grad_(True)
+    x, y, v = t64(x), t64(y), t64(v)
+    wt = torch.ones(x.shape[0], dtype=F64) if weights is None else t64(weights)
+    with torch.enable_grad():
+        L = model.weighted_inner_loss(w, th, x, y, wt)
+        (g,) = torch.autograd.grad(L, th, create_graph=True)
+        (hv,) = torch.autograd.grad((g * v).sum(), th)
+    return hv.numpy()
+
+
+def tangent_losses(w, theta, x, y, v):
+    """Per-example directional derivatives dl_b/d theta . v (the mixed term of Eq. 7 for
+    per-example weights), via the transpose of the per-example-loss VJP."""
+    th = t64(theta).clone().requires_grad_(True)
+    x, y, v = t64(x), t64(y), t64(v)
+    c = torch.zeros(x.shape[0], dtype=F64, requires_grad=True)
+    with torch.enable_grad():
+        l = model.losses(w, th, x, y)
+        (jtc,) = torch.autograd.grad(l, th, c, create_graph=True)
+        (ldot,) = torch.autograd.grad((jtc * v).sum(), c)
+    return ldot.numpy()
+
+
+def per_example_losses(w, theta, x, y):
+    with torch.no_grad():
+        return model.losses(w, t64(theta), t64(x), t64(y)).numpy()

@@ -1,0 +1,201 @@
+"""Seeded synthetic workloads for the Truncated-BPTT meta-gradient (shared input recipe).
+
+This module is the only code shared by the CPU oracle and the CUDA path.  It holds the
+workload shapes and draws their inputs; it contains none of the meta-gradient arithmetic
+(no loss, no gradient, no update rule).  The one model evaluation in here is the random
+*teacher* network that labels regression inputs, i.e. data generation.
+
+Every random array comes from ``numpy.random.Generator(PCG64(SeedSequence([seed, k])))``
+with a fixed stream index ``k`` per role, so the oracle and the GPU path see bit-identical
+inputs.  Values that the bf16 path consumes are rounded to bf16 (round-to-nearest-even)
+here, once, and handed to both sides as float32 arrays holding bf16-representable values.
+
+Workloads (problem statement: bilevel problem of Eq. 1 unrolled as Eq. 2; meta-parameters
+as in the loss-weighting and learned-learning-rate tasks of Section 5):
+
+* ``tiny``  - 16->32->1 tanh MLP, squared loss, B=8, T=4 SGD steps, alpha=0.1, per-example
+  weight logits, fp32.
+* ``wide``  - 1024-wide 4-hidden-layer GELU MLP with a 10-class softmax head, B=256, T=16,
+  alpha=0.05, per-example weight logits, outer batch 1024, bf16 GEMMs.
+* ``deep``  - 8 Linear 4096->4096 layers (SiLU after the first 7), regression onto a random
+  teacher, per-parameter log learning rates, SGD with momentum 0.9, B=512, T=32, bf16 GEMMs.
+"""
+from __future__ import annotations
+
+import copy
+import math
+from dataclasses import dataclass, field, replace
+from typing import Optional
+
+import numpy as np
+
+# Stream indices (one per role).  Changing one changes every stored expected value.
+_STREAMS = {"x": 1, "teacher": 2, "noise": 3, "theta0": 4, "eta": 5, "outer": 6,
+            "tokens": 7, "labels": 8, "outer_noise": 9, "outer_labels": 10, "dir": 11}
+
+
+def rng(seed: int, stream: str) -> np.random.Generator:
+    return np.random.Generator(np.random.PCG64(np.random.SeedSequence([seed, _STREAMS[stream]])))
+
+
+def round_bf16(a: np.ndarray) -> np.ndarray:
+    """Round float values to the nearest bf16 (ties to even); returned as float32."""
+    f = np.ascontiguousarray(a, dtype=np.float32)
+    u = f.view(np.uint32).astype(np.uint64)
+    u = (u + 0x7FFF + ((u >> 16) & 1)) & 0xFFFF0000
+    return u.astype(np.uint32).view(np.float32)
+
+
+# meta-parameter kinds (bit mask, same values as the C header)
+EXAMPLE_WEIGHTS = 1
+PARAM_LOGLR = 2
+SCALAR_LOGLR = 4
+
+
+@dataclass
+class Workload:
+    name: str
+    dims: list                      # MLP layer widths [d_in, h1, ..., d_out]
+    act: str                        # hidden activation: ident|tanh|gelu|silu
+    loss: str                       # squared | ce
+    precision: str                  # fp32 | bf16
+    B: int
+    T: int
+    B_outer: int
+    alpha: float = 0.0              # constant lr (when no log-lr meta-parameter)
+    momentum: float = 0.0
+    meta_kind: int = EXAMPLE_WEIGHTS
+    loglr_mean: float = 0.0
+    loglr_std: float = 0.0
+    eta_std: float = 1.0            # example-logit std
+    noise_std: float = 0.0          # regression-target noise std
+    seed: int = 0
+    has_bias: bool = True
+    extra: dict = field(default_factory=dict)
+
+    @property
+    def n_layers(self) -> int:
+        return len(self.dims) - 1
+
+    @property
+    def n_params(self) -> int:
+        return sum(self.dims[i] * self.dims[i + 1] + (self.dims[i + 1] if self.has_bias else 0)
+                   for i in range(self.n_layers))
+
+    @property
+    def n_eta(self) -> int:
+        n = 0
+        if self.meta_kind & EXAMPLE_WEIGHTS:
+            n += self.T * self.B
+        if self.meta_kind & PARAM_LOGLR:
+            n += self.n_params
+        if self.meta_kind & SCALAR_LOGLR:
+            n += 1
+        return n
+
+    def layer_offsets(self):
+        """(W offset, b offset) of each layer in the flat parameter vector.
+
+        Layout: for each layer l, W_l as [d_l][d_{l+1}] row-major, then b_l [d_{l+1}].
+        """
+        offs, o = [], 0
+        for i in range(self.n_layers):
+            din, dout = self.dims[i], self.dims[i + 1]
+            ow = o
+            o += din * dout
+            ob = o if self.has_bias else -1
+            if self.has_bias:
+                o += dout
+            offs.append((ow, ob))
+        return offs
+
+    def with_(self, **kw) -> "Workload":
+        return replace(copy.deepcopy(self), **kw)
+
+
+WORKLOADS = {
+    "tiny": Workload("tiny", [16, 32, 1], "tanh", "squared", "fp32", B=8, T=4, B_outer=8,
+                     alpha=0.1, noise_std=0.1),
+    "wide": Workload("wide", [1024] * 5 + [10], "gelu", "ce", "bf16", B=256, T=16,
+                     B_outer=1024, alpha=0.05),
+    "deep": Workload("deep", [4096] * 9, "silu", "squared", "bf16", B=512, T=32,
+                     B_outer=512, momentum=0.9, meta_kind=PARAM_LOGLR,
+                     loglr_mean=math.log(1e-2), loglr_std=0.1),
+}
+
+
+def glorot_params(w: Workload, g: np.random.Generator) -> np.ndarray:
+    """Glorot-uniform weights, zero biases, in the flat layout of ``layer_offsets``."""
+    theta = np.zeros(w.n_params, dtype=np.float64)
+    for i, (ow, ob) in enumerate(w.layer_offsets()):
+        din, dout = w.dims[i], w.dims[i + 1]
+        lim = math.sqrt(6.0 / (din + dout))
+        theta[ow:ow + din * dout] = g.uniform(-lim, lim, size=din * dout)
+    return theta.astype(np.float32)
+
+
+def _teacher_outputs(w: Workload, x: np.ndarray) -> np.ndarray:
+    """Labels for regression workloads: a Glorot-initialised copy of the architecture
+    (own stream) evaluated in float32.  Data generation only."""
+    tw = glorot_params(w, rng(w.seed, "teacher"))
+    h = x.astype(np.float32)
+    for i, (ow, ob) in enumerate(w.layer_offsets()):
+        din, dout = w.dims[i], w.dims[i + 1]
+        W = tw[ow:ow + din * dout].reshape(din, dout)
+        h = h @ W
+        if ob >= 0:
+            h = h + tw[ob:ob + dout]
+        if i + 1 < w.n_layers:
+            if w.act == "tanh":
+                h = np.tanh(h)
+            elif w.act == "gelu":
+                from scipy.special import erf
+                h = (0.5 * h * (1.0 + erf(h / math.sqrt(2.0)))).astype(np.float32)
+            elif w.act == "silu":
+                h = h / (1.0 + np.exp(-h))
+    return h.astype(np.float32)
+
+
+@dataclass
+class Inputs:
+    theta0: np.ndarray      # [P] float32
+    eta: np.ndarray         # [n_eta] float32
+    inner_x: np.ndarray     # [T, B, d_in] float32 (bf16-representable for bf16 workloads)
+    inner_y: np.ndarray     # [T, B] int32 labels or [T, B, d_out] float32 targets
+    outer_x: np.ndarray     # [B_outer, d_in]
+    outer_y: np.ndarray     # [B_outer] int32 or [B_outer, d_out] float32
+
+
+def make_inputs(w: Workload) -> Inputs:
+    """Draw every input of one meta-gradient call for workload ``w``."""
+    din, dout = w.dims[0], w.dims[-1]
+    rd = round_bf16 if w.precision == "bf16" else (lambda a: np.asarray(a, np.float32))
+    x = rd(rng(w.seed, "x").standard_normal((w.T, w.B, din)))
+    ox = rd(rng(w.seed, "outer").standard_normal((w.B_outer, din)))
+    if w.loss == "ce":
+        y = rng(w.seed, "labels").integers(0, dout, size=(w.T, w.B)).astype(np.int32)
+        oy = rng(w.seed, "outer_labels").integers(0, dout, size=(w.B_outer,)).astype(np.int32)
+    else:
+        y = _teacher_outputs(w, x.reshape(-1, din)).reshape(w.T, w.B, dout)
+        oy = _teacher_outputs(w, ox)
+        if w.noise_std > 0:
+            y = (y + w.noise_std * rng(w.seed, "noise").standard_normal(y.shape)).astype(np.float32)
+            oy = (oy + w.noise_std * rng(w.seed, "outer_noise").standard_normal(oy.shape)).astype(np.float32)
+    theta0 = glorot_params(w, rng(w.seed, "theta0"))
+    ge = rng(w.seed, "eta")
+    parts = []
+    if w.meta_kind & EXAMPLE_WEIGHTS:
+        parts.append(w.eta_std * ge.standard_normal(w.T * w.B))
+    if w.meta_kind & PARAM_LOGLR:
+        parts.append(w.loglr_mean + w.loglr_std * ge.standard_normal(w.n_params))
+    if w.meta_kind & SCALAR_LOGLR:
+        parts.append(np.array([w.extra.get("scalar_loglr", math.log(1e-3))]))
+    eta = np.concatenate(parts).astype(np.float32)
+    return Inputs(theta0, eta, np.ascontiguousarray(x, np.float32), y,
+                  np.ascontiguousarray(ox, np.float32), oy)
+
+
+def random_direction(n: int, seed: int = 0, k: int = 0) -> np.ndarray:
+    """A seeded Gaussian direction of length n (HVP tangents, directional checks)."""
+    g = np.random.Generator(np.random.PCG64(np.random.SeedSequence([seed, _STREAMS["dir"], k])))
+    return g.standard_normal(n).astype(np.float32)

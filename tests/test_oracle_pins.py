@@ -1,0 +1,220 @@
+"""Pins of the CPU oracle against facts other than itself (no GPU needed).
+
+* P1  central finite differences of V(eta) (the meta-gradient is the exact derivative of
+      the unrolled program, Eq. 2 / Proposition 3.1), on several small MLP workloads
+      covering every activation, both losses, momentum and all meta-parameter kinds.
+* P2  linear model with squared loss: Hessian = kron(X^T W X / (B*O), I_O) in closed form,
+      and the whole meta-gradient through the explicit-matrix adjoint recurrence of Eq. 5.
+* P3  Hessian symmetry u^T (H v) = v^T (H u) (Schwarz, Eqs. 6-7) and linearity.
+* P4  explicit Hessian of a 8->16->1 tanh MLP by finite differences of the gradient, which
+      is itself pinned to finite differences of the plain forward loss.
+* P5  special cases: alpha = 0 gives zero weight meta-gradient and dV/dtheta_0 = grad V;
+      T = 1 gives d eta_b = -(alpha/B) sigma'(eta_b) grad l_b(theta_0) . grad V(theta_1).
+* tangent losses dl_b/dtheta . v against finite differences of l_b.
+"""
+import math
+
+import numpy as np
+import pytest
+
+from paper_2505_00793_gb300 import synth
+from oracle import metagrad as om
+
+EX, PLR, SLR = synth.EXAMPLE_WEIGHTS, synth.PARAM_LOGLR, synth.SCALAR_LOGLR
+
+
+def _rel(a, b):
+    a, b = np.asarray(a, np.float64), np.asarray(b, np.float64)
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
+
+
+def _fd_eta(w, inp, idx, h=1e-5, dirs=None):
+    eta = inp.eta.astype(np.float64)
+    out = []
+    for i in idx:
+        e = np.zeros_like(eta)
+        e[i] = h
+        out.append((om.value(w, inp, eta + e) - om.value(w, inp, eta - e)) / (2 * h))
+    return np.array(out)
+
+
+SMALL = {
+    "tiny": synth.WORKLOADS["tiny"],
+    "ce_gelu": synth.Workload("ce_gelu", [6, 8, 8, 4], "gelu", "ce", "fp32", B=5, T=3,
+                              B_outer=7, alpha=0.3),
+    "mom_plr_silu": synth.Workload("mom_plr_silu", [4, 6, 3], "silu", "squared", "fp32", B=6,
+                                   T=3, B_outer=5, momentum=0.9, meta_kind=PLR,
+                                   loglr_mean=math.log(0.2), loglr_std=0.1),
+    "ex_slr_tanh_mom": synth.Workload("ex_slr_tanh_mom", [5, 7, 2], "tanh", "squared", "fp32",
+                                      B=4, T=3, B_outer=6, momentum=0.5, meta_kind=EX | SLR,
+                                      noise_std=0.1, extra={"scalar_loglr": math.log(0.3)}),
+}
+
+
+@pytest.mark.parametrize("name", list(SMALL))
+def test_p1_finite_differences(name):
+    w = SMALL[name]
+    inp = synth.make_inputs(w)
+    res = om.meta_grad(w, inp)
+    n = w.n_eta
+    idx = list(range(n)) if n <= 64 else list(np.random.default_rng(0).choice(n, 40, replace=False))
+    fd = _fd_eta(w, inp, idx)
+    assert _rel(res["d_eta"][idx], fd) < 1e-6, (res["d_eta"][idx], fd)
+    assert np.abs(res["d_eta"][idx]).max() > 1e-6  # non-trivial
+
+
+def test_p1_theta0_finite_differences():
+    w = SMALL["ce_gelu"]
+    inp = synth.make_inputs(w)
+    res = om.meta_grad(w, inp)
+    rng = np.random.default_rng(1)
+    for k in rng.choice(w.n_params, 6, replace=False):
+        h = 1e-5
+        ip = synth.Inputs(inp.theta0.astype(np.float64).copy(), inp.eta, inp.inner_x, inp.inner_y,
+                          inp.outer_x, inp.outer_y)
+        im = synth.Inputs(inp.theta0.astype(np.float64).copy(), inp.eta, inp.inner_x, inp.inner_y,
+                          inp.outer_x, inp.outer_y)
+        ip.theta0[k] += h
+        im.theta0[k] -= h
+        fd = (om.value(w, ip) - om.value(w, im)) / (2 * h)
+        assert abs(res["d_theta0"][k] - fd) <= 1e-6 * (abs(fd) + 1e-3)
+
+
+def _linear_workload(B=6, T=3, din=4, dout=3):
+    return synth.Workload("lin", [din, dout], "ident", "squared", "fp32", B=B, T=T, B_outer=5,
+                          alpha=0.2, noise_std=0.1)
+
+
+def _xt(x):
+    return np.concatenate([x, np.ones((x.shape[0], 1))], axis=1)
+
+
+def test_p2_linear_hessian_closed_form():
+    w = _linear_workload()
+    inp = synth.make_inputs(w)
+    ex = 1.0 / (1.0 + np.exp(-inp.eta.astype(np.float64).reshape(w.T, w.B)))
+    X = _xt(inp.inner_x[0].astype(np.float64))
+    O = w.dims[-1]
+    H = np.kron(X.T @ np.diag(ex[0]) @ X / (w.B * O), np.eye(O))
+    v = synth.random_direction(w.n_params, 3)
+    hv = om.hvp(w, inp.theta0, inp.inner_x[0], inp.inner_y[0], v, ex[0])
+    assert _rel(hv, H @ v) < 1e-12
+
+
+def test_p2_linear_meta_grad_closed_form():
+    w = _linear_workload()
+    inp = synth.make_inputs(w)
+    O, B = w.dims[-1], w.B
+    eta = inp.eta.astype(np.float64).reshape(w.T, B)
+    wts = 1.0 / (1.0 + np.exp(-eta))
+    theta = inp.theta0.astype(np.float64)
+    Xs = [_xt(inp.inner_x[t].astype(np.float64)) for t in range(w.T)]
+    Ys = [inp.inner_y[t].astype(np.float64) for t in range(w.T)]
+
+    def resid(theta, X, Y):  # f - y, with theta as [(din+1), O]
+        return X @ theta.reshape(-1, O) - Y
+
+    thetas = [theta]
+    for t in range(w.T):
+        r = resid(thetas[-1], Xs[t], Ys[t])
+        g = (Xs[t].T @ (wts[t][:, None] * r) / (B * O)).reshape(-1)
+        thetas.append(thetas[-1] - w.alpha * g)
+    Xo = _xt(inp.outer_x.astype(np.float64))
+    ro = resid(thetas[-1], Xo, inp.outer_y.astype(np.float64))
+    tb = (Xo.T @ ro / (w.B_outer * O)).reshape(-1)
+    d_eta = np.zeros((w.T, B))
+    for t in range(w.T - 1, -1, -1):
+        X = Xs[t]
+        H = np.kron(X.T @ np.diag(wts[t]) @ X / (B * O), np.eye(O))
+        r = resid(thetas[t], X, Ys[t])
+        for b in range(B):
+            grad_lb = np.outer(X[b], r[b]).reshape(-1) / O
+            d_eta[t, b] = wts[t, b] * (1 - wts[t, b]) * (-w.alpha / B) * grad_lb @ tb
+        tb = tb - w.alpha * H @ tb
+    res = om.meta_grad(w, inp)
+    assert _rel(res["d_eta"], d_eta.reshape(-1)) < 1e-12
+    assert _rel(res["d_theta0"], tb) < 1e-12
+
+
+def _mlp8():
+    return synth.Workload("h8", [8, 16, 1], "tanh", "squared", "fp32", B=10, T=1, B_outer=4,
+                          alpha=0.1, noise_std=0.1)
+
+
+def test_p3_symmetry_and_linearity():
+    for w in (_mlp8(), SMALL["ce_gelu"], SMALL["mom_plr_silu"]):
+        inp = synth.make_inputs(w)
+        u = synth.random_direction(w.n_params, 0, 1).astype(np.float64)
+        v = synth.random_direction(w.n_params, 0, 2).astype(np.float64)
+        wt = np.linspace(0.2, 1.0, w.B)
+        args = (inp.theta0, inp.inner_x[0], inp.inner_y[0])
+        hu = om.hvp(w, *args, u, wt)
+        hv = om.hvp(w, *args, v, wt)
+        assert abs(u @ hv - v @ hu) <= 1e-12 * (abs(u @ hv) + 1e-12)
+        huv = om.hvp(w, *args, 2.0 * u - 3.0 * v, wt)
+        assert _rel(huv, 2.0 * hu - 3.0 * hv) < 1e-12
+
+
+def test_p4_explicit_hessian():
+    w = _mlp8()
+    inp = synth.make_inputs(w)
+    P = w.n_params
+    assert P == 161
+    x, y = inp.inner_x[0], inp.inner_y[0]
+    theta = inp.theta0.astype(np.float64)
+    # gradient vs finite differences of the plain forward loss
+    from oracle import model
+    import torch
+
+    def L(th):
+        return float(model.weighted_inner_loss(w, torch.from_numpy(th), torch.from_numpy(x.astype(np.float64)),
+                                               torch.from_numpy(y.astype(np.float64)),
+                                               torch.ones(w.B, dtype=torch.float64)))
+    g = om.grad(w, theta, x, y)
+    h = 1e-6
+    gfd = np.array([(L(theta + h * e) - L(theta - h * e)) / (2 * h) for e in np.eye(P)])
+    assert _rel(g, gfd) < 1e-7
+    # Hessian column by column from finite differences of the gradient
+    h = 1e-5
+    Hfd = np.stack([(om.grad(w, theta + h * e, x, y) - om.grad(w, theta - h * e, x, y)) / (2 * h)
+                    for e in np.eye(P)], axis=1)
+    assert _rel(Hfd, Hfd.T) < 1e-7
+    v = synth.random_direction(P, 0, 5)
+    assert _rel(om.hvp(w, theta, x, y, v), Hfd @ v) < 1e-7
+
+
+def test_p5_alpha_zero():
+    w = SMALL["tiny"].with_(alpha=0.0)
+    inp = synth.make_inputs(w)
+    res = om.meta_grad(w, inp)
+    assert np.abs(res["d_eta"]).max() == 0.0
+    gV = om.grad(w, inp.theta0, inp.outer_x, inp.outer_y)
+    assert _rel(res["d_theta0"], gV) < 1e-14
+
+
+def test_p5_single_step():
+    w = SMALL["tiny"].with_(T=1)
+    inp = synth.make_inputs(w)
+    res = om.meta_grad(w, inp)
+    thetas, _ = om.rollout(w, inp)
+    gV = om.grad(w, thetas[1].numpy(), inp.outer_x, inp.outer_y)
+    eta = inp.eta.astype(np.float64)
+    s = 1 / (1 + np.exp(-eta))
+    expect = []
+    for b in range(w.B):
+        glb = om.grad(w, inp.theta0, inp.inner_x[0][b:b + 1], inp.inner_y[0][b:b + 1])
+        expect.append(-(w.alpha / w.B) * s[b] * (1 - s[b]) * glb @ gV)
+    assert _rel(res["d_eta"], expect) < 1e-12
+
+
+def test_tangent_losses_fd():
+    for w in (SMALL["ce_gelu"], _mlp8()):
+        inp = synth.make_inputs(w)
+        v = synth.random_direction(w.n_params, 0, 7)
+        theta = inp.theta0.astype(np.float64)
+        x, y = inp.inner_x[0], inp.inner_y[0]
+        ld = om.tangent_losses(w, theta, x, y, v)
+        h = 1e-6
+        fd = (om.per_example_losses(w, theta + h * v, x, y)
+              - om.per_example_losses(w, theta - h * v, x, y)) / (2 * h)
+        assert _rel(ld, fd) < 1e-7
