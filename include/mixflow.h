@@ -1,0 +1,206 @@
+/*
+ * mixflow.h - C ABI of the GB300 mixed-mode (forward-over-reverse) meta-gradient library.
+ *
+ * The library computes the meta-gradient dV/d eta of a Truncated-BPTT bilevel problem
+ * (Eq. 1 of "Scalable Meta-Learning via Mixed-Mode Differentiation", unrolled as Eq. 2):
+ *
+ *     m_{t+1}     = mu * m_t + grad_theta L_t(theta_t),             m_0 = 0
+ *     theta_{t+1} = theta_t - lr (*) m_{t+1},                        t = 0..T-1
+ *     L_t(theta)  = (1/B) sum_b w_{t,b} l_b(theta; x_{t,b}),  w_{t,b} = sigmoid(eta_{t,b})
+ *     V           = (1/B_outer) sum_b l_b(theta_T; outer batch)
+ *
+ * with lr = alpha, or exp(eta_lr) per parameter, or exp(eta_s) for one scalar log-lr.
+ * The backward sweep walks t = T-1..0 using the reparameterisation of Eq. 3 and the
+ * symmetry identities of Eqs. 6-7: every vector-Hessian and vector-mixed-derivative product
+ * of the recurrence Eq. 5 is evaluated as a Hessian-vector product by forward-over-reverse
+ * differentiation (Section 3, Proposition 3.1, Algorithm 2):
+ *
+ *     theta_bar_T = grad V(theta_T),  m_bar_T = 0
+ *     u_t         = m_bar_{t+1} - lr (*) theta_bar_{t+1}
+ *     theta_bar_t = theta_bar_{t+1} + H_t u_t              (H_t = Hessian of L_t at theta_t)
+ *     m_bar_t     = mu * u_t
+ *     d eta_{t,b} = sigmoid'(eta_{t,b}) / B * (grad l_b(theta_t) . u_t)
+ *     d eta_lr   += -lr (*) m_{t+1} (*) theta_bar_{t+1}
+ *
+ * Inner models: multilayer perceptrons (MF_ARCH_MLP).  Parameters are one flat float32
+ * vector: for each layer l, W_l as [d_l][d_{l+1}] row-major, then b_l [d_{l+1}].
+ *
+ * Conventions for every call:
+ *  - Tensor arguments are device pointers owned by the caller (e.g. torch CUDA tensors),
+ *    unless stated otherwise.  They must stay valid until the stream work completes.
+ *  - Calls enqueue work on `stream` (a cudaStream_t; NULL = legacy default stream) and
+ *    return without synchronising, except where stated.  Argument errors are returned
+ *    immediately; errors found on the device (non-finite values, a kernel wait that ran out
+ *    of time) are reported by mf_sync().
+ *  - Library workspace (the theta_t checkpoint store, activations) is obtained through the
+ *    allocator set with mf_set_allocator (default: cudaMallocAsync on the call's stream),
+ *    kept in the handle between calls with the same or smaller shape, and released by
+ *    mf_release_workspace() or mf_destroy().
+ *  - A handle is not thread-safe; use one handle per host thread.
+ */
+#ifndef MIXFLOW_H
+#define MIXFLOW_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct mf_ctx* mf_handle;
+
+typedef enum {
+  MF_OK = 0,
+  MF_ERR_INVALID_ARG = 1,   /* a NULL pointer, a bad size or an inconsistent descriptor */
+  MF_ERR_UNSUPPORTED = 2,   /* valid request this build does not implement */
+  MF_ERR_OOM = 3,           /* the allocator returned NULL */
+  MF_ERR_CUDA = 4,          /* a CUDA runtime call failed; see mf_last_error() */
+  MF_ERR_NONFINITE = 5,     /* a NaN/Inf reached the adjoint or the updated parameters */
+  MF_ERR_TIMEOUT = 6        /* a bounded device-side wait ran out of time */
+} mf_status;
+
+enum { MF_ARCH_MLP = 0, MF_ARCH_DECODER = 1 };
+enum { MF_ACT_IDENT = 0, MF_ACT_TANH = 1, MF_ACT_GELU = 2, MF_ACT_SILU = 3 };
+enum { MF_LOSS_SQUARED = 0, MF_LOSS_SOFTMAX_CE = 1, MF_LOSS_NEXT_TOKEN_CE = 2 };
+enum { MF_PREC_FP32 = 0, MF_PREC_BF16 = 1 };
+enum { MF_META_EXAMPLE_WEIGHTS = 1, MF_META_PARAM_LOGLR = 2, MF_META_SCALAR_LOGLR = 4 };
+enum { MF_HVP_MIXED_FOR = 0, MF_HVP_REV_REV = 1 };
+
+#define MF_MAX_LAYERS 32
+
+/* Inner model (Eq. 1's L and V).
+ *  arch       MF_ARCH_MLP.
+ *  n_layers   number of Linear layers, 1..MF_MAX_LAYERS.
+ *  dims       n_layers+1 widths: dims[0] = input size, dims[n_layers] = output size.
+ *  act        activation after every layer but the last (MF_ACT_*).
+ *  has_bias   1 = every layer has a bias vector.
+ *  loss       MF_LOSS_SQUARED: l_b = 1/2 mean_o (f_bo - y_bo)^2, y float32 [rows][d_out];
+ *             MF_LOSS_SOFTMAX_CE: l_b = logsumexp(f_b) - f_{b,y_b}, y int32 [rows].
+ *  precision  MF_PREC_FP32: float32 inputs, float32 GEMMs (SIMT);
+ *             MF_PREC_BF16: bf16 inputs, bf16 tensor-core GEMMs with float32 accumulation;
+ *             parameters, optimiser state, adjoints and meta-gradients stay float32.
+ *  The remaining fields are reserved for MF_ARCH_DECODER and must be 0 for MLPs. */
+typedef struct {
+  int arch;
+  int n_layers;
+  int dims[MF_MAX_LAYERS + 1];
+  int act;
+  int has_bias;
+  int loss;
+  int precision;
+  int d_model, n_heads, d_ff, vocab, seq_len;
+  float rope_base, rms_eps;
+} mf_model_desc;
+
+/* Inner loop (Eq. 2) and meta-parameters.
+ *  T          inner steps (>= 1);  B rows per inner batch;  B_outer rows of the outer batch.
+ *  alpha      constant learning rate (used when no log-lr meta-parameter is set).
+ *  momentum   heavy-ball coefficient mu in [0, 1) (0 = plain SGD).
+ *  meta_kind  bit mask of MF_META_*; eta is laid out as [T*B example-weight logits]
+ *             [P per-parameter log-lrs][1 scalar log-lr], in that order, for the bits set.
+ *             PARAM_LOGLR and SCALAR_LOGLR are mutually exclusive.
+ *  hvp_mode   MF_HVP_MIXED_FOR (this build's sweep; MF_HVP_REV_REV is reserved).
+ *  ckpt_every 1 = keep every theta_t in the checkpoint store (the only value accepted). */
+typedef struct {
+  int T, B, B_outer;
+  float alpha, momentum;
+  int meta_kind;
+  int hvp_mode;
+  int ckpt_every;
+} mf_loop_desc;
+
+/* Create a handle for one inner-model architecture.  *out receives a library-owned handle.
+ * Errors: MF_ERR_INVALID_ARG (bad descriptor), MF_ERR_UNSUPPORTED (decoder arch),
+ * MF_ERR_CUDA (no usable device). */
+mf_status mf_create(const mf_model_desc* desc, mf_handle* out);
+
+/* Release the handle and its workspace (synchronises the device first). */
+mf_status mf_destroy(mf_handle h);
+
+/* Route workspace allocations through caller callbacks (e.g. PyTorch's caching allocator).
+ * alloc(bytes, stream, ctx) returns a device pointer or NULL; free(ptr, bytes, stream, ctx).
+ * Pass alloc = free = NULL to restore the default.  Releases the current workspace. */
+mf_status mf_set_allocator(mf_handle h, void* (*alloc)(size_t, void*, void*),
+                           void (*free_fn)(void*, size_t, void*, void*), void* ctx);
+
+/* Number of parameters P = |theta| and of meta-parameters |eta| for loop descriptor `loop`
+ * (loop may be NULL, then *n_eta is set to 0).  Host-only. */
+mf_status mf_param_count(mf_handle h, const mf_loop_desc* loop, int64_t* n_params,
+                         int64_t* n_eta);
+
+/* Bytes of workspace mf_meta_grad needs for `loop` (checkpoint store + activations). */
+mf_status mf_workspace_bytes(mf_handle h, const mf_loop_desc* loop, size_t* bytes);
+
+/* Free the cached workspace now (the next call allocates it again). */
+mf_status mf_release_workspace(mf_handle h);
+
+/* Inner rollout only (Eq. 2, Algorithm 2's loop): theta0 [P] float32, eta as above,
+ * inner_x [T][B][d_in] (bf16 for MF_PREC_BF16, float32 for MF_PREC_FP32), inner_y
+ * [T][B] int32 labels or [T][B][d_out] float32 targets.  Writes thetaT [P]. */
+mf_status mf_inner_rollout(mf_handle h, const mf_loop_desc* loop, const float* theta0,
+                           const float* eta, const void* inner_x, const void* inner_y,
+                           float* thetaT, void* stream);
+
+/* One fwdrev_grad backward step (Section 3.1): at parameters theta [P], on the batch
+ * x [B][d_in] / y [B] or [B][d_out] with per-example loss weights ex_w [B] (NULL = all 1),
+ * for L = (1/B) sum_b ex_w_b l_b:
+ *   Hv [P]             = (d^2 L / d theta^2) v        (forward-over-reverse)
+ *   tangent_losses [B] = grad l_b(theta) . v           (nullable; the mixed term per example)
+ *   grad [P]           = grad L(theta)                 (nullable)
+ * hvp_mode must be MF_HVP_MIXED_FOR. */
+mf_status mf_hvp(mf_handle h, int B, const float* theta, const void* x, const void* y,
+                 const float* ex_w, const float* v, float* Hv, float* tangent_losses,
+                 float* grad, int hvp_mode, void* stream);
+
+/* The meta-gradient (Algorithm 2): rollout storing theta_t (and m_t when lr is a
+ * meta-parameter), outer gradient (Eq. 4), then the mixed-mode reverse sweep t = T-1..0.
+ *   d_eta [n_eta]      dV/d eta (same layout as eta).
+ *   d_theta0 [P]       dV/d theta_0 (nullable).
+ *   outer_loss [1]     V (nullable, device float).
+ * outer_x [B_outer][d_in], outer_y [B_outer] int32 or [B_outer][d_out] float32. */
+mf_status mf_meta_grad(mf_handle h, const mf_loop_desc* loop, const float* theta0,
+                       const float* eta, const void* inner_x, const void* inner_y,
+                       const void* outer_x, const void* outer_y, float* d_eta,
+                       float* d_theta0, float* outer_loss, void* stream);
+
+/* Wait for the handle's last stream and report device-side errors (MF_ERR_NONFINITE,
+ * MF_ERR_TIMEOUT, MF_ERR_CUDA).  Clears the device status word. */
+mf_status mf_sync(mf_handle h);
+
+/* Static description of a status code, and the handle's last error message. */
+const char* mf_status_string(mf_status s);
+const char* mf_last_error(mf_handle h);
+
+/* Diagnostics.  mf_stats: kernel launches issued by the handle since creation and the
+ * largest workspace it has held.  mf_set_kernel_timing(h, 1) records CUDA events around
+ * every launch of the bf16 dual GEMM (slower; for measurement);  mf_kernel_time returns
+ * the summed milliseconds and launch count of that kernel since the last reset, plus its
+ * algorithmic flops (2*M*N*K per accumulated product term), then resets. */
+mf_status mf_stats(mf_handle h, uint64_t* launches, size_t* peak_workspace_bytes);
+mf_status mf_set_kernel_timing(mf_handle h, int enable);
+mf_status mf_kernel_time(mf_handle h, double* ms, uint64_t* launches, double* flops);
+
+/* Host-side fault injection for tests: kind 1 = the next workspace allocation fails;
+ * kind 2 = the next mf_sync reports MF_ERR_TIMEOUT as if a device wait had expired;
+ * kind 0 clears.  Nothing is done on the GPU. */
+mf_status mf_inject_fault(mf_handle h, int kind);
+
+/* Building block exposed for tests and profiling: the bf16 dual GEMM of the sweep.
+ * All operands K-major, row-major with leading dimension in elements (multiple of 8):
+ *   A0, A1 [M][K] bf16;  B0, B1 [N][K] bf16;  C0, C1 [M][N] float32 (ldc).
+ * `terms` selects the products summed into each accumulator:
+ *   bit 0: C0 += A0 B0^T   bit 1: C0 += A1 B0^T   bit 2: C0 += A0 B1^T
+ *   bit 3: C1 += A1 B0^T   bit 4: C1 += A0 B1^T
+ * The forward tangent of a dual Linear layer is terms = 1|8|16:  C0 = A0 B0^T (primal),
+ * C1 = A1 B0^T + A0 B1^T (tangent).  bias0/bias1 [N] float32 are added when non-NULL.
+ * Runs on tcgen05 tensor cores with TMEM accumulators and TMA-fed shared memory. */
+mf_status mf_dual_gemm_bf16(int M, int N, int K, const void* A0, int lda0, const void* A1,
+                            int lda1, const void* B0, int ldb0, const void* B1, int ldb1,
+                            float* C0, int ldc0, const float* bias0, float* C1, int ldc1,
+                            const float* bias1, unsigned terms, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MIXFLOW_H */

@@ -1,0 +1,793 @@
+// Host runtime of the library: handle, workspace, the MLP executor (dual forward, dual loss,
+// dual backward as sequences of kernel launches), the rollout with its theta_t checkpoint
+// store, the mixed-mode reverse sweep, and the C ABI of include/mixflow.h.
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <algorithm>
+#include <string>
+#include <utility>
+#include <vector>
+
+#include "../../include/mixflow.h"
+#include "internal.h"
+
+using mf::GemmArgs;
+
+namespace {
+
+constexpr size_t ALIGN = 256;
+inline size_t align_up(size_t x, size_t a = ALIGN) { return (x + a - 1) / a * a; }
+inline int ld8(int x) { return (x + 7) / 8 * 8; }
+
+}  // namespace
+
+struct mf_ctx {
+  mf_model_desc md;
+  int L = 0;
+  std::vector<int> dims;
+  std::vector<int64_t> woff, boff;
+  int64_t P = 0;
+  int maxd = 0;
+  bool bf16 = false;
+
+  void* (*ualloc)(size_t, void*, void*) = nullptr;
+  void (*ufree)(void*, size_t, void*, void*) = nullptr;
+  void* uctx = nullptr;
+
+  void* ws = nullptr;
+  size_t ws_bytes = 0;
+  size_t peak = 0;
+  int* d_status = nullptr;
+  std::string err;
+  uint64_t launches = 0;
+  cudaStream_t last_stream = nullptr;
+  int fault = 0;
+
+  bool timing = false;
+  std::vector<std::pair<cudaEvent_t, cudaEvent_t>> evs;
+  double timed_flops = 0.0;
+};
+
+namespace {
+
+mf_status fail(mf_ctx* h, mf_status s, const std::string& msg) {
+  if (h) h->err = msg;
+  return s;
+}
+
+#define MF_CUDA(h, call)                                                          \
+  do {                                                                            \
+    cudaError_t e_ = (call);                                                      \
+    if (e_ != cudaSuccess)                                                        \
+      return fail(h, MF_ERR_CUDA, std::string(#call) + ": " + cudaGetErrorString(e_)); \
+  } while (0)
+
+// ---- workspace layout -------------------------------------------------------------------
+struct Plan {
+  int rows = 0;          // max rows of any batch
+  int ldR = 0;           // leading dim of transposed activations (multiple of 8)
+  int T = 0;
+  bool store_all = true; // keep theta_0..theta_T
+  int n_theta_slots = 0, n_m_slots = 0;
+  int nb = 0;            // adjoint partial blocks per step
+  size_t bytes = 0;
+  // offsets
+  size_t o_theta = 0, o_m = 0, o_g = 0, o_tbar = 0, o_u = 0, o_part = 0, o_l = 0, o_ld = 0;
+  std::vector<size_t> o_Wb, o_WbT, o_Ub, o_UbT, o_A, o_Ad, o_AT, o_AdT, o_Z, o_Zd;
+  size_t o_dZ = 0, o_dZd = 0, o_dZT = 0, o_dZdT = 0, o_dZ32 = 0, o_dZd32 = 0, o_dA = 0, o_dAd = 0;
+};
+
+Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slots,
+               bool with_partials) {
+  Plan p;
+  p.rows = rows;
+  p.ldR = ld8(rows);
+  p.T = T;
+  p.n_theta_slots = n_theta_slots;
+  p.n_m_slots = n_m_slots;
+  const size_t es = h->bf16 ? 2 : 4;
+  size_t o = 0;
+  auto take = [&](size_t bytes) { size_t r = o; o += align_up(bytes); return r; };
+  const size_t P4 = static_cast<size_t>(h->P) * 4;
+  p.o_theta = take(P4 * n_theta_slots);
+  p.o_m = take(P4 * n_m_slots);
+  p.o_g = take(P4);
+  p.o_tbar = take(P4);
+  p.o_u = take(P4);
+  p.nb = mf::adjoint_partials_blocks(h->P);
+  p.o_part = take(with_partials ? static_cast<size_t>(p.nb) * (T > 0 ? T : 1) * 4 : 4);
+  p.o_l = take(static_cast<size_t>(rows) * 4);
+  p.o_ld = take(static_cast<size_t>(rows) * 4);
+  const int L = h->L;
+  p.o_Wb.resize(L); p.o_WbT.resize(L); p.o_Ub.resize(L); p.o_UbT.resize(L);
+  p.o_A.resize(L); p.o_Ad.resize(L); p.o_AT.resize(L); p.o_AdT.resize(L);
+  p.o_Z.resize(L); p.o_Zd.resize(L);
+  for (int l = 0; l < L; ++l) {
+    const int din = h->dims[l], dout = h->dims[l + 1];
+    p.o_Wb[l] = take(static_cast<size_t>(din) * ld8(dout) * es);
+    p.o_WbT[l] = take(static_cast<size_t>(dout) * ld8(din) * es);
+    p.o_Ub[l] = take(static_cast<size_t>(din) * ld8(dout) * es);
+    p.o_UbT[l] = take(static_cast<size_t>(dout) * ld8(din) * es);
+    p.o_A[l] = take(static_cast<size_t>(rows) * ld8(din) * es);
+    p.o_Ad[l] = take(static_cast<size_t>(rows) * ld8(din) * es);
+    p.o_AT[l] = take(static_cast<size_t>(din) * p.ldR * es);
+    p.o_AdT[l] = take(static_cast<size_t>(din) * p.ldR * es);
+    p.o_Z[l] = take(static_cast<size_t>(rows) * dout * 4);
+    p.o_Zd[l] = take(static_cast<size_t>(rows) * dout * 4);
+  }
+  const int md = h->maxd;
+  p.o_dZ = take(static_cast<size_t>(rows) * ld8(md) * es);
+  p.o_dZd = take(static_cast<size_t>(rows) * ld8(md) * es);
+  p.o_dZT = take(static_cast<size_t>(md) * p.ldR * es);
+  p.o_dZdT = take(static_cast<size_t>(md) * p.ldR * es);
+  p.o_dZ32 = take(static_cast<size_t>(rows) * md * 4);
+  p.o_dZd32 = take(static_cast<size_t>(rows) * md * 4);
+  p.o_dA = take(static_cast<size_t>(rows) * md * 4);
+  p.o_dAd = take(static_cast<size_t>(rows) * md * 4);
+  p.bytes = o;
+  return p;
+}
+
+void release_ws(mf_ctx* h) {
+  if (!h->ws) return;
+  cudaDeviceSynchronize();
+  if (h->ufree) h->ufree(h->ws, h->ws_bytes, nullptr, h->uctx);
+  else cudaFree(h->ws);
+  h->ws = nullptr;
+  h->ws_bytes = 0;
+}
+
+mf_status ensure_ws(mf_ctx* h, size_t bytes, cudaStream_t s) {
+  if (h->fault == 1) {
+    h->fault = 0;
+    return fail(h, MF_ERR_OOM, "injected allocation failure");
+  }
+  if (h->ws && h->ws_bytes >= bytes) return MF_OK;
+  release_ws(h);
+  void* p = nullptr;
+  if (h->ualloc) {
+    p = h->ualloc(bytes, static_cast<void*>(s), h->uctx);
+  } else if (cudaMalloc(&p, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    p = nullptr;
+  }
+  if (!p) return fail(h, MF_ERR_OOM, "workspace allocation of " + std::to_string(bytes) + " bytes failed");
+  h->ws = p;
+  h->ws_bytes = bytes;
+  h->peak = std::max(h->peak, bytes);
+  return MF_OK;
+}
+
+// ---- the MLP executor --------------------------------------------------------------------
+template <typename T>
+struct Exec {
+  mf_ctx* h;
+  const Plan& p;
+  cudaStream_t s;
+  char* base;
+  mf_status st = MF_OK;
+
+  Exec(mf_ctx* h_, const Plan& p_, cudaStream_t s_)
+      : h(h_), p(p_), s(s_), base(static_cast<char*>(h_->ws)) {}
+
+  template <typename U> U* at(size_t off) const { return reinterpret_cast<U*>(base + off); }
+  float* theta_slot(int t) const { return at<float>(p.o_theta) + static_cast<int64_t>(t) * h->P; }
+  float* m_slot(int j) const { return at<float>(p.o_m) + static_cast<int64_t>(j) * h->P; }
+
+  void launched(int n = 1) { h->launches += n; }
+
+  void check(cudaError_t e, const char* what) {
+    if (e != cudaSuccess && st == MF_OK) {
+      st = MF_ERR_CUDA;
+      h->err = std::string(what) + ": " + cudaGetErrorString(e);
+    }
+  }
+
+  void gemm(GemmArgs g) {
+    if (st != MF_OK) return;
+    g.status = h->d_status;
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    const bool tc = h->bf16;
+    if (tc && h->timing) {
+      cudaEventCreate(&e0);
+      cudaEventCreate(&e1);
+      cudaEventRecord(e0, s);
+    }
+    cudaError_t e;
+    const char* why = "";
+    if (tc) e = mf::tc_gemm(g, s, &why);
+    else e = mf::simt_gemm(g, s);
+    if (e != cudaSuccess) {
+      st = MF_ERR_CUDA;
+      h->err = std::string("dual GEMM launch failed: ") + cudaGetErrorString(e) + " " + why;
+      return;
+    }
+    launched();
+    if (tc && h->timing) {
+      cudaEventRecord(e1, s);
+      h->evs.emplace_back(e0, e1);
+      h->timed_flops += 2.0 * g.M * g.N * static_cast<double>(g.K) * mf::term_count(g.terms);
+    }
+  }
+
+  // bf16 (or fp32) operand copies of the weights of theta (or of the tangent u).
+  void cast_params(const float* theta, bool tangent) {
+    for (int l = 0; l < h->L; ++l) {
+      const int din = h->dims[l], dout = h->dims[l + 1];
+      T* W = at<T>(tangent ? p.o_Ub[l] : p.o_Wb[l]);
+      T* WT = at<T>(tangent ? p.o_UbT[l] : p.o_WbT[l]);
+      mf::cast_transpose<T>(theta + h->woff[l], din, dout, W, ld8(dout), WT, ld8(din), s);
+      launched();
+    }
+  }
+
+  // Forward pass of `rows` examples: primal (z) or dual (z, z_dot along u).
+  void forward(int rows, const T* x, const float* theta, const float* u, bool dual) {
+    const int din0 = h->dims[0];
+    mf::transpose<T>(x, rows, din0, din0, at<T>(p.o_AT[0]), p.ldR, s);
+    launched();
+    for (int l = 0; l < h->L; ++l) {
+      const int din = h->dims[l], dout = h->dims[l + 1];
+      GemmArgs g;
+      g.M = rows; g.N = dout; g.K = din;
+      g.A0 = l == 0 ? static_cast<const void*>(x) : at<T>(p.o_A[l]);
+      g.lda0 = l == 0 ? din : ld8(din);
+      g.A1 = l == 0 ? nullptr : at<T>(p.o_Ad[l]);
+      g.lda1 = ld8(din);
+      g.B0 = at<T>(p.o_WbT[l]); g.ldb0 = ld8(din);
+      g.B1 = at<T>(p.o_UbT[l]); g.ldb1 = ld8(din);
+      g.C0 = at<float>(p.o_Z[l]); g.ldc0 = dout;
+      g.bias0 = h->md.has_bias ? theta + h->boff[l] : nullptr;
+      g.terms = mf::T_C0_A0B0;
+      if (dual) {
+        g.terms |= mf::T_C1_A0B1 | (l > 0 ? mf::T_C1_A1B0 : 0u);
+        g.C1 = at<float>(p.o_Zd[l]); g.ldc1 = dout;
+        g.bias1 = h->md.has_bias ? u + h->boff[l] : nullptr;
+      }
+      gemm(g);
+      if (l + 1 < h->L) {
+        mf::act_fwd<T>(h->md.act, at<float>(p.o_Z[l]), dual ? at<float>(p.o_Zd[l]) : nullptr, rows,
+                       dout, at<T>(p.o_A[l + 1]), at<T>(p.o_Ad[l + 1]), ld8(dout),
+                       at<T>(p.o_AT[l + 1]), at<T>(p.o_AdT[l + 1]), p.ldR, s);
+        launched();
+      }
+    }
+  }
+
+  // Loss seeds at the head: d f (and its tangent) into the backward buffers.
+  void loss(int rows, bool dual, const void* y, const float* eta_w, const float* ex_w,
+            float* l_out, float* ld_out, float* d_eta) {
+    const int L = h->L, C = h->dims[L];
+    mf::LossArgs a;
+    a.loss = h->md.loss == MF_LOSS_SOFTMAX_CE ? 1 : 0;
+    a.rows = rows; a.cols = C;
+    a.F = at<float>(p.o_Z[L - 1]);
+    a.Fd = dual ? at<float>(p.o_Zd[L - 1]) : nullptr;
+    if (a.loss == 0) a.Yf = static_cast<const float*>(y);
+    else a.Yi = static_cast<const int*>(y);
+    a.eta_w = eta_w; a.ex_w = ex_w;
+    a.inv_norm = 1.f / static_cast<float>(rows);
+    a.l = l_out; a.ld = ld_out; a.d_eta = d_eta;
+    a.dF32 = at<float>(p.o_dZ32); a.dFd32 = dual ? at<float>(p.o_dZd32) : nullptr;
+    a.dF = at<T>(p.o_dZ); a.dFd = dual ? at<T>(p.o_dZd) : nullptr;
+    a.ldo = ld8(C);
+    a.status = h->d_status;
+    mf::loss_seed<T>(a, s);
+    launched();
+    mf::transpose<T>(at<T>(p.o_dZ), rows, C, ld8(C), at<T>(p.o_dZT), p.ldR, s);
+    launched();
+    if (dual) {
+      mf::transpose<T>(at<T>(p.o_dZd), rows, C, ld8(C), at<T>(p.o_dZdT), p.ldR, s);
+      launched();
+    }
+  }
+
+  // Backward pass.  Primal: out_g = grad L.  Dual: out_h = H u (and out_g = grad L if given).
+  void backward(int rows, bool dual, float* out_h, float* out_g) {
+    for (int l = h->L - 1; l >= 0; --l) {
+      const int din = h->dims[l], dout = h->dims[l + 1];
+      // weight product: grad W = a^T dz ;  (H u)_W = a_dot^T dz + a^T dz_dot
+      GemmArgs g;
+      g.M = din; g.N = dout; g.K = rows;
+      g.A0 = at<T>(p.o_AT[l]); g.lda0 = p.ldR;
+      g.A1 = at<T>(p.o_AdT[l]); g.lda1 = p.ldR;
+      g.B0 = at<T>(p.o_dZT); g.ldb0 = p.ldR;
+      g.B1 = at<T>(p.o_dZdT); g.ldb1 = p.ldR;
+      if (!dual) {
+        g.terms = mf::T_C0_A0B0;
+        g.C0 = out_g + h->woff[l]; g.ldc0 = dout;
+      } else if (out_g) {
+        g.terms = mf::T_C0_A0B0 | mf::T_C1_A0B1 | (l > 0 ? mf::T_C1_A1B0 : 0u);
+        g.C0 = out_g + h->woff[l]; g.ldc0 = dout;
+        g.C1 = out_h + h->woff[l]; g.ldc1 = dout;
+      } else {
+        g.terms = mf::T_C0_A0B1 | (l > 0 ? mf::T_C0_A1B0 : 0u);
+        g.C0 = out_h + h->woff[l]; g.ldc0 = dout;
+      }
+      gemm(g);
+      if (h->md.has_bias) {
+        if (dual) { mf::colsum(at<float>(p.o_dZd32), rows, dout, out_h + h->boff[l], s); launched(); }
+        if (out_g) {
+          mf::colsum(at<float>(p.o_dZ32), rows, dout, out_g + h->boff[l], s);
+          launched();
+        }
+      }
+      if (l == 0) break;
+      // data product: da = dz W^T ;  da_dot = dz_dot W^T + dz U^T
+      GemmArgs d;
+      d.M = rows; d.N = din; d.K = dout;
+      d.A0 = at<T>(p.o_dZ); d.lda0 = ld8(dout);
+      d.A1 = at<T>(p.o_dZd); d.lda1 = ld8(dout);
+      d.B0 = at<T>(p.o_Wb[l]); d.ldb0 = ld8(dout);
+      d.B1 = at<T>(p.o_Ub[l]); d.ldb1 = ld8(dout);
+      d.C0 = at<float>(p.o_dA); d.ldc0 = din;
+      d.terms = mf::T_C0_A0B0;
+      if (dual) {
+        d.terms |= mf::T_C1_A1B0 | mf::T_C1_A0B1;
+        d.C1 = at<float>(p.o_dAd); d.ldc1 = din;
+      }
+      gemm(d);
+      mf::act_bwd<T>(h->md.act, at<float>(p.o_Z[l - 1]), dual ? at<float>(p.o_Zd[l - 1]) : nullptr,
+                     at<float>(p.o_dA), dual ? at<float>(p.o_dAd) : nullptr, rows, din,
+                     at<T>(p.o_dZ), at<T>(p.o_dZd), ld8(din), at<T>(p.o_dZT), at<T>(p.o_dZdT),
+                     p.ldR, at<float>(p.o_dZ32), dual ? at<float>(p.o_dZd32) : nullptr, s);
+      launched();
+    }
+  }
+};
+
+mf_status validate_loop(mf_ctx* h, const mf_loop_desc* lp) {
+  if (!lp) return fail(h, MF_ERR_INVALID_ARG, "loop descriptor is NULL");
+  if (lp->T < 1 || lp->B < 1 || lp->B_outer < 1)
+    return fail(h, MF_ERR_INVALID_ARG, "T, B and B_outer must be >= 1");
+  if (lp->meta_kind & ~7) return fail(h, MF_ERR_INVALID_ARG, "unknown meta_kind bits");
+  if ((lp->meta_kind & MF_META_PARAM_LOGLR) && (lp->meta_kind & MF_META_SCALAR_LOGLR))
+    return fail(h, MF_ERR_INVALID_ARG, "PARAM_LOGLR and SCALAR_LOGLR are mutually exclusive");
+  if (!(lp->momentum >= 0.f && lp->momentum < 1.f))
+    return fail(h, MF_ERR_INVALID_ARG, "momentum must be in [0, 1)");
+  if (lp->hvp_mode != MF_HVP_MIXED_FOR)
+    return fail(h, MF_ERR_UNSUPPORTED, "only MF_HVP_MIXED_FOR is implemented");
+  if (lp->ckpt_every != 1 && lp->ckpt_every != 0)
+    return fail(h, MF_ERR_UNSUPPORTED, "only ckpt_every = 1 is implemented");
+  return MF_OK;
+}
+
+int64_t n_eta_of(const mf_ctx* h, const mf_loop_desc* lp) {
+  int64_t n = 0;
+  if (lp->meta_kind & MF_META_EXAMPLE_WEIGHTS) n += static_cast<int64_t>(lp->T) * lp->B;
+  if (lp->meta_kind & MF_META_PARAM_LOGLR) n += h->P;
+  if (lp->meta_kind & MF_META_SCALAR_LOGLR) n += 1;
+  return n;
+}
+
+mf_status check_x(mf_ctx* h, const void* x, int rows) {
+  if (!h->bf16) return MF_OK;
+  const int din = h->dims[0];
+  if ((reinterpret_cast<uintptr_t>(x) & 15) || (din % 8) != 0 ||
+      ((static_cast<int64_t>(rows) * din * 2) % 16) != 0)
+    return fail(h, MF_ERR_INVALID_ARG,
+                "bf16 inputs must be 16-byte aligned with d_in a multiple of 8");
+  return MF_OK;
+}
+
+size_t y_stride_bytes(const mf_ctx* h, int rows) {
+  return h->md.loss == MF_LOSS_SOFTMAX_CE ? static_cast<size_t>(rows) * 4
+                                          : static_cast<size_t>(rows) * h->dims[h->L] * 4;
+}
+
+struct LrSel {
+  mf::LrArgs lr;
+  bool lr_meta = false;
+  int64_t off_plr = -1, off_slr = -1;
+};
+
+LrSel lr_select(const mf_ctx* h, const mf_loop_desc* lp, const float* eta) {
+  LrSel r;
+  int64_t o = 0;
+  if (lp->meta_kind & MF_META_EXAMPLE_WEIGHTS) o += static_cast<int64_t>(lp->T) * lp->B;
+  r.lr.alpha = lp->alpha;
+  if (lp->meta_kind & MF_META_PARAM_LOGLR) {
+    r.off_plr = o;
+    r.lr.plr = eta + o;
+    r.lr_meta = true;
+    o += h->P;
+  }
+  if (lp->meta_kind & MF_META_SCALAR_LOGLR) {
+    r.off_slr = o;
+    r.lr.slr = eta + o;
+    r.lr_meta = true;
+  }
+  return r;
+}
+
+// Inner rollout (Eq. 2).  With store_all, theta slot t holds theta_t and m slot j holds
+// m_{j+1} when the learning rate is a meta-parameter; otherwise two theta slots ping-pong.
+template <typename E>
+void rollout(Exec<E>& ex, const mf_loop_desc* lp, const float* eta, const void* inner_x,
+             const void* inner_y, const LrSel& lr, bool store_all, float** theta_T) {
+  mf_ctx* h = ex.h;
+  const int B = lp->B, din = h->dims[0];
+  const size_t xs = static_cast<size_t>(B) * din * (h->bf16 ? 2 : 4);
+  const size_t ys = y_stride_bytes(h, B);
+  float* m_run = (lp->momentum != 0.f && !lr.lr_meta) ? ex.template at<float>(ex.p.o_u) : nullptr;
+  if (m_run) { mf::fill(m_run, h->P, 0.f, ex.s); ex.launched(); }
+  const float* m_prev = nullptr;
+  for (int t = 0; t < lp->T; ++t) {
+    float* th = ex.theta_slot(store_all ? t : (t & 1));
+    float* th_next = ex.theta_slot(store_all ? t + 1 : ((t + 1) & 1));
+    const E* x = reinterpret_cast<const E*>(static_cast<const char*>(inner_x) + xs * t);
+    const void* y = static_cast<const char*>(inner_y) + ys * t;
+    ex.cast_params(th, false);
+    ex.forward(B, x, th, nullptr, false);
+    const float* ew = (lp->meta_kind & MF_META_EXAMPLE_WEIGHTS) ? eta + static_cast<int64_t>(t) * B : nullptr;
+    ex.loss(B, false, y, ew, nullptr, nullptr, nullptr, nullptr);
+    float* g = ex.template at<float>(ex.p.o_g);
+    ex.backward(B, false, nullptr, g);
+    float* m_out = nullptr;
+    if (lr.lr_meta && store_all) m_out = ex.m_slot(t);
+    else if (lr.lr_meta) m_out = ex.m_slot(0);
+    else if (m_run) m_out = m_run;
+    const float* m_in = lr.lr_meta ? m_prev : m_run;
+    mf::rollout_update(h->P, th, m_in, g, lp->momentum, lr.lr, th_next, m_out, h->d_status, ex.s);
+    ex.launched();
+    m_prev = m_out;
+    if (ex.st != MF_OK) return;
+  }
+  *theta_T = ex.theta_slot(store_all ? lp->T : (lp->T & 1));
+}
+
+template <typename E>
+mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
+                         const float* eta, const void* inner_x, const void* inner_y,
+                         const void* outer_x, const void* outer_y, float* d_eta,
+                         float* d_theta0, float* outer_loss, cudaStream_t s) {
+  const int T = lp->T, B = lp->B, Bo = lp->B_outer;
+  const LrSel lr = lr_select(h, lp, eta);
+  const bool scalar_lr = lp->meta_kind & MF_META_SCALAR_LOGLR;
+  Plan plan = make_plan(h, std::max(B, Bo), T, T + 1, lr.lr_meta ? T : 0, scalar_lr);
+  mf_status st = ensure_ws(h, plan.bytes, s);
+  if (st != MF_OK) return st;
+  Exec<E> ex(h, plan, s);
+  MF_CUDA(h, cudaMemcpyAsync(ex.theta_slot(0), theta0, h->P * 4, cudaMemcpyDeviceToDevice, s));
+  const int64_t ne = n_eta_of(h, lp);
+  MF_CUDA(h, cudaMemsetAsync(d_eta, 0, ne * 4, s));
+
+  // 1. rollout with the theta_t store
+  float* thT = nullptr;
+  rollout<E>(ex, lp, eta, inner_x, inner_y, lr, true, &thT);
+  if (ex.st != MF_OK) return ex.st;
+
+  // 2. outer gradient theta_bar_T = grad V(theta_T)  (Eq. 4)
+  float* tbar = ex.template at<float>(plan.o_tbar);
+  float* u = ex.template at<float>(plan.o_u);
+  float* Hu = ex.template at<float>(plan.o_g);
+  float* part = ex.template at<float>(plan.o_part);
+  ex.cast_params(thT, false);
+  ex.forward(Bo, static_cast<const E*>(outer_x), thT, nullptr, false);
+  ex.loss(Bo, false, outer_y, nullptr, nullptr, ex.template at<float>(plan.o_l), nullptr, nullptr);
+  ex.backward(Bo, false, nullptr, tbar);
+  if (outer_loss) {
+    mf::sum_scaled(ex.template at<float>(plan.o_l), Bo, 1.f / Bo, outer_loss, s);
+    ex.launched();
+  }
+  float* d_plr = lr.off_plr >= 0 ? d_eta + lr.off_plr : nullptr;
+  // u_{T-1} = -lr theta_bar_T ;  d eta_lr += -lr m_T theta_bar_T
+  mf::adjoint_update(h->P, tbar, nullptr, lr.lr_meta ? ex.m_slot(T - 1) : nullptr, nullptr, u,
+                     lp->momentum, lr.lr, d_plr, scalar_lr ? part + (T - 1) * plan.nb : nullptr,
+                     plan.nb, h->d_status, s);
+  ex.launched();
+
+  // 3. reverse sweep t = T-1..0 with forward-over-reverse Hessian-vector products
+  const int din = h->dims[0];
+  const size_t xs = static_cast<size_t>(B) * din * (h->bf16 ? 2 : 4);
+  const size_t ys = y_stride_bytes(h, B);
+  for (int t = T - 1; t >= 0; --t) {
+    const float* th = ex.theta_slot(t);
+    const E* x = reinterpret_cast<const E*>(static_cast<const char*>(inner_x) + xs * t);
+    const void* y = static_cast<const char*>(inner_y) + ys * t;
+    ex.cast_params(th, false);
+    ex.cast_params(u, true);
+    ex.forward(B, x, th, u, true);
+    const bool exw = lp->meta_kind & MF_META_EXAMPLE_WEIGHTS;
+    const float* ew = exw ? eta + static_cast<int64_t>(t) * B : nullptr;
+    float* de = exw ? d_eta + static_cast<int64_t>(t) * B : nullptr;
+    ex.loss(B, true, y, ew, nullptr, nullptr, ex.template at<float>(plan.o_ld), de);
+    ex.backward(B, true, Hu, nullptr);
+    if (t > 0) {
+      // theta_bar_t = theta_bar_{t+1} + H u ; d eta_lr += -lr m_t theta_bar_t ;
+      // u_{t-1} = mu u_t - lr theta_bar_t
+      mf::adjoint_update(h->P, tbar, Hu, lr.lr_meta ? ex.m_slot(t - 1) : nullptr, u, u,
+                         lp->momentum, lr.lr, d_plr,
+                         scalar_lr ? part + (t - 1) * plan.nb : nullptr, plan.nb, h->d_status, s);
+    } else {
+      mf::adjoint_update(h->P, tbar, Hu, nullptr, nullptr, nullptr, lp->momentum, lr.lr, nullptr,
+                         nullptr, 0, h->d_status, s);
+    }
+    ex.launched();
+    if (ex.st != MF_OK) return ex.st;
+  }
+  if (scalar_lr) {
+    mf::sum_scaled(part, T * plan.nb, 1.f, d_eta + lr.off_slr, s);
+    ex.launched();
+  }
+  if (d_theta0) MF_CUDA(h, cudaMemcpyAsync(d_theta0, tbar, h->P * 4, cudaMemcpyDeviceToDevice, s));
+  MF_CUDA(h, cudaGetLastError());
+  return ex.st;
+}
+
+template <typename E>
+mf_status rollout_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0, const float* eta,
+                       const void* inner_x, const void* inner_y, float* thetaT, cudaStream_t s) {
+  const LrSel lr = lr_select(h, lp, eta);
+  Plan plan = make_plan(h, lp->B, lp->T, 2, lr.lr_meta ? 1 : 0, false);
+  mf_status st = ensure_ws(h, plan.bytes, s);
+  if (st != MF_OK) return st;
+  Exec<E> ex(h, plan, s);
+  MF_CUDA(h, cudaMemcpyAsync(ex.theta_slot(0), theta0, h->P * 4, cudaMemcpyDeviceToDevice, s));
+  // with the learning rate as a meta-parameter the ping-pong variant keeps m in m slot 0
+  float* thT = nullptr;
+  rollout<E>(ex, lp, eta, inner_x, inner_y, lr, false, &thT);
+  if (ex.st != MF_OK) return ex.st;
+  MF_CUDA(h, cudaMemcpyAsync(thetaT, thT, h->P * 4, cudaMemcpyDeviceToDevice, s));
+  return MF_OK;
+}
+
+template <typename E>
+mf_status hvp_impl(mf_ctx* h, int B, const float* theta, const void* x, const void* y,
+                   const float* ex_w, const float* v, float* Hv, float* tl, float* grad,
+                   cudaStream_t s) {
+  Plan plan = make_plan(h, B, 1, 0, 0, false);
+  mf_status st = ensure_ws(h, plan.bytes, s);
+  if (st != MF_OK) return st;
+  Exec<E> ex(h, plan, s);
+  ex.cast_params(theta, false);
+  ex.cast_params(v, true);
+  ex.forward(B, static_cast<const E*>(x), theta, v, true);
+  ex.loss(B, true, y, nullptr, ex_w, nullptr, tl, nullptr);
+  ex.backward(B, true, Hv, grad);
+  MF_CUDA(h, cudaGetLastError());
+  return ex.st;
+}
+
+}  // namespace
+
+// ======================================= C ABI ============================================
+extern "C" {
+
+const char* mf_status_string(mf_status s) {
+  switch (s) {
+    case MF_OK: return "ok";
+    case MF_ERR_INVALID_ARG: return "invalid argument";
+    case MF_ERR_UNSUPPORTED: return "unsupported";
+    case MF_ERR_OOM: return "out of memory";
+    case MF_ERR_CUDA: return "CUDA error";
+    case MF_ERR_NONFINITE: return "non-finite value";
+    case MF_ERR_TIMEOUT: return "device wait timed out";
+  }
+  return "unknown status";
+}
+
+const char* mf_last_error(mf_handle h) { return h ? h->err.c_str() : "NULL handle"; }
+
+mf_status mf_create(const mf_model_desc* d, mf_handle* out) {
+  if (!d || !out) return MF_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (d->arch == MF_ARCH_DECODER) return MF_ERR_UNSUPPORTED;
+  if (d->arch != MF_ARCH_MLP) return MF_ERR_INVALID_ARG;
+  if (d->n_layers < 1 || d->n_layers > MF_MAX_LAYERS) return MF_ERR_INVALID_ARG;
+  for (int i = 0; i <= d->n_layers; ++i)
+    if (d->dims[i] < 1 || d->dims[i] > (1 << 20)) return MF_ERR_INVALID_ARG;
+  if (d->act < MF_ACT_IDENT || d->act > MF_ACT_SILU) return MF_ERR_INVALID_ARG;
+  if (d->loss != MF_LOSS_SQUARED && d->loss != MF_LOSS_SOFTMAX_CE) {
+    return d->loss == MF_LOSS_NEXT_TOKEN_CE ? MF_ERR_UNSUPPORTED : MF_ERR_INVALID_ARG;
+  }
+  if (d->precision != MF_PREC_FP32 && d->precision != MF_PREC_BF16) return MF_ERR_INVALID_ARG;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) { cudaGetLastError(); return MF_ERR_CUDA; }
+  mf_ctx* h = new mf_ctx();
+  h->md = *d;
+  h->L = d->n_layers;
+  h->dims.assign(d->dims, d->dims + d->n_layers + 1);
+  int64_t o = 0;
+  for (int l = 0; l < h->L; ++l) {
+    h->woff.push_back(o);
+    o += static_cast<int64_t>(h->dims[l]) * h->dims[l + 1];
+    h->boff.push_back(d->has_bias ? o : -1);
+    if (d->has_bias) o += h->dims[l + 1];
+  }
+  h->P = o;
+  h->maxd = *std::max_element(h->dims.begin(), h->dims.end());
+  h->bf16 = d->precision == MF_PREC_BF16;
+  if (cudaMalloc(&h->d_status, sizeof(int)) != cudaSuccess ||
+      cudaMemset(h->d_status, 0, sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    delete h;
+    return MF_ERR_CUDA;
+  }
+  *out = h;
+  return MF_OK;
+}
+
+mf_status mf_destroy(mf_handle h) {
+  if (!h) return MF_ERR_INVALID_ARG;
+  cudaDeviceSynchronize();
+  release_ws(h);
+  for (auto& e : h->evs) { cudaEventDestroy(e.first); cudaEventDestroy(e.second); }
+  if (h->d_status) cudaFree(h->d_status);
+  delete h;
+  return MF_OK;
+}
+
+mf_status mf_set_allocator(mf_handle h, void* (*alloc)(size_t, void*, void*),
+                           void (*free_fn)(void*, size_t, void*, void*), void* ctx) {
+  if (!h) return MF_ERR_INVALID_ARG;
+  if ((alloc == nullptr) != (free_fn == nullptr))
+    return fail(h, MF_ERR_INVALID_ARG, "alloc and free must both be set or both NULL");
+  release_ws(h);
+  h->ualloc = alloc;
+  h->ufree = free_fn;
+  h->uctx = ctx;
+  return MF_OK;
+}
+
+mf_status mf_param_count(mf_handle h, const mf_loop_desc* lp, int64_t* n_params, int64_t* n_eta) {
+  if (!h) return MF_ERR_INVALID_ARG;
+  if (n_params) *n_params = h->P;
+  if (n_eta) *n_eta = lp ? n_eta_of(h, lp) : 0;
+  return MF_OK;
+}
+
+mf_status mf_workspace_bytes(mf_handle h, const mf_loop_desc* lp, size_t* bytes) {
+  if (!h || !bytes) return MF_ERR_INVALID_ARG;
+  mf_status st = validate_loop(h, lp);
+  if (st != MF_OK) return st;
+  const bool lr_meta = lp->meta_kind & (MF_META_PARAM_LOGLR | MF_META_SCALAR_LOGLR);
+  *bytes = make_plan(h, std::max(lp->B, lp->B_outer), lp->T, lp->T + 1, lr_meta ? lp->T : 0,
+                     lp->meta_kind & MF_META_SCALAR_LOGLR).bytes;
+  return MF_OK;
+}
+
+mf_status mf_release_workspace(mf_handle h) {
+  if (!h) return MF_ERR_INVALID_ARG;
+  release_ws(h);
+  return MF_OK;
+}
+
+mf_status mf_inner_rollout(mf_handle h, const mf_loop_desc* lp, const float* theta0,
+                           const float* eta, const void* inner_x, const void* inner_y,
+                           float* thetaT, void* stream) {
+  if (!h) return MF_ERR_INVALID_ARG;
+  mf_status st = validate_loop(h, lp);
+  if (st != MF_OK) return st;
+  if (!theta0 || !inner_x || !inner_y || !thetaT || (n_eta_of(h, lp) > 0 && !eta))
+    return fail(h, MF_ERR_INVALID_ARG, "NULL tensor argument");
+  if ((st = check_x(h, inner_x, lp->B)) != MF_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  h->last_stream = s;
+  return h->bf16 ? rollout_impl<__nv_bfloat16>(h, lp, theta0, eta, inner_x, inner_y, thetaT, s)
+                 : rollout_impl<float>(h, lp, theta0, eta, inner_x, inner_y, thetaT, s);
+}
+
+mf_status mf_hvp(mf_handle h, int B, const float* theta, const void* x, const void* y,
+                 const float* ex_w, const float* v, float* Hv, float* tangent_losses, float* grad,
+                 int hvp_mode, void* stream) {
+  if (!h) return MF_ERR_INVALID_ARG;
+  if (B < 1) return fail(h, MF_ERR_INVALID_ARG, "B must be >= 1");
+  if (hvp_mode != MF_HVP_MIXED_FOR) return fail(h, MF_ERR_UNSUPPORTED, "only MF_HVP_MIXED_FOR is implemented");
+  if (!theta || !x || !y || !v || !Hv) return fail(h, MF_ERR_INVALID_ARG, "NULL tensor argument");
+  mf_status st = check_x(h, x, B);
+  if (st != MF_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  h->last_stream = s;
+  return h->bf16 ? hvp_impl<__nv_bfloat16>(h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, s)
+                 : hvp_impl<float>(h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, s);
+}
+
+mf_status mf_meta_grad(mf_handle h, const mf_loop_desc* lp, const float* theta0, const float* eta,
+                       const void* inner_x, const void* inner_y, const void* outer_x,
+                       const void* outer_y, float* d_eta, float* d_theta0, float* outer_loss,
+                       void* stream) {
+  if (!h) return MF_ERR_INVALID_ARG;
+  mf_status st = validate_loop(h, lp);
+  if (st != MF_OK) return st;
+  if (!theta0 || !inner_x || !inner_y || !outer_x || !outer_y)
+    return fail(h, MF_ERR_INVALID_ARG, "NULL tensor argument");
+  if (n_eta_of(h, lp) > 0 && (!eta || !d_eta))
+    return fail(h, MF_ERR_INVALID_ARG, "eta and d_eta are required when meta_kind != 0");
+  if (n_eta_of(h, lp) == 0 && !d_theta0)
+    return fail(h, MF_ERR_INVALID_ARG, "nothing to compute: meta_kind = 0 and d_theta0 = NULL");
+  if ((st = check_x(h, inner_x, lp->B)) != MF_OK) return st;
+  if ((st = check_x(h, outer_x, lp->B_outer)) != MF_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  h->last_stream = s;
+  return h->bf16 ? meta_grad_impl<__nv_bfloat16>(h, lp, theta0, eta, inner_x, inner_y, outer_x,
+                                                 outer_y, d_eta, d_theta0, outer_loss, s)
+                 : meta_grad_impl<float>(h, lp, theta0, eta, inner_x, inner_y, outer_x, outer_y,
+                                         d_eta, d_theta0, outer_loss, s);
+}
+
+mf_status mf_sync(mf_handle h) {
+  if (!h) return MF_ERR_INVALID_ARG;
+  cudaError_t e = cudaStreamSynchronize(h->last_stream);
+  if (e != cudaSuccess) return fail(h, MF_ERR_CUDA, std::string("stream: ") + cudaGetErrorString(e));
+  int v = 0;
+  e = cudaMemcpy(&v, h->d_status, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return fail(h, MF_ERR_CUDA, std::string("status read: ") + cudaGetErrorString(e));
+  if (h->fault == 2) { h->fault = 0; v = mf::DEV_TIMEOUT; }
+  if (v != 0) {
+    cudaMemset(h->d_status, 0, sizeof(int));
+    if (v == mf::DEV_TIMEOUT) return fail(h, MF_ERR_TIMEOUT, "a device-side wait ran out of time");
+    if (v == mf::DEV_NONFINITE) return fail(h, MF_ERR_NONFINITE, "non-finite value in the adjoint or the parameters");
+    if (v == 1) return fail(h, MF_ERR_INVALID_ARG, "a class label is out of range");
+    return fail(h, MF_ERR_CUDA, "device status " + std::to_string(v));
+  }
+  return MF_OK;
+}
+
+mf_status mf_stats(mf_handle h, uint64_t* launches, size_t* peak) {
+  if (!h) return MF_ERR_INVALID_ARG;
+  if (launches) *launches = h->launches;
+  if (peak) *peak = h->peak;
+  return MF_OK;
+}
+
+mf_status mf_set_kernel_timing(mf_handle h, int enable) {
+  if (!h) return MF_ERR_INVALID_ARG;
+  h->timing = enable != 0;
+  return MF_OK;
+}
+
+mf_status mf_kernel_time(mf_handle h, double* ms, uint64_t* launches, double* flops) {
+  if (!h) return MF_ERR_INVALID_ARG;
+  double tot = 0.0;
+  uint64_t n = 0;
+  if (!h->evs.empty()) {
+    cudaError_t e = cudaEventSynchronize(h->evs.back().second);
+    if (e != cudaSuccess) return fail(h, MF_ERR_CUDA, cudaGetErrorString(e));
+  }
+  for (auto& pr : h->evs) {
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, pr.first, pr.second) == cudaSuccess) { tot += t; ++n; }
+    cudaEventDestroy(pr.first);
+    cudaEventDestroy(pr.second);
+  }
+  h->evs.clear();
+  if (ms) *ms = tot;
+  if (launches) *launches = n;
+  if (flops) *flops = h->timed_flops;
+  h->timed_flops = 0.0;
+  return MF_OK;
+}
+
+mf_status mf_inject_fault(mf_handle h, int kind) {
+  if (!h || kind < 0 || kind > 2) return MF_ERR_INVALID_ARG;
+  h->fault = kind;
+  return MF_OK;
+}
+
+mf_status mf_dual_gemm_bf16(int M, int N, int K, const void* A0, int lda0, const void* A1,
+                            int lda1, const void* B0, int ldb0, const void* B1, int ldb1,
+                            float* C0, int ldc0, const float* bias0, float* C1, int ldc1,
+                            const float* bias1, unsigned terms, void* stream) {
+  if (M < 1 || N < 1 || K < 1 || (terms & ~31u) || !(terms & 31u)) return MF_ERR_INVALID_ARG;
+  const bool acc0 = terms & (mf::T_C0_A0B0 | mf::T_C0_A1B0 | mf::T_C0_A0B1);
+  const bool acc1 = terms & (mf::T_C1_A1B0 | mf::T_C1_A0B1);
+  if ((acc0 && (!C0 || ldc0 < N)) || (acc1 && (!C1 || ldc1 < N))) return MF_ERR_INVALID_ARG;
+  GemmArgs g;
+  g.M = M; g.N = N; g.K = K;
+  g.A0 = A0; g.lda0 = lda0; g.A1 = A1; g.lda1 = lda1;
+  g.B0 = B0; g.ldb0 = ldb0; g.B1 = B1; g.ldb1 = ldb1;
+  g.C0 = acc0 ? C0 : nullptr; g.ldc0 = ldc0; g.bias0 = bias0;
+  g.C1 = acc1 ? C1 : nullptr; g.ldc1 = ldc1; g.bias1 = bias1;
+  g.terms = terms;
+  const char* why = "";
+  cudaError_t e = mf::tc_gemm(g, static_cast<cudaStream_t>(stream), &why);
+  if (e == cudaErrorInvalidValue) { cudaGetLastError(); return MF_ERR_INVALID_ARG; }
+  return e == cudaSuccess ? MF_OK : MF_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,246 @@
+"""ctypes binding of ``libmixflow.so`` (the C ABI of ``include/mixflow.h``).
+
+Argument marshalling only: every step of the meta-gradient runs in the library's CUDA
+kernels.  Functions keep the C names; ``MixFlow`` wraps a handle and takes torch tensors
+(device memory and streams come from PyTorch).  Importing this module raises if the
+library has not been built - there is no fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", "libmixflow.so")
+
+MF_MAX_LAYERS = 32
+MF_ARCH_MLP, MF_ARCH_DECODER = 0, 1
+ACTS = {"ident": 0, "tanh": 1, "gelu": 2, "silu": 3}
+LOSSES = {"squared": 0, "ce": 1, "next_token_ce": 2}
+PRECISIONS = {"fp32": 0, "bf16": 1}
+MF_META_EXAMPLE_WEIGHTS, MF_META_PARAM_LOGLR, MF_META_SCALAR_LOGLR = 1, 2, 4
+MF_HVP_MIXED_FOR, MF_HVP_REV_REV = 0, 1
+STATUS = {0: "MF_OK", 1: "MF_ERR_INVALID_ARG", 2: "MF_ERR_UNSUPPORTED", 3: "MF_ERR_OOM",
+          4: "MF_ERR_CUDA", 5: "MF_ERR_NONFINITE", 6: "MF_ERR_TIMEOUT"}
+
+# Every symbol include/mixflow.h declares (checked by the CPU test suite).
+EXPORTS = ["mf_create", "mf_destroy", "mf_set_allocator", "mf_param_count",
+           "mf_workspace_bytes", "mf_release_workspace", "mf_inner_rollout", "mf_hvp",
+           "mf_meta_grad", "mf_sync", "mf_status_string", "mf_last_error", "mf_stats",
+           "mf_set_kernel_timing", "mf_kernel_time", "mf_inject_fault", "mf_dual_gemm_bf16"]
+
+
+class mf_model_desc(C.Structure):
+    _fields_ = [("arch", C.c_int), ("n_layers", C.c_int), ("dims", C.c_int * (MF_MAX_LAYERS + 1)),
+                ("act", C.c_int), ("has_bias", C.c_int), ("loss", C.c_int), ("precision", C.c_int),
+                ("d_model", C.c_int), ("n_heads", C.c_int), ("d_ff", C.c_int), ("vocab", C.c_int),
+                ("seq_len", C.c_int), ("rope_base", C.c_float), ("rms_eps", C.c_float)]
+
+
+class mf_loop_desc(C.Structure):
+    _fields_ = [("T", C.c_int), ("B", C.c_int), ("B_outer", C.c_int), ("alpha", C.c_float),
+                ("momentum", C.c_float), ("meta_kind", C.c_int), ("hvp_mode", C.c_int),
+                ("ckpt_every", C.c_int)]
+
+
+class MixflowError(RuntimeError):
+    def __init__(self, status, msg=""):
+        super().__init__(f"{STATUS.get(status, status)}: {msg}")
+        self.status = status
+
+
+def load(path: str = LIB_PATH) -> C.CDLL:
+    if not os.path.exists(path):
+        raise ImportError(f"native library missing: {path} (run __graft_entry__.build())")
+    lib = C.CDLL(path)
+    vp, i64p, u64p, szp, dblp = C.c_void_p, C.POINTER(C.c_int64), C.POINTER(C.c_uint64), \
+        C.POINTER(C.c_size_t), C.POINTER(C.c_double)
+    H = C.c_void_p
+    sig = {
+        "mf_create": ([C.POINTER(mf_model_desc), C.POINTER(H)], C.c_int),
+        "mf_destroy": ([H], C.c_int),
+        "mf_set_allocator": ([H, vp, vp, vp], C.c_int),
+        "mf_param_count": ([H, C.POINTER(mf_loop_desc), i64p, i64p], C.c_int),
+        "mf_workspace_bytes": ([H, C.POINTER(mf_loop_desc), szp], C.c_int),
+        "mf_release_workspace": ([H], C.c_int),
+        "mf_inner_rollout": ([H, C.POINTER(mf_loop_desc), vp, vp, vp, vp, vp, vp], C.c_int),
+        "mf_hvp": ([H, C.c_int, vp, vp, vp, vp, vp, vp, vp, vp, C.c_int, vp], C.c_int),
+        "mf_meta_grad": ([H, C.POINTER(mf_loop_desc), vp, vp, vp, vp, vp, vp, vp, vp, vp, vp], C.c_int),
+        "mf_sync": ([H], C.c_int),
+        "mf_status_string": ([C.c_int], C.c_char_p),
+        "mf_last_error": ([H], C.c_char_p),
+        "mf_stats": ([H, u64p, szp], C.c_int),
+        "mf_set_kernel_timing": ([H, C.c_int], C.c_int),
+        "mf_kernel_time": ([H, dblp, u64p, dblp], C.c_int),
+        "mf_inject_fault": ([H, C.c_int], C.c_int),
+        "mf_dual_gemm_bf16": ([C.c_int, C.c_int, C.c_int, vp, C.c_int, vp, C.c_int, vp, C.c_int, vp,
+                               C.c_int, vp, C.c_int, vp, vp, C.c_int, vp, C.c_uint, vp], C.c_int),
+    }
+    for name, (args, res) in sig.items():
+        f = getattr(lib, name)
+        f.argtypes = args
+        f.restype = res
+    return lib
+
+
+_lib = None
+
+
+def lib() -> C.CDLL:
+    global _lib
+    if _lib is None:
+        _lib = load()
+    return _lib
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    return C.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return C.c_void_p(stream.cuda_stream)
+
+
+def model_desc_for(w) -> mf_model_desc:
+    """mf_model_desc of a ``synth.Workload`` (MLP)."""
+    d = mf_model_desc()
+    d.arch = MF_ARCH_MLP
+    d.n_layers = len(w.dims) - 1
+    for i, v in enumerate(w.dims):
+        d.dims[i] = v
+    d.act = ACTS[w.act]
+    d.has_bias = 1 if w.has_bias else 0
+    d.loss = LOSSES[w.loss]
+    d.precision = PRECISIONS[w.precision]
+    return d
+
+
+def loop_desc_for(w, hvp_mode: int = MF_HVP_MIXED_FOR) -> mf_loop_desc:
+    l = mf_loop_desc()
+    l.T, l.B, l.B_outer = w.T, w.B, w.B_outer
+    l.alpha, l.momentum = w.alpha, w.momentum
+    l.meta_kind = w.meta_kind
+    l.hvp_mode = hvp_mode
+    l.ckpt_every = 1
+    return l
+
+
+def mf_dual_gemm_bf16(M, N, K, A0, A1, B0, B1, C0, C1, terms, bias0=None, bias1=None,
+                      stream=None):
+    """C0/C1 (float32) = selected products of bf16 K-major operands (see mixflow.h)."""
+    ld = lambda t: (t.stride(0) if t is not None else 0)
+    st = lib().mf_dual_gemm_bf16(M, N, K, _ptr(A0), ld(A0), _ptr(A1), ld(A1), _ptr(B0), ld(B0),
+                                 _ptr(B1), ld(B1), _ptr(C0), ld(C0), _ptr(bias0), _ptr(C1),
+                                 ld(C1), _ptr(bias1), terms, _stream(stream))
+    if st != 0:
+        raise MixflowError(st, "mf_dual_gemm_bf16")
+
+
+class MixFlow:
+    """One library handle for one inner-model architecture."""
+
+    def __init__(self, desc: mf_model_desc):
+        self._lib = lib()
+        self.desc = desc
+        h = C.c_void_p()
+        st = self._lib.mf_create(C.byref(desc), C.byref(h))
+        if st != 0:
+            raise MixflowError(st, "mf_create")
+        self.h = h
+
+    @classmethod
+    def for_workload(cls, w):
+        return cls(model_desc_for(w))
+
+    def close(self):
+        if getattr(self, "h", None):
+            self._lib.mf_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _check(self, st, what):
+        if st != 0:
+            raise MixflowError(st, f"{what}: {self._lib.mf_last_error(self.h).decode()}")
+
+    def param_count(self, loop=None):
+        n, e = C.c_int64(), C.c_int64()
+        self._check(self._lib.mf_param_count(self.h, C.byref(loop) if loop else None,
+                                             C.byref(n), C.byref(e)), "mf_param_count")
+        return n.value, e.value
+
+    def workspace_bytes(self, loop):
+        b = C.c_size_t()
+        self._check(self._lib.mf_workspace_bytes(self.h, C.byref(loop), C.byref(b)),
+                    "mf_workspace_bytes")
+        return b.value
+
+    def release_workspace(self):
+        self._check(self._lib.mf_release_workspace(self.h), "mf_release_workspace")
+
+    def meta_grad(self, loop, theta0, eta, inner_x, inner_y, outer_x, outer_y, d_eta,
+                  d_theta0=None, outer_loss=None, stream=None):
+        st = self._lib.mf_meta_grad(self.h, C.byref(loop), _ptr(theta0), _ptr(eta), _ptr(inner_x),
+                                    _ptr(inner_y), _ptr(outer_x), _ptr(outer_y), _ptr(d_eta),
+                                    _ptr(d_theta0), _ptr(outer_loss), _stream(stream))
+        self._check(st, "mf_meta_grad")
+
+    def inner_rollout(self, loop, theta0, eta, inner_x, inner_y, thetaT, stream=None):
+        st = self._lib.mf_inner_rollout(self.h, C.byref(loop), _ptr(theta0), _ptr(eta),
+                                        _ptr(inner_x), _ptr(inner_y), _ptr(thetaT), _stream(stream))
+        self._check(st, "mf_inner_rollout")
+
+    def hvp(self, B, theta, x, y, v, Hv, ex_w=None, tangent_losses=None, grad=None,
+            hvp_mode=MF_HVP_MIXED_FOR, stream=None):
+        st = self._lib.mf_hvp(self.h, B, _ptr(theta), _ptr(x), _ptr(y), _ptr(ex_w), _ptr(v),
+                              _ptr(Hv), _ptr(tangent_losses), _ptr(grad), hvp_mode, _stream(stream))
+        self._check(st, "mf_hvp")
+
+    def sync(self):
+        self._check(self._lib.mf_sync(self.h), "mf_sync")
+
+    def stats(self):
+        n, p = C.c_uint64(), C.c_size_t()
+        self._check(self._lib.mf_stats(self.h, C.byref(n), C.byref(p)), "mf_stats")
+        return n.value, p.value
+
+    def set_kernel_timing(self, on: bool):
+        self._check(self._lib.mf_set_kernel_timing(self.h, 1 if on else 0), "mf_set_kernel_timing")
+
+    def kernel_time(self):
+        ms, n, fl = C.c_double(), C.c_uint64(), C.c_double()
+        self._check(self._lib.mf_kernel_time(self.h, C.byref(ms), C.byref(n), C.byref(fl)),
+                    "mf_kernel_time")
+        return ms.value, n.value, fl.value
+
+    def inject_fault(self, kind: int):
+        self._check(self._lib.mf_inject_fault(self.h, kind), "mf_inject_fault")
+
+
+def to_device_inputs(w, inp, device="cuda"):
+    """Move a ``synth.Inputs`` to the device with the dtypes the ABI expects."""
+    import torch
+    xdt = torch.bfloat16 if w.precision == "bf16" else torch.float32
+
+    def xt(a):
+        return torch.from_numpy(np.ascontiguousarray(a, np.float32)).to(device).to(xdt).contiguous()
+
+    def yt(a):
+        if a.dtype.kind in "iu":
+            return torch.from_numpy(np.ascontiguousarray(a, np.int32)).to(device)
+        return torch.from_numpy(np.ascontiguousarray(a, np.float32)).to(device)
+
+    f = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.float32)).to(device)
+    return dict(theta0=f(inp.theta0), eta=f(inp.eta), inner_x=xt(inp.inner_x),
+                inner_y=yt(inp.inner_y), outer_x=xt(inp.outer_x), outer_y=yt(inp.outer_y))

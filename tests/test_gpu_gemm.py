@@ -1,0 +1,67 @@
+"""The tcgen05 dual GEMM against float64 products of the same bf16 operands.
+
+Shapes span several 128 x BN tiles, ragged M/N/K tails and every product-term mask the
+sweep uses (primal, dual forward, dual input layer, weight-tangent sum)."""
+import numpy as np
+import pytest
+
+from gpu_util import need_gpu, rel_l2
+
+SHAPES = [(128, 128, 64), (256, 1024, 1024), (256, 10, 1024), (1024, 1024, 512),
+          (77, 45, 136), (130, 300, 8), (512, 4096, 256), (300, 16, 40)]
+MASKS = [1, 1 | 8 | 16, 1 | 16, 2 | 4, 4, 1 | 2 | 4 | 8 | 16]
+
+
+def _ref(A0, A1, B0, B1, mask):
+    a0, a1, b0, b1 = (x.double().cpu() for x in (A0, A1, B0, B1))
+    c0 = None
+    c1 = None
+    terms0 = [(1, a0, b0), (2, a1, b0), (4, a0, b1)]
+    terms1 = [(8, a1, b0), (16, a0, b1)]
+    for bit, a, b in terms0:
+        if mask & bit:
+            c0 = a @ b.T if c0 is None else c0 + a @ b.T
+    for bit, a, b in terms1:
+        if mask & bit:
+            c1 = a @ b.T if c1 is None else c1 + a @ b.T
+    return c0, c1
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("shape", SHAPES)
+@pytest.mark.parametrize("mask", MASKS)
+def test_dual_gemm(shape, mask):
+    torch, native = need_gpu()
+    M, N, K = shape
+    g = torch.Generator(device="cpu").manual_seed(M * 131 + N * 7 + K + mask)
+    mk = lambda r: (torch.randn(r, K, generator=g)).to(torch.bfloat16).cuda()
+    A0, A1, B0, B1 = mk(M), mk(M), mk(N), mk(N)
+    C0 = torch.full((M, N), float("nan"), device="cuda")
+    C1 = torch.full((M, N), float("nan"), device="cuda")
+    bias0 = torch.randn(N, generator=g).cuda()
+    bias1 = torch.randn(N, generator=g).cuda()
+    native.mf_dual_gemm_bf16(M, N, K, A0, A1, B0, B1, C0, C1, mask, bias0, bias1)
+    torch.cuda.synchronize()
+    r0, r1 = _ref(A0, A1, B0, B1, mask)
+    if r0 is not None:
+        r0 = r0 + bias0.double().cpu()
+        assert rel_l2(C0.cpu().numpy(), r0.numpy()) < 1e-5
+    if r1 is not None:
+        r1 = r1 + bias1.double().cpu()
+        assert rel_l2(C1.cpu().numpy(), r1.numpy()) < 1e-5
+
+
+@pytest.mark.gpu
+def test_dual_gemm_strided_operands():
+    """Leading dimensions larger than K (padded operand buffers)."""
+    torch, native = need_gpu()
+    M, N, K, ld = 200, 96, 72, 88
+    g = torch.Generator(device="cpu").manual_seed(3)
+    A0 = torch.randn(M, ld, generator=g).to(torch.bfloat16).cuda()
+    B0 = torch.randn(N, ld, generator=g).to(torch.bfloat16).cuda()
+    C0 = torch.zeros(M, N + 8, device="cuda")
+    native.mf_dual_gemm_bf16(M, N, K, A0, None, B0, None, C0, None, 1)
+    torch.cuda.synchronize()
+    ref = A0[:, :K].double().cpu() @ B0[:, :K].double().cpu().T
+    assert rel_l2(C0[:, :N].cpu().numpy(), ref.numpy()) < 1e-5
+    assert float(C0[:, N:].abs().max()) == 0.0
