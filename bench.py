@@ -1,0 +1,297 @@
+"""Benchmark: mixed-mode (forward-over-reverse) Truncated-BPTT meta-gradient steps per second.
+
+One step = one full ``mf_meta_grad`` call on the "wide" workload: a 1024-wide, 4-hidden-layer
+GELU MLP with a 10-class softmax head, B = 256 examples per inner step, T = 16 SGD steps
+(alpha = 0.05), per-example weight logits (T*B = 4096 meta-parameters), outer batch 1024,
+bf16 tensor-core GEMMs with float32 accumulation and float32 parameters/adjoints.  Inputs are
+seeded synthetic data resident in HBM when the timed region starts.
+
+Prints one JSON line (rank 0).  ``--impl reference`` times the CPU float64 oracle instead.
+Multi-GPU runs are independent replicas (weak scaling), one process per GPU under torchrun.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = "wide"
+REF_T_SAMPLE = 4
+WORKLOAD_DESC = ("wide MLP 1024-1024x4-10 GELU, softmax-CE, B=256, T=16 SGD alpha=0.05, "
+                 "per-example weight logits (4096), outer batch 1024, bf16 GEMMs / fp32 state")
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return p, "measured"
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", "-i", str(gpu_index), f"--query-gpu={self.Q}",
+                                       "--format=csv,noheader,nounits", "-lms", "200"],
+                                      stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return None
+        self.p.terminate()
+        try:
+            self.p.wait(timeout=5)
+        except Exception:
+            self.p.kill()
+        self.f.seek(0)
+        rows = [r.split(",") for r in self.f.read().strip().splitlines() if r.strip()]
+        os.unlink(self.f.name)
+        sm, smax, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            r = [x.strip() for x in r]
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                smax = max(smax, float(r[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, r[5:9]):
+                if v.lower() in ("active", "1", "yes"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def cpu_oracle_time(w, t_sample=None):
+    """Wall time of the float64 oracle meta-gradient on workload w, run on the first
+    ``t_sample`` inner steps (all T when None) and scaled by T / t_sample.  Scaling also
+    multiplies the outer-gradient part, so a sampled figure over-states the oracle's time
+    slightly.  Returns (seconds for the full workload, seconds spent, threads)."""
+    import torch
+    from paper_2505_00793_gb300 import synth
+    from oracle import metagrad as om
+    ts = w.T if t_sample is None else min(t_sample, w.T)
+    ws = w.with_(T=ts)
+    inp = synth.make_inputs(ws)
+    t0 = time.perf_counter()
+    om.meta_grad(ws, inp)
+    spent = time.perf_counter() - t0
+    return spent * w.T / ts, spent, torch.get_num_threads()
+
+
+def run_reference(args):
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return 0
+    from paper_2505_00793_gb300 import synth
+    w = synth.WORKLOADS[WORKLOAD]
+    for _ in range(args.warmup):
+        cpu_oracle_time(w, REF_T_SAMPLE)
+    est = []
+    for _ in range(args.steps):
+        full, spent, cores = cpu_oracle_time(w, REF_T_SAMPLE)
+        est.append(full)
+    ms = 1000.0 * statistics.mean(est)
+    value = 1000.0 / ms
+    sample = (f"per step: oracle meta-gradient over the first {REF_T_SAMPLE} of the 16 inner "
+              f"steps of the same workload, time scaled by 16/{REF_T_SAMPLE}")
+    print(json.dumps({
+        "impl": "reference", "metric": "meta-grad steps/s", "value": value, "unit": "meta-steps/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": WORKLOAD_DESC},
+        "cpu_baseline": {"value": value, "unit": "meta-steps/s", "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "meta-steps/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }), flush=True)
+    return 0
+
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+    from paper_2505_00793_gb300 import native, synth
+
+    ws, rank, local = _dist()
+    torch.cuda.set_device(local)
+    if ws > 1:
+        dist.init_process_group("nccl")
+    w = synth.WORKLOADS[WORKLOAD]
+    inp = synth.make_inputs(w)
+    d = native.to_device_inputs(w, inp)
+    mf = native.MixFlow.for_workload(w)
+    loop = native.loop_desc_for(w)
+    d_eta = torch.empty(w.n_eta, device="cuda")
+    V = torch.empty(1, device="cuda")
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(256 * 1024 * 1024 // 4, device="cuda")   # > 129 MB L2
+
+    def step():
+        mf.meta_grad(loop, d["theta0"], d["eta"], d["inner_x"], d["inner_y"], d["outer_x"],
+                     d["outer_y"], d_eta, None, V, stream=stream)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    mf.sync()
+
+    def barrier():
+        if ws > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    # ---- timed region: K steps, L2 flushed before each (outside the step's events) -------
+    clk = ClockSampler(local)
+    time.sleep(0.3)
+    launches0, _ = mf.stats()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    barrier()
+    for e0, e1 in evs:
+        flush.fill_(1.0)
+        e0.record(stream)
+        step()
+        e1.record(stream)
+    barrier()
+    clocks = clk.stop()
+    mf.sync()
+    launches1, peak_ws = mf.stats()
+    ms_steps = [e0.elapsed_time(e1) for e0, e1 in evs]
+    total_ms = sum(ms_steps)
+    if ws > 1:
+        t = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t)
+    ms_per_step = total_ms / args.steps
+    value = ws * 1000.0 / ms_per_step
+
+    # ---- dominant kernel (tcgen05 dual GEMM): per-launch CUDA events over the same steps ---
+    mf.set_kernel_timing(True)
+    mf.kernel_time()
+    for _ in range(args.steps):
+        flush.fill_(1.0)
+        step()
+    mf.sync()
+    g_ms, g_n, g_flops = mf.kernel_time()
+    mf.set_kernel_timing(False)
+    peaks, peak_src = _peaks()
+    g_tflops = g_flops / (g_ms * 1e-3) / 1e12 if g_ms > 0 else 0.0
+    peak_tc = peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"])
+
+    # ---- end to end through the public API with host buffers -------------------------------
+    pin = {k: v.cpu().pin_memory() for k, v in d.items()}
+    h_eta = torch.empty(w.n_eta, pin_memory=True)
+    h_V = torch.empty(1, pin_memory=True)
+    h2d = sum(v.numel() * v.element_size() for v in pin.values())
+    d2h = h_eta.numel() * 4 + 4
+    for _ in range(2):
+        for k in d:
+            d[k].copy_(pin[k], non_blocking=True)
+        step()
+        h_eta.copy_(d_eta, non_blocking=True)
+        h_V.copy_(V, non_blocking=True)
+    barrier()
+    e_evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+             for _ in range(args.steps)]
+    for e0, e1 in e_evs:
+        flush.fill_(1.0)
+        e0.record(stream)
+        for k in d:
+            d[k].copy_(pin[k], non_blocking=True)
+        step()
+        h_eta.copy_(d_eta, non_blocking=True)
+        h_V.copy_(V, non_blocking=True)
+        e1.record(stream)
+    barrier()
+    e2e_ms = sum(e0.elapsed_time(e1) for e0, e1 in e_evs) / args.steps
+    if ws > 1:
+        t = torch.tensor([e2e_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t)
+    mf.sync()
+
+    inputs_bytes = h2d
+    peak_hbm_gb = (peak_ws + inputs_bytes + w.n_eta * 4) / 1e9
+
+    out = None
+    if rank == 0:
+        cpu = None
+        if ws == 1 and not args.no_cpu_baseline:
+            full_s, spent, cores = cpu_oracle_time(w)
+            cpu = {"value": 1.0 / full_s, "unit": "meta-steps/s", "cores": cores, "kind": "oracle",
+                   "sample": f"one full oracle meta-gradient of the workload (T=16, {spent:.1f} s "
+                             "of CPU work)"}
+        out = {
+            "metric": "meta-grad steps/s", "value": value, "unit": "meta-steps/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD_DESC, "parallelism": f"replicas x{ws}",
+                       "l2": "flushed before every timed step (256 MB write outside the step events)"},
+            "roofline": {"bound": "tensor", "kernel": "tc_dual_gemm_kernel (tcgen05 dual GEMM)",
+                         "achieved": g_tflops, "peak": peak_tc, "unit": "TFLOP/s",
+                         "frac": g_tflops / peak_tc, "traffic": None,
+                         "peak_source": f"{peak_src} bf16_tflops_sustained",
+                         "launches_per_step": g_n / max(args.steps, 1),
+                         "avg_launch_us": 1000.0 * g_ms / max(g_n, 1),
+                         "share_of_step": g_ms / args.steps / ms_per_step},
+            "hvp_tflops": g_tflops,
+            "peak_hbm_gb": peak_hbm_gb,
+            "cpu_baseline": cpu,
+            "e2e": {"value": ws * 1000.0 / e2e_ms, "unit": "meta-steps/s",
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": int(launches1 - launches0),
+            "clocks": clocks,
+        }
+        print(json.dumps(out), flush=True)
+    mf.close()
+    if ws > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="mixflow", choices=["mixflow", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())
