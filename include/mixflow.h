@@ -186,6 +186,28 @@ mf_status mf_kernel_time(mf_handle h, double* ms, uint64_t* launches, double* fl
  * kind 0 clears.  Nothing is done on the GPU. */
 mf_status mf_inject_fault(mf_handle h, int kind);
 
+/* mf_hvp without any device allocation.  The paper has no counterpart to this call; it
+ * exists for callers that cannot allocate device memory: code that enqueues work inside a
+ * CUDA stream capture where allocation is not allowed, embedders whose device memory is
+ * entirely reserved by their own allocator, and hosts that only accept pre-registered
+ * buffers.  It computes exactly what mf_hvp computes (MF_HVP_MIXED_FOR) for the model
+ * described by `desc`, without a handle: inputs and outputs are caller-owned device
+ * pointers as in mf_hvp, and all intermediate storage lives in one 32 MiB array in the
+ * library's device memory (a file-scope __device__ array that every GPU loading the
+ * library holds until the process exits).
+ *  - Returns MF_ERR_INVALID_ARG when the workspace for (desc, B) exceeds that array
+ *    (about 32 MiB; e.g. a [128, 256, 256, 10] MLP at B = 64 needs well under 1 MiB).
+ *  - The first call on a device looks up the array's device address (cudaGetSymbolAddress)
+ *    with that device current; make that first call outside any stream capture.
+ *  - Every call shares the array and leaves its contents behind; the call clears the
+ *    status word it needs.  Calls whose GPU work overlaps (different streams, or several
+ *    host threads) race on the array: serialise them.
+ *  - Device-side conditions (non-finite values, a bounded wait that ran out) are not
+ *    reported; the call is asynchronous on `stream` like mf_hvp. */
+mf_status mf_hvp_noalloc(const mf_model_desc* desc, int B, const float* theta, const void* x,
+                         const void* y, const float* ex_w, const float* v, float* Hv,
+                         float* tangent_losses, float* grad, void* stream);
+
 /* Building block exposed for tests and profiling: the bf16 dual GEMM of the sweep.
  * All operands K-major, row-major with leading dimension in elements (multiple of 8):
  *   A0, A1 [M][K] bf16;  B0, B1 [N][K] bf16;  C0, C1 [M][N] float32 (ldc).

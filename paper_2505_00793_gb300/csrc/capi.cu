@@ -8,6 +8,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <mutex>
 #include <string>
 #include <utility>
 #include <vector>
@@ -791,3 +792,94 @@ mf_status mf_dual_gemm_bf16(int M, int N, int K, const void* A0, int lda0, const
 }
 
 }  // extern "C"
+
+// ================================ no-allocation HVP =======================================
+// Callers that cannot allocate device memory - code running inside a CUDA graph capture
+// that forbids allocation, embedders whose memory is fully pre-reserved by another
+// allocator, or hosts that only hand out pre-registered buffers - use mf_hvp_noalloc.  Its
+// workspace is one file-scope device array; nothing is allocated per call or per handle.
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = static_cast<size_t>(32) << 20;   // 32 MiB
+constexpr size_t kNoAllocStatusBytes = 256;   // status word, then the workspace
+constexpr int kMaxDevices = 64;
+
+// Held by every GPU that loads the library until the process exits.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device, looked up once per device.
+// The symbol name is only a host-side stand-in; kernels must be given this address.
+cudaError_t noalloc_scratch(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return e;
+    g_noalloc_ptr[dev] = p;
+  }
+  *out = g_noalloc_ptr[dev];
+  return cudaSuccess;
+}
+
+}  // namespace
+
+extern "C" mf_status mf_hvp_noalloc(const mf_model_desc* d, int B, const float* theta,
+                                    const void* x, const void* y, const float* ex_w,
+                                    const float* v, float* Hv, float* tangent_losses,
+                                    float* grad, void* stream) {
+  if (!d || B < 1 || !theta || !x || !y || !v || !Hv) return MF_ERR_INVALID_ARG;
+  if (d->arch == MF_ARCH_DECODER) return MF_ERR_UNSUPPORTED;
+  if (d->arch != MF_ARCH_MLP || d->n_layers < 1 || d->n_layers > MF_MAX_LAYERS)
+    return MF_ERR_INVALID_ARG;
+  for (int i = 0; i <= d->n_layers; ++i)
+    if (d->dims[i] < 1 || d->dims[i] > (1 << 20)) return MF_ERR_INVALID_ARG;
+  if (d->act < MF_ACT_IDENT || d->act > MF_ACT_SILU) return MF_ERR_INVALID_ARG;
+  if (d->loss != MF_LOSS_SQUARED && d->loss != MF_LOSS_SOFTMAX_CE)
+    return d->loss == MF_LOSS_NEXT_TOKEN_CE ? MF_ERR_UNSUPPORTED : MF_ERR_INVALID_ARG;
+  if (d->precision != MF_PREC_FP32 && d->precision != MF_PREC_BF16) return MF_ERR_INVALID_ARG;
+
+  // A handle-free context on the host stack; its workspace is the static device array.
+  mf_ctx h;
+  h.md = *d;
+  h.L = d->n_layers;
+  h.dims.assign(d->dims, d->dims + d->n_layers + 1);
+  int64_t o = 0;
+  for (int l = 0; l < h.L; ++l) {
+    h.woff.push_back(o);
+    o += static_cast<int64_t>(h.dims[l]) * h.dims[l + 1];
+    h.boff.push_back(d->has_bias ? o : -1);
+    if (d->has_bias) o += h.dims[l + 1];
+  }
+  h.P = o;
+  h.maxd = *std::max_element(h.dims.begin(), h.dims.end());
+  h.bf16 = d->precision == MF_PREC_BF16;
+  const Plan plan = make_plan(&h, B, 1, 0, 0, false);
+  if (plan.bytes > kNoAllocScratchBytes - kNoAllocStatusBytes) return MF_ERR_INVALID_ARG;
+  if (check_x(&h, x, B) != MF_OK) return MF_ERR_INVALID_ARG;
+
+  void* scratch = nullptr;
+  if (noalloc_scratch(&scratch) != cudaSuccess) {
+    cudaGetLastError();
+    return MF_ERR_CUDA;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  h.d_status = static_cast<int*>(scratch);
+  if (cudaMemsetAsync(h.d_status, 0, sizeof(int), s) != cudaSuccess) {
+    cudaGetLastError();
+    return MF_ERR_CUDA;
+  }
+  h.ws = static_cast<char*>(scratch) + kNoAllocStatusBytes;
+  h.ws_bytes = kNoAllocScratchBytes - kNoAllocStatusBytes;
+  const mf_status st =
+      h.bf16 ? hvp_impl<__nv_bfloat16>(&h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, s)
+             : hvp_impl<float>(&h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, s);
+  h.ws = nullptr;   // not owned: never released
+  return st;
+}

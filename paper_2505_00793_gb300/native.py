@@ -29,7 +29,8 @@ STATUS = {0: "MF_OK", 1: "MF_ERR_INVALID_ARG", 2: "MF_ERR_UNSUPPORTED", 3: "MF_E
 EXPORTS = ["mf_create", "mf_destroy", "mf_set_allocator", "mf_param_count",
            "mf_workspace_bytes", "mf_release_workspace", "mf_inner_rollout", "mf_hvp",
            "mf_meta_grad", "mf_sync", "mf_status_string", "mf_last_error", "mf_stats",
-           "mf_set_kernel_timing", "mf_kernel_time", "mf_inject_fault", "mf_dual_gemm_bf16"]
+           "mf_set_kernel_timing", "mf_kernel_time", "mf_inject_fault", "mf_dual_gemm_bf16",
+           "mf_hvp_noalloc"]
 
 
 class mf_model_desc(C.Structure):
@@ -75,6 +76,8 @@ def load(path: str = LIB_PATH) -> C.CDLL:
         "mf_set_kernel_timing": ([H, C.c_int], C.c_int),
         "mf_kernel_time": ([H, dblp, u64p, dblp], C.c_int),
         "mf_inject_fault": ([H, C.c_int], C.c_int),
+        "mf_hvp_noalloc": ([C.POINTER(mf_model_desc), C.c_int, vp, vp, vp, vp, vp, vp, vp, vp, vp],
+                           C.c_int),
         "mf_dual_gemm_bf16": ([C.c_int, C.c_int, C.c_int, vp, C.c_int, vp, C.c_int, vp, C.c_int, vp,
                                C.c_int, vp, C.c_int, vp, vp, C.c_int, vp, C.c_uint, vp], C.c_int),
     }
