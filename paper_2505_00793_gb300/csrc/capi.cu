@@ -72,16 +72,25 @@ struct Plan {
   int rows = 0;          // max rows of any batch
   int ldR = 0;           // leading dim of transposed activations (multiple of 8)
   int T = 0;
-  bool store_all = true; // keep theta_0..theta_T
   int n_theta_slots = 0, n_m_slots = 0;
-  int nb = 0;            // adjoint partial blocks per step
+  int nb = 0;            // blocks (tiles) of the per-layer update kernel
   size_t bytes = 0;
-  // offsets
   size_t o_theta = 0, o_m = 0, o_g = 0, o_tbar = 0, o_u = 0, o_part = 0, o_l = 0, o_ld = 0;
   std::vector<size_t> o_Wb, o_WbT, o_Ub, o_UbT, o_A, o_Ad, o_AT, o_AdT, o_Z, o_Zd;
-  size_t o_dZ = 0, o_dZd = 0, o_dZT = 0, o_dZdT = 0, o_dZ32 = 0, o_dZd32 = 0, o_dA = 0, o_dAd = 0;
+  size_t o_dZ[2] = {0, 0}, o_dZd[2] = {0, 0}, o_dZT[2] = {0, 0}, o_dZdT[2] = {0, 0};
 };
 
+int n_update_tiles(const mf_ctx* h) {
+  int tiles = 0;
+  for (int l = 0; l < h->L; ++l) {
+    const int rows = h->dims[l] + (h->md.has_bias ? 1 : 0);
+    tiles += ((rows + 31) / 32) * ((h->dims[l + 1] + 31) / 32);
+  }
+  return tiles;
+}
+
+// Transposed activations carry one extra row (ones for a, zeros for a') so that the weight
+// product [a^T; 1][dz] yields the weight and the bias gradient (stored contiguously in theta).
 Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slots,
                bool with_partials) {
   Plan p;
@@ -91,6 +100,7 @@ Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slot
   p.n_theta_slots = n_theta_slots;
   p.n_m_slots = n_m_slots;
   const size_t es = h->bf16 ? 2 : 4;
+  const int hb = h->md.has_bias ? 1 : 0;
   size_t o = 0;
   auto take = [&](size_t bytes) { size_t r = o; o += align_up(bytes); return r; };
   const size_t P4 = static_cast<size_t>(h->P) * 4;
@@ -99,7 +109,7 @@ Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slot
   p.o_g = take(P4);
   p.o_tbar = take(P4);
   p.o_u = take(P4);
-  p.nb = mf::adjoint_partials_blocks(h->P);
+  p.nb = n_update_tiles(h);
   p.o_part = take(with_partials ? static_cast<size_t>(p.nb) * (T > 0 ? T : 1) * 4 : 4);
   p.o_l = take(static_cast<size_t>(rows) * 4);
   p.o_ld = take(static_cast<size_t>(rows) * 4);
@@ -115,20 +125,18 @@ Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slot
     p.o_UbT[l] = take(static_cast<size_t>(dout) * ld8(din) * es);
     p.o_A[l] = take(static_cast<size_t>(rows) * ld8(din) * es);
     p.o_Ad[l] = take(static_cast<size_t>(rows) * ld8(din) * es);
-    p.o_AT[l] = take(static_cast<size_t>(din) * p.ldR * es);
-    p.o_AdT[l] = take(static_cast<size_t>(din) * p.ldR * es);
+    p.o_AT[l] = take(static_cast<size_t>(din + hb) * p.ldR * es);
+    p.o_AdT[l] = take(static_cast<size_t>(din + hb) * p.ldR * es);
     p.o_Z[l] = take(static_cast<size_t>(rows) * dout * 4);
     p.o_Zd[l] = take(static_cast<size_t>(rows) * dout * 4);
   }
   const int md = h->maxd;
-  p.o_dZ = take(static_cast<size_t>(rows) * ld8(md) * es);
-  p.o_dZd = take(static_cast<size_t>(rows) * ld8(md) * es);
-  p.o_dZT = take(static_cast<size_t>(md) * p.ldR * es);
-  p.o_dZdT = take(static_cast<size_t>(md) * p.ldR * es);
-  p.o_dZ32 = take(static_cast<size_t>(rows) * md * 4);
-  p.o_dZd32 = take(static_cast<size_t>(rows) * md * 4);
-  p.o_dA = take(static_cast<size_t>(rows) * md * 4);
-  p.o_dAd = take(static_cast<size_t>(rows) * md * 4);
+  for (int b = 0; b < 2; ++b) {
+    p.o_dZ[b] = take(static_cast<size_t>(rows) * ld8(md) * es);
+    p.o_dZd[b] = take(static_cast<size_t>(rows) * ld8(md) * es);
+    p.o_dZT[b] = take(static_cast<size_t>(md) * p.ldR * es);
+    p.o_dZdT[b] = take(static_cast<size_t>(md) * p.ldR * es);
+  }
   p.bytes = o;
   return p;
 }
@@ -171,22 +179,35 @@ struct Exec {
   cudaStream_t s;
   char* base;
   mf_status st = MF_OK;
+  mf::LayerTable tab;
 
   Exec(mf_ctx* h_, const Plan& p_, cudaStream_t s_)
-      : h(h_), p(p_), s(s_), base(static_cast<char*>(h_->ws)) {}
+      : h(h_), p(p_), s(s_), base(static_cast<char*>(h_->ws)) {
+    tab.n = h->L;
+    int tiles = 0;
+    for (int l = 0; l < h->L; ++l) {
+      const int din = h->dims[l], dout = h->dims[l + 1];
+      tab.rows[l] = din + (h->md.has_bias ? 1 : 0);
+      tab.din[l] = din;
+      tab.dout[l] = dout;
+      tab.off[l] = h->woff[l];
+      tab.tile0[l] = tiles;
+      tiles += ((tab.rows[l] + 31) / 32) * ((dout + 31) / 32);
+      tab.ldw[l] = ld8(dout);
+      tab.ldwt[l] = ld8(din);
+      tab.W[l] = at<T>(p.o_Wb[l]);
+      tab.WT[l] = at<T>(p.o_WbT[l]);
+      tab.U[l] = at<T>(p.o_Ub[l]);
+      tab.UT[l] = at<T>(p.o_UbT[l]);
+    }
+    tab.tile0[h->L] = tiles;
+  }
 
   template <typename U> U* at(size_t off) const { return reinterpret_cast<U*>(base + off); }
   float* theta_slot(int t) const { return at<float>(p.o_theta) + static_cast<int64_t>(t) * h->P; }
   float* m_slot(int j) const { return at<float>(p.o_m) + static_cast<int64_t>(j) * h->P; }
 
   void launched(int n = 1) { h->launches += n; }
-
-  void check(cudaError_t e, const char* what) {
-    if (e != cudaSuccess && st == MF_OK) {
-      st = MF_ERR_CUDA;
-      h->err = std::string(what) + ": " + cudaGetErrorString(e);
-    }
-  }
 
   void gemm(GemmArgs g) {
     if (st != MF_OK) return;
@@ -215,18 +236,34 @@ struct Exec {
     }
   }
 
-  // bf16 (or fp32) operand copies of the weights of theta (or of the tangent u).
-  void cast_params(const float* theta, bool tangent) {
+  // Bias rows of the augmented transposed activations (ones for a, zeros for a').
+  void prepare() {
+    if (!h->md.has_bias) return;
+    mf::RowFill f;
     for (int l = 0; l < h->L; ++l) {
-      const int din = h->dims[l], dout = h->dims[l + 1];
-      T* W = at<T>(tangent ? p.o_Ub[l] : p.o_Wb[l]);
-      T* WT = at<T>(tangent ? p.o_UbT[l] : p.o_WbT[l]);
-      mf::cast_transpose<T>(theta + h->woff[l], din, dout, W, ld8(dout), WT, ld8(din), s);
-      launched();
+      f.dst[f.n] = at<T>(p.o_AT[l]); f.row[f.n] = h->dims[l]; f.ld[f.n] = p.ldR; f.value[f.n] = 1.f; ++f.n;
+      f.dst[f.n] = at<T>(p.o_AdT[l]); f.row[f.n] = h->dims[l]; f.ld[f.n] = p.ldR; f.value[f.n] = 0.f; ++f.n;
     }
+    mf::fill_rows<T>(f, p.ldR, s);
+    launched();
   }
 
-  // Forward pass of `rows` examples: primal (z) or dual (z, z_dot along u).
+  void update(const mf::LayerUpdArgs& a) {
+    mf::layer_update<T>(tab, a, s);
+    launched();
+  }
+
+  // Cast parameters (or the tangent) into the GEMM operand copies.
+  void cast_params(const float* theta, bool tangent) {
+    mf::LayerUpdArgs a;
+    a.mode = mf::LU_CAST;
+    a.cast_src = theta;
+    a.cast_src_to_u = tangent;
+    update(a);
+  }
+
+  // Forward pass of `rows` examples: primal (z) or dual (z, z_dot along u).  Hidden layers
+  // fuse bias, activation and its tangent into the GEMM epilogue.
   void forward(int rows, const T* x, const float* theta, const float* u, bool dual) {
     const int din0 = h->dims[0];
     mf::transpose<T>(x, rows, din0, din0, at<T>(p.o_AT[0]), p.ldR, s);
@@ -249,20 +286,24 @@ struct Exec {
         g.C1 = at<float>(p.o_Zd[l]); g.ldc1 = dout;
         g.bias1 = h->md.has_bias ? u + h->boff[l] : nullptr;
       }
-      gemm(g);
       if (l + 1 < h->L) {
-        mf::act_fwd<T>(h->md.act, at<float>(p.o_Z[l]), dual ? at<float>(p.o_Zd[l]) : nullptr, rows,
-                       dout, at<T>(p.o_A[l + 1]), at<T>(p.o_Ad[l + 1]), ld8(dout),
-                       at<T>(p.o_AT[l + 1]), at<T>(p.o_AdT[l + 1]), p.ldR, s);
-        launched();
+        g.epi.mode = mf::EPI_ACT_FWD;
+        g.epi.act = h->md.act;
+        g.epi.A = at<T>(p.o_A[l + 1]);
+        g.epi.Ad = dual ? at<T>(p.o_Ad[l + 1]) : nullptr;
+        g.epi.lda = ld8(dout);
+        g.epi.AT = at<T>(p.o_AT[l + 1]);
+        g.epi.AdT = dual ? at<T>(p.o_AdT[l + 1]) : nullptr;
+        g.epi.ldt = p.ldR;
       }
+      gemm(g);
     }
   }
 
-  // Loss seeds at the head: d f (and its tangent) into the backward buffers.
+  // Loss seeds at the head: d f (and its tangent) into backward buffer set (L-1) & 1.
   void loss(int rows, bool dual, const void* y, const float* eta_w, const float* ex_w,
             float* l_out, float* ld_out, float* d_eta) {
-    const int L = h->L, C = h->dims[L];
+    const int L = h->L, C = h->dims[L], b = (L - 1) & 1;
     mf::LossArgs a;
     a.loss = h->md.loss == MF_LOSS_SOFTMAX_CE ? 1 : 0;
     a.rows = rows; a.cols = C;
@@ -273,31 +314,32 @@ struct Exec {
     a.eta_w = eta_w; a.ex_w = ex_w;
     a.inv_norm = 1.f / static_cast<float>(rows);
     a.l = l_out; a.ld = ld_out; a.d_eta = d_eta;
-    a.dF32 = at<float>(p.o_dZ32); a.dFd32 = dual ? at<float>(p.o_dZd32) : nullptr;
-    a.dF = at<T>(p.o_dZ); a.dFd = dual ? at<T>(p.o_dZd) : nullptr;
+    a.dF = at<T>(p.o_dZ[b]); a.dFd = dual ? at<T>(p.o_dZd[b]) : nullptr;
     a.ldo = ld8(C);
     a.status = h->d_status;
     mf::loss_seed<T>(a, s);
     launched();
-    mf::transpose<T>(at<T>(p.o_dZ), rows, C, ld8(C), at<T>(p.o_dZT), p.ldR, s);
+    mf::transpose<T>(at<T>(p.o_dZ[b]), rows, C, ld8(C), at<T>(p.o_dZT[b]), p.ldR, s);
     launched();
     if (dual) {
-      mf::transpose<T>(at<T>(p.o_dZd), rows, C, ld8(C), at<T>(p.o_dZdT), p.ldR, s);
+      mf::transpose<T>(at<T>(p.o_dZd[b]), rows, C, ld8(C), at<T>(p.o_dZdT[b]), p.ldR, s);
       launched();
     }
   }
 
   // Backward pass.  Primal: out_g = grad L.  Dual: out_h = H u (and out_g = grad L if given).
+  // Weight products write the weight and bias rows of theta's layout in one GEMM; the data
+  // products fuse the activation backward (and its tangent) into the epilogue.
   void backward(int rows, bool dual, float* out_h, float* out_g) {
+    const int hb = h->md.has_bias ? 1 : 0;
     for (int l = h->L - 1; l >= 0; --l) {
-      const int din = h->dims[l], dout = h->dims[l + 1];
-      // weight product: grad W = a^T dz ;  (H u)_W = a_dot^T dz + a^T dz_dot
+      const int din = h->dims[l], dout = h->dims[l + 1], b = l & 1;
       GemmArgs g;
-      g.M = din; g.N = dout; g.K = rows;
+      g.M = din + hb; g.N = dout; g.K = rows;
       g.A0 = at<T>(p.o_AT[l]); g.lda0 = p.ldR;
       g.A1 = at<T>(p.o_AdT[l]); g.lda1 = p.ldR;
-      g.B0 = at<T>(p.o_dZT); g.ldb0 = p.ldR;
-      g.B1 = at<T>(p.o_dZdT); g.ldb1 = p.ldR;
+      g.B0 = at<T>(p.o_dZT[b]); g.ldb0 = p.ldR;
+      g.B1 = at<T>(p.o_dZdT[b]); g.ldb1 = p.ldR;
       if (!dual) {
         g.terms = mf::T_C0_A0B0;
         g.C0 = out_g + h->woff[l]; g.ldc0 = dout;
@@ -310,33 +352,27 @@ struct Exec {
         g.C0 = out_h + h->woff[l]; g.ldc0 = dout;
       }
       gemm(g);
-      if (h->md.has_bias) {
-        if (dual) { mf::colsum(at<float>(p.o_dZd32), rows, dout, out_h + h->boff[l], s); launched(); }
-        if (out_g) {
-          mf::colsum(at<float>(p.o_dZ32), rows, dout, out_g + h->boff[l], s);
-          launched();
-        }
-      }
       if (l == 0) break;
-      // data product: da = dz W^T ;  da_dot = dz_dot W^T + dz U^T
+      // data product: da = dz W^T ; da' = dz' W^T + dz U^T ; epilogue -> dz, dz' of layer l-1
       GemmArgs d;
       d.M = rows; d.N = din; d.K = dout;
-      d.A0 = at<T>(p.o_dZ); d.lda0 = ld8(dout);
-      d.A1 = at<T>(p.o_dZd); d.lda1 = ld8(dout);
+      d.A0 = at<T>(p.o_dZ[b]); d.lda0 = ld8(dout);
+      d.A1 = at<T>(p.o_dZd[b]); d.lda1 = ld8(dout);
       d.B0 = at<T>(p.o_Wb[l]); d.ldb0 = ld8(dout);
       d.B1 = at<T>(p.o_Ub[l]); d.ldb1 = ld8(dout);
-      d.C0 = at<float>(p.o_dA); d.ldc0 = din;
-      d.terms = mf::T_C0_A0B0;
-      if (dual) {
-        d.terms |= mf::T_C1_A1B0 | mf::T_C1_A0B1;
-        d.C1 = at<float>(p.o_dAd); d.ldc1 = din;
-      }
+      d.terms = dual ? (mf::T_C0_A0B0 | mf::T_C1_A1B0 | mf::T_C1_A0B1) : mf::T_C0_A0B0;
+      d.epi.mode = mf::EPI_ACT_BWD;
+      d.epi.act = h->md.act;
+      d.epi.Z = at<float>(p.o_Z[l - 1]);
+      d.epi.Zd = dual ? at<float>(p.o_Zd[l - 1]) : nullptr;
+      d.epi.ldz = din;
+      d.epi.A = at<T>(p.o_dZ[b ^ 1]);
+      d.epi.Ad = dual ? at<T>(p.o_dZd[b ^ 1]) : nullptr;
+      d.epi.lda = ld8(din);
+      d.epi.AT = at<T>(p.o_dZT[b ^ 1]);
+      d.epi.AdT = dual ? at<T>(p.o_dZdT[b ^ 1]) : nullptr;
+      d.epi.ldt = p.ldR;
       gemm(d);
-      mf::act_bwd<T>(h->md.act, at<float>(p.o_Z[l - 1]), dual ? at<float>(p.o_Zd[l - 1]) : nullptr,
-                     at<float>(p.o_dA), dual ? at<float>(p.o_dAd) : nullptr, rows, din,
-                     at<T>(p.o_dZ), at<T>(p.o_dZd), ld8(din), at<T>(p.o_dZT), at<T>(p.o_dZdT),
-                     p.ldR, at<float>(p.o_dZ32), dual ? at<float>(p.o_dZd32) : nullptr, s);
-      launched();
     }
   }
 };
@@ -407,6 +443,7 @@ LrSel lr_select(const mf_ctx* h, const mf_loop_desc* lp, const float* eta) {
 
 // Inner rollout (Eq. 2).  With store_all, theta slot t holds theta_t and m slot j holds
 // m_{j+1} when the learning rate is a meta-parameter; otherwise two theta slots ping-pong.
+// Each step's update (K4) also casts theta_{t+1} into the GEMM operand copies.
 template <typename E>
 void rollout(Exec<E>& ex, const mf_loop_desc* lp, const float* eta, const void* inner_x,
              const void* inner_y, const LrSel& lr, bool store_all, float** theta_T) {
@@ -417,12 +454,12 @@ void rollout(Exec<E>& ex, const mf_loop_desc* lp, const float* eta, const void* 
   float* m_run = (lp->momentum != 0.f && !lr.lr_meta) ? ex.template at<float>(ex.p.o_u) : nullptr;
   if (m_run) { mf::fill(m_run, h->P, 0.f, ex.s); ex.launched(); }
   const float* m_prev = nullptr;
+  ex.cast_params(ex.theta_slot(0), false);
   for (int t = 0; t < lp->T; ++t) {
     float* th = ex.theta_slot(store_all ? t : (t & 1));
     float* th_next = ex.theta_slot(store_all ? t + 1 : ((t + 1) & 1));
     const E* x = reinterpret_cast<const E*>(static_cast<const char*>(inner_x) + xs * t);
     const void* y = static_cast<const char*>(inner_y) + ys * t;
-    ex.cast_params(th, false);
     ex.forward(B, x, th, nullptr, false);
     const float* ew = (lp->meta_kind & MF_META_EXAMPLE_WEIGHTS) ? eta + static_cast<int64_t>(t) * B : nullptr;
     ex.loss(B, false, y, ew, nullptr, nullptr, nullptr, nullptr);
@@ -432,9 +469,17 @@ void rollout(Exec<E>& ex, const mf_loop_desc* lp, const float* eta, const void* 
     if (lr.lr_meta && store_all) m_out = ex.m_slot(t);
     else if (lr.lr_meta) m_out = ex.m_slot(0);
     else if (m_run) m_out = m_run;
-    const float* m_in = lr.lr_meta ? m_prev : m_run;
-    mf::rollout_update(h->P, th, m_in, g, lp->momentum, lr.lr, th_next, m_out, h->d_status, ex.s);
-    ex.launched();
+    mf::LayerUpdArgs a;
+    a.mode = mf::LU_ROLLOUT;
+    a.theta = th;
+    a.m = lr.lr_meta ? m_prev : m_run;
+    a.g = g;
+    a.theta_out = th_next;
+    a.m_out = m_out;
+    a.mu = lp->momentum;
+    a.lr = lr.lr;
+    a.status = h->d_status;
+    ex.update(a);
     m_prev = m_out;
     if (ex.st != MF_OK) return;
   }
@@ -455,19 +500,19 @@ mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
   Exec<E> ex(h, plan, s);
   MF_CUDA(h, cudaMemcpyAsync(ex.theta_slot(0), theta0, h->P * 4, cudaMemcpyDeviceToDevice, s));
   const int64_t ne = n_eta_of(h, lp);
-  MF_CUDA(h, cudaMemsetAsync(d_eta, 0, ne * 4, s));
+  if (ne > 0) MF_CUDA(h, cudaMemsetAsync(d_eta, 0, ne * 4, s));
+  ex.prepare();
 
   // 1. rollout with the theta_t store
   float* thT = nullptr;
   rollout<E>(ex, lp, eta, inner_x, inner_y, lr, true, &thT);
   if (ex.st != MF_OK) return ex.st;
 
-  // 2. outer gradient theta_bar_T = grad V(theta_T)  (Eq. 4)
+  // 2. outer gradient theta_bar_T = grad V(theta_T)  (Eq. 4); theta_T is already cast
   float* tbar = ex.template at<float>(plan.o_tbar);
   float* u = ex.template at<float>(plan.o_u);
   float* Hu = ex.template at<float>(plan.o_g);
   float* part = ex.template at<float>(plan.o_part);
-  ex.cast_params(thT, false);
   ex.forward(Bo, static_cast<const E*>(outer_x), thT, nullptr, false);
   ex.loss(Bo, false, outer_y, nullptr, nullptr, ex.template at<float>(plan.o_l), nullptr, nullptr);
   ex.backward(Bo, false, nullptr, tbar);
@@ -476,39 +521,54 @@ mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
     ex.launched();
   }
   float* d_plr = lr.off_plr >= 0 ? d_eta + lr.off_plr : nullptr;
-  // u_{T-1} = -lr theta_bar_T ;  d eta_lr += -lr m_T theta_bar_T
-  mf::adjoint_update(h->P, tbar, nullptr, lr.lr_meta ? ex.m_slot(T - 1) : nullptr, nullptr, u,
-                     lp->momentum, lr.lr, d_plr, scalar_lr ? part + (T - 1) * plan.nb : nullptr,
-                     plan.nb, h->d_status, s);
-  ex.launched();
+  // u_{T-1} = -lr theta_bar_T ;  d eta_lr += -lr m_T theta_bar_T ; cast theta_{T-1}, u_{T-1}
+  {
+    mf::LayerUpdArgs a;
+    a.mode = mf::LU_ADJOINT;
+    a.theta_bar = tbar;
+    a.m_adj = lr.lr_meta ? ex.m_slot(T - 1) : nullptr;
+    a.u_out = u;
+    a.d_plr = d_plr;
+    a.partials = scalar_lr ? part + static_cast<int64_t>(T - 1) * plan.nb : nullptr;
+    a.cast_src = ex.theta_slot(T - 1);
+    a.mu = lp->momentum;
+    a.lr = lr.lr;
+    a.status = h->d_status;
+    ex.update(a);
+  }
 
   // 3. reverse sweep t = T-1..0 with forward-over-reverse Hessian-vector products
   const int din = h->dims[0];
   const size_t xs = static_cast<size_t>(B) * din * (h->bf16 ? 2 : 4);
   const size_t ys = y_stride_bytes(h, B);
+  const bool exw = lp->meta_kind & MF_META_EXAMPLE_WEIGHTS;
   for (int t = T - 1; t >= 0; --t) {
     const float* th = ex.theta_slot(t);
     const E* x = reinterpret_cast<const E*>(static_cast<const char*>(inner_x) + xs * t);
     const void* y = static_cast<const char*>(inner_y) + ys * t;
-    ex.cast_params(th, false);
-    ex.cast_params(u, true);
     ex.forward(B, x, th, u, true);
-    const bool exw = lp->meta_kind & MF_META_EXAMPLE_WEIGHTS;
     const float* ew = exw ? eta + static_cast<int64_t>(t) * B : nullptr;
     float* de = exw ? d_eta + static_cast<int64_t>(t) * B : nullptr;
     ex.loss(B, true, y, ew, nullptr, nullptr, ex.template at<float>(plan.o_ld), de);
     ex.backward(B, true, Hu, nullptr);
+    // theta_bar_t = theta_bar_{t+1} + H u ; d eta_lr += -lr m_t theta_bar_t ;
+    // u_{t-1} = mu u_t - lr theta_bar_t ; cast theta_{t-1}, u_{t-1}
+    mf::LayerUpdArgs a;
+    a.mode = mf::LU_ADJOINT;
+    a.theta_bar = tbar;
+    a.Hu = Hu;
     if (t > 0) {
-      // theta_bar_t = theta_bar_{t+1} + H u ; d eta_lr += -lr m_t theta_bar_t ;
-      // u_{t-1} = mu u_t - lr theta_bar_t
-      mf::adjoint_update(h->P, tbar, Hu, lr.lr_meta ? ex.m_slot(t - 1) : nullptr, u, u,
-                         lp->momentum, lr.lr, d_plr,
-                         scalar_lr ? part + (t - 1) * plan.nb : nullptr, plan.nb, h->d_status, s);
-    } else {
-      mf::adjoint_update(h->P, tbar, Hu, nullptr, nullptr, nullptr, lp->momentum, lr.lr, nullptr,
-                         nullptr, 0, h->d_status, s);
+      a.m_adj = lr.lr_meta ? ex.m_slot(t - 1) : nullptr;
+      a.u_in = u;
+      a.u_out = u;
+      a.d_plr = d_plr;
+      a.partials = scalar_lr ? part + static_cast<int64_t>(t - 1) * plan.nb : nullptr;
+      a.cast_src = ex.theta_slot(t - 1);
     }
-    ex.launched();
+    a.mu = lp->momentum;
+    a.lr = lr.lr;
+    a.status = h->d_status;
+    ex.update(a);
     if (ex.st != MF_OK) return ex.st;
   }
   if (scalar_lr) {
@@ -529,7 +589,7 @@ mf_status rollout_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0, c
   if (st != MF_OK) return st;
   Exec<E> ex(h, plan, s);
   MF_CUDA(h, cudaMemcpyAsync(ex.theta_slot(0), theta0, h->P * 4, cudaMemcpyDeviceToDevice, s));
-  // with the learning rate as a meta-parameter the ping-pong variant keeps m in m slot 0
+  ex.prepare();
   float* thT = nullptr;
   rollout<E>(ex, lp, eta, inner_x, inner_y, lr, false, &thT);
   if (ex.st != MF_OK) return ex.st;
@@ -545,6 +605,7 @@ mf_status hvp_impl(mf_ctx* h, int B, const float* theta, const void* x, const vo
   mf_status st = ensure_ws(h, plan.bytes, s);
   if (st != MF_OK) return st;
   Exec<E> ex(h, plan, s);
+  ex.prepare();
   ex.cast_params(theta, false);
   ex.cast_params(v, true);
   ex.forward(B, static_cast<const E*>(x), theta, v, true);

@@ -17,6 +17,20 @@ enum : unsigned {
 
 inline int term_count(unsigned t) { return __builtin_popcount(t & 31u); }
 
+enum Act : int { ACT_IDENT = 0, ACT_TANH = 1, ACT_GELU = 2, ACT_SILU = 3 };
+enum EpiMode : int { EPI_STORE = 0, EPI_ACT_FWD = 1, EPI_ACT_BWD = 2 };
+
+// Fused epilogue of a dual GEMM (see device_math.cuh for the element rules).  The A family
+// outputs have the operand element type of the GEMM backend (bf16 for tensor cores, float
+// for the SIMT path): A/Ad row-major [M][lda], AT/AdT transposed [N][ldt]; each nullable.
+struct EpiParams {
+  int mode = EPI_STORE;
+  int act = ACT_IDENT;
+  void* A = nullptr; void* Ad = nullptr; int lda = 0;
+  void* AT = nullptr; void* AdT = nullptr; int ldt = 0;
+  const float* Z = nullptr; const float* Zd = nullptr; int ldz = 0;   // EPI_ACT_BWD inputs
+};
+
 // C[m][n] (+)= sum over selected terms of X[m][k] * Y[n][k]   (both operands K-major).
 struct GemmArgs {
   int M = 0, N = 0, K = 0;
@@ -27,36 +41,35 @@ struct GemmArgs {
   float* C0 = nullptr; int ldc0 = 0; const float* bias0 = nullptr;
   float* C1 = nullptr; int ldc1 = 0; const float* bias1 = nullptr;
   unsigned terms = 0;
+  EpiParams epi;
+  int split_k = 0;         // 0 = choose automatically, else 1/2/4/8 (tensor-core path)
+  int bn = 0, ka = 0;      // tile width / K atoms per stage; 0 = choose automatically
   int* status = nullptr;   // device status word (timeouts), may be null
 };
 
 // tcgen05 bf16 GEMM (tc_gemm.cu).  Returns cudaSuccess or the launch error; sets *why on a
 // host-side rejection (bad alignment/ld) and returns cudaErrorInvalidValue.
 cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why);
+// Activation-epilogue instances (tc_gemm_act.cu), called by tc_gemm.
+cudaError_t tc_gemm_act(const GemmArgs& a, cudaStream_t s, const char** why, int bn, int ka);
 // SIMT float32 GEMM with the same semantics (simt_gemm.cu).
 cudaError_t simt_gemm(const GemmArgs& a, cudaStream_t s);
 
 // ---- elementwise / row kernels (kernels.cu); T is float or __nv_bfloat16 -------------
-enum Act : int { ACT_IDENT = 0, ACT_TANH = 1, ACT_GELU = 2, ACT_SILU = 3 };
-
-// W [rows][cols] float32 (ld = cols) -> Wo [rows][ldo] (T), WoT [cols][ldoT] (T).
-template <typename T>
-void cast_transpose(const float* W, int rows, int cols, T* Wo, int ldo, T* WoT, int ldoT,
-                    cudaStream_t s);
 // X [rows][ld] (T) -> XT [cols][ldT] (T)
 template <typename T>
 void transpose(const T* X, int rows, int cols, int ld, T* XT, int ldT, cudaStream_t s);
-
-// Dual activation forward: a = phi(z), a_dot = phi'(z) z_dot (when Zd != null).
+// Set one row (columns 0..cols-1) of each listed matrix to a value: the bias row of the
+// augmented transposed activations [a^T; 1] and [a'^T; 0] of the weight products.
+struct RowFill {
+  int n = 0;
+  void* dst[64];
+  int row[64];
+  int ld[64];
+  float value[64];
+};
 template <typename T>
-void act_fwd(int act, const float* Z, const float* Zd, int rows, int cols, T* A, T* Ad,
-             int ld, T* AT, T* AdT, int ldT, cudaStream_t s);
-// Dual activation backward: dz = phi'(z) da ; dz_dot = phi''(z) z_dot da + phi'(z) da_dot.
-// Writes T copies (normal + transposed) and float32 copies (for bias reductions).
-template <typename T>
-void act_bwd(int act, const float* Z, const float* Zd, const float* dA, const float* dAd,
-             int rows, int cols, T* dZ, T* dZd, int ld, T* dZT, T* dZdT, int ldT,
-             float* dZ32, float* dZd32, cudaStream_t s);
+void fill_rows(const RowFill& f, int cols, cudaStream_t s);
 
 struct LossArgs {
   int loss = 0;            // 0 squared, 1 softmax CE
@@ -69,15 +82,12 @@ struct LossArgs {
   float* l = nullptr;      // per-example loss [rows] (nullable)
   float* ld = nullptr;     // per-example tangent loss [rows] (nullable)
   float* d_eta = nullptr;  // += sigmoid'(eta_w) * ld * inv_norm  [rows] (nullable)
-  float* dF32 = nullptr; float* dFd32 = nullptr;   // seeds float32 [rows][cols]
   void* dF = nullptr; void* dFd = nullptr; int ldo = 0; // seeds in T [rows][ldo]
   int* status = nullptr;
 };
 template <typename T>
 void loss_seed(const LossArgs& a, cudaStream_t s);
 
-// out[n] = sum_{r<rows} X[r][n]  (deterministic, float32)
-void colsum(const float* X, int rows, int cols, float* out, cudaStream_t s);
 // out[0] = scale * sum_i x[i] (deterministic, one block)
 void sum_scaled(const float* x, int n, float scale, float* out, cudaStream_t s);
 
@@ -87,19 +97,40 @@ struct LrArgs {
   const float* slr = nullptr;   // scalar log-lr [1]
 };
 
-// Rollout update (K4):  m' = mu m + g ;  theta' = theta - lr m'   (m may be null = 0)
-void rollout_update(int64_t P, const float* theta, const float* m, const float* g, float mu,
-                    LrArgs lr, float* theta_out, float* m_out, int* status, cudaStream_t s);
+// Per-layer view of the flat parameter vector for the fused update/cast kernel.  Layer l
+// occupies rows[l] x dout[l] floats at off[l] (W_l rows, then the bias row when present);
+// its first din[l] rows are cast to the GEMM operand copies W (row-major [din][ldw]) and
+// WT (transposed [dout][ldwt]), or U / UT for the tangent.
+constexpr int kMaxLayers = 32;
+struct LayerTable {
+  int n = 0;
+  int rows[kMaxLayers], din[kMaxLayers], dout[kMaxLayers];
+  int64_t off[kMaxLayers];
+  int tile0[kMaxLayers + 1];
+  int ldw[kMaxLayers], ldwt[kMaxLayers];
+  void* W[kMaxLayers]; void* WT[kMaxLayers]; void* U[kMaxLayers]; void* UT[kMaxLayers];
+};
 
-// Adjoint update (K5):  theta_bar += Hu (Hu nullable);
-//   if m != null: d_plr += -lr m theta_bar  (per parameter)  or partial[blk] = sum(-lr m theta_bar)
-//   u = mu u - lr theta_bar   (u_in nullable = 0)
-void adjoint_update(int64_t P, float* theta_bar, const float* Hu, const float* m,
-                    const float* u_in, float* u_out, float mu, LrArgs lr, float* d_plr,
-                    float* partials, int n_partials, int* status, cudaStream_t s);
-int adjoint_partials_blocks(int64_t P);
+enum LuMode : int { LU_CAST = 0, LU_ROLLOUT = 1, LU_ADJOINT = 2 };
+struct LayerUpdArgs {
+  int mode = LU_CAST;
+  const float* cast_src = nullptr;  // parameters to cast into W/WT (nullable)
+  bool cast_src_to_u = false;       // LU_CAST: write into U/UT instead of W/WT
+  // LU_ROLLOUT (K4):  m' = mu m + g ; theta' = theta - lr m' ; cast theta' into W/WT
+  const float* theta = nullptr; const float* m = nullptr; const float* g = nullptr;
+  float* theta_out = nullptr; float* m_out = nullptr;
+  // LU_ADJOINT (K5):  theta_bar += Hu ; d eta_lr from m_adj ; u' = mu u - lr theta_bar ;
+  //                   cast u' into U/UT
+  float* theta_bar = nullptr; const float* Hu = nullptr; const float* m_adj = nullptr;
+  const float* u_in = nullptr; float* u_out = nullptr; float* d_plr = nullptr;
+  float* partials = nullptr;       // scalar log-lr: one partial per block (tile)
+  float mu = 0.f;
+  LrArgs lr;
+  int* status = nullptr;
+};
+template <typename T>
+void layer_update(const LayerTable& tab, const LayerUpdArgs& a, cudaStream_t s);
 
 void fill(float* p, int64_t n, float v, cudaStream_t s);
-void copy_f32(float* dst, const float* src, int64_t n, cudaStream_t s);
 
 }  // namespace mf

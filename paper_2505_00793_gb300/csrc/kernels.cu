@@ -1,76 +1,24 @@
 // Elementwise, row and update kernels of the mixed-mode sweep (HBM-bound work).
 //
-//  * dual activation forward / backward (the tangent rules of a = phi(z) and of its VJP),
-//    writing both the row-major operand and its transpose for the next tensor-core GEMM;
 //  * per-example loss seeds with the tangent per-example loss (the mixed term of Eq. 7 for
 //    per-example weights) and d eta_{t,b} = sigmoid'(eta_{t,b}) * l'_b / B;
-//  * the inner-step update (Eq. 2) and the adjoint update of the reverse sweep (Eq. 5 with
-//    the Hessian product supplied by the forward-over-reverse pass).
+//  * the fused per-layer update kernel: the inner-step update of Eq. 2 (rollout) or the
+//    adjoint update of the reverse sweep (Eq. 5 with the Hessian product supplied by the
+//    forward-over-reverse pass), each fused with the cast of the next step's parameters /
+//    tangent into the row-major and transposed GEMM operand copies;
+//  * transposes, row fills and a deterministic sum.
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <math.h>
 #include <stdint.h>
 
+#include "device_math.cuh"
 #include "internal.h"
 
 namespace mf {
 namespace {
 
-template <typename T> __device__ __forceinline__ T to_t(float x);
-template <> __device__ __forceinline__ float to_t<float>(float x) { return x; }
-template <> __device__ __forceinline__ __nv_bfloat16 to_t<__nv_bfloat16>(float x) {
-  return __float2bfloat16_rn(x);
-}
-
-// phi, phi', phi'' of the hidden activations.
-__device__ __forceinline__ void act_eval(int act, float z, float& f, float& d1, float& d2) {
-  switch (act) {
-    case ACT_TANH: {
-      const float t = tanhf(z);
-      f = t; d1 = 1.f - t * t; d2 = -2.f * t * d1;
-      break;
-    }
-    case ACT_GELU: {   // x * Phi(x): phi' = Phi + x pdf, phi'' = pdf (2 - x^2)
-      const float cdf = 0.5f * (1.f + erff(z * 0.70710678118654752f));
-      const float pdf = 0.39894228040143268f * expf(-0.5f * z * z);
-      f = z * cdf; d1 = cdf + z * pdf; d2 = pdf * (2.f - z * z);
-      break;
-    }
-    case ACT_SILU: {   // x * s(x): phi' = s (1 + x (1 - s)), phi'' = s (1 - s) (2 + x (1 - 2 s))
-      const float sg = 1.f / (1.f + expf(-z));
-      f = z * sg; d1 = sg * (1.f + z * (1.f - sg));
-      d2 = sg * (1.f - sg) * (2.f + z * (1.f - 2.f * sg));
-      break;
-    }
-    default:
-      f = z; d1 = 1.f; d2 = 0.f;
-  }
-}
-
 constexpr int TILE = 32, TROWS = 8;
-
-template <typename T>
-__global__ void cast_transpose_kernel(const float* __restrict__ W, int rows, int cols,
-                                      T* __restrict__ Wo, int ldo, T* __restrict__ WoT, int ldoT) {
-  __shared__ float tile[TILE][TILE + 1];
-  const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
-  const int tx = threadIdx.x, ty = threadIdx.y;
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int r = r0 + i, c = c0 + tx;
-    float v = 0.f;
-    if (r < rows && c < cols) {
-      v = W[static_cast<int64_t>(r) * cols + c];
-      if (Wo) Wo[static_cast<int64_t>(r) * ldo + c] = to_t<T>(v);
-    }
-    tile[i][tx] = v;
-  }
-  if (!WoT) return;
-  __syncthreads();
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int c = c0 + i, r = r0 + tx;
-    if (c < cols && r < rows) WoT[static_cast<int64_t>(c) * ldoT + r] = to_t<T>(tile[tx][i]);
-  }
-}
 
 template <typename T>
 __global__ void transpose_kernel(const T* __restrict__ X, int rows, int cols, int ld,
@@ -90,82 +38,12 @@ __global__ void transpose_kernel(const T* __restrict__ X, int rows, int cols, in
 }
 
 template <typename T>
-__global__ void act_fwd_kernel(int act, const float* __restrict__ Z, const float* __restrict__ Zd,
-                               int rows, int cols, T* __restrict__ A, T* __restrict__ Ad, int ld,
-                               T* __restrict__ AT, T* __restrict__ AdT, int ldT) {
-  __shared__ float ta[TILE][TILE + 1];
-  __shared__ float tad[TILE][TILE + 1];
-  const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
-  const int tx = threadIdx.x, ty = threadIdx.y;
-  const bool dual = Zd != nullptr;
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int r = r0 + i, c = c0 + tx;
-    float a = 0.f, ad = 0.f;
-    if (r < rows && c < cols) {
-      const int64_t o = static_cast<int64_t>(r) * cols + c;
-      float d1, d2;
-      act_eval(act, Z[o], a, d1, d2);
-      A[static_cast<int64_t>(r) * ld + c] = to_t<T>(a);
-      if (dual) {
-        ad = d1 * Zd[o];
-        Ad[static_cast<int64_t>(r) * ld + c] = to_t<T>(ad);
-      }
-    }
-    ta[i][tx] = a;
-    tad[i][tx] = ad;
-  }
-  __syncthreads();
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int c = c0 + i, r = r0 + tx;
-    if (c < cols && r < rows) {
-      const int64_t o = static_cast<int64_t>(c) * ldT + r;
-      AT[o] = to_t<T>(ta[tx][i]);
-      if (dual) AdT[o] = to_t<T>(tad[tx][i]);
-    }
-  }
-}
-
-template <typename T>
-__global__ void act_bwd_kernel(int act, const float* __restrict__ Z, const float* __restrict__ Zd,
-                               const float* __restrict__ dA, const float* __restrict__ dAd,
-                               int rows, int cols, T* __restrict__ dZ, T* __restrict__ dZd, int ld,
-                               T* __restrict__ dZT, T* __restrict__ dZdT, int ldT,
-                               float* __restrict__ dZ32, float* __restrict__ dZd32) {
-  __shared__ float t0[TILE][TILE + 1];
-  __shared__ float t1[TILE][TILE + 1];
-  const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
-  const int tx = threadIdx.x, ty = threadIdx.y;
-  const bool dual = dAd != nullptr;
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int r = r0 + i, c = c0 + tx;
-    float g = 0.f, gd = 0.f;
-    if (r < rows && c < cols) {
-      const int64_t o = static_cast<int64_t>(r) * cols + c;
-      float f, d1, d2;
-      act_eval(act, Z[o], f, d1, d2);
-      const float da = dA[o];
-      g = d1 * da;
-      const int64_t on = static_cast<int64_t>(r) * ld + c;
-      dZ[on] = to_t<T>(g);
-      if (dZ32) dZ32[o] = g;
-      if (dual) {
-        gd = d2 * Zd[o] * da + d1 * dAd[o];
-        dZd[on] = to_t<T>(gd);
-        if (dZd32) dZd32[o] = gd;
-      }
-    }
-    t0[i][tx] = g;
-    t1[i][tx] = gd;
-  }
-  __syncthreads();
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int c = c0 + i, r = r0 + tx;
-    if (c < cols && r < rows) {
-      const int64_t o = static_cast<int64_t>(c) * ldT + r;
-      dZT[o] = to_t<T>(t0[tx][i]);
-      if (dual) dZdT[o] = to_t<T>(t1[tx][i]);
-    }
-  }
+__global__ void fill_rows_kernel(const RowFill f, int cols) {
+  const int k = blockIdx.y;
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= f.n || c >= cols) return;
+  T* dst = static_cast<T*>(f.dst[k]);
+  dst[static_cast<int64_t>(f.row[k]) * f.ld[k] + c] = to_t<T>(f.value[k]);
 }
 
 __device__ __forceinline__ float warp_sum(float v) {
@@ -197,7 +75,6 @@ __global__ void loss_seed_kernel(const LossArgs a) {
   T* dF = static_cast<T*>(a.dF);
   T* dFd = static_cast<T*>(a.dFd);
   const int64_t orow = static_cast<int64_t>(row) * a.ldo;
-  const int64_t frow = static_cast<int64_t>(row) * C;
   float l = 0.f, ld = 0.f;
   if (a.loss == 0) {
     const float* y = a.Yf + static_cast<int64_t>(row) * C;
@@ -207,14 +84,8 @@ __global__ void loss_seed_kernel(const LossArgs a) {
       const float r = f[c] - y[c];
       s2 += r * r;
       if (fd) s1 += r * fd[c];
-      const float g = scale * r * invC;
-      if (dF) dF[orow + c] = to_t<T>(g);
-      if (a.dF32) a.dF32[frow + c] = g;
-      if (fd) {
-        const float gd = scale * fd[c] * invC;
-        if (dFd) dFd[orow + c] = to_t<T>(gd);
-        if (a.dFd32) a.dFd32[frow + c] = gd;
-      }
+      if (dF) dF[orow + c] = to_t<T>(scale * r * invC);
+      if (fd && dFd) dFd[orow + c] = to_t<T>(scale * fd[c] * invC);
     }
     l = 0.5f * warp_sum(s2) * invC;
     ld = warp_sum(s1) * invC;
@@ -238,14 +109,8 @@ __global__ void loss_seed_kernel(const LossArgs a) {
     }
     for (int c = lane; c < C; c += 32) {
       const float pc = expf(f[c] - lse);
-      const float g = scale * (pc - (c == y ? 1.f : 0.f));
-      if (dF) dF[orow + c] = to_t<T>(g);
-      if (a.dF32) a.dF32[frow + c] = g;
-      if (fd) {
-        const float gd = scale * pc * (fd[c] - pf);
-        if (dFd) dFd[orow + c] = to_t<T>(gd);
-        if (a.dFd32) a.dFd32[frow + c] = gd;
-      }
+      if (dF) dF[orow + c] = to_t<T>(scale * (pc - (c == y ? 1.f : 0.f)));
+      if (fd && dFd) dFd[orow + c] = to_t<T>(scale * pc * (fd[c] - pf));
     }
     l = lse - f[y];
     if (fd) ld = pf - fd[y];
@@ -255,15 +120,6 @@ __global__ void loss_seed_kernel(const LossArgs a) {
     if (a.ld) a.ld[row] = ld;
     if (a.d_eta && a.eta_w) a.d_eta[row] = sg * (1.f - sg) * ld * a.inv_norm;
   }
-}
-
-__global__ void colsum_kernel(const float* __restrict__ X, int rows, int cols,
-                              float* __restrict__ out) {
-  const int c = blockIdx.x * blockDim.x + threadIdx.x;
-  if (c >= cols) return;
-  float s = 0.f;
-  for (int r = 0; r < rows; ++r) s += X[static_cast<int64_t>(r) * cols + c];
-  out[c] = s;
 }
 
 __global__ void sum_scaled_kernel(const float* __restrict__ x, int n, float scale,
@@ -287,52 +143,86 @@ __device__ __forceinline__ float lr_at(const LrArgs& lr, int64_t i) {
   return lr.alpha;
 }
 
-__global__ void rollout_update_kernel(int64_t P, const float* __restrict__ theta,
-                                      const float* __restrict__ m, const float* __restrict__ g,
-                                      float mu, LrArgs lr, float* __restrict__ theta_out,
-                                      float* __restrict__ m_out, int* status) {
-  bool bad = false;
-  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < P;
-       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const float mn = (m ? mu * m[i] : 0.f) + g[i];
-    const float tn = theta[i] - lr_at(lr, i) * mn;
-    if (m_out) m_out[i] = mn;
-    theta_out[i] = tn;
-    bad |= !isfinite(tn);
-  }
-  if (bad && status) atomicExch(status, DEV_NONFINITE);
-}
-
-__global__ void adjoint_update_kernel(int64_t P, float* __restrict__ theta_bar,
-                                      const float* __restrict__ Hu, const float* __restrict__ m,
-                                      const float* __restrict__ u_in, float* __restrict__ u_out,
-                                      float mu, LrArgs lr, float* __restrict__ d_plr,
-                                      float* __restrict__ partials, int* status) {
-  __shared__ float red[32];
+// One 32 x 32 tile of one layer's [rows][dout] slice of the flat parameter vector per block.
+template <typename T>
+__global__ void __launch_bounds__(TILE * TROWS) layer_update_kernel(const LayerTable tab,
+                                                                    const LayerUpdArgs a) {
+  __shared__ float tw[TILE][TILE + 1];   // values cast into W / WT
+  __shared__ float tu[TILE][TILE + 1];   // values cast into U / UT
+  __shared__ float red[TILE * TROWS / 32];
+  int l = 0;
+  while (l + 1 < tab.n && static_cast<int>(blockIdx.x) >= tab.tile0[l + 1]) ++l;
+  const int t = blockIdx.x - tab.tile0[l];
+  const int dout = tab.dout[l], rows = tab.rows[l], din = tab.din[l];
+  const int tiles_c = (dout + TILE - 1) / TILE;
+  const int r0 = (t / tiles_c) * TILE, c0 = (t % tiles_c) * TILE;
+  const int tx = threadIdx.x, ty = threadIdx.y;
+  const bool cast_w = (a.mode == LU_ROLLOUT) || (a.mode == LU_CAST && !a.cast_src_to_u) ||
+                      (a.mode == LU_ADJOINT && a.cast_src);
+  const bool cast_u = (a.mode == LU_CAST && a.cast_src_to_u) || (a.mode == LU_ADJOINT && a.u_out);
   bool bad = false;
   float acc = 0.f;
-  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < P;
-       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const float tb = theta_bar[i] + (Hu ? Hu[i] : 0.f);
-    theta_bar[i] = tb;
-    bad |= !isfinite(tb);
-    const float r = lr_at(lr, i);
-    if (m) {
-      const float contrib = -r * m[i] * tb;
-      if (d_plr) d_plr[i] += contrib;
-      else acc += contrib;
+  for (int i = ty; i < TILE; i += TROWS) {
+    const int r = r0 + i, c = c0 + tx;
+    float vw = 0.f, vu = 0.f;
+    if (r < rows && c < dout) {
+      const int64_t k = tab.off[l] + static_cast<int64_t>(r) * dout + c;
+      if (a.mode == LU_ROLLOUT) {
+        const float mn = (a.m ? a.mu * a.m[k] : 0.f) + a.g[k];
+        const float tn = a.theta[k] - lr_at(a.lr, k) * mn;
+        a.theta_out[k] = tn;
+        if (a.m_out) a.m_out[k] = mn;
+        bad |= !isfinite(tn);
+        vw = tn;
+      } else if (a.mode == LU_ADJOINT) {
+        const float tb = a.theta_bar[k] + (a.Hu ? a.Hu[k] : 0.f);
+        a.theta_bar[k] = tb;
+        bad |= !isfinite(tb);
+        const float lr = lr_at(a.lr, k);
+        if (a.m_adj) {
+          const float contrib = -lr * a.m_adj[k] * tb;
+          if (a.d_plr) a.d_plr[k] += contrib;
+          else acc += contrib;
+        }
+        if (a.u_out) {
+          vu = (a.u_in ? a.mu * a.u_in[k] : 0.f) - lr * tb;
+          a.u_out[k] = vu;
+        }
+        if (a.cast_src) vw = a.cast_src[k];
+      } else {
+        const float v = a.cast_src[k];
+        vw = v;
+        vu = v;
+      }
     }
-    if (u_out) u_out[i] = (u_in ? mu * u_in[i] : 0.f) - r * tb;
+    tw[i][tx] = vw;
+    tu[i][tx] = vu;
+    // row-major operand copies (only the din weight rows; the bias row stays float32)
+    if (r < din && c < dout) {
+      const int64_t o = static_cast<int64_t>(r) * tab.ldw[l] + c;
+      if (cast_w) static_cast<T*>(tab.W[l])[o] = to_t<T>(vw);
+      if (cast_u) static_cast<T*>(tab.U[l])[o] = to_t<T>(vu);
+    }
   }
-  if (bad && status) atomicExch(status, DEV_NONFINITE);
-  if (partials) {
+  if (bad && a.status) atomicExch(a.status, DEV_NONFINITE);
+  if (a.partials) {
     acc = warp_sum(acc);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
-    __syncthreads();
-    if (threadIdx.x < 32) {
-      float v = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.f;
-      v = warp_sum(v);
-      if (threadIdx.x == 0) partials[blockIdx.x] = v;
+    const int lin = ty * TILE + tx;
+    if ((lin & 31) == 0) red[lin >> 5] = acc;
+  }
+  __syncthreads();
+  if (a.partials && ty == 0) {
+    float v = tx < (TILE * TROWS / 32) ? red[tx] : 0.f;
+    v = warp_sum(v);
+    if (tx == 0) a.partials[blockIdx.x] = v;
+  }
+  // transposed operand copies [dout][ldwt]
+  for (int i = ty; i < TILE; i += TROWS) {
+    const int c = c0 + i, r = r0 + tx;
+    if (c < dout && r < din) {
+      const int64_t o = static_cast<int64_t>(c) * tab.ldwt[l] + r;
+      if (cast_w) static_cast<T*>(tab.WT[l])[o] = to_t<T>(tw[tx][i]);
+      if (cast_u) static_cast<T*>(tab.UT[l])[o] = to_t<T>(tu[tx][i]);
     }
   }
 }
@@ -343,23 +233,7 @@ __global__ void fill_kernel(float* p, int64_t n, float v) {
     p[i] = v;
 }
 
-int grid_for(int64_t n, int threads) {
-  int64_t b = (n + threads - 1) / threads;
-  const int64_t cap = 152 * 16;
-  if (b > cap) b = cap;
-  if (b < 1) b = 1;
-  return static_cast<int>(b);
-}
-
 }  // namespace
-
-template <typename T>
-void cast_transpose(const float* W, int rows, int cols, T* Wo, int ldo, T* WoT, int ldoT,
-                    cudaStream_t s) {
-  if (rows <= 0 || cols <= 0) return;
-  dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE);
-  cast_transpose_kernel<T><<<grid, dim3(TILE, TROWS), 0, s>>>(W, rows, cols, Wo, ldo, WoT, ldoT);
-}
 
 template <typename T>
 void transpose(const T* X, int rows, int cols, int ld, T* XT, int ldT, cudaStream_t s) {
@@ -369,22 +243,10 @@ void transpose(const T* X, int rows, int cols, int ld, T* XT, int ldT, cudaStrea
 }
 
 template <typename T>
-void act_fwd(int act, const float* Z, const float* Zd, int rows, int cols, T* A, T* Ad, int ld,
-             T* AT, T* AdT, int ldT, cudaStream_t s) {
-  if (rows <= 0 || cols <= 0) return;
-  dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE);
-  act_fwd_kernel<T><<<grid, dim3(TILE, TROWS), 0, s>>>(act, Z, Zd, rows, cols, A, Ad, ld, AT,
-                                                        AdT, ldT);
-}
-
-template <typename T>
-void act_bwd(int act, const float* Z, const float* Zd, const float* dA, const float* dAd,
-             int rows, int cols, T* dZ, T* dZd, int ld, T* dZT, T* dZdT, int ldT, float* dZ32,
-             float* dZd32, cudaStream_t s) {
-  if (rows <= 0 || cols <= 0) return;
-  dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE);
-  act_bwd_kernel<T><<<grid, dim3(TILE, TROWS), 0, s>>>(act, Z, Zd, dA, dAd, rows, cols, dZ, dZd,
-                                                        ld, dZT, dZdT, ldT, dZ32, dZd32);
+void fill_rows(const RowFill& f, int cols, cudaStream_t s) {
+  if (f.n <= 0 || cols <= 0) return;
+  dim3 grid((cols + 255) / 256, f.n);
+  fill_rows_kernel<T><<<grid, 256, 0, s>>>(f, cols);
 }
 
 template <typename T>
@@ -394,49 +256,29 @@ void loss_seed(const LossArgs& a, cudaStream_t s) {
   loss_seed_kernel<T><<<(a.rows + warps - 1) / warps, warps * 32, 0, s>>>(a);
 }
 
-void colsum(const float* X, int rows, int cols, float* out, cudaStream_t s) {
-  if (cols <= 0) return;
-  colsum_kernel<<<(cols + 255) / 256, 256, 0, s>>>(X, rows, cols, out);
-}
-
 void sum_scaled(const float* x, int n, float scale, float* out, cudaStream_t s) {
   sum_scaled_kernel<<<1, 1024, 0, s>>>(x, n, scale, out);
 }
 
-void rollout_update(int64_t P, const float* theta, const float* m, const float* g, float mu,
-                    LrArgs lr, float* theta_out, float* m_out, int* status, cudaStream_t s) {
-  rollout_update_kernel<<<grid_for(P, 256), 256, 0, s>>>(P, theta, m, g, mu, lr, theta_out, m_out,
-                                                         status);
-}
-
-int adjoint_partials_blocks(int64_t P) { return grid_for(P, 256); }
-
-void adjoint_update(int64_t P, float* theta_bar, const float* Hu, const float* m,
-                    const float* u_in, float* u_out, float mu, LrArgs lr, float* d_plr,
-                    float* partials, int n_partials, int* status, cudaStream_t s) {
-  const int g = grid_for(P, 256);
-  (void)n_partials;
-  adjoint_update_kernel<<<g, 256, 0, s>>>(P, theta_bar, Hu, m, u_in, u_out, mu, lr, d_plr,
-                                          partials, status);
+template <typename T>
+void layer_update(const LayerTable& tab, const LayerUpdArgs& a, cudaStream_t s) {
+  const int blocks = tab.tile0[tab.n];
+  if (blocks <= 0) return;
+  layer_update_kernel<T><<<blocks, dim3(TILE, TROWS), 0, s>>>(tab, a);
 }
 
 void fill(float* p, int64_t n, float v, cudaStream_t s) {
   if (n <= 0) return;
-  fill_kernel<<<grid_for(n, 256), 256, 0, s>>>(p, n, v);
+  int64_t b = (n + 255) / 256;
+  if (b > 152 * 16) b = 152 * 16;
+  fill_kernel<<<static_cast<int>(b), 256, 0, s>>>(p, n, v);
 }
 
-void copy_f32(float* dst, const float* src, int64_t n, cudaStream_t s) {
-  if (n > 0) cudaMemcpyAsync(dst, src, n * sizeof(float), cudaMemcpyDeviceToDevice, s);
-}
-
-#define MF_INST(T)                                                                           \
-  template void cast_transpose<T>(const float*, int, int, T*, int, T*, int, cudaStream_t);  \
-  template void transpose<T>(const T*, int, int, int, T*, int, cudaStream_t);               \
-  template void act_fwd<T>(int, const float*, const float*, int, int, T*, T*, int, T*, T*,  \
-                           int, cudaStream_t);                                              \
-  template void act_bwd<T>(int, const float*, const float*, const float*, const float*, int, \
-                           int, T*, T*, int, T*, T*, int, float*, float*, cudaStream_t);     \
-  template void loss_seed<T>(const LossArgs&, cudaStream_t);
+#define MF_INST(T)                                                                 \
+  template void transpose<T>(const T*, int, int, int, T*, int, cudaStream_t);     \
+  template void fill_rows<T>(const RowFill&, int, cudaStream_t);                  \
+  template void loss_seed<T>(const LossArgs&, cudaStream_t);                      \
+  template void layer_update<T>(const LayerTable&, const LayerUpdArgs&, cudaStream_t);
 MF_INST(float)
 MF_INST(__nv_bfloat16)
 #undef MF_INST

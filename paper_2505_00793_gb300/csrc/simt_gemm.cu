@@ -1,10 +1,12 @@
 // Float32 dual GEMM on the CUDA cores, for the float32-precision path (small models whose
 // meta-gradient is checked at 1e-4 relative error, below what bf16/tf32 operands allow).
-// Same term semantics as the tensor-core kernel: C_j = sum of selected X Y^T products,
-// both operands K-major.  64x64 output tile per block, 256 threads, 4x4 per thread.
+// Same term semantics and fused epilogues as the tensor-core kernel: C_j = sum of selected
+// X Y^T products (both operands K-major), then the per-element epilogue of device_math.cuh.
+// 64x64 output tile per block, 256 threads, 4x4 outputs per thread and accumulator.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "device_math.cuh"
 #include "internal.h"
 
 namespace mf {
@@ -18,6 +20,7 @@ struct SimtParams {
   const float* A[2]; int lda[2];
   const float* B[2]; int ldb[2];
   float* C[2]; int ldc[2]; const float* bias[2];
+  EpiParams epi;
 };
 
 __global__ void __launch_bounds__(256) simt_dual_gemm_kernel(const SimtParams p) {
@@ -25,52 +28,69 @@ __global__ void __launch_bounds__(256) simt_dual_gemm_kernel(const SimtParams p)
   __shared__ float Bs[TK][TN + 1];
   const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
   const int m0 = blockIdx.y * TM, n0 = blockIdx.x * TN;
-  // term list: (acc, a index, b index)
   const int tacc[5] = {0, 0, 0, 1, 1};
   const int ta[5] = {0, 1, 0, 1, 0};
   const int tb[5] = {0, 0, 1, 0, 1};
-  for (int acc = 0; acc < 2; ++acc) {
-    bool any = false;
-    float c[4][4] = {};
-    for (int t = 0; t < 5; ++t) {
-      if (!(p.terms & (1u << t)) || tacc[t] != acc) continue;
-      any = true;
-      const float* A = p.A[ta[t]];
-      const float* B = p.B[tb[t]];
-      const int lda = p.lda[ta[t]], ldb = p.ldb[tb[t]];
-      for (int k0 = 0; k0 < p.K; k0 += TK) {
-        for (int i = threadIdx.x; i < TM * TK; i += 256) {
-          const int r = i / TK, kk = i % TK;
-          const int gm = m0 + r, gk = k0 + kk;
-          As[kk][r] = (gm < p.M && gk < p.K) ? A[static_cast<int64_t>(gm) * lda + gk] : 0.f;
-          const int gn = n0 + r;
-          Bs[kk][r] = (gn < p.N && gk < p.K) ? B[static_cast<int64_t>(gn) * ldb + gk] : 0.f;
-        }
-        __syncthreads();
+  float c[2][4][4] = {};
+  for (int t = 0; t < 5; ++t) {
+    if (!(p.terms & (1u << t))) continue;
+    const int acc = tacc[t];
+    const float* A = p.A[ta[t]];
+    const float* B = p.B[tb[t]];
+    const int lda = p.lda[ta[t]], ldb = p.ldb[tb[t]];
+    for (int k0 = 0; k0 < p.K; k0 += TK) {
+      for (int i = threadIdx.x; i < TM * TK; i += 256) {
+        const int r = i / TK, kk = i % TK;
+        const int gm = m0 + r, gk = k0 + kk;
+        As[kk][r] = (gm < p.M && gk < p.K) ? A[static_cast<int64_t>(gm) * lda + gk] : 0.f;
+        const int gn = n0 + r;
+        Bs[kk][r] = (gn < p.N && gk < p.K) ? B[static_cast<int64_t>(gn) * ldb + gk] : 0.f;
+      }
+      __syncthreads();
 #pragma unroll
-        for (int kk = 0; kk < TK; ++kk) {
-          float a[4], b[4];
+      for (int kk = 0; kk < TK; ++kk) {
+        float a[4], b[4];
 #pragma unroll
-          for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
+        for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
 #pragma unroll
-          for (int j = 0; j < 4; ++j) b[j] = Bs[kk][tx * 4 + j];
+        for (int j = 0; j < 4; ++j) b[j] = Bs[kk][tx * 4 + j];
+        if (acc == 0) {
 #pragma unroll
           for (int i = 0; i < 4; ++i)
 #pragma unroll
-            for (int j = 0; j < 4; ++j) c[i][j] = fmaf(a[i], b[j], c[i][j]);
+            for (int j = 0; j < 4; ++j) c[0][i][j] = fmaf(a[i], b[j], c[0][i][j]);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 4; ++j) c[1][i][j] = fmaf(a[i], b[j], c[1][i][j]);
         }
-        __syncthreads();
       }
+      __syncthreads();
     }
-    if (!any || !p.C[acc]) continue;
-    for (int i = 0; i < 4; ++i) {
-      const int gm = m0 + ty * 4 + i;
-      if (gm >= p.M) continue;
-      for (int j = 0; j < 4; ++j) {
-        const int gn = n0 + tx * 4 + j;
-        if (gn >= p.N) continue;
-        p.C[acc][static_cast<int64_t>(gm) * p.ldc[acc] + gn] =
-            c[i][j] + (p.bias[acc] ? p.bias[acc][gn] : 0.f);
+  }
+  const bool dual = (p.terms & (T_C1_A1B0 | T_C1_A0B1)) != 0;
+  const EpiParams& e = p.epi;
+  float* A = static_cast<float*>(e.A);
+  float* Ad = static_cast<float*>(e.Ad);
+  float* AT = static_cast<float*>(e.AT);
+  float* AdT = static_cast<float*>(e.AdT);
+  for (int i = 0; i < 4; ++i) {
+    const int gm = m0 + ty * 4 + i;
+    if (gm >= p.M) continue;
+    for (int j = 0; j < 4; ++j) {
+      const int gn = n0 + tx * 4 + j;
+      if (gn >= p.N) continue;
+      const EpiOut o = epi_eval(e, gm, gn, c[0][i][j], c[1][i][j], p.bias[0], p.bias[1], dual);
+      if (p.C[0]) p.C[0][static_cast<int64_t>(gm) * p.ldc[0] + gn] = o.c0;
+      if (p.C[1] && dual) p.C[1][static_cast<int64_t>(gm) * p.ldc[1] + gn] = o.c1;
+      if (e.mode != EPI_STORE) {
+        if (A) A[static_cast<int64_t>(gm) * e.lda + gn] = o.o0;
+        if (AT) AT[static_cast<int64_t>(gn) * e.ldt + gm] = o.o0;
+        if (dual) {
+          if (Ad) Ad[static_cast<int64_t>(gm) * e.lda + gn] = o.o1;
+          if (AdT) AdT[static_cast<int64_t>(gn) * e.ldt + gm] = o.o1;
+        }
       }
     }
   }
@@ -88,6 +108,7 @@ cudaError_t simt_gemm(const GemmArgs& a, cudaStream_t s) {
   p.B[1] = static_cast<const float*>(a.B1); p.ldb[1] = a.ldb1;
   p.C[0] = a.C0; p.ldc[0] = a.ldc0; p.bias[0] = a.bias0;
   p.C[1] = a.C1; p.ldc[1] = a.ldc1; p.bias[1] = a.bias1;
+  p.epi = a.epi;
   dim3 grid((a.N + TN - 1) / TN, (a.M + TM - 1) / TM);
   simt_dual_gemm_kernel<<<grid, 256, 0, s>>>(p);
   return cudaGetLastError();

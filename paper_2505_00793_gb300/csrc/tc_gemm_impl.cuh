@@ -1,0 +1,829 @@
+// Dual-number bf16 GEMM on the 5th-generation tensor cores (tcgen05 + TMEM + TMA), sm_103a.
+//
+// One launch evaluates a Linear layer of the forward-over-reverse pass (Section 2.2's
+// forward-over-reverse HVP applied layer by layer): the primal product P = A B^T and its
+// tangent P' = A' B^T + A B'^T share the A and B shared-memory tiles, so four TMA tiles
+// feed three tensor-core products per K block.  Every product term is optional (bit mask),
+// which gives the primal-only layer, the input layer (A' = 0) and the weight-tangent
+// product [a'; a]^T [dz; dz'] from the same kernel.
+//
+// CTA = 6 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues tcgen05.mma from
+// one thread, warps 2..5 drain the accumulators (tcgen05.ld) and run the fused epilogue
+// (bias, activation and its derivatives, bf16 operand stores for the next GEMM in both
+// row-major and transposed layouts).  Tile 128 x BN x (64 KA) (bf16, 128-byte swizzle, KA
+// swizzle atoms per pipeline stage), multi-stage mbarrier pipeline.  Row-major outputs are
+// staged in swizzled shared memory and written by per-warp TMA stores (coalesced); the
+// transposed operand copies are written directly (consecutive lanes = consecutive rows).  GEMMs with few output tiles split K across a thread-block
+// cluster of S CTAs; the partial accumulators meet in distributed shared memory and each
+// CTA reduces 128/S rows in a fixed order (deterministic).  Every mbarrier wait is bounded;
+// on expiry the CTA records DEV_TIMEOUT and carries on to the end without further waits.
+// Implementation of the tcgen05 dual GEMM, included by tc_gemm.cu (plain stores) and by
+// tc_gemm_act.cu (activation epilogues).  The epilogue mode and the activation are template
+// parameters so that each kernel instance carries only its own per-element code.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+#include <string.h>
+
+#include "device_math.cuh"
+#include "internal.h"
+
+namespace mf {
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;                 // bf16 elements per 128-byte swizzle row
+constexpr int MAX_STAGES = 8;
+constexpr int THREADS = 192;
+constexpr long long WAIT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
+
+struct TcParams {
+  int M, N, K;
+  unsigned terms;
+  int stages;
+  int split;
+  int tma_store;          // 1: row-major outputs through TMA stores
+  int st_c0, st_c1, st_a, st_ad;   // which row-major outputs exist
+  int a0_off, a1_off, b0_off, b1_off, stage_bytes, tx_bytes;
+  float* C0; int ldc0; const float* bias0;
+  float* C1; int ldc1; const float* bias1;
+  EpiParams epi;
+  int* status;
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait: returns false (and flags the status word) if the phase never completes.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* status) {
+  if (mbar_try_wait(bar, parity)) return true;
+  long long t0 = clock64();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (clock64() - t0 > WAIT_CYCLES) {
+      if (status) atomicExch(status, DEV_TIMEOUT);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                            int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row groups of
+// 1024 bytes (stride byte offset), descriptor version 1.
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(1) << 16;              // leading byte offset (unused here)
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;      // stride byte offset
+  d |= static_cast<uint64_t>(1) << 46;              // version
+  d |= static_cast<uint64_t>(2) << 61;              // SWIZZLE_128B
+  return d;
+}
+
+// TMEM allocation size: a power of two >= 32 columns covering the accumulators.
+__host__ __device__ constexpr uint32_t tmem_cols(int needed) {
+  return needed <= 32 ? 32u : needed <= 64 ? 64u : needed <= 128 ? 128u : needed <= 256 ? 256u : 512u;
+}
+
+// Instruction descriptor, kind::f16: D f32, A/B bf16, both K-major, M = 128, N = BN.
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(n >> 3) << 17) |
+         (static_cast<uint32_t>(m >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t dtmem, uint64_t ad, uint64_t bd,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(dtmem),
+      "l"(ad), "l"(bd), "r"(idesc), "r"(accumulate));
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t dsmem_addr(uint32_t local_addr, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local_addr), "r"(rank));
+  return remote;
+}
+
+__device__ __forceinline__ void st_dsmem4(uint32_t remote_addr, float a, float b, float c, float d) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(remote_addr), "f"(a),
+               "f"(b), "f"(c), "f"(d)
+               : "memory");
+}
+
+__device__ __forceinline__ void epi_bar() {   // the 4 epilogue warps only
+  asm volatile("bar.sync 1, 128;" ::: "memory");
+}
+
+// Row-per-thread epilogue for 16 consecutive columns (no split): float32 outputs, the
+// row-major bf16 operand rows and the transposed bf16 operand columns.
+template <int MODE, int ACT>
+__device__ __forceinline__ void epilogue16(const TcParams& p, int row, int col0,
+                                           const float (&v0)[16], const float (&v1)[16],
+                                           bool dual) {
+  const EpiParams e = p.epi;
+  const bool rowok = row < p.M;
+  float o0[16], o1[16], c0[16], c1[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const int n = col0 + j;
+    const bool ok = rowok && n < p.N;
+    EpiOut o;
+    if (ok) o = epi_eval_t<MODE, ACT>(e, row, n, v0[j], v1[j], p.bias0, p.bias1, dual);
+    else o.c0 = o.c1 = o.o0 = o.o1 = 0.f;
+    c0[j] = o.c0; c1[j] = o.c1; o0[j] = o.o0; o1[j] = o.o1;
+  }
+  const bool full = rowok && col0 + 16 <= p.N;
+  if (rowok) {
+    if (p.C0) {
+      float* dst = p.C0 + static_cast<int64_t>(row) * p.ldc0 + col0;
+      if (full && !(p.ldc0 & 3) && !(reinterpret_cast<uintptr_t>(p.C0) & 15)) {
+#pragma unroll
+        for (int j = 0; j < 16; j += 4)
+          *reinterpret_cast<float4*>(dst + j) = make_float4(c0[j], c0[j + 1], c0[j + 2], c0[j + 3]);
+      } else {
+        for (int j = 0; j < 16; ++j) if (col0 + j < p.N) dst[j] = c0[j];
+      }
+    }
+    if (p.C1 && dual) {
+      float* dst = p.C1 + static_cast<int64_t>(row) * p.ldc1 + col0;
+      if (full && !(p.ldc1 & 3) && !(reinterpret_cast<uintptr_t>(p.C1) & 15)) {
+#pragma unroll
+        for (int j = 0; j < 16; j += 4)
+          *reinterpret_cast<float4*>(dst + j) = make_float4(c1[j], c1[j + 1], c1[j + 2], c1[j + 3]);
+      } else {
+        for (int j = 0; j < 16; ++j) if (col0 + j < p.N) dst[j] = c1[j];
+      }
+    }
+  }
+  if constexpr (MODE == EPI_STORE) return;
+  // row-major operand copies (ld multiple of 8 elements, col0 multiple of 16)
+  __nv_bfloat16* A = static_cast<__nv_bfloat16*>(e.A);
+  __nv_bfloat16* Ad = static_cast<__nv_bfloat16*>(e.Ad);
+  if (rowok) {
+    for (int w = 0; w < 2; ++w) {
+      __nv_bfloat16* X = w == 0 ? A : Ad;
+      const float* o = w == 0 ? o0 : o1;
+      if (!X || (w == 1 && !dual)) continue;
+      __nv_bfloat16* dst = X + static_cast<int64_t>(row) * e.lda + col0;
+      if (full) {
+        uint4 q0 = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]),
+                              pack_bf16x2(o[4], o[5]), pack_bf16x2(o[6], o[7]));
+        uint4 q1 = make_uint4(pack_bf16x2(o[8], o[9]), pack_bf16x2(o[10], o[11]),
+                              pack_bf16x2(o[12], o[13]), pack_bf16x2(o[14], o[15]));
+        reinterpret_cast<uint4*>(dst)[0] = q0;
+        reinterpret_cast<uint4*>(dst)[1] = q1;
+      } else {
+        for (int j = 0; j < 16; ++j) if (col0 + j < p.N) dst[j] = __float2bfloat16_rn(o[j]);
+      }
+    }
+  }
+  // transposed operand copies: for each column, the 32 lanes of the warp write 32
+  // consecutive rows (coalesced)
+  __nv_bfloat16* AT = static_cast<__nv_bfloat16*>(e.AT);
+  __nv_bfloat16* AdT = static_cast<__nv_bfloat16*>(e.AdT);
+  if (rowok) {
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const int n = col0 + j;
+      if (n >= p.N) break;
+      if (AT) AT[static_cast<int64_t>(n) * e.ldt + row] = __float2bfloat16_rn(o0[j]);
+      if (AdT && dual) AdT[static_cast<int64_t>(n) * e.ldt + row] = __float2bfloat16_rn(o1[j]);
+    }
+  }
+}
+
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(x), "r"(y), "r"(smem_u32(src))
+      : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+// Per-warp staging of a 32-row slab of the tile for TMA stores (128-byte swizzle: the
+// 16-byte chunk j of row r sits at chunk position j ^ (r % 8) of the row's 128 bytes).
+// Layout per warp: C0 [2 boxes of 32x32 f32] | C1 [2 boxes] | A [32x64 bf16] | Ad [32x64].
+constexpr int STG_F32_BOX = 32 * 32 * 4;          // 4 KB
+constexpr int STG_BF16_BOX = 32 * 64 * 2;         // 4 KB
+constexpr int STG_WARP = 4 * STG_F32_BOX + 2 * STG_BF16_BOX;   // 24 KB
+
+// TMA-store epilogue of one warp (32 rows) over the tile's BN columns, 64 at a time.
+template <int BN, int MODE, int ACT>
+__device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMap* mC0,
+                                             const CUtensorMap* mC1, const CUtensorMap* mA,
+                                             const CUtensorMap* mAd, uint8_t* stg, uint32_t taddr,
+                                             int q, int lane, int m0, int n0, bool dual) {
+  const EpiParams e = p.epi;
+  const int row = m0 + q * 32 + lane;
+  const bool rowok = row < p.M;
+  uint8_t* sC0 = stg;
+  uint8_t* sC1 = stg + 2 * STG_F32_BOX;
+  uint8_t* sA = stg + 4 * STG_F32_BOX;
+  uint8_t* sAd = sA + STG_BF16_BOX;
+  const int sw = lane & 7;
+  __nv_bfloat16* AT = static_cast<__nv_bfloat16*>(e.AT);
+  __nv_bfloat16* AdT = static_cast<__nv_bfloat16*>(e.AdT);
+  for (int c = 0; c < BN; c += 64) {
+    if (c > 0) {
+      if (lane == 0) bulk_wait_read();
+      __syncwarp();
+    }
+#pragma unroll 1
+    for (int sub = 0; sub < 4; ++sub) {
+      const int cc = c + sub * 16;          // tile column of this 16-column group
+      if (cc >= BN) break;
+      float v0[16], v1[16];
+      tmem_ld16(taddr + cc, v0);
+      if (dual) tmem_ld16(taddr + BN + cc, v1);
+      else {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v1[j] = 0.f;
+      }
+      float c0[16], c1[16], o0[16], o1[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const int n = n0 + cc + j;
+        EpiOut o;
+        if (rowok && n < p.N) o = epi_eval_t<MODE, ACT>(e, row, n, v0[j], v1[j], p.bias0, p.bias1, dual);
+        else o.c0 = o.c1 = o.o0 = o.o1 = 0.f;
+        c0[j] = o.c0; c1[j] = o.c1; o0[j] = o.o0; o1[j] = o.o1;
+      }
+      // float32 slabs: box (sub / 2), chunks (sub % 2) * 4 .. + 3 of the 128-byte row
+      const int fb = (sub >> 1) * STG_F32_BOX + lane * 128;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int pos = ((((sub & 1) * 4) + k) ^ sw) * 16;
+        if (p.st_c0)
+          *reinterpret_cast<float4*>(sC0 + fb + pos) =
+              make_float4(c0[4 * k], c0[4 * k + 1], c0[4 * k + 2], c0[4 * k + 3]);
+        if (p.st_c1)
+          *reinterpret_cast<float4*>(sC1 + fb + pos) =
+              make_float4(c1[4 * k], c1[4 * k + 1], c1[4 * k + 2], c1[4 * k + 3]);
+      }
+      // bf16 slabs: chunks sub * 2 .. + 1 of the 128-byte row
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        const int pos = (((sub * 2) + k) ^ sw) * 16;
+        if (p.st_a)
+          *reinterpret_cast<uint4*>(sA + lane * 128 + pos) =
+              make_uint4(pack_bf16x2(o0[8 * k], o0[8 * k + 1]), pack_bf16x2(o0[8 * k + 2], o0[8 * k + 3]),
+                         pack_bf16x2(o0[8 * k + 4], o0[8 * k + 5]), pack_bf16x2(o0[8 * k + 6], o0[8 * k + 7]));
+        if (p.st_ad)
+          *reinterpret_cast<uint4*>(sAd + lane * 128 + pos) =
+              make_uint4(pack_bf16x2(o1[8 * k], o1[8 * k + 1]), pack_bf16x2(o1[8 * k + 2], o1[8 * k + 3]),
+                         pack_bf16x2(o1[8 * k + 4], o1[8 * k + 5]), pack_bf16x2(o1[8 * k + 6], o1[8 * k + 7]));
+      }
+      // transposed operand copies, coalesced across the warp's rows
+      if (MODE != EPI_STORE && rowok) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const int n = n0 + cc + j;
+          if (n >= p.N) break;
+          if (AT) AT[static_cast<int64_t>(n) * e.ldt + row] = __float2bfloat16_rn(o0[j]);
+          if (AdT && dual) AdT[static_cast<int64_t>(n) * e.ldt + row] = __float2bfloat16_rn(o1[j]);
+        }
+      }
+    }
+    fence_proxy_async();
+    __syncwarp();
+    if (lane == 0) {
+      const int y = m0 + q * 32;
+      if (y < p.M) {
+        for (int b = 0; b < 2; ++b) {
+          const int x = n0 + c + 32 * b;
+          if (x >= p.N) continue;
+          if (p.st_c0) tma_store_2d(mC0, sC0 + b * STG_F32_BOX, x, y);
+          if (p.st_c1) tma_store_2d(mC1, sC1 + b * STG_F32_BOX, x, y);
+        }
+        if (n0 + c < p.N) {
+          if (p.st_a) tma_store_2d(mA, sA, n0 + c, y);
+          if (p.st_ad) tma_store_2d(mAd, sAd, n0 + c, y);
+        }
+      }
+      bulk_commit();
+    }
+  }
+  if (lane == 0) bulk_wait_all();
+  __syncwarp();
+}
+
+template <int BN, int KA, int MODE, int ACT>
+__global__ void __launch_bounds__(THREADS, 1)
+    tc_dual_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
+                        const __grid_constant__ CUtensorMap tmA1,
+                        const __grid_constant__ CUtensorMap tmB0,
+                        const __grid_constant__ CUtensorMap tmB1,
+                        const __grid_constant__ CUtensorMap tmC0,
+                        const __grid_constant__ CUtensorMap tmC1,
+                        const __grid_constant__ CUtensorMap tmA,
+                        const __grid_constant__ CUtensorMap tmAd, const TcParams prm) {
+  // Work on a register copy: a reference into the parameter block would be re-read after
+  // every asm statement with a memory clobber (mbarrier waits, commits, stores).
+  const TcParams p = prm;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[MAX_STAGES];
+  __shared__ __align__(8) uint64_t empty_bar[MAX_STAGES];
+  __shared__ __align__(8) uint64_t acc_bar;
+  __shared__ uint32_t tmem_slot;
+
+  constexpr int SK = BK * KA;            // K elements per pipeline stage
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int m0 = blockIdx.y * BM;
+  const int n0 = blockIdx.x * BN;
+  const int S = p.split;
+  const int nkb = (p.K + SK - 1) / SK;
+  const int kper = (nkb + S - 1) / S;
+  const int kb0 = static_cast<int>(blockIdx.z) * kper;
+  const int nk = max(0, min(nkb, kb0 + kper) - kb0);
+  const unsigned terms = p.terms;
+  const bool dual = (terms & (T_C1_A1B0 | T_C1_A0B1)) != 0;
+  const uint32_t ncols = tmem_cols(dual ? 2 * BN : BN);
+  constexpr int A_ATOM = BM * BK * 2, B_ATOM = BN * BK * 2;
+
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < p.stages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], 1);
+    }
+    mbar_init(&acc_bar, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&tmem_slot)),
+                 "r"(ncols));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---- TMA producer: KA swizzle atoms per operand per stage -------------------------
+      const int stages = p.stages, stage_bytes = p.stage_bytes, tx_bytes = p.tx_bytes;
+      const int a0_off = p.a0_off, a1_off = p.a1_off, b0_off = p.b0_off, b1_off = p.b1_off;
+      int* const status = p.status;
+      for (int i = 0; i < nk; ++i) {
+        const int s = i % stages;
+        const uint32_t ph = (i / stages) & 1;
+        if (!mbar_wait(&empty_bar[s], ph ^ 1, status)) break;
+        uint8_t* st = smem + s * stage_bytes;
+        mbar_expect_tx(&full_bar[s], tx_bytes);
+        const int k = (kb0 + i) * SK;
+#pragma unroll
+        for (int a = 0; a < KA; ++a) {
+          const int ka = k + a * BK;
+          if (a0_off >= 0) tma_load_2d(st + a0_off + a * A_ATOM, &tmA0, &full_bar[s], ka, m0);
+          if (a1_off >= 0) tma_load_2d(st + a1_off + a * A_ATOM, &tmA1, &full_bar[s], ka, m0);
+          if (b0_off >= 0) tma_load_2d(st + b0_off + a * B_ATOM, &tmB0, &full_bar[s], ka, n0);
+          if (b1_off >= 0) tma_load_2d(st + b1_off + a * B_ATOM, &tmB1, &full_bar[s], ka, n0);
+        }
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0 && nk > 0) {
+      // ---- MMA issuer (single thread) -----------------------------------------------
+      constexpr uint32_t idesc = idesc_bf16(BM, BN);
+      const uint32_t d0 = tbase;
+      const uint32_t d1 = tbase + BN;
+      const int stages = p.stages, stage_bytes = p.stage_bytes;
+      const int a0_off = p.a0_off, a1_off = p.a1_off, b0_off = p.b0_off, b1_off = p.b1_off;
+      int* const status = p.status;
+      const uint32_t sbase = smem_u32(smem);
+      bool started0 = false, started1 = false;
+      for (int i = 0; i < nk; ++i) {
+        const int s = i % stages;
+        const uint32_t ph = (i / stages) & 1;
+        if (!mbar_wait(&full_bar[s], ph, status)) break;
+        tc_fence_after();
+        const uint32_t st = sbase + s * stage_bytes;
+#pragma unroll
+        for (int a = 0; a < KA; ++a) {
+          const uint64_t a0 = a0_off >= 0 ? sdesc_sw128(st + a0_off + a * A_ATOM) : 0;
+          const uint64_t a1 = a1_off >= 0 ? sdesc_sw128(st + a1_off + a * A_ATOM) : 0;
+          const uint64_t b0 = b0_off >= 0 ? sdesc_sw128(st + b0_off + a * B_ATOM) : 0;
+          const uint64_t b1 = b1_off >= 0 ? sdesc_sw128(st + b1_off + a * B_ATOM) : 0;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            const uint64_t adv = static_cast<uint64_t>(kk * 2);   // 32 bytes per K=16 step
+            if (terms & T_C0_A0B0) { mma_bf16(d0, a0 + adv, b0 + adv, idesc, started0); started0 = true; }
+            if (terms & T_C0_A1B0) { mma_bf16(d0, a1 + adv, b0 + adv, idesc, started0); started0 = true; }
+            if (terms & T_C0_A0B1) { mma_bf16(d0, a0 + adv, b1 + adv, idesc, started0); started0 = true; }
+            if (terms & T_C1_A1B0) { mma_bf16(d1, a1 + adv, b0 + adv, idesc, started1); started1 = true; }
+            if (terms & T_C1_A0B1) { mma_bf16(d1, a0 + adv, b1 + adv, idesc, started1); started1 = true; }
+          }
+        }
+        mma_commit(&empty_bar[s]);
+      }
+      mma_commit(&acc_bar);
+    }
+    __syncwarp();
+  } else {
+    // ---- accumulator drain: warps 2..5, TMEM lane quadrant = warp % 4 ---------------
+    const int q = warp & 3;
+    const int r = q * 32 + lane;   // row within the tile
+    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    const bool ok = nk > 0 && mbar_wait(&acc_bar, 0, p.status);
+    tc_fence_after();
+    if (S == 1) {
+      if (ok) {
+        if (p.tma_store) {
+          epilogue_tma<BN, MODE, ACT>(p, &tmC0, &tmC1, &tmA, &tmAd, smem + q * STG_WARP, tbase + lane_off,
+                           q, lane, m0, n0, dual);
+        } else {
+#pragma unroll 1
+          for (int c = 0; c < BN; c += 16) {
+            float v0[16], v1[16];
+            tmem_ld16(tbase + lane_off + c, v0);
+            if (dual) tmem_ld16(tbase + lane_off + BN + c, v1);
+            else {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) v1[j] = 0.f;
+            }
+            if (n0 + c < p.N) epilogue16<MODE, ACT>(p, m0 + r, n0 + c, v0, v1, dual);
+          }
+        }
+      }
+    }
+    tc_fence_before();
+  }
+
+  if (S > 1) {
+    // Split K: CTA z of the cluster owns tile rows [z*128/S, (z+1)*128/S).  After a first
+    // cluster barrier (every CTA is done with its pipeline buffers), each CTA pushes its
+    // partial rows into the owner's receive buffer R[acc][src rank][row][BN + 4] with remote
+    // shared-memory stores; after the second barrier each owner sums the S slabs in rank
+    // order (deterministic) and runs the epilogue for its rows.
+    constexpr int LDP = BN + 4;
+    const int nacc = dual ? 2 : 1;
+    const int rows_per = BM / S;
+    const uint32_t z = blockIdx.z;
+    const uint32_t rbase = smem_u32(smem);
+    __syncwarp();
+    cluster_sync_all();
+    if (warp >= 2) {
+      tc_fence_after();
+      const int q = warp & 3;
+      const int r = q * 32 + lane;
+      const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+      const bool ok = nk > 0;
+      const uint32_t owner = static_cast<uint32_t>(r / rows_per);
+      const int rr = r % rows_per;
+      for (int a = 0; a < nacc; ++a) {
+        const uint32_t row_addr = dsmem_addr(
+            rbase + static_cast<uint32_t>((((a * S + z) * rows_per + rr) * LDP) * 4), owner);
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 16) {
+          float v[16];
+          if (ok) {
+            tmem_ld16(tbase + lane_off + a * BN + c, v);
+          } else {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) v[j] = 0.f;
+          }
+#pragma unroll
+          for (int j = 0; j < 16; j += 4)
+            st_dsmem4(row_addr + static_cast<uint32_t>((c + j) * 4), v[j], v[j + 1], v[j + 2], v[j + 3]);
+        }
+      }
+      tc_fence_before();
+    }
+    __syncwarp();
+    cluster_sync_all();   // every partial row has reached its owner
+    if (warp >= 2) {
+      const int e = threadIdx.x - 64;            // 0..127
+      const int r_begin = static_cast<int>(z) * rows_per;
+      float* Rcv = reinterpret_cast<float*>(smem);          // [acc][S][rows_per][LDP]
+      float* R = Rcv + nacc * BM * LDP;                     // reduced rows [acc][rows_per][LDP]
+      // Phase A: sum the S received slabs in rank order (local shared memory).
+      constexpr int VPR = BN / 4;                // float4 per row
+      const int nvec = rows_per * VPR;
+      for (int a = 0; a < nacc; ++a) {
+        for (int it = e; it < nvec; it += 128) {
+          const int rr = it / VPR, c4 = (it % VPR) * 4;
+          float4 acc = *reinterpret_cast<const float4*>(Rcv + ((a * S) * rows_per + rr) * LDP + c4);
+          for (int k = 1; k < S; ++k) {
+            const float4 v = *reinterpret_cast<const float4*>(Rcv + ((a * S + k) * rows_per + rr) * LDP + c4);
+            acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+          }
+          *reinterpret_cast<float4*>(R + (a * rows_per + rr) * LDP + c4) = acc;
+        }
+      }
+      epi_bar();
+      // Phase B: fused epilogue, one column per thread, 8-row chunks (the transposed bf16
+      // operand gets one 16-byte store per chunk; row-major stores are coalesced across
+      // consecutive columns)
+      const int tpc = 128 / (BN < 128 ? BN : 128);   // threads per column
+      const EpiParams ep = p.epi;
+      __nv_bfloat16* AT = static_cast<__nv_bfloat16*>(ep.AT);
+      __nv_bfloat16* AdT = static_cast<__nv_bfloat16*>(ep.AdT);
+      __nv_bfloat16* A = static_cast<__nv_bfloat16*>(ep.A);
+      __nv_bfloat16* Ad = static_cast<__nv_bfloat16*>(ep.Ad);
+      for (int col = e % BN; col < BN; col += 128) {
+        const int n = n0 + col;
+        for (int ch = (e % 128) / (BN < 128 ? BN : 128); ch * 8 < rows_per; ch += tpc) {
+          float t0[8], t1[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int rr = ch * 8 + j;
+            const float v0 = R[rr * LDP + col];
+            const float v1 = dual ? R[(rows_per + rr) * LDP + col] : 0.f;
+            const int m = m0 + r_begin + rr;
+            t0[j] = t1[j] = 0.f;
+            if (m < p.M && n < p.N) {
+              const EpiOut o = epi_eval_t<MODE, ACT>(ep, m, n, v0, v1, p.bias0, p.bias1, dual);
+              if (p.C0) p.C0[static_cast<int64_t>(m) * p.ldc0 + n] = o.c0;
+              if (p.C1 && dual) p.C1[static_cast<int64_t>(m) * p.ldc1 + n] = o.c1;
+              if (MODE != EPI_STORE) {
+                if (A) A[static_cast<int64_t>(m) * ep.lda + n] = __float2bfloat16_rn(o.o0);
+                if (Ad && dual) Ad[static_cast<int64_t>(m) * ep.lda + n] = __float2bfloat16_rn(o.o1);
+              }
+              t0[j] = o.o0;
+              t1[j] = o.o1;
+            }
+          }
+          if (MODE != EPI_STORE && n < p.N) {
+            const int mb = m0 + r_begin + ch * 8;
+            for (int w = 0; w < 2; ++w) {
+              __nv_bfloat16* X = w == 0 ? AT : AdT;
+              const float* t = w == 0 ? t0 : t1;
+              if (!X || (w == 1 && !dual)) continue;
+              __nv_bfloat16* dst = X + static_cast<int64_t>(n) * ep.ldt + mb;
+              if (mb + 8 <= p.M) {
+                *reinterpret_cast<uint4*>(dst) =
+                    make_uint4(pack_bf16x2(t[0], t[1]), pack_bf16x2(t[2], t[3]),
+                               pack_bf16x2(t[4], t[5]), pack_bf16x2(t[6], t[7]));
+              } else {
+                for (int j = 0; j < 8; ++j) if (mb + j < p.M) dst[j] = __float2bfloat16_rn(t[j]);
+              }
+            }
+          }
+        }
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tbase),
+                 "r"(ncols));
+  }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion,
+                                  CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                         cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  }
+  return fn;
+}
+
+// 2-D tensor map, 128-byte swizzle: inner extent `inner` elements, `rows` rows, row pitch
+// `ld` elements, box box_inner x box_rows.
+bool make_map2(CUtensorMap* m, CUtensorMapDataType dt, int esize, const void* ptr, int inner,
+               int rows, int ld, int box_inner, int box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * esize};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(box_inner), static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, dt, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+         CUDA_SUCCESS;
+}
+
+// K-major bf16 operand [rows][K] (leading dimension ld), box 64 x box_rows.
+bool make_map(CUtensorMap* m, const void* ptr, int K, int rows, int ld, int box_rows) {
+  return make_map2(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, ptr, K, rows, ld, BK, box_rows);
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+// Split of K across a cluster: double S while the grid stays within ~1.2 waves of 152 SMs
+// and every split keeps at least two K stages.
+int choose_split(int tiles, int nkb) {
+  int S = 1;
+  while (S < 4 && tiles * S * 2 <= 184 && (nkb + 2 * S - 1) / (2 * S) >= 2) S *= 2;
+  return S;
+}
+
+template <int BN, int KA, int MODE, int ACT>
+cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
+  const unsigned t = a.terms;
+  const bool useA0 = t & (T_C0_A0B0 | T_C0_A0B1 | T_C1_A0B1);
+  const bool useA1 = t & (T_C0_A1B0 | T_C1_A1B0);
+  const bool useB0 = t & (T_C0_A0B0 | T_C0_A1B0 | T_C1_A1B0);
+  const bool useB1 = t & (T_C0_A0B1 | T_C1_A0B1);
+  const bool dual = t & (T_C1_A1B0 | T_C1_A0B1);
+  TcParams p;
+  memset(&p, 0, sizeof(p));
+  p.M = a.M; p.N = a.N; p.K = a.K; p.terms = t;
+  const int a_bytes = KA * BM * BK * 2, b_bytes = KA * BN * BK * 2;
+  int off = 0;
+  p.a0_off = useA0 ? (off += a_bytes, off - a_bytes) : -1;
+  p.a1_off = useA1 ? (off += a_bytes, off - a_bytes) : -1;
+  p.b0_off = useB0 ? (off += b_bytes, off - b_bytes) : -1;
+  p.b1_off = useB1 ? (off += b_bytes, off - b_bytes) : -1;
+  p.stage_bytes = off;
+  p.tx_bytes = off;
+  const int budget = 220 * 1024;
+  int stages = budget / off;
+  if (stages > MAX_STAGES) stages = MAX_STAGES;
+  if (stages < 2) { *why = "tile does not fit shared memory"; return cudaErrorInvalidValue; }
+  p.stages = stages;
+  p.C0 = a.C0; p.ldc0 = a.ldc0; p.bias0 = a.bias0;
+  p.C1 = dual ? a.C1 : nullptr; p.ldc1 = a.ldc1; p.bias1 = a.bias1;
+  p.epi = a.epi;
+  p.status = a.status;
+
+  const int tiles_n = (a.N + BN - 1) / BN, tiles_m = (a.M + BM - 1) / BM;
+  const int nkb = (a.K + BK * KA - 1) / (BK * KA);
+  int S = a.split_k > 0 ? a.split_k : (BN > 128 ? 1 : choose_split(tiles_n * tiles_m, nkb));
+  if (S != 1 && S != 2 && S != 4 && S != 8) { *why = "split_k must be 1, 2, 4 or 8"; return cudaErrorInvalidValue; }
+  if (BN > 128) S = 1;
+  if (S > nkb) S = 1;
+  p.split = S;
+
+  CUtensorMap mA0, mA1, mB0, mB1, mC0, mC1, mA, mAd;
+  memset(&mA0, 0, sizeof(mA0)); memset(&mA1, 0, sizeof(mA1));
+  memset(&mB0, 0, sizeof(mB0)); memset(&mB1, 0, sizeof(mB1));
+  memset(&mC0, 0, sizeof(mC0)); memset(&mC1, 0, sizeof(mC1));
+  memset(&mA, 0, sizeof(mA)); memset(&mAd, 0, sizeof(mAd));
+  if (useA0 && !make_map(&mA0, a.A0, a.K, a.M, a.lda0, BM)) { *why = "tensor map A0"; return cudaErrorInvalidValue; }
+  if (useA1 && !make_map(&mA1, a.A1, a.K, a.M, a.lda1, BM)) { *why = "tensor map A1"; return cudaErrorInvalidValue; }
+  if (useB0 && !make_map(&mB0, a.B0, a.K, a.N, a.ldb0, BN)) { *why = "tensor map B0"; return cudaErrorInvalidValue; }
+  if (useB1 && !make_map(&mB1, a.B1, a.K, a.N, a.ldb1, BN)) { *why = "tensor map B1"; return cudaErrorInvalidValue; }
+
+  // Row-major outputs through TMA stores when every one of them is aligned for it.
+  const bool act = a.epi.mode != EPI_STORE;
+  p.st_c0 = p.C0 != nullptr;
+  p.st_c1 = p.C1 != nullptr;
+  p.st_a = act && a.epi.A != nullptr;
+  p.st_ad = act && dual && a.epi.Ad != nullptr;
+  bool tma_ok = S == 1 && BN >= 64;   // store boxes are 64 columns wide
+  if (p.st_c0) tma_ok = tma_ok && aligned16(p.C0) && !(p.ldc0 & 3);
+  if (p.st_c1) tma_ok = tma_ok && aligned16(p.C1) && !(p.ldc1 & 3);
+  if (p.st_a) tma_ok = tma_ok && aligned16(a.epi.A) && !(a.epi.lda & 7);
+  if (p.st_ad) tma_ok = tma_ok && aligned16(a.epi.Ad) && !(a.epi.lda & 7);
+  if (tma_ok && p.st_c0)
+    tma_ok = make_map2(&mC0, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, p.C0, a.N, a.M, p.ldc0, 32, 32);
+  if (tma_ok && p.st_c1)
+    tma_ok = make_map2(&mC1, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, p.C1, a.N, a.M, p.ldc1, 32, 32);
+  if (tma_ok && p.st_a)
+    tma_ok = make_map2(&mA, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, a.epi.A, a.N, a.M, a.epi.lda, 64, 32);
+  if (tma_ok && p.st_ad)
+    tma_ok = make_map2(&mAd, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, a.epi.Ad, a.N, a.M, a.epi.lda, 64, 32);
+  p.tma_store = tma_ok ? 1 : 0;
+
+  int need = stages * off;
+  if (S > 1) {
+    // split-K: partial tiles [acc][128][BN+4] plus this CTA's reduced rows [acc][128/S][BN+4]
+    const int partial_bytes = (dual ? 2 : 1) * (BM + BM / S) * (BN + 4) * 4;
+    if (partial_bytes > need) need = partial_bytes;
+  }
+  if (p.tma_store && 4 * STG_WARP > need) need = 4 * STG_WARP;
+  const int smem = need + 1024;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(tc_dual_gemm_kernel<BN, KA, MODE, ACT>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, 225 * 1024);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  if (smem > 225 * 1024) { *why = "shared memory budget exceeded"; return cudaErrorInvalidValue; }
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3(tiles_n, tiles_m, S);
+  cfg.blockDim = dim3(THREADS, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = S;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, tc_dual_gemm_kernel<BN, KA, MODE, ACT>, mA0, mA1, mB0, mB1, mC0, mC1, mA,
+                            mAd, p);
+}
+
+// Dispatch over the tile width for one epilogue (MODE, ACT).
+template <int MODE, int ACT>
+cudaError_t launch_bn(const GemmArgs& a, cudaStream_t s, const char** why, int bn, int ka) {
+  (void)ka;
+  switch (bn) {
+    case 16: return launch_cfg<16, 1, MODE, ACT>(a, s, why);
+    case 32: return launch_cfg<32, 1, MODE, ACT>(a, s, why);
+    case 64: return launch_cfg<64, 1, MODE, ACT>(a, s, why);
+    case 128: return launch_cfg<128, 1, MODE, ACT>(a, s, why);
+    case 256: return launch_cfg<256, 1, MODE, ACT>(a, s, why);
+  }
+  *why = "unsupported tile width";
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace
+}  // namespace mf

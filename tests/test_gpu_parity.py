@@ -39,6 +39,9 @@ BF16_CASES = {
     "deep_small": synth.Workload("deep_small", [256] * 5, "silu", "squared", "bf16", B=64, T=6,
                                  B_outer=64, momentum=0.9, meta_kind=PLR,
                                  loglr_mean=math.log(1e-2), loglr_std=0.1),
+    # K large enough for the cluster split-K path (S = 2 and 4) with ragged M = 100 / 120
+    "wide_split": synth.Workload("wide_split", [1024, 384, 200, 10], "gelu", "ce", "bf16", B=100,
+                                 T=3, B_outer=120, alpha=0.05),
     "mlp_ex_slr": synth.Workload("mlp_ex_slr", [64, 192, 130, 8], "tanh", "squared", "bf16",
                                  B=48, T=4, B_outer=32, momentum=0.5, meta_kind=EX | SLR,
                                  noise_std=0.1, extra={"scalar_loglr": math.log(0.05)}),
@@ -187,9 +190,11 @@ def test_special_cases_on_gpu():
 
 
 @pytest.mark.gpu
-def test_deterministic_repeat():
-    """Two calls on the same inputs give bit-identical meta-gradients (fixed-order sums)."""
-    w = BF16_CASES["mlp_ex_slr"]
+@pytest.mark.parametrize("name", ["mlp_ex_slr", "wide_split"])
+def test_deterministic_repeat(name):
+    """Two calls on the same inputs give bit-identical meta-gradients (fixed-order sums,
+    including the cluster split-K reduction)."""
+    w = BF16_CASES[name]
     inp = synth.make_inputs(w)
     a = run_meta_grad(w, inp)
     b = run_meta_grad(w, inp)
