@@ -174,12 +174,20 @@ const char* mf_last_error(mf_handle h);
 
 /* Diagnostics.  mf_stats: kernel launches issued by the handle since creation and the
  * largest workspace it has held.  mf_set_kernel_timing(h, 1) records CUDA events around
- * every launch of the bf16 dual GEMM (slower; for measurement);  mf_kernel_time returns
- * the summed milliseconds and launch count of that kernel since the last reset, plus its
- * algorithmic flops (2*M*N*K per accumulated product term), then resets. */
+ * every launch of the bf16 dual GEMM (inside the captured graph when graphs are in use);
+ * mf_kernel_time synchronises and returns the summed milliseconds and launch count of that
+ * kernel since the last reset - for graph replays, those of the most recent replay - plus
+ * its algorithmic flops (2*M*N*K per accumulated product term), then resets. */
 mf_status mf_stats(mf_handle h, uint64_t* launches, size_t* peak_workspace_bytes);
 mf_status mf_set_kernel_timing(mf_handle h, int enable);
 mf_status mf_kernel_time(mf_handle h, double* ms, uint64_t* launches, double* flops);
+
+/* Library options.  MF_OPT_CUDA_GRAPHS (default 1): a call of mf_meta_grad, mf_inner_rollout
+ * or mf_hvp repeated with the same shapes and pointers is captured into a CUDA graph on its
+ * second occurrence and replayed afterwards, on a library-owned stream that is ordered after
+ * and before the caller's stream with events.  0 launches every kernel individually. */
+enum { MF_OPT_CUDA_GRAPHS = 1 };
+mf_status mf_set_option(mf_handle h, int option, int value);
 
 /* Host-side fault injection for tests: kind 1 = the next workspace allocation fails;
  * kind 2 = the next mf_sync reports MF_ERR_TIMEOUT as if a device wait had expired;

@@ -51,6 +51,22 @@ struct mf_ctx {
   bool timing = false;
   std::vector<std::pair<cudaEvent_t, cudaEvent_t>> evs;
   double timed_flops = 0.0;
+
+  // CUDA graphs: a call repeated with the same shapes and pointers is captured once (on the
+  // second occurrence) and replayed from then on, on the library's own stream.
+  struct GraphCache {
+    uint64_t key = 0, pending = 0;
+    cudaGraphExec_t exec = nullptr;
+    uint64_t launches = 0;
+    // kernel timing: event pairs recorded inside the graph (re-recorded by each replay)
+    std::vector<std::pair<cudaEvent_t, cudaEvent_t>> evs;
+    double flops = 0.0;
+  };
+  GraphCache* timed_replay = nullptr;   // graph whose events hold the last replay's times
+  bool use_graphs = true;
+  GraphCache g_meta, g_roll, g_hvp;
+  cudaStream_t gstream = nullptr;
+  cudaEvent_t ev_in = nullptr, ev_out = nullptr;
 };
 
 namespace {
@@ -141,7 +157,10 @@ Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slot
   return p;
 }
 
+void drop_graphs(mf_ctx* h);
+
 void release_ws(mf_ctx* h) {
+  drop_graphs(h);
   if (!h->ws) return;
   cudaDeviceSynchronize();
   if (h->ufree) h->ufree(h->ws, h->ws_bytes, nullptr, h->uctx);
@@ -169,6 +188,99 @@ mf_status ensure_ws(mf_ctx* h, size_t bytes, cudaStream_t s) {
   h->ws_bytes = bytes;
   h->peak = std::max(h->peak, bytes);
   return MF_OK;
+}
+
+// ---- CUDA graph replay ---------------------------------------------------------------------
+uint64_t mix_key(uint64_t h, uint64_t v) {
+  h ^= v + 0x9e3779b97f4a7c15ULL + (h << 6) + (h >> 2);
+  return h;
+}
+
+void drop_graph(mf_ctx::GraphCache& g) {
+  if (g.exec) cudaGraphExecDestroy(g.exec);
+  g.exec = nullptr;
+  g.key = g.pending = 0;
+  for (auto& e : g.evs) { cudaEventDestroy(e.first); cudaEventDestroy(e.second); }
+  g.evs.clear();
+  g.flops = 0.0;
+}
+
+void drop_graphs(mf_ctx* h) {
+  h->timed_replay = nullptr;
+  drop_graph(h->g_meta);
+  drop_graph(h->g_roll);
+  drop_graph(h->g_hvp);
+}
+
+mf_status graph_launch(mf_ctx* h, mf_ctx::GraphCache& g, cudaStream_t user) {
+  MF_CUDA(h, cudaEventRecord(h->ev_in, user));
+  MF_CUDA(h, cudaStreamWaitEvent(h->gstream, h->ev_in, 0));
+  MF_CUDA(h, cudaGraphLaunch(g.exec, h->gstream));
+  MF_CUDA(h, cudaEventRecord(h->ev_out, h->gstream));
+  MF_CUDA(h, cudaStreamWaitEvent(user, h->ev_out, 0));
+  h->launches += g.launches;
+  h->timed_replay = g.evs.empty() ? nullptr : &g;
+  return MF_OK;
+}
+
+// Runs body(stream) eagerly, or replays / captures it as a CUDA graph.  The first call with
+// a given key runs eagerly (it may allocate the workspace and set kernel attributes); the
+// second captures on the library stream; later ones replay.
+template <typename F>
+mf_status run_graphed(mf_ctx* h, mf_ctx::GraphCache& g, uint64_t key, cudaStream_t user, F&& body) {
+  key = mix_key(key, reinterpret_cast<uintptr_t>(h->ws));
+  key = mix_key(key, h->ws_bytes);
+  key = mix_key(key, h->timing ? 1 : 0);
+  if (!h->use_graphs || !h->gstream) return body(user);
+  if (g.exec && g.key == key) return graph_launch(h, g, user);
+  if (g.pending != key) {
+    if (g.exec) drop_graph(g);
+    g.pending = key;
+    return body(user);
+  }
+  // second identical call: capture
+  if (h->ws == nullptr) return body(user);
+  const uint64_t l0 = h->launches;
+  // events recorded while capturing belong to the graph
+  std::vector<std::pair<cudaEvent_t, cudaEvent_t>> outer_evs;
+  outer_evs.swap(h->evs);
+  const double outer_flops = h->timed_flops;
+  h->timed_flops = 0.0;
+  MF_CUDA(h, cudaStreamBeginCapture(h->gstream, cudaStreamCaptureModeThreadLocal));
+  const mf_status st = body(h->gstream);
+  cudaGraph_t graph = nullptr;
+  const cudaError_t ce = cudaStreamEndCapture(h->gstream, &graph);
+  std::vector<std::pair<cudaEvent_t, cudaEvent_t>> graph_evs;
+  graph_evs.swap(h->evs);
+  h->evs.swap(outer_evs);
+  const double graph_flops = h->timed_flops;
+  h->timed_flops = outer_flops;
+  if (st != MF_OK || ce != cudaSuccess || !graph) {
+    if (graph) cudaGraphDestroy(graph);
+    for (auto& e : graph_evs) { cudaEventDestroy(e.first); cudaEventDestroy(e.second); }
+    cudaGetLastError();
+    h->launches = l0;
+    g.pending = 0;
+    if (st != MF_OK) return st;
+    return fail(h, MF_ERR_CUDA, std::string("graph capture failed: ") + cudaGetErrorString(ce));
+  }
+  cudaGraphExec_t exec = nullptr;
+  const cudaError_t ie = cudaGraphInstantiate(&exec, graph, 0);
+  cudaGraphDestroy(graph);
+  if (ie != cudaSuccess) {
+    for (auto& e : graph_evs) { cudaEventDestroy(e.first); cudaEventDestroy(e.second); }
+    cudaGetLastError();
+    h->launches = l0;
+    g.pending = 0;
+    return fail(h, MF_ERR_CUDA, std::string("graph instantiate failed: ") + cudaGetErrorString(ie));
+  }
+  g.exec = exec;
+  g.key = key;
+  g.evs.swap(graph_evs);
+  g.flops = graph_flops;
+  g.launches = h->launches - l0;
+  h->launches = l0;
+  return graph_launch(h, g, user);
 }
 
 // ---- the MLP executor --------------------------------------------------------------------
@@ -213,11 +325,16 @@ struct Exec {
     if (st != MF_OK) return;
     g.status = h->d_status;
     cudaEvent_t e0 = nullptr, e1 = nullptr;
+    unsigned ev_flags = cudaEventRecordDefault;
     const bool tc = h->bf16;
     if (tc && h->timing) {
       cudaEventCreate(&e0);
       cudaEventCreate(&e1);
-      cudaEventRecord(e0, s);
+      // inside a stream capture an external record becomes an event-record graph node
+      cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+      cudaStreamIsCapturing(s, &cs);
+      ev_flags = cs == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : cudaEventRecordDefault;
+      cudaEventRecordWithFlags(e0, s, ev_flags);
     }
     cudaError_t e;
     const char* why = "";
@@ -230,7 +347,7 @@ struct Exec {
     }
     launched();
     if (tc && h->timing) {
-      cudaEventRecord(e1, s);
+      cudaEventRecordWithFlags(e1, s, ev_flags);
       h->evs.emplace_back(e0, e1);
       h->timed_flops += 2.0 * g.M * g.N * static_cast<double>(g.K) * mf::term_count(g.terms);
     }
@@ -665,8 +782,12 @@ mf_status mf_create(const mf_model_desc* d, mf_handle* out) {
   h->maxd = *std::max_element(h->dims.begin(), h->dims.end());
   h->bf16 = d->precision == MF_PREC_BF16;
   if (cudaMalloc(&h->d_status, sizeof(int)) != cudaSuccess ||
-      cudaMemset(h->d_status, 0, sizeof(int)) != cudaSuccess) {
+      cudaMemset(h->d_status, 0, sizeof(int)) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&h->gstream, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_in, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_out, cudaEventDisableTiming) != cudaSuccess) {
     cudaGetLastError();
+    if (h->d_status) cudaFree(h->d_status);
     delete h;
     return MF_ERR_CUDA;
   }
@@ -679,7 +800,11 @@ mf_status mf_destroy(mf_handle h) {
   cudaDeviceSynchronize();
   release_ws(h);
   for (auto& e : h->evs) { cudaEventDestroy(e.first); cudaEventDestroy(e.second); }
+  drop_graphs(h);
   if (h->d_status) cudaFree(h->d_status);
+  if (h->gstream) cudaStreamDestroy(h->gstream);
+  if (h->ev_in) cudaEventDestroy(h->ev_in);
+  if (h->ev_out) cudaEventDestroy(h->ev_out);
   delete h;
   return MF_OK;
 }
@@ -730,8 +855,19 @@ mf_status mf_inner_rollout(mf_handle h, const mf_loop_desc* lp, const float* the
   if ((st = check_x(h, inner_x, lp->B)) != MF_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   h->last_stream = s;
-  return h->bf16 ? rollout_impl<__nv_bfloat16>(h, lp, theta0, eta, inner_x, inner_y, thetaT, s)
-                 : rollout_impl<float>(h, lp, theta0, eta, inner_x, inner_y, thetaT, s);
+  uint64_t key = 0x726f6c6cULL;
+  for (uint64_t v : {static_cast<uint64_t>(lp->T), static_cast<uint64_t>(lp->B),
+                     static_cast<uint64_t>(lp->meta_kind),
+                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->alpha)),
+                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->momentum)),
+                     reinterpret_cast<uint64_t>(theta0), reinterpret_cast<uint64_t>(eta),
+                     reinterpret_cast<uint64_t>(inner_x), reinterpret_cast<uint64_t>(inner_y),
+                     reinterpret_cast<uint64_t>(thetaT)})
+    key = mix_key(key, v);
+  return run_graphed(h, h->g_roll, key, s, [&](cudaStream_t st) {
+    return h->bf16 ? rollout_impl<__nv_bfloat16>(h, lp, theta0, eta, inner_x, inner_y, thetaT, st)
+                   : rollout_impl<float>(h, lp, theta0, eta, inner_x, inner_y, thetaT, st);
+  });
 }
 
 mf_status mf_hvp(mf_handle h, int B, const float* theta, const void* x, const void* y,
@@ -745,8 +881,17 @@ mf_status mf_hvp(mf_handle h, int B, const float* theta, const void* x, const vo
   if (st != MF_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   h->last_stream = s;
-  return h->bf16 ? hvp_impl<__nv_bfloat16>(h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, s)
-                 : hvp_impl<float>(h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, s);
+  uint64_t key = 0x687670ULL;
+  for (uint64_t v2 : {static_cast<uint64_t>(B), reinterpret_cast<uint64_t>(theta),
+                      reinterpret_cast<uint64_t>(x), reinterpret_cast<uint64_t>(y),
+                      reinterpret_cast<uint64_t>(ex_w), reinterpret_cast<uint64_t>(v),
+                      reinterpret_cast<uint64_t>(Hv), reinterpret_cast<uint64_t>(tangent_losses),
+                      reinterpret_cast<uint64_t>(grad)})
+    key = mix_key(key, v2);
+  return run_graphed(h, h->g_hvp, key, s, [&](cudaStream_t st) {
+    return h->bf16 ? hvp_impl<__nv_bfloat16>(h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, st)
+                   : hvp_impl<float>(h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, st);
+  });
 }
 
 mf_status mf_meta_grad(mf_handle h, const mf_loop_desc* lp, const float* theta0, const float* eta,
@@ -766,15 +911,29 @@ mf_status mf_meta_grad(mf_handle h, const mf_loop_desc* lp, const float* theta0,
   if ((st = check_x(h, outer_x, lp->B_outer)) != MF_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   h->last_stream = s;
-  return h->bf16 ? meta_grad_impl<__nv_bfloat16>(h, lp, theta0, eta, inner_x, inner_y, outer_x,
-                                                 outer_y, d_eta, d_theta0, outer_loss, s)
-                 : meta_grad_impl<float>(h, lp, theta0, eta, inner_x, inner_y, outer_x, outer_y,
-                                         d_eta, d_theta0, outer_loss, s);
+  uint64_t key = 0x6d657461ULL;
+  for (uint64_t v : {static_cast<uint64_t>(lp->T), static_cast<uint64_t>(lp->B),
+                     static_cast<uint64_t>(lp->B_outer), static_cast<uint64_t>(lp->meta_kind),
+                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->alpha)),
+                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->momentum)),
+                     reinterpret_cast<uint64_t>(theta0), reinterpret_cast<uint64_t>(eta),
+                     reinterpret_cast<uint64_t>(inner_x), reinterpret_cast<uint64_t>(inner_y),
+                     reinterpret_cast<uint64_t>(outer_x), reinterpret_cast<uint64_t>(outer_y),
+                     reinterpret_cast<uint64_t>(d_eta), reinterpret_cast<uint64_t>(d_theta0),
+                     reinterpret_cast<uint64_t>(outer_loss)})
+    key = mix_key(key, v);
+  return run_graphed(h, h->g_meta, key, s, [&](cudaStream_t st) {
+    return h->bf16 ? meta_grad_impl<__nv_bfloat16>(h, lp, theta0, eta, inner_x, inner_y, outer_x,
+                                                   outer_y, d_eta, d_theta0, outer_loss, st)
+                   : meta_grad_impl<float>(h, lp, theta0, eta, inner_x, inner_y, outer_x, outer_y,
+                                           d_eta, d_theta0, outer_loss, st);
+  });
 }
 
 mf_status mf_sync(mf_handle h) {
   if (!h) return MF_ERR_INVALID_ARG;
   cudaError_t e = cudaStreamSynchronize(h->last_stream);
+  if (e == cudaSuccess && h->gstream) e = cudaStreamSynchronize(h->gstream);
   if (e != cudaSuccess) return fail(h, MF_ERR_CUDA, std::string("stream: ") + cudaGetErrorString(e));
   int v = 0;
   e = cudaMemcpy(&v, h->d_status, sizeof(int), cudaMemcpyDeviceToHost);
@@ -807,6 +966,19 @@ mf_status mf_kernel_time(mf_handle h, double* ms, uint64_t* launches, double* fl
   if (!h) return MF_ERR_INVALID_ARG;
   double tot = 0.0;
   uint64_t n = 0;
+  double fl = h->timed_flops;
+  if (h->timed_replay) {
+    // one replay's worth of in-graph event pairs (each replay re-records them)
+    auto& g = *h->timed_replay;
+    cudaError_t e = cudaEventSynchronize(g.evs.back().second);
+    if (e != cudaSuccess) return fail(h, MF_ERR_CUDA, cudaGetErrorString(e));
+    for (auto& pr : g.evs) {
+      float t = 0.f;
+      if (cudaEventElapsedTime(&t, pr.first, pr.second) == cudaSuccess) { tot += t; ++n; }
+    }
+    fl += g.flops;
+    h->timed_replay = nullptr;
+  }
   if (!h->evs.empty()) {
     cudaError_t e = cudaEventSynchronize(h->evs.back().second);
     if (e != cudaSuccess) return fail(h, MF_ERR_CUDA, cudaGetErrorString(e));
@@ -820,9 +992,19 @@ mf_status mf_kernel_time(mf_handle h, double* ms, uint64_t* launches, double* fl
   h->evs.clear();
   if (ms) *ms = tot;
   if (launches) *launches = n;
-  if (flops) *flops = h->timed_flops;
+  if (flops) *flops = fl;
   h->timed_flops = 0.0;
   return MF_OK;
+}
+
+mf_status mf_set_option(mf_handle h, int option, int value) {
+  if (!h) return MF_ERR_INVALID_ARG;
+  if (option == MF_OPT_CUDA_GRAPHS) {
+    h->use_graphs = value != 0;
+    if (!h->use_graphs) drop_graphs(h);
+    return MF_OK;
+  }
+  return fail(h, MF_ERR_INVALID_ARG, "unknown option");
 }
 
 mf_status mf_inject_fault(mf_handle h, int kind) {

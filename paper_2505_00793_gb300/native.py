@@ -22,6 +22,7 @@ LOSSES = {"squared": 0, "ce": 1, "next_token_ce": 2}
 PRECISIONS = {"fp32": 0, "bf16": 1}
 MF_META_EXAMPLE_WEIGHTS, MF_META_PARAM_LOGLR, MF_META_SCALAR_LOGLR = 1, 2, 4
 MF_HVP_MIXED_FOR, MF_HVP_REV_REV = 0, 1
+MF_OPT_CUDA_GRAPHS = 1
 STATUS = {0: "MF_OK", 1: "MF_ERR_INVALID_ARG", 2: "MF_ERR_UNSUPPORTED", 3: "MF_ERR_OOM",
           4: "MF_ERR_CUDA", 5: "MF_ERR_NONFINITE", 6: "MF_ERR_TIMEOUT"}
 
@@ -30,7 +31,7 @@ EXPORTS = ["mf_create", "mf_destroy", "mf_set_allocator", "mf_param_count",
            "mf_workspace_bytes", "mf_release_workspace", "mf_inner_rollout", "mf_hvp",
            "mf_meta_grad", "mf_sync", "mf_status_string", "mf_last_error", "mf_stats",
            "mf_set_kernel_timing", "mf_kernel_time", "mf_inject_fault", "mf_dual_gemm_bf16",
-           "mf_hvp_noalloc"]
+           "mf_hvp_noalloc", "mf_set_option"]
 
 
 class mf_model_desc(C.Structure):
@@ -76,6 +77,7 @@ def load(path: str = LIB_PATH) -> C.CDLL:
         "mf_set_kernel_timing": ([H, C.c_int], C.c_int),
         "mf_kernel_time": ([H, dblp, u64p, dblp], C.c_int),
         "mf_inject_fault": ([H, C.c_int], C.c_int),
+        "mf_set_option": ([H, C.c_int, C.c_int], C.c_int),
         "mf_hvp_noalloc": ([C.POINTER(mf_model_desc), C.c_int, vp, vp, vp, vp, vp, vp, vp, vp, vp],
                            C.c_int),
         "mf_dual_gemm_bf16": ([C.c_int, C.c_int, C.c_int, vp, C.c_int, vp, C.c_int, vp, C.c_int, vp,
@@ -226,6 +228,9 @@ class MixFlow:
         self._check(self._lib.mf_kernel_time(self.h, C.byref(ms), C.byref(n), C.byref(fl)),
                     "mf_kernel_time")
         return ms.value, n.value, fl.value
+
+    def set_option(self, option: int, value: int):
+        self._check(self._lib.mf_set_option(self.h, option, value), "mf_set_option")
 
     def inject_fault(self, kind: int):
         self._check(self._lib.mf_inject_fault(self.h, kind), "mf_inject_fault")

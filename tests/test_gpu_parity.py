@@ -200,3 +200,39 @@ def test_deterministic_repeat(name):
     b = run_meta_grad(w, inp)
     assert np.array_equal(a["d_eta"], b["d_eta"])
     assert np.array_equal(a["d_theta0"], b["d_theta0"])
+
+
+@pytest.mark.gpu
+def test_graph_replay_matches_eager():
+    """Repeated calls with the same pointers run eagerly, then capture a CUDA graph, then
+    replay it; new input values behind the same pointers must be picked up by the replay."""
+    torch, native = need_gpu()
+    w = BF16_CASES["wide_split"]
+    inp = synth.make_inputs(w)
+    mf = native.MixFlow.for_workload(w)
+    loop = native.loop_desc_for(w)
+    d = native.to_device_inputs(w, inp)
+    d_eta = torch.empty(w.n_eta, device="cuda")
+    d_th = torch.empty(w.n_params, device="cuda")
+    outs = []
+    for call in range(4):
+        if call == 3:   # new inputs behind the same pointers
+            d["eta"].mul_(-0.5)
+        mf.meta_grad(loop, d["theta0"], d["eta"], d["inner_x"], d["inner_y"], d["outer_x"],
+                     d["outer_y"], d_eta, d_th)
+        mf.sync()
+        outs.append((d_eta.cpu().numpy().copy(), d_th.cpu().numpy().copy()))
+    for k in (1, 2):
+        assert np.array_equal(outs[0][0], outs[k][0]) and np.array_equal(outs[0][1], outs[k][1])
+    eta2 = (inp.eta.astype(np.float64) * -0.5).astype(np.float32)
+    ref = om.meta_grad(w, synth.Inputs(inp.theta0, eta2, inp.inner_x, inp.inner_y, inp.outer_x,
+                                       inp.outer_y))
+    assert rel_l2(outs[3][0], ref["d_eta"]) < 2e-2
+    # graphs off: same numbers as the eager first call
+    mf.set_option(native.MF_OPT_CUDA_GRAPHS, 0)
+    d["eta"].mul_(-2.0)
+    mf.meta_grad(loop, d["theta0"], d["eta"], d["inner_x"], d["inner_y"], d["outer_x"],
+                 d["outer_y"], d_eta, d_th)
+    mf.sync()
+    assert np.array_equal(d_eta.cpu().numpy(), outs[0][0])
+    mf.close()
