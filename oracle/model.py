@@ -4,7 +4,8 @@ Test infrastructure only (see ``oracle/__init__.py``).
 
 The paper leaves the inner model abstract (L(theta, eta, x) in Eq. 1); the workloads fix it
 as a multilayer perceptron with a flat parameter vector laid out per layer as W_l
-[d_l, d_{l+1}] row-major followed by b_l [d_{l+1}].  Per-example losses:
+[d_l, d_{l+1}] row-major followed by b_l [d_{l+1}].  The decoder-only transformer of the language-modelling tasks (Section 5: Chinchilla-style
+models with RoPE) is written out in ``decoder_logits``.  Per-example losses:
 
 * squared:  l_b = 1/2 * mean_o (f_bo - y_bo)^2
 * ce:       l_b = logsumexp(f_b) - f_{b, y_b}     (natural log)
@@ -68,7 +69,69 @@ def per_example_loss(w, f: torch.Tensor, y: torch.Tensor) -> torch.Tensor:
     raise ValueError(w.loss)
 
 
+def decoder_unpack(w, theta):
+    """Named views into the flat decoder parameter vector (``Workload.decoder_layout``)."""
+    out, o = {}, 0
+    for name, n in w.decoder_layout():
+        out[name] = theta[o:o + n]
+        o += n
+    return out
+
+
+def rmsnorm(x, g, eps):
+    """y = g * x / sqrt(mean(x^2) + eps) over the last axis (pre-norm of the decoder blocks)."""
+    return g * x * torch.rsqrt((x * x).mean(dim=-1, keepdim=True) + eps)
+
+
+def rope(x, base):
+    """Rotary position embedding, rotate-half form, over the last axis of [B, H, S, dh]:
+    out = x cos(p w) + rot(x) sin(p w), rot(x) = [-x2, x1], w_j = base^(-2 (j mod dh/2) / dh)."""
+    S, dh = x.shape[-2], x.shape[-1]
+    half = dh // 2
+    j = torch.arange(half, dtype=F64)
+    inv = base ** (-2.0 * j / dh)
+    ang = torch.arange(S, dtype=F64)[:, None] * inv[None, :]       # [S, half]
+    cos = torch.cat([torch.cos(ang), torch.cos(ang)], dim=-1)
+    sin = torch.cat([torch.sin(ang), torch.sin(ang)], dim=-1)
+    rot = torch.cat([-x[..., half:], x[..., :half]], dim=-1)
+    return x * cos + rot * sin
+
+
+def decoder_logits(w, theta, ids):
+    """Decoder-only transformer: token embedding, n_blocks pre-RMSNorm blocks (causal
+    multi-head attention with RoPE, GELU MLP, residual connections), final RMSNorm, untied
+    head.  ids [B, S+1]; returns logits [B, S, V] for positions 0..S-1."""
+    P = decoder_unpack(w, theta)
+    d, H, F, V = w.d_model, w.n_heads, w.d_ff, w.vocab
+    dh = d // H
+    B, S = ids.shape[0], ids.shape[1] - 1
+    x = P["E"].reshape(V, d)[ids[:, :S]]                            # [B, S, d]
+    mask = torch.triu(torch.ones(S, S, dtype=torch.bool), diagonal=1)
+    for l in range(w.n_blocks):
+        h = rmsnorm(x, P[f"g1.{l}"], w.rms_eps)
+        qkv = h @ P[f"Wqkv.{l}"].reshape(d, 3 * d)
+        q, k, v = (t.reshape(B, S, H, dh).transpose(1, 2) for t in qkv.split(d, dim=-1))
+        q, k = rope(q, w.rope_base), rope(k, w.rope_base)
+        s = (q @ k.transpose(-1, -2)) / math.sqrt(dh)
+        s = s.masked_fill(mask, float("-inf"))
+        o = torch.softmax(s, dim=-1) @ v                             # [B, H, S, dh]
+        x = x + o.transpose(1, 2).reshape(B, S, d) @ P[f"Wo.{l}"].reshape(d, d)
+        h2 = rmsnorm(x, P[f"g2.{l}"], w.rms_eps)
+        x = x + act("gelu", h2 @ P[f"W1.{l}"].reshape(d, F)) @ P[f"W2.{l}"].reshape(F, d)
+    return rmsnorm(x, P["gf"], w.rms_eps) @ P["Wh"].reshape(d, V)
+
+
+def decoder_losses(w, theta, ids):
+    """Per-sequence next-token cross-entropy, mean over the S predicted positions."""
+    f = decoder_logits(w, theta, ids)
+    tgt = ids[:, 1:].long()
+    ce = torch.logsumexp(f, dim=-1) - f.gather(-1, tgt[..., None])[..., 0]
+    return ce.mean(dim=1)
+
+
 def losses(w, theta, x, y):
+    if getattr(w, "arch", "mlp") == "decoder":
+        return decoder_losses(w, theta, x.long())
     return per_example_loss(w, mlp_forward(w, theta, x), y)
 
 

@@ -19,6 +19,12 @@ as in the loss-weighting and learned-learning-rate tasks of Section 5):
   alpha=0.05, per-example weight logits, outer batch 1024, bf16 GEMMs.
 * ``deep``  - 8 Linear 4096->4096 layers (SiLU after the first 7), regression onto a random
   teacher, per-parameter log learning rates, SGD with momentum 0.9, B=512, T=32, bf16 GEMMs.
+* ``decoder_small`` - decoder-only transformer, 6 layers, d_model 512, 8 heads, MLP 2048
+  GELU, pre-RMSNorm, RoPE, causal attention, vocabulary 8192, sequences of 256 tokens with
+  ids drawn from a Zipf(1.1) law truncated to the vocabulary, batch 16, T=8 SGD steps,
+  alpha=1e-3, per-sequence weight logits, next-token cross-entropy.
+* ``decoder_large`` - 12 layers, d_model 1024, 16 heads, MLP 4096, sequences of 1024, batch 8,
+  vocabulary 32768, T=16 heavy-ball (0.9) steps, per-sequence weights plus a scalar log-lr.
 """
 from __future__ import annotations
 
@@ -55,7 +61,7 @@ SCALAR_LOGLR = 4
 @dataclass
 class Workload:
     name: str
-    dims: list                      # MLP layer widths [d_in, h1, ..., d_out]
+    dims: list                      # MLP layer widths [d_in, h1, ..., d_out] (MLP only)
     act: str                        # hidden activation: ident|tanh|gelu|silu
     loss: str                       # squared | ce
     precision: str                  # fp32 | bf16
@@ -72,6 +78,18 @@ class Workload:
     seed: int = 0
     has_bias: bool = True
     extra: dict = field(default_factory=dict)
+    # decoder-only transformer (arch == "decoder"); dims/act/has_bias unused there
+    arch: str = "mlp"
+    d_model: int = 0
+    n_heads: int = 0
+    d_ff: int = 0
+    vocab: int = 0
+    seq: int = 0
+    n_blocks: int = 0
+    zipf_s: float = 1.1
+    init_std: float = 0.02
+    rope_base: float = 10000.0
+    rms_eps: float = 1e-6
 
     @property
     def n_layers(self) -> int:
@@ -79,8 +97,22 @@ class Workload:
 
     @property
     def n_params(self) -> int:
+        if self.arch == "decoder":
+            return sum(n for _, n in self.decoder_layout())
         return sum(self.dims[i] * self.dims[i + 1] + (self.dims[i + 1] if self.has_bias else 0)
                    for i in range(self.n_layers))
+
+    def decoder_layout(self):
+        """(name, size) of each decoder tensor in flat-parameter order: embedding E [V][d];
+        per block g1 [d], Wqkv [d][3d], Wo [d][d], g2 [d], W1 [d][dff], W2 [dff][d]; final gain
+        gf [d]; head Wh [d][V]."""
+        d, V, F = self.d_model, self.vocab, self.d_ff
+        out = [("E", V * d)]
+        for l in range(self.n_blocks):
+            out += [(f"g1.{l}", d), (f"Wqkv.{l}", d * 3 * d), (f"Wo.{l}", d * d),
+                    (f"g2.{l}", d), (f"W1.{l}", d * F), (f"W2.{l}", F * d)]
+        out += [("gf", d), ("Wh", d * V)]
+        return out
 
     @property
     def n_eta(self) -> int:
@@ -113,6 +145,14 @@ class Workload:
         return replace(copy.deepcopy(self), **kw)
 
 
+def decoder(name, d, H, F, L, V, S, B, T, B_outer, alpha=0.0, momentum=0.0,
+            meta_kind=EXAMPLE_WEIGHTS, **kw):
+    return Workload(name, [], "gelu", "next_token_ce", "bf16", B=B, T=T, B_outer=B_outer,
+                    alpha=alpha, momentum=momentum, meta_kind=meta_kind, has_bias=False,
+                    arch="decoder", d_model=d, n_heads=H, d_ff=F, vocab=V, seq=S, n_blocks=L,
+                    **kw)
+
+
 WORKLOADS = {
     "tiny": Workload("tiny", [16, 32, 1], "tanh", "squared", "fp32", B=8, T=4, B_outer=8,
                      alpha=0.1, noise_std=0.1),
@@ -121,6 +161,11 @@ WORKLOADS = {
     "deep": Workload("deep", [4096] * 9, "silu", "squared", "bf16", B=512, T=32,
                      B_outer=512, momentum=0.9, meta_kind=PARAM_LOGLR,
                      loglr_mean=math.log(1e-2), loglr_std=0.1),
+    "decoder_small": decoder("decoder_small", 512, 8, 2048, 6, 8192, 256, B=16, T=8, B_outer=16,
+                             alpha=1e-3),
+    "decoder_large": decoder("decoder_large", 1024, 16, 4096, 12, 32768, 1024, B=8, T=16,
+                             B_outer=8, momentum=0.9, meta_kind=EXAMPLE_WEIGHTS | SCALAR_LOGLR,
+                             extra={"scalar_loglr": math.log(1e-3)}),
 }
 
 
@@ -166,8 +211,42 @@ class Inputs:
     outer_y: np.ndarray     # [B_outer] int32 or [B_outer, d_out] float32
 
 
+def zipf_ids(g: np.random.Generator, shape, V: int, s: float) -> np.ndarray:
+    """Token ids from p(k) ~ k^-s on k = 1..V (truncated Zipf), id = k - 1, by inverse CDF."""
+    p = np.arange(1, V + 1, dtype=np.float64) ** (-s)
+    cdf = np.cumsum(p / p.sum())
+    u = g.random(size=shape)
+    return np.minimum(np.searchsorted(cdf, u, side="right"), V - 1).astype(np.int32)
+
+
+def decoder_params(w: Workload, g: np.random.Generator) -> np.ndarray:
+    """N(0, init_std) matrices, unit RMSNorm gains, in the layout of ``decoder_layout``."""
+    parts = []
+    for name, n in w.decoder_layout():
+        if name.startswith("g"):
+            parts.append(np.ones(n))
+        else:
+            parts.append(w.init_std * g.standard_normal(n))
+    return np.concatenate(parts).astype(np.float32)
+
+
 def make_inputs(w: Workload) -> Inputs:
     """Draw every input of one meta-gradient call for workload ``w``."""
+    if w.arch == "decoder":
+        ids = zipf_ids(rng(w.seed, "tokens"), (w.T, w.B, w.seq + 1), w.vocab, w.zipf_s)
+        oids = zipf_ids(rng(w.seed, "outer"), (w.B_outer, w.seq + 1), w.vocab, w.zipf_s)
+        theta0 = decoder_params(w, rng(w.seed, "theta0"))
+        ge = rng(w.seed, "eta")
+        parts = []
+        if w.meta_kind & EXAMPLE_WEIGHTS:
+            parts.append(w.eta_std * ge.standard_normal(w.T * w.B))
+        if w.meta_kind & PARAM_LOGLR:
+            parts.append(w.loglr_mean + w.loglr_std * ge.standard_normal(w.n_params))
+        if w.meta_kind & SCALAR_LOGLR:
+            parts.append(np.array([w.extra.get("scalar_loglr", math.log(1e-3))]))
+        eta = np.concatenate(parts).astype(np.float32)
+        # token ids double as inputs (positions 0..S-1) and targets (positions 1..S)
+        return Inputs(theta0, eta, ids, ids, oids, oids)
     din, dout = w.dims[0], w.dims[-1]
     rd = round_bf16 if w.precision == "bf16" else (lambda a: np.asarray(a, np.float32))
     x = rd(rng(w.seed, "x").standard_normal((w.T, w.B, din)))

@@ -218,3 +218,66 @@ def test_tangent_losses_fd():
         fd = (om.per_example_losses(w, theta + h * v, x, y)
               - om.per_example_losses(w, theta - h * v, x, y)) / (2 * h)
         assert _rel(ld, fd) < 1e-7
+
+
+# ---- decoder-only transformer -------------------------------------------------------------
+DEC = {
+    "dec_ex": synth.decoder("dec_ex", 16, 2, 32, 2, 32, 8, B=3, T=2, B_outer=2, alpha=0.1),
+    "dec_mom_slr": synth.decoder("dec_mom_slr", 16, 4, 24, 1, 24, 6, B=2, T=3, B_outer=2,
+                                 momentum=0.9, meta_kind=EX | SLR,
+                                 extra={"scalar_loglr": math.log(0.2)}),
+}
+
+
+@pytest.mark.parametrize("name", list(DEC))
+def test_p1_decoder_finite_differences(name):
+    w = DEC[name]
+    inp = synth.make_inputs(w)
+    res = om.meta_grad(w, inp)
+    idx = list(range(w.n_eta))
+    fd = _fd_eta(w, inp, idx)
+    assert _rel(res["d_eta"], fd) < 1e-6, (res["d_eta"], fd)
+    assert np.abs(res["d_eta"]).max() > 1e-7
+
+
+def test_decoder_model_properties():
+    """Semantics of the oracle's decoder: RoPE keeps norms and makes q.k depend on the
+    position difference only; attention is causal; RMSNorm is scale invariant."""
+    import torch
+    from oracle import model
+    g = torch.Generator().manual_seed(0)
+    q = torch.randn(1, 1, 1, 8, generator=g, dtype=torch.float64)
+    k = torch.randn(1, 1, 1, 8, generator=g, dtype=torch.float64)
+    S = 12
+    qs = model.rope(q.expand(1, 1, S, 8).clone(), 10000.0)[0, 0]
+    ks = model.rope(k.expand(1, 1, S, 8).clone(), 10000.0)[0, 0]
+    assert torch.allclose(qs.norm(dim=-1), q.norm().expand(S), rtol=1e-12)
+    dots = qs @ ks.T
+    for shift in range(S):
+        diag = torch.diagonal(dots, offset=shift)
+        assert torch.allclose(diag, diag[0].expand_as(diag), rtol=1e-10, atol=1e-12)
+    x = torch.randn(4, 8, generator=g, dtype=torch.float64)
+    gain = torch.rand(8, generator=g, dtype=torch.float64) + 0.5
+    assert torch.allclose(model.rmsnorm(3.7 * x, gain, 0.0), model.rmsnorm(x, gain, 0.0))
+    w = DEC["dec_ex"]
+    inp = synth.make_inputs(w)
+    theta = torch.from_numpy(inp.theta0.astype(np.float64))
+    ids = torch.from_numpy(inp.inner_x[0].astype(np.int64))
+    ids2 = ids.clone()
+    ids2[:, 5:] = (ids2[:, 5:] + 7) % w.vocab           # change the future only
+    f1 = model.decoder_logits(w, theta, ids)
+    f2 = model.decoder_logits(w, theta, ids2)
+    assert torch.equal(f1[:, :5], f2[:, :5])
+    assert not torch.allclose(f1[:, 5:], f2[:, 5:])
+
+
+def test_zipf_ids_law():
+    """Token ids follow the truncated Zipf(1.1) law (inverse-CDF sampling)."""
+    g = np.random.default_rng(3)
+    V = 50
+    ids = synth.zipf_ids(g, (200000,), V, 1.1)
+    assert ids.min() >= 0 and ids.max() < V
+    p = np.arange(1, V + 1, dtype=np.float64) ** -1.1
+    p /= p.sum()
+    emp = np.bincount(ids, minlength=V) / ids.size
+    assert np.abs(emp - p).max() < 4e-3
