@@ -22,8 +22,16 @@
  *     d eta_{t,b} = sigmoid'(eta_{t,b}) / B * (grad l_b(theta_t) . u_t)
  *     d eta_lr   += -lr (*) m_{t+1} (*) theta_bar_{t+1}
  *
- * Inner models: multilayer perceptrons (MF_ARCH_MLP).  Parameters are one flat float32
- * vector: for each layer l, W_l as [d_l][d_{l+1}] row-major, then b_l [d_{l+1}].
+ * Inner models:
+ *  - MF_ARCH_MLP: multilayer perceptrons.  Parameters are one flat float32 vector: for each
+ *    layer l, W_l as [d_l][d_{l+1}] row-major, then b_l [d_{l+1}].
+ *  - MF_ARCH_DECODER: decoder-only transformer (the language models of Section 5): token
+ *    embedding, n_layers blocks of pre-RMSNorm causal multi-head attention with RoPE
+ *    (rotate-half, angle s * rope_base^(-2j/dh)) and pre-RMSNorm GELU MLP with residual
+ *    connections, final RMSNorm, untied head; per-sequence next-token cross-entropy (mean
+ *    over the seq_len predicted positions).  No biases.  Flat parameter order: E [vocab][d];
+ *    per block g1 [d], Wqkv [d][3d] (q | k | v columns, heads contiguous), Wo [d][d],
+ *    g2 [d], W1 [d][d_ff], W2 [d_ff][d]; then gf [d], Wh [d][vocab].
  *
  * Conventions for every call:
  *  - Tensor arguments are device pointers owned by the caller (e.g. torch CUDA tensors),
@@ -76,11 +84,15 @@ enum { MF_HVP_MIXED_FOR = 0, MF_HVP_REV_REV = 1 };
  *  act        activation after every layer but the last (MF_ACT_*).
  *  has_bias   1 = every layer has a bias vector.
  *  loss       MF_LOSS_SQUARED: l_b = 1/2 mean_o (f_bo - y_bo)^2, y float32 [rows][d_out];
- *             MF_LOSS_SOFTMAX_CE: l_b = logsumexp(f_b) - f_{b,y_b}, y int32 [rows].
+ *             MF_LOSS_SOFTMAX_CE: l_b = logsumexp(f_b) - f_{b,y_b}, y int32 [rows];
+ *             MF_LOSS_NEXT_TOKEN_CE (decoder only): x = y = int32 token ids [rows][seq_len+1],
+ *             inputs ids[:, 0:S], targets ids[:, 1:S+1].
  *  precision  MF_PREC_FP32: float32 inputs, float32 GEMMs (SIMT);
  *             MF_PREC_BF16: bf16 inputs, bf16 tensor-core GEMMs with float32 accumulation;
  *             parameters, optimiser state, adjoints and meta-gradients stay float32.
- *  The remaining fields are reserved for MF_ARCH_DECODER and must be 0 for MLPs. */
+ *  Decoder fields (MF_ARCH_DECODER; n_layers = blocks): d_model, n_heads (d_model/n_heads a
+ *  multiple of 8), d_ff, vocab, seq_len (multiples of 8), rope_base (0 = 10000),
+ *  rms_eps (0 = 1e-6).  dims/act/has_bias are ignored for decoders. */
 typedef struct {
   int arch;
   int n_layers;
@@ -111,8 +123,7 @@ typedef struct {
 } mf_loop_desc;
 
 /* Create a handle for one inner-model architecture.  *out receives a library-owned handle.
- * Errors: MF_ERR_INVALID_ARG (bad descriptor), MF_ERR_UNSUPPORTED (decoder arch),
- * MF_ERR_CUDA (no usable device). */
+ * Errors: MF_ERR_INVALID_ARG (bad descriptor), MF_ERR_CUDA (no usable device). */
 mf_status mf_create(const mf_model_desc* desc, mf_handle* out);
 
 /* Release the handle and its workspace (synchronises the device first). */

@@ -14,6 +14,7 @@
 #include <vector>
 
 #include "../../include/mixflow.h"
+#include "decoder_layout.h"
 #include "internal.h"
 
 using mf::GemmArgs;
@@ -28,6 +29,8 @@ inline int ld8(int x) { return (x + 7) / 8 * 8; }
 
 struct mf_ctx {
   mf_model_desc md;
+  bool decoder = false;
+  DecLayout Ly;
   int L = 0;
   std::vector<int> dims;
   std::vector<int64_t> woff, boff;
@@ -283,6 +286,8 @@ mf_status run_graphed(mf_ctx* h, mf_ctx::GraphCache& g, uint64_t key, cudaStream
   return graph_launch(h, g, user);
 }
 
+size_t y_stride_bytes(const mf_ctx* h, int rows);
+
 // ---- the MLP executor --------------------------------------------------------------------
 template <typename T>
 struct Exec {
@@ -318,6 +323,17 @@ struct Exec {
   template <typename U> U* at(size_t off) const { return reinterpret_cast<U*>(base + off); }
   float* theta_slot(int t) const { return at<float>(p.o_theta) + static_cast<int64_t>(t) * h->P; }
   float* m_slot(int j) const { return at<float>(p.o_m) + static_cast<int64_t>(j) * h->P; }
+  float* g_buf() const { return at<float>(p.o_g); }
+  float* tbar_buf() const { return at<float>(p.o_tbar); }
+  float* u_buf() const { return at<float>(p.o_u); }
+  float* part_buf() const { return at<float>(p.o_part); }
+  float* l_buf() const { return at<float>(p.o_l); }
+  float* ld_buf() const { return at<float>(p.o_ld); }
+  int nb() const { return p.nb; }
+  size_t x_step_bytes(int rows) const {
+    return static_cast<size_t>(rows) * h->dims[0] * (h->bf16 ? 2 : 4);
+  }
+  size_t y_step_bytes(int rows) const { return y_stride_bytes(h, rows); }
 
   void launched(int n = 1) { h->launches += n; }
 
@@ -381,7 +397,8 @@ struct Exec {
 
   // Forward pass of `rows` examples: primal (z) or dual (z, z_dot along u).  Hidden layers
   // fuse bias, activation and its tangent into the GEMM epilogue.
-  void forward(int rows, const T* x, const float* theta, const float* u, bool dual) {
+  void forward(int rows, const void* xv, const float* theta, const float* u, bool dual) {
+    const T* x = static_cast<const T*>(xv);
     const int din0 = h->dims[0];
     mf::transpose<T>(x, rows, din0, din0, at<T>(p.o_AT[0]), p.ldR, s);
     launched();
@@ -494,6 +511,8 @@ struct Exec {
   }
 };
 
+#include "decoder_exec.cuh"
+
 mf_status validate_loop(mf_ctx* h, const mf_loop_desc* lp) {
   if (!lp) return fail(h, MF_ERR_INVALID_ARG, "loop descriptor is NULL");
   if (lp->T < 1 || lp->B < 1 || lp->B_outer < 1)
@@ -519,7 +538,7 @@ int64_t n_eta_of(const mf_ctx* h, const mf_loop_desc* lp) {
 }
 
 mf_status check_x(mf_ctx* h, const void* x, int rows) {
-  if (!h->bf16) return MF_OK;
+  if (!h->bf16 || h->decoder) return MF_OK;
   const int din = h->dims[0];
   if ((reinterpret_cast<uintptr_t>(x) & 15) || (din % 8) != 0 ||
       ((static_cast<int64_t>(rows) * din * 2) % 16) != 0)
@@ -560,27 +579,28 @@ LrSel lr_select(const mf_ctx* h, const mf_loop_desc* lp, const float* eta) {
 
 // Inner rollout (Eq. 2).  With store_all, theta slot t holds theta_t and m slot j holds
 // m_{j+1} when the learning rate is a meta-parameter; otherwise two theta slots ping-pong.
-// Each step's update (K4) also casts theta_{t+1} into the GEMM operand copies.
-template <typename E>
-void rollout(Exec<E>& ex, const mf_loop_desc* lp, const float* eta, const void* inner_x,
+// Each step's update (K4) also casts theta_{t+1} into the GEMM operand copies.  X is the
+// model executor (MLP or decoder).
+template <typename X>
+void rollout(X& ex, const mf_loop_desc* lp, const float* eta, const void* inner_x,
              const void* inner_y, const LrSel& lr, bool store_all, float** theta_T) {
   mf_ctx* h = ex.h;
-  const int B = lp->B, din = h->dims[0];
-  const size_t xs = static_cast<size_t>(B) * din * (h->bf16 ? 2 : 4);
-  const size_t ys = y_stride_bytes(h, B);
-  float* m_run = (lp->momentum != 0.f && !lr.lr_meta) ? ex.template at<float>(ex.p.o_u) : nullptr;
+  const int B = lp->B;
+  const size_t xs = ex.x_step_bytes(B);
+  const size_t ys = ex.y_step_bytes(B);
+  float* m_run = (lp->momentum != 0.f && !lr.lr_meta) ? ex.u_buf() : nullptr;
   if (m_run) { mf::fill(m_run, h->P, 0.f, ex.s); ex.launched(); }
   const float* m_prev = nullptr;
   ex.cast_params(ex.theta_slot(0), false);
   for (int t = 0; t < lp->T; ++t) {
     float* th = ex.theta_slot(store_all ? t : (t & 1));
     float* th_next = ex.theta_slot(store_all ? t + 1 : ((t + 1) & 1));
-    const E* x = reinterpret_cast<const E*>(static_cast<const char*>(inner_x) + xs * t);
+    const void* x = static_cast<const char*>(inner_x) + xs * t;
     const void* y = static_cast<const char*>(inner_y) + ys * t;
     ex.forward(B, x, th, nullptr, false);
     const float* ew = (lp->meta_kind & MF_META_EXAMPLE_WEIGHTS) ? eta + static_cast<int64_t>(t) * B : nullptr;
     ex.loss(B, false, y, ew, nullptr, nullptr, nullptr, nullptr);
-    float* g = ex.template at<float>(ex.p.o_g);
+    float* g = ex.g_buf();
     ex.backward(B, false, nullptr, g);
     float* m_out = nullptr;
     if (lr.lr_meta && store_all) m_out = ex.m_slot(t);
@@ -603,18 +623,17 @@ void rollout(Exec<E>& ex, const mf_loop_desc* lp, const float* eta, const void* 
   *theta_T = ex.theta_slot(store_all ? lp->T : (lp->T & 1));
 }
 
-template <typename E>
-mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
-                         const float* eta, const void* inner_x, const void* inner_y,
-                         const void* outer_x, const void* outer_y, float* d_eta,
-                         float* d_theta0, float* outer_loss, cudaStream_t s) {
+// Algorithm 2 once the workspace is in place: rollout, outer gradient (Eq. 4), then the
+// reverse sweep t = T-1..0 with forward-over-reverse Hessian-vector products.
+template <typename X>
+mf_status meta_grad_run(X& ex, const mf_loop_desc* lp, const float* theta0, const float* eta,
+                        const void* inner_x, const void* inner_y, const void* outer_x,
+                        const void* outer_y, float* d_eta, float* d_theta0, float* outer_loss) {
+  mf_ctx* h = ex.h;
+  cudaStream_t s = ex.s;
   const int T = lp->T, B = lp->B, Bo = lp->B_outer;
   const LrSel lr = lr_select(h, lp, eta);
   const bool scalar_lr = lp->meta_kind & MF_META_SCALAR_LOGLR;
-  Plan plan = make_plan(h, std::max(B, Bo), T, T + 1, lr.lr_meta ? T : 0, scalar_lr);
-  mf_status st = ensure_ws(h, plan.bytes, s);
-  if (st != MF_OK) return st;
-  Exec<E> ex(h, plan, s);
   MF_CUDA(h, cudaMemcpyAsync(ex.theta_slot(0), theta0, h->P * 4, cudaMemcpyDeviceToDevice, s));
   const int64_t ne = n_eta_of(h, lp);
   if (ne > 0) MF_CUDA(h, cudaMemsetAsync(d_eta, 0, ne * 4, s));
@@ -622,19 +641,20 @@ mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
 
   // 1. rollout with the theta_t store
   float* thT = nullptr;
-  rollout<E>(ex, lp, eta, inner_x, inner_y, lr, true, &thT);
+  rollout(ex, lp, eta, inner_x, inner_y, lr, true, &thT);
   if (ex.st != MF_OK) return ex.st;
 
   // 2. outer gradient theta_bar_T = grad V(theta_T)  (Eq. 4); theta_T is already cast
-  float* tbar = ex.template at<float>(plan.o_tbar);
-  float* u = ex.template at<float>(plan.o_u);
-  float* Hu = ex.template at<float>(plan.o_g);
-  float* part = ex.template at<float>(plan.o_part);
-  ex.forward(Bo, static_cast<const E*>(outer_x), thT, nullptr, false);
-  ex.loss(Bo, false, outer_y, nullptr, nullptr, ex.template at<float>(plan.o_l), nullptr, nullptr);
+  float* tbar = ex.tbar_buf();
+  float* u = ex.u_buf();
+  float* Hu = ex.g_buf();
+  float* part = ex.part_buf();
+  const int nb = ex.nb();
+  ex.forward(Bo, outer_x, thT, nullptr, false);
+  ex.loss(Bo, false, outer_y, nullptr, nullptr, ex.l_buf(), nullptr, nullptr);
   ex.backward(Bo, false, nullptr, tbar);
   if (outer_loss) {
-    mf::sum_scaled(ex.template at<float>(plan.o_l), Bo, 1.f / Bo, outer_loss, s);
+    mf::sum_scaled(ex.l_buf(), Bo, 1.f / Bo, outer_loss, s);
     ex.launched();
   }
   float* d_plr = lr.off_plr >= 0 ? d_eta + lr.off_plr : nullptr;
@@ -646,7 +666,7 @@ mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
     a.m_adj = lr.lr_meta ? ex.m_slot(T - 1) : nullptr;
     a.u_out = u;
     a.d_plr = d_plr;
-    a.partials = scalar_lr ? part + static_cast<int64_t>(T - 1) * plan.nb : nullptr;
+    a.partials = scalar_lr ? part + static_cast<int64_t>(T - 1) * nb : nullptr;
     a.cast_src = ex.theta_slot(T - 1);
     a.mu = lp->momentum;
     a.lr = lr.lr;
@@ -654,19 +674,18 @@ mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
     ex.update(a);
   }
 
-  // 3. reverse sweep t = T-1..0 with forward-over-reverse Hessian-vector products
-  const int din = h->dims[0];
-  const size_t xs = static_cast<size_t>(B) * din * (h->bf16 ? 2 : 4);
-  const size_t ys = y_stride_bytes(h, B);
+  // 3. reverse sweep
+  const size_t xs = ex.x_step_bytes(B);
+  const size_t ys = ex.y_step_bytes(B);
   const bool exw = lp->meta_kind & MF_META_EXAMPLE_WEIGHTS;
   for (int t = T - 1; t >= 0; --t) {
     const float* th = ex.theta_slot(t);
-    const E* x = reinterpret_cast<const E*>(static_cast<const char*>(inner_x) + xs * t);
+    const void* x = static_cast<const char*>(inner_x) + xs * t;
     const void* y = static_cast<const char*>(inner_y) + ys * t;
     ex.forward(B, x, th, u, true);
     const float* ew = exw ? eta + static_cast<int64_t>(t) * B : nullptr;
     float* de = exw ? d_eta + static_cast<int64_t>(t) * B : nullptr;
-    ex.loss(B, true, y, ew, nullptr, nullptr, ex.template at<float>(plan.o_ld), de);
+    ex.loss(B, true, y, ew, nullptr, nullptr, ex.ld_buf(), de);
     ex.backward(B, true, Hu, nullptr);
     // theta_bar_t = theta_bar_{t+1} + H u ; d eta_lr += -lr m_t theta_bar_t ;
     // u_{t-1} = mu u_t - lr theta_bar_t ; cast theta_{t-1}, u_{t-1}
@@ -679,7 +698,7 @@ mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
       a.u_in = u;
       a.u_out = u;
       a.d_plr = d_plr;
-      a.partials = scalar_lr ? part + static_cast<int64_t>(t - 1) * plan.nb : nullptr;
+      a.partials = scalar_lr ? part + static_cast<int64_t>(t - 1) * nb : nullptr;
       a.cast_src = ex.theta_slot(t - 1);
     }
     a.mu = lp->momentum;
@@ -689,7 +708,7 @@ mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
     if (ex.st != MF_OK) return ex.st;
   }
   if (scalar_lr) {
-    mf::sum_scaled(part, T * plan.nb, 1.f, d_eta + lr.off_slr, s);
+    mf::sum_scaled(part, T * nb, 1.f, d_eta + lr.off_slr, s);
     ex.launched();
   }
   if (d_theta0) MF_CUDA(h, cudaMemcpyAsync(d_theta0, tbar, h->P * 4, cudaMemcpyDeviceToDevice, s));
@@ -697,39 +716,81 @@ mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
   return ex.st;
 }
 
-template <typename E>
-mf_status rollout_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0, const float* eta,
-                       const void* inner_x, const void* inner_y, float* thetaT, cudaStream_t s) {
+template <typename X>
+mf_status rollout_run(X& ex, const mf_loop_desc* lp, const float* theta0, const float* eta,
+                      const void* inner_x, const void* inner_y, float* thetaT) {
+  mf_ctx* h = ex.h;
   const LrSel lr = lr_select(h, lp, eta);
-  Plan plan = make_plan(h, lp->B, lp->T, 2, lr.lr_meta ? 1 : 0, false);
+  MF_CUDA(h, cudaMemcpyAsync(ex.theta_slot(0), theta0, h->P * 4, cudaMemcpyDeviceToDevice, ex.s));
+  ex.prepare();
+  float* thT = nullptr;
+  rollout(ex, lp, eta, inner_x, inner_y, lr, false, &thT);
+  if (ex.st != MF_OK) return ex.st;
+  MF_CUDA(h, cudaMemcpyAsync(thetaT, thT, h->P * 4, cudaMemcpyDeviceToDevice, ex.s));
+  return MF_OK;
+}
+
+template <typename X>
+mf_status hvp_run(X& ex, int B, const float* theta, const void* x, const void* y,
+                  const float* ex_w, const float* v, float* Hv, float* tl, float* grad) {
+  mf_ctx* h = ex.h;
+  ex.prepare();
+  ex.cast_params(theta, false);
+  ex.cast_params(v, true);
+  ex.forward(B, x, theta, v, true);
+  ex.loss(B, true, y, nullptr, ex_w, nullptr, tl, nullptr);
+  ex.backward(B, true, Hv, grad);
+  MF_CUDA(h, cudaGetLastError());
+  return ex.st;
+}
+
+// Plan the workspace for the handle's model, allocate it, and run f(executor).
+template <typename E, typename F>
+mf_status with_exec(mf_ctx* h, int rows, int T, int theta_slots, int m_slots, bool partials,
+                    cudaStream_t s, F&& f) {
+  if (h->decoder) {
+    DecPlan plan = make_dec_plan(h, h->Ly, rows, T, theta_slots, m_slots, partials);
+    mf_status st = ensure_ws(h, plan.bytes, s);
+    if (st != MF_OK) return st;
+    DecExec<E> ex(h, plan, h->Ly, s);
+    return f(ex);
+  }
+  Plan plan = make_plan(h, rows, T, theta_slots, m_slots, partials);
   mf_status st = ensure_ws(h, plan.bytes, s);
   if (st != MF_OK) return st;
   Exec<E> ex(h, plan, s);
-  MF_CUDA(h, cudaMemcpyAsync(ex.theta_slot(0), theta0, h->P * 4, cudaMemcpyDeviceToDevice, s));
-  ex.prepare();
-  float* thT = nullptr;
-  rollout<E>(ex, lp, eta, inner_x, inner_y, lr, false, &thT);
-  if (ex.st != MF_OK) return ex.st;
-  MF_CUDA(h, cudaMemcpyAsync(thetaT, thT, h->P * 4, cudaMemcpyDeviceToDevice, s));
-  return MF_OK;
+  return f(ex);
+}
+
+template <typename E>
+mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
+                         const float* eta, const void* inner_x, const void* inner_y,
+                         const void* outer_x, const void* outer_y, float* d_eta,
+                         float* d_theta0, float* outer_loss, cudaStream_t s) {
+  const bool lr_meta = lp->meta_kind & (MF_META_PARAM_LOGLR | MF_META_SCALAR_LOGLR);
+  return with_exec<E>(h, std::max(lp->B, lp->B_outer), lp->T, lp->T + 1, lr_meta ? lp->T : 0,
+                      lp->meta_kind & MF_META_SCALAR_LOGLR, s, [&](auto& ex) {
+                        return meta_grad_run(ex, lp, theta0, eta, inner_x, inner_y, outer_x,
+                                             outer_y, d_eta, d_theta0, outer_loss);
+                      });
+}
+
+template <typename E>
+mf_status rollout_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0, const float* eta,
+                       const void* inner_x, const void* inner_y, float* thetaT, cudaStream_t s) {
+  const bool lr_meta = lp->meta_kind & (MF_META_PARAM_LOGLR | MF_META_SCALAR_LOGLR);
+  return with_exec<E>(h, lp->B, lp->T, 2, lr_meta ? 1 : 0, false, s, [&](auto& ex) {
+    return rollout_run(ex, lp, theta0, eta, inner_x, inner_y, thetaT);
+  });
 }
 
 template <typename E>
 mf_status hvp_impl(mf_ctx* h, int B, const float* theta, const void* x, const void* y,
                    const float* ex_w, const float* v, float* Hv, float* tl, float* grad,
                    cudaStream_t s) {
-  Plan plan = make_plan(h, B, 1, 0, 0, false);
-  mf_status st = ensure_ws(h, plan.bytes, s);
-  if (st != MF_OK) return st;
-  Exec<E> ex(h, plan, s);
-  ex.prepare();
-  ex.cast_params(theta, false);
-  ex.cast_params(v, true);
-  ex.forward(B, static_cast<const E*>(x), theta, v, true);
-  ex.loss(B, true, y, nullptr, ex_w, nullptr, tl, nullptr);
-  ex.backward(B, true, Hv, grad);
-  MF_CUDA(h, cudaGetLastError());
-  return ex.st;
+  return with_exec<E>(h, B, 1, 0, 0, false, s, [&](auto& ex) {
+    return hvp_run(ex, B, theta, x, y, ex_w, v, Hv, tl, grad);
+  });
 }
 
 }  // namespace
@@ -755,22 +816,37 @@ const char* mf_last_error(mf_handle h) { return h ? h->err.c_str() : "NULL handl
 mf_status mf_create(const mf_model_desc* d, mf_handle* out) {
   if (!d || !out) return MF_ERR_INVALID_ARG;
   *out = nullptr;
-  if (d->arch == MF_ARCH_DECODER) return MF_ERR_UNSUPPORTED;
-  if (d->arch != MF_ARCH_MLP) return MF_ERR_INVALID_ARG;
-  if (d->n_layers < 1 || d->n_layers > MF_MAX_LAYERS) return MF_ERR_INVALID_ARG;
-  for (int i = 0; i <= d->n_layers; ++i)
-    if (d->dims[i] < 1 || d->dims[i] > (1 << 20)) return MF_ERR_INVALID_ARG;
-  if (d->act < MF_ACT_IDENT || d->act > MF_ACT_SILU) return MF_ERR_INVALID_ARG;
-  if (d->loss != MF_LOSS_SQUARED && d->loss != MF_LOSS_SOFTMAX_CE) {
-    return d->loss == MF_LOSS_NEXT_TOKEN_CE ? MF_ERR_UNSUPPORTED : MF_ERR_INVALID_ARG;
-  }
   if (d->precision != MF_PREC_FP32 && d->precision != MF_PREC_BF16) return MF_ERR_INVALID_ARG;
+  const bool decoder = d->arch == MF_ARCH_DECODER;
+  if (decoder) {
+    if (d->loss != MF_LOSS_NEXT_TOKEN_CE || d->n_layers < 1 || d->n_layers > 30 ||
+        d->d_model < 8 || d->n_heads < 1 || d->d_model % d->n_heads != 0 ||
+        (d->d_model / d->n_heads) % 8 != 0 || d->d_ff < 8 || d->d_ff % 8 != 0 ||
+        d->d_model % 8 != 0 || d->vocab < 2 || d->vocab % 8 != 0 || d->seq_len < 8 ||
+        d->seq_len % 8 != 0)
+      return MF_ERR_INVALID_ARG;
+  } else {
+    if (d->arch != MF_ARCH_MLP) return MF_ERR_INVALID_ARG;
+    if (d->n_layers < 1 || d->n_layers > MF_MAX_LAYERS) return MF_ERR_INVALID_ARG;
+    for (int i = 0; i <= d->n_layers; ++i)
+      if (d->dims[i] < 1 || d->dims[i] > (1 << 20)) return MF_ERR_INVALID_ARG;
+    if (d->act < MF_ACT_IDENT || d->act > MF_ACT_SILU) return MF_ERR_INVALID_ARG;
+    if (d->loss != MF_LOSS_SQUARED && d->loss != MF_LOSS_SOFTMAX_CE) return MF_ERR_INVALID_ARG;
+  }
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) { cudaGetLastError(); return MF_ERR_CUDA; }
   mf_ctx* h = new mf_ctx();
   h->md = *d;
-  h->L = d->n_layers;
-  h->dims.assign(d->dims, d->dims + d->n_layers + 1);
+  h->decoder = decoder;
+  if (decoder) {
+    h->Ly = dec_layout(*d);
+    h->P = dec_param_count(h->Ly);
+    h->bf16 = d->precision == MF_PREC_BF16;
+    h->dims.assign(1, d->d_model);
+    h->maxd = d->d_model;
+  }
+  h->L = decoder ? 0 : d->n_layers;
+  if (!decoder) h->dims.assign(d->dims, d->dims + d->n_layers + 1);
   int64_t o = 0;
   for (int l = 0; l < h->L; ++l) {
     h->woff.push_back(o);
@@ -778,9 +854,11 @@ mf_status mf_create(const mf_model_desc* d, mf_handle* out) {
     h->boff.push_back(d->has_bias ? o : -1);
     if (d->has_bias) o += h->dims[l + 1];
   }
-  h->P = o;
-  h->maxd = *std::max_element(h->dims.begin(), h->dims.end());
-  h->bf16 = d->precision == MF_PREC_BF16;
+  if (!decoder) {
+    h->P = o;
+    h->maxd = *std::max_element(h->dims.begin(), h->dims.end());
+    h->bf16 = d->precision == MF_PREC_BF16;
+  }
   if (cudaMalloc(&h->d_status, sizeof(int)) != cudaSuccess ||
       cudaMemset(h->d_status, 0, sizeof(int)) != cudaSuccess ||
       cudaStreamCreateWithFlags(&h->gstream, cudaStreamNonBlocking) != cudaSuccess ||
@@ -833,6 +911,11 @@ mf_status mf_workspace_bytes(mf_handle h, const mf_loop_desc* lp, size_t* bytes)
   mf_status st = validate_loop(h, lp);
   if (st != MF_OK) return st;
   const bool lr_meta = lp->meta_kind & (MF_META_PARAM_LOGLR | MF_META_SCALAR_LOGLR);
+  if (h->decoder) {
+    *bytes = make_dec_plan(h, h->Ly, std::max(lp->B, lp->B_outer), lp->T, lp->T + 1,
+                           lr_meta ? lp->T : 0, lp->meta_kind & MF_META_SCALAR_LOGLR).bytes;
+    return MF_OK;
+  }
   *bytes = make_plan(h, std::max(lp->B, lp->B_outer), lp->T, lp->T + 1, lr_meta ? lp->T : 0,
                      lp->meta_kind & MF_META_SCALAR_LOGLR).bytes;
   return MF_OK;
@@ -1078,7 +1161,7 @@ extern "C" mf_status mf_hvp_noalloc(const mf_model_desc* d, int B, const float* 
                                     const float* v, float* Hv, float* tangent_losses,
                                     float* grad, void* stream) {
   if (!d || B < 1 || !theta || !x || !y || !v || !Hv) return MF_ERR_INVALID_ARG;
-  if (d->arch == MF_ARCH_DECODER) return MF_ERR_UNSUPPORTED;
+  if (d->arch == MF_ARCH_DECODER) return MF_ERR_UNSUPPORTED;   // MLP models only
   if (d->arch != MF_ARCH_MLP || d->n_layers < 1 || d->n_layers > MF_MAX_LAYERS)
     return MF_ERR_INVALID_ARG;
   for (int i = 0; i <= d->n_layers; ++i)

@@ -1,0 +1,690 @@
+// Row and elementwise kernels of the dual (primal + tangent) decoder-only transformer:
+// embedding gather and deterministic scatter-add, fused residual + RMSNorm forward and its
+// dual backward, RoPE with the head split (and its transpose for the backward), causal
+// softmax with its tangent, the softmax backward with its tangent, next-token
+// cross-entropy with per-sequence weights (the mixed term of Eq. 7 per sequence), and
+// deterministic column reductions for the RMSNorm gains.
+//
+// Notation (per token row): n = x r, r = (mean x^2 + eps)^-1/2, h = g n;
+// tangents carry a dot: r' = -r^3 mean(x x'), n' = x' r + x r', h' = g' n + g n'.
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <math.h>
+#include <stdint.h>
+
+#include "device_math.cuh"
+#include "internal.h"
+
+namespace mf {
+namespace {
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// Block-wide sum of two values (fixed reduction order), blockDim.x a multiple of 32, <= 1024.
+__device__ __forceinline__ float2 block_sum2(float a, float b) {
+  __shared__ float2 red[32];
+  a = warp_sum(a);
+  b = warp_sum(b);
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();
+  if (l == 0) red[w] = make_float2(a, b);
+  __syncthreads();
+  float2 r = make_float2(0.f, 0.f);
+  const int nw = blockDim.x >> 5;
+  if (w == 0) {
+    float2 v = l < nw ? red[l] : make_float2(0.f, 0.f);
+    v.x = warp_sum(v.x);
+    v.y = warp_sum(v.y);
+    if (l == 0) red[0] = v;
+  }
+  __syncthreads();
+  r = red[0];
+  return r;
+}
+
+__device__ __forceinline__ float ld_t(const float* p, int64_t i) { return p[i]; }
+__device__ __forceinline__ float ld_t(const __nv_bfloat16* p, int64_t i) { return __bfloat162float(p[i]); }
+
+// x[r] = E[id(r)], x'[r] = U_E[id(r)]  (ids [B][S+1]; row r = b S + s uses ids[b][s])
+__global__ void embed_fwd_kernel(const int* __restrict__ ids, int S, int d, int V,
+                                 const float* __restrict__ E, const float* __restrict__ UE,
+                                 float* __restrict__ x, float* __restrict__ xd, int* status) {
+  const int r = blockIdx.x;
+  const int b = r / S, s = r % S;
+  int id = ids[static_cast<int64_t>(b) * (S + 1) + s];
+  if (id < 0 || id >= V) {
+    if (threadIdx.x == 0 && status) atomicExch(status, 1);
+    id = 0;
+  }
+  for (int j = threadIdx.x; j < d; j += blockDim.x) {
+    x[static_cast<int64_t>(r) * d + j] = E[static_cast<int64_t>(id) * d + j];
+    if (xd) xd[static_cast<int64_t>(r) * d + j] = UE[static_cast<int64_t>(id) * d + j];
+  }
+}
+
+// Fused residual add + RMSNorm (dual).  x = x_in (+ y); stores x (float32), r, r', and
+// h = g x r (and h') in T, row-major [N][ldh].
+template <typename T>
+__global__ void rmsnorm_fwd_kernel(int d, float eps, const float* __restrict__ x_in,
+                                   const float* __restrict__ y, const float* __restrict__ xd_in,
+                                   const float* __restrict__ yd, const float* __restrict__ g,
+                                   const float* __restrict__ gd, float* __restrict__ x_out,
+                                   float* __restrict__ xd_out, float* __restrict__ rr,
+                                   float* __restrict__ rrd, T* __restrict__ h, T* __restrict__ hd,
+                                   int ldh) {
+  const int r = blockIdx.x;
+  const int64_t o = static_cast<int64_t>(r) * d;
+  const bool dual = xd_in != nullptr;
+  float s2 = 0.f, s1 = 0.f;
+  for (int j = threadIdx.x; j < d; j += blockDim.x) {
+    float v = x_in[o + j] + (y ? y[o + j] : 0.f);
+    x_out[o + j] = v;
+    s2 += v * v;
+    if (dual) {
+      const float vd = xd_in[o + j] + (yd ? yd[o + j] : 0.f);
+      xd_out[o + j] = vd;
+      s1 += v * vd;
+    }
+  }
+  const float2 sums = block_sum2(s2, s1);
+  const float inv_d = 1.f / static_cast<float>(d);
+  const float rs = rsqrtf(sums.x * inv_d + eps);
+  const float rsd = -rs * rs * rs * sums.y * inv_d;
+  if (threadIdx.x == 0) {
+    rr[r] = rs;
+    if (dual) rrd[r] = rsd;
+  }
+  const int64_t oh = static_cast<int64_t>(r) * ldh;
+  for (int j = threadIdx.x; j < d; j += blockDim.x) {
+    const float v = x_out[o + j];
+    const float n = v * rs;
+    h[oh + j] = to_t<T>(g[j] * n);
+    if (dual) {
+      const float nd = xd_out[o + j] * rs + v * rsd;
+      hd[oh + j] = to_t<T>(gd[j] * n + g[j] * nd);
+    }
+  }
+}
+
+// Dual RMSNorm backward, accumulated into the residual gradient:
+//   dx += r (dn - n c),  c = mean(dn n),  dn = dy g
+//   dx' += r' (dn - n c) + r (dn' - n' c - n c'),  dn' = dy' g + dy g',  c' = mean(dn' n + dn n')
+template <typename T>
+__global__ void rmsnorm_bwd_kernel(int d, const float* __restrict__ x, const float* __restrict__ xd,
+                                   const float* __restrict__ rr, const float* __restrict__ rrd,
+                                   const float* __restrict__ g, const float* __restrict__ gd,
+                                   const float* __restrict__ dy, const float* __restrict__ dyd,
+                                   float* __restrict__ dx, float* __restrict__ dxd) {
+  const int r = blockIdx.x;
+  const int64_t o = static_cast<int64_t>(r) * d;
+  const bool dual = dyd != nullptr;
+  const float rs = rr[r];
+  const float rsd = dual ? rrd[r] : 0.f;
+  float sc = 0.f, scd = 0.f;
+  for (int j = threadIdx.x; j < d; j += blockDim.x) {
+    const float n = x[o + j] * rs;
+    const float dn = dy[o + j] * g[j];
+    sc += dn * n;
+    if (dual) {
+      const float nd = xd[o + j] * rs + x[o + j] * rsd;
+      const float dnd = dyd[o + j] * g[j] + dy[o + j] * gd[j];
+      scd += dnd * n + dn * nd;
+    }
+  }
+  const float2 sums = block_sum2(sc, scd);
+  const float inv_d = 1.f / static_cast<float>(d);
+  const float c = sums.x * inv_d, cd = sums.y * inv_d;
+  for (int j = threadIdx.x; j < d; j += blockDim.x) {
+    const float n = x[o + j] * rs;
+    const float dn = dy[o + j] * g[j];
+    dx[o + j] += rs * (dn - n * c);
+    if (dual) {
+      const float nd = xd[o + j] * rs + x[o + j] * rsd;
+      const float dnd = dyd[o + j] * g[j] + dy[o + j] * gd[j];
+      dxd[o + j] += rsd * (dn - n * c) + rs * (dnd - nd * c - n * cd);
+    }
+  }
+}
+
+// Gain gradients: dg_j = sum_r dy_rj n_rj ;  dg'_j = sum_r (dy'_rj n_rj + dy_rj n'_rj).
+// Block (32 columns x 32 row lanes); each lane sums a strided set of rows, then the 32
+// partials are added in a fixed order (deterministic).
+__global__ void gain_grad_kernel(int N, int d, const float* __restrict__ x,
+                                 const float* __restrict__ xd, const float* __restrict__ rr,
+                                 const float* __restrict__ rrd, const float* __restrict__ dy,
+                                 const float* __restrict__ dyd, float* __restrict__ dg,
+                                 float* __restrict__ dgd) {
+  __shared__ float sp[32][33];
+  __shared__ float spd[32][33];
+  const int j = blockIdx.x * 32 + threadIdx.x;
+  const bool dual = dyd != nullptr;
+  float a = 0.f, ad = 0.f;
+  if (j < d) {
+    for (int r = threadIdx.y; r < N; r += 32) {
+      const int64_t o = static_cast<int64_t>(r) * d + j;
+      const float n = x[o] * rr[r];
+      a += dy[o] * n;
+      if (dual) {
+        const float nd = xd[o] * rr[r] + x[o] * rrd[r];
+        ad += dyd[o] * n + dy[o] * nd;
+      }
+    }
+  }
+  sp[threadIdx.y][threadIdx.x] = a;
+  spd[threadIdx.y][threadIdx.x] = ad;
+  __syncthreads();
+  if (threadIdx.y == 0 && j < d) {
+    float s = 0.f, sd = 0.f;
+    for (int k = 0; k < 32; ++k) { s += sp[k][threadIdx.x]; sd += spd[k][threadIdx.x]; }
+    if (dg) dg[j] = s;
+    if (dual && dgd) dgd[j] = sd;
+  }
+}
+
+// RoPE (rotate-half) on q and k, q scaled by 1/sqrt(dh), head split.  qkv [N][3d] float32
+// (token-major) -> Q, K, V [B*H][S][dh] in T.  Angle of pair j at position s:
+// s * base^(-2 j / dh).
+template <typename T>
+__global__ void rope_split_kernel(int S, int H, int dh, float base, float qscale,
+                                  const float* __restrict__ qkv, T* __restrict__ Q,
+                                  T* __restrict__ K, T* __restrict__ Vv) {
+  const int r = blockIdx.x;                 // token row
+  const int b = r / S, s = r % S;
+  const int d = H * dh, half = dh / 2;
+  const float* row = qkv + static_cast<int64_t>(r) * 3 * d;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    const int h = c / dh, e = c % dh;
+    const int j = e < half ? e : e - half;
+    const float ang = static_cast<float>(s) * powf(base, -2.f * static_cast<float>(j) / static_cast<float>(dh));
+    float sn, cs;
+    sincosf(ang, &sn, &cs);
+    const float q = row[c], k = row[d + c];
+    const float qo = e < half ? -row[c + half] : row[c - half];
+    const float ko = e < half ? -row[d + c + half] : row[d + c - half];
+    const int64_t o = ((static_cast<int64_t>(b) * H + h) * S + s) * dh + e;
+    Q[o] = to_t<T>((q * cs + qo * sn) * qscale);
+    K[o] = to_t<T>(k * cs + ko * sn);
+    Vv[o] = to_t<T>(row[2 * d + c]);
+  }
+}
+
+// Transpose of the RoPE/split map for the backward: dQ, dK, dV [B*H][S][dh] (float32) ->
+// dqkv [N][3d] row-major (T):  dq = R^T(dQ) qscale, dk = R^T(dK), dv = dV, with
+// R^T(y) = y cos + [y2, -y1] sin.
+template <typename T>
+__global__ void rope_merge_kernel(int S, int H, int dh, float base, float qscale,
+                                  const float* __restrict__ dQ, const float* __restrict__ dK,
+                                  const float* __restrict__ dV, T* __restrict__ out, int ldo) {
+  const int r = blockIdx.x;
+  const int b = r / S, s = r % S;
+  const int d = H * dh, half = dh / 2;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    const int h = c / dh, e = c % dh;
+    const int j = e < half ? e : e - half;
+    const float ang = static_cast<float>(s) * powf(base, -2.f * static_cast<float>(j) / static_cast<float>(dh));
+    float sn, cs;
+    sincosf(ang, &sn, &cs);
+    const int64_t o = ((static_cast<int64_t>(b) * H + h) * S + s) * dh;
+    const float q = dQ[o + e], k = dK[o + e];
+    const float qo = e < half ? dQ[o + e + half] : -dQ[o + e - half];
+    const float ko = e < half ? dK[o + e + half] : -dK[o + e - half];
+    T* row = out + static_cast<int64_t>(r) * ldo;
+    row[c] = to_t<T>((q * cs + qo * sn) * qscale);
+    row[d + c] = to_t<T>(k * cs + ko * sn);
+    row[2 * d + c] = to_t<T>(dV[o + e]);
+  }
+}
+
+// Head merge: O [B*H][S][dh] (float32) -> [N][ldo] (T) token-major, column h*dh + e.
+template <typename T>
+__global__ void head_merge_kernel(int S, int H, int dh, const float* __restrict__ O,
+                                  T* __restrict__ out, int ldo) {
+  const int r = blockIdx.x;
+  const int b = r / S, s = r % S;
+  const int d = H * dh;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    const int h = c / dh, e = c % dh;
+    out[static_cast<int64_t>(r) * ldo + c] =
+        to_t<T>(O[((static_cast<int64_t>(b) * H + h) * S + s) * dh + e]);
+  }
+}
+
+// Head split of a token-major float32 gradient [N][d] -> [B*H][S][dh] (T).
+template <typename T>
+__global__ void head_split_kernel(int S, int H, int dh, const float* __restrict__ X,
+                                  T* __restrict__ out) {
+  const int r = blockIdx.x;
+  const int b = r / S, s = r % S;
+  const int d = H * dh;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    const int h = c / dh, e = c % dh;
+    out[((static_cast<int64_t>(b) * H + h) * S + s) * dh + e] =
+        to_t<T>(X[static_cast<int64_t>(r) * d + c]);
+  }
+}
+
+// Causal softmax with tangent, one warp per score row (q): P = softmax(S), keys k > q masked;
+// P' = P (S' - sum_k P S').
+template <typename T>
+__global__ void softmax_fwd_kernel(int S, int rows, const float* __restrict__ Sc,
+                                   const float* __restrict__ Scd, T* __restrict__ P,
+                                   T* __restrict__ Pd) {
+  const int warps = blockDim.x >> 5;
+  const int row = blockIdx.x * warps + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const int q = row % S;
+  const int64_t o = static_cast<int64_t>(row) * S;
+  float mx = -INFINITY;
+  for (int k = lane; k <= q; k += 32) mx = fmaxf(mx, Sc[o + k]);
+  mx = warp_max(mx);
+  float se = 0.f;
+  for (int k = lane; k <= q; k += 32) se += expf(Sc[o + k] - mx);
+  se = warp_sum(se);
+  const float inv = 1.f / se;
+  float ps = 0.f;
+  if (Scd) {
+    for (int k = lane; k <= q; k += 32) ps += expf(Sc[o + k] - mx) * inv * Scd[o + k];
+    ps = warp_sum(ps);
+  }
+  for (int k = lane; k < S; k += 32) {
+    float p = 0.f, pd = 0.f;
+    if (k <= q) {
+      p = expf(Sc[o + k] - mx) * inv;
+      if (Scd) pd = p * (Scd[o + k] - ps);
+    }
+    P[o + k] = to_t<T>(p);
+    if (Pd) Pd[o + k] = to_t<T>(pd);
+  }
+}
+
+// Softmax backward with tangent, one warp per row:
+//   D = sum_k P dP,  D' = sum_k (P' dP + P dP'),
+//   dS = P (dP - D),  dS' = P' (dP - D) + P (dP' - D').
+template <typename T>
+__global__ void softmax_bwd_kernel(int S, int rows, const T* __restrict__ P,
+                                   const T* __restrict__ Pd, const float* __restrict__ dP,
+                                   const float* __restrict__ dPd, T* __restrict__ dS,
+                                   T* __restrict__ dSd) {
+  const int warps = blockDim.x >> 5;
+  const int row = blockIdx.x * warps + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const int64_t o = static_cast<int64_t>(row) * S;
+  const bool dual = dPd != nullptr;
+  float D = 0.f, Dd = 0.f;
+  for (int k = lane; k < S; k += 32) {
+    const float p = ld_t(P, o + k);
+    D += p * dP[o + k];
+    if (dual) Dd += ld_t(Pd, o + k) * dP[o + k] + p * dPd[o + k];
+  }
+  D = warp_sum(D);
+  if (dual) Dd = warp_sum(Dd);
+  for (int k = lane; k < S; k += 32) {
+    const float p = ld_t(P, o + k);
+    const float g = dP[o + k] - D;
+    dS[o + k] = to_t<T>(p * g);
+    if (dual) dSd[o + k] = to_t<T>(ld_t(Pd, o + k) * g + p * (dPd[o + k] - Dd));
+  }
+}
+
+// Next-token cross-entropy row statistics, one block per token row r = b S + s, target
+// ids[b][s+1]:  lse, l = lse - f_y, l' = p.f' - f'_y (with p = softmax(f)).
+__global__ void ce_stats_kernel(int S, int V, const int* __restrict__ ids,
+                                const float* __restrict__ F, const float* __restrict__ Fd,
+                                float* __restrict__ lse, float* __restrict__ l,
+                                float* __restrict__ pf, float* __restrict__ ld, int* status) {
+  const int r = blockIdx.x;
+  const int b = r / S, s = r % S;
+  int y = ids[static_cast<int64_t>(b) * (S + 1) + s + 1];
+  if (y < 0 || y >= V) {
+    if (threadIdx.x == 0 && status) atomicExch(status, 1);
+    y = 0;
+  }
+  const float* f = F + static_cast<int64_t>(r) * V;
+  __shared__ float red[32];
+  float mx = -INFINITY;
+  for (int c = threadIdx.x; c < V; c += blockDim.x) mx = fmaxf(mx, f[c]);
+  mx = warp_max(mx);
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  if (lane == 0) red[w] = mx;
+  __syncthreads();
+  if (w == 0) {
+    float v = lane < nw ? red[lane] : -INFINITY;
+    v = warp_max(v);
+    if (lane == 0) red[0] = v;
+  }
+  __syncthreads();
+  mx = red[0];
+  __syncthreads();
+  float se = 0.f;
+  for (int c = threadIdx.x; c < V; c += blockDim.x) se += expf(f[c] - mx);
+  const float2 a = block_sum2(se, 0.f);
+  const float lz = mx + logf(a.x);
+  float pfd = 0.f;
+  if (Fd) {
+    const float* fd = Fd + static_cast<int64_t>(r) * V;
+    for (int c = threadIdx.x; c < V; c += blockDim.x) pfd += expf(f[c] - lz) * fd[c];
+  }
+  const float2 bsum = block_sum2(pfd, 0.f);
+  if (threadIdx.x == 0) {
+    lse[r] = lz;
+    l[r] = lz - f[y];
+    if (Fd) {
+      pf[r] = bsum.x;
+      ld[r] = bsum.x - Fd[static_cast<int64_t>(r) * V + y];
+    }
+  }
+}
+
+// Cross-entropy seeds over a [rows x V] tile grid: dF = c (p - onehot), dF' = c p (f' - p.f'),
+// with c = w_b / (B S).  Writes row-major [N][ldo].
+template <typename T>
+__global__ void ce_seed_kernel(int S, int V, const int* __restrict__ ids,
+                               const float* __restrict__ F, const float* __restrict__ Fd,
+                               const float* __restrict__ lse, const float* __restrict__ pf,
+                               const float* __restrict__ eta_w, const float* __restrict__ ex_w,
+                               float inv_norm, T* __restrict__ dF, T* __restrict__ dFd, int ldo) {
+  const int r = blockIdx.y;
+  const int b = r / S, s = r % S;
+  const int y = ids[static_cast<int64_t>(b) * (S + 1) + s + 1];
+  float w = 1.f;
+  if (ex_w) w = ex_w[b];
+  else if (eta_w) w = 1.f / (1.f + expf(-eta_w[b]));
+  const float c = w * inv_norm;
+  const float lz = lse[r];
+  const float pfr = Fd ? pf[r] : 0.f;
+  for (int col = blockIdx.x * blockDim.x + threadIdx.x; col < V; col += gridDim.x * blockDim.x) {
+    const int64_t o = static_cast<int64_t>(r) * V + col;
+    const float p = expf(F[o] - lz);
+    dF[static_cast<int64_t>(r) * ldo + col] = to_t<T>(c * (p - (col == y ? 1.f : 0.f)));
+    if (Fd) dFd[static_cast<int64_t>(r) * ldo + col] = to_t<T>(c * p * (Fd[o] - pfr));
+  }
+}
+
+// Per-sequence reductions, one warp per sequence: l_b = mean_s l_bs, l'_b = mean_s l'_bs;
+// d eta_b = sigmoid'(eta_b) l'_b / B; optional outputs.
+__global__ void seq_reduce_kernel(int B, int S, const float* __restrict__ l,
+                                  const float* __restrict__ ld, const float* __restrict__ eta_w,
+                                  float invB, float* __restrict__ l_seq, float* __restrict__ ld_seq,
+                                  float* __restrict__ d_eta) {
+  const int warps = blockDim.x >> 5;
+  const int b = blockIdx.x * warps + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (b >= B) return;
+  float a = 0.f, ad = 0.f;
+  for (int s = lane; s < S; s += 32) {
+    a += l[static_cast<int64_t>(b) * S + s];
+    if (ld) ad += ld[static_cast<int64_t>(b) * S + s];
+  }
+  a = warp_sum(a) / static_cast<float>(S);
+  ad = warp_sum(ad) / static_cast<float>(S);
+  if (lane == 0) {
+    if (l_seq) l_seq[b] = a;
+    if (ld_seq) ld_seq[b] = ad;
+    if (d_eta && eta_w) {
+      const float sg = 1.f / (1.f + expf(-eta_w[b]));
+      d_eta[b] = sg * (1.f - sg) * ad * invB;
+    }
+  }
+}
+
+// ---- deterministic embedding scatter-add --------------------------------------------------
+__global__ void token_count_kernel(int N, int S, int V, const int* __restrict__ ids,
+                                   int* __restrict__ count) {
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= N) return;
+  int id = ids[static_cast<int64_t>(r / S) * (S + 1) + r % S];
+  if (id < 0 || id >= V) id = 0;
+  atomicAdd(&count[id], 1);
+}
+
+// Exclusive scan of count[0..V) into start[0..V] (one block).
+__global__ void scan_kernel(int V, const int* __restrict__ count, int* __restrict__ start) {
+  __shared__ int part[1024];
+  const int per = (V + blockDim.x - 1) / blockDim.x;
+  const int b0 = threadIdx.x * per;
+  int s = 0;
+  for (int i = b0; i < b0 + per && i < V; ++i) s += count[i];
+  part[threadIdx.x] = s;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int acc = 0;
+    for (int i = 0; i < static_cast<int>(blockDim.x); ++i) {
+      const int v = part[i];
+      part[i] = acc;
+      acc += v;
+    }
+    start[V] = acc;
+  }
+  __syncthreads();
+  int acc = part[threadIdx.x];
+  for (int i = b0; i < b0 + per && i < V; ++i) {
+    start[i] = acc;
+    acc += count[i];
+  }
+}
+
+// Stable placement: token r goes to start[id] + (number of earlier tokens with the same id).
+__global__ void token_place_kernel(int N, int S, int V, const int* __restrict__ ids,
+                                   const int* __restrict__ start, int* __restrict__ order) {
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= N) return;
+  auto id_of = [&](int t) {
+    int v = ids[static_cast<int64_t>(t / S) * (S + 1) + t % S];
+    return (v < 0 || v >= V) ? 0 : v;
+  };
+  const int id = id_of(r);
+  int rank = 0;
+  for (int t = 0; t < r; ++t) rank += id_of(t) == id;
+  order[start[id] + rank] = r;
+}
+
+// dE[v] = sum over tokens with id v (in position order) of dx[token]; one block per id.
+__global__ void embed_bwd_kernel(int d, const int* __restrict__ start,
+                                 const int* __restrict__ order, const float* __restrict__ dx,
+                                 const float* __restrict__ dxd, float* __restrict__ dE,
+                                 float* __restrict__ dEd) {
+  const int v = blockIdx.x;
+  const int a = start[v], e = start[v + 1];
+  for (int j = threadIdx.x; j < d; j += blockDim.x) {
+    float s = 0.f, sd = 0.f;
+    for (int k = a; k < e; ++k) {
+      const int64_t o = static_cast<int64_t>(order[k]) * d + j;
+      s += dx[o];
+      if (dxd) sd += dxd[o];
+    }
+    if (dE) dE[static_cast<int64_t>(v) * d + j] = s;
+    if (dEd) dEd[static_cast<int64_t>(v) * d + j] = sd;
+  }
+}
+
+constexpr int TILE = 32, TROWS = 8;
+
+// Batched transpose: X [batch][rows][ld] -> XT [batch][cols][ldT].
+template <typename TI, typename TO>
+__global__ void transpose_b_kernel(const TI* __restrict__ X, int rows, int cols, int ld,
+                                   int64_t bsX, TO* __restrict__ XT, int ldT, int64_t bsT) {
+  __shared__ float tile[TILE][TILE + 1];
+  const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
+  X += blockIdx.z * bsX;
+  XT += blockIdx.z * bsT;
+  const int tx = threadIdx.x, ty = threadIdx.y;
+  for (int i = ty; i < TILE; i += TROWS) {
+    const int r = r0 + i, c = c0 + tx;
+    if (r < rows && c < cols) tile[i][tx] = ld_t(X, static_cast<int64_t>(r) * ld + c);
+  }
+  __syncthreads();
+  for (int i = ty; i < TILE; i += TROWS) {
+    const int c = c0 + i, r = r0 + tx;
+    if (c < cols && r < rows) XT[static_cast<int64_t>(c) * ldT + r] = to_t<TO>(tile[tx][i]);
+  }
+}
+
+// Row-major cast (with a leading dimension) float32 -> T.
+template <typename T>
+__global__ void cast_rows_kernel(const float* __restrict__ X, int rows, int cols, T* __restrict__ Y,
+                                 int ldy) {
+  const int64_t n = static_cast<int64_t>(rows) * cols;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t r = i / cols, c = i % cols;
+    Y[r * ldy + c] = to_t<T>(X[i]);
+  }
+}
+
+int blocks_for(int64_t n) {
+  int64_t b = (n + 255) / 256;
+  if (b > 152 * 16) b = 152 * 16;
+  return static_cast<int>(b < 1 ? 1 : b);
+}
+
+}  // namespace
+
+// ---- launchers -------------------------------------------------------------------------------
+void dec_embed_fwd(int N, int S, int d, int V, const int* ids, const float* E, const float* UE,
+                   float* x, float* xd, int* status, cudaStream_t s) {
+  embed_fwd_kernel<<<N, 256, 0, s>>>(ids, S, d, V, E, UE, x, xd, status);
+}
+
+template <typename T>
+void dec_rmsnorm_fwd(int N, int d, float eps, const float* x_in, const float* y, const float* xd_in,
+                     const float* yd, const float* g, const float* gd, float* x_out, float* xd_out,
+                     float* r, float* rd, T* h, T* hd, int ldh, cudaStream_t s) {
+  rmsnorm_fwd_kernel<T><<<N, 256, 0, s>>>(d, eps, x_in, y, xd_in, yd, g, gd, x_out, xd_out, r, rd,
+                                          h, hd, ldh);
+}
+
+template <typename T>
+void dec_rmsnorm_bwd(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
+                     const float* g, const float* gd, const float* dy, const float* dyd, float* dx,
+                     float* dxd, cudaStream_t s) {
+  rmsnorm_bwd_kernel<T><<<N, 256, 0, s>>>(d, x, xd, r, rd, g, gd, dy, dyd, dx, dxd);
+}
+
+void dec_gain_grad(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
+                   const float* dy, const float* dyd, float* dg, float* dgd, cudaStream_t s) {
+  gain_grad_kernel<<<(d + 31) / 32, dim3(32, 32), 0, s>>>(N, d, x, xd, r, rd, dy, dyd, dg, dgd);
+}
+
+template <typename T>
+void dec_rope_split(int N, int S, int H, int dh, float base, float qscale, const float* qkv, T* Q,
+                    T* K, T* V, cudaStream_t s) {
+  rope_split_kernel<T><<<N, 256, 0, s>>>(S, H, dh, base, qscale, qkv, Q, K, V);
+}
+
+template <typename T>
+void dec_rope_merge(int N, int S, int H, int dh, float base, float qscale, const float* dQ,
+                    const float* dK, const float* dV, T* out, int ldo, cudaStream_t s) {
+  rope_merge_kernel<T><<<N, 256, 0, s>>>(S, H, dh, base, qscale, dQ, dK, dV, out, ldo);
+}
+
+template <typename T>
+void dec_head_merge(int N, int S, int H, int dh, const float* O, T* out, int ldo, cudaStream_t s) {
+  head_merge_kernel<T><<<N, 256, 0, s>>>(S, H, dh, O, out, ldo);
+}
+
+template <typename T>
+void dec_head_split(int N, int S, int H, int dh, const float* X, T* out, cudaStream_t s) {
+  head_split_kernel<T><<<N, 256, 0, s>>>(S, H, dh, X, out);
+}
+
+template <typename T>
+void dec_softmax_fwd(int S, int rows, const float* Sc, const float* Scd, T* P, T* Pd,
+                     cudaStream_t s) {
+  softmax_fwd_kernel<T><<<(rows + 7) / 8, 256, 0, s>>>(S, rows, Sc, Scd, P, Pd);
+}
+
+template <typename T>
+void dec_softmax_bwd(int S, int rows, const T* P, const T* Pd, const float* dP, const float* dPd,
+                     T* dS, T* dSd, cudaStream_t s) {
+  softmax_bwd_kernel<T><<<(rows + 7) / 8, 256, 0, s>>>(S, rows, P, Pd, dP, dPd, dS, dSd);
+}
+
+void dec_ce_stats(int N, int S, int V, const int* ids, const float* F, const float* Fd, float* lse,
+                  float* l, float* pf, float* ld, int* status, cudaStream_t s) {
+  ce_stats_kernel<<<N, 512, 0, s>>>(S, V, ids, F, Fd, lse, l, pf, ld, status);
+}
+
+template <typename T>
+void dec_ce_seed(int N, int S, int V, const int* ids, const float* F, const float* Fd,
+                 const float* lse, const float* pf, const float* eta_w, const float* ex_w,
+                 float inv_norm, T* dF, T* dFd, int ldo, cudaStream_t s) {
+  dim3 grid((V + 255) / 256 > 16 ? 16 : (V + 255) / 256, N);
+  ce_seed_kernel<T><<<grid, 256, 0, s>>>(S, V, ids, F, Fd, lse, pf, eta_w, ex_w, inv_norm, dF, dFd,
+                                         ldo);
+}
+
+void dec_seq_reduce(int B, int S, const float* l, const float* ld, const float* eta_w, float invB,
+                    float* l_seq, float* ld_seq, float* d_eta, cudaStream_t s) {
+  seq_reduce_kernel<<<(B + 7) / 8, 256, 0, s>>>(B, S, l, ld, eta_w, invB, l_seq, ld_seq, d_eta);
+}
+
+void dec_token_csr(int N, int S, int V, const int* ids, int* count, int* start, int* order,
+                   cudaStream_t s) {
+  cudaMemsetAsync(count, 0, sizeof(int) * V, s);
+  token_count_kernel<<<(N + 255) / 256, 256, 0, s>>>(N, S, V, ids, count);
+  scan_kernel<<<1, 1024, 0, s>>>(V, count, start);
+  token_place_kernel<<<(N + 255) / 256, 256, 0, s>>>(N, S, V, ids, start, order);
+}
+
+void dec_embed_bwd(int V, int d, const int* start, const int* order, const float* dx,
+                   const float* dxd, float* dE, float* dEd, cudaStream_t s) {
+  embed_bwd_kernel<<<V, 256, 0, s>>>(d, start, order, dx, dxd, dE, dEd);
+}
+
+template <typename TI, typename TO>
+void transpose_batched(const TI* X, int rows, int cols, int ld, int64_t bsX, TO* XT, int ldT,
+                       int64_t bsT, int batch, cudaStream_t s) {
+  if (rows <= 0 || cols <= 0 || batch <= 0) return;
+  dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE, batch);
+  transpose_b_kernel<TI, TO><<<grid, dim3(TILE, TROWS), 0, s>>>(X, rows, cols, ld, bsX, XT, ldT, bsT);
+}
+
+template <typename T>
+void cast_rows(const float* X, int rows, int cols, T* Y, int ldy, cudaStream_t s) {
+  cast_rows_kernel<T><<<blocks_for(static_cast<int64_t>(rows) * cols), 256, 0, s>>>(X, rows, cols, Y, ldy);
+}
+
+#define MF_DEC_INST(T)                                                                            \
+  template void dec_rmsnorm_fwd<T>(int, int, float, const float*, const float*, const float*,      \
+                                   const float*, const float*, const float*, float*, float*,       \
+                                   float*, float*, T*, T*, int, cudaStream_t);                     \
+  template void dec_rmsnorm_bwd<T>(int, int, const float*, const float*, const float*,             \
+                                   const float*, const float*, const float*, const float*,         \
+                                   const float*, float*, float*, cudaStream_t);                    \
+  template void dec_rope_split<T>(int, int, int, int, float, float, const float*, T*, T*, T*,      \
+                                  cudaStream_t);                                                   \
+  template void dec_rope_merge<T>(int, int, int, int, float, float, const float*, const float*,    \
+                                  const float*, T*, int, cudaStream_t);                            \
+  template void dec_head_merge<T>(int, int, int, int, const float*, T*, int, cudaStream_t);       \
+  template void dec_head_split<T>(int, int, int, int, const float*, T*, cudaStream_t);            \
+  template void dec_softmax_fwd<T>(int, int, const float*, const float*, T*, T*, cudaStream_t);   \
+  template void dec_softmax_bwd<T>(int, int, const T*, const T*, const float*, const float*, T*,  \
+                                   T*, cudaStream_t);                                              \
+  template void dec_ce_seed<T>(int, int, int, const int*, const float*, const float*,              \
+                               const float*, const float*, const float*, const float*, float, T*,  \
+                               T*, int, cudaStream_t);                                             \
+  template void cast_rows<T>(const float*, int, int, T*, int, cudaStream_t);
+MF_DEC_INST(float)
+MF_DEC_INST(__nv_bfloat16)
+#undef MF_DEC_INST
+template void transpose_batched<float, float>(const float*, int, int, int, int64_t, float*, int,
+                                              int64_t, int, cudaStream_t);
+template void transpose_batched<__nv_bfloat16, __nv_bfloat16>(const __nv_bfloat16*, int, int, int,
+                                                              int64_t, __nv_bfloat16*, int, int64_t,
+                                                              int, cudaStream_t);
+template void transpose_batched<float, __nv_bfloat16>(const float*, int, int, int, int64_t,
+                                                      __nv_bfloat16*, int, int64_t, int,
+                                                      cudaStream_t);
+
+}  // namespace mf

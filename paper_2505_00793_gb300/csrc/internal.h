@@ -42,6 +42,8 @@ struct GemmArgs {
   float* C1 = nullptr; int ldc1 = 0; const float* bias1 = nullptr;
   unsigned terms = 0;
   EpiParams epi;
+  int batch = 1;           // independent GEMMs of the same shape (attention heads)
+  int64_t bsA0 = 0, bsA1 = 0, bsB0 = 0, bsB1 = 0, bsC0 = 0, bsC1 = 0;   // batch strides (elements)
   int split_k = 0;         // 0 = choose automatically, else 1/2/4/8 (tensor-core path)
   int bn = 0, ka = 0;      // tile width / K atoms per stage; 0 = choose automatically
   int* status = nullptr;   // device status word (timeouts), may be null
@@ -101,7 +103,7 @@ struct LrArgs {
 // occupies rows[l] x dout[l] floats at off[l] (W_l rows, then the bias row when present);
 // its first din[l] rows are cast to the GEMM operand copies W (row-major [din][ldw]) and
 // WT (transposed [dout][ldwt]), or U / UT for the tangent.
-constexpr int kMaxLayers = 32;
+constexpr int kMaxLayers = 96;
 struct LayerTable {
   int n = 0;
   int rows[kMaxLayers], din[kMaxLayers], dout[kMaxLayers];
@@ -132,5 +134,52 @@ template <typename T>
 void layer_update(const LayerTable& tab, const LayerUpdArgs& a, cudaStream_t s);
 
 void fill(float* p, int64_t n, float v, cudaStream_t s);
+
+// ---- decoder-only transformer kernels (decoder_kernels.cu) ------------------------------
+void dec_embed_fwd(int N, int S, int d, int V, const int* ids, const float* E, const float* UE,
+                   float* x, float* xd, int* status, cudaStream_t s);
+template <typename T>
+void dec_rmsnorm_fwd(int N, int d, float eps, const float* x_in, const float* y, const float* xd_in,
+                     const float* yd, const float* g, const float* gd, float* x_out, float* xd_out,
+                     float* r, float* rd, T* h, T* hd, int ldh, cudaStream_t s);
+template <typename T>
+void dec_rmsnorm_bwd(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
+                     const float* g, const float* gd, const float* dy, const float* dyd, float* dx,
+                     float* dxd, cudaStream_t s);
+void dec_gain_grad(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
+                   const float* dy, const float* dyd, float* dg, float* dgd, cudaStream_t s);
+template <typename T>
+void dec_rope_split(int N, int S, int H, int dh, float base, float qscale, const float* qkv, T* Q,
+                    T* K, T* V, cudaStream_t s);
+template <typename T>
+void dec_rope_merge(int N, int S, int H, int dh, float base, float qscale, const float* dQ,
+                    const float* dK, const float* dV, T* out, int ldo, cudaStream_t s);
+template <typename T>
+void dec_head_merge(int N, int S, int H, int dh, const float* O, T* out, int ldo, cudaStream_t s);
+template <typename T>
+void dec_head_split(int N, int S, int H, int dh, const float* X, T* out, cudaStream_t s);
+template <typename T>
+void dec_softmax_fwd(int S, int rows, const float* Sc, const float* Scd, T* P, T* Pd,
+                     cudaStream_t s);
+template <typename T>
+void dec_softmax_bwd(int S, int rows, const T* P, const T* Pd, const float* dP, const float* dPd,
+                     T* dS, T* dSd, cudaStream_t s);
+void dec_ce_stats(int N, int S, int V, const int* ids, const float* F, const float* Fd, float* lse,
+                  float* l, float* pf, float* ld, int* status, cudaStream_t s);
+template <typename T>
+void dec_ce_seed(int N, int S, int V, const int* ids, const float* F, const float* Fd,
+                 const float* lse, const float* pf, const float* eta_w, const float* ex_w,
+                 float inv_norm, T* dF, T* dFd, int ldo, cudaStream_t s);
+void dec_seq_reduce(int B, int S, const float* l, const float* ld, const float* eta_w, float invB,
+                    float* l_seq, float* ld_seq, float* d_eta, cudaStream_t s);
+void dec_token_csr(int N, int S, int V, const int* ids, int* count, int* start, int* order,
+                   cudaStream_t s);
+void dec_embed_bwd(int V, int d, const int* start, const int* order, const float* dx,
+                   const float* dxd, float* dE, float* dEd, cudaStream_t s);
+template <typename TI, typename TO>
+void transpose_batched(const TI* X, int rows, int cols, int ld, int64_t bsX, TO* XT, int ldT,
+                       int64_t bsT, int batch, cudaStream_t s);
+template <typename T>
+void cast_rows(const float* X, int rows, int cols, T* Y, int ldy, cudaStream_t s);
 
 }  // namespace mf

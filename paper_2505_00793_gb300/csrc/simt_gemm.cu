@@ -21,9 +21,16 @@ struct SimtParams {
   const float* B[2]; int ldb[2];
   float* C[2]; int ldc[2]; const float* bias[2];
   EpiParams epi;
+  int64_t bsA[2], bsB[2], bsC[2];   // batch strides (blockIdx.z = batch index)
 };
 
-__global__ void __launch_bounds__(256) simt_dual_gemm_kernel(const SimtParams p) {
+__global__ void __launch_bounds__(256) simt_dual_gemm_kernel(SimtParams p) {
+  const int64_t bz = blockIdx.z;
+  for (int i = 0; i < 2; ++i) {
+    if (p.A[i]) p.A[i] += bz * p.bsA[i];
+    if (p.B[i]) p.B[i] += bz * p.bsB[i];
+    if (p.C[i]) p.C[i] += bz * p.bsC[i];
+  }
   __shared__ float As[TK][TM + 1];
   __shared__ float Bs[TK][TN + 1];
   const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
@@ -109,7 +116,10 @@ cudaError_t simt_gemm(const GemmArgs& a, cudaStream_t s) {
   p.C[0] = a.C0; p.ldc[0] = a.ldc0; p.bias[0] = a.bias0;
   p.C[1] = a.C1; p.ldc[1] = a.ldc1; p.bias[1] = a.bias1;
   p.epi = a.epi;
-  dim3 grid((a.N + TN - 1) / TN, (a.M + TM - 1) / TM);
+  p.bsA[0] = a.bsA0; p.bsA[1] = a.bsA1; p.bsB[0] = a.bsB0; p.bsB[1] = a.bsB1;
+  p.bsC[0] = a.bsC0; p.bsC[1] = a.bsC1;
+  if (a.batch > 1 && a.epi.mode != EPI_STORE) return cudaErrorInvalidValue;
+  dim3 grid((a.N + TN - 1) / TN, (a.M + TM - 1) / TM, a.batch < 1 ? 1 : a.batch);
   simt_dual_gemm_kernel<<<grid, 256, 0, s>>>(p);
   return cudaGetLastError();
 }

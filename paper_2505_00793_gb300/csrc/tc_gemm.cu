@@ -39,6 +39,18 @@ cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why) {
       return cudaErrorInvalidValue;
     }
   }
+  if (a.batch > 1 && a.epi.mode != EPI_STORE) {
+    *why = "batched GEMMs support the plain-store epilogue only";
+    return cudaErrorInvalidValue;
+  }
+  if (a.batch > 1) {
+    const int64_t bs[4] = {a.bsA0, a.bsA1, a.bsB0, a.bsB1};
+    for (int i = 0; i < 4; ++i)
+      if ((a.terms & uses[i]) && (bs[i] & 7)) {
+        *why = "operand batch strides must be multiples of 8 elements";
+        return cudaErrorInvalidValue;
+      }
+  }
   if (a.epi.mode != EPI_STORE) {
     const void* outs[4] = {a.epi.A, a.epi.Ad, a.epi.AT, a.epi.AdT};
     for (int i = 0; i < 4; ++i)
@@ -56,7 +68,7 @@ cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why) {
     // Narrow outputs take the narrowest tile; otherwise 64-wide tiles while a 128-wide grid
     // would leave most SMs idle (small-batch layers), else 128 (dual) or 256 columns.
     const bool dual = a.terms & (T_C1_A1B0 | T_C1_A0B1);
-    const int tiles_m = (a.M + 127) / 128;
+    const int tiles_m = ((a.M + 127) / 128) * (a.batch < 1 ? 1 : a.batch);
     if (a.N <= 16) bn = 16;
     else if (a.N <= 32) bn = 32;
     else if (a.N <= 64 || tiles_m * ((a.N + 127) / 128) < 76) bn = 64;

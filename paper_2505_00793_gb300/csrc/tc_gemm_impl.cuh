@@ -45,6 +45,8 @@ struct TcParams {
   int stages;
   int split;
   int tma_store;          // 1: row-major outputs through TMA stores
+  int batch;              // independent GEMMs; blockIdx.z = batch index * split + split index
+  int64_t bsC0, bsC1;     // batch strides of C0 / C1 (direct-store paths)
   int st_c0, st_c1, st_a, st_ad;   // which row-major outputs exist
   int a0_off, a1_off, b0_off, b1_off, stage_bytes, tx_bytes;
   float* C0; int ldc0; const float* bias0;
@@ -92,12 +94,13 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* s
   }
 }
 
-__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar,
-                                            int x, int y) {
+// Every operand map is 3-D {K, rows, batch}; non-batched GEMMs have batch extent 1.
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                            int x, int y, int z) {
   asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
       : "memory");
 }
 
@@ -269,11 +272,12 @@ __device__ __forceinline__ void fence_proxy_async() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int x, int y,
+                                             int z) {
   asm volatile(
-      "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+      "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
           reinterpret_cast<uint64_t>(map)),
-      "r"(x), "r"(y), "r"(smem_u32(src))
+      "r"(x), "r"(y), "r"(z), "r"(smem_u32(src))
       : "memory");
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
@@ -294,7 +298,7 @@ template <int BN, int MODE, int ACT>
 __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMap* mC0,
                                              const CUtensorMap* mC1, const CUtensorMap* mA,
                                              const CUtensorMap* mAd, uint8_t* stg, uint32_t taddr,
-                                             int q, int lane, int m0, int n0, bool dual) {
+                                             int q, int lane, int m0, int n0, bool dual, int bz) {
   const EpiParams e = p.epi;
   const int row = m0 + q * 32 + lane;
   const bool rowok = row < p.M;
@@ -374,12 +378,12 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
         for (int b = 0; b < 2; ++b) {
           const int x = n0 + c + 32 * b;
           if (x >= p.N) continue;
-          if (p.st_c0) tma_store_2d(mC0, sC0 + b * STG_F32_BOX, x, y);
-          if (p.st_c1) tma_store_2d(mC1, sC1 + b * STG_F32_BOX, x, y);
+          if (p.st_c0) tma_store_3d(mC0, sC0 + b * STG_F32_BOX, x, y, bz);
+          if (p.st_c1) tma_store_3d(mC1, sC1 + b * STG_F32_BOX, x, y, bz);
         }
         if (n0 + c < p.N) {
-          if (p.st_a) tma_store_2d(mA, sA, n0 + c, y);
-          if (p.st_ad) tma_store_2d(mAd, sAd, n0 + c, y);
+          if (p.st_a) tma_store_3d(mA, sA, n0 + c, y, bz);
+          if (p.st_ad) tma_store_3d(mAd, sAd, n0 + c, y, bz);
         }
       }
       bulk_commit();
@@ -401,7 +405,11 @@ __global__ void __launch_bounds__(THREADS, 1)
                         const __grid_constant__ CUtensorMap tmAd, const TcParams prm) {
   // Work on a register copy: a reference into the parameter block would be re-read after
   // every asm statement with a memory clobber (mbarrier waits, commits, stores).
-  const TcParams p = prm;
+  TcParams p = prm;
+  const int bz = static_cast<int>(blockIdx.z) / p.split;     // batch index
+  const int zs = static_cast<int>(blockIdx.z) % p.split;     // split index (cluster rank)
+  if (p.C0) p.C0 += bz * p.bsC0;
+  if (p.C1) p.C1 += bz * p.bsC1;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[MAX_STAGES];
   __shared__ __align__(8) uint64_t empty_bar[MAX_STAGES];
@@ -416,7 +424,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int S = p.split;
   const int nkb = (p.K + SK - 1) / SK;
   const int kper = (nkb + S - 1) / S;
-  const int kb0 = static_cast<int>(blockIdx.z) * kper;
+  const int kb0 = zs * kper;
   const int nk = max(0, min(nkb, kb0 + kper) - kb0);
   const unsigned terms = p.terms;
   const bool dual = (terms & (T_C1_A1B0 | T_C1_A0B1)) != 0;
@@ -461,10 +469,10 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int a = 0; a < KA; ++a) {
           const int ka = k + a * BK;
-          if (a0_off >= 0) tma_load_2d(st + a0_off + a * A_ATOM, &tmA0, &full_bar[s], ka, m0);
-          if (a1_off >= 0) tma_load_2d(st + a1_off + a * A_ATOM, &tmA1, &full_bar[s], ka, m0);
-          if (b0_off >= 0) tma_load_2d(st + b0_off + a * B_ATOM, &tmB0, &full_bar[s], ka, n0);
-          if (b1_off >= 0) tma_load_2d(st + b1_off + a * B_ATOM, &tmB1, &full_bar[s], ka, n0);
+          if (a0_off >= 0) tma_load_3d(st + a0_off + a * A_ATOM, &tmA0, &full_bar[s], ka, m0, bz);
+          if (a1_off >= 0) tma_load_3d(st + a1_off + a * A_ATOM, &tmA1, &full_bar[s], ka, m0, bz);
+          if (b0_off >= 0) tma_load_3d(st + b0_off + a * B_ATOM, &tmB0, &full_bar[s], ka, n0, bz);
+          if (b1_off >= 0) tma_load_3d(st + b1_off + a * B_ATOM, &tmB1, &full_bar[s], ka, n0, bz);
         }
       }
     }
@@ -518,7 +526,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (ok) {
         if (p.tma_store) {
           epilogue_tma<BN, MODE, ACT>(p, &tmC0, &tmC1, &tmA, &tmAd, smem + q * STG_WARP, tbase + lane_off,
-                           q, lane, m0, n0, dual);
+                           q, lane, m0, n0, dual, bz);
         } else {
 #pragma unroll 1
           for (int c = 0; c < BN; c += 16) {
@@ -546,7 +554,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     constexpr int LDP = BN + 4;
     const int nacc = dual ? 2 : 1;
     const int rows_per = BM / S;
-    const uint32_t z = blockIdx.z;
+    const uint32_t z = static_cast<uint32_t>(zs);
     const uint32_t rbase = smem_u32(smem);
     __syncwarp();
     cluster_sync_all();
@@ -681,22 +689,29 @@ EncodeTiledFn encode_fn() {
 // 2-D tensor map, 128-byte swizzle: inner extent `inner` elements, `rows` rows, row pitch
 // `ld` elements, box box_inner x box_rows.
 bool make_map2(CUtensorMap* m, CUtensorMapDataType dt, int esize, const void* ptr, int inner,
-               int rows, int ld, int box_inner, int box_rows) {
+               int rows, int ld, int box_inner, int box_rows, int batch = 1,
+               int64_t bstride = 0) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
-  cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows)};
-  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * esize};
-  cuuint32_t box[2] = {static_cast<cuuint32_t>(box_inner), static_cast<cuuint32_t>(box_rows)};
-  cuuint32_t estr[2] = {1, 1};
-  return fn(m, dt, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+  if (batch < 1) batch = 1;
+  if (batch == 1) bstride = static_cast<int64_t>(ld) * rows;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows),
+                        static_cast<cuuint64_t>(batch)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(ld) * esize,
+                           static_cast<cuuint64_t>(bstride) * esize};
+  cuuint32_t box[3] = {static_cast<cuuint32_t>(box_inner), static_cast<cuuint32_t>(box_rows), 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, dt, 3, const_cast<void*>(ptr), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
          CUDA_SUCCESS;
 }
 
 // K-major bf16 operand [rows][K] (leading dimension ld), box 64 x box_rows.
-bool make_map(CUtensorMap* m, const void* ptr, int K, int rows, int ld, int box_rows) {
-  return make_map2(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, ptr, K, rows, ld, BK, box_rows);
+bool make_map(CUtensorMap* m, const void* ptr, int K, int rows, int ld, int box_rows,
+              int batch = 1, int64_t bstride = 0) {
+  return make_map2(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, ptr, K, rows, ld, BK, box_rows, batch,
+                   bstride);
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
@@ -740,7 +755,8 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
 
   const int tiles_n = (a.N + BN - 1) / BN, tiles_m = (a.M + BM - 1) / BM;
   const int nkb = (a.K + BK * KA - 1) / (BK * KA);
-  int S = a.split_k > 0 ? a.split_k : (BN > 128 ? 1 : choose_split(tiles_n * tiles_m, nkb));
+  int S = a.split_k > 0 ? a.split_k
+                        : (BN > 128 ? 1 : choose_split(tiles_n * tiles_m * (a.batch < 1 ? 1 : a.batch), nkb));
   if (S != 1 && S != 2 && S != 4 && S != 8) { *why = "split_k must be 1, 2, 4 or 8"; return cudaErrorInvalidValue; }
   if (BN > 128) S = 1;
   if (S > nkb) S = 1;
@@ -751,10 +767,14 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
   memset(&mB0, 0, sizeof(mB0)); memset(&mB1, 0, sizeof(mB1));
   memset(&mC0, 0, sizeof(mC0)); memset(&mC1, 0, sizeof(mC1));
   memset(&mA, 0, sizeof(mA)); memset(&mAd, 0, sizeof(mAd));
-  if (useA0 && !make_map(&mA0, a.A0, a.K, a.M, a.lda0, BM)) { *why = "tensor map A0"; return cudaErrorInvalidValue; }
-  if (useA1 && !make_map(&mA1, a.A1, a.K, a.M, a.lda1, BM)) { *why = "tensor map A1"; return cudaErrorInvalidValue; }
-  if (useB0 && !make_map(&mB0, a.B0, a.K, a.N, a.ldb0, BN)) { *why = "tensor map B0"; return cudaErrorInvalidValue; }
-  if (useB1 && !make_map(&mB1, a.B1, a.K, a.N, a.ldb1, BN)) { *why = "tensor map B1"; return cudaErrorInvalidValue; }
+  const int nb = a.batch < 1 ? 1 : a.batch;
+  if (useA0 && !make_map(&mA0, a.A0, a.K, a.M, a.lda0, BM, nb, a.bsA0)) { *why = "tensor map A0"; return cudaErrorInvalidValue; }
+  if (useA1 && !make_map(&mA1, a.A1, a.K, a.M, a.lda1, BM, nb, a.bsA1)) { *why = "tensor map A1"; return cudaErrorInvalidValue; }
+  if (useB0 && !make_map(&mB0, a.B0, a.K, a.N, a.ldb0, BN, nb, a.bsB0)) { *why = "tensor map B0"; return cudaErrorInvalidValue; }
+  if (useB1 && !make_map(&mB1, a.B1, a.K, a.N, a.ldb1, BN, nb, a.bsB1)) { *why = "tensor map B1"; return cudaErrorInvalidValue; }
+  p.batch = nb;
+  p.bsC0 = a.bsC0;
+  p.bsC1 = a.bsC1;
 
   // Row-major outputs through TMA stores when every one of them is aligned for it.
   const bool act = a.epi.mode != EPI_STORE;
@@ -767,10 +787,13 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
   if (p.st_c1) tma_ok = tma_ok && aligned16(p.C1) && !(p.ldc1 & 3);
   if (p.st_a) tma_ok = tma_ok && aligned16(a.epi.A) && !(a.epi.lda & 7);
   if (p.st_ad) tma_ok = tma_ok && aligned16(a.epi.Ad) && !(a.epi.lda & 7);
+  if (nb > 1) tma_ok = tma_ok && !(a.bsC0 & 3) && !(a.bsC1 & 3);
   if (tma_ok && p.st_c0)
-    tma_ok = make_map2(&mC0, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, p.C0, a.N, a.M, p.ldc0, 32, 32);
+    tma_ok = make_map2(&mC0, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, p.C0, a.N, a.M, p.ldc0, 32, 32, nb,
+                       a.bsC0);
   if (tma_ok && p.st_c1)
-    tma_ok = make_map2(&mC1, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, p.C1, a.N, a.M, p.ldc1, 32, 32);
+    tma_ok = make_map2(&mC1, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, p.C1, a.N, a.M, p.ldc1, 32, 32, nb,
+                       a.bsC1);
   if (tma_ok && p.st_a)
     tma_ok = make_map2(&mA, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, a.epi.A, a.N, a.M, a.epi.lda, 64, 32);
   if (tma_ok && p.st_ad)
@@ -795,7 +818,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
   if (smem > 225 * 1024) { *why = "shared memory budget exceeded"; return cudaErrorInvalidValue; }
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof(cfg));
-  cfg.gridDim = dim3(tiles_n, tiles_m, S);
+  cfg.gridDim = dim3(tiles_n, tiles_m, S * nb);
   cfg.blockDim = dim3(THREADS, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;

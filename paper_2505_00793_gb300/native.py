@@ -114,8 +114,16 @@ def _stream(stream):
 
 
 def model_desc_for(w) -> mf_model_desc:
-    """mf_model_desc of a ``synth.Workload`` (MLP)."""
+    """mf_model_desc of a ``synth.Workload`` (MLP or decoder-only transformer)."""
     d = mf_model_desc()
+    if getattr(w, "arch", "mlp") == "decoder":
+        d.arch = MF_ARCH_DECODER
+        d.n_layers = w.n_blocks
+        d.d_model, d.n_heads, d.d_ff, d.vocab, d.seq_len = w.d_model, w.n_heads, w.d_ff, w.vocab, w.seq
+        d.rope_base, d.rms_eps = w.rope_base, w.rms_eps
+        d.loss = LOSSES["next_token_ce"]
+        d.precision = PRECISIONS[w.precision]
+        return d
     d.arch = MF_ARCH_MLP
     d.n_layers = len(w.dims) - 1
     for i, v in enumerate(w.dims):
@@ -239,6 +247,12 @@ class MixFlow:
 def to_device_inputs(w, inp, device="cuda"):
     """Move a ``synth.Inputs`` to the device with the dtypes the ABI expects."""
     import torch
+    if getattr(w, "arch", "mlp") == "decoder":
+        ids = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.int32)).to(device)
+        f = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.float32)).to(device)
+        ix, ox = ids(inp.inner_x), ids(inp.outer_x)
+        return dict(theta0=f(inp.theta0), eta=f(inp.eta), inner_x=ix, inner_y=ix, outer_x=ox,
+                    outer_y=ox)
     xdt = torch.bfloat16 if w.precision == "bf16" else torch.float32
 
     def xt(a):
