@@ -91,3 +91,10 @@ def test_decoder_hvp(name, tol):
     assert rel_l2(Hv.cpu().numpy(), om.hvp(w, inp.theta0, ids, ids, v, wt)) < tol
     assert rel_l2(tl.cpu().numpy(), om.tangent_losses(w, inp.theta0, ids, ids, v)) < tol
     mf.close()
+
+
+@pytest.mark.gpu
+def test_decoder_small_full_size_single_step():
+    """The 27M-parameter decoder (d 512, 8 heads, MLP 2048, 6 blocks, vocabulary 8192,
+    16 sequences of 256 tokens) at T = 1, every output against the oracle."""
+    _check(synth.WORKLOADS["decoder_small"].with_(T=1), 2e-2)
