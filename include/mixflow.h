@@ -41,7 +41,7 @@
  *    immediately; errors found on the device (non-finite values, a kernel wait that ran out
  *    of time) are reported by mf_sync().
  *  - Library workspace (the theta_t checkpoint store, activations) is obtained through the
- *    allocator set with mf_set_allocator (default: cudaMallocAsync on the call's stream),
+ *    allocator set with mf_set_allocator (default: cudaMalloc, freed with cudaFree),
  *    kept in the handle between calls with the same or smaller shape, and released by
  *    mf_release_workspace() or mf_destroy().
  *  - A handle is not thread-safe; use one handle per host thread.
@@ -112,7 +112,11 @@ typedef struct {
  *  meta_kind  bit mask of MF_META_*; eta is laid out as [T*B example-weight logits]
  *             [P per-parameter log-lrs][1 scalar log-lr], in that order, for the bits set.
  *             PARAM_LOGLR and SCALAR_LOGLR are mutually exclusive.
- *  hvp_mode   MF_HVP_MIXED_FOR (this build's sweep; MF_HVP_REV_REV is reserved).
+ *  hvp_mode   MF_HVP_MIXED_FOR: each step's Hessian-vector product is forward-over-reverse
+ *             (Algorithm 2, the mixed-mode sweep).  MF_HVP_REV_REV: reverse-over-reverse
+ *             (Algorithm 1's schedule: the inner backward is kept whole and differentiated
+ *             again in reverse), the standard-AD baseline; same result, more workspace.
+ *             MF_HVP_REV_REV is implemented for MF_ARCH_MLP only (UNSUPPORTED otherwise).
  *  ckpt_every 1 = keep every theta_t in the checkpoint store (the only value accepted). */
 typedef struct {
   int T, B, B_outer;
@@ -140,7 +144,8 @@ mf_status mf_set_allocator(mf_handle h, void* (*alloc)(size_t, void*, void*),
 mf_status mf_param_count(mf_handle h, const mf_loop_desc* loop, int64_t* n_params,
                          int64_t* n_eta);
 
-/* Bytes of workspace mf_meta_grad needs for `loop` (checkpoint store + activations). */
+/* Bytes of workspace mf_meta_grad needs for `loop` (checkpoint store + activations; with
+ * MF_HVP_REV_REV also the stored inner backward graph). */
 mf_status mf_workspace_bytes(mf_handle h, const mf_loop_desc* loop, size_t* bytes);
 
 /* Free the cached workspace now (the next call allocates it again). */
@@ -159,7 +164,8 @@ mf_status mf_inner_rollout(mf_handle h, const mf_loop_desc* loop, const float* t
  *   Hv [P]             = (d^2 L / d theta^2) v        (forward-over-reverse)
  *   tangent_losses [B] = grad l_b(theta) . v           (nullable; the mixed term per example)
  *   grad [P]           = grad L(theta)                 (nullable)
- * hvp_mode must be MF_HVP_MIXED_FOR. */
+ * hvp_mode MF_HVP_MIXED_FOR (forward-over-reverse) or MF_HVP_REV_REV (reverse-over-reverse,
+ * MLP models only; returns MF_ERR_UNSUPPORTED for the decoder). */
 mf_status mf_hvp(mf_handle h, int B, const float* theta, const void* x, const void* y,
                  const float* ex_w, const float* v, float* Hv, float* tangent_losses,
                  float* grad, int hvp_mode, void* stream);
@@ -232,7 +238,7 @@ mf_status mf_hvp_noalloc(const mf_model_desc* desc, int B, const float* theta, c
  *   A0, A1 [M][K] bf16;  B0, B1 [N][K] bf16;  C0, C1 [M][N] float32 (ldc).
  * `terms` selects the products summed into each accumulator:
  *   bit 0: C0 += A0 B0^T   bit 1: C0 += A1 B0^T   bit 2: C0 += A0 B1^T
- *   bit 3: C1 += A1 B0^T   bit 4: C1 += A0 B1^T
+ *   bit 3: C1 += A1 B0^T   bit 4: C1 += A0 B1^T   bit 5: C0 += A1 B1^T
  * The forward tangent of a dual Linear layer is terms = 1|8|16:  C0 = A0 B0^T (primal),
  * C1 = A1 B0^T + A0 B1^T (tangent).  bias0/bias1 [N] float32 are added when non-NULL.
  * Runs on tcgen05 tensor cores with TMEM accumulators and TMA-fed shared memory. */

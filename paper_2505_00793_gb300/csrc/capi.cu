@@ -97,6 +97,10 @@ struct Plan {
   size_t o_theta = 0, o_m = 0, o_g = 0, o_tbar = 0, o_u = 0, o_part = 0, o_l = 0, o_ld = 0;
   std::vector<size_t> o_Wb, o_WbT, o_Ub, o_UbT, o_A, o_Ad, o_AT, o_AdT, o_Z, o_Zd;
   size_t o_dZ[2] = {0, 0}, o_dZd[2] = {0, 0}, o_dZT[2] = {0, 0}, o_dZdT[2] = {0, 0};
+  // reverse-over-reverse: the stored reverse graph (per-layer dz, da) and the adjoints
+  bool ror = false;
+  std::vector<size_t> o_SZ, o_SZT, o_SA, o_DAB, o_DABT, o_ZP;
+  size_t o_DZB = 0, o_ZB = 0, o_ZBT = 0, o_AB = 0;
 };
 
 int n_update_tiles(const mf_ctx* h) {
@@ -111,8 +115,9 @@ int n_update_tiles(const mf_ctx* h) {
 // Transposed activations carry one extra row (ones for a, zeros for a') so that the weight
 // product [a^T; 1][dz] yields the weight and the bias gradient (stored contiguously in theta).
 Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slots,
-               bool with_partials) {
+               bool with_partials, bool ror = false) {
   Plan p;
+  p.ror = ror;
   p.rows = rows;
   p.ldR = ld8(rows);
   p.T = T;
@@ -155,6 +160,23 @@ Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slot
     p.o_dZd[b] = take(static_cast<size_t>(rows) * ld8(md) * es);
     p.o_dZT[b] = take(static_cast<size_t>(md) * p.ldR * es);
     p.o_dZdT[b] = take(static_cast<size_t>(md) * p.ldR * es);
+  }
+  if (ror) {
+    p.o_SZ.resize(L); p.o_SZT.resize(L); p.o_SA.resize(L); p.o_DAB.resize(L); p.o_DABT.resize(L);
+    p.o_ZP.resize(L);
+    for (int l = 0; l < L; ++l) {
+      const int din = h->dims[l], dout = h->dims[l + 1];
+      p.o_SZ[l] = take(static_cast<size_t>(rows) * ld8(dout) * es);
+      p.o_SZT[l] = take(static_cast<size_t>(dout) * p.ldR * es);
+      p.o_SA[l] = take(static_cast<size_t>(rows) * din * 4);
+      p.o_DAB[l] = take(static_cast<size_t>(rows) * ld8(dout) * es);
+      p.o_DABT[l] = take(static_cast<size_t>(dout + 1) * p.ldR * es);
+      p.o_ZP[l] = take(static_cast<size_t>(rows) * dout * 4);
+    }
+    p.o_DZB = take(static_cast<size_t>(rows) * md * 4);
+    p.o_ZB = take(static_cast<size_t>(rows) * ld8(md) * es);
+    p.o_ZBT = take(static_cast<size_t>(md) * p.ldR * es);
+    p.o_AB = take(static_cast<size_t>(rows) * md * 4);
   }
   p.bytes = o;
   return p;
@@ -297,6 +319,11 @@ struct Exec {
   char* base;
   mf_status st = MF_OK;
   mf::LayerTable tab;
+  bool ror_store = false;   // primal backward keeps every layer's dz (and da) for RoR
+
+  // backward seed buffers of layer l (ping-pong, or the stored reverse graph)
+  T* dz_buf(int l) const { return ror_store ? at<T>(p.o_SZ[l]) : at<T>(p.o_dZ[l & 1]); }
+  T* dzT_buf(int l) const { return ror_store ? at<T>(p.o_SZT[l]) : at<T>(p.o_dZT[l & 1]); }
 
   Exec(mf_ctx* h_, const Plan& p_, cudaStream_t s_)
       : h(h_), p(p_), s(s_), base(static_cast<char*>(h_->ws)) {
@@ -377,6 +404,12 @@ struct Exec {
       f.dst[f.n] = at<T>(p.o_AT[l]); f.row[f.n] = h->dims[l]; f.ld[f.n] = p.ldR; f.value[f.n] = 1.f; ++f.n;
       f.dst[f.n] = at<T>(p.o_AdT[l]); f.row[f.n] = h->dims[l]; f.ld[f.n] = p.ldR; f.value[f.n] = 0.f; ++f.n;
     }
+    if (p.ror) {
+      for (int l = 0; l + 1 < h->L; ++l) {
+        f.dst[f.n] = at<T>(p.o_DABT[l]); f.row[f.n] = h->dims[l + 1]; f.ld[f.n] = p.ldR;
+        f.value[f.n] = 0.f; ++f.n;
+      }
+    }
     mf::fill_rows<T>(f, p.ldR, s);
     launched();
   }
@@ -437,7 +470,7 @@ struct Exec {
   // Loss seeds at the head: d f (and its tangent) into backward buffer set (L-1) & 1.
   void loss(int rows, bool dual, const void* y, const float* eta_w, const float* ex_w,
             float* l_out, float* ld_out, float* d_eta) {
-    const int L = h->L, C = h->dims[L], b = (L - 1) & 1;
+    const int L = h->L, C = h->dims[L];
     mf::LossArgs a;
     a.loss = h->md.loss == MF_LOSS_SOFTMAX_CE ? 1 : 0;
     a.rows = rows; a.cols = C;
@@ -448,12 +481,13 @@ struct Exec {
     a.eta_w = eta_w; a.ex_w = ex_w;
     a.inv_norm = 1.f / static_cast<float>(rows);
     a.l = l_out; a.ld = ld_out; a.d_eta = d_eta;
-    a.dF = at<T>(p.o_dZ[b]); a.dFd = dual ? at<T>(p.o_dZd[b]) : nullptr;
+    const int b = (L - 1) & 1;
+    a.dF = dz_buf(L - 1); a.dFd = dual ? at<T>(p.o_dZd[b]) : nullptr;
     a.ldo = ld8(C);
     a.status = h->d_status;
     mf::loss_seed<T>(a, s);
     launched();
-    mf::transpose<T>(at<T>(p.o_dZ[b]), rows, C, ld8(C), at<T>(p.o_dZT[b]), p.ldR, s);
+    mf::transpose<T>(dz_buf(L - 1), rows, C, ld8(C), dzT_buf(L - 1), p.ldR, s);
     launched();
     if (dual) {
       mf::transpose<T>(at<T>(p.o_dZd[b]), rows, C, ld8(C), at<T>(p.o_dZdT[b]), p.ldR, s);
@@ -472,7 +506,7 @@ struct Exec {
       g.M = din + hb; g.N = dout; g.K = rows;
       g.A0 = at<T>(p.o_AT[l]); g.lda0 = p.ldR;
       g.A1 = at<T>(p.o_AdT[l]); g.lda1 = p.ldR;
-      g.B0 = at<T>(p.o_dZT[b]); g.ldb0 = p.ldR;
+      g.B0 = dzT_buf(l); g.ldb0 = p.ldR;
       g.B1 = at<T>(p.o_dZdT[b]); g.ldb1 = p.ldR;
       if (!dual) {
         g.terms = mf::T_C0_A0B0;
@@ -485,12 +519,12 @@ struct Exec {
         g.terms = mf::T_C0_A0B1 | (l > 0 ? mf::T_C0_A1B0 : 0u);
         g.C0 = out_h + h->woff[l]; g.ldc0 = dout;
       }
-      gemm(g);
+      if (dual || out_g) gemm(g);
       if (l == 0) break;
       // data product: da = dz W^T ; da' = dz' W^T + dz U^T ; epilogue -> dz, dz' of layer l-1
       GemmArgs d;
       d.M = rows; d.N = din; d.K = dout;
-      d.A0 = at<T>(p.o_dZ[b]); d.lda0 = ld8(dout);
+      d.A0 = dz_buf(l); d.lda0 = ld8(dout);
       d.A1 = at<T>(p.o_dZd[b]); d.lda1 = ld8(dout);
       d.B0 = at<T>(p.o_Wb[l]); d.ldb0 = ld8(dout);
       d.B1 = at<T>(p.o_Ub[l]); d.ldb1 = ld8(dout);
@@ -500,12 +534,100 @@ struct Exec {
       d.epi.Z = at<float>(p.o_Z[l - 1]);
       d.epi.Zd = dual ? at<float>(p.o_Zd[l - 1]) : nullptr;
       d.epi.ldz = din;
-      d.epi.A = at<T>(p.o_dZ[b ^ 1]);
+      if (ror_store) { d.C0 = at<float>(p.o_SA[l]); d.ldc0 = din; }
+      d.epi.A = dz_buf(l - 1);
       d.epi.Ad = dual ? at<T>(p.o_dZd[b ^ 1]) : nullptr;
       d.epi.lda = ld8(din);
-      d.epi.AT = at<T>(p.o_dZT[b ^ 1]);
+      d.epi.AT = dzT_buf(l - 1);
       d.epi.AdT = dual ? at<T>(p.o_dZdT[b ^ 1]) : nullptr;
       d.epi.ldt = p.ldR;
+      gemm(d);
+    }
+  }
+
+  // Hessian-vector product by reverse-over-reverse (Algorithm 1's schedule): primal forward,
+  // primal backward keeping every layer's dz and da (the reverse graph), then the adjoint of
+  // the backward in forward layer order and the adjoint of the forward in reverse order.
+  // Writes Hv, and per example l'_b (ld_out) and d eta (from the loss Hessian step).
+  void ror_hvp(int rows, const void* x, const float* theta, const float* u, const void* y,
+               const float* eta_w, const float* ex_w, float* Hv, float* grad, float* ld_out,
+               float* d_eta) {
+    const int L = h->L, hb = h->md.has_bias ? 1 : 0;
+    forward(rows, x, theta, nullptr, false);
+    ror_store = true;
+    loss(rows, false, y, eta_w, ex_w, nullptr, nullptr, nullptr);
+    backward(rows, false, nullptr, grad);
+    ror_store = false;
+    // adjoint of the backward pass, layers 0..L-1: dzbar_l = a_{l-1} V_l + c_l + dabar_{l-1} W_l
+    for (int l = 0; l < L; ++l) {
+      const int din = h->dims[l], dout = h->dims[l + 1];
+      GemmArgs g;
+      g.M = rows; g.N = dout; g.K = din;
+      g.A0 = l == 0 ? x : static_cast<const void*>(at<T>(p.o_A[l]));
+      g.lda0 = l == 0 ? din : ld8(din);
+      g.A1 = l == 0 ? nullptr : at<T>(p.o_DAB[l - 1]);
+      g.lda1 = ld8(din);
+      g.B0 = at<T>(p.o_WbT[l]); g.ldb0 = ld8(din);
+      g.B1 = at<T>(p.o_UbT[l]); g.ldb1 = ld8(din);
+      g.terms = mf::T_C0_A0B1 | (l > 0 ? mf::T_C0_A1B0 : 0u);
+      g.C0 = at<float>(p.o_DZB); g.ldc0 = dout;
+      g.bias0 = h->md.has_bias ? u + h->boff[l] : nullptr;
+      gemm(g);
+      if (l + 1 < L) {
+        mf::ror_fwd_elem<T>(h->md.act, at<float>(p.o_DZB), at<float>(p.o_Z[l]),
+                            at<float>(p.o_SA[l + 1]), rows, dout, at<T>(p.o_DAB[l]), ld8(dout),
+                            at<T>(p.o_DABT[l]), p.ldR, at<float>(p.o_ZP[l]), s);
+        launched();
+      } else {
+        // loss Hessian along dzbar (this is the forward tangent of the logits): zbar_{L-1},
+        // the per-example directional losses and the weight meta-gradient
+        mf::LossArgs a;
+        a.loss = h->md.loss == MF_LOSS_SOFTMAX_CE ? 1 : 0;
+        a.rows = rows; a.cols = dout;
+        a.F = at<float>(p.o_Z[l]);
+        a.Fd = at<float>(p.o_DZB);
+        if (a.loss == 0) a.Yf = static_cast<const float*>(y);
+        else a.Yi = static_cast<const int*>(y);
+        a.eta_w = eta_w; a.ex_w = ex_w;
+        a.inv_norm = 1.f / static_cast<float>(rows);
+        a.ld = ld_out; a.d_eta = d_eta;
+        a.dF = nullptr; a.dFd = at<T>(p.o_ZB);
+        a.ldo = ld8(dout);
+        a.status = h->d_status;
+        mf::loss_seed<T>(a, s);
+        launched();
+        mf::transpose<T>(at<T>(p.o_ZB), rows, dout, ld8(dout), at<T>(p.o_ZBT), p.ldR, s);
+        launched();
+      }
+    }
+    // adjoint of the forward pass, layers L-1..0
+    for (int l = L - 1; l >= 0; --l) {
+      const int din = h->dims[l], dout = h->dims[l + 1];
+      if (l + 1 < L) {
+        mf::ror_bwd_elem<T>(h->md.act, at<float>(p.o_ZP[l]), at<float>(p.o_AB), at<float>(p.o_Z[l]),
+                            rows, dout, at<T>(p.o_ZB), ld8(dout), at<T>(p.o_ZBT), p.ldR, s);
+        launched();
+      }
+      // (H v)_{W_l, b_l} = [a_{l-1}^T; 1] zbar_l + [dabar_{l-1}^T; 0] dz_l
+      GemmArgs g;
+      g.M = din + hb; g.N = dout; g.K = rows;
+      g.A0 = at<T>(p.o_AT[l]); g.lda0 = p.ldR;
+      g.A1 = l > 0 ? at<T>(p.o_DABT[l - 1]) : nullptr; g.lda1 = p.ldR;
+      g.B0 = at<T>(p.o_ZBT); g.ldb0 = p.ldR;
+      g.B1 = at<T>(p.o_SZT[l]); g.ldb1 = p.ldR;
+      g.terms = mf::T_C0_A0B0 | (l > 0 ? mf::T_C0_A1B1 : 0u);
+      g.C0 = Hv + h->woff[l]; g.ldc0 = dout;
+      gemm(g);
+      if (l == 0) break;
+      // abar_{l-1} = zbar_l W_l^T + dz_l V_l^T
+      GemmArgs d;
+      d.M = rows; d.N = din; d.K = dout;
+      d.A0 = at<T>(p.o_ZB); d.lda0 = ld8(dout);
+      d.A1 = at<T>(p.o_SZ[l]); d.lda1 = ld8(dout);
+      d.B0 = at<T>(p.o_Wb[l]); d.ldb0 = ld8(dout);
+      d.B1 = at<T>(p.o_Ub[l]); d.ldb1 = ld8(dout);
+      d.terms = mf::T_C0_A0B0 | mf::T_C0_A1B1;
+      d.C0 = at<float>(p.o_AB); d.ldc0 = din;
       gemm(d);
     }
   }
@@ -522,8 +644,10 @@ mf_status validate_loop(mf_ctx* h, const mf_loop_desc* lp) {
     return fail(h, MF_ERR_INVALID_ARG, "PARAM_LOGLR and SCALAR_LOGLR are mutually exclusive");
   if (!(lp->momentum >= 0.f && lp->momentum < 1.f))
     return fail(h, MF_ERR_INVALID_ARG, "momentum must be in [0, 1)");
-  if (lp->hvp_mode != MF_HVP_MIXED_FOR)
-    return fail(h, MF_ERR_UNSUPPORTED, "only MF_HVP_MIXED_FOR is implemented");
+  if (lp->hvp_mode != MF_HVP_MIXED_FOR && lp->hvp_mode != MF_HVP_REV_REV)
+    return fail(h, MF_ERR_INVALID_ARG, "unknown hvp_mode");
+  if (lp->hvp_mode == MF_HVP_REV_REV && h->decoder)
+    return fail(h, MF_ERR_UNSUPPORTED, "reverse-over-reverse is implemented for MLP models");
   if (lp->ckpt_every != 1 && lp->ckpt_every != 0)
     return fail(h, MF_ERR_UNSUPPORTED, "only ckpt_every = 1 is implemented");
   return MF_OK;
@@ -682,11 +806,15 @@ mf_status meta_grad_run(X& ex, const mf_loop_desc* lp, const float* theta0, cons
     const float* th = ex.theta_slot(t);
     const void* x = static_cast<const char*>(inner_x) + xs * t;
     const void* y = static_cast<const char*>(inner_y) + ys * t;
-    ex.forward(B, x, th, u, true);
     const float* ew = exw ? eta + static_cast<int64_t>(t) * B : nullptr;
     float* de = exw ? d_eta + static_cast<int64_t>(t) * B : nullptr;
-    ex.loss(B, true, y, ew, nullptr, nullptr, ex.ld_buf(), de);
-    ex.backward(B, true, Hu, nullptr);
+    if (lp->hvp_mode == MF_HVP_REV_REV) {
+      ex.ror_hvp(B, x, th, u, y, ew, nullptr, Hu, nullptr, ex.ld_buf(), de);
+    } else {
+      ex.forward(B, x, th, u, true);
+      ex.loss(B, true, y, ew, nullptr, nullptr, ex.ld_buf(), de);
+      ex.backward(B, true, Hu, nullptr);
+    }
     // theta_bar_t = theta_bar_{t+1} + H u ; d eta_lr += -lr m_t theta_bar_t ;
     // u_{t-1} = mu u_t - lr theta_bar_t ; cast theta_{t-1}, u_{t-1}
     mf::LayerUpdArgs a;
@@ -732,14 +860,19 @@ mf_status rollout_run(X& ex, const mf_loop_desc* lp, const float* theta0, const 
 
 template <typename X>
 mf_status hvp_run(X& ex, int B, const float* theta, const void* x, const void* y,
-                  const float* ex_w, const float* v, float* Hv, float* tl, float* grad) {
+                  const float* ex_w, const float* v, float* Hv, float* tl, float* grad,
+                  bool ror) {
   mf_ctx* h = ex.h;
   ex.prepare();
   ex.cast_params(theta, false);
   ex.cast_params(v, true);
-  ex.forward(B, x, theta, v, true);
-  ex.loss(B, true, y, nullptr, ex_w, nullptr, tl, nullptr);
-  ex.backward(B, true, Hv, grad);
+  if (ror) {
+    ex.ror_hvp(B, x, theta, v, y, nullptr, ex_w, Hv, grad, tl, nullptr);
+  } else {
+    ex.forward(B, x, theta, v, true);
+    ex.loss(B, true, y, nullptr, ex_w, nullptr, tl, nullptr);
+    ex.backward(B, true, Hv, grad);
+  }
   MF_CUDA(h, cudaGetLastError());
   return ex.st;
 }
@@ -747,7 +880,7 @@ mf_status hvp_run(X& ex, int B, const float* theta, const void* x, const void* y
 // Plan the workspace for the handle's model, allocate it, and run f(executor).
 template <typename E, typename F>
 mf_status with_exec(mf_ctx* h, int rows, int T, int theta_slots, int m_slots, bool partials,
-                    cudaStream_t s, F&& f) {
+                    bool ror, cudaStream_t s, F&& f) {
   if (h->decoder) {
     DecPlan plan = make_dec_plan(h, h->Ly, rows, T, theta_slots, m_slots, partials);
     mf_status st = ensure_ws(h, plan.bytes, s);
@@ -755,7 +888,7 @@ mf_status with_exec(mf_ctx* h, int rows, int T, int theta_slots, int m_slots, bo
     DecExec<E> ex(h, plan, h->Ly, s);
     return f(ex);
   }
-  Plan plan = make_plan(h, rows, T, theta_slots, m_slots, partials);
+  Plan plan = make_plan(h, rows, T, theta_slots, m_slots, partials, ror);
   mf_status st = ensure_ws(h, plan.bytes, s);
   if (st != MF_OK) return st;
   Exec<E> ex(h, plan, s);
@@ -769,7 +902,8 @@ mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
                          float* d_theta0, float* outer_loss, cudaStream_t s) {
   const bool lr_meta = lp->meta_kind & (MF_META_PARAM_LOGLR | MF_META_SCALAR_LOGLR);
   return with_exec<E>(h, std::max(lp->B, lp->B_outer), lp->T, lp->T + 1, lr_meta ? lp->T : 0,
-                      lp->meta_kind & MF_META_SCALAR_LOGLR, s, [&](auto& ex) {
+                      lp->meta_kind & MF_META_SCALAR_LOGLR, lp->hvp_mode == MF_HVP_REV_REV, s,
+                      [&](auto& ex) {
                         return meta_grad_run(ex, lp, theta0, eta, inner_x, inner_y, outer_x,
                                              outer_y, d_eta, d_theta0, outer_loss);
                       });
@@ -779,7 +913,7 @@ template <typename E>
 mf_status rollout_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0, const float* eta,
                        const void* inner_x, const void* inner_y, float* thetaT, cudaStream_t s) {
   const bool lr_meta = lp->meta_kind & (MF_META_PARAM_LOGLR | MF_META_SCALAR_LOGLR);
-  return with_exec<E>(h, lp->B, lp->T, 2, lr_meta ? 1 : 0, false, s, [&](auto& ex) {
+  return with_exec<E>(h, lp->B, lp->T, 2, lr_meta ? 1 : 0, false, false, s, [&](auto& ex) {
     return rollout_run(ex, lp, theta0, eta, inner_x, inner_y, thetaT);
   });
 }
@@ -787,9 +921,9 @@ mf_status rollout_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0, c
 template <typename E>
 mf_status hvp_impl(mf_ctx* h, int B, const float* theta, const void* x, const void* y,
                    const float* ex_w, const float* v, float* Hv, float* tl, float* grad,
-                   cudaStream_t s) {
-  return with_exec<E>(h, B, 1, 0, 0, false, s, [&](auto& ex) {
-    return hvp_run(ex, B, theta, x, y, ex_w, v, Hv, tl, grad);
+                   bool ror, cudaStream_t s) {
+  return with_exec<E>(h, B, 1, 0, 0, false, ror, s, [&](auto& ex) {
+    return hvp_run(ex, B, theta, x, y, ex_w, v, Hv, tl, grad, ror);
   });
 }
 
@@ -917,7 +1051,7 @@ mf_status mf_workspace_bytes(mf_handle h, const mf_loop_desc* lp, size_t* bytes)
     return MF_OK;
   }
   *bytes = make_plan(h, std::max(lp->B, lp->B_outer), lp->T, lp->T + 1, lr_meta ? lp->T : 0,
-                     lp->meta_kind & MF_META_SCALAR_LOGLR).bytes;
+                     lp->meta_kind & MF_META_SCALAR_LOGLR, lp->hvp_mode == MF_HVP_REV_REV).bytes;
   return MF_OK;
 }
 
@@ -958,22 +1092,27 @@ mf_status mf_hvp(mf_handle h, int B, const float* theta, const void* x, const vo
                  int hvp_mode, void* stream) {
   if (!h) return MF_ERR_INVALID_ARG;
   if (B < 1) return fail(h, MF_ERR_INVALID_ARG, "B must be >= 1");
-  if (hvp_mode != MF_HVP_MIXED_FOR) return fail(h, MF_ERR_UNSUPPORTED, "only MF_HVP_MIXED_FOR is implemented");
+  if (hvp_mode != MF_HVP_MIXED_FOR && hvp_mode != MF_HVP_REV_REV)
+    return fail(h, MF_ERR_INVALID_ARG, "unknown hvp_mode");
+  if (hvp_mode == MF_HVP_REV_REV && h->decoder)
+    return fail(h, MF_ERR_UNSUPPORTED, "reverse-over-reverse is implemented for MLP models");
+  const bool ror = hvp_mode == MF_HVP_REV_REV;
   if (!theta || !x || !y || !v || !Hv) return fail(h, MF_ERR_INVALID_ARG, "NULL tensor argument");
   mf_status st = check_x(h, x, B);
   if (st != MF_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   h->last_stream = s;
   uint64_t key = 0x687670ULL;
-  for (uint64_t v2 : {static_cast<uint64_t>(B), reinterpret_cast<uint64_t>(theta),
+  for (uint64_t v2 : {static_cast<uint64_t>(B), static_cast<uint64_t>(hvp_mode),
+                      reinterpret_cast<uint64_t>(theta),
                       reinterpret_cast<uint64_t>(x), reinterpret_cast<uint64_t>(y),
                       reinterpret_cast<uint64_t>(ex_w), reinterpret_cast<uint64_t>(v),
                       reinterpret_cast<uint64_t>(Hv), reinterpret_cast<uint64_t>(tangent_losses),
                       reinterpret_cast<uint64_t>(grad)})
     key = mix_key(key, v2);
   return run_graphed(h, h->g_hvp, key, s, [&](cudaStream_t st) {
-    return h->bf16 ? hvp_impl<__nv_bfloat16>(h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, st)
-                   : hvp_impl<float>(h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, st);
+    return h->bf16 ? hvp_impl<__nv_bfloat16>(h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, ror, st)
+                   : hvp_impl<float>(h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, ror, st);
   });
 }
 
@@ -997,6 +1136,7 @@ mf_status mf_meta_grad(mf_handle h, const mf_loop_desc* lp, const float* theta0,
   uint64_t key = 0x6d657461ULL;
   for (uint64_t v : {static_cast<uint64_t>(lp->T), static_cast<uint64_t>(lp->B),
                      static_cast<uint64_t>(lp->B_outer), static_cast<uint64_t>(lp->meta_kind),
+                     static_cast<uint64_t>(lp->hvp_mode),
                      static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->alpha)),
                      static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->momentum)),
                      reinterpret_cast<uint64_t>(theta0), reinterpret_cast<uint64_t>(eta),
@@ -1100,8 +1240,8 @@ mf_status mf_dual_gemm_bf16(int M, int N, int K, const void* A0, int lda0, const
                             int lda1, const void* B0, int ldb0, const void* B1, int ldb1,
                             float* C0, int ldc0, const float* bias0, float* C1, int ldc1,
                             const float* bias1, unsigned terms, void* stream) {
-  if (M < 1 || N < 1 || K < 1 || (terms & ~31u) || !(terms & 31u)) return MF_ERR_INVALID_ARG;
-  const bool acc0 = terms & (mf::T_C0_A0B0 | mf::T_C0_A1B0 | mf::T_C0_A0B1);
+  if (M < 1 || N < 1 || K < 1 || (terms & ~mf::T_ALL) || !(terms & mf::T_ALL)) return MF_ERR_INVALID_ARG;
+  const bool acc0 = terms & (mf::T_C0_A0B0 | mf::T_C0_A1B0 | mf::T_C0_A0B1 | mf::T_C0_A1B1);
   const bool acc1 = terms & (mf::T_C1_A1B0 | mf::T_C1_A0B1);
   if ((acc0 && (!C0 || ldc0 < N)) || (acc1 && (!C1 || ldc1 < N))) return MF_ERR_INVALID_ARG;
   GemmArgs g;
@@ -1204,8 +1344,8 @@ extern "C" mf_status mf_hvp_noalloc(const mf_model_desc* d, int B, const float* 
   h.ws = static_cast<char*>(scratch) + kNoAllocStatusBytes;
   h.ws_bytes = kNoAllocScratchBytes - kNoAllocStatusBytes;
   const mf_status st =
-      h.bf16 ? hvp_impl<__nv_bfloat16>(&h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, s)
-             : hvp_impl<float>(&h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, s);
+      h.bf16 ? hvp_impl<__nv_bfloat16>(&h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, false, s)
+             : hvp_impl<float>(&h, B, theta, x, y, ex_w, v, Hv, tangent_losses, grad, false, s);
   h.ws = nullptr;   // not owned: never released
   return st;
 }

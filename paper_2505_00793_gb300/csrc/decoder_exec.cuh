@@ -640,4 +640,11 @@ struct DecExec {
     launched();
     chk("decoder backward");
   }
+
+  // Reverse-over-reverse is built for MLP models only; the entry points reject it for the
+  // decoder before an executor exists, so this is never reached.
+  void ror_hvp(int, const void*, const float*, const float*, const void*, const float*,
+               const float*, float*, float*, float*, float*) {
+    st = MF_ERR_UNSUPPORTED;
+  }
 };

@@ -12,10 +12,12 @@ enum : int { DEV_OK = 0, DEV_NONFINITE = 5, DEV_TIMEOUT = 6 };
 
 // GEMM product terms (same bit meaning as mf_dual_gemm_bf16's `terms`).
 enum : unsigned {
-  T_C0_A0B0 = 1u, T_C0_A1B0 = 2u, T_C0_A0B1 = 4u, T_C1_A1B0 = 8u, T_C1_A0B1 = 16u
+  T_C0_A0B0 = 1u, T_C0_A1B0 = 2u, T_C0_A0B1 = 4u, T_C1_A1B0 = 8u, T_C1_A0B1 = 16u,
+  T_C0_A1B1 = 32u
 };
+constexpr unsigned T_ALL = 63u;
 
-inline int term_count(unsigned t) { return __builtin_popcount(t & 31u); }
+inline int term_count(unsigned t) { return __builtin_popcount(t & T_ALL); }
 
 enum Act : int { ACT_IDENT = 0, ACT_TANH = 1, ACT_GELU = 2, ACT_SILU = 3 };
 enum EpiMode : int { EPI_STORE = 0, EPI_ACT_FWD = 1, EPI_ACT_BWD = 2 };
@@ -134,6 +136,15 @@ template <typename T>
 void layer_update(const LayerTable& tab, const LayerUpdArgs& a, cudaStream_t s);
 
 void fill(float* p, int64_t n, float v, cudaStream_t s);
+
+// Reverse-over-reverse element kernels (MLP): dabar = dzbar phi'(z), zpart = dzbar phi''(z) da;
+// zbar = zpart + abar phi'(z).  T outputs row-major and transposed.
+template <typename T>
+void ror_fwd_elem(int act, const float* dzbar, const float* Z, const float* dA, int rows, int cols,
+                  T* dab, int ld, T* dabT, int ldT, float* zpart, cudaStream_t s);
+template <typename T>
+void ror_bwd_elem(int act, const float* zpart, const float* abar, const float* Z, int rows,
+                  int cols, T* zb, int ld, T* zbT, int ldT, cudaStream_t s);
 
 // ---- decoder-only transformer kernels (decoder_kernels.cu) ------------------------------
 void dec_embed_fwd(int N, int S, int d, int V, const int* ids, const float* E, const float* UE,

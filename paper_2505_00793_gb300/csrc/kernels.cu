@@ -227,6 +227,64 @@ __global__ void __launch_bounds__(TILE * TROWS) layer_update_kernel(const LayerT
   }
 }
 
+// Reverse-over-reverse, forward layer order: from dzbar (the adjoint of the backward's dz):
+//   dabar = dzbar phi'(z)  (T, row-major and transposed),  zpart = dzbar phi''(z) da.
+template <typename T>
+__global__ void ror_fwd_elem_kernel(int act, const float* __restrict__ dzbar,
+                                    const float* __restrict__ Z, const float* __restrict__ dA,
+                                    int rows, int cols, T* __restrict__ dab, int ld,
+                                    T* __restrict__ dabT, int ldT, float* __restrict__ zpart) {
+  __shared__ float tile[TILE][TILE + 1];
+  const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
+  const int tx = threadIdx.x, ty = threadIdx.y;
+  for (int i = ty; i < TILE; i += TROWS) {
+    const int r = r0 + i, c = c0 + tx;
+    float v = 0.f;
+    if (r < rows && c < cols) {
+      const int64_t o = static_cast<int64_t>(r) * cols + c;
+      float f, d1, d2;
+      act_eval(act, Z[o], f, d1, d2);
+      v = dzbar[o] * d1;
+      zpart[o] = dzbar[o] * d2 * dA[o];
+      dab[static_cast<int64_t>(r) * ld + c] = to_t<T>(v);
+    }
+    tile[i][tx] = v;
+  }
+  __syncthreads();
+  for (int i = ty; i < TILE; i += TROWS) {
+    const int c = c0 + i, r = r0 + tx;
+    if (c < cols && r < rows) dabT[static_cast<int64_t>(c) * ldT + r] = to_t<T>(tile[tx][i]);
+  }
+}
+
+// Reverse-over-reverse, reverse layer order:  zbar = zpart + abar phi'(z)  (T, both layouts).
+template <typename T>
+__global__ void ror_bwd_elem_kernel(int act, const float* __restrict__ zpart,
+                                    const float* __restrict__ abar, const float* __restrict__ Z,
+                                    int rows, int cols, T* __restrict__ zb, int ld,
+                                    T* __restrict__ zbT, int ldT) {
+  __shared__ float tile[TILE][TILE + 1];
+  const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
+  const int tx = threadIdx.x, ty = threadIdx.y;
+  for (int i = ty; i < TILE; i += TROWS) {
+    const int r = r0 + i, c = c0 + tx;
+    float v = 0.f;
+    if (r < rows && c < cols) {
+      const int64_t o = static_cast<int64_t>(r) * cols + c;
+      float f, d1, d2;
+      act_eval(act, Z[o], f, d1, d2);
+      v = zpart[o] + abar[o] * d1;
+      zb[static_cast<int64_t>(r) * ld + c] = to_t<T>(v);
+    }
+    tile[i][tx] = v;
+  }
+  __syncthreads();
+  for (int i = ty; i < TILE; i += TROWS) {
+    const int c = c0 + i, r = r0 + tx;
+    if (c < cols && r < rows) zbT[static_cast<int64_t>(c) * ldT + r] = to_t<T>(tile[tx][i]);
+  }
+}
+
 __global__ void fill_kernel(float* p, int64_t n, float v) {
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x)
@@ -267,6 +325,24 @@ void layer_update(const LayerTable& tab, const LayerUpdArgs& a, cudaStream_t s) 
   layer_update_kernel<T><<<blocks, dim3(TILE, TROWS), 0, s>>>(tab, a);
 }
 
+template <typename T>
+void ror_fwd_elem(int act, const float* dzbar, const float* Z, const float* dA, int rows, int cols,
+                  T* dab, int ld, T* dabT, int ldT, float* zpart, cudaStream_t s) {
+  if (rows <= 0 || cols <= 0) return;
+  dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE);
+  ror_fwd_elem_kernel<T><<<grid, dim3(TILE, TROWS), 0, s>>>(act, dzbar, Z, dA, rows, cols, dab, ld,
+                                                             dabT, ldT, zpart);
+}
+
+template <typename T>
+void ror_bwd_elem(int act, const float* zpart, const float* abar, const float* Z, int rows,
+                  int cols, T* zb, int ld, T* zbT, int ldT, cudaStream_t s) {
+  if (rows <= 0 || cols <= 0) return;
+  dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE);
+  ror_bwd_elem_kernel<T><<<grid, dim3(TILE, TROWS), 0, s>>>(act, zpart, abar, Z, rows, cols, zb, ld,
+                                                             zbT, ldT);
+}
+
 void fill(float* p, int64_t n, float v, cudaStream_t s) {
   if (n <= 0) return;
   int64_t b = (n + 255) / 256;
@@ -278,7 +354,11 @@ void fill(float* p, int64_t n, float v, cudaStream_t s) {
   template void transpose<T>(const T*, int, int, int, T*, int, cudaStream_t);     \
   template void fill_rows<T>(const RowFill&, int, cudaStream_t);                  \
   template void loss_seed<T>(const LossArgs&, cudaStream_t);                      \
-  template void layer_update<T>(const LayerTable&, const LayerUpdArgs&, cudaStream_t);
+  template void layer_update<T>(const LayerTable&, const LayerUpdArgs&, cudaStream_t);        \
+  template void ror_fwd_elem<T>(int, const float*, const float*, const float*, int, int, T*, int, \
+                                T*, int, float*, cudaStream_t);                                   \
+  template void ror_bwd_elem<T>(int, const float*, const float*, const float*, int, int, T*, int,  \
+                                T*, int, cudaStream_t);
 MF_INST(float)
 MF_INST(__nv_bfloat16)
 #undef MF_INST

@@ -35,11 +35,11 @@ __global__ void __launch_bounds__(256) simt_dual_gemm_kernel(SimtParams p) {
   __shared__ float Bs[TK][TN + 1];
   const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
   const int m0 = blockIdx.y * TM, n0 = blockIdx.x * TN;
-  const int tacc[5] = {0, 0, 0, 1, 1};
-  const int ta[5] = {0, 1, 0, 1, 0};
-  const int tb[5] = {0, 0, 1, 0, 1};
+  const int tacc[6] = {0, 0, 0, 1, 1, 0};
+  const int ta[6] = {0, 1, 0, 1, 0, 1};
+  const int tb[6] = {0, 0, 1, 0, 1, 1};
   float c[2][4][4] = {};
-  for (int t = 0; t < 5; ++t) {
+  for (int t = 0; t < 6; ++t) {
     if (!(p.terms & (1u << t))) continue;
     const int acc = tacc[t];
     const float* A = p.A[ta[t]];

@@ -24,14 +24,14 @@ namespace mf {
 cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why) {
   static const char* dummy;
   if (!why) why = &dummy;
-  if (a.M <= 0 || a.N <= 0 || a.K <= 0 || (a.terms & 31u) == 0) {
+  if (a.M <= 0 || a.N <= 0 || a.K <= 0 || (a.terms & T_ALL) == 0 || (a.terms & ~T_ALL)) {
     *why = "empty GEMM";
     return cudaErrorInvalidValue;
   }
   const void* ptrs[4] = {a.A0, a.A1, a.B0, a.B1};
   const int lds[4] = {a.lda0, a.lda1, a.ldb0, a.ldb1};
-  const unsigned uses[4] = {T_C0_A0B0 | T_C0_A0B1 | T_C1_A0B1, T_C0_A1B0 | T_C1_A1B0,
-                            T_C0_A0B0 | T_C0_A1B0 | T_C1_A1B0, T_C0_A0B1 | T_C1_A0B1};
+  const unsigned uses[4] = {T_C0_A0B0 | T_C0_A0B1 | T_C1_A0B1, T_C0_A1B0 | T_C1_A1B0 | T_C0_A1B1,
+                            T_C0_A0B0 | T_C0_A1B0 | T_C1_A1B0, T_C0_A0B1 | T_C1_A0B1 | T_C0_A1B1};
   for (int i = 0; i < 4; ++i) {
     if (!(a.terms & uses[i])) continue;
     if (!ptrs[i] || (reinterpret_cast<uintptr_t>(ptrs[i]) & 15) || (lds[i] & 7) || lds[i] < a.K) {

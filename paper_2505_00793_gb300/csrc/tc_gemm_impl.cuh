@@ -508,6 +508,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (terms & T_C0_A0B1) { mma_bf16(d0, a0 + adv, b1 + adv, idesc, started0); started0 = true; }
             if (terms & T_C1_A1B0) { mma_bf16(d1, a1 + adv, b0 + adv, idesc, started1); started1 = true; }
             if (terms & T_C1_A0B1) { mma_bf16(d1, a0 + adv, b1 + adv, idesc, started1); started1 = true; }
+            if (terms & T_C0_A1B1) { mma_bf16(d0, a1 + adv, b1 + adv, idesc, started0); started0 = true; }
           }
         }
         mma_commit(&empty_bar[s]);
@@ -728,9 +729,9 @@ template <int BN, int KA, int MODE, int ACT>
 cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
   const unsigned t = a.terms;
   const bool useA0 = t & (T_C0_A0B0 | T_C0_A0B1 | T_C1_A0B1);
-  const bool useA1 = t & (T_C0_A1B0 | T_C1_A1B0);
+  const bool useA1 = t & (T_C0_A1B0 | T_C1_A1B0 | T_C0_A1B1);
   const bool useB0 = t & (T_C0_A0B0 | T_C0_A1B0 | T_C1_A1B0);
-  const bool useB1 = t & (T_C0_A0B1 | T_C1_A0B1);
+  const bool useB1 = t & (T_C0_A0B1 | T_C1_A0B1 | T_C0_A1B1);
   const bool dual = t & (T_C1_A1B0 | T_C1_A0B1);
   TcParams p;
   memset(&p, 0, sizeof(p));

@@ -9,14 +9,14 @@ from gpu_util import need_gpu, rel_l2
 
 SHAPES = [(128, 128, 64), (256, 1024, 1024), (256, 10, 1024), (1024, 1024, 512),
           (77, 45, 136), (130, 300, 8), (512, 4096, 256), (300, 16, 40)]
-MASKS = [1, 1 | 8 | 16, 1 | 16, 2 | 4, 4, 1 | 2 | 4 | 8 | 16]
+MASKS = [1, 1 | 8 | 16, 1 | 16, 2 | 4, 4, 1 | 2 | 4 | 8 | 16, 1 | 32, 2 | 4 | 32]
 
 
 def _ref(A0, A1, B0, B1, mask):
     a0, a1, b0, b1 = (x.double().cpu() for x in (A0, A1, B0, B1))
     c0 = None
     c1 = None
-    terms0 = [(1, a0, b0), (2, a1, b0), (4, a0, b1)]
+    terms0 = [(1, a0, b0), (2, a1, b0), (4, a0, b1), (32, a1, b1)]
     terms1 = [(8, a1, b0), (16, a0, b1)]
     for bit, a, b in terms0:
         if mask & bit:
