@@ -202,8 +202,15 @@ mf_status mf_kernel_time(mf_handle h, double* ms, uint64_t* launches, double* fl
 /* Library options.  MF_OPT_CUDA_GRAPHS (default 1): a call of mf_meta_grad, mf_inner_rollout
  * or mf_hvp repeated with the same shapes and pointers is captured into a CUDA graph on its
  * second occurrence and replayed afterwards, on a library-owned stream that is ordered after
- * and before the caller's stream with events.  0 launches every kernel individually. */
-enum { MF_OPT_CUDA_GRAPHS = 1 };
+ * and before the caller's stream with events.  0 launches every kernel individually.
+ * MF_OPT_PDL (default 1, process-wide): kernels are launched with programmatic dependent
+ * launch, so each one's launch and prologue overlap the tail of the previous kernel on the
+ * stream (memory effects keep stream order).  0 launches them with plain stream order.
+ * Setting it drops the handle's captured graphs.
+ * MF_OPT_CONCURRENT (default 1): in each backward layer the weight product and the data
+ * product run on two streams (parallel branches of a captured graph); 0 runs them in
+ * sequence on the call's stream. */
+enum { MF_OPT_CUDA_GRAPHS = 1, MF_OPT_PDL = 2, MF_OPT_CONCURRENT = 3 };
 mf_status mf_set_option(mf_handle h, int option, int value);
 
 /* Host-side fault injection for tests: kind 1 = the next workspace allocation fails;

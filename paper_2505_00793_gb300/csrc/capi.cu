@@ -16,6 +16,7 @@
 #include "../../include/mixflow.h"
 #include "decoder_layout.h"
 #include "internal.h"
+#include "launch.cuh"
 
 using mf::GemmArgs;
 
@@ -70,6 +71,12 @@ struct mf_ctx {
   GraphCache g_meta, g_roll, g_hvp;
   cudaStream_t gstream = nullptr;
   cudaEvent_t ev_in = nullptr, ev_out = nullptr;
+  // Side stream for independent GEMMs of one backward layer (the weight product runs next
+  // to the data product); forked from and joined back into the working stream with events,
+  // which a stream capture turns into parallel graph branches.
+  cudaStream_t sstream = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  bool concurrent = true;
 };
 
 namespace {
@@ -364,8 +371,24 @@ struct Exec {
 
   void launched(int n = 1) { h->launches += n; }
 
-  void gemm(GemmArgs g) {
+  // Fork the side stream off the working stream / join it back (see mf_ctx::sstream).
+  bool can_fork() const { return h->concurrent && h->sstream && h->ev_fork && h->ev_join; }
+  void fork() {
+    if (cudaEventRecord(h->ev_fork, s) != cudaSuccess ||
+        cudaStreamWaitEvent(h->sstream, h->ev_fork, 0) != cudaSuccess) {
+      st = MF_ERR_CUDA; h->err = "stream fork failed";
+    }
+  }
+  void join() {
+    if (cudaEventRecord(h->ev_join, h->sstream) != cudaSuccess ||
+        cudaStreamWaitEvent(s, h->ev_join, 0) != cudaSuccess) {
+      st = MF_ERR_CUDA; h->err = "stream join failed";
+    }
+  }
+
+  void gemm(GemmArgs g, cudaStream_t on = nullptr) {
     if (st != MF_OK) return;
+    const cudaStream_t s = on ? on : this->s;
     g.status = h->d_status;
     cudaEvent_t e0 = nullptr, e1 = nullptr;
     unsigned ev_flags = cudaEventRecordDefault;
@@ -519,8 +542,11 @@ struct Exec {
         g.terms = mf::T_C0_A0B1 | (l > 0 ? mf::T_C0_A1B0 : 0u);
         g.C0 = out_h + h->woff[l]; g.ldc0 = dout;
       }
-      if (dual || out_g) gemm(g);
-      if (l == 0) break;
+      const bool wgemm = dual || out_g;
+      if (l == 0) {
+        if (wgemm) gemm(g);
+        break;
+      }
       // data product: da = dz W^T ; da' = dz' W^T + dz U^T ; epilogue -> dz, dz' of layer l-1
       GemmArgs d;
       d.M = rows; d.N = din; d.K = dout;
@@ -541,7 +567,18 @@ struct Exec {
       d.epi.AT = dzT_buf(l - 1);
       d.epi.AdT = dual ? at<T>(p.o_dZdT[b ^ 1]) : nullptr;
       d.epi.ldt = p.ldR;
-      gemm(d);
+      // The weight product reads layer l's seeds and writes its slice of the output; the
+      // data product reads the same seeds and writes layer l-1's (the other ping-pong set):
+      // they are independent and run side by side, joined before layer l-1 overwrites.
+      if (wgemm && can_fork()) {
+        fork();
+        gemm(g, h->sstream);
+        gemm(d);
+        join();
+      } else {
+        if (wgemm) gemm(g);
+        gemm(d);
+      }
     }
   }
 
@@ -927,6 +964,17 @@ mf_status hvp_impl(mf_ctx* h, int B, const float* theta, const void* x, const vo
   });
 }
 
+void destroy_handle_objects(mf_ctx* h) {
+  if (h->d_status) cudaFree(h->d_status);
+  if (h->gstream) cudaStreamDestroy(h->gstream);
+  if (h->sstream) cudaStreamDestroy(h->sstream);
+  for (cudaEvent_t e : {h->ev_in, h->ev_out, h->ev_fork, h->ev_join})
+    if (e) cudaEventDestroy(e);
+  h->d_status = nullptr;
+  h->gstream = h->sstream = nullptr;
+  h->ev_in = h->ev_out = h->ev_fork = h->ev_join = nullptr;
+}
+
 }  // namespace
 
 // ======================================= C ABI ============================================
@@ -997,9 +1045,12 @@ mf_status mf_create(const mf_model_desc* d, mf_handle* out) {
       cudaMemset(h->d_status, 0, sizeof(int)) != cudaSuccess ||
       cudaStreamCreateWithFlags(&h->gstream, cudaStreamNonBlocking) != cudaSuccess ||
       cudaEventCreateWithFlags(&h->ev_in, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_out, cudaEventDisableTiming) != cudaSuccess) {
+      cudaEventCreateWithFlags(&h->ev_out, cudaEventDisableTiming) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&h->sstream, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess) {
     cudaGetLastError();
-    if (h->d_status) cudaFree(h->d_status);
+    destroy_handle_objects(h);
     delete h;
     return MF_ERR_CUDA;
   }
@@ -1013,10 +1064,7 @@ mf_status mf_destroy(mf_handle h) {
   release_ws(h);
   for (auto& e : h->evs) { cudaEventDestroy(e.first); cudaEventDestroy(e.second); }
   drop_graphs(h);
-  if (h->d_status) cudaFree(h->d_status);
-  if (h->gstream) cudaStreamDestroy(h->gstream);
-  if (h->ev_in) cudaEventDestroy(h->ev_in);
-  if (h->ev_out) cudaEventDestroy(h->ev_out);
+  destroy_handle_objects(h);
   delete h;
   return MF_OK;
 }
@@ -1225,6 +1273,16 @@ mf_status mf_set_option(mf_handle h, int option, int value) {
   if (option == MF_OPT_CUDA_GRAPHS) {
     h->use_graphs = value != 0;
     if (!h->use_graphs) drop_graphs(h);
+    return MF_OK;
+  }
+  if (option == MF_OPT_PDL) {
+    mf::g_pdl = value != 0;
+    drop_graphs(h);
+    return MF_OK;
+  }
+  if (option == MF_OPT_CONCURRENT) {
+    h->concurrent = value != 0;
+    drop_graphs(h);
     return MF_OK;
   }
   return fail(h, MF_ERR_INVALID_ARG, "unknown option");

@@ -14,6 +14,7 @@
 
 #include "device_math.cuh"
 #include "internal.h"
+#include "launch.cuh"
 
 namespace mf {
 namespace {
@@ -58,6 +59,7 @@ __device__ __forceinline__ float ld_t(const __nv_bfloat16* p, int64_t i) { retur
 __global__ void embed_fwd_kernel(const int* __restrict__ ids, int S, int d, int V,
                                  const float* __restrict__ E, const float* __restrict__ UE,
                                  float* __restrict__ x, float* __restrict__ xd, int* status) {
+  pdl_entry();
   const int r = blockIdx.x;
   const int b = r / S, s = r % S;
   int id = ids[static_cast<int64_t>(b) * (S + 1) + s];
@@ -81,6 +83,7 @@ __global__ void rmsnorm_fwd_kernel(int d, float eps, const float* __restrict__ x
                                    float* __restrict__ xd_out, float* __restrict__ rr,
                                    float* __restrict__ rrd, T* __restrict__ h, T* __restrict__ hd,
                                    int ldh) {
+  pdl_entry();
   const int r = blockIdx.x;
   const int64_t o = static_cast<int64_t>(r) * d;
   const bool dual = xd_in != nullptr;
@@ -124,6 +127,7 @@ __global__ void rmsnorm_bwd_kernel(int d, const float* __restrict__ x, const flo
                                    const float* __restrict__ g, const float* __restrict__ gd,
                                    const float* __restrict__ dy, const float* __restrict__ dyd,
                                    float* __restrict__ dx, float* __restrict__ dxd) {
+  pdl_entry();
   const int r = blockIdx.x;
   const int64_t o = static_cast<int64_t>(r) * d;
   const bool dual = dyd != nullptr;
@@ -163,6 +167,7 @@ __global__ void gain_grad_kernel(int N, int d, const float* __restrict__ x,
                                  const float* __restrict__ rrd, const float* __restrict__ dy,
                                  const float* __restrict__ dyd, float* __restrict__ dg,
                                  float* __restrict__ dgd) {
+  pdl_entry();
   __shared__ float sp[32][33];
   __shared__ float spd[32][33];
   const int j = blockIdx.x * 32 + threadIdx.x;
@@ -197,6 +202,7 @@ template <typename T>
 __global__ void rope_split_kernel(int S, int H, int dh, float base, float qscale,
                                   const float* __restrict__ qkv, T* __restrict__ Q,
                                   T* __restrict__ K, T* __restrict__ Vv) {
+  pdl_entry();
   const int r = blockIdx.x;                 // token row
   const int b = r / S, s = r % S;
   const int d = H * dh, half = dh / 2;
@@ -224,6 +230,7 @@ template <typename T>
 __global__ void rope_merge_kernel(int S, int H, int dh, float base, float qscale,
                                   const float* __restrict__ dQ, const float* __restrict__ dK,
                                   const float* __restrict__ dV, T* __restrict__ out, int ldo) {
+  pdl_entry();
   const int r = blockIdx.x;
   const int b = r / S, s = r % S;
   const int d = H * dh, half = dh / 2;
@@ -248,6 +255,7 @@ __global__ void rope_merge_kernel(int S, int H, int dh, float base, float qscale
 template <typename T>
 __global__ void head_merge_kernel(int S, int H, int dh, const float* __restrict__ O,
                                   T* __restrict__ out, int ldo) {
+  pdl_entry();
   const int r = blockIdx.x;
   const int b = r / S, s = r % S;
   const int d = H * dh;
@@ -262,6 +270,7 @@ __global__ void head_merge_kernel(int S, int H, int dh, const float* __restrict_
 template <typename T>
 __global__ void head_split_kernel(int S, int H, int dh, const float* __restrict__ X,
                                   T* __restrict__ out) {
+  pdl_entry();
   const int r = blockIdx.x;
   const int b = r / S, s = r % S;
   const int d = H * dh;
@@ -278,6 +287,7 @@ template <typename T>
 __global__ void softmax_fwd_kernel(int S, int rows, const float* __restrict__ Sc,
                                    const float* __restrict__ Scd, T* __restrict__ P,
                                    T* __restrict__ Pd) {
+  pdl_entry();
   const int warps = blockDim.x >> 5;
   const int row = blockIdx.x * warps + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -315,6 +325,7 @@ __global__ void softmax_bwd_kernel(int S, int rows, const T* __restrict__ P,
                                    const T* __restrict__ Pd, const float* __restrict__ dP,
                                    const float* __restrict__ dPd, T* __restrict__ dS,
                                    T* __restrict__ dSd) {
+  pdl_entry();
   const int warps = blockDim.x >> 5;
   const int row = blockIdx.x * warps + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -343,6 +354,7 @@ __global__ void ce_stats_kernel(int S, int V, const int* __restrict__ ids,
                                 const float* __restrict__ F, const float* __restrict__ Fd,
                                 float* __restrict__ lse, float* __restrict__ l,
                                 float* __restrict__ pf, float* __restrict__ ld, int* status) {
+  pdl_entry();
   const int r = blockIdx.x;
   const int b = r / S, s = r % S;
   int y = ids[static_cast<int64_t>(b) * (S + 1) + s + 1];
@@ -394,6 +406,7 @@ __global__ void ce_seed_kernel(int S, int V, const int* __restrict__ ids,
                                const float* __restrict__ lse, const float* __restrict__ pf,
                                const float* __restrict__ eta_w, const float* __restrict__ ex_w,
                                float inv_norm, T* __restrict__ dF, T* __restrict__ dFd, int ldo) {
+  pdl_entry();
   const int r = blockIdx.y;
   const int b = r / S, s = r % S;
   const int y = ids[static_cast<int64_t>(b) * (S + 1) + s + 1];
@@ -417,6 +430,7 @@ __global__ void seq_reduce_kernel(int B, int S, const float* __restrict__ l,
                                   const float* __restrict__ ld, const float* __restrict__ eta_w,
                                   float invB, float* __restrict__ l_seq, float* __restrict__ ld_seq,
                                   float* __restrict__ d_eta) {
+  pdl_entry();
   const int warps = blockDim.x >> 5;
   const int b = blockIdx.x * warps + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -441,6 +455,7 @@ __global__ void seq_reduce_kernel(int B, int S, const float* __restrict__ l,
 // ---- deterministic embedding scatter-add --------------------------------------------------
 __global__ void token_count_kernel(int N, int S, int V, const int* __restrict__ ids,
                                    int* __restrict__ count) {
+  pdl_entry();
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= N) return;
   int id = ids[static_cast<int64_t>(r / S) * (S + 1) + r % S];
@@ -450,6 +465,7 @@ __global__ void token_count_kernel(int N, int S, int V, const int* __restrict__ 
 
 // Exclusive scan of count[0..V) into start[0..V] (one block).
 __global__ void scan_kernel(int V, const int* __restrict__ count, int* __restrict__ start) {
+  pdl_entry();
   __shared__ int part[1024];
   const int per = (V + blockDim.x - 1) / blockDim.x;
   const int b0 = threadIdx.x * per;
@@ -477,6 +493,7 @@ __global__ void scan_kernel(int V, const int* __restrict__ count, int* __restric
 // Stable placement: token r goes to start[id] + (number of earlier tokens with the same id).
 __global__ void token_place_kernel(int N, int S, int V, const int* __restrict__ ids,
                                    const int* __restrict__ start, int* __restrict__ order) {
+  pdl_entry();
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= N) return;
   auto id_of = [&](int t) {
@@ -494,6 +511,7 @@ __global__ void embed_bwd_kernel(int d, const int* __restrict__ start,
                                  const int* __restrict__ order, const float* __restrict__ dx,
                                  const float* __restrict__ dxd, float* __restrict__ dE,
                                  float* __restrict__ dEd) {
+  pdl_entry();
   const int v = blockIdx.x;
   const int a = start[v], e = start[v + 1];
   for (int j = threadIdx.x; j < d; j += blockDim.x) {
@@ -514,6 +532,7 @@ constexpr int TILE = 32, TROWS = 8;
 template <typename TI, typename TO>
 __global__ void transpose_b_kernel(const TI* __restrict__ X, int rows, int cols, int ld,
                                    int64_t bsX, TO* __restrict__ XT, int ldT, int64_t bsT) {
+  pdl_entry();
   __shared__ float tile[TILE][TILE + 1];
   const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
   X += blockIdx.z * bsX;
@@ -534,6 +553,7 @@ __global__ void transpose_b_kernel(const TI* __restrict__ X, int rows, int cols,
 template <typename T>
 __global__ void cast_rows_kernel(const float* __restrict__ X, int rows, int cols, T* __restrict__ Y,
                                  int ldy) {
+  pdl_entry();
   const int64_t n = static_cast<int64_t>(rows) * cols;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -553,14 +573,14 @@ int blocks_for(int64_t n) {
 // ---- launchers -------------------------------------------------------------------------------
 void dec_embed_fwd(int N, int S, int d, int V, const int* ids, const float* E, const float* UE,
                    float* x, float* xd, int* status, cudaStream_t s) {
-  embed_fwd_kernel<<<N, 256, 0, s>>>(ids, S, d, V, E, UE, x, xd, status);
+  launch_k(embed_fwd_kernel, dim3(N), dim3(256), 0, s, ids, S, d, V, E, UE, x, xd, status);
 }
 
 template <typename T>
 void dec_rmsnorm_fwd(int N, int d, float eps, const float* x_in, const float* y, const float* xd_in,
                      const float* yd, const float* g, const float* gd, float* x_out, float* xd_out,
                      float* r, float* rd, T* h, T* hd, int ldh, cudaStream_t s) {
-  rmsnorm_fwd_kernel<T><<<N, 256, 0, s>>>(d, eps, x_in, y, xd_in, yd, g, gd, x_out, xd_out, r, rd,
+  launch_k(rmsnorm_fwd_kernel<T>, dim3(N), dim3(256), 0, s, d, eps, x_in, y, xd_in, yd, g, gd, x_out, xd_out, r, rd,
                                           h, hd, ldh);
 }
 
@@ -568,51 +588,51 @@ template <typename T>
 void dec_rmsnorm_bwd(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
                      const float* g, const float* gd, const float* dy, const float* dyd, float* dx,
                      float* dxd, cudaStream_t s) {
-  rmsnorm_bwd_kernel<T><<<N, 256, 0, s>>>(d, x, xd, r, rd, g, gd, dy, dyd, dx, dxd);
+  launch_k(rmsnorm_bwd_kernel<T>, dim3(N), dim3(256), 0, s, d, x, xd, r, rd, g, gd, dy, dyd, dx, dxd);
 }
 
 void dec_gain_grad(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
                    const float* dy, const float* dyd, float* dg, float* dgd, cudaStream_t s) {
-  gain_grad_kernel<<<(d + 31) / 32, dim3(32, 32), 0, s>>>(N, d, x, xd, r, rd, dy, dyd, dg, dgd);
+  launch_k(gain_grad_kernel, dim3((d + 31) / 32), dim3(dim3(32, 32)), 0, s, N, d, x, xd, r, rd, dy, dyd, dg, dgd);
 }
 
 template <typename T>
 void dec_rope_split(int N, int S, int H, int dh, float base, float qscale, const float* qkv, T* Q,
                     T* K, T* V, cudaStream_t s) {
-  rope_split_kernel<T><<<N, 256, 0, s>>>(S, H, dh, base, qscale, qkv, Q, K, V);
+  launch_k(rope_split_kernel<T>, dim3(N), dim3(256), 0, s, S, H, dh, base, qscale, qkv, Q, K, V);
 }
 
 template <typename T>
 void dec_rope_merge(int N, int S, int H, int dh, float base, float qscale, const float* dQ,
                     const float* dK, const float* dV, T* out, int ldo, cudaStream_t s) {
-  rope_merge_kernel<T><<<N, 256, 0, s>>>(S, H, dh, base, qscale, dQ, dK, dV, out, ldo);
+  launch_k(rope_merge_kernel<T>, dim3(N), dim3(256), 0, s, S, H, dh, base, qscale, dQ, dK, dV, out, ldo);
 }
 
 template <typename T>
 void dec_head_merge(int N, int S, int H, int dh, const float* O, T* out, int ldo, cudaStream_t s) {
-  head_merge_kernel<T><<<N, 256, 0, s>>>(S, H, dh, O, out, ldo);
+  launch_k(head_merge_kernel<T>, dim3(N), dim3(256), 0, s, S, H, dh, O, out, ldo);
 }
 
 template <typename T>
 void dec_head_split(int N, int S, int H, int dh, const float* X, T* out, cudaStream_t s) {
-  head_split_kernel<T><<<N, 256, 0, s>>>(S, H, dh, X, out);
+  launch_k(head_split_kernel<T>, dim3(N), dim3(256), 0, s, S, H, dh, X, out);
 }
 
 template <typename T>
 void dec_softmax_fwd(int S, int rows, const float* Sc, const float* Scd, T* P, T* Pd,
                      cudaStream_t s) {
-  softmax_fwd_kernel<T><<<(rows + 7) / 8, 256, 0, s>>>(S, rows, Sc, Scd, P, Pd);
+  launch_k(softmax_fwd_kernel<T>, dim3((rows + 7) / 8), dim3(256), 0, s, S, rows, Sc, Scd, P, Pd);
 }
 
 template <typename T>
 void dec_softmax_bwd(int S, int rows, const T* P, const T* Pd, const float* dP, const float* dPd,
                      T* dS, T* dSd, cudaStream_t s) {
-  softmax_bwd_kernel<T><<<(rows + 7) / 8, 256, 0, s>>>(S, rows, P, Pd, dP, dPd, dS, dSd);
+  launch_k(softmax_bwd_kernel<T>, dim3((rows + 7) / 8), dim3(256), 0, s, S, rows, P, Pd, dP, dPd, dS, dSd);
 }
 
 void dec_ce_stats(int N, int S, int V, const int* ids, const float* F, const float* Fd, float* lse,
                   float* l, float* pf, float* ld, int* status, cudaStream_t s) {
-  ce_stats_kernel<<<N, 512, 0, s>>>(S, V, ids, F, Fd, lse, l, pf, ld, status);
+  launch_k(ce_stats_kernel, dim3(N), dim3(512), 0, s, S, V, ids, F, Fd, lse, l, pf, ld, status);
 }
 
 template <typename T>
@@ -620,26 +640,26 @@ void dec_ce_seed(int N, int S, int V, const int* ids, const float* F, const floa
                  const float* lse, const float* pf, const float* eta_w, const float* ex_w,
                  float inv_norm, T* dF, T* dFd, int ldo, cudaStream_t s) {
   dim3 grid((V + 255) / 256 > 16 ? 16 : (V + 255) / 256, N);
-  ce_seed_kernel<T><<<grid, 256, 0, s>>>(S, V, ids, F, Fd, lse, pf, eta_w, ex_w, inv_norm, dF, dFd,
+  launch_k(ce_seed_kernel<T>, dim3(grid), dim3(256), 0, s, S, V, ids, F, Fd, lse, pf, eta_w, ex_w, inv_norm, dF, dFd,
                                          ldo);
 }
 
 void dec_seq_reduce(int B, int S, const float* l, const float* ld, const float* eta_w, float invB,
                     float* l_seq, float* ld_seq, float* d_eta, cudaStream_t s) {
-  seq_reduce_kernel<<<(B + 7) / 8, 256, 0, s>>>(B, S, l, ld, eta_w, invB, l_seq, ld_seq, d_eta);
+  launch_k(seq_reduce_kernel, dim3((B + 7) / 8), dim3(256), 0, s, B, S, l, ld, eta_w, invB, l_seq, ld_seq, d_eta);
 }
 
 void dec_token_csr(int N, int S, int V, const int* ids, int* count, int* start, int* order,
                    cudaStream_t s) {
   cudaMemsetAsync(count, 0, sizeof(int) * V, s);
-  token_count_kernel<<<(N + 255) / 256, 256, 0, s>>>(N, S, V, ids, count);
-  scan_kernel<<<1, 1024, 0, s>>>(V, count, start);
-  token_place_kernel<<<(N + 255) / 256, 256, 0, s>>>(N, S, V, ids, start, order);
+  launch_k(token_count_kernel, dim3((N + 255) / 256), dim3(256), 0, s, N, S, V, ids, count);
+  launch_k(scan_kernel, dim3(1), dim3(1024), 0, s, V, count, start);
+  launch_k(token_place_kernel, dim3((N + 255) / 256), dim3(256), 0, s, N, S, V, ids, start, order);
 }
 
 void dec_embed_bwd(int V, int d, const int* start, const int* order, const float* dx,
                    const float* dxd, float* dE, float* dEd, cudaStream_t s) {
-  embed_bwd_kernel<<<V, 256, 0, s>>>(d, start, order, dx, dxd, dE, dEd);
+  launch_k(embed_bwd_kernel, dim3(V), dim3(256), 0, s, d, start, order, dx, dxd, dE, dEd);
 }
 
 template <typename TI, typename TO>
@@ -647,12 +667,12 @@ void transpose_batched(const TI* X, int rows, int cols, int ld, int64_t bsX, TO*
                        int64_t bsT, int batch, cudaStream_t s) {
   if (rows <= 0 || cols <= 0 || batch <= 0) return;
   dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE, batch);
-  transpose_b_kernel<TI, TO><<<grid, dim3(TILE, TROWS), 0, s>>>(X, rows, cols, ld, bsX, XT, ldT, bsT);
+  launch_k(transpose_b_kernel<TI, TO>, dim3(grid), dim3(TILE, TROWS), 0, s, X, rows, cols, ld, bsX, XT, ldT, bsT);
 }
 
 template <typename T>
 void cast_rows(const float* X, int rows, int cols, T* Y, int ldy, cudaStream_t s) {
-  cast_rows_kernel<T><<<blocks_for(static_cast<int64_t>(rows) * cols), 256, 0, s>>>(X, rows, cols, Y, ldy);
+  launch_k(cast_rows_kernel<T>, dim3(blocks_for(static_cast<int64_t>(rows) * cols)), dim3(256), 0, s, X, rows, cols, Y, ldy);
 }
 
 #define MF_DEC_INST(T)                                                                            \

@@ -14,8 +14,11 @@
 
 #include "device_math.cuh"
 #include "internal.h"
+#include "launch.cuh"
 
 namespace mf {
+
+int g_pdl = 1;
 namespace {
 
 constexpr int TILE = 32, TROWS = 8;
@@ -23,6 +26,7 @@ constexpr int TILE = 32, TROWS = 8;
 template <typename T>
 __global__ void transpose_kernel(const T* __restrict__ X, int rows, int cols, int ld,
                                  T* __restrict__ XT, int ldT) {
+  pdl_entry();
   __shared__ T tile[TILE][TILE + 1];
   const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
   const int tx = threadIdx.x, ty = threadIdx.y;
@@ -39,6 +43,7 @@ __global__ void transpose_kernel(const T* __restrict__ X, int rows, int cols, in
 
 template <typename T>
 __global__ void fill_rows_kernel(const RowFill f, int cols) {
+  pdl_entry();
   const int k = blockIdx.y;
   const int c = blockIdx.x * blockDim.x + threadIdx.x;
   if (k >= f.n || c >= cols) return;
@@ -61,6 +66,7 @@ __device__ __forceinline__ float warp_max(float v) {
 // l = logsumexp(f) - f_y.  Seeds scaled by w_b / B.
 template <typename T>
 __global__ void loss_seed_kernel(const LossArgs a) {
+  pdl_entry();
   const int warps = blockDim.x >> 5;
   const int row = blockIdx.x * warps + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -124,6 +130,7 @@ __global__ void loss_seed_kernel(const LossArgs a) {
 
 __global__ void sum_scaled_kernel(const float* __restrict__ x, int n, float scale,
                                   float* __restrict__ out) {
+  pdl_entry();
   __shared__ float red[32];
   float s = 0.f;
   for (int i = threadIdx.x; i < n; i += blockDim.x) s += x[i];
@@ -147,6 +154,7 @@ __device__ __forceinline__ float lr_at(const LrArgs& lr, int64_t i) {
 template <typename T>
 __global__ void __launch_bounds__(TILE * TROWS) layer_update_kernel(const LayerTable tab,
                                                                     const LayerUpdArgs a) {
+  pdl_entry();
   __shared__ float tw[TILE][TILE + 1];   // values cast into W / WT
   __shared__ float tu[TILE][TILE + 1];   // values cast into U / UT
   __shared__ float red[TILE * TROWS / 32];
@@ -234,6 +242,7 @@ __global__ void ror_fwd_elem_kernel(int act, const float* __restrict__ dzbar,
                                     const float* __restrict__ Z, const float* __restrict__ dA,
                                     int rows, int cols, T* __restrict__ dab, int ld,
                                     T* __restrict__ dabT, int ldT, float* __restrict__ zpart) {
+  pdl_entry();
   __shared__ float tile[TILE][TILE + 1];
   const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
   const int tx = threadIdx.x, ty = threadIdx.y;
@@ -263,6 +272,7 @@ __global__ void ror_bwd_elem_kernel(int act, const float* __restrict__ zpart,
                                     const float* __restrict__ abar, const float* __restrict__ Z,
                                     int rows, int cols, T* __restrict__ zb, int ld,
                                     T* __restrict__ zbT, int ldT) {
+  pdl_entry();
   __shared__ float tile[TILE][TILE + 1];
   const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
   const int tx = threadIdx.x, ty = threadIdx.y;
@@ -286,6 +296,7 @@ __global__ void ror_bwd_elem_kernel(int act, const float* __restrict__ zpart,
 }
 
 __global__ void fill_kernel(float* p, int64_t n, float v) {
+  pdl_entry();
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x)
     p[i] = v;
@@ -297,32 +308,32 @@ template <typename T>
 void transpose(const T* X, int rows, int cols, int ld, T* XT, int ldT, cudaStream_t s) {
   if (rows <= 0 || cols <= 0) return;
   dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE);
-  transpose_kernel<T><<<grid, dim3(TILE, TROWS), 0, s>>>(X, rows, cols, ld, XT, ldT);
+  launch_k(transpose_kernel<T>, dim3(grid), dim3(TILE, TROWS), 0, s, X, rows, cols, ld, XT, ldT);
 }
 
 template <typename T>
 void fill_rows(const RowFill& f, int cols, cudaStream_t s) {
   if (f.n <= 0 || cols <= 0) return;
   dim3 grid((cols + 255) / 256, f.n);
-  fill_rows_kernel<T><<<grid, 256, 0, s>>>(f, cols);
+  launch_k(fill_rows_kernel<T>, dim3(grid), dim3(256), 0, s, f, cols);
 }
 
 template <typename T>
 void loss_seed(const LossArgs& a, cudaStream_t s) {
   if (a.rows <= 0) return;
   const int warps = 8;
-  loss_seed_kernel<T><<<(a.rows + warps - 1) / warps, warps * 32, 0, s>>>(a);
+  launch_k(loss_seed_kernel<T>, dim3((a.rows + warps - 1) / warps), dim3(warps * 32), 0, s, a);
 }
 
 void sum_scaled(const float* x, int n, float scale, float* out, cudaStream_t s) {
-  sum_scaled_kernel<<<1, 1024, 0, s>>>(x, n, scale, out);
+  launch_k(sum_scaled_kernel, dim3(1), dim3(1024), 0, s, x, n, scale, out);
 }
 
 template <typename T>
 void layer_update(const LayerTable& tab, const LayerUpdArgs& a, cudaStream_t s) {
   const int blocks = tab.tile0[tab.n];
   if (blocks <= 0) return;
-  layer_update_kernel<T><<<blocks, dim3(TILE, TROWS), 0, s>>>(tab, a);
+  launch_k(layer_update_kernel<T>, dim3(blocks), dim3(TILE, TROWS), 0, s, tab, a);
 }
 
 template <typename T>
@@ -330,7 +341,7 @@ void ror_fwd_elem(int act, const float* dzbar, const float* Z, const float* dA, 
                   T* dab, int ld, T* dabT, int ldT, float* zpart, cudaStream_t s) {
   if (rows <= 0 || cols <= 0) return;
   dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE);
-  ror_fwd_elem_kernel<T><<<grid, dim3(TILE, TROWS), 0, s>>>(act, dzbar, Z, dA, rows, cols, dab, ld,
+  launch_k(ror_fwd_elem_kernel<T>, dim3(grid), dim3(TILE, TROWS), 0, s, act, dzbar, Z, dA, rows, cols, dab, ld,
                                                              dabT, ldT, zpart);
 }
 
@@ -339,7 +350,7 @@ void ror_bwd_elem(int act, const float* zpart, const float* abar, const float* Z
                   int cols, T* zb, int ld, T* zbT, int ldT, cudaStream_t s) {
   if (rows <= 0 || cols <= 0) return;
   dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE);
-  ror_bwd_elem_kernel<T><<<grid, dim3(TILE, TROWS), 0, s>>>(act, zpart, abar, Z, rows, cols, zb, ld,
+  launch_k(ror_bwd_elem_kernel<T>, dim3(grid), dim3(TILE, TROWS), 0, s, act, zpart, abar, Z, rows, cols, zb, ld,
                                                              zbT, ldT);
 }
 
@@ -347,7 +358,7 @@ void fill(float* p, int64_t n, float v, cudaStream_t s) {
   if (n <= 0) return;
   int64_t b = (n + 255) / 256;
   if (b > 152 * 16) b = 152 * 16;
-  fill_kernel<<<static_cast<int>(b), 256, 0, s>>>(p, n, v);
+  launch_k(fill_kernel, dim3(static_cast<int>(b)), dim3(256), 0, s, p, n, v);
 }
 
 #define MF_INST(T)                                                                 \

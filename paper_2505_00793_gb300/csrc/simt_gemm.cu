@@ -8,6 +8,7 @@
 
 #include "device_math.cuh"
 #include "internal.h"
+#include "launch.cuh"
 
 namespace mf {
 namespace {
@@ -25,6 +26,7 @@ struct SimtParams {
 };
 
 __global__ void __launch_bounds__(256) simt_dual_gemm_kernel(SimtParams p) {
+  pdl_entry();
   const int64_t bz = blockIdx.z;
   for (int i = 0; i < 2; ++i) {
     if (p.A[i]) p.A[i] += bz * p.bsA[i];
@@ -120,7 +122,7 @@ cudaError_t simt_gemm(const GemmArgs& a, cudaStream_t s) {
   p.bsC[0] = a.bsC0; p.bsC[1] = a.bsC1;
   if (a.batch > 1 && a.epi.mode != EPI_STORE) return cudaErrorInvalidValue;
   dim3 grid((a.N + TN - 1) / TN, (a.M + TM - 1) / TM, a.batch < 1 ? 1 : a.batch);
-  simt_dual_gemm_kernel<<<grid, 256, 0, s>>>(p);
+  launch_k(simt_dual_gemm_kernel, dim3(grid), dim3(256), 0, s, p);
   return cudaGetLastError();
 }
 

@@ -29,6 +29,7 @@
 
 #include "device_math.cuh"
 #include "internal.h"
+#include "launch.cuh"
 
 namespace mf {
 namespace {
@@ -95,6 +96,10 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* s
 }
 
 // Every operand map is 3-D {K, rows, batch}; non-batched GEMMs have batch extent 1.
+__device__ __forceinline__ void prefetch_tmap(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint64_t* bar,
                                             int x, int y, int z) {
   asm volatile(
@@ -441,6 +446,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     mbar_init(&acc_bar, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    // the descriptors are kernel parameters, not data of the previous kernel
+    if (p.a0_off >= 0) prefetch_tmap(&tmA0);
+    if (p.a1_off >= 0) prefetch_tmap(&tmA1);
+    if (p.b0_off >= 0) prefetch_tmap(&tmB0);
+    if (p.b1_off >= 0) prefetch_tmap(&tmB1);
   }
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -452,6 +462,9 @@ __global__ void __launch_bounds__(THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tbase = tmem_slot;
+  // Everything above overlaps the previous kernel under programmatic dependent launch;
+  // from here on the kernel reads and writes global memory.
+  pdl_entry();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -823,13 +836,15 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
   cfg.blockDim = dim3(THREADS, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 1;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = S;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = g_pdl ? 1 : 0;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, tc_dual_gemm_kernel<BN, KA, MODE, ACT>, mA0, mA1, mB0, mB1, mC0, mC1, mA,
                             mAd, p);
 }

@@ -236,3 +236,31 @@ def test_graph_replay_matches_eager():
     mf.sync()
     assert np.array_equal(d_eta.cpu().numpy(), outs[0][0])
     mf.close()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("option", ["MF_OPT_PDL", "MF_OPT_CONCURRENT"])
+def test_launch_options_bit_identical(option):
+    """Programmatic dependent launch and the two-stream backward change when kernels may
+    run, not what they compute or the order of dependent memory effects: the meta-gradient
+    is bit-identical with the option on and off, eager and replayed."""
+    torch, native = need_gpu()
+    opt = getattr(native, option)
+    w = BF16_CASES["wide_ragged"]
+    inp = synth.make_inputs(w)
+    outs = []
+    for val in (1, 0, 1):
+        mf = native.MixFlow.for_workload(w)
+        mf.set_option(opt, val)
+        loop = native.loop_desc_for(w)
+        d = native.to_device_inputs(w, inp)
+        d_eta = torch.empty(w.n_eta, device="cuda")
+        d_th = torch.empty(w.n_params, device="cuda")
+        for _ in range(3):   # eager, capture, replay
+            mf.meta_grad(loop, d["theta0"], d["eta"], d["inner_x"], d["inner_y"], d["outer_x"],
+                         d["outer_y"], d_eta, d_th)
+        mf.sync()
+        outs.append((d_eta.cpu().numpy(), d_th.cpu().numpy()))
+        mf.close()
+    for k in (1, 2):
+        assert np.array_equal(outs[0][0], outs[k][0]) and np.array_equal(outs[0][1], outs[k][1])
