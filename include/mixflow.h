@@ -209,8 +209,12 @@ mf_status mf_kernel_time(mf_handle h, double* ms, uint64_t* launches, double* fl
  * Setting it drops the handle's captured graphs.
  * MF_OPT_CONCURRENT (default 1): in each backward layer the weight product and the data
  * product run on two streams (parallel branches of a captured graph); 0 runs them in
- * sequence on the call's stream. */
-enum { MF_OPT_CUDA_GRAPHS = 1, MF_OPT_PDL = 2, MF_OPT_CONCURRENT = 3 };
+ * sequence on the call's stream.
+ * MF_OPT_GEMM_2SM (process-wide): 1 (default) computes a bf16 GEMM with 256-row tiles on
+ * CTA pairs (tcgen05 cta_group::2) when its grid of pairs fills the GPU, 0 never, 2 for
+ * every GEMM with more than 128 rows (for tests).  Results are identical up to the
+ * summation order within a tile, which both forms share. */
+enum { MF_OPT_CUDA_GRAPHS = 1, MF_OPT_PDL = 2, MF_OPT_CONCURRENT = 3, MF_OPT_GEMM_2SM = 4 };
 mf_status mf_set_option(mf_handle h, int option, int value);
 
 /* Host-side fault injection for tests: kind 1 = the next workspace allocation fails;

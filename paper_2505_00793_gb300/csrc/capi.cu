@@ -1280,6 +1280,12 @@ mf_status mf_set_option(mf_handle h, int option, int value) {
     drop_graphs(h);
     return MF_OK;
   }
+  if (option == MF_OPT_GEMM_2SM) {
+    if (value < 0 || value > 2) return fail(h, MF_ERR_INVALID_ARG, "MF_OPT_GEMM_2SM takes 0, 1 or 2");
+    mf::g_pair_mode = value;
+    drop_graphs(h);
+    return MF_OK;
+  }
   if (option == MF_OPT_CONCURRENT) {
     h->concurrent = value != 0;
     drop_graphs(h);

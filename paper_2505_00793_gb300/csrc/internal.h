@@ -48,6 +48,7 @@ struct GemmArgs {
   int64_t bsA0 = 0, bsA1 = 0, bsB0 = 0, bsB1 = 0, bsC0 = 0, bsC1 = 0;   // batch strides (elements)
   int split_k = 0;         // 0 = choose automatically, else 1/2/4/8 (tensor-core path)
   int bn = 0, ka = 0;      // tile width / K atoms per stage; 0 = choose automatically
+  int pair = 0;            // 2-SM tiles (tensor-core path): 0 automatic, 1 always, -1 never
   int* status = nullptr;   // device status word (timeouts), may be null
 };
 
@@ -55,7 +56,10 @@ struct GemmArgs {
 // host-side rejection (bad alignment/ld) and returns cudaErrorInvalidValue.
 cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why);
 // Activation-epilogue instances (tc_gemm_act.cu), called by tc_gemm.
-cudaError_t tc_gemm_act(const GemmArgs& a, cudaStream_t s, const char** why, int bn, int ka);
+cudaError_t tc_gemm_act(const GemmArgs& a, cudaStream_t s, const char** why, int bn, int pair);
+// Process-wide choice of 2-SM tiles for GEMMs that leave it automatic: 0 never, 1 when the
+// grid fills the GPU (default), 2 whenever M > 128.
+extern int g_pair_mode;
 // SIMT float32 GEMM with the same semantics (simt_gemm.cu).
 cudaError_t simt_gemm(const GemmArgs& a, cudaStream_t s);
 

@@ -21,6 +21,8 @@
 
 namespace mf {
 
+int g_pair_mode = 1;
+
 cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why) {
   static const char* dummy;
   if (!why) why = &dummy;
@@ -63,21 +65,32 @@ cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why) {
       return cudaErrorInvalidValue;
     }
   }
-  int bn = a.bn, ka = a.ka;
+  int bn = a.bn, pair = 0;
+  const int nbatch = a.batch < 1 ? 1 : a.batch;
+  if (a.pair >= 0 && a.split_k <= 1 && a.M > 128 && (bn == 0 || bn == 128 || bn == 256)) {
+    // 2-SM tiles (256 rows per CTA pair) when the pair grid fills the GPU
+    const int pairs_m = ((a.M + 255) / 256) * nbatch;
+    if (a.pair == 1 || g_pair_mode == 2) {
+      pair = 1;
+      if (bn == 0) bn = a.N > 128 ? 256 : 128;
+    } else if (g_pair_mode == 1 && bn == 0 && a.M >= 256) {
+      if (pairs_m * ((a.N + 255) / 256) >= 76) { pair = 1; bn = 256; }
+      else if (pairs_m * ((a.N + 127) / 128) >= 60) { pair = 1; bn = 128; }
+    }
+  }
   if (bn == 0) {
     // Narrow outputs take the narrowest tile; otherwise 64-wide tiles while a 128-wide grid
     // would leave most SMs idle (small-batch layers), else 128 (dual) or 256 columns.
     const bool dual = a.terms & (T_C1_A1B0 | T_C1_A0B1);
-    const int tiles_m = ((a.M + 127) / 128) * (a.batch < 1 ? 1 : a.batch);
+    const int tiles_m = ((a.M + 127) / 128) * nbatch;
     if (a.N <= 16) bn = 16;
     else if (a.N <= 32) bn = 32;
     else if (a.N <= 64 || tiles_m * ((a.N + 127) / 128) < 76) bn = 64;
     else if (dual || tiles_m * ((a.N + 255) / 256) < 152) bn = 128;
     else bn = 256;
   }
-  if (ka == 0) ka = 1;
-  if (a.epi.mode == EPI_STORE) return launch_bn<EPI_STORE, ACT_IDENT>(a, s, why, bn, ka);
-  return tc_gemm_act(a, s, why, bn, ka);
+  if (a.epi.mode == EPI_STORE) return launch_bn<EPI_STORE, ACT_IDENT>(a, s, why, bn, pair);
+  return tc_gemm_act(a, s, why, bn, pair);
 }
 
 }  // namespace mf

@@ -50,6 +50,7 @@ struct TcParams {
   int64_t bsC0, bsC1;     // batch strides of C0 / C1 (direct-store paths)
   int st_c0, st_c1, st_a, st_ad;   // which row-major outputs exist
   int a0_off, a1_off, b0_off, b1_off, stage_bytes, tx_bytes;
+  int nsub;               // TMEM blocks per logical accumulator (1, 2 or 4)
   float* C0; int ldc0; const float* bias0;
   float* C1; int ldc1; const float* bias1;
   EpiParams epi;
@@ -167,6 +168,28 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Accumulators.  Logical accumulator c (0: C0, 1: C1) owns nsub blocks of BN TMEM columns
+// at (c * nsub + j) * BN.  Successive products into one logical accumulator rotate over its
+// blocks: an MMA into a block waits for the previous MMA into the same block (its
+// read-modify-write of TMEM), so rotating keeps several MMAs in flight.  The epilogue sums
+// the blocks in order j = 0..nsub-1 (deterministic).
+template <int BN>
+__device__ __forceinline__ void ld_acc16(uint32_t taddr, int c, int nsub, int col,
+                                         float (&v)[16]) {
+  tmem_ld16(taddr + static_cast<uint32_t>(c * nsub * BN + col), v);
+  for (int j = 1; j < nsub; ++j) {
+    float t[16];
+    tmem_ld16(taddr + static_cast<uint32_t>((c * nsub + j) * BN + col), t);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] += t[i];
+  }
+}
+
+// The most blocks (up to 4) that fit 512 TMEM columns.
+__host__ __device__ constexpr int acc_blocks(int nlogical, int bn) {
+  return nlogical * 4 * bn <= 512 ? 4 : nlogical * 2 * bn <= 512 ? 2 : 1;
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
@@ -324,8 +347,8 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
       const int cc = c + sub * 16;          // tile column of this 16-column group
       if (cc >= BN) break;
       float v0[16], v1[16];
-      tmem_ld16(taddr + cc, v0);
-      if (dual) tmem_ld16(taddr + BN + cc, v1);
+      ld_acc16<BN>(taddr, 0, p.nsub, cc, v0);
+      if (dual) ld_acc16<BN>(taddr, 1, p.nsub, cc, v1);
       else {
 #pragma unroll
         for (int j = 0; j < 16; ++j) v1[j] = 0.f;
@@ -398,6 +421,107 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
   __syncwarp();
 }
 
+__device__ __forceinline__ void mma_bf16_pair(uint32_t dtmem, uint64_t ad, uint64_t bd,
+                                              uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(dtmem),
+      "l"(ad), "l"(bd), "r"(idesc), "r"(accumulate));
+}
+
+// Arrive once on the barrier at this shared-memory offset in both CTAs of the pair when
+// the pair's previously issued MMAs have completed.
+__device__ __forceinline__ void mma_commit_pair(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(static_cast<uint16_t>(3))
+      : "memory");
+}
+
+struct MmaLoop {
+  int nk, stages, stage_bytes, a0_off, a1_off, b0_off, b1_off;
+  uint32_t sbase, tbase;
+  uint64_t* full_bar;
+  uint64_t* empty_bar;
+  int* status;
+};
+
+// The MMA issuer's loop over K blocks.  TERMS != 0 fixes the product mask at compile time
+// (TERMS = 0 reads `terms` at run time) so that the issue sequence is straight-line code:
+// a single thread issues every tcgen05.mma, and instructions between MMAs delay the tensor
+// pipe.  Products of K slice kk go to accumulator block kk mod NSUB (see ld_acc16).  PAIR
+// issues the M = 256 form for a CTA pair and multicasts the commits to both CTAs.
+template <int BN, int KA, unsigned TERMS, int NSUB, bool PAIR>
+__device__ __forceinline__ void mma_loop(const MmaLoop& L, unsigned terms_rt, int nsub_rt) {
+  constexpr int A_ATOM = BM * BK * 2, B_ATOM = (PAIR ? BN / 2 : BN) * BK * 2;
+  constexpr uint32_t idesc = idesc_bf16(PAIR ? 2 * BM : BM, BN);
+  const unsigned terms = TERMS ? TERMS : terms_rt;
+  const uint32_t nsub = NSUB ? static_cast<uint32_t>(NSUB) : static_cast<uint32_t>(nsub_rt);
+  for (int i = 0; i < L.nk; ++i) {
+    const int s = i % L.stages;
+    const uint32_t ph = (i / L.stages) & 1;
+    if (!mbar_wait(&L.full_bar[s], ph, L.status)) break;
+    tc_fence_after();
+    const uint32_t st = L.sbase + s * L.stage_bytes;
+#pragma unroll
+    for (int a = 0; a < KA; ++a) {
+      const uint64_t a0 = L.a0_off >= 0 ? sdesc_sw128(st + L.a0_off + a * A_ATOM) : 0;
+      const uint64_t a1 = L.a1_off >= 0 ? sdesc_sw128(st + L.a1_off + a * A_ATOM) : 0;
+      const uint64_t b0 = L.b0_off >= 0 ? sdesc_sw128(st + L.b0_off + a * B_ATOM) : 0;
+      const uint64_t b1 = L.b1_off >= 0 ? sdesc_sw128(st + L.b1_off + a * B_ATOM) : 0;
+#pragma unroll
+      for (int kk = 0; kk < BK / 16; ++kk) {
+        const uint64_t adv = static_cast<uint64_t>(kk * 2);   // 32 bytes per K=16 step
+        const uint32_t blk = static_cast<uint32_t>(kk) & (nsub - 1);
+        const uint32_t t0 = L.tbase + blk * BN, t1 = L.tbase + (nsub + blk) * BN;
+        uint32_t f0 = (i == 0 && a == 0 && static_cast<uint32_t>(kk) < nsub) ? 0u : 1u;
+        uint32_t f1 = f0;
+        auto mma = [&](uint32_t d, uint64_t ad, uint64_t bd, uint32_t f) {
+          if constexpr (PAIR) mma_bf16_pair(d, ad, bd, idesc, f);
+          else mma_bf16(d, ad, bd, idesc, f);
+        };
+        if (terms & T_C0_A0B0) { mma(t0, a0 + adv, b0 + adv, f0); f0 = 1; }
+        if (terms & T_C1_A1B0) { mma(t1, a1 + adv, b0 + adv, f1); f1 = 1; }
+        if (terms & T_C0_A1B0) { mma(t0, a1 + adv, b0 + adv, f0); f0 = 1; }
+        if (terms & T_C1_A0B1) { mma(t1, a0 + adv, b1 + adv, f1); f1 = 1; }
+        if (terms & T_C0_A0B1) { mma(t0, a0 + adv, b1 + adv, f0); f0 = 1; }
+        if (terms & T_C0_A1B1) { mma(t0, a1 + adv, b1 + adv, f0); f0 = 1; }
+      }
+    }
+    if constexpr (PAIR) mma_commit_pair(&L.empty_bar[s]);
+    else mma_commit(&L.empty_bar[s]);
+  }
+}
+
+// Dispatch of the MMA loop over the product masks the library issues; anything else takes
+// the run-time mask.  Plain-store GEMMs carry the weight products and the head layer,
+// activation epilogues the forward and data products.
+template <int BN, int KA, int MODE, bool PAIR>
+__device__ __forceinline__ void mma_dispatch(const MmaLoop& L, unsigned terms, int nsub) {
+  constexpr int N1 = acc_blocks(1, BN), N2 = acc_blocks(2, BN);
+  switch (terms) {
+    case T_C0_A0B0: mma_loop<BN, KA, T_C0_A0B0, N1, PAIR>(L, terms, nsub); return;
+    case T_C0_A0B0 | T_C1_A1B0 | T_C1_A0B1:
+      mma_loop<BN, KA, T_C0_A0B0 | T_C1_A1B0 | T_C1_A0B1, N2, PAIR>(L, terms, nsub); return;
+    case T_C0_A0B0 | T_C1_A0B1:
+      mma_loop<BN, KA, T_C0_A0B0 | T_C1_A0B1, N2, PAIR>(L, terms, nsub); return;
+    default: break;
+  }
+  if constexpr (MODE == EPI_STORE) {
+    switch (terms) {
+      case T_C0_A0B1: mma_loop<BN, KA, T_C0_A0B1, N1, PAIR>(L, terms, nsub); return;
+      case T_C0_A1B0 | T_C0_A0B1:
+        mma_loop<BN, KA, T_C0_A1B0 | T_C0_A0B1, N1, PAIR>(L, terms, nsub); return;
+      case T_C0_A0B0 | T_C0_A1B1:
+        mma_loop<BN, KA, T_C0_A0B0 | T_C0_A1B1, N1, PAIR>(L, terms, nsub); return;
+      default: break;
+    }
+  }
+  mma_loop<BN, KA, 0, 0, PAIR>(L, terms, nsub);
+}
+
 template <int BN, int KA, int MODE, int ACT>
 __global__ void __launch_bounds__(THREADS, 1)
     tc_dual_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
@@ -433,7 +557,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int nk = max(0, min(nkb, kb0 + kper) - kb0);
   const unsigned terms = p.terms;
   const bool dual = (terms & (T_C1_A1B0 | T_C1_A0B1)) != 0;
-  const uint32_t ncols = tmem_cols(dual ? 2 * BN : BN);
+  const uint32_t ncols = tmem_cols((dual ? 2 : 1) * p.nsub * BN);
   constexpr int A_ATOM = BM * BK * 2, B_ATOM = BN * BK * 2;
 
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -493,39 +617,12 @@ __global__ void __launch_bounds__(THREADS, 1)
   } else if (warp == 1) {
     if (lane == 0 && nk > 0) {
       // ---- MMA issuer (single thread) -----------------------------------------------
-      constexpr uint32_t idesc = idesc_bf16(BM, BN);
-      const uint32_t d0 = tbase;
-      const uint32_t d1 = tbase + BN;
-      const int stages = p.stages, stage_bytes = p.stage_bytes;
-      const int a0_off = p.a0_off, a1_off = p.a1_off, b0_off = p.b0_off, b1_off = p.b1_off;
-      int* const status = p.status;
-      const uint32_t sbase = smem_u32(smem);
-      bool started0 = false, started1 = false;
-      for (int i = 0; i < nk; ++i) {
-        const int s = i % stages;
-        const uint32_t ph = (i / stages) & 1;
-        if (!mbar_wait(&full_bar[s], ph, status)) break;
-        tc_fence_after();
-        const uint32_t st = sbase + s * stage_bytes;
-#pragma unroll
-        for (int a = 0; a < KA; ++a) {
-          const uint64_t a0 = a0_off >= 0 ? sdesc_sw128(st + a0_off + a * A_ATOM) : 0;
-          const uint64_t a1 = a1_off >= 0 ? sdesc_sw128(st + a1_off + a * A_ATOM) : 0;
-          const uint64_t b0 = b0_off >= 0 ? sdesc_sw128(st + b0_off + a * B_ATOM) : 0;
-          const uint64_t b1 = b1_off >= 0 ? sdesc_sw128(st + b1_off + a * B_ATOM) : 0;
-#pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint64_t adv = static_cast<uint64_t>(kk * 2);   // 32 bytes per K=16 step
-            if (terms & T_C0_A0B0) { mma_bf16(d0, a0 + adv, b0 + adv, idesc, started0); started0 = true; }
-            if (terms & T_C0_A1B0) { mma_bf16(d0, a1 + adv, b0 + adv, idesc, started0); started0 = true; }
-            if (terms & T_C0_A0B1) { mma_bf16(d0, a0 + adv, b1 + adv, idesc, started0); started0 = true; }
-            if (terms & T_C1_A1B0) { mma_bf16(d1, a1 + adv, b0 + adv, idesc, started1); started1 = true; }
-            if (terms & T_C1_A0B1) { mma_bf16(d1, a0 + adv, b1 + adv, idesc, started1); started1 = true; }
-            if (terms & T_C0_A1B1) { mma_bf16(d0, a1 + adv, b1 + adv, idesc, started0); started0 = true; }
-          }
-        }
-        mma_commit(&empty_bar[s]);
-      }
+      MmaLoop L;
+      L.nk = nk; L.stages = p.stages; L.stage_bytes = p.stage_bytes;
+      L.a0_off = p.a0_off; L.a1_off = p.a1_off; L.b0_off = p.b0_off; L.b1_off = p.b1_off;
+      L.sbase = smem_u32(smem); L.tbase = tbase;
+      L.full_bar = full_bar; L.empty_bar = empty_bar; L.status = p.status;
+      mma_dispatch<BN, KA, MODE, false>(L, terms, p.nsub);
       mma_commit(&acc_bar);
     }
     __syncwarp();
@@ -545,8 +642,8 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll 1
           for (int c = 0; c < BN; c += 16) {
             float v0[16], v1[16];
-            tmem_ld16(tbase + lane_off + c, v0);
-            if (dual) tmem_ld16(tbase + lane_off + BN + c, v1);
+            ld_acc16<BN>(tbase + lane_off, 0, p.nsub, c, v0);
+            if (dual) ld_acc16<BN>(tbase + lane_off, 1, p.nsub, c, v1);
             else {
 #pragma unroll
               for (int j = 0; j < 16; ++j) v1[j] = 0.f;
@@ -587,7 +684,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int c = 0; c < BN; c += 16) {
           float v[16];
           if (ok) {
-            tmem_ld16(tbase + lane_off + a * BN + c, v);
+            ld_acc16<BN>(tbase + lane_off, a, p.nsub, c, v);
           } else {
 #pragma unroll
             for (int j = 0; j < 16; ++j) v[j] = 0.f;
@@ -757,6 +854,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
   p.b1_off = useB1 ? (off += b_bytes, off - b_bytes) : -1;
   p.stage_bytes = off;
   p.tx_bytes = off;
+  p.nsub = acc_blocks(dual ? 2 : 1, BN);
   const int budget = 220 * 1024;
   int stages = budget / off;
   if (stages > MAX_STAGES) stages = MAX_STAGES;
@@ -849,10 +947,265 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
                             mAd, p);
 }
 
+// ================================ 2-SM tiles (cta_group::2) ================================
+// A cluster of two CTAs (a CTA pair on two SMs) computes a 256 x BN tile: each CTA stages
+// its own 128 rows of A and one half (BN/2 rows) of B, the even CTA issues
+// tcgen05.mma.cta_group::2 (M = 256) that reads both CTAs' shared memory and accumulates
+// rows 0..127 in its TMEM and rows 128..255 in the odd CTA's TMEM.  Per SM this halves the
+// B bytes per flop against the one-SM tile, so the same shared memory holds a deeper
+// pipeline.  Both CTAs' TMA loads signal the even CTA's full barriers; the MMA completion
+// is multicast to both CTAs' empty barriers and accumulator barrier.  No split of K.
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void tma_load_3d_pair(void* dst, const CUtensorMap* map,
+                                                 uint32_t bar_cluster, int x, int y, int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar_cluster)
+      : "memory");
+}
+
+template <int BN, int MODE, int ACT>
+__global__ void __launch_bounds__(THREADS, 1)
+    tc2_dual_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
+                         const __grid_constant__ CUtensorMap tmA1,
+                         const __grid_constant__ CUtensorMap tmB0,
+                         const __grid_constant__ CUtensorMap tmB1,
+                         const __grid_constant__ CUtensorMap tmC0,
+                         const __grid_constant__ CUtensorMap tmC1,
+                         const __grid_constant__ CUtensorMap tmA,
+                         const __grid_constant__ CUtensorMap tmAd, const TcParams prm) {
+  TcParams p = prm;
+  const int bz = static_cast<int>(blockIdx.z);
+  if (p.C0) p.C0 += bz * p.bsC0;
+  if (p.C1) p.C1 += bz * p.bsC1;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[MAX_STAGES];
+  __shared__ __align__(8) uint64_t empty_bar[MAX_STAGES];
+  __shared__ __align__(8) uint64_t acc_bar;
+  __shared__ uint32_t tmem_slot;
+
+  constexpr int BH = BN / 2;                 // B rows staged by each CTA
+  const uint32_t rank = cluster_rank();      // 0: issues the MMAs, 1: its peer
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int m0 = static_cast<int>(blockIdx.x >> 1) * (2 * BM) + static_cast<int>(rank) * BM;
+  const int n0 = blockIdx.y * BN;
+  const int nk = (p.K + BK - 1) / BK;
+  const unsigned terms = p.terms;
+  const bool dual = (terms & (T_C1_A1B0 | T_C1_A0B1)) != 0;
+  const uint32_t ncols = tmem_cols((dual ? 2 : 1) * p.nsub * BN);
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < p.stages; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], 1);
+    }
+    mbar_init(&acc_bar, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    if (p.a0_off >= 0) prefetch_tmap(&tmA0);
+    if (p.a1_off >= 0) prefetch_tmap(&tmA1);
+    if (p.b0_off >= 0) prefetch_tmap(&tmB0);
+    if (p.b1_off >= 0) prefetch_tmap(&tmB1);
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&tmem_slot)),
+                 "r"(ncols));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;");
+  }
+  tc_fence_before();
+  cluster_sync_all();          // both CTAs' barriers initialised and TMEM allocated
+  tc_fence_after();
+  const uint32_t tbase = tmem_slot;
+  pdl_entry();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      const int stages = p.stages, stage_bytes = p.stage_bytes;
+      const int a0_off = p.a0_off, a1_off = p.a1_off, b0_off = p.b0_off, b1_off = p.b1_off;
+      int* const status = p.status;
+      const uint32_t full0 = dsmem_addr(smem_u32(&full_bar[0]), 0);   // even CTA's barriers
+      const int nb0 = n0 + static_cast<int>(rank) * BH;
+      for (int i = 0; i < nk; ++i) {
+        const int s = i % stages;
+        const uint32_t ph = (i / stages) & 1;
+        if (!mbar_wait(&empty_bar[s], ph ^ 1, status)) break;
+        if (rank == 0) mbar_expect_tx(&full_bar[s], 2 * stage_bytes);
+        const uint32_t bar = full0 + static_cast<uint32_t>(s) * 8u;
+        uint8_t* st = smem + s * stage_bytes;
+        const int k = i * BK;
+        if (a0_off >= 0) tma_load_3d_pair(st + a0_off, &tmA0, bar, k, m0, bz);
+        if (a1_off >= 0) tma_load_3d_pair(st + a1_off, &tmA1, bar, k, m0, bz);
+        if (b0_off >= 0) tma_load_3d_pair(st + b0_off, &tmB0, bar, k, nb0, bz);
+        if (b1_off >= 0) tma_load_3d_pair(st + b1_off, &tmB1, bar, k, nb0, bz);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (rank == 0 && lane == 0) {
+      MmaLoop L;
+      L.nk = nk; L.stages = p.stages; L.stage_bytes = p.stage_bytes;
+      L.a0_off = p.a0_off; L.a1_off = p.a1_off; L.b0_off = p.b0_off; L.b1_off = p.b1_off;
+      L.sbase = smem_u32(smem); L.tbase = tbase;
+      L.full_bar = full_bar; L.empty_bar = empty_bar; L.status = p.status;
+      mma_dispatch<BN, 1, MODE, true>(L, terms, p.nsub);
+      mma_commit_pair(&acc_bar);
+    }
+    __syncwarp();
+  } else {
+    // accumulator drain: this CTA's 128 rows of the pair tile, TMEM lane quadrant = warp % 4
+    const int q = warp & 3;
+    const int r = q * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    const bool ok = mbar_wait(&acc_bar, 0, p.status);
+    tc_fence_after();
+    if (ok) {
+      if (p.tma_store) {
+        epilogue_tma<BN, MODE, ACT>(p, &tmC0, &tmC1, &tmA, &tmAd, smem + q * STG_WARP,
+                                    tbase + lane_off, q, lane, m0, n0, dual, bz);
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 16) {
+          float v0[16], v1[16];
+          ld_acc16<BN>(tbase + lane_off, 0, p.nsub, c, v0);
+          if (dual) ld_acc16<BN>(tbase + lane_off, 1, p.nsub, c, v1);
+          else {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) v1[j] = 0.f;
+          }
+          if (n0 + c < p.N) epilogue16<MODE, ACT>(p, m0 + r, n0 + c, v0, v1, dual);
+        }
+      }
+    }
+    tc_fence_before();
+  }
+  __syncthreads();
+  cluster_sync_all();          // both CTAs have drained their TMEM
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tbase),
+                 "r"(ncols));
+  }
+}
+
+template <int BN, int MODE, int ACT>
+cudaError_t launch_cfg2(const GemmArgs& a, cudaStream_t s, const char** why) {
+  constexpr int BH = BN / 2;
+  const unsigned t = a.terms;
+  const bool useA0 = t & (T_C0_A0B0 | T_C0_A0B1 | T_C1_A0B1);
+  const bool useA1 = t & (T_C0_A1B0 | T_C1_A1B0 | T_C0_A1B1);
+  const bool useB0 = t & (T_C0_A0B0 | T_C0_A1B0 | T_C1_A1B0);
+  const bool useB1 = t & (T_C0_A0B1 | T_C1_A0B1 | T_C0_A1B1);
+  const bool dual = t & (T_C1_A1B0 | T_C1_A0B1);
+  TcParams p;
+  memset(&p, 0, sizeof(p));
+  p.M = a.M; p.N = a.N; p.K = a.K; p.terms = t;
+  const int a_bytes = BM * BK * 2, b_bytes = BH * BK * 2;
+  int off = 0;
+  p.a0_off = useA0 ? (off += a_bytes, off - a_bytes) : -1;
+  p.a1_off = useA1 ? (off += a_bytes, off - a_bytes) : -1;
+  p.b0_off = useB0 ? (off += b_bytes, off - b_bytes) : -1;
+  p.b1_off = useB1 ? (off += b_bytes, off - b_bytes) : -1;
+  p.stage_bytes = off;
+  p.tx_bytes = off;
+  p.nsub = acc_blocks(dual ? 2 : 1, BN);
+  int stages = (220 * 1024) / off;
+  if (stages > MAX_STAGES) stages = MAX_STAGES;
+  if (stages < 2) { *why = "tile does not fit shared memory"; return cudaErrorInvalidValue; }
+  p.stages = stages;
+  p.split = 1;
+  p.C0 = a.C0; p.ldc0 = a.ldc0; p.bias0 = a.bias0;
+  p.C1 = dual ? a.C1 : nullptr; p.ldc1 = a.ldc1; p.bias1 = a.bias1;
+  p.epi = a.epi;
+  p.status = a.status;
+  const int nb = a.batch < 1 ? 1 : a.batch;
+  const int pairs_m = (a.M + 2 * BM - 1) / (2 * BM), tiles_n = (a.N + BN - 1) / BN;
+
+  CUtensorMap mA0, mA1, mB0, mB1, mC0, mC1, mA, mAd;
+  memset(&mA0, 0, sizeof(mA0)); memset(&mA1, 0, sizeof(mA1));
+  memset(&mB0, 0, sizeof(mB0)); memset(&mB1, 0, sizeof(mB1));
+  memset(&mC0, 0, sizeof(mC0)); memset(&mC1, 0, sizeof(mC1));
+  memset(&mA, 0, sizeof(mA)); memset(&mAd, 0, sizeof(mAd));
+  if (useA0 && !make_map(&mA0, a.A0, a.K, a.M, a.lda0, BM, nb, a.bsA0)) { *why = "tensor map A0"; return cudaErrorInvalidValue; }
+  if (useA1 && !make_map(&mA1, a.A1, a.K, a.M, a.lda1, BM, nb, a.bsA1)) { *why = "tensor map A1"; return cudaErrorInvalidValue; }
+  if (useB0 && !make_map(&mB0, a.B0, a.K, a.N, a.ldb0, BH, nb, a.bsB0)) { *why = "tensor map B0"; return cudaErrorInvalidValue; }
+  if (useB1 && !make_map(&mB1, a.B1, a.K, a.N, a.ldb1, BH, nb, a.bsB1)) { *why = "tensor map B1"; return cudaErrorInvalidValue; }
+  p.batch = nb;
+  p.bsC0 = a.bsC0;
+  p.bsC1 = a.bsC1;
+
+  const bool act = a.epi.mode != EPI_STORE;
+  p.st_c0 = p.C0 != nullptr;
+  p.st_c1 = p.C1 != nullptr;
+  p.st_a = act && a.epi.A != nullptr;
+  p.st_ad = act && dual && a.epi.Ad != nullptr;
+  bool tma_ok = true;
+  if (p.st_c0) tma_ok = tma_ok && aligned16(p.C0) && !(p.ldc0 & 3);
+  if (p.st_c1) tma_ok = tma_ok && aligned16(p.C1) && !(p.ldc1 & 3);
+  if (p.st_a) tma_ok = tma_ok && aligned16(a.epi.A) && !(a.epi.lda & 7);
+  if (p.st_ad) tma_ok = tma_ok && aligned16(a.epi.Ad) && !(a.epi.lda & 7);
+  if (nb > 1) tma_ok = tma_ok && !(a.bsC0 & 3) && !(a.bsC1 & 3);
+  if (tma_ok && p.st_c0)
+    tma_ok = make_map2(&mC0, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, p.C0, a.N, a.M, p.ldc0, 32, 32, nb,
+                       a.bsC0);
+  if (tma_ok && p.st_c1)
+    tma_ok = make_map2(&mC1, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, p.C1, a.N, a.M, p.ldc1, 32, 32, nb,
+                       a.bsC1);
+  if (tma_ok && p.st_a)
+    tma_ok = make_map2(&mA, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, a.epi.A, a.N, a.M, a.epi.lda, 64, 32);
+  if (tma_ok && p.st_ad)
+    tma_ok = make_map2(&mAd, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, a.epi.Ad, a.N, a.M, a.epi.lda, 64, 32);
+  p.tma_store = tma_ok ? 1 : 0;
+
+  int need = stages * off;
+  if (p.tma_store && 4 * STG_WARP > need) need = 4 * STG_WARP;
+  const int smem = need + 1024;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(tc2_dual_gemm_kernel<BN, MODE, ACT>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, 225 * 1024);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  if (smem > 225 * 1024) { *why = "shared memory budget exceeded"; return cudaErrorInvalidValue; }
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3(2 * pairs_m, tiles_n, nb);
+  cfg.blockDim = dim3(THREADS, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = g_pdl ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, tc2_dual_gemm_kernel<BN, MODE, ACT>, mA0, mA1, mB0, mB1, mC0,
+                            mC1, mA, mAd, p);
+}
+
 // Dispatch over the tile width for one epilogue (MODE, ACT).
+// pair = 1 selects the 2-SM tile (bn 128 or 256).
 template <int MODE, int ACT>
-cudaError_t launch_bn(const GemmArgs& a, cudaStream_t s, const char** why, int bn, int ka) {
-  (void)ka;
+cudaError_t launch_bn(const GemmArgs& a, cudaStream_t s, const char** why, int bn, int pair) {
+  if (pair) {
+    if (bn == 128) return launch_cfg2<128, MODE, ACT>(a, s, why);
+    if (bn == 256) return launch_cfg2<256, MODE, ACT>(a, s, why);
+    *why = "2-SM tiles are 128 or 256 columns wide";
+    return cudaErrorInvalidValue;
+  }
   switch (bn) {
     case 16: return launch_cfg<16, 1, MODE, ACT>(a, s, why);
     case 32: return launch_cfg<32, 1, MODE, ACT>(a, s, why);

@@ -65,3 +65,28 @@ def test_dual_gemm_strided_operands():
     ref = A0[:, :K].double().cpu() @ B0[:, :K].double().cpu().T
     assert rel_l2(C0[:, :N].cpu().numpy(), ref.numpy()) < 1e-5
     assert float(C0[:, N:].abs().max()) == 0.0
+
+
+def _set_pair_mode(native, value):
+    """MF_OPT_GEMM_2SM is process-wide; any handle can set it."""
+    from paper_2505_00793_gb300 import synth
+    mf = native.MixFlow.for_workload(synth.WORKLOADS["tiny"])
+    mf.set_option(native.MF_OPT_GEMM_2SM, value)
+    mf.close()
+
+
+PAIR_SHAPES = [(256, 1024, 1024), (1024, 1024, 512), (130, 300, 8), (512, 4096, 256),
+               (300, 16, 40), (600, 520, 200), (256, 256, 64), (1000, 130, 1096)]
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("shape", PAIR_SHAPES)
+@pytest.mark.parametrize("mask", MASKS)
+def test_dual_gemm_pair_tiles(shape, mask):
+    """The same products on 256-row tiles computed by CTA pairs (tcgen05 cta_group::2)."""
+    torch, native = need_gpu()
+    _set_pair_mode(native, 2)
+    try:
+        test_dual_gemm(shape, mask)
+    finally:
+        _set_pair_mode(native, 1)

@@ -264,3 +264,17 @@ def test_launch_options_bit_identical(option):
         mf.close()
     for k in (1, 2):
         assert np.array_equal(outs[0][0], outs[k][0]) and np.array_equal(outs[0][1], outs[k][1])
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name", ["wide_small", "wide_split", "mlp_ex_slr"])
+def test_meta_grad_bf16_pair_tiles(name):
+    """Every GEMM with more than 128 rows on 256-row CTA-pair tiles."""
+    torch, native = need_gpu()
+    mf = native.MixFlow.for_workload(synth.WORKLOADS["tiny"])
+    mf.set_option(native.MF_OPT_GEMM_2SM, 2)
+    try:
+        _check(BF16_CASES[name], 2e-2)
+    finally:
+        mf.set_option(native.MF_OPT_GEMM_2SM, 1)
+        mf.close()
