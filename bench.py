@@ -8,6 +8,11 @@ seeded synthetic data resident in HBM when the timed region starts.
 
 Prints one JSON line (rank 0).  ``--impl reference`` times the CPU float64 oracle instead.
 Multi-GPU runs are independent replicas (weak scaling), one process per GPU under torchrun.
+
+``--workload`` measures another configuration the same way (deep MLP, the two decoder-only
+transformers); ``--hvp-mode rr`` runs the reverse-over-reverse sweep instead of the
+mixed-mode one (MLPs), for the memory comparison.  Those lines skip the CPU baseline unless
+``--cpu-baseline`` is given.
 """
 from __future__ import annotations
 
@@ -25,8 +30,19 @@ sys.path.insert(0, ROOT)
 
 WORKLOAD = "wide"
 REF_T_SAMPLE = 4
-WORKLOAD_DESC = ("wide MLP 1024-1024x4-10 GELU, softmax-CE, B=256, T=16 SGD alpha=0.05, "
-                 "per-example weight logits (4096), outer batch 1024, bf16 GEMMs / fp32 state")
+WORKLOAD_DESCS = {
+    "wide": ("wide MLP 1024-1024x4-10 GELU, softmax-CE, B=256, T=16 SGD alpha=0.05, "
+             "per-example weight logits (4096), outer batch 1024, bf16 GEMMs / fp32 state"),
+    "deep": ("deep MLP 8 x 4096 SiLU, squared loss on a teacher, B=512, T=32 momentum 0.9, "
+             "per-parameter log learning rates (134M), outer batch 512, bf16 GEMMs / fp32 state"),
+    "decoder_small": ("decoder-only transformer 6 x d512, 8 heads, MLP 2048 GELU, vocab 8192, "
+                      "S=256, B=16 sequences, T=8 SGD alpha=1e-3, per-sequence weights, outer 16, "
+                      "Zipf(1.1) token ids, bf16 GEMMs / fp32 state"),
+    "decoder_large": ("decoder-only transformer 12 x d1024, 16 heads, MLP 4096 GELU, vocab 32768, "
+                      "S=1024, B=8, T=16 momentum 0.9, per-sequence weights + scalar log-lr, outer 8, "
+                      "Zipf(1.1) token ids, bf16 GEMMs / fp32 state"),
+}
+WORKLOAD_DESC = WORKLOAD_DESCS[WORKLOAD]
 
 
 def _dist():
@@ -146,11 +162,12 @@ def run_gpu(args):
     torch.cuda.set_device(local)
     if ws > 1:
         dist.init_process_group("nccl")
-    w = synth.WORKLOADS[WORKLOAD]
+    w = synth.WORKLOADS[args.workload]
     inp = synth.make_inputs(w)
     d = native.to_device_inputs(w, inp)
     mf = native.MixFlow.for_workload(w)
-    loop = native.loop_desc_for(w)
+    rr = args.hvp_mode == "rr"
+    loop = native.loop_desc_for(w, native.MF_HVP_REV_REV if rr else native.MF_HVP_MIXED_FOR)
     d_eta = torch.empty(w.n_eta, device="cuda")
     V = torch.empty(1, device="cuda")
     stream = torch.cuda.current_stream()
@@ -209,6 +226,7 @@ def run_gpu(args):
         e0.record(stream)
         step()
         e1.record(stream)
+        e1.synchronize()
         ms_, n_, fl_ = mf.kernel_time()
         g_ms += ms_; g_n += n_; g_flops += fl_
         t_ms += e0.elapsed_time(e1)
@@ -251,11 +269,17 @@ def run_gpu(args):
 
     inputs_bytes = h2d
     peak_hbm_gb = (peak_ws + inputs_bytes + w.n_eta * 4) / 1e9
+    # static part (Section 4's accounting): the theta_t store (and m_t store when the learning
+    # rate is a meta-parameter), the inputs, eta and d eta; the rest is the sweep's dynamic memory
+    lr_meta = bool(w.meta_kind & (synth.PARAM_LOGLR | synth.SCALAR_LOGLR))
+    store = (w.T + 1 + (w.T if lr_meta else 0)) * w.n_params * 4
+    static_gb = (store + inputs_bytes + w.n_eta * 4) / 1e9
 
     out = None
     if rank == 0:
         cpu = None
-        if ws == 1 and not args.no_cpu_baseline:
+        default = args.workload == WORKLOAD and not rr
+        if ws == 1 and not args.no_cpu_baseline and (default or args.cpu_baseline):
             full_s, spent, cores = cpu_oracle_time(w)
             cpu = {"value": 1.0 / full_s, "unit": "meta-steps/s", "cores": cores, "kind": "oracle",
                    "sample": f"one full oracle meta-gradient of the workload (T=16, {spent:.1f} s "
@@ -265,7 +289,9 @@ def run_gpu(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic",
-            "config": {"workload": WORKLOAD_DESC, "parallelism": f"replicas x{ws}",
+            "config": {"workload": WORKLOAD_DESCS[args.workload]
+                       + ("; reverse-over-reverse HVPs" if rr else ""),
+                       "parallelism": f"replicas x{ws}",
                        "l2": "flushed before every timed step (256 MB write outside the step events)"},
             "roofline": {"bound": "tensor", "kernel": "tc_dual_gemm_kernel (tcgen05 dual GEMM)",
                          "achieved": g_tflops, "peak": peak_tc, "unit": "TFLOP/s",
@@ -276,6 +302,9 @@ def run_gpu(args):
                          "share_of_step": g_ms / max(t_ms, 1e-9)},
             "hvp_tflops": g_tflops,
             "peak_hbm_gb": peak_hbm_gb,
+            "hbm": {"total_gb": peak_hbm_gb, "static_gb": static_gb,
+                    "dynamic_gb": peak_hbm_gb - static_gb,
+                    "hvp_mode": "reverse-over-reverse" if rr else "mixed forward-over-reverse"},
             "cpu_baseline": cpu,
             "e2e": {"value": ws * 1000.0 / e2e_ms, "unit": "meta-steps/s",
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
@@ -297,6 +326,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="mixflow", choices=["mixflow", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-baseline", action="store_true",
+                    help="also time the oracle for a non-default workload or mode")
+    ap.add_argument("--workload", default=WORKLOAD, choices=sorted(WORKLOAD_DESCS))
+    ap.add_argument("--hvp-mode", default="for", choices=["for", "rr"])
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

@@ -37,7 +37,9 @@ namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;                 // bf16 elements per 128-byte swizzle row
 constexpr int MAX_STAGES = 8;
-constexpr int THREADS = 192;
+constexpr int EPI_WARPS = 8;                     // two per TMEM lane quadrant
+constexpr int EPI_THREADS = 32 * EPI_WARPS;
+constexpr int THREADS = 64 + EPI_THREADS;        // producer warp, MMA warp, epilogue
 constexpr long long WAIT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
 
 struct TcParams {
@@ -214,8 +216,8 @@ __device__ __forceinline__ void st_dsmem4(uint32_t remote_addr, float a, float b
                : "memory");
 }
 
-__device__ __forceinline__ void epi_bar() {   // the 4 epilogue warps only
-  asm volatile("bar.sync 1, 128;" ::: "memory");
+__device__ __forceinline__ void epi_bar() {   // the epilogue warps only
+  asm volatile("bar.sync 1, %0;" ::"n"(EPI_THREADS) : "memory");
 }
 
 // Row-per-thread epilogue for 16 consecutive columns (no split): float32 outputs, the
@@ -326,7 +328,8 @@ template <int BN, int MODE, int ACT>
 __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMap* mC0,
                                              const CUtensorMap* mC1, const CUtensorMap* mA,
                                              const CUtensorMap* mAd, uint8_t* stg, uint32_t taddr,
-                                             int q, int lane, int m0, int n0, bool dual, int bz) {
+                                             int q, int lane, int m0, int n0, bool dual, int bz,
+                                             int c_begin, int c_end) {
   const EpiParams e = p.epi;
   const int row = m0 + q * 32 + lane;
   const bool rowok = row < p.M;
@@ -337,8 +340,8 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
   const int sw = lane & 7;
   __nv_bfloat16* AT = static_cast<__nv_bfloat16*>(e.AT);
   __nv_bfloat16* AdT = static_cast<__nv_bfloat16*>(e.AdT);
-  for (int c = 0; c < BN; c += 64) {
-    if (c > 0) {
+  for (int c = c_begin; c < c_end; c += 64) {
+    if (c > c_begin) {
       if (lane == 0) bulk_wait_read();
       __syncwarp();
     }
@@ -459,6 +462,9 @@ __device__ __forceinline__ void mma_loop(const MmaLoop& L, unsigned terms_rt, in
   constexpr uint32_t idesc = idesc_bf16(PAIR ? 2 * BM : BM, BN);
   const unsigned terms = TERMS ? TERMS : terms_rt;
   const uint32_t nsub = NSUB ? static_cast<uint32_t>(NSUB) : static_cast<uint32_t>(nsub_rt);
+  // products into C0 / C1 per K slice
+  const uint32_t p0 = __popc(terms & (T_C0_A0B0 | T_C0_A1B0 | T_C0_A0B1 | T_C0_A1B1));
+  const uint32_t p1 = __popc(terms & (T_C1_A1B0 | T_C1_A0B1));
   for (int i = 0; i < L.nk; ++i) {
     const int s = i % L.stages;
     const uint32_t ph = (i / L.stages) & 1;
@@ -473,21 +479,26 @@ __device__ __forceinline__ void mma_loop(const MmaLoop& L, unsigned terms_rt, in
       const uint64_t b1 = L.b1_off >= 0 ? sdesc_sw128(st + L.b1_off + a * B_ATOM) : 0;
 #pragma unroll
       for (int kk = 0; kk < BK / 16; ++kk) {
+        // The j-th product of K slice kk into accumulator c goes to block
+        // (kk * P_c + j) mod nsub (P_c products into c per slice); the first product into
+        // a block overwrites it.
         const uint64_t adv = static_cast<uint64_t>(kk * 2);   // 32 bytes per K=16 step
-        const uint32_t blk = static_cast<uint32_t>(kk) & (nsub - 1);
-        const uint32_t t0 = L.tbase + blk * BN, t1 = L.tbase + (nsub + blk) * BN;
-        uint32_t f0 = (i == 0 && a == 0 && static_cast<uint32_t>(kk) < nsub) ? 0u : 1u;
-        uint32_t f1 = f0;
-        auto mma = [&](uint32_t d, uint64_t ad, uint64_t bd, uint32_t f) {
-          if constexpr (PAIR) mma_bf16_pair(d, ad, bd, idesc, f);
-          else mma_bf16(d, ad, bd, idesc, f);
+        const bool first = i == 0 && a == 0;
+        uint32_t q0 = static_cast<uint32_t>(kk) * p0, q1 = static_cast<uint32_t>(kk) * p1;
+        auto mma = [&](uint32_t c, uint64_t ad, uint64_t bd) {
+          uint32_t& q = c ? q1 : q0;
+          const uint32_t blk = c * nsub + (q & (nsub - 1));
+          const uint32_t f = (first && q < nsub) ? 0u : 1u;
+          ++q;
+          if constexpr (PAIR) mma_bf16_pair(L.tbase + blk * BN, ad, bd, idesc, f);
+          else mma_bf16(L.tbase + blk * BN, ad, bd, idesc, f);
         };
-        if (terms & T_C0_A0B0) { mma(t0, a0 + adv, b0 + adv, f0); f0 = 1; }
-        if (terms & T_C1_A1B0) { mma(t1, a1 + adv, b0 + adv, f1); f1 = 1; }
-        if (terms & T_C0_A1B0) { mma(t0, a1 + adv, b0 + adv, f0); f0 = 1; }
-        if (terms & T_C1_A0B1) { mma(t1, a0 + adv, b1 + adv, f1); f1 = 1; }
-        if (terms & T_C0_A0B1) { mma(t0, a0 + adv, b1 + adv, f0); f0 = 1; }
-        if (terms & T_C0_A1B1) { mma(t0, a1 + adv, b1 + adv, f0); f0 = 1; }
+        if (terms & T_C0_A0B0) mma(0, a0 + adv, b0 + adv);
+        if (terms & T_C1_A1B0) mma(1, a1 + adv, b0 + adv);
+        if (terms & T_C0_A1B0) mma(0, a1 + adv, b0 + adv);
+        if (terms & T_C1_A0B1) mma(1, a0 + adv, b1 + adv);
+        if (terms & T_C0_A0B1) mma(0, a0 + adv, b1 + adv);
+        if (terms & T_C0_A1B1) mma(0, a1 + adv, b1 + adv);
       }
     }
     if constexpr (PAIR) mma_commit_pair(&L.empty_bar[s]);
@@ -627,20 +638,24 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     __syncwarp();
   } else {
-    // ---- accumulator drain: warps 2..5, TMEM lane quadrant = warp % 4 ---------------
+    // ---- accumulator drain: TMEM lane quadrant = warp % 4; the two warps of a quadrant
+    // take one column half each (tiles of 128 or more columns) --------------------------
     const int q = warp & 3;
     const int r = q * 32 + lane;   // row within the tile
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    const int half = (warp - 2) >> 2;
+    const int c_begin = BN >= 128 ? half * (BN / 2) : 0;
+    const int c_end = BN >= 128 ? c_begin + BN / 2 : (half == 0 ? BN : 0);
     const bool ok = nk > 0 && mbar_wait(&acc_bar, 0, p.status);
     tc_fence_after();
     if (S == 1) {
       if (ok) {
         if (p.tma_store) {
-          epilogue_tma<BN, MODE, ACT>(p, &tmC0, &tmC1, &tmA, &tmAd, smem + q * STG_WARP, tbase + lane_off,
-                           q, lane, m0, n0, dual, bz);
+          epilogue_tma<BN, MODE, ACT>(p, &tmC0, &tmC1, &tmA, &tmAd, smem + (warp - 2) * STG_WARP,
+                                      tbase + lane_off, q, lane, m0, n0, dual, bz, c_begin, c_end);
         } else {
 #pragma unroll 1
-          for (int c = 0; c < BN; c += 16) {
+          for (int c = c_begin; c < c_end; c += 16) {
             float v0[16], v1[16];
             ld_acc16<BN>(tbase + lane_off, 0, p.nsub, c, v0);
             if (dual) ld_acc16<BN>(tbase + lane_off, 1, p.nsub, c, v1);
@@ -674,6 +689,9 @@ __global__ void __launch_bounds__(THREADS, 1)
       const int q = warp & 3;
       const int r = q * 32 + lane;
       const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+      const int half = (warp - 2) >> 2;
+      const int c_begin = BN >= 32 ? half * (BN / 2) : 0;
+      const int c_end = BN >= 32 ? c_begin + BN / 2 : (half == 0 ? BN : 0);
       const bool ok = nk > 0;
       const uint32_t owner = static_cast<uint32_t>(r / rows_per);
       const int rr = r % rows_per;
@@ -681,7 +699,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         const uint32_t row_addr = dsmem_addr(
             rbase + static_cast<uint32_t>((((a * S + z) * rows_per + rr) * LDP) * 4), owner);
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 16) {
+        for (int c = c_begin; c < c_end; c += 16) {
           float v[16];
           if (ok) {
             ld_acc16<BN>(tbase + lane_off, a, p.nsub, c, v);
@@ -699,7 +717,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncwarp();
     cluster_sync_all();   // every partial row has reached its owner
     if (warp >= 2) {
-      const int e = threadIdx.x - 64;            // 0..127
+      const int e = threadIdx.x - 64;            // 0 .. EPI_THREADS-1
       const int r_begin = static_cast<int>(z) * rows_per;
       float* Rcv = reinterpret_cast<float*>(smem);          // [acc][S][rows_per][LDP]
       float* R = Rcv + nacc * BM * LDP;                     // reduced rows [acc][rows_per][LDP]
@@ -707,7 +725,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       constexpr int VPR = BN / 4;                // float4 per row
       const int nvec = rows_per * VPR;
       for (int a = 0; a < nacc; ++a) {
-        for (int it = e; it < nvec; it += 128) {
+        for (int it = e; it < nvec; it += EPI_THREADS) {
           const int rr = it / VPR, c4 = (it % VPR) * 4;
           float4 acc = *reinterpret_cast<const float4*>(Rcv + ((a * S) * rows_per + rr) * LDP + c4);
           for (int k = 1; k < S; ++k) {
@@ -721,15 +739,16 @@ __global__ void __launch_bounds__(THREADS, 1)
       // Phase B: fused epilogue, one column per thread, 8-row chunks (the transposed bf16
       // operand gets one 16-byte store per chunk; row-major stores are coalesced across
       // consecutive columns)
-      const int tpc = 128 / (BN < 128 ? BN : 128);   // threads per column
+      constexpr int CW = BN < EPI_THREADS ? BN : EPI_THREADS;
+      const int tpc = EPI_THREADS / CW;          // threads per column
       const EpiParams ep = p.epi;
       __nv_bfloat16* AT = static_cast<__nv_bfloat16*>(ep.AT);
       __nv_bfloat16* AdT = static_cast<__nv_bfloat16*>(ep.AdT);
       __nv_bfloat16* A = static_cast<__nv_bfloat16*>(ep.A);
       __nv_bfloat16* Ad = static_cast<__nv_bfloat16*>(ep.Ad);
-      for (int col = e % BN; col < BN; col += 128) {
+      for (int col = e % BN; col < BN; col += EPI_THREADS) {
         const int n = n0 + col;
-        for (int ch = (e % 128) / (BN < 128 ? BN : 128); ch * 8 < rows_per; ch += tpc) {
+        for (int ch = e / CW; ch * 8 < rows_per; ch += tpc) {
           float t0[8], t1[8];
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
@@ -918,7 +937,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
     const int partial_bytes = (dual ? 2 : 1) * (BM + BM / S) * (BN + 4) * 4;
     if (partial_bytes > need) need = partial_bytes;
   }
-  if (p.tma_store && 4 * STG_WARP > need) need = 4 * STG_WARP;
+  if (p.tma_store && EPI_WARPS * STG_WARP > need) need = EPI_WARPS * STG_WARP;
   const int smem = need + 1024;
   static bool attr_set = false;
   if (!attr_set) {
@@ -1062,19 +1081,21 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     __syncwarp();
   } else {
-    // accumulator drain: this CTA's 128 rows of the pair tile, TMEM lane quadrant = warp % 4
+    // accumulator drain: this CTA's 128 rows of the pair tile, TMEM lane quadrant = warp % 4,
+    // one column half per warp of a quadrant
     const int q = warp & 3;
     const int r = q * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    const int c_begin = ((warp - 2) >> 2) * (BN / 2), c_end = c_begin + BN / 2;
     const bool ok = mbar_wait(&acc_bar, 0, p.status);
     tc_fence_after();
     if (ok) {
       if (p.tma_store) {
-        epilogue_tma<BN, MODE, ACT>(p, &tmC0, &tmC1, &tmA, &tmAd, smem + q * STG_WARP,
-                                    tbase + lane_off, q, lane, m0, n0, dual, bz);
+        epilogue_tma<BN, MODE, ACT>(p, &tmC0, &tmC1, &tmA, &tmAd, smem + (warp - 2) * STG_WARP,
+                                    tbase + lane_off, q, lane, m0, n0, dual, bz, c_begin, c_end);
       } else {
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 16) {
+        for (int c = c_begin; c < c_end; c += 16) {
           float v0[16], v1[16];
           ld_acc16<BN>(tbase + lane_off, 0, p.nsub, c, v0);
           if (dual) ld_acc16<BN>(tbase + lane_off, 1, p.nsub, c, v1);
@@ -1167,7 +1188,7 @@ cudaError_t launch_cfg2(const GemmArgs& a, cudaStream_t s, const char** why) {
   p.tma_store = tma_ok ? 1 : 0;
 
   int need = stages * off;
-  if (p.tma_store && 4 * STG_WARP > need) need = 4 * STG_WARP;
+  if (p.tma_store && EPI_WARPS * STG_WARP > need) need = EPI_WARPS * STG_WARP;
   const int smem = need + 1024;
   static bool attr_set = false;
   if (!attr_set) {
