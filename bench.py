@@ -107,6 +107,24 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def _dram_traffic():
+    """DRAM bytes per launch of the dominant kernel from the committed ncu capture, or None
+    when the kernel's sources changed since the counters were taken."""
+    import hashlib
+    try:
+        with open(os.path.join(ROOT, "profiles", "tc_dual_gemm_wide_traffic.json")) as f:
+            rec = json.load(f)
+        h = hashlib.sha256()
+        for name in rec["source_files"]:
+            with open(os.path.join(ROOT, name), "rb") as src:
+                h.update(src.read())
+        if h.hexdigest() != rec["source_sha256"]:
+            return None
+        return rec["traffic_bytes_per_launch"]
+    except Exception:
+        return None
+
+
 def cpu_oracle_time(w, t_sample=None):
     """Wall time of the float64 oracle meta-gradient on workload w, run on the first
     ``t_sample`` inner steps (all T when None) and scaled by T / t_sample.  Scaling also
@@ -295,7 +313,8 @@ def run_gpu(args):
                        "l2": "flushed before every timed step (256 MB write outside the step events)"},
             "roofline": {"bound": "tensor", "kernel": "tc_dual_gemm_kernel (tcgen05 dual GEMM)",
                          "achieved": g_tflops, "peak": peak_tc, "unit": "TFLOP/s",
-                         "frac": g_tflops / peak_tc, "traffic": None,
+                         "frac": g_tflops / peak_tc,
+                         "traffic": _dram_traffic() if args.workload == WORKLOAD else None,
                          "peak_source": f"{peak_src} bf16_tflops_sustained",
                          "launches_per_step": g_n / max(args.steps, 1),
                          "avg_launch_us": 1000.0 * g_ms / max(g_n, 1),
