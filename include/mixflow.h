@@ -116,7 +116,8 @@ typedef struct {
  *             (Algorithm 2, the mixed-mode sweep).  MF_HVP_REV_REV: reverse-over-reverse
  *             (Algorithm 1's schedule: the inner backward is kept whole and differentiated
  *             again in reverse), the standard-AD baseline; same result, more workspace.
- *             MF_HVP_REV_REV is implemented for MF_ARCH_MLP only (UNSUPPORTED otherwise).
+ *             MLPs keep every layer's dz and da; the decoder keeps the residual-stream
+ *             cotangent at every block output and recomputes the cotangents inside a block.
  *  ckpt_every 1 = keep every theta_t in the checkpoint store (the only value accepted). */
 typedef struct {
   int T, B, B_outer;
@@ -164,8 +165,7 @@ mf_status mf_inner_rollout(mf_handle h, const mf_loop_desc* loop, const float* t
  *   Hv [P]             = (d^2 L / d theta^2) v        (forward-over-reverse)
  *   tangent_losses [B] = grad l_b(theta) . v           (nullable; the mixed term per example)
  *   grad [P]           = grad L(theta)                 (nullable)
- * hvp_mode MF_HVP_MIXED_FOR (forward-over-reverse) or MF_HVP_REV_REV (reverse-over-reverse,
- * MLP models only; returns MF_ERR_UNSUPPORTED for the decoder). */
+ * hvp_mode MF_HVP_MIXED_FOR (forward-over-reverse) or MF_HVP_REV_REV (reverse-over-reverse). */
 mf_status mf_hvp(mf_handle h, int B, const float* theta, const void* x, const void* y,
                  const float* ex_w, const float* v, float* Hv, float* tangent_losses,
                  float* grad, int hvp_mode, void* stream);

@@ -683,8 +683,7 @@ mf_status validate_loop(mf_ctx* h, const mf_loop_desc* lp) {
     return fail(h, MF_ERR_INVALID_ARG, "momentum must be in [0, 1)");
   if (lp->hvp_mode != MF_HVP_MIXED_FOR && lp->hvp_mode != MF_HVP_REV_REV)
     return fail(h, MF_ERR_INVALID_ARG, "unknown hvp_mode");
-  if (lp->hvp_mode == MF_HVP_REV_REV && h->decoder)
-    return fail(h, MF_ERR_UNSUPPORTED, "reverse-over-reverse is implemented for MLP models");
+
   if (lp->ckpt_every != 1 && lp->ckpt_every != 0)
     return fail(h, MF_ERR_UNSUPPORTED, "only ckpt_every = 1 is implemented");
   return MF_OK;
@@ -919,7 +918,7 @@ template <typename E, typename F>
 mf_status with_exec(mf_ctx* h, int rows, int T, int theta_slots, int m_slots, bool partials,
                     bool ror, cudaStream_t s, F&& f) {
   if (h->decoder) {
-    DecPlan plan = make_dec_plan(h, h->Ly, rows, T, theta_slots, m_slots, partials);
+    DecPlan plan = make_dec_plan(h, h->Ly, rows, T, theta_slots, m_slots, partials, ror);
     mf_status st = ensure_ws(h, plan.bytes, s);
     if (st != MF_OK) return st;
     DecExec<E> ex(h, plan, h->Ly, s);
@@ -1095,7 +1094,8 @@ mf_status mf_workspace_bytes(mf_handle h, const mf_loop_desc* lp, size_t* bytes)
   const bool lr_meta = lp->meta_kind & (MF_META_PARAM_LOGLR | MF_META_SCALAR_LOGLR);
   if (h->decoder) {
     *bytes = make_dec_plan(h, h->Ly, std::max(lp->B, lp->B_outer), lp->T, lp->T + 1,
-                           lr_meta ? lp->T : 0, lp->meta_kind & MF_META_SCALAR_LOGLR).bytes;
+                           lr_meta ? lp->T : 0, lp->meta_kind & MF_META_SCALAR_LOGLR,
+                           lp->hvp_mode == MF_HVP_REV_REV).bytes;
     return MF_OK;
   }
   *bytes = make_plan(h, std::max(lp->B, lp->B_outer), lp->T, lp->T + 1, lr_meta ? lp->T : 0,
@@ -1142,8 +1142,7 @@ mf_status mf_hvp(mf_handle h, int B, const float* theta, const void* x, const vo
   if (B < 1) return fail(h, MF_ERR_INVALID_ARG, "B must be >= 1");
   if (hvp_mode != MF_HVP_MIXED_FOR && hvp_mode != MF_HVP_REV_REV)
     return fail(h, MF_ERR_INVALID_ARG, "unknown hvp_mode");
-  if (hvp_mode == MF_HVP_REV_REV && h->decoder)
-    return fail(h, MF_ERR_UNSUPPORTED, "reverse-over-reverse is implemented for MLP models");
+
   const bool ror = hvp_mode == MF_HVP_REV_REV;
   if (!theta || !x || !y || !v || !Hv) return fail(h, MF_ERR_INVALID_ARG, "NULL tensor argument");
   mf_status st = check_x(h, x, B);

@@ -54,11 +54,16 @@ struct DecPlan {
   size_t dOh = 0, dOhd = 0, dOhT = 0, dOhdT = 0, dP = 0, dPd = 0, dS = 0, dSd = 0, dST = 0,
          dSdT = 0, PT = 0, PdT = 0, dQ = 0, dQd = 0, dK = 0, dKd = 0, dV = 0, dVd = 0;
   size_t dqkv = 0, dqkvd = 0, dqkvT = 0, dqkvdT = 0, dz1 = 0, dz1d = 0, dz1T = 0, dz1dT = 0;
+  // reverse-over-reverse: the inner backward's residual-stream cotangent at the output of
+  // every block (the stored reverse graph, at block granularity)
+  bool ror = false;
+  std::vector<size_t> dxs;
 };
 
 DecPlan make_dec_plan(const mf_ctx* h, const DecLayout& Ly, int rows, int T, int n_theta_slots,
-                      int n_m_slots, bool with_partials) {
+                      int n_m_slots, bool with_partials, bool ror = false) {
   DecPlan p;
+  p.ror = ror;
   p.rows = rows;
   p.N = rows * Ly.S;
   p.ldN = ld8(p.N);
@@ -138,6 +143,8 @@ DecPlan make_dec_plan(const mf_ctx* h, const DecLayout& Ly, int rows, int T, int
   const size_t head4 = static_cast<size_t>(BH) * S * Ly.dh * 4;
   p.dQ = take(head4); p.dQd = take(head4); p.dK = take(head4); p.dKd = take(head4);
   p.dV = take(head4); p.dVd = take(head4);
+  if (ror)
+    for (int l = 0; l < Ly.L; ++l) p.dxs.push_back(take(Nd4));
   p.dqkv = take(N * 3 * d * es); p.dqkvd = take(N * 3 * d * es);
   p.dqkvT = take(3 * d * p.ldN * es); p.dqkvdT = take(3 * d * p.ldN * es);
   p.dz1 = take(N * F * es); p.dz1d = take(N * F * es);
@@ -161,6 +168,9 @@ struct DecExec {
   bool dual_cur = false;
   const float* theta_cur = nullptr;
   const float* u_cur = nullptr;
+  // reverse-over-reverse: 1 = the primal backward stores each block's output cotangent,
+  // 2 = the second-order backward restarts every block from the stored cotangent
+  int ror_mode = 0;
 
   DecExec(mf_ctx* h_, const DecPlan& p_, const DecLayout& L_, cudaStream_t s_)
       : h(h_), p(p_), Ly(L_), s(s_), base(static_cast<char*>(h_->ws)) {
@@ -452,6 +462,7 @@ struct DecExec {
   // weight product into out (grad) / outh (tangent): [A^T][seed] with K = tokens
   void wprod(int M, int Nn, const T* AT_, const T* AdT_, const T* ST_, const T* SdT_, bool dual,
              float* outg, float* outh) {
+    if (!dual && !outg) return;   // primal backward kept only for its cotangents
     GemmArgs g;
     g.M = M; g.N = Nn; g.K = rows_cur * Ly.S;
     g.A0 = AT_; g.A1 = AdT_; g.lda0 = g.lda1 = p.ldN;
@@ -509,6 +520,13 @@ struct DecExec {
                       at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr, G(Ly.gf), Hh(Ly.gf), s);
     launched(2);
     for (int l = Ly.L - 1; l >= 0; --l) {
+      if (ror_mode == 1) {
+        cudaMemcpyAsync(at<float>(p.dxs[l]), at<float>(p.dx), static_cast<size_t>(N) * d * 4,
+                        cudaMemcpyDeviceToDevice, s);
+      } else if (ror_mode == 2) {
+        cudaMemcpyAsync(at<float>(p.dx), at<float>(p.dxs[l]), static_cast<size_t>(N) * d * 4,
+                        cudaMemcpyDeviceToDevice, s);
+      }
       // ---- MLP branch: seed = dx -------------------------------------------------------
       seed_from(at<float>(p.dx), at<float>(p.dxd), dual);
       wprod(F, d, at<T>(p.a1T[l]), at<T>(p.a1dT[l]), at<T>(p.dyT), at<T>(p.dydT), dual, G(Ly.W2[l]),
@@ -641,10 +659,25 @@ struct DecExec {
     chk("decoder backward");
   }
 
-  // Reverse-over-reverse is built for MLP models only; the entry points reject it for the
-  // decoder before an executor exists, so this is never reached.
-  void ror_hvp(int, const void*, const float*, const float*, const void*, const float*,
-               const float*, float*, float*, float*, float*) {
-    st = MF_ERR_UNSUPPORTED;
+  // Hessian-vector product by reverse-over-reverse (Algorithm 1's schedule) at block
+  // granularity: primal forward and primal backward, which stores the residual-stream
+  // cotangent at the output of every block (the reverse graph); then the tangent pass in
+  // forward order (the adjoint of the backward, by the symmetry of Eqs. 6-7) and the
+  // second-order backward in reverse order, which restarts each block from its stored
+  // cotangent and recomputes the cotangents inside the block (block rematerialisation of
+  // the inner backward, the granularity at which the forward keeps its activations).
+  void ror_hvp(int rows, const void* x, const float* theta, const float* u, const void* y,
+               const float* eta_w, const float* ex_w, float* Hv, float* grad, float* ld_out,
+               float* d_eta) {
+    forward(rows, x, theta, nullptr, false);
+    loss(rows, false, y, eta_w, ex_w, nullptr, nullptr, nullptr);
+    ror_mode = 1;
+    backward(rows, false, nullptr, grad);
+    ror_mode = 0;
+    forward(rows, x, theta, u, true);
+    loss(rows, true, y, eta_w, ex_w, nullptr, ld_out, d_eta);
+    ror_mode = 2;
+    backward(rows, true, Hv, nullptr);
+    ror_mode = 0;
   }
 };

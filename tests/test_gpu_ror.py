@@ -3,9 +3,9 @@
 The two modes compute the same mathematical object (Eqs. 6-7: the Hessian is symmetric, so
 differentiating the backward pass in reverse equals pushing a tangent forward through it).
 Checked here: each mode against the float64 oracle, the two modes against each other at
-float32 (where only the summation order differs), the full meta-gradient in both modes,
-graph replay, and that the stored backward graph makes reverse-over-reverse need more
-workspace than the mixed-mode sweep."""
+float32 (where only the summation order differs), the full meta-gradient in both modes for
+MLPs and the decoder, graph replay, and that the stored backward graph makes
+reverse-over-reverse need more workspace than the mixed-mode sweep."""
 import numpy as np
 import pytest
 
@@ -129,10 +129,38 @@ def test_ror_needs_more_workspace():
 
 
 @pytest.mark.gpu
-def test_ror_rejected_for_decoder():
+@pytest.mark.parametrize("name,tol,tol_modes", [("dec32_a", 1e-4, 1e-5), ("dec32_mom", 1e-4, 1e-5),
+                                               ("dec16_small", 2e-2, 5e-3), ("dec16_mom", 2e-2, 5e-3)])
+def test_ror_decoder_meta_grad(name, tol, tol_modes):
+    """Decoder reverse-over-reverse (block-granular reverse graph): against the oracle, and
+    against the mixed-mode sweep (float32: same arithmetic up to summation order; bf16: the
+    primal-only and dual GEMMs may tile differently)."""
+    from test_gpu_decoder import BF16 as DBF16, FP32 as DFP32
+    w = DFP32.get(name) or DBF16[name]
+    inp = synth.make_inputs(w)
+    ref = om.meta_grad(w, inp)
+    (de_r, dt_r, V_r), ws_r = _meta(w, inp, REVREV)
+    (de_m, dt_m, _), ws_m = _meta(w, inp, MIXED)
+    assert rel_l2(de_r, ref["d_eta"]) < tol
+    assert rel_l2(dt_r, ref["d_theta0"]) < tol
+    assert abs(V_r - ref["V"]) <= tol * abs(ref["V"])
+    assert rel_l2(de_r, de_m) < tol_modes
+    assert rel_l2(dt_r, dt_m) < tol_modes
+    assert ws_r > ws_m
+
+
+@pytest.mark.gpu
+def test_ror_decoder_hvp():
     torch, native = need_gpu()
-    w = synth.WORKLOADS["decoder_small"]
-    mf = native.MixFlow.for_workload(w)
-    with pytest.raises(RuntimeError, match="UNSUPPORTED"):
-        mf.workspace_bytes(native.loop_desc_for(w, hvp_mode=REVREV))
-    mf.close()
+    from test_gpu_decoder import FP32 as DFP32
+    w = DFP32["dec32_mom"]
+    inp = synth.make_inputs(w)
+    v = synth.random_direction(w.n_params, 5, 11)
+    wt = np.linspace(0.25, 1.0, w.B).astype(np.float32)
+    hv_r, g_r, tl_r = _hvp(w, inp, REVREV, v, wt)
+    hv_m, g_m, tl_m = _hvp(w, inp, MIXED, v, wt)
+    x, y = inp.inner_x[0], inp.inner_y[0]
+    assert rel_l2(hv_r, om.hvp(w, inp.theta0, x, y, v, wt)) < 1e-4
+    assert rel_l2(hv_r, hv_m) < 1e-5
+    assert rel_l2(g_r, g_m) < 1e-5
+    assert rel_l2(tl_r, tl_m) < 1e-5
