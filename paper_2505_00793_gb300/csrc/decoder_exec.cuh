@@ -39,7 +39,7 @@ struct DecPlan {
   int nb = 0;
   size_t bytes = 0;
   size_t o_theta = 0, o_m = 0, o_g = 0, o_tbar = 0, o_u = 0, o_part = 0, o_l = 0, o_ld = 0;
-  size_t o_count = 0, o_start = 0, o_order = 0;
+  size_t o_count = 0, o_start = 0, o_order = 0, o_order_tmp = 0, gpart = 0;
   // per tensor operand copies (index = tensor index; 0 when not cast)
   std::vector<size_t> o_W, o_WT, o_U, o_UT;
   // per block activations
@@ -88,6 +88,8 @@ DecPlan make_dec_plan(const mf_ctx* h, const DecLayout& Ly, int rows, int T, int
   p.o_count = take(static_cast<size_t>(V) * 4);
   p.o_start = take(static_cast<size_t>(V + 1) * 4);
   p.o_order = take(static_cast<size_t>(N) * 4);
+  p.o_order_tmp = take(static_cast<size_t>(N) * 4);
+  p.gpart = take(static_cast<size_t>(2) * mf::dec_gain_chunks(static_cast<int>(N)) * d * 4);
   for (const auto& t : tens) {
     if (t.cast) {
       p.o_W.push_back(take(static_cast<size_t>(t.rows) * ld8(t.cols) * es));
@@ -501,7 +503,8 @@ struct DecExec {
     const float* u = u_cur;
     auto G = [&](int64_t off) { return out_g ? out_g + off : nullptr; };
     auto Hh = [&](int64_t off) { return dual ? out_h + off : nullptr; };
-    mf::dec_token_csr(N, S, V, ids_cur, at<int>(p.o_count), at<int>(p.o_start), at<int>(p.o_order), s);
+    mf::dec_token_csr(N, S, V, ids_cur, at<int>(p.o_count), at<int>(p.o_start), at<int>(p.o_order),
+                      at<int>(p.o_order_tmp), s);
     launched(3);
     // head: dWh = hf^T dF ; dhf = dF Wh^T
     wprod(d, V, at<T>(p.hfT), at<T>(p.hfdT), at<T>(p.dFT), at<T>(p.dFdT), dual, G(Ly.Wh), Hh(Ly.Wh));
@@ -517,7 +520,8 @@ struct DecExec {
                            theta_cur + Ly.gf, dual ? u + Ly.gf : nullptr, at<float>(p.dh),
                            dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx), at<float>(p.dxd), s);
     mf::dec_gain_grad(N, d, at<float>(p.xf), at<float>(p.xfd), at<float>(p.rf), at<float>(p.rfd),
-                      at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr, G(Ly.gf), Hh(Ly.gf), s);
+                      at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr, G(Ly.gf), Hh(Ly.gf),
+                      at<float>(p.gpart), s);
     launched(2);
     for (int l = Ly.L - 1; l >= 0; --l) {
       if (ror_mode == 1) {
@@ -556,7 +560,7 @@ struct DecExec {
       }
       mf::dec_gain_grad(N, d, at<float>(p.x2[l]), at<float>(p.x2d[l]), at<float>(p.r2[l]),
                         at<float>(p.r2d[l]), at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr,
-                        G(Ly.g2[l]), Hh(Ly.g2[l]), s);
+                        G(Ly.g2[l]), Hh(Ly.g2[l]), at<float>(p.gpart), s);
       mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.x2[l]), at<float>(p.x2d[l]), at<float>(p.r2[l]),
                              at<float>(p.r2d[l]), theta_cur + Ly.g2[l], dual ? u + Ly.g2[l] : nullptr,
                              at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx),
@@ -646,7 +650,7 @@ struct DecExec {
       }
       mf::dec_gain_grad(N, d, at<float>(p.x1[l]), at<float>(p.x1d[l]), at<float>(p.r1[l]),
                         at<float>(p.r1d[l]), at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr,
-                        G(Ly.g1[l]), Hh(Ly.g1[l]), s);
+                        G(Ly.g1[l]), Hh(Ly.g1[l]), at<float>(p.gpart), s);
       mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.x1[l]), at<float>(p.x1d[l]), at<float>(p.r1[l]),
                              at<float>(p.r1d[l]), theta_cur + Ly.g1[l], dual ? u + Ly.g1[l] : nullptr,
                              at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx),

@@ -159,22 +159,26 @@ __global__ void rmsnorm_bwd_kernel(int d, const float* __restrict__ x, const flo
   }
 }
 
-// Gain gradients: dg_j = sum_r dy_rj n_rj ;  dg'_j = sum_r (dy'_rj n_rj + dy_rj n'_rj).
-// Block (32 columns x 32 row lanes); each lane sums a strided set of rows, then the 32
-// partials are added in a fixed order (deterministic).
-__global__ void gain_grad_kernel(int N, int d, const float* __restrict__ x,
-                                 const float* __restrict__ xd, const float* __restrict__ rr,
-                                 const float* __restrict__ rrd, const float* __restrict__ dy,
-                                 const float* __restrict__ dyd, float* __restrict__ dg,
-                                 float* __restrict__ dgd) {
+// RMSNorm gain gradient: dg[j] = sum_r dy[r][j] x[r][j] r_r (and its tangent), as a
+// fixed-order two-stage reduction: stage 1 sums 256-row chunks (one partial row per chunk),
+// stage 2 sums the chunk partials in chunk order.
+constexpr int GG_ROWS = 256;
+
+__global__ void gain_grad_partial_kernel(int N, int d, const float* __restrict__ x,
+                                         const float* __restrict__ xd, const float* __restrict__ rr,
+                                         const float* __restrict__ rrd, const float* __restrict__ dy,
+                                         const float* __restrict__ dyd, float* __restrict__ part,
+                                         float* __restrict__ partd) {
   pdl_entry();
-  __shared__ float sp[32][33];
-  __shared__ float spd[32][33];
+  __shared__ float sp[8][33];
+  __shared__ float spd[8][33];
   const int j = blockIdx.x * 32 + threadIdx.x;
+  const int r0 = blockIdx.y * GG_ROWS;
+  const int r1 = min(N, r0 + GG_ROWS);
   const bool dual = dyd != nullptr;
   float a = 0.f, ad = 0.f;
   if (j < d) {
-    for (int r = threadIdx.y; r < N; r += 32) {
+    for (int r = r0 + threadIdx.y; r < r1; r += 8) {
       const int64_t o = static_cast<int64_t>(r) * d + j;
       const float n = x[o] * rr[r];
       a += dy[o] * n;
@@ -188,11 +192,27 @@ __global__ void gain_grad_kernel(int N, int d, const float* __restrict__ x,
   spd[threadIdx.y][threadIdx.x] = ad;
   __syncthreads();
   if (threadIdx.y == 0 && j < d) {
-    float s = 0.f, sd = 0.f;
-    for (int k = 0; k < 32; ++k) { s += sp[k][threadIdx.x]; sd += spd[k][threadIdx.x]; }
-    if (dg) dg[j] = s;
-    if (dual && dgd) dgd[j] = sd;
+    float t = 0.f, td = 0.f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) { t += sp[k][threadIdx.x]; td += spd[k][threadIdx.x]; }
+    part[static_cast<int64_t>(blockIdx.y) * d + j] = t;
+    if (dual) partd[static_cast<int64_t>(blockIdx.y) * d + j] = td;
   }
+}
+
+__global__ void gain_grad_final_kernel(int nchunk, int d, const float* __restrict__ part,
+                                       const float* __restrict__ partd, float* __restrict__ dg,
+                                       float* __restrict__ dgd) {
+  pdl_entry();
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j >= d) return;
+  float t = 0.f, td = 0.f;
+  for (int c = 0; c < nchunk; ++c) {
+    t += part[static_cast<int64_t>(c) * d + j];
+    if (partd) td += partd[static_cast<int64_t>(c) * d + j];
+  }
+  if (dg) dg[j] = t;
+  if (partd && dgd) dgd[j] = td;
 }
 
 // RoPE (rotate-half) on q and k, q scaled by 1/sqrt(dh), head split.  qkv [N][3d] float32
@@ -490,20 +510,40 @@ __global__ void scan_kernel(int V, const int* __restrict__ count, int* __restric
   }
 }
 
-// Stable placement: token r goes to start[id] + (number of earlier tokens with the same id).
-__global__ void token_place_kernel(int N, int S, int V, const int* __restrict__ ids,
-                                   const int* __restrict__ start, int* __restrict__ order) {
+// Placement in two steps: every token takes a free slot of its id's segment (atomic, any
+// order), then each segment is put in position order (stable, deterministic): an entry's
+// rank is the number of entries of the segment at earlier positions.
+__global__ void token_scatter_kernel(int N, int S, int V, const int* __restrict__ ids,
+                                     const int* __restrict__ start, int* __restrict__ count,
+                                     int* __restrict__ tmp) {
   pdl_entry();
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= N) return;
-  auto id_of = [&](int t) {
-    int v = ids[static_cast<int64_t>(t / S) * (S + 1) + t % S];
-    return (v < 0 || v >= V) ? 0 : v;
-  };
-  const int id = id_of(r);
-  int rank = 0;
-  for (int t = 0; t < r; ++t) rank += id_of(t) == id;
-  order[start[id] + rank] = r;
+  int id = ids[static_cast<int64_t>(r / S) * (S + 1) + r % S];
+  if (id < 0 || id >= V) id = 0;
+  const int slot = atomicSub(&count[id], 1) - 1;
+  tmp[start[id] + slot] = r;
+}
+
+constexpr int SEG_SMEM = 4096;
+
+__global__ void token_order_kernel(const int* __restrict__ start, const int* __restrict__ tmp,
+                                   int* __restrict__ order) {
+  pdl_entry();
+  __shared__ int seg[SEG_SMEM];
+  const int v = blockIdx.x;
+  const int a = start[v], L = start[v + 1] - a;
+  if (L == 0) return;
+  const bool staged = L <= SEG_SMEM;
+  if (staged)
+    for (int i = threadIdx.x; i < L; i += blockDim.x) seg[i] = tmp[a + i];
+  __syncthreads();
+  for (int i = threadIdx.x; i < L; i += blockDim.x) {
+    const int pi = staged ? seg[i] : tmp[a + i];
+    int rank = 0;
+    for (int k = 0; k < L; ++k) rank += (staged ? seg[k] : tmp[a + k]) < pi;
+    order[a + rank] = pi;
+  }
 }
 
 // dE[v] = sum over tokens with id v (in position order) of dx[token]; one block per id.
@@ -591,9 +631,18 @@ void dec_rmsnorm_bwd(int N, int d, const float* x, const float* xd, const float*
   launch_k(rmsnorm_bwd_kernel<T>, dim3(N), dim3(256), 0, s, d, x, xd, r, rd, g, gd, dy, dyd, dx, dxd);
 }
 
+int dec_gain_chunks(int N) { return (N + GG_ROWS - 1) / GG_ROWS; }
+
 void dec_gain_grad(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
-                   const float* dy, const float* dyd, float* dg, float* dgd, cudaStream_t s) {
-  launch_k(gain_grad_kernel, dim3((d + 31) / 32), dim3(dim3(32, 32)), 0, s, N, d, x, xd, r, rd, dy, dyd, dg, dgd);
+                   const float* dy, const float* dyd, float* dg, float* dgd, float* part,
+                   cudaStream_t s) {
+  if (!dg && !(dyd && dgd)) return;
+  const int nchunk = dec_gain_chunks(N);
+  float* partd = dyd ? part + static_cast<int64_t>(nchunk) * d : nullptr;
+  launch_k(gain_grad_partial_kernel, dim3((d + 31) / 32, nchunk), dim3(32, 8), 0, s, N, d, x, xd,
+           r, rd, dy, dyd, part, partd);
+  launch_k(gain_grad_final_kernel, dim3((d + 255) / 256), dim3(256), 0, s, nchunk, d, part, partd,
+           dg, dgd);
 }
 
 template <typename T>
@@ -650,11 +699,13 @@ void dec_seq_reduce(int B, int S, const float* l, const float* ld, const float* 
 }
 
 void dec_token_csr(int N, int S, int V, const int* ids, int* count, int* start, int* order,
-                   cudaStream_t s) {
+                   int* tmp, cudaStream_t s) {
   cudaMemsetAsync(count, 0, sizeof(int) * V, s);
   launch_k(token_count_kernel, dim3((N + 255) / 256), dim3(256), 0, s, N, S, V, ids, count);
   launch_k(scan_kernel, dim3(1), dim3(1024), 0, s, V, count, start);
-  launch_k(token_place_kernel, dim3((N + 255) / 256), dim3(256), 0, s, N, S, V, ids, start, order);
+  launch_k(token_scatter_kernel, dim3((N + 255) / 256), dim3(256), 0, s, N, S, V, ids, start,
+           count, tmp);
+  launch_k(token_order_kernel, dim3(V), dim3(256), 0, s, start, tmp, order);
 }
 
 void dec_embed_bwd(int V, int d, const int* start, const int* order, const float* dx,

@@ -161,8 +161,11 @@ template <typename T>
 void dec_rmsnorm_bwd(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
                      const float* g, const float* gd, const float* dy, const float* dyd, float* dx,
                      float* dxd, cudaStream_t s);
+int dec_gain_chunks(int N);
+// part: scratch of 2 * dec_gain_chunks(N) * d floats
 void dec_gain_grad(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
-                   const float* dy, const float* dyd, float* dg, float* dgd, cudaStream_t s);
+                   const float* dy, const float* dyd, float* dg, float* dgd, float* part,
+                   cudaStream_t s);
 template <typename T>
 void dec_rope_split(int N, int S, int H, int dh, float base, float qscale, const float* qkv, T* Q,
                     T* K, T* V, cudaStream_t s);
@@ -187,8 +190,9 @@ void dec_ce_seed(int N, int S, int V, const int* ids, const float* F, const floa
                  float inv_norm, T* dF, T* dFd, int ldo, cudaStream_t s);
 void dec_seq_reduce(int B, int S, const float* l, const float* ld, const float* eta_w, float invB,
                     float* l_seq, float* ld_seq, float* d_eta, cudaStream_t s);
+// tmp: scratch of N ints
 void dec_token_csr(int N, int S, int V, const int* ids, int* count, int* start, int* order,
-                   cudaStream_t s);
+                   int* tmp, cudaStream_t s);
 void dec_embed_bwd(int V, int d, const int* start, const int* order, const float* dx,
                    const float* dxd, float* dE, float* dEd, cudaStream_t s);
 template <typename TI, typename TO>
