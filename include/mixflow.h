@@ -252,6 +252,8 @@ mf_status mf_hvp_noalloc(const mf_model_desc* desc, int B, const float* theta, c
  *   bit 3: C1 += A1 B0^T   bit 4: C1 += A0 B1^T   bit 5: C0 += A1 B1^T
  * The forward tangent of a dual Linear layer is terms = 1|8|16:  C0 = A0 B0^T (primal),
  * C1 = A1 B0^T + A0 B1^T (tangent).  bias0/bias1 [N] float32 are added when non-NULL.
+ * Layout flags in the same word: bit 8 - A0, A1 are MN-major, stored [K][M] (element (m, k)
+ * at k * lda + m, lda >= M); bit 9 - B0, B1 are MN-major, stored [K][N] (ldb >= N).
  * Runs on tcgen05 tensor cores with TMEM accumulators and TMA-fed shared memory. */
 mf_status mf_dual_gemm_bf16(int M, int N, int K, const void* A0, int lda0, const void* A1,
                             int lda1, const void* B0, int ldb0, const void* B1, int ldb1,

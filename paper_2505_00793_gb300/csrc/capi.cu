@@ -96,18 +96,18 @@ mf_status fail(mf_ctx* h, mf_status s, const std::string& msg) {
 // ---- workspace layout -------------------------------------------------------------------
 struct Plan {
   int rows = 0;          // max rows of any batch
-  int ldR = 0;           // leading dim of transposed activations (multiple of 8)
   int T = 0;
   int n_theta_slots = 0, n_m_slots = 0;
   int nb = 0;            // blocks (tiles) of the per-layer update kernel
   size_t bytes = 0;
   size_t o_theta = 0, o_m = 0, o_g = 0, o_tbar = 0, o_u = 0, o_part = 0, o_l = 0, o_ld = 0;
-  std::vector<size_t> o_Wb, o_WbT, o_Ub, o_UbT, o_A, o_Ad, o_AT, o_AdT, o_Z, o_Zd;
-  size_t o_dZ[2] = {0, 0}, o_dZd[2] = {0, 0}, o_dZT[2] = {0, 0}, o_dZdT[2] = {0, 0};
+  std::vector<size_t> o_Wb, o_Ub, o_A, o_Ad, o_Z, o_Zd;
+  std::vector<int> lda;  // leading dim of layer l's input activations (room for the bias column)
+  size_t o_dZ[2] = {0, 0}, o_dZd[2] = {0, 0};
   // reverse-over-reverse: the stored reverse graph (per-layer dz, da) and the adjoints
   bool ror = false;
-  std::vector<size_t> o_SZ, o_SZT, o_SA, o_DAB, o_DABT, o_ZP;
-  size_t o_DZB = 0, o_ZB = 0, o_ZBT = 0, o_AB = 0;
+  std::vector<size_t> o_SZ, o_SA, o_DAB, o_ZP;
+  size_t o_DZB = 0, o_ZB = 0, o_AB = 0;
 };
 
 int n_update_tiles(const mf_ctx* h) {
@@ -119,14 +119,15 @@ int n_update_tiles(const mf_ctx* h) {
   return tiles;
 }
 
-// Transposed activations carry one extra row (ones for a, zeros for a') so that the weight
-// product [a^T; 1][dz] yields the weight and the bias gradient (stored contiguously in theta).
+// Activations a [rows][din] carry one extra column (ones for a, zeros for a') so that the
+// weight product [a 1]^T dz, read MN-major straight from the row-major activations, yields
+// the weight and the bias gradient (stored contiguously in theta).  No operand is stored
+// transposed: the forward product reads W [din][dout] MN-major as well.
 Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slots,
                bool with_partials, bool ror = false) {
   Plan p;
   p.ror = ror;
   p.rows = rows;
-  p.ldR = ld8(rows);
   p.T = T;
   p.n_theta_slots = n_theta_slots;
   p.n_m_slots = n_m_slots;
@@ -145,19 +146,15 @@ Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slot
   p.o_l = take(static_cast<size_t>(rows) * 4);
   p.o_ld = take(static_cast<size_t>(rows) * 4);
   const int L = h->L;
-  p.o_Wb.resize(L); p.o_WbT.resize(L); p.o_Ub.resize(L); p.o_UbT.resize(L);
-  p.o_A.resize(L); p.o_Ad.resize(L); p.o_AT.resize(L); p.o_AdT.resize(L);
-  p.o_Z.resize(L); p.o_Zd.resize(L);
+  p.o_Wb.resize(L); p.o_Ub.resize(L); p.o_A.resize(L); p.o_Ad.resize(L);
+  p.o_Z.resize(L); p.o_Zd.resize(L); p.lda.resize(L);
   for (int l = 0; l < L; ++l) {
     const int din = h->dims[l], dout = h->dims[l + 1];
+    p.lda[l] = ld8(din + hb);
     p.o_Wb[l] = take(static_cast<size_t>(din) * ld8(dout) * es);
-    p.o_WbT[l] = take(static_cast<size_t>(dout) * ld8(din) * es);
     p.o_Ub[l] = take(static_cast<size_t>(din) * ld8(dout) * es);
-    p.o_UbT[l] = take(static_cast<size_t>(dout) * ld8(din) * es);
-    p.o_A[l] = take(static_cast<size_t>(rows) * ld8(din) * es);
-    p.o_Ad[l] = take(static_cast<size_t>(rows) * ld8(din) * es);
-    p.o_AT[l] = take(static_cast<size_t>(din + hb) * p.ldR * es);
-    p.o_AdT[l] = take(static_cast<size_t>(din + hb) * p.ldR * es);
+    p.o_A[l] = take(static_cast<size_t>(rows) * p.lda[l] * es);
+    p.o_Ad[l] = take(static_cast<size_t>(rows) * p.lda[l] * es);
     p.o_Z[l] = take(static_cast<size_t>(rows) * dout * 4);
     p.o_Zd[l] = take(static_cast<size_t>(rows) * dout * 4);
   }
@@ -165,24 +162,18 @@ Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slot
   for (int b = 0; b < 2; ++b) {
     p.o_dZ[b] = take(static_cast<size_t>(rows) * ld8(md) * es);
     p.o_dZd[b] = take(static_cast<size_t>(rows) * ld8(md) * es);
-    p.o_dZT[b] = take(static_cast<size_t>(md) * p.ldR * es);
-    p.o_dZdT[b] = take(static_cast<size_t>(md) * p.ldR * es);
   }
   if (ror) {
-    p.o_SZ.resize(L); p.o_SZT.resize(L); p.o_SA.resize(L); p.o_DAB.resize(L); p.o_DABT.resize(L);
-    p.o_ZP.resize(L);
+    p.o_SZ.resize(L); p.o_SA.resize(L); p.o_DAB.resize(L); p.o_ZP.resize(L);
     for (int l = 0; l < L; ++l) {
       const int din = h->dims[l], dout = h->dims[l + 1];
       p.o_SZ[l] = take(static_cast<size_t>(rows) * ld8(dout) * es);
-      p.o_SZT[l] = take(static_cast<size_t>(dout) * p.ldR * es);
       p.o_SA[l] = take(static_cast<size_t>(rows) * din * 4);
-      p.o_DAB[l] = take(static_cast<size_t>(rows) * ld8(dout) * es);
-      p.o_DABT[l] = take(static_cast<size_t>(dout + 1) * p.ldR * es);
+      p.o_DAB[l] = take(static_cast<size_t>(rows) * ld8(dout + hb) * es);
       p.o_ZP[l] = take(static_cast<size_t>(rows) * dout * 4);
     }
     p.o_DZB = take(static_cast<size_t>(rows) * md * 4);
     p.o_ZB = take(static_cast<size_t>(rows) * ld8(md) * es);
-    p.o_ZBT = take(static_cast<size_t>(md) * p.ldR * es);
     p.o_AB = take(static_cast<size_t>(rows) * md * 4);
   }
   p.bytes = o;
@@ -330,7 +321,6 @@ struct Exec {
 
   // backward seed buffers of layer l (ping-pong, or the stored reverse graph)
   T* dz_buf(int l) const { return ror_store ? at<T>(p.o_SZ[l]) : at<T>(p.o_dZ[l & 1]); }
-  T* dzT_buf(int l) const { return ror_store ? at<T>(p.o_SZT[l]) : at<T>(p.o_dZT[l & 1]); }
 
   Exec(mf_ctx* h_, const Plan& p_, cudaStream_t s_)
       : h(h_), p(p_), s(s_), base(static_cast<char*>(h_->ws)) {
@@ -345,11 +335,11 @@ struct Exec {
       tab.tile0[l] = tiles;
       tiles += ((tab.rows[l] + 31) / 32) * ((dout + 31) / 32);
       tab.ldw[l] = ld8(dout);
-      tab.ldwt[l] = ld8(din);
+      tab.ldwt[l] = 0;
       tab.W[l] = at<T>(p.o_Wb[l]);
-      tab.WT[l] = at<T>(p.o_WbT[l]);
+      tab.WT[l] = nullptr;         // every product reads W row-major (K- or MN-major)
       tab.U[l] = at<T>(p.o_Ub[l]);
-      tab.UT[l] = at<T>(p.o_UbT[l]);
+      tab.UT[l] = nullptr;
     }
     tab.tile0[h->L] = tiles;
   }
@@ -419,21 +409,22 @@ struct Exec {
     }
   }
 
-  // Bias rows of the augmented transposed activations (ones for a, zeros for a').
+  // Bias columns of the augmented activations (ones for a, zeros for a' and for the
+  // reverse-over-reverse adjoint activations).
   void prepare() {
     if (!h->md.has_bias) return;
-    mf::RowFill f;
+    mf::ColFill f;
     for (int l = 0; l < h->L; ++l) {
-      f.dst[f.n] = at<T>(p.o_AT[l]); f.row[f.n] = h->dims[l]; f.ld[f.n] = p.ldR; f.value[f.n] = 1.f; ++f.n;
-      f.dst[f.n] = at<T>(p.o_AdT[l]); f.row[f.n] = h->dims[l]; f.ld[f.n] = p.ldR; f.value[f.n] = 0.f; ++f.n;
+      f.dst[f.n] = at<T>(p.o_A[l]); f.col[f.n] = h->dims[l]; f.ld[f.n] = p.lda[l]; f.value[f.n] = 1.f; ++f.n;
+      f.dst[f.n] = at<T>(p.o_Ad[l]); f.col[f.n] = h->dims[l]; f.ld[f.n] = p.lda[l]; f.value[f.n] = 0.f; ++f.n;
     }
     if (p.ror) {
       for (int l = 0; l + 1 < h->L; ++l) {
-        f.dst[f.n] = at<T>(p.o_DABT[l]); f.row[f.n] = h->dims[l + 1]; f.ld[f.n] = p.ldR;
+        f.dst[f.n] = at<T>(p.o_DAB[l]); f.col[f.n] = h->dims[l + 1]; f.ld[f.n] = p.lda[l + 1];
         f.value[f.n] = 0.f; ++f.n;
       }
     }
-    mf::fill_rows<T>(f, p.ldR, s);
+    mf::fill_cols<T>(f, p.rows, s);
     launched();
   }
 
@@ -454,20 +445,24 @@ struct Exec {
   // Forward pass of `rows` examples: primal (z) or dual (z, z_dot along u).  Hidden layers
   // fuse bias, activation and its tangent into the GEMM epilogue.
   void forward(int rows, const void* xv, const float* theta, const float* u, bool dual) {
-    const T* x = static_cast<const T*>(xv);
     const int din0 = h->dims[0];
-    mf::transpose<T>(x, rows, din0, din0, at<T>(p.o_AT[0]), p.ldR, s);
-    launched();
+    const size_t es = sizeof(T);
+    // inputs into the augmented layer-0 activations (the bias column is already set)
+    if (cudaMemcpy2DAsync(at<T>(p.o_A[0]), p.lda[0] * es, xv, din0 * es, din0 * es, rows,
+                          cudaMemcpyDeviceToDevice, s) != cudaSuccess && st == MF_OK) {
+      st = MF_ERR_CUDA;
+      h->err = "input copy failed";
+    }
     for (int l = 0; l < h->L; ++l) {
       const int din = h->dims[l], dout = h->dims[l + 1];
       GemmArgs g;
       g.M = rows; g.N = dout; g.K = din;
-      g.A0 = l == 0 ? static_cast<const void*>(x) : at<T>(p.o_A[l]);
-      g.lda0 = l == 0 ? din : ld8(din);
+      g.A0 = at<T>(p.o_A[l]); g.lda0 = p.lda[l];
       g.A1 = l == 0 ? nullptr : at<T>(p.o_Ad[l]);
-      g.lda1 = ld8(din);
-      g.B0 = at<T>(p.o_WbT[l]); g.ldb0 = ld8(din);
-      g.B1 = at<T>(p.o_UbT[l]); g.ldb1 = ld8(din);
+      g.lda1 = p.lda[l];
+      g.B0 = at<T>(p.o_Wb[l]); g.ldb0 = ld8(dout);   // W [din][dout]: MN-major
+      g.B1 = at<T>(p.o_Ub[l]); g.ldb1 = ld8(dout);
+      g.b_mn = true;
       g.C0 = at<float>(p.o_Z[l]); g.ldc0 = dout;
       g.bias0 = h->md.has_bias ? theta + h->boff[l] : nullptr;
       g.terms = mf::T_C0_A0B0;
@@ -481,10 +476,7 @@ struct Exec {
         g.epi.act = h->md.act;
         g.epi.A = at<T>(p.o_A[l + 1]);
         g.epi.Ad = dual ? at<T>(p.o_Ad[l + 1]) : nullptr;
-        g.epi.lda = ld8(dout);
-        g.epi.AT = at<T>(p.o_AT[l + 1]);
-        g.epi.AdT = dual ? at<T>(p.o_AdT[l + 1]) : nullptr;
-        g.epi.ldt = p.ldR;
+        g.epi.lda = p.lda[l + 1];
       }
       gemm(g);
     }
@@ -510,12 +502,6 @@ struct Exec {
     a.status = h->d_status;
     mf::loss_seed<T>(a, s);
     launched();
-    mf::transpose<T>(dz_buf(L - 1), rows, C, ld8(C), dzT_buf(L - 1), p.ldR, s);
-    launched();
-    if (dual) {
-      mf::transpose<T>(at<T>(p.o_dZd[b]), rows, C, ld8(C), at<T>(p.o_dZdT[b]), p.ldR, s);
-      launched();
-    }
   }
 
   // Backward pass.  Primal: out_g = grad L.  Dual: out_h = H u (and out_g = grad L if given).
@@ -525,12 +511,15 @@ struct Exec {
     const int hb = h->md.has_bias ? 1 : 0;
     for (int l = h->L - 1; l >= 0; --l) {
       const int din = h->dims[l], dout = h->dims[l + 1], b = l & 1;
+      // [a 1]^T dz and [a' 0]^T dz + [a 1]^T dz': activations [rows][din+1] and seeds
+      // [rows][dout] are read MN-major (K = rows)
       GemmArgs g;
       g.M = din + hb; g.N = dout; g.K = rows;
-      g.A0 = at<T>(p.o_AT[l]); g.lda0 = p.ldR;
-      g.A1 = at<T>(p.o_AdT[l]); g.lda1 = p.ldR;
-      g.B0 = dzT_buf(l); g.ldb0 = p.ldR;
-      g.B1 = at<T>(p.o_dZdT[b]); g.ldb1 = p.ldR;
+      g.A0 = at<T>(p.o_A[l]); g.lda0 = p.lda[l];
+      g.A1 = at<T>(p.o_Ad[l]); g.lda1 = p.lda[l];
+      g.B0 = dz_buf(l); g.ldb0 = ld8(dout);
+      g.B1 = at<T>(p.o_dZd[b]); g.ldb1 = ld8(dout);
+      g.a_mn = g.b_mn = true;
       if (!dual) {
         g.terms = mf::T_C0_A0B0;
         g.C0 = out_g + h->woff[l]; g.ldc0 = dout;
@@ -564,9 +553,6 @@ struct Exec {
       d.epi.A = dz_buf(l - 1);
       d.epi.Ad = dual ? at<T>(p.o_dZd[b ^ 1]) : nullptr;
       d.epi.lda = ld8(din);
-      d.epi.AT = dzT_buf(l - 1);
-      d.epi.AdT = dual ? at<T>(p.o_dZdT[b ^ 1]) : nullptr;
-      d.epi.ldt = p.ldR;
       // The weight product reads layer l's seeds and writes its slice of the output; the
       // data product reads the same seeds and writes layer l-1's (the other ping-pong set):
       // they are independent and run side by side, joined before layer l-1 overwrites.
@@ -600,20 +586,20 @@ struct Exec {
       const int din = h->dims[l], dout = h->dims[l + 1];
       GemmArgs g;
       g.M = rows; g.N = dout; g.K = din;
-      g.A0 = l == 0 ? x : static_cast<const void*>(at<T>(p.o_A[l]));
-      g.lda0 = l == 0 ? din : ld8(din);
+      g.A0 = at<T>(p.o_A[l]); g.lda0 = p.lda[l];
       g.A1 = l == 0 ? nullptr : at<T>(p.o_DAB[l - 1]);
-      g.lda1 = ld8(din);
-      g.B0 = at<T>(p.o_WbT[l]); g.ldb0 = ld8(din);
-      g.B1 = at<T>(p.o_UbT[l]); g.ldb1 = ld8(din);
+      g.lda1 = p.lda[l];
+      g.B0 = at<T>(p.o_Wb[l]); g.ldb0 = ld8(dout);
+      g.B1 = at<T>(p.o_Ub[l]); g.ldb1 = ld8(dout);
+      g.b_mn = true;
       g.terms = mf::T_C0_A0B1 | (l > 0 ? mf::T_C0_A1B0 : 0u);
       g.C0 = at<float>(p.o_DZB); g.ldc0 = dout;
       g.bias0 = h->md.has_bias ? u + h->boff[l] : nullptr;
       gemm(g);
       if (l + 1 < L) {
         mf::ror_fwd_elem<T>(h->md.act, at<float>(p.o_DZB), at<float>(p.o_Z[l]),
-                            at<float>(p.o_SA[l + 1]), rows, dout, at<T>(p.o_DAB[l]), ld8(dout),
-                            at<T>(p.o_DABT[l]), p.ldR, at<float>(p.o_ZP[l]), s);
+                            at<float>(p.o_SA[l + 1]), rows, dout, at<T>(p.o_DAB[l]), p.lda[l + 1],
+                            nullptr, 0, at<float>(p.o_ZP[l]), s);
         launched();
       } else {
         // loss Hessian along dzbar (this is the forward tangent of the logits): zbar_{L-1},
@@ -633,8 +619,6 @@ struct Exec {
         a.status = h->d_status;
         mf::loss_seed<T>(a, s);
         launched();
-        mf::transpose<T>(at<T>(p.o_ZB), rows, dout, ld8(dout), at<T>(p.o_ZBT), p.ldR, s);
-        launched();
       }
     }
     // adjoint of the forward pass, layers L-1..0
@@ -642,16 +626,17 @@ struct Exec {
       const int din = h->dims[l], dout = h->dims[l + 1];
       if (l + 1 < L) {
         mf::ror_bwd_elem<T>(h->md.act, at<float>(p.o_ZP[l]), at<float>(p.o_AB), at<float>(p.o_Z[l]),
-                            rows, dout, at<T>(p.o_ZB), ld8(dout), at<T>(p.o_ZBT), p.ldR, s);
+                            rows, dout, at<T>(p.o_ZB), ld8(dout), nullptr, 0, s);
         launched();
       }
       // (H v)_{W_l, b_l} = [a_{l-1}^T; 1] zbar_l + [dabar_{l-1}^T; 0] dz_l
       GemmArgs g;
       g.M = din + hb; g.N = dout; g.K = rows;
-      g.A0 = at<T>(p.o_AT[l]); g.lda0 = p.ldR;
-      g.A1 = l > 0 ? at<T>(p.o_DABT[l - 1]) : nullptr; g.lda1 = p.ldR;
-      g.B0 = at<T>(p.o_ZBT); g.ldb0 = p.ldR;
-      g.B1 = at<T>(p.o_SZT[l]); g.ldb1 = p.ldR;
+      g.A0 = at<T>(p.o_A[l]); g.lda0 = p.lda[l];
+      g.A1 = l > 0 ? at<T>(p.o_DAB[l - 1]) : nullptr; g.lda1 = p.lda[l];
+      g.B0 = at<T>(p.o_ZB); g.ldb0 = ld8(dout);
+      g.B1 = at<T>(p.o_SZ[l]); g.ldb1 = ld8(dout);
+      g.a_mn = g.b_mn = true;
       g.terms = mf::T_C0_A0B0 | (l > 0 ? mf::T_C0_A1B1 : 0u);
       g.C0 = Hv + h->woff[l]; g.ldc0 = dout;
       gemm(g);
@@ -1303,6 +1288,9 @@ mf_status mf_dual_gemm_bf16(int M, int N, int K, const void* A0, int lda0, const
                             int lda1, const void* B0, int ldb0, const void* B1, int ldb1,
                             float* C0, int ldc0, const float* bias0, float* C1, int ldc1,
                             const float* bias1, unsigned terms, void* stream) {
+  constexpr unsigned kAmn = 1u << 8, kBmn = 1u << 9;
+  const bool a_mn = terms & kAmn, b_mn = terms & kBmn;
+  terms &= ~(kAmn | kBmn);
   if (M < 1 || N < 1 || K < 1 || (terms & ~mf::T_ALL) || !(terms & mf::T_ALL)) return MF_ERR_INVALID_ARG;
   const bool acc0 = terms & (mf::T_C0_A0B0 | mf::T_C0_A1B0 | mf::T_C0_A0B1 | mf::T_C0_A1B1);
   const bool acc1 = terms & (mf::T_C1_A1B0 | mf::T_C1_A0B1);
@@ -1314,6 +1302,8 @@ mf_status mf_dual_gemm_bf16(int M, int N, int K, const void* A0, int lda0, const
   g.C0 = acc0 ? C0 : nullptr; g.ldc0 = ldc0; g.bias0 = bias0;
   g.C1 = acc1 ? C1 : nullptr; g.ldc1 = ldc1; g.bias1 = bias1;
   g.terms = terms;
+  g.a_mn = a_mn;
+  g.b_mn = b_mn;
   const char* why = "";
   cudaError_t e = mf::tc_gemm(g, static_cast<cudaStream_t>(stream), &why);
   if (e == cudaErrorInvalidValue) { cudaGetLastError(); return MF_ERR_INVALID_ARG; }

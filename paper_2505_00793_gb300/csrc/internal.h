@@ -49,6 +49,9 @@ struct GemmArgs {
   int split_k = 0;         // 0 = choose automatically, else 1/2/4/8 (tensor-core path)
   int bn = 0, ka = 0;      // tile width / K atoms per stage; 0 = choose automatically
   int pair = 0;            // 2-SM tiles (tensor-core path): 0 automatic, 1 always, -1 never
+  // Operand layouts: K-major (default, X[row][k] at row * ld + k) or MN-major
+  // (X[row][k] at k * ld + row), for A0/A1 and for B0/B1.
+  bool a_mn = false, b_mn = false;
   int* status = nullptr;   // device status word (timeouts), may be null
 };
 
@@ -78,6 +81,17 @@ struct RowFill {
 };
 template <typename T>
 void fill_rows(const RowFill& f, int cols, cudaStream_t s);
+
+// Column fills: dst[n][r * ld[n] + col[n]] = value[n] for r < rows.
+struct ColFill {
+  int n = 0;
+  void* dst[64];
+  int col[64];
+  int ld[64];
+  float value[64];
+};
+template <typename T>
+void fill_cols(const ColFill& f, int rows, cudaStream_t s);
 
 struct LossArgs {
   int loss = 0;            // 0 squared, 1 softmax CE

@@ -51,6 +51,15 @@ __global__ void fill_rows_kernel(const RowFill f, int cols) {
   dst[static_cast<int64_t>(f.row[k]) * f.ld[k] + c] = to_t<T>(f.value[k]);
 }
 
+template <typename T>
+__global__ void fill_cols_kernel(const ColFill f, int rows) {
+  pdl_entry();
+  const int n = blockIdx.y;
+  T* dst = static_cast<T*>(f.dst[n]);
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < rows; r += gridDim.x * blockDim.x)
+    dst[static_cast<int64_t>(r) * f.ld[n] + f.col[n]] = to_t<T>(f.value[n]);
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -229,8 +238,8 @@ __global__ void __launch_bounds__(TILE * TROWS) layer_update_kernel(const LayerT
     const int c = c0 + i, r = r0 + tx;
     if (c < dout && r < din) {
       const int64_t o = static_cast<int64_t>(c) * tab.ldwt[l] + r;
-      if (cast_w) static_cast<T*>(tab.WT[l])[o] = to_t<T>(tw[tx][i]);
-      if (cast_u) static_cast<T*>(tab.UT[l])[o] = to_t<T>(tu[tx][i]);
+      if (cast_w && tab.WT[l]) static_cast<T*>(tab.WT[l])[o] = to_t<T>(tw[tx][i]);
+      if (cast_u && tab.UT[l]) static_cast<T*>(tab.UT[l])[o] = to_t<T>(tu[tx][i]);
     }
   }
 }
@@ -262,7 +271,7 @@ __global__ void ror_fwd_elem_kernel(int act, const float* __restrict__ dzbar,
   __syncthreads();
   for (int i = ty; i < TILE; i += TROWS) {
     const int c = c0 + i, r = r0 + tx;
-    if (c < cols && r < rows) dabT[static_cast<int64_t>(c) * ldT + r] = to_t<T>(tile[tx][i]);
+    if (dabT && c < cols && r < rows) dabT[static_cast<int64_t>(c) * ldT + r] = to_t<T>(tile[tx][i]);
   }
 }
 
@@ -291,7 +300,7 @@ __global__ void ror_bwd_elem_kernel(int act, const float* __restrict__ zpart,
   __syncthreads();
   for (int i = ty; i < TILE; i += TROWS) {
     const int c = c0 + i, r = r0 + tx;
-    if (c < cols && r < rows) zbT[static_cast<int64_t>(c) * ldT + r] = to_t<T>(tile[tx][i]);
+    if (zbT && c < cols && r < rows) zbT[static_cast<int64_t>(c) * ldT + r] = to_t<T>(tile[tx][i]);
   }
 }
 
@@ -316,6 +325,12 @@ void fill_rows(const RowFill& f, int cols, cudaStream_t s) {
   if (f.n <= 0 || cols <= 0) return;
   dim3 grid((cols + 255) / 256, f.n);
   launch_k(fill_rows_kernel<T>, dim3(grid), dim3(256), 0, s, f, cols);
+}
+
+template <typename T>
+void fill_cols(const ColFill& f, int rows, cudaStream_t s) {
+  if (f.n == 0 || rows <= 0) return;
+  launch_k(fill_cols_kernel<T>, dim3((rows + 255) / 256, f.n), dim3(256), 0, s, f, rows);
 }
 
 template <typename T>
@@ -364,6 +379,7 @@ void fill(float* p, int64_t n, float v, cudaStream_t s) {
 #define MF_INST(T)                                                                 \
   template void transpose<T>(const T*, int, int, int, T*, int, cudaStream_t);     \
   template void fill_rows<T>(const RowFill&, int, cudaStream_t);                  \
+  template void fill_cols<T>(const ColFill&, int, cudaStream_t);                  \
   template void loss_seed<T>(const LossArgs&, cudaStream_t);                      \
   template void layer_update<T>(const LayerTable&, const LayerUpdArgs&, cudaStream_t);        \
   template void ror_fwd_elem<T>(int, const float*, const float*, const float*, int, int, T*, int, \

@@ -20,6 +20,7 @@ struct SimtParams {
   unsigned terms;
   const float* A[2]; int lda[2];
   const float* B[2]; int ldb[2];
+  int a_mn, b_mn;                  // MN-major operands: X[row][k] at k * ld + row
   float* C[2]; int ldc[2]; const float* bias[2];
   EpiParams epi;
   int64_t bsA[2], bsB[2], bsC[2];   // batch strides (blockIdx.z = batch index)
@@ -51,9 +52,13 @@ __global__ void __launch_bounds__(256) simt_dual_gemm_kernel(SimtParams p) {
       for (int i = threadIdx.x; i < TM * TK; i += 256) {
         const int r = i / TK, kk = i % TK;
         const int gm = m0 + r, gk = k0 + kk;
-        As[kk][r] = (gm < p.M && gk < p.K) ? A[static_cast<int64_t>(gm) * lda + gk] : 0.f;
+        As[kk][r] = (gm < p.M && gk < p.K)
+                        ? A[p.a_mn ? static_cast<int64_t>(gk) * lda + gm : static_cast<int64_t>(gm) * lda + gk]
+                        : 0.f;
         const int gn = n0 + r;
-        Bs[kk][r] = (gn < p.N && gk < p.K) ? B[static_cast<int64_t>(gn) * ldb + gk] : 0.f;
+        Bs[kk][r] = (gn < p.N && gk < p.K)
+                        ? B[p.b_mn ? static_cast<int64_t>(gk) * ldb + gn : static_cast<int64_t>(gn) * ldb + gk]
+                        : 0.f;
       }
       __syncthreads();
 #pragma unroll
@@ -118,6 +123,8 @@ cudaError_t simt_gemm(const GemmArgs& a, cudaStream_t s) {
   p.C[0] = a.C0; p.ldc[0] = a.ldc0; p.bias[0] = a.bias0;
   p.C[1] = a.C1; p.ldc[1] = a.ldc1; p.bias[1] = a.bias1;
   p.epi = a.epi;
+  p.a_mn = a.a_mn ? 1 : 0;
+  p.b_mn = a.b_mn ? 1 : 0;
   p.bsA[0] = a.bsA0; p.bsA[1] = a.bsA1; p.bsB[0] = a.bsB0; p.bsB[1] = a.bsB1;
   p.bsC[0] = a.bsC0; p.bsC[1] = a.bsC1;
   if (a.batch > 1 && a.epi.mode != EPI_STORE) return cudaErrorInvalidValue;

@@ -36,8 +36,10 @@ cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why) {
                             T_C0_A0B0 | T_C0_A1B0 | T_C1_A1B0, T_C0_A0B1 | T_C1_A0B1 | T_C0_A1B1};
   for (int i = 0; i < 4; ++i) {
     if (!(a.terms & uses[i])) continue;
-    if (!ptrs[i] || (reinterpret_cast<uintptr_t>(ptrs[i]) & 15) || (lds[i] & 7) || lds[i] < a.K) {
-      *why = "operand pointer must be 16-byte aligned with ld a multiple of 8 and >= K";
+    const bool mn = i < 2 ? a.a_mn : a.b_mn;
+    const int minld = mn ? (i < 2 ? a.M : a.N) : a.K;   // K-major rows hold K, MN-major rows M/N
+    if (!ptrs[i] || (reinterpret_cast<uintptr_t>(ptrs[i]) & 15) || (lds[i] & 7) || lds[i] < minld) {
+      *why = "operand pointer must be 16-byte aligned with ld a multiple of 8 and >= its row length";
       return cudaErrorInvalidValue;
     }
   }
@@ -89,6 +91,7 @@ cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why) {
     else if (dual || tiles_m * ((a.N + 255) / 256) < 152) bn = 128;
     else bn = 256;
   }
+  if (a.b_mn && bn < 64) bn = 64;   // MN-major B is staged in 64-row boxes
   if (a.epi.mode == EPI_STORE) return launch_bn<EPI_STORE, ACT_IDENT>(a, s, why, bn, pair);
   return tc_gemm_act(a, s, why, bn, pair);
 }

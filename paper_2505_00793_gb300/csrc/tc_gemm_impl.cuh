@@ -53,6 +53,7 @@ struct TcParams {
   int st_c0, st_c1, st_a, st_ad;   // which row-major outputs exist
   int a0_off, a1_off, b0_off, b1_off, stage_bytes, tx_bytes;
   int nsub;               // TMEM blocks per logical accumulator (1, 2 or 4)
+  int a_mn, b_mn;         // operands stored MN-major ([K][rows]) instead of K-major
   float* C0; int ldc0; const float* bias0;
   float* C1; int ldc1; const float* bias1;
   EpiParams epi;
@@ -126,6 +127,20 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
   d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
   d |= static_cast<uint64_t>(1) << 16;              // leading byte offset (unused here)
   d |= static_cast<uint64_t>(1024 >> 4) << 32;      // stride byte offset
+  d |= static_cast<uint64_t>(1) << 46;              // version
+  d |= static_cast<uint64_t>(2) << 61;              // SWIZZLE_128B
+  return d;
+}
+
+// MN-major operand ([K][rows] in memory, rows contiguous), 128-byte swizzle, staged as
+// boxes of 64 rows x 64 K (8 KB, K rows of 128 bytes): 8-row K groups 1024 bytes apart
+// (stride byte offset), 64-row blocks 8 KB apart (leading byte offset).
+constexpr int MN_BOX = 64 * BK * 2;
+__device__ __forceinline__ uint64_t sdesc_mn_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(MN_BOX >> 4) << 16;    // leading byte offset: next 64 rows
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;      // stride byte offset: next 8 K rows
   d |= static_cast<uint64_t>(1) << 46;              // version
   d |= static_cast<uint64_t>(2) << 61;              // SWIZZLE_128B
   return d;
@@ -445,6 +460,7 @@ __device__ __forceinline__ void mma_commit_pair(uint64_t* bar) {
 
 struct MmaLoop {
   int nk, stages, stage_bytes, a0_off, a1_off, b0_off, b1_off;
+  int a_mn, b_mn;
   uint32_t sbase, tbase;
   uint64_t* full_bar;
   uint64_t* empty_bar;
@@ -459,7 +475,11 @@ struct MmaLoop {
 template <int BN, int KA, unsigned TERMS, int NSUB, bool PAIR>
 __device__ __forceinline__ void mma_loop(const MmaLoop& L, unsigned terms_rt, int nsub_rt) {
   constexpr int A_ATOM = BM * BK * 2, B_ATOM = (PAIR ? BN / 2 : BN) * BK * 2;
-  constexpr uint32_t idesc = idesc_bf16(PAIR ? 2 * BM : BM, BN);
+  // bits 15 / 16 of the instruction descriptor: A / B MN-major
+  const uint32_t idesc = idesc_bf16(PAIR ? 2 * BM : BM, BN) | (static_cast<uint32_t>(L.a_mn) << 15) |
+                         (static_cast<uint32_t>(L.b_mn) << 16);
+  // descriptor advance per K=16 slice, in 16-byte units: 32 bytes K-major, 16 rows MN-major
+  const uint64_t stepA = L.a_mn ? 128u : 2u, stepB = L.b_mn ? 128u : 2u;
   const unsigned terms = TERMS ? TERMS : terms_rt;
   const uint32_t nsub = NSUB ? static_cast<uint32_t>(NSUB) : static_cast<uint32_t>(nsub_rt);
   // products into C0 / C1 per K slice
@@ -473,16 +493,23 @@ __device__ __forceinline__ void mma_loop(const MmaLoop& L, unsigned terms_rt, in
     const uint32_t st = L.sbase + s * L.stage_bytes;
 #pragma unroll
     for (int a = 0; a < KA; ++a) {
-      const uint64_t a0 = L.a0_off >= 0 ? sdesc_sw128(st + L.a0_off + a * A_ATOM) : 0;
-      const uint64_t a1 = L.a1_off >= 0 ? sdesc_sw128(st + L.a1_off + a * A_ATOM) : 0;
-      const uint64_t b0 = L.b0_off >= 0 ? sdesc_sw128(st + L.b0_off + a * B_ATOM) : 0;
-      const uint64_t b1 = L.b1_off >= 0 ? sdesc_sw128(st + L.b1_off + a * B_ATOM) : 0;
+      auto descA = [&](int off) {
+        return L.a_mn ? sdesc_mn_sw128(st + off) : sdesc_sw128(st + off + a * A_ATOM);
+      };
+      auto descB = [&](int off) {
+        return L.b_mn ? sdesc_mn_sw128(st + off) : sdesc_sw128(st + off + a * B_ATOM);
+      };
+      const uint64_t a0 = L.a0_off >= 0 ? descA(L.a0_off) : 0;
+      const uint64_t a1 = L.a1_off >= 0 ? descA(L.a1_off) : 0;
+      const uint64_t b0 = L.b0_off >= 0 ? descB(L.b0_off) : 0;
+      const uint64_t b1 = L.b1_off >= 0 ? descB(L.b1_off) : 0;
 #pragma unroll
       for (int kk = 0; kk < BK / 16; ++kk) {
         // The j-th product of K slice kk into accumulator c goes to block
         // (kk * P_c + j) mod nsub (P_c products into c per slice); the first product into
         // a block overwrites it.
-        const uint64_t adv = static_cast<uint64_t>(kk * 2);   // 32 bytes per K=16 step
+        const uint64_t advA = static_cast<uint64_t>(kk) * stepA;
+        const uint64_t advB = static_cast<uint64_t>(kk) * stepB;
         const bool first = i == 0 && a == 0;
         uint32_t q0 = static_cast<uint32_t>(kk) * p0, q1 = static_cast<uint32_t>(kk) * p1;
         auto mma = [&](uint32_t c, uint64_t ad, uint64_t bd) {
@@ -493,12 +520,12 @@ __device__ __forceinline__ void mma_loop(const MmaLoop& L, unsigned terms_rt, in
           if constexpr (PAIR) mma_bf16_pair(L.tbase + blk * BN, ad, bd, idesc, f);
           else mma_bf16(L.tbase + blk * BN, ad, bd, idesc, f);
         };
-        if (terms & T_C0_A0B0) mma(0, a0 + adv, b0 + adv);
-        if (terms & T_C1_A1B0) mma(1, a1 + adv, b0 + adv);
-        if (terms & T_C0_A1B0) mma(0, a1 + adv, b0 + adv);
-        if (terms & T_C1_A0B1) mma(1, a0 + adv, b1 + adv);
-        if (terms & T_C0_A0B1) mma(0, a0 + adv, b1 + adv);
-        if (terms & T_C0_A1B1) mma(0, a1 + adv, b1 + adv);
+        if (terms & T_C0_A0B0) mma(0, a0 + advA, b0 + advB);
+        if (terms & T_C1_A1B0) mma(1, a1 + advA, b0 + advB);
+        if (terms & T_C0_A1B0) mma(0, a1 + advA, b0 + advB);
+        if (terms & T_C1_A0B1) mma(1, a0 + advA, b1 + advB);
+        if (terms & T_C0_A0B1) mma(0, a0 + advA, b1 + advB);
+        if (terms & T_C0_A1B1) mma(0, a1 + advA, b1 + advB);
       }
     }
     if constexpr (PAIR) mma_commit_pair(&L.empty_bar[s]);
@@ -617,10 +644,24 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int a = 0; a < KA; ++a) {
           const int ka = k + a * BK;
-          if (a0_off >= 0) tma_load_3d(st + a0_off + a * A_ATOM, &tmA0, &full_bar[s], ka, m0, bz);
-          if (a1_off >= 0) tma_load_3d(st + a1_off + a * A_ATOM, &tmA1, &full_bar[s], ka, m0, bz);
-          if (b0_off >= 0) tma_load_3d(st + b0_off + a * B_ATOM, &tmB0, &full_bar[s], ka, n0, bz);
-          if (b1_off >= 0) tma_load_3d(st + b1_off + a * B_ATOM, &tmB1, &full_bar[s], ka, n0, bz);
+          if (p.a_mn) {   // MN-major: boxes of 64 rows x 64 K at (row, k)
+            for (int j = 0; j < BM / 64; ++j) {
+              if (a0_off >= 0) tma_load_3d(st + a0_off + j * MN_BOX, &tmA0, &full_bar[s], m0 + 64 * j, ka, bz);
+              if (a1_off >= 0) tma_load_3d(st + a1_off + j * MN_BOX, &tmA1, &full_bar[s], m0 + 64 * j, ka, bz);
+            }
+          } else {
+            if (a0_off >= 0) tma_load_3d(st + a0_off + a * A_ATOM, &tmA0, &full_bar[s], ka, m0, bz);
+            if (a1_off >= 0) tma_load_3d(st + a1_off + a * A_ATOM, &tmA1, &full_bar[s], ka, m0, bz);
+          }
+          if (p.b_mn) {
+            for (int j = 0; j < BN / 64; ++j) {
+              if (b0_off >= 0) tma_load_3d(st + b0_off + j * MN_BOX, &tmB0, &full_bar[s], n0 + 64 * j, ka, bz);
+              if (b1_off >= 0) tma_load_3d(st + b1_off + j * MN_BOX, &tmB1, &full_bar[s], n0 + 64 * j, ka, bz);
+            }
+          } else {
+            if (b0_off >= 0) tma_load_3d(st + b0_off + a * B_ATOM, &tmB0, &full_bar[s], ka, n0, bz);
+            if (b1_off >= 0) tma_load_3d(st + b1_off + a * B_ATOM, &tmB1, &full_bar[s], ka, n0, bz);
+          }
         }
       }
     }
@@ -632,6 +673,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       L.nk = nk; L.stages = p.stages; L.stage_bytes = p.stage_bytes;
       L.a0_off = p.a0_off; L.a1_off = p.a1_off; L.b0_off = p.b0_off; L.b1_off = p.b1_off;
       L.sbase = smem_u32(smem); L.tbase = tbase;
+      L.a_mn = p.a_mn; L.b_mn = p.b_mn;
       L.full_bar = full_bar; L.empty_bar = empty_bar; L.status = p.status;
       mma_dispatch<BN, KA, MODE, false>(L, terms, p.nsub);
       mma_commit(&acc_bar);
@@ -844,6 +886,14 @@ bool make_map(CUtensorMap* m, const void* ptr, int K, int rows, int ld, int box_
                    bstride);
 }
 
+// Operand map: K-major [rows][K] (box 64 K x box_rows) or MN-major [K][rows] (boxes of 64
+// rows x 64 K; the kernel issues box_rows / 64 of them per stage).
+bool make_op_map(CUtensorMap* m, const void* ptr, int K, int rows, int ld, int box_rows, int batch,
+                 int64_t bstride, bool mn) {
+  if (!mn) return make_map(m, ptr, K, rows, ld, box_rows, batch, bstride);
+  return make_map2(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, ptr, rows, K, ld, 64, BK, batch, bstride);
+}
+
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 // Split of K across a cluster: double S while the grid stays within ~1.2 waves of 152 SMs
@@ -899,10 +949,12 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
   memset(&mC0, 0, sizeof(mC0)); memset(&mC1, 0, sizeof(mC1));
   memset(&mA, 0, sizeof(mA)); memset(&mAd, 0, sizeof(mAd));
   const int nb = a.batch < 1 ? 1 : a.batch;
-  if (useA0 && !make_map(&mA0, a.A0, a.K, a.M, a.lda0, BM, nb, a.bsA0)) { *why = "tensor map A0"; return cudaErrorInvalidValue; }
-  if (useA1 && !make_map(&mA1, a.A1, a.K, a.M, a.lda1, BM, nb, a.bsA1)) { *why = "tensor map A1"; return cudaErrorInvalidValue; }
-  if (useB0 && !make_map(&mB0, a.B0, a.K, a.N, a.ldb0, BN, nb, a.bsB0)) { *why = "tensor map B0"; return cudaErrorInvalidValue; }
-  if (useB1 && !make_map(&mB1, a.B1, a.K, a.N, a.ldb1, BN, nb, a.bsB1)) { *why = "tensor map B1"; return cudaErrorInvalidValue; }
+  p.a_mn = a.a_mn ? 1 : 0;
+  p.b_mn = a.b_mn ? 1 : 0;
+  if (useA0 && !make_op_map(&mA0, a.A0, a.K, a.M, a.lda0, BM, nb, a.bsA0, a.a_mn)) { *why = "tensor map A0"; return cudaErrorInvalidValue; }
+  if (useA1 && !make_op_map(&mA1, a.A1, a.K, a.M, a.lda1, BM, nb, a.bsA1, a.a_mn)) { *why = "tensor map A1"; return cudaErrorInvalidValue; }
+  if (useB0 && !make_op_map(&mB0, a.B0, a.K, a.N, a.ldb0, BN, nb, a.bsB0, a.b_mn)) { *why = "tensor map B0"; return cudaErrorInvalidValue; }
+  if (useB1 && !make_op_map(&mB1, a.B1, a.K, a.N, a.ldb1, BN, nb, a.bsB1, a.b_mn)) { *why = "tensor map B1"; return cudaErrorInvalidValue; }
   p.batch = nb;
   p.bsC0 = a.bsC0;
   p.bsC1 = a.bsC1;
@@ -1062,10 +1114,24 @@ __global__ void __launch_bounds__(THREADS, 1)
         const uint32_t bar = full0 + static_cast<uint32_t>(s) * 8u;
         uint8_t* st = smem + s * stage_bytes;
         const int k = i * BK;
-        if (a0_off >= 0) tma_load_3d_pair(st + a0_off, &tmA0, bar, k, m0, bz);
-        if (a1_off >= 0) tma_load_3d_pair(st + a1_off, &tmA1, bar, k, m0, bz);
-        if (b0_off >= 0) tma_load_3d_pair(st + b0_off, &tmB0, bar, k, nb0, bz);
-        if (b1_off >= 0) tma_load_3d_pair(st + b1_off, &tmB1, bar, k, nb0, bz);
+        if (p.a_mn) {
+          for (int j = 0; j < BM / 64; ++j) {
+            if (a0_off >= 0) tma_load_3d_pair(st + a0_off + j * MN_BOX, &tmA0, bar, m0 + 64 * j, k, bz);
+            if (a1_off >= 0) tma_load_3d_pair(st + a1_off + j * MN_BOX, &tmA1, bar, m0 + 64 * j, k, bz);
+          }
+        } else {
+          if (a0_off >= 0) tma_load_3d_pair(st + a0_off, &tmA0, bar, k, m0, bz);
+          if (a1_off >= 0) tma_load_3d_pair(st + a1_off, &tmA1, bar, k, m0, bz);
+        }
+        if (p.b_mn) {
+          for (int j = 0; j < BH / 64; ++j) {
+            if (b0_off >= 0) tma_load_3d_pair(st + b0_off + j * MN_BOX, &tmB0, bar, nb0 + 64 * j, k, bz);
+            if (b1_off >= 0) tma_load_3d_pair(st + b1_off + j * MN_BOX, &tmB1, bar, nb0 + 64 * j, k, bz);
+          }
+        } else {
+          if (b0_off >= 0) tma_load_3d_pair(st + b0_off, &tmB0, bar, k, nb0, bz);
+          if (b1_off >= 0) tma_load_3d_pair(st + b1_off, &tmB1, bar, k, nb0, bz);
+        }
       }
     }
     __syncwarp();
@@ -1075,6 +1141,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       L.nk = nk; L.stages = p.stages; L.stage_bytes = p.stage_bytes;
       L.a0_off = p.a0_off; L.a1_off = p.a1_off; L.b0_off = p.b0_off; L.b1_off = p.b1_off;
       L.sbase = smem_u32(smem); L.tbase = tbase;
+      L.a_mn = p.a_mn; L.b_mn = p.b_mn;
       L.full_bar = full_bar; L.empty_bar = empty_bar; L.status = p.status;
       mma_dispatch<BN, 1, MODE, true>(L, terms, p.nsub);
       mma_commit_pair(&acc_bar);
@@ -1156,10 +1223,12 @@ cudaError_t launch_cfg2(const GemmArgs& a, cudaStream_t s, const char** why) {
   memset(&mB0, 0, sizeof(mB0)); memset(&mB1, 0, sizeof(mB1));
   memset(&mC0, 0, sizeof(mC0)); memset(&mC1, 0, sizeof(mC1));
   memset(&mA, 0, sizeof(mA)); memset(&mAd, 0, sizeof(mAd));
-  if (useA0 && !make_map(&mA0, a.A0, a.K, a.M, a.lda0, BM, nb, a.bsA0)) { *why = "tensor map A0"; return cudaErrorInvalidValue; }
-  if (useA1 && !make_map(&mA1, a.A1, a.K, a.M, a.lda1, BM, nb, a.bsA1)) { *why = "tensor map A1"; return cudaErrorInvalidValue; }
-  if (useB0 && !make_map(&mB0, a.B0, a.K, a.N, a.ldb0, BH, nb, a.bsB0)) { *why = "tensor map B0"; return cudaErrorInvalidValue; }
-  if (useB1 && !make_map(&mB1, a.B1, a.K, a.N, a.ldb1, BH, nb, a.bsB1)) { *why = "tensor map B1"; return cudaErrorInvalidValue; }
+  p.a_mn = a.a_mn ? 1 : 0;
+  p.b_mn = a.b_mn ? 1 : 0;
+  if (useA0 && !make_op_map(&mA0, a.A0, a.K, a.M, a.lda0, BM, nb, a.bsA0, a.a_mn)) { *why = "tensor map A0"; return cudaErrorInvalidValue; }
+  if (useA1 && !make_op_map(&mA1, a.A1, a.K, a.M, a.lda1, BM, nb, a.bsA1, a.a_mn)) { *why = "tensor map A1"; return cudaErrorInvalidValue; }
+  if (useB0 && !make_op_map(&mB0, a.B0, a.K, a.N, a.ldb0, BH, nb, a.bsB0, a.b_mn)) { *why = "tensor map B0"; return cudaErrorInvalidValue; }
+  if (useB1 && !make_op_map(&mB1, a.B1, a.K, a.N, a.ldb1, BH, nb, a.bsB1, a.b_mn)) { *why = "tensor map B1"; return cudaErrorInvalidValue; }
   p.batch = nb;
   p.bsC0 = a.bsC0;
   p.bsC1 = a.bsC1;

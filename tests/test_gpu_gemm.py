@@ -90,3 +90,43 @@ def test_dual_gemm_pair_tiles(shape, mask):
         test_dual_gemm(shape, mask)
     finally:
         _set_pair_mode(native, 1)
+
+
+MN_SHAPES = [(256, 1024, 1024), (1025, 1024, 256), (300, 10, 72), (130, 200, 40), (1000, 520, 200)]
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("shape", MN_SHAPES)
+@pytest.mark.parametrize("layout", [1, 2, 3])
+@pytest.mark.parametrize("mask", [1, 1 | 8 | 16, 2 | 4, 1 | 32])
+@pytest.mark.parametrize("pair_mode", [1, 2])
+def test_dual_gemm_mn_major(shape, layout, mask, pair_mode):
+    """Operands stored MN-major ([K][rows], rows contiguous; layout bit 0 for A, bit 1 for B),
+    on one-SM and CTA-pair tiles."""
+    torch, native = need_gpu()
+    M, N, K = shape
+    g = torch.Generator(device="cpu").manual_seed(M * 17 + N * 3 + K + mask + layout)
+    ld8 = lambda n: (n + 7) // 8 * 8
+    def op(rows, mn):
+        x = torch.randn(rows, K, generator=g).to(torch.bfloat16)
+        if not mn:
+            return x, x.cuda()
+        store = torch.zeros(K, ld8(rows), dtype=torch.bfloat16)
+        store[:, :rows] = x.t()
+        return x, store.cuda()
+    a_mn, b_mn = bool(layout & 1), bool(layout & 2)
+    (a0, A0), (a1, A1) = op(M, a_mn), op(M, a_mn)
+    (b0, B0), (b1, B1) = op(N, b_mn), op(N, b_mn)
+    C0 = torch.full((M, N), float("nan"), device="cuda")
+    C1 = torch.full((M, N), float("nan"), device="cuda")
+    _set_pair_mode(native, pair_mode)
+    try:
+        native.mf_dual_gemm_bf16(M, N, K, A0, A1, B0, B1, C0, C1, mask | (layout << 8))
+        torch.cuda.synchronize()
+    finally:
+        _set_pair_mode(native, 1)
+    r0, r1 = _ref(a0, a1, b0, b1, mask)
+    if r0 is not None:
+        assert rel_l2(C0.cpu().numpy(), r0.numpy()) < 1e-5
+    if r1 is not None:
+        assert rel_l2(C1.cpu().numpy(), r1.numpy()) < 1e-5
