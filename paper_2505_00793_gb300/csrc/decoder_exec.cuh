@@ -41,19 +41,19 @@ struct DecPlan {
   size_t o_theta = 0, o_m = 0, o_g = 0, o_tbar = 0, o_u = 0, o_part = 0, o_l = 0, o_ld = 0;
   size_t o_count = 0, o_start = 0, o_order = 0, o_order_tmp = 0, gpart = 0;
   // per tensor operand copies (index = tensor index; 0 when not cast)
-  std::vector<size_t> o_W, o_WT, o_U, o_UT;
+  std::vector<size_t> o_W, o_U;
   // per block activations
-  std::vector<size_t> x1, x1d, r1, r1d, x2, x2d, r2, r2d, h1, h1d, h1T, h1dT, h2, h2d, h2T, h2dT;
-  std::vector<size_t> Q, Qd, K, Kd, Vv, Vd, QT, QdT, KT, KdT, VT, VdT, P, Pd, Om, Omd, OmT, OmdT;
-  std::vector<size_t> z1, z1d, a1, a1d, a1T, a1dT;
-  size_t x0 = 0, x0d = 0, xf = 0, xfd = 0, rf = 0, rfd = 0, hf = 0, hfd = 0, hfT = 0, hfdT = 0;
-  size_t Fl = 0, Fld = 0, lse = 0, ltok = 0, pf = 0, ldtok = 0, dF = 0, dFd = 0, dFT = 0, dFdT = 0;
+  std::vector<size_t> x1, x1d, r1, r1d, x2, x2d, r2, r2d, h1, h1d, h2, h2d;
+  std::vector<size_t> Q, Qd, K, Kd, Vv, Vd, P, Pd, Om, Omd;
+  std::vector<size_t> z1, z1d, a1, a1d;
+  size_t x0 = 0, x0d = 0, xf = 0, xfd = 0, rf = 0, rfd = 0, hf = 0, hfd = 0;
+  size_t Fl = 0, Fld = 0, lse = 0, ltok = 0, pf = 0, ldtok = 0, dF = 0, dFd = 0;
   // scratch reused by every block
   size_t qkv = 0, qkvd = 0, Sc = 0, Scd = 0, O = 0, Od = 0, y = 0, yd = 0, yprev = 0;
-  size_t dx = 0, dxd = 0, dh = 0, dhd = 0, dy = 0, dyd = 0, dyT = 0, dydT = 0;
-  size_t dOh = 0, dOhd = 0, dOhT = 0, dOhdT = 0, dP = 0, dPd = 0, dS = 0, dSd = 0, dST = 0,
-         dSdT = 0, PT = 0, PdT = 0, dQ = 0, dQd = 0, dK = 0, dKd = 0, dV = 0, dVd = 0;
-  size_t dqkv = 0, dqkvd = 0, dqkvT = 0, dqkvdT = 0, dz1 = 0, dz1d = 0, dz1T = 0, dz1dT = 0;
+  size_t dx = 0, dxd = 0, dh = 0, dhd = 0, dy = 0, dyd = 0;
+  size_t dOh = 0, dOhd = 0, dP = 0, dPd = 0, dS = 0, dSd = 0;
+  size_t dQ = 0, dQd = 0, dK = 0, dKd = 0, dV = 0, dVd = 0;
+  size_t dqkv = 0, dqkvd = 0, dz1 = 0, dz1d = 0;
   // reverse-over-reverse: the inner backward's residual-stream cotangent at the output of
   // every block (the stored reverse graph, at block granularity)
   bool ror = false;
@@ -93,14 +93,12 @@ DecPlan make_dec_plan(const mf_ctx* h, const DecLayout& Ly, int rows, int T, int
   for (const auto& t : tens) {
     if (t.cast) {
       p.o_W.push_back(take(static_cast<size_t>(t.rows) * ld8(t.cols) * es));
-      p.o_WT.push_back(take(static_cast<size_t>(t.cols) * ld8(t.rows) * es));
       p.o_U.push_back(take(static_cast<size_t>(t.rows) * ld8(t.cols) * es));
-      p.o_UT.push_back(take(static_cast<size_t>(t.cols) * ld8(t.rows) * es));
     } else {
-      p.o_W.push_back(0); p.o_WT.push_back(0); p.o_U.push_back(0); p.o_UT.push_back(0);
+      p.o_W.push_back(0); p.o_U.push_back(0);
     }
   }
-  const size_t Nd4 = N * d * 4, NdT = N * d * es, NdTt = d * p.ldN * es;
+  const size_t Nd4 = N * d * 4, NdT = N * d * es;
   const size_t head = static_cast<size_t>(BH) * S * Ly.dh * es;
   const size_t SS = static_cast<size_t>(BH) * S * S;
   for (int l = 0; l < Ly.L; ++l) {
@@ -109,48 +107,37 @@ DecPlan make_dec_plan(const mf_ctx* h, const DecLayout& Ly, int rows, int T, int
     p.x2.push_back(take(Nd4)); p.x2d.push_back(take(Nd4));
     p.r2.push_back(take(N * 4)); p.r2d.push_back(take(N * 4));
     p.h1.push_back(take(NdT)); p.h1d.push_back(take(NdT));
-    p.h1T.push_back(take(NdTt)); p.h1dT.push_back(take(NdTt));
     p.h2.push_back(take(NdT)); p.h2d.push_back(take(NdT));
-    p.h2T.push_back(take(NdTt)); p.h2dT.push_back(take(NdTt));
     p.Q.push_back(take(head)); p.Qd.push_back(take(head));
     p.K.push_back(take(head)); p.Kd.push_back(take(head));
     p.Vv.push_back(take(head)); p.Vd.push_back(take(head));
-    p.QT.push_back(take(head)); p.QdT.push_back(take(head));
-    p.KT.push_back(take(head)); p.KdT.push_back(take(head));
-    p.VT.push_back(take(head)); p.VdT.push_back(take(head));
     p.P.push_back(take(SS * es)); p.Pd.push_back(take(SS * es));
     p.Om.push_back(take(NdT)); p.Omd.push_back(take(NdT));
-    p.OmT.push_back(take(NdTt)); p.OmdT.push_back(take(NdTt));
     p.z1.push_back(take(N * F * 4)); p.z1d.push_back(take(N * F * 4));
     p.a1.push_back(take(N * F * es)); p.a1d.push_back(take(N * F * es));
-    p.a1T.push_back(take(F * p.ldN * es)); p.a1dT.push_back(take(F * p.ldN * es));
   }
   p.x0 = take(Nd4); p.x0d = take(Nd4);
   p.xf = take(Nd4); p.xfd = take(Nd4); p.rf = take(N * 4); p.rfd = take(N * 4);
-  p.hf = take(NdT); p.hfd = take(NdT); p.hfT = take(NdTt); p.hfdT = take(NdTt);
+  p.hf = take(NdT); p.hfd = take(NdT);
   p.Fl = take(N * V * 4); p.Fld = take(N * V * 4);
   p.lse = take(N * 4); p.ltok = take(N * 4); p.pf = take(N * 4); p.ldtok = take(N * 4);
   p.dF = take(N * V * es); p.dFd = take(N * V * es);
-  p.dFT = take(V * p.ldN * es); p.dFdT = take(V * p.ldN * es);
   p.qkv = take(N * 3 * d * 4); p.qkvd = take(N * 3 * d * 4);
   p.Sc = take(SS * 4); p.Scd = take(SS * 4);
   p.O = take(static_cast<size_t>(BH) * S * Ly.dh * 4); p.Od = take(static_cast<size_t>(BH) * S * Ly.dh * 4);
   p.y = take(Nd4); p.yd = take(Nd4);
   p.dx = take(Nd4); p.dxd = take(Nd4); p.dh = take(Nd4); p.dhd = take(Nd4);
-  p.dy = take(NdT); p.dyd = take(NdT); p.dyT = take(NdTt); p.dydT = take(NdTt);
-  p.dOh = take(head); p.dOhd = take(head); p.dOhT = take(head); p.dOhdT = take(head);
+  p.dy = take(NdT); p.dyd = take(NdT);
+  p.dOh = take(head); p.dOhd = take(head);
   p.dP = take(SS * 4); p.dPd = take(SS * 4);
-  p.dS = take(SS * es); p.dSd = take(SS * es); p.dST = take(SS * es); p.dSdT = take(SS * es);
-  p.PT = take(SS * es); p.PdT = take(SS * es);
+  p.dS = take(SS * es); p.dSd = take(SS * es);
   const size_t head4 = static_cast<size_t>(BH) * S * Ly.dh * 4;
   p.dQ = take(head4); p.dQd = take(head4); p.dK = take(head4); p.dKd = take(head4);
   p.dV = take(head4); p.dVd = take(head4);
   if (ror)
     for (int l = 0; l < Ly.L; ++l) p.dxs.push_back(take(Nd4));
   p.dqkv = take(N * 3 * d * es); p.dqkvd = take(N * 3 * d * es);
-  p.dqkvT = take(3 * d * p.ldN * es); p.dqkvdT = take(3 * d * p.ldN * es);
   p.dz1 = take(N * F * es); p.dz1d = take(N * F * es);
-  p.dz1T = take(F * p.ldN * es); p.dz1dT = take(F * p.ldN * es);
   p.bytes = o;
   return p;
 }
@@ -188,11 +175,11 @@ struct DecExec {
       tab.tile0[i] = tiles;
       tiles += ((t.rows + 31) / 32) * ((t.cols + 31) / 32);
       tab.ldw[i] = ld8(t.cols);
-      tab.ldwt[i] = ld8(t.rows);
-      tab.W[i] = t.cast ? at<T>(p.o_W[i]) : nullptr;
-      tab.WT[i] = t.cast ? at<T>(p.o_WT[i]) : nullptr;
+      tab.ldwt[i] = 0;
+      tab.W[i] = t.cast ? at<T>(p.o_W[i]) : nullptr;   // read K- or MN-major, never transposed
+      tab.WT[i] = nullptr;
       tab.U[i] = t.cast ? at<T>(p.o_U[i]) : nullptr;
-      tab.UT[i] = t.cast ? at<T>(p.o_UT[i]) : nullptr;
+      tab.UT[i] = nullptr;
     }
     tab.tile0[tab.n] = tiles;
   }
@@ -226,9 +213,9 @@ struct DecExec {
     return -1;
   }
   T* W(int64_t off) const { return at<T>(p.o_W[tidx(off)]); }
-  T* WT(int64_t off) const { return at<T>(p.o_WT[tidx(off)]); }
+
   T* Uw(int64_t off) const { return at<T>(p.o_U[tidx(off)]); }
-  T* UT(int64_t off) const { return at<T>(p.o_UT[tidx(off)]); }
+
 
   void gemm(GemmArgs g) {
     if (st != MF_OK) return;
@@ -293,19 +280,9 @@ struct DecExec {
     update(a);
   }
 
-  void tr(const T* X, int rows, int cols, int ld, T* XT, int ldT) {
-    mf::transpose_batched<T, T>(X, rows, cols, ld, 0, XT, ldT, 0, 1, s);
-    launched();
-  }
-  void trb(const T* X, int rows, int cols, T* XT, int batch) {
-    mf::transpose_batched<T, T>(X, rows, cols, cols, static_cast<int64_t>(rows) * cols, XT, rows,
-                                static_cast<int64_t>(rows) * cols, batch, s);
-    launched();
-  }
-
   void forward(int rows, const void* x, const float* theta, const float* u, bool dual) {
     const int S = Ly.S, d = Ly.d, H = Ly.H, dh = Ly.dh, F = Ly.F, V = Ly.V;
-    const int N = rows * S, BH = rows * H, ldN = p.ldN;
+    const int N = rows * S, BH = rows * H;
     const int* ids = static_cast<const int*>(x);
     rows_cur = rows;
     ids_cur = ids;
@@ -327,12 +304,11 @@ struct DecExec {
                              at<float>(p.r1[l]), at<float>(p.r1d[l]), at<T>(p.h1[l]), at<T>(p.h1d[l]),
                              d, s);
       launched();
-      tr(at<T>(p.h1[l]), N, d, d, at<T>(p.h1T[l]), ldN);
-      if (dual) tr(at<T>(p.h1d[l]), N, d, d, at<T>(p.h1dT[l]), ldN);
-      // q k v = h Wqkv
+      // q k v = h Wqkv   (weights [d][3d] read MN-major)
       {
-        GemmArgs g = lin(N, 3 * d, d, at<T>(p.h1[l]), at<T>(p.h1d[l]), d, WT(Ly.Wqkv[l]),
-                         UT(Ly.Wqkv[l]), ld8(d), dual);
+        GemmArgs g = lin(N, 3 * d, d, at<T>(p.h1[l]), at<T>(p.h1d[l]), d, W(Ly.Wqkv[l]),
+                         Uw(Ly.Wqkv[l]), ld8(3 * d), dual);
+        g.b_mn = true;
         g.C0 = at<float>(p.qkv); g.ldc0 = 3 * d;
         g.C1 = at<float>(p.qkvd); g.ldc1 = 3 * d;
         if (!dual) g.terms = mf::T_C0_A0B0;
@@ -347,8 +323,7 @@ struct DecExec {
                               at<T>(p.Kd[l]), at<T>(p.Vd[l]), s);
         launched();
       }
-      trb(at<T>(p.Vv[l]), S, dh, at<T>(p.VT[l]), BH);
-      if (dual) trb(at<T>(p.Vd[l]), S, dh, at<T>(p.VdT[l]), BH);
+
       // scores S = Q K^T (dual: Q' K^T + Q K'^T), batch over B*H
       {
         GemmArgs g = lin(S, S, dh, at<T>(p.Q[l]), at<T>(p.Qd[l]), dh, at<T>(p.K[l]), at<T>(p.Kd[l]),
@@ -361,10 +336,11 @@ struct DecExec {
       mf::dec_softmax_fwd<T>(S, BH * S, at<float>(p.Sc), dual ? at<float>(p.Scd) : nullptr,
                              at<T>(p.P[l]), dual ? at<T>(p.Pd[l]) : nullptr, s);
       launched();
-      // O = P V (dual: P' V + P V')
+      // O = P V (dual: P' V + P V'); V [S][dh] read MN-major
       {
-        GemmArgs g = lin(S, dh, S, at<T>(p.P[l]), at<T>(p.Pd[l]), S, at<T>(p.VT[l]),
-                         at<T>(p.VdT[l]), S, dual);
+        GemmArgs g = lin(S, dh, S, at<T>(p.P[l]), at<T>(p.Pd[l]), S, at<T>(p.Vv[l]),
+                         at<T>(p.Vd[l]), dh, dual);
+        g.b_mn = true;
         batched(g, BH, ss, hs, hs);
         g.C0 = at<float>(p.O); g.ldc0 = dh;
         g.C1 = at<float>(p.Od); g.ldc1 = dh;
@@ -372,16 +348,15 @@ struct DecExec {
       }
       mf::dec_head_merge<T>(N, S, H, dh, at<float>(p.O), at<T>(p.Om[l]), d, s);
       launched();
-      tr(at<T>(p.Om[l]), N, d, d, at<T>(p.OmT[l]), ldN);
       if (dual) {
         mf::dec_head_merge<T>(N, S, H, dh, at<float>(p.Od), at<T>(p.Omd[l]), d, s);
         launched();
-        tr(at<T>(p.Omd[l]), N, d, d, at<T>(p.OmdT[l]), ldN);
       }
       // y = O Wo
       {
-        GemmArgs g = lin(N, d, d, at<T>(p.Om[l]), at<T>(p.Omd[l]), d, WT(Ly.Wo[l]), UT(Ly.Wo[l]),
+        GemmArgs g = lin(N, d, d, at<T>(p.Om[l]), at<T>(p.Omd[l]), d, W(Ly.Wo[l]), Uw(Ly.Wo[l]),
                          ld8(d), dual);
+        g.b_mn = true;
         g.C0 = at<float>(p.y); g.ldc0 = d;
         g.C1 = at<float>(p.yd); g.ldc1 = d;
         gemm(g);
@@ -393,12 +368,11 @@ struct DecExec {
                              at<float>(p.x2d[l]), at<float>(p.r2[l]), at<float>(p.r2d[l]),
                              at<T>(p.h2[l]), at<T>(p.h2d[l]), d, s);
       launched();
-      tr(at<T>(p.h2[l]), N, d, d, at<T>(p.h2T[l]), ldN);
-      if (dual) tr(at<T>(p.h2d[l]), N, d, d, at<T>(p.h2dT[l]), ldN);
       // a = GELU(h2 W1) fused; z kept for the backward
       {
-        GemmArgs g = lin(N, F, d, at<T>(p.h2[l]), at<T>(p.h2d[l]), d, WT(Ly.W1[l]), UT(Ly.W1[l]),
-                         ld8(d), dual);
+        GemmArgs g = lin(N, F, d, at<T>(p.h2[l]), at<T>(p.h2d[l]), d, W(Ly.W1[l]), Uw(Ly.W1[l]),
+                         ld8(F), dual);
+        g.b_mn = true;
         g.C0 = at<float>(p.z1[l]); g.ldc0 = F;
         g.C1 = at<float>(p.z1d[l]); g.ldc1 = F;
         g.epi.mode = mf::EPI_ACT_FWD;
@@ -406,15 +380,13 @@ struct DecExec {
         g.epi.A = at<T>(p.a1[l]);
         g.epi.Ad = dual ? at<T>(p.a1d[l]) : nullptr;
         g.epi.lda = F;
-        g.epi.AT = at<T>(p.a1T[l]);
-        g.epi.AdT = dual ? at<T>(p.a1dT[l]) : nullptr;
-        g.epi.ldt = ldN;
         gemm(g);
       }
       // y = a W2  (added to x2 by the next RMSNorm)
       {
-        GemmArgs g = lin(N, d, F, at<T>(p.a1[l]), at<T>(p.a1d[l]), F, WT(Ly.W2[l]), UT(Ly.W2[l]),
-                         ld8(F), dual);
+        GemmArgs g = lin(N, d, F, at<T>(p.a1[l]), at<T>(p.a1d[l]), F, W(Ly.W2[l]), Uw(Ly.W2[l]),
+                         ld8(d), dual);
+        g.b_mn = true;
         g.C0 = at<float>(p.y); g.ldc0 = d;
         g.C1 = at<float>(p.yd); g.ldc1 = d;
         gemm(g);
@@ -428,10 +400,9 @@ struct DecExec {
                            dual ? u + Ly.gf : nullptr, at<float>(p.xf), at<float>(p.xfd),
                            at<float>(p.rf), at<float>(p.rfd), at<T>(p.hf), at<T>(p.hfd), d, s);
     launched();
-    tr(at<T>(p.hf), N, d, d, at<T>(p.hfT), ldN);
-    if (dual) tr(at<T>(p.hfd), N, d, d, at<T>(p.hfdT), ldN);
     {
-      GemmArgs g = lin(N, V, d, at<T>(p.hf), at<T>(p.hfd), d, WT(Ly.Wh), UT(Ly.Wh), ld8(d), dual);
+      GemmArgs g = lin(N, V, d, at<T>(p.hf), at<T>(p.hfd), d, W(Ly.Wh), Uw(Ly.Wh), ld8(V), dual);
+      g.b_mn = true;
       g.C0 = at<float>(p.Fl); g.ldc0 = V;
       g.C1 = at<float>(p.Fld); g.ldc1 = V;
       gemm(g);
@@ -443,7 +414,7 @@ struct DecExec {
   void loss(int rows, bool dual, const void* y, const float* eta_w, const float* ex_w,
             float* l_out, float* ld_out, float* d_eta) {
     (void)y;
-    const int S = Ly.S, V = Ly.V, N = rows * S, ldN = p.ldN;
+    const int S = Ly.S, V = Ly.V, N = rows * S;
     mf::dec_ce_stats(N, S, V, ids_cur, at<float>(p.Fl), dual ? at<float>(p.Fld) : nullptr,
                      at<float>(p.lse), at<float>(p.ltok), at<float>(p.pf), at<float>(p.ldtok),
                      h->d_status, s);
@@ -453,22 +424,22 @@ struct DecExec {
                        1.f / (static_cast<float>(rows) * S), at<T>(p.dF),
                        dual ? at<T>(p.dFd) : nullptr, V, s);
     launched();
-    tr(at<T>(p.dF), N, V, V, at<T>(p.dFT), ldN);
-    if (dual) tr(at<T>(p.dFd), N, V, V, at<T>(p.dFdT), ldN);
     mf::dec_seq_reduce(rows, S, at<float>(p.ltok), dual ? at<float>(p.ldtok) : nullptr, eta_w,
                        1.f / rows, l_out, ld_out, d_eta, s);
     launched();
     chk("decoder loss");
   }
 
-  // weight product into out (grad) / outh (tangent): [A^T][seed] with K = tokens
-  void wprod(int M, int Nn, const T* AT_, const T* AdT_, const T* ST_, const T* SdT_, bool dual,
+  // weight product into out (grad) / outh (tangent): A^T seed with K = tokens; the
+  // activations A [tokens][M] and the seeds [tokens][Nn] are read MN-major
+  void wprod(int M, int Nn, const T* A_, const T* Ad_, const T* S_, const T* Sd_, bool dual,
              float* outg, float* outh) {
     if (!dual && !outg) return;   // primal backward kept only for its cotangents
     GemmArgs g;
     g.M = M; g.N = Nn; g.K = rows_cur * Ly.S;
-    g.A0 = AT_; g.A1 = AdT_; g.lda0 = g.lda1 = p.ldN;
-    g.B0 = ST_; g.B1 = SdT_; g.ldb0 = g.ldb1 = p.ldN;
+    g.A0 = A_; g.A1 = Ad_; g.lda0 = g.lda1 = M;
+    g.B0 = S_; g.B1 = Sd_; g.ldb0 = g.ldb1 = Nn;
+    g.a_mn = g.b_mn = true;
     if (!dual) {
       g.terms = mf::T_C0_A0B0;
       g.C0 = outg; g.ldc0 = Nn;
@@ -483,16 +454,14 @@ struct DecExec {
     gemm(g);
   }
 
-  // residual gradient (float32) -> bf16 seed, row-major and transposed
+  // residual gradient (float32) -> operand-type seed
   void seed_from(const float* X, const float* Xd, bool dual) {
     const int N = rows_cur * Ly.S, d = Ly.d;
     mf::cast_rows<T>(X, N, d, at<T>(p.dy), d, s);
     launched();
-    tr(at<T>(p.dy), N, d, d, at<T>(p.dyT), p.ldN);
     if (dual) {
       mf::cast_rows<T>(Xd, N, d, at<T>(p.dyd), d, s);
       launched();
-      tr(at<T>(p.dyd), N, d, d, at<T>(p.dydT), p.ldN);
     }
   }
 
@@ -507,7 +476,7 @@ struct DecExec {
                       at<int>(p.o_order_tmp), s);
     launched(3);
     // head: dWh = hf^T dF ; dhf = dF Wh^T
-    wprod(d, V, at<T>(p.hfT), at<T>(p.hfdT), at<T>(p.dFT), at<T>(p.dFdT), dual, G(Ly.Wh), Hh(Ly.Wh));
+    wprod(d, V, at<T>(p.hf), at<T>(p.hfd), at<T>(p.dF), at<T>(p.dFd), dual, G(Ly.Wh), Hh(Ly.Wh));
     {
       GemmArgs g = lin(N, d, V, at<T>(p.dF), at<T>(p.dFd), V, W(Ly.Wh), Uw(Ly.Wh), ld8(V), dual);
       g.C0 = at<float>(p.dh); g.ldc0 = d;
@@ -533,7 +502,7 @@ struct DecExec {
       }
       // ---- MLP branch: seed = dx -------------------------------------------------------
       seed_from(at<float>(p.dx), at<float>(p.dxd), dual);
-      wprod(F, d, at<T>(p.a1T[l]), at<T>(p.a1dT[l]), at<T>(p.dyT), at<T>(p.dydT), dual, G(Ly.W2[l]),
+      wprod(F, d, at<T>(p.a1[l]), at<T>(p.a1d[l]), at<T>(p.dy), at<T>(p.dyd), dual, G(Ly.W2[l]),
             Hh(Ly.W2[l]));
       {
         GemmArgs g = lin(N, F, d, at<T>(p.dy), at<T>(p.dyd), d, W(Ly.W2[l]), Uw(Ly.W2[l]), ld8(d), dual);
@@ -545,12 +514,9 @@ struct DecExec {
         g.epi.A = at<T>(p.dz1);
         g.epi.Ad = dual ? at<T>(p.dz1d) : nullptr;
         g.epi.lda = F;
-        g.epi.AT = at<T>(p.dz1T);
-        g.epi.AdT = dual ? at<T>(p.dz1dT) : nullptr;
-        g.epi.ldt = p.ldN;
         gemm(g);
       }
-      wprod(d, F, at<T>(p.h2T[l]), at<T>(p.h2dT[l]), at<T>(p.dz1T), at<T>(p.dz1dT), dual, G(Ly.W1[l]),
+      wprod(d, F, at<T>(p.h2[l]), at<T>(p.h2d[l]), at<T>(p.dz1), at<T>(p.dz1d), dual, G(Ly.W1[l]),
             Hh(Ly.W1[l]));
       {
         GemmArgs g = lin(N, d, F, at<T>(p.dz1), at<T>(p.dz1d), F, W(Ly.W1[l]), Uw(Ly.W1[l]), ld8(F), dual);
@@ -568,7 +534,7 @@ struct DecExec {
       launched(2);
       // ---- attention branch: seed = dx --------------------------------------------------
       seed_from(at<float>(p.dx), at<float>(p.dxd), dual);
-      wprod(d, d, at<T>(p.OmT[l]), at<T>(p.OmdT[l]), at<T>(p.dyT), at<T>(p.dydT), dual, G(Ly.Wo[l]),
+      wprod(d, d, at<T>(p.Om[l]), at<T>(p.Omd[l]), at<T>(p.dy), at<T>(p.dyd), dual, G(Ly.Wo[l]),
             Hh(Ly.Wo[l]));
       {
         GemmArgs g = lin(N, d, d, at<T>(p.dy), at<T>(p.dyd), d, W(Ly.Wo[l]), Uw(Ly.Wo[l]), ld8(d), dual);
@@ -578,11 +544,9 @@ struct DecExec {
       }
       mf::dec_head_split<T>(N, S, H, dh, at<float>(p.dh), at<T>(p.dOh), s);
       launched();
-      trb(at<T>(p.dOh), S, dh, at<T>(p.dOhT), BH);
       if (dual) {
         mf::dec_head_split<T>(N, S, H, dh, at<float>(p.dhd), at<T>(p.dOhd), s);
         launched();
-        trb(at<T>(p.dOhd), S, dh, at<T>(p.dOhdT), BH);
       }
       // dP = dO V^T (dual: dO' V^T + dO V'^T)
       {
@@ -596,33 +560,27 @@ struct DecExec {
                              at<float>(p.dP), dual ? at<float>(p.dPd) : nullptr, at<T>(p.dS),
                              dual ? at<T>(p.dSd) : nullptr, s);
       launched();
-      trb(at<T>(p.P[l]), S, S, at<T>(p.PT), BH);
-      trb(at<T>(p.dS), S, S, at<T>(p.dST), BH);
-      trb(at<T>(p.Q[l]), S, dh, at<T>(p.QT[l]), BH);
-      trb(at<T>(p.K[l]), S, dh, at<T>(p.KT[l]), BH);
-      if (dual) {
-        trb(at<T>(p.Pd[l]), S, S, at<T>(p.PdT), BH);
-        trb(at<T>(p.dSd), S, S, at<T>(p.dSdT), BH);
-        trb(at<T>(p.Qd[l]), S, dh, at<T>(p.QdT[l]), BH);
-        trb(at<T>(p.Kd[l]), S, dh, at<T>(p.KdT[l]), BH);
-      }
-      // dV = P^T dO ; dQ = dS K ; dK = dS^T Q   (each with its tangent)
+      // dV = P^T dO ; dQ = dS K ; dK = dS^T Q   (each with its tangent); P, dS, dO, K, Q
+      // are read in place (MN-major where the product contracts over their row index)
       {
-        GemmArgs g = lin(S, dh, S, at<T>(p.PT), at<T>(p.PdT), S, at<T>(p.dOhT), at<T>(p.dOhdT), S, dual);
+        GemmArgs g = lin(S, dh, S, at<T>(p.P[l]), at<T>(p.Pd[l]), S, at<T>(p.dOh), at<T>(p.dOhd), dh, dual);
+        g.a_mn = g.b_mn = true;
         batched(g, BH, ss, hs, hs);
         g.C0 = at<float>(p.dV); g.ldc0 = dh;
         g.C1 = at<float>(p.dVd); g.ldc1 = dh;
         gemm(g);
       }
       {
-        GemmArgs g = lin(S, dh, S, at<T>(p.dS), at<T>(p.dSd), S, at<T>(p.KT[l]), at<T>(p.KdT[l]), S, dual);
+        GemmArgs g = lin(S, dh, S, at<T>(p.dS), at<T>(p.dSd), S, at<T>(p.K[l]), at<T>(p.Kd[l]), dh, dual);
+        g.b_mn = true;
         batched(g, BH, ss, hs, hs);
         g.C0 = at<float>(p.dQ); g.ldc0 = dh;
         g.C1 = at<float>(p.dQd); g.ldc1 = dh;
         gemm(g);
       }
       {
-        GemmArgs g = lin(S, dh, S, at<T>(p.dST), at<T>(p.dSdT), S, at<T>(p.QT[l]), at<T>(p.QdT[l]), S, dual);
+        GemmArgs g = lin(S, dh, S, at<T>(p.dS), at<T>(p.dSd), S, at<T>(p.Q[l]), at<T>(p.Qd[l]), dh, dual);
+        g.a_mn = g.b_mn = true;
         batched(g, BH, ss, hs, hs);
         g.C0 = at<float>(p.dK); g.ldc0 = dh;
         g.C1 = at<float>(p.dKd); g.ldc1 = dh;
@@ -632,14 +590,12 @@ struct DecExec {
       mf::dec_rope_merge<T>(N, S, H, dh, Ly.base, qscale, at<float>(p.dQ), at<float>(p.dK),
                             at<float>(p.dV), at<T>(p.dqkv), 3 * d, s);
       launched();
-      tr(at<T>(p.dqkv), N, 3 * d, 3 * d, at<T>(p.dqkvT), p.ldN);
       if (dual) {
         mf::dec_rope_merge<T>(N, S, H, dh, Ly.base, qscale, at<float>(p.dQd), at<float>(p.dKd),
                               at<float>(p.dVd), at<T>(p.dqkvd), 3 * d, s);
         launched();
-        tr(at<T>(p.dqkvd), N, 3 * d, 3 * d, at<T>(p.dqkvdT), p.ldN);
       }
-      wprod(d, 3 * d, at<T>(p.h1T[l]), at<T>(p.h1dT[l]), at<T>(p.dqkvT), at<T>(p.dqkvdT), dual,
+      wprod(d, 3 * d, at<T>(p.h1[l]), at<T>(p.h1d[l]), at<T>(p.dqkv), at<T>(p.dqkvd), dual,
             G(Ly.Wqkv[l]), Hh(Ly.Wqkv[l]));
       {
         GemmArgs g = lin(N, d, 3 * d, at<T>(p.dqkv), at<T>(p.dqkvd), 3 * d, W(Ly.Wqkv[l]),
