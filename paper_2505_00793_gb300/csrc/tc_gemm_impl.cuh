@@ -37,9 +37,19 @@ namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;                 // bf16 elements per 128-byte swizzle row
 constexpr int MAX_STAGES = 8;
-constexpr int EPI_WARPS = 8;                     // two per TMEM lane quadrant
+// Epilogue warps: one-SM tiles (small grids, split K) drain with sixteen warps storing
+// straight from registers; CTA-pair tiles with eight warps through TMA-store staging
+// (STG_WARP bytes of shared memory per warp).  Warps sharing a TMEM lane quadrant split its
+// columns.
+constexpr int EPI_WARPS = 16;
+constexpr int EPI_GROUPS = EPI_WARPS / 4;
+constexpr bool EPI_TMA = false;
 constexpr int EPI_THREADS = 32 * EPI_WARPS;
 constexpr int THREADS = 64 + EPI_THREADS;        // producer warp, MMA warp, epilogue
+constexpr int EPI_WARPS2 = 8;
+constexpr int EPI_GROUPS2 = EPI_WARPS2 / 4;
+constexpr bool EPI_TMA2 = true;
+constexpr int THREADS2 = 64 + 32 * EPI_WARPS2;
 constexpr long long WAIT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
 
 struct TcParams {
@@ -685,9 +695,13 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int q = warp & 3;
     const int r = q * 32 + lane;   // row within the tile
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
-    const int half = (warp - 2) >> 2;
-    const int c_begin = BN >= 128 ? half * (BN / 2) : 0;
-    const int c_end = BN >= 128 ? c_begin + BN / 2 : (half == 0 ? BN : 0);
+    // columns of this warp: BN / EPI_GROUPS per group (16-column granularity; TMA-store
+    // chunks of 64), narrow tiles on group 0 only
+    const int grp = (warp - 2) >> 2;
+    constexpr int GW = EPI_TMA ? 64 : 16;
+    constexpr int CG = BN / EPI_GROUPS >= GW ? BN / EPI_GROUPS : BN;
+    const int c_begin = CG < BN ? grp * CG : 0;
+    const int c_end = CG < BN ? c_begin + CG : (grp == 0 ? BN : 0);
     const bool ok = nk > 0 && mbar_wait(&acc_bar, 0, p.status);
     tc_fence_after();
     if (S == 1) {
@@ -731,9 +745,10 @@ __global__ void __launch_bounds__(THREADS, 1)
       const int q = warp & 3;
       const int r = q * 32 + lane;
       const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
-      const int half = (warp - 2) >> 2;
-      const int c_begin = BN >= 32 ? half * (BN / 2) : 0;
-      const int c_end = BN >= 32 ? c_begin + BN / 2 : (half == 0 ? BN : 0);
+      const int grp = (warp - 2) >> 2;
+      constexpr int CG = BN / EPI_GROUPS >= 16 ? BN / EPI_GROUPS : BN;
+      const int c_begin = CG < BN ? grp * CG : 0;
+      const int c_end = CG < BN ? c_begin + CG : (grp == 0 ? BN : 0);
       const bool ok = nk > 0;
       const uint32_t owner = static_cast<uint32_t>(r / rows_per);
       const int rr = r % rows_per;
@@ -965,7 +980,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
   p.st_c1 = p.C1 != nullptr;
   p.st_a = act && a.epi.A != nullptr;
   p.st_ad = act && dual && a.epi.Ad != nullptr;
-  bool tma_ok = S == 1 && BN >= 64;   // store boxes are 64 columns wide
+  bool tma_ok = EPI_TMA && S == 1 && BN >= 64;   // store boxes are 64 columns wide
   if (p.st_c0) tma_ok = tma_ok && aligned16(p.C0) && !(p.ldc0 & 3);
   if (p.st_c1) tma_ok = tma_ok && aligned16(p.C1) && !(p.ldc1 & 3);
   if (p.st_a) tma_ok = tma_ok && aligned16(a.epi.A) && !(a.epi.lda & 7);
@@ -1043,7 +1058,7 @@ __device__ __forceinline__ void tma_load_3d_pair(void* dst, const CUtensorMap* m
 }
 
 template <int BN, int MODE, int ACT>
-__global__ void __launch_bounds__(THREADS, 1)
+__global__ void __launch_bounds__(THREADS2, 1)
     tc2_dual_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
                          const __grid_constant__ CUtensorMap tmA1,
                          const __grid_constant__ CUtensorMap tmB0,
@@ -1153,7 +1168,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int q = warp & 3;
     const int r = q * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
-    const int c_begin = ((warp - 2) >> 2) * (BN / 2), c_end = c_begin + BN / 2;
+    constexpr int CG = BN / EPI_GROUPS2;
+    const int c_begin = ((warp - 2) >> 2) * CG, c_end = c_begin + CG;
     const bool ok = mbar_wait(&acc_bar, 0, p.status);
     tc_fence_after();
     if (ok) {
@@ -1238,7 +1254,7 @@ cudaError_t launch_cfg2(const GemmArgs& a, cudaStream_t s, const char** why) {
   p.st_c1 = p.C1 != nullptr;
   p.st_a = act && a.epi.A != nullptr;
   p.st_ad = act && dual && a.epi.Ad != nullptr;
-  bool tma_ok = true;
+  bool tma_ok = EPI_TMA2;
   if (p.st_c0) tma_ok = tma_ok && aligned16(p.C0) && !(p.ldc0 & 3);
   if (p.st_c1) tma_ok = tma_ok && aligned16(p.C1) && !(p.ldc1 & 3);
   if (p.st_a) tma_ok = tma_ok && aligned16(a.epi.A) && !(a.epi.lda & 7);
@@ -1257,7 +1273,7 @@ cudaError_t launch_cfg2(const GemmArgs& a, cudaStream_t s, const char** why) {
   p.tma_store = tma_ok ? 1 : 0;
 
   int need = stages * off;
-  if (p.tma_store && EPI_WARPS * STG_WARP > need) need = EPI_WARPS * STG_WARP;
+  if (p.tma_store && EPI_WARPS2 * STG_WARP > need) need = EPI_WARPS2 * STG_WARP;
   const int smem = need + 1024;
   static bool attr_set = false;
   if (!attr_set) {
@@ -1270,7 +1286,7 @@ cudaError_t launch_cfg2(const GemmArgs& a, cudaStream_t s, const char** why) {
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof(cfg));
   cfg.gridDim = dim3(2 * pairs_m, tiles_n, nb);
-  cfg.blockDim = dim3(THREADS, 1, 1);
+  cfg.blockDim = dim3(THREADS2, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
