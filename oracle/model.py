@@ -9,6 +9,8 @@ models with RoPE) is written out in ``decoder_logits``.  Per-example losses:
 
 * squared:  l_b = 1/2 * mean_o (f_bo - y_bo)^2
 * ce:       l_b = logsumexp(f_b) - f_{b, y_b}     (natural log)
+* chain_mse (the motivating example of Section 3): l_b = mean_o (y_M(f_bo) - y_bo)^2 with the
+  recursion y_0 = f, y_i = i * (2 + sin y_{i-1}) ** cos y_{i-1}, i = 1..M (Eq. 8).
 
 The weighted inner loss of the loss-weighting task (Section 5, L = alpha(eta, x) * NTP) is
 L_t = (1/B) sum_b sigmoid(eta_{t,b}) l_b, normalised by B, not by the sum of weights.
@@ -59,10 +61,20 @@ def mlp_forward(w, theta: torch.Tensor, x: torch.Tensor) -> torch.Tensor:
     return h
 
 
+def chain(f: torch.Tensor, M: int) -> torch.Tensor:
+    """The M-step elementwise recursion of the motivating example (Eq. 8)."""
+    y = f
+    for i in range(1, M + 1):
+        y = i * (2.0 + torch.sin(y)) ** torch.cos(y)
+    return y
+
+
 def per_example_loss(w, f: torch.Tensor, y: torch.Tensor) -> torch.Tensor:
     """Vector of per-example losses l_b (shape [B])."""
     if w.loss == "squared":
         return 0.5 * ((f - y) ** 2).mean(dim=1)
+    if w.loss == "chain_mse":
+        return ((chain(f, w.extra["chain_steps"]) - y) ** 2).mean(dim=1)
     if w.loss == "ce":
         lse = torch.logsumexp(f, dim=1)
         return lse - f.gather(1, y.long().view(-1, 1)).view(-1)

@@ -25,6 +25,12 @@ as in the loss-weighting and learned-learning-rate tasks of Section 5):
   alpha=1e-3, per-sequence weight logits, next-token cross-entropy.
 * ``decoder_large`` - 12 layers, d_model 1024, 16 heads, MLP 4096, sequences of 1024, batch 8,
   vocabulary 32768, T=16 heavy-ball (0.9) steps, per-sequence weights plus a scalar log-lr.
+* ``toy`` - the motivating example of Section 3: one D x D linear map followed by an M-step
+  elementwise recursion, mean-squared error on random targets, B=1024, D=4096, T=2 SGD steps
+  with lr 1e-3; the meta-parameter is the initial point theta_0 (MAML-style), so the
+  meta-gradient is d V / d theta_0 (meta_kind 0).  Inputs, targets and theta_0 are standard
+  normal; ``toy_bf16`` scales theta_0 by 1/sqrt(D) so that the recursion sees O(1) inputs
+  and bf16 GEMM operands stay meaningful.
 """
 from __future__ import annotations
 
@@ -37,7 +43,8 @@ import numpy as np
 
 # Stream indices (one per role).  Changing one changes every stored expected value.
 _STREAMS = {"x": 1, "teacher": 2, "noise": 3, "theta0": 4, "eta": 5, "outer": 6,
-            "tokens": 7, "labels": 8, "outer_noise": 9, "outer_labels": 10, "dir": 11}
+            "tokens": 7, "labels": 8, "outer_noise": 9, "outer_labels": 10, "dir": 11,
+            "targets": 12}
 
 
 def rng(seed: int, stream: str) -> np.random.Generator:
@@ -63,7 +70,7 @@ class Workload:
     name: str
     dims: list                      # MLP layer widths [d_in, h1, ..., d_out] (MLP only)
     act: str                        # hidden activation: ident|tanh|gelu|silu
-    loss: str                       # squared | ce
+    loss: str                       # squared | ce | chain_mse (toy task; extra["chain_steps"])
     precision: str                  # fp32 | bf16
     B: int
     T: int
@@ -169,6 +176,18 @@ WORKLOADS = {
 }
 
 
+def toy(name, D, B, M, T=2, precision="bf16", init_std=None, **kw):
+    """Motivating example: x theta followed by the M-step recursion, MSE, theta_0 meta-gradient."""
+    return Workload(name, [D, D], "ident", "chain_mse", precision, B=B, T=T, B_outer=B,
+                    alpha=1e-3, meta_kind=0, has_bias=False,
+                    init_std=1.0 if init_std is None else init_std,
+                    extra={"chain_steps": M}, **kw)
+
+
+WORKLOADS["toy"] = toy("toy", 4096, 1024, 8, precision="bf16", init_std=1.0 / 64.0)
+WORKLOADS["toy_fp32"] = toy("toy_fp32", 4096, 1024, 8, precision="fp32")
+
+
 def glorot_params(w: Workload, g: np.random.Generator) -> np.ndarray:
     """Glorot-uniform weights, zero biases, in the flat layout of ``layer_offsets``."""
     theta = np.zeros(w.n_params, dtype=np.float64)
@@ -251,6 +270,14 @@ def make_inputs(w: Workload) -> Inputs:
     rd = round_bf16 if w.precision == "bf16" else (lambda a: np.asarray(a, np.float32))
     x = rd(rng(w.seed, "x").standard_normal((w.T, w.B, din)))
     ox = rd(rng(w.seed, "outer").standard_normal((w.B_outer, din)))
+    if w.loss == "chain_mse":
+        # motivating example: standard-normal targets and theta_0 (scaled by init_std)
+        gt = rng(w.seed, "targets")
+        y = gt.standard_normal((w.T, w.B, dout)).astype(np.float32)
+        oy = gt.standard_normal((w.B_outer, dout)).astype(np.float32)
+        theta0 = (w.init_std * rng(w.seed, "theta0").standard_normal(w.n_params)).astype(np.float32)
+        return Inputs(theta0, np.zeros(0, np.float32), np.ascontiguousarray(x, np.float32), y,
+                      np.ascontiguousarray(ox, np.float32), oy)
     if w.loss == "ce":
         y = rng(w.seed, "labels").integers(0, dout, size=(w.T, w.B)).astype(np.int32)
         oy = rng(w.seed, "outer_labels").integers(0, dout, size=(w.B_outer,)).astype(np.int32)

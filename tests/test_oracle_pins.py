@@ -281,3 +281,49 @@ def test_zipf_ids_law():
     p /= p.sum()
     emp = np.bincount(ids, minlength=V) / ids.size
     assert np.abs(emp - p).max() < 4e-3
+
+
+# ---- motivating example of Section 3 (Eq. 8): theta_0 meta-gradient through the recursion
+TOY = synth.toy("toy_tiny", 4, 3, 3, precision="fp32")
+
+
+def test_toy_theta0_finite_differences():
+    """Every component of dV/dtheta_0 (MAML-style meta-parameter) against central finite
+    differences of the unrolled program, through the 3-step recursion."""
+    w = TOY
+    inp = synth.make_inputs(w)
+    res = om.meta_grad(w, inp)
+    h = 1e-6
+    fd = []
+    for k in range(w.n_params):
+        th_p = inp.theta0.astype(np.float64).copy()
+        th_m = th_p.copy()
+        th_p[k] += h
+        th_m[k] -= h
+        vp = om.value(w, synth.Inputs(th_p, inp.eta, inp.inner_x, inp.inner_y, inp.outer_x, inp.outer_y))
+        vm = om.value(w, synth.Inputs(th_m, inp.eta, inp.inner_x, inp.inner_y, inp.outer_x, inp.outer_y))
+        fd.append((vp - vm) / (2 * h))
+    assert _rel(res["d_theta0"], fd) < 1e-6
+    assert np.abs(res["d_theta0"]).max() > 1e-3
+
+
+def test_toy_zero_steps_is_linear_closed_form():
+    """With M = 0 the example is a linear model with L = mean((x W - y)^2): gradient
+    (2/(B O)) X^T (X W - Y), Hessian (2/(B O)) X^T X (x) I, adjoint recurrence of Eq. 5."""
+    w = synth.toy("toy_lin", 5, 4, 0, T=3, precision="fp32")
+    inp = synth.make_inputs(w)
+    D, B = w.dims[0], w.B
+    W = inp.theta0.astype(np.float64).reshape(D, D)
+    Xs = [inp.inner_x[t].astype(np.float64) for t in range(w.T)]
+    Ys = [inp.inner_y[t].astype(np.float64) for t in range(w.T)]
+    Ws = [W]
+    for t in range(w.T):
+        g = 2.0 / (B * D) * Xs[t].T @ (Xs[t] @ Ws[-1] - Ys[t])
+        Ws.append(Ws[-1] - w.alpha * g)
+    Xo, Yo = inp.outer_x.astype(np.float64), inp.outer_y.astype(np.float64)
+    tb = (2.0 / (w.B_outer * D) * Xo.T @ (Xo @ Ws[-1] - Yo)).reshape(-1)
+    for t in range(w.T - 1, -1, -1):
+        H = np.kron(2.0 / (B * D) * Xs[t].T @ Xs[t], np.eye(D))
+        tb = tb - w.alpha * H @ tb
+    res = om.meta_grad(w, inp)
+    assert _rel(res["d_theta0"], tb) < 1e-12
