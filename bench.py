@@ -10,7 +10,7 @@ Prints one JSON line (rank 0).  ``--impl reference`` times the CPU float64 oracl
 Multi-GPU runs are independent replicas (weak scaling), one process per GPU under torchrun.
 
 ``--workload`` measures another configuration the same way (deep MLP, the two decoder-only
-transformers); ``--hvp-mode rr`` runs the reverse-over-reverse sweep instead of the
+transformers, the motivating example of Section 3 with ``--chain-steps M``); ``--hvp-mode rr`` runs the reverse-over-reverse sweep instead of the
 mixed-mode one (MLPs), for the memory comparison.  Those lines skip the CPU baseline unless
 ``--cpu-baseline`` is given.
 """
@@ -41,6 +41,9 @@ WORKLOAD_DESCS = {
     "decoder_large": ("decoder-only transformer 12 x d1024, 16 heads, MLP 4096 GELU, vocab 32768, "
                       "S=1024, B=8, T=16 momentum 0.9, per-sequence weights + scalar log-lr, outer 8, "
                       "Zipf(1.1) token ids, bf16 GEMMs / fp32 state"),
+    "toy": ("motivating example of Section 3: y_0 = x theta (4096 x 4096, no bias), M = 8 steps "
+            "of y_i = i (2 + sin y_{i-1})^cos y_{i-1}, MSE on N(0,1) targets, B=1024, T=2 SGD "
+            "alpha=1e-3, theta_0 meta-gradient (16.8M), outer batch 1024, bf16 GEMMs / fp32 state"),
 }
 WORKLOAD_DESC = WORKLOAD_DESCS[WORKLOAD]
 
@@ -50,6 +53,28 @@ def _dist():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     return ws, rank, local
+
+
+def _max_over_ranks(x: float, ws: int, device) -> float:
+    """The largest of the ranks' values (the slowest replica sets the job's time)."""
+    if ws <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t)
+
+
+def _job_rate(total_ms: float, steps: int, ws: int, device):
+    """(ms per step of the slowest rank, whole-job meta-steps/s over all ranks)."""
+    ms = _max_over_ranks(total_ms, ws, device) / steps
+    return ms, ws * 1000.0 / ms
+
+
+def _replica_workload(w, rank: int):
+    """Replica r solves its own problem: the same shapes and distributions, seed + r."""
+    return w if rank == 0 else w.with_(seed=w.seed + rank)
 
 
 def _peaks():
@@ -181,19 +206,25 @@ def run_gpu(args):
     if ws > 1:
         dist.init_process_group("nccl")
     w = synth.WORKLOADS[args.workload]
+    if args.chain_steps is not None:
+        w = w.with_(extra={**w.extra, "chain_steps": args.chain_steps})
+    w = _replica_workload(w, rank)
     inp = synth.make_inputs(w)
     d = native.to_device_inputs(w, inp)
     mf = native.MixFlow.for_workload(w)
     rr = args.hvp_mode == "rr"
     loop = native.loop_desc_for(w, native.MF_HVP_REV_REV if rr else native.MF_HVP_MIXED_FOR)
     d_eta = torch.empty(w.n_eta, device="cuda")
+    # the meta-gradient lands in d_eta, or in d theta_0 when theta_0 is the meta-parameter
+    d_th = torch.empty(w.n_params, device="cuda") if w.n_eta == 0 else None
+    d_out = d_eta if d_th is None else d_th
     V = torch.empty(1, device="cuda")
     stream = torch.cuda.current_stream()
     flush = torch.empty(256 * 1024 * 1024 // 4, device="cuda")   # > 129 MB L2
 
     def step():
         mf.meta_grad(loop, d["theta0"], d["eta"], d["inner_x"], d["inner_y"], d["outer_x"],
-                     d["outer_y"], d_eta, None, V, stream=stream)
+                     d["outer_y"], d_eta, d_th, V, stream=stream)
 
     for _ in range(max(args.warmup, 3)):
         step()
@@ -220,14 +251,8 @@ def run_gpu(args):
     clocks = clk.stop()
     mf.sync()
     launches1, peak_ws = mf.stats()
-    ms_steps = [e0.elapsed_time(e1) for e0, e1 in evs]
-    total_ms = sum(ms_steps)
-    if ws > 1:
-        t = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t)
-    ms_per_step = total_ms / args.steps
-    value = ws * 1000.0 / ms_per_step
+    total_ms = sum(e0.elapsed_time(e1) for e0, e1 in evs)
+    ms_per_step, value = _job_rate(total_ms, args.steps, ws, "cuda")
 
     # ---- dominant kernel (tcgen05 dual GEMM): CUDA events around each of its launches,
     # recorded inside the replayed graph, over K more steps of the same workload ---------
@@ -255,7 +280,7 @@ def run_gpu(args):
 
     # ---- end to end through the public API with host buffers -------------------------------
     pin = {k: v.cpu().pin_memory() for k, v in d.items()}
-    h_eta = torch.empty(w.n_eta, pin_memory=True)
+    h_eta = torch.empty(d_out.numel(), pin_memory=True)
     h_V = torch.empty(1, pin_memory=True)
     h2d = sum(v.numel() * v.element_size() for v in pin.values())
     d2h = h_eta.numel() * 4 + 4
@@ -263,7 +288,7 @@ def run_gpu(args):
         for k in d:
             d[k].copy_(pin[k], non_blocking=True)
         step()
-        h_eta.copy_(d_eta, non_blocking=True)
+        h_eta.copy_(d_out, non_blocking=True)
         h_V.copy_(V, non_blocking=True)
     barrier()
     e_evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -274,24 +299,21 @@ def run_gpu(args):
         for k in d:
             d[k].copy_(pin[k], non_blocking=True)
         step()
-        h_eta.copy_(d_eta, non_blocking=True)
+        h_eta.copy_(d_out, non_blocking=True)
         h_V.copy_(V, non_blocking=True)
         e1.record(stream)
     barrier()
-    e2e_ms = sum(e0.elapsed_time(e1) for e0, e1 in e_evs) / args.steps
-    if ws > 1:
-        t = torch.tensor([e2e_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t)
+    _, e2e_value = _job_rate(sum(e0.elapsed_time(e1) for e0, e1 in e_evs), args.steps, ws,
+                             "cuda")
     mf.sync()
 
     inputs_bytes = h2d
-    peak_hbm_gb = (peak_ws + inputs_bytes + w.n_eta * 4) / 1e9
+    peak_hbm_gb = (peak_ws + inputs_bytes + d_out.numel() * 4) / 1e9
     # static part (Section 4's accounting): the theta_t store (and m_t store when the learning
     # rate is a meta-parameter), the inputs, eta and d eta; the rest is the sweep's dynamic memory
     lr_meta = bool(w.meta_kind & (synth.PARAM_LOGLR | synth.SCALAR_LOGLR))
     store = (w.T + 1 + (w.T if lr_meta else 0)) * w.n_params * 4
-    static_gb = (store + inputs_bytes + w.n_eta * 4) / 1e9
+    static_gb = (store + inputs_bytes + d_out.numel() * 4) / 1e9
 
     out = None
     if rank == 0:
@@ -308,7 +330,9 @@ def run_gpu(args):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic",
             "config": {"workload": WORKLOAD_DESCS[args.workload]
-                       + ("; reverse-over-reverse HVPs" if rr else ""),
+                       + ("; reverse-over-reverse HVPs" if rr else "")
+                       + (f"; M overridden to {args.chain_steps}"
+                          if args.chain_steps is not None else ""),
                        "parallelism": f"replicas x{ws}",
                        "l2": "flushed before every timed step (256 MB write outside the step events)"},
             "roofline": {"bound": "tensor", "kernel": "tc_dual_gemm_kernel (tcgen05 dual GEMM)",
@@ -325,7 +349,7 @@ def run_gpu(args):
                     "dynamic_gb": peak_hbm_gb - static_gb,
                     "hvp_mode": "reverse-over-reverse" if rr else "mixed forward-over-reverse"},
             "cpu_baseline": cpu,
-            "e2e": {"value": ws * 1000.0 / e2e_ms, "unit": "meta-steps/s",
+            "e2e": {"value": e2e_value, "unit": "meta-steps/s",
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": int(launches1 - launches0),
             "clocks": clocks,
@@ -348,6 +372,8 @@ def main():
     ap.add_argument("--cpu-baseline", action="store_true",
                     help="also time the oracle for a non-default workload or mode")
     ap.add_argument("--workload", default=WORKLOAD, choices=sorted(WORKLOAD_DESCS))
+    ap.add_argument("--chain-steps", type=int, default=None,
+                    help="M of the motivating example's recursion (--workload toy)")
     ap.add_argument("--hvp-mode", default="for", choices=["for", "rr"])
     args = ap.parse_args()
     if args.impl == "reference":

@@ -70,7 +70,8 @@ typedef enum {
 
 enum { MF_ARCH_MLP = 0, MF_ARCH_DECODER = 1 };
 enum { MF_ACT_IDENT = 0, MF_ACT_TANH = 1, MF_ACT_GELU = 2, MF_ACT_SILU = 3 };
-enum { MF_LOSS_SQUARED = 0, MF_LOSS_SOFTMAX_CE = 1, MF_LOSS_NEXT_TOKEN_CE = 2 };
+enum { MF_LOSS_SQUARED = 0, MF_LOSS_SOFTMAX_CE = 1, MF_LOSS_NEXT_TOKEN_CE = 2,
+       MF_LOSS_CHAIN_MSE = 3 };
 enum { MF_PREC_FP32 = 0, MF_PREC_BF16 = 1 };
 enum { MF_META_EXAMPLE_WEIGHTS = 1, MF_META_PARAM_LOGLR = 2, MF_META_SCALAR_LOGLR = 4 };
 enum { MF_HVP_MIXED_FOR = 0, MF_HVP_REV_REV = 1 };
@@ -86,13 +87,22 @@ enum { MF_HVP_MIXED_FOR = 0, MF_HVP_REV_REV = 1 };
  *  loss       MF_LOSS_SQUARED: l_b = 1/2 mean_o (f_bo - y_bo)^2, y float32 [rows][d_out];
  *             MF_LOSS_SOFTMAX_CE: l_b = logsumexp(f_b) - f_{b,y_b}, y int32 [rows];
  *             MF_LOSS_NEXT_TOKEN_CE (decoder only): x = y = int32 token ids [rows][seq_len+1],
- *             inputs ids[:, 0:S], targets ids[:, 1:S+1].
+ *             inputs ids[:, 0:S], targets ids[:, 1:S+1];
+ *             MF_LOSS_CHAIN_MSE (MLP; the motivating example of Section 3, Eq. 8): the
+ *             output f passes through y_0 = f, y_i = i (2 + sin y_{i-1})^cos y_{i-1},
+ *             i = 1..chain_steps, and l_b = mean_o (y_M,bo - y_bo)^2 (no 1/2), y float32
+ *             [rows][d_out].  In the mixed mode the recursion is evaluated inside the loss
+ *             kernel with its first and second derivatives and nothing of it is stored;
+ *             under MF_HVP_REV_REV the loss records the chain's tape (y_0..y_{M-1} and the
+ *             adjoints ybar_1..ybar_M, 2 M floats per output element) and the adjoint of its
+ *             backward reads it back, as reverse mode through the recursion does.
  *  precision  MF_PREC_FP32: float32 inputs, float32 GEMMs (SIMT);
  *             MF_PREC_BF16: bf16 inputs, bf16 tensor-core GEMMs with float32 accumulation;
  *             parameters, optimiser state, adjoints and meta-gradients stay float32.
  *  Decoder fields (MF_ARCH_DECODER; n_layers = blocks): d_model, n_heads (d_model/n_heads a
  *  multiple of 8), d_ff, vocab, seq_len (multiples of 8), rope_base (0 = 10000),
- *  rms_eps (0 = 1e-6).  dims/act/has_bias are ignored for decoders. */
+ *  rms_eps (0 = 1e-6).  dims/act/has_bias are ignored for decoders.
+ *  chain_steps  M of MF_LOSS_CHAIN_MSE (0..4096; ignored for other losses). */
 typedef struct {
   int arch;
   int n_layers;
@@ -103,6 +113,7 @@ typedef struct {
   int precision;
   int d_model, n_heads, d_ff, vocab, seq_len;
   float rope_base, rms_eps;
+  int chain_steps;
 } mf_model_desc;
 
 /* Inner loop (Eq. 2) and meta-parameters.
@@ -116,8 +127,9 @@ typedef struct {
  *             (Algorithm 2, the mixed-mode sweep).  MF_HVP_REV_REV: reverse-over-reverse
  *             (Algorithm 1's schedule: the inner backward is kept whole and differentiated
  *             again in reverse), the standard-AD baseline; same result, more workspace.
- *             MLPs keep every layer's dz and da; the decoder keeps the residual-stream
- *             cotangent at every block output and recomputes the cotangents inside a block.
+ *             MLPs keep every layer's dz and da (and the chain loss its tape); the decoder
+ *             keeps the residual-stream cotangent at every block output and recomputes the
+ *             cotangents inside a block.
  *  ckpt_every 1 = keep every theta_t in the checkpoint store (the only value accepted). */
 typedef struct {
   int T, B, B_outer;

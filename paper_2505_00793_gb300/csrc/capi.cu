@@ -108,6 +108,8 @@ struct Plan {
   bool ror = false;
   std::vector<size_t> o_SZ, o_SA, o_DAB, o_ZP;
   size_t o_DZB = 0, o_ZB = 0, o_AB = 0;
+  // ... and, for the chain loss, its tape: y_0..y_{M-1} and y-bar_1..y-bar_M per element
+  size_t o_CH = 0;
 };
 
 int n_update_tiles(const mf_ctx* h) {
@@ -175,6 +177,8 @@ Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slot
     p.o_DZB = take(static_cast<size_t>(rows) * md * 4);
     p.o_ZB = take(static_cast<size_t>(rows) * ld8(md) * es);
     p.o_AB = take(static_cast<size_t>(rows) * md * 4);
+    if (h->md.loss == MF_LOSS_CHAIN_MSE && h->md.chain_steps > 0)
+      p.o_CH = take(2 * static_cast<size_t>(h->md.chain_steps) * rows * h->dims[L] * 4);
   }
   p.bytes = o;
   return p;
@@ -321,6 +325,10 @@ struct Exec {
 
   // backward seed buffers of layer l (ping-pong, or the stored reverse graph)
   T* dz_buf(int l) const { return ror_store ? at<T>(p.o_SZ[l]) : at<T>(p.o_dZ[l & 1]); }
+  // loss kernel selector: 0 squared, 1 softmax CE, 2 chain MSE
+  int loss_kind() const {
+    return h->md.loss == MF_LOSS_SOFTMAX_CE ? 1 : h->md.loss == MF_LOSS_CHAIN_MSE ? 2 : 0;
+  }
 
   Exec(mf_ctx* h_, const Plan& p_, cudaStream_t s_)
       : h(h_), p(p_), s(s_), base(static_cast<char*>(h_->ws)) {
@@ -487,11 +495,12 @@ struct Exec {
             float* l_out, float* ld_out, float* d_eta) {
     const int L = h->L, C = h->dims[L];
     mf::LossArgs a;
-    a.loss = h->md.loss == MF_LOSS_SOFTMAX_CE ? 1 : 0;
+    a.loss = loss_kind();
+    a.chain = h->md.chain_steps;
     a.rows = rows; a.cols = C;
     a.F = at<float>(p.o_Z[L - 1]);
     a.Fd = dual ? at<float>(p.o_Zd[L - 1]) : nullptr;
-    if (a.loss == 0) a.Yf = static_cast<const float*>(y);
+    if (a.loss != 1) a.Yf = static_cast<const float*>(y);
     else a.Yi = static_cast<const int*>(y);
     a.eta_w = eta_w; a.ex_w = ex_w;
     a.inv_norm = 1.f / static_cast<float>(rows);
@@ -500,6 +509,10 @@ struct Exec {
     a.dF = dz_buf(L - 1); a.dFd = dual ? at<T>(p.o_dZd[b]) : nullptr;
     a.ldo = ld8(C);
     a.status = h->d_status;
+    if (ror_store && a.loss == 2 && a.chain > 0) {   // reverse mode records the chain's tape
+      a.tape = at<float>(p.o_CH);
+      a.ror = 1;
+    }
     mf::loss_seed<T>(a, s);
     launched();
   }
@@ -605,11 +618,12 @@ struct Exec {
         // loss Hessian along dzbar (this is the forward tangent of the logits): zbar_{L-1},
         // the per-example directional losses and the weight meta-gradient
         mf::LossArgs a;
-        a.loss = h->md.loss == MF_LOSS_SOFTMAX_CE ? 1 : 0;
+        a.loss = loss_kind();
+        a.chain = h->md.chain_steps;
         a.rows = rows; a.cols = dout;
         a.F = at<float>(p.o_Z[l]);
         a.Fd = at<float>(p.o_DZB);
-        if (a.loss == 0) a.Yf = static_cast<const float*>(y);
+        if (a.loss != 1) a.Yf = static_cast<const float*>(y);
         else a.Yi = static_cast<const int*>(y);
         a.eta_w = eta_w; a.ex_w = ex_w;
         a.inv_norm = 1.f / static_cast<float>(rows);
@@ -617,6 +631,10 @@ struct Exec {
         a.dF = nullptr; a.dFd = at<T>(p.o_ZB);
         a.ldo = ld8(dout);
         a.status = h->d_status;
+        if (a.loss == 2 && a.chain > 0) {   // adjoint of the chain's backward, from its tape
+          a.tape = at<float>(p.o_CH);
+          a.ror = 2;
+        }
         mf::loss_seed<T>(a, s);
         launched();
       }
@@ -997,7 +1015,10 @@ mf_status mf_create(const mf_model_desc* d, mf_handle* out) {
     for (int i = 0; i <= d->n_layers; ++i)
       if (d->dims[i] < 1 || d->dims[i] > (1 << 20)) return MF_ERR_INVALID_ARG;
     if (d->act < MF_ACT_IDENT || d->act > MF_ACT_SILU) return MF_ERR_INVALID_ARG;
-    if (d->loss != MF_LOSS_SQUARED && d->loss != MF_LOSS_SOFTMAX_CE) return MF_ERR_INVALID_ARG;
+    if (d->loss != MF_LOSS_SQUARED && d->loss != MF_LOSS_SOFTMAX_CE && d->loss != MF_LOSS_CHAIN_MSE)
+      return MF_ERR_INVALID_ARG;
+    if (d->loss == MF_LOSS_CHAIN_MSE && (d->chain_steps < 0 || d->chain_steps > 4096))
+      return MF_ERR_INVALID_ARG;
   }
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) { cudaGetLastError(); return MF_ERR_CUDA; }
@@ -1360,8 +1381,10 @@ extern "C" mf_status mf_hvp_noalloc(const mf_model_desc* d, int B, const float* 
   for (int i = 0; i <= d->n_layers; ++i)
     if (d->dims[i] < 1 || d->dims[i] > (1 << 20)) return MF_ERR_INVALID_ARG;
   if (d->act < MF_ACT_IDENT || d->act > MF_ACT_SILU) return MF_ERR_INVALID_ARG;
-  if (d->loss != MF_LOSS_SQUARED && d->loss != MF_LOSS_SOFTMAX_CE)
+  if (d->loss != MF_LOSS_SQUARED && d->loss != MF_LOSS_SOFTMAX_CE && d->loss != MF_LOSS_CHAIN_MSE)
     return d->loss == MF_LOSS_NEXT_TOKEN_CE ? MF_ERR_UNSUPPORTED : MF_ERR_INVALID_ARG;
+  if (d->loss == MF_LOSS_CHAIN_MSE && (d->chain_steps < 0 || d->chain_steps > 4096))
+    return MF_ERR_INVALID_ARG;
   if (d->precision != MF_PREC_FP32 && d->precision != MF_PREC_BF16) return MF_ERR_INVALID_ARG;
 
   // A handle-free context on the host stack; its workspace is the static device array.

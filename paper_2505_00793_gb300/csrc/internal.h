@@ -94,7 +94,8 @@ template <typename T>
 void fill_cols(const ColFill& f, int rows, cudaStream_t s);
 
 struct LossArgs {
-  int loss = 0;            // 0 squared, 1 softmax CE
+  int loss = 0;            // 0 squared, 1 softmax CE, 2 chain MSE (motivating example)
+  int chain = 0;           // chain MSE: steps M of the recursion
   int rows = 0, cols = 0;
   const float* F = nullptr;  const float* Fd = nullptr;  // logits [rows][cols], tangent
   const float* Yf = nullptr; const int* Yi = nullptr;    // targets
@@ -106,6 +107,11 @@ struct LossArgs {
   float* d_eta = nullptr;  // += sigmoid'(eta_w) * ld * inv_norm  [rows] (nullable)
   void* dF = nullptr; void* dFd = nullptr; int ldo = 0; // seeds in T [rows][ldo]
   int* status = nullptr;
+  // chain MSE by reverse-over-reverse: tape [2M][rows*cols] floats; ror = 1 records it in the
+  // primal loss (writes dF), ror = 2 runs the adjoint of the chain's backward along Fd
+  // (writes dFd, ld, d_eta) and overwrites the y-bar half with partial adjoints
+  float* tape = nullptr;
+  int ror = 0;
 };
 template <typename T>
 void loss_seed(const LossArgs& a, cudaStream_t s);

@@ -137,6 +137,176 @@ __global__ void loss_seed_kernel(const LossArgs a) {
   }
 }
 
+// Motivating example of Section 3 (Eq. 8): the model output is f = x theta followed by the
+// elementwise recursion y_0 = f, y_i = i (2 + sin y_{i-1})^cos y_{i-1}, i = 1..M, and
+// l_b = mean_o (y_M - t)^2.  Per element the recursion is carried with its first and second
+// derivatives in f (y', y''), so the loss seed 2/C r y' and its tangent 2/C (y'^2 + r y'') f'
+// come out of one pass; nothing of the recursion is stored.  One block per example.
+__device__ __forceinline__ void chain_eval(float f, int M, float& y, float& d1, float& d2) {
+  y = f; d1 = 1.f; d2 = 0.f;
+  for (int i = 1; i <= M; ++i) {
+    float sn, cs;
+    sincosf(y, &sn, &cs);
+    const float b = 2.f + sn;                 // >= 1
+    const float lb = logf(b);
+    const float g1 = -sn * lb + cs * cs / b;  // d/dy [cos y log(2 + sin y)]
+    const float g2 = -cs * lb - 3.f * sn * cs / b - cs * cs * cs / (b * b);
+    const float yi = static_cast<float>(i) * expf(cs * lb);
+    const float f1 = yi * g1, f2 = yi * (g1 * g1 + g2);
+    d2 = f2 * d1 * d1 + f1 * d2;
+    d1 = f1 * d1;
+    y = yi;
+  }
+}
+
+template <typename T>
+__global__ void chain_loss_kernel(const LossArgs a) {
+  pdl_entry();
+  __shared__ float red[2][8];
+  const int row = blockIdx.x;
+  const int C = a.cols;
+  const float* f = a.F + static_cast<int64_t>(row) * C;
+  const float* fd = a.Fd ? a.Fd + static_cast<int64_t>(row) * C : nullptr;
+  const float* t = a.Yf + static_cast<int64_t>(row) * C;
+  float w = 1.f, sg = 0.f;
+  if (a.ex_w) w = a.ex_w[row];
+  else if (a.eta_w) { sg = 1.f / (1.f + expf(-a.eta_w[row])); w = sg; }
+  const float invC = 1.f / static_cast<float>(C);
+  const float scale = w * a.inv_norm;
+  T* dF = static_cast<T*>(a.dF);
+  T* dFd = static_cast<T*>(a.dFd);
+  const int64_t orow = static_cast<int64_t>(row) * a.ldo;
+  float s2 = 0.f, s1 = 0.f;
+  bool bad = false;
+  for (int c = threadIdx.x; c < C; c += blockDim.x) {
+    float y, d1, d2;
+    chain_eval(f[c], a.chain, y, d1, d2);
+    const float r = y - t[c];
+    bad |= !isfinite(y) || !isfinite(d1);
+    s2 += r * r;
+    if (dF) dF[orow + c] = to_t<T>(scale * 2.f * invC * r * d1);
+    if (fd) {
+      const float ad = d1 * fd[c];
+      s1 += r * ad;
+      if (dFd) dFd[orow + c] = to_t<T>(scale * 2.f * invC * (d1 * ad + r * d2 * fd[c]));
+    }
+  }
+  if (bad && a.status) atomicExch(a.status, DEV_NONFINITE);
+  s2 = warp_sum(s2);
+  s1 = warp_sum(s1);
+  const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) { red[0][wid] = s2; red[1][wid] = s1; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float l = 0.f, ld = 0.f;
+    for (int k = 0; k < static_cast<int>(blockDim.x >> 5); ++k) { l += red[0][k]; ld += red[1][k]; }
+    l *= invC;
+    ld *= 2.f * invC;
+    if (a.l) a.l[row] = l;
+    if (a.ld) a.ld[row] = ld;
+    if (a.d_eta && a.eta_w) a.d_eta[row] = sg * (1.f - sg) * ld * a.inv_norm;
+  }
+}
+
+// The same loss by reverse-over-reverse (Algorithm 1's schedule applied inside the chain).
+// ror = 1, primal: forward y_i = phi_i(y_{i-1}) recording y_0..y_{M-1}, then the backward
+// ybar_M = c r, ybar_{i-1} = ybar_i phi_i'(y_{i-1}) recording ybar_1..ybar_M, with
+// c = 2 w / (B C) and phi_i' = y_i (d/dy)[cos y log(2 + sin y)]; dF = ybar_0.
+// ror = 2, adjoint of that backward along a_0 = Fd (the incoming adjoint of ybar_0): forward
+// a_i = a_{i-1} phi_i'(y_{i-1}) leaving yhat_{i-1} = a_{i-1} ybar_i phi_i''(y_{i-1}) in
+// ybar_i's slot, then yhat_M = c a_M and back yhat_{i-1} += yhat_i phi_i'(y_{i-1});
+// dFd = yhat_0, and ld = 2/C sum r a_M.  Both phases read the tape back instead of carrying
+// derivatives, so the tape (2 M floats per element) is what this mode holds beyond the
+// mixed mode.  Tape slot k of element e = row * C + c is at tape[k * rows * C + e].
+__device__ __forceinline__ float chain_step(int i, float y, float& g1, float& g2) {
+  float sn, cs;
+  sincosf(y, &sn, &cs);
+  const float b = 2.f + sn;
+  const float lb = logf(b);
+  g1 = -sn * lb + cs * cs / b;
+  g2 = -cs * lb - 3.f * sn * cs / b - cs * cs * cs / (b * b);
+  return static_cast<float>(i) * expf(cs * lb);
+}
+
+template <typename T>
+__global__ void chain_ror_kernel(const LossArgs a) {
+  pdl_entry();
+  __shared__ float red[2][8];
+  const int row = blockIdx.x;
+  const int C = a.cols, M = a.chain;
+  const int64_t E = static_cast<int64_t>(a.rows) * C;
+  const float* f = a.F + static_cast<int64_t>(row) * C;
+  const float* t = a.Yf + static_cast<int64_t>(row) * C;
+  float w = 1.f, sg = 0.f;
+  if (a.ex_w) w = a.ex_w[row];
+  else if (a.eta_w) { sg = 1.f / (1.f + expf(-a.eta_w[row])); w = sg; }
+  const float invC = 1.f / static_cast<float>(C);
+  const float cw = w * a.inv_norm * 2.f * invC;
+  const int64_t orow = static_cast<int64_t>(row) * a.ldo;
+  float s2 = 0.f, s1 = 0.f;
+  bool bad = false;
+  float g1, g2;
+  for (int c = threadIdx.x; c < C; c += blockDim.x) {
+    float* tp = a.tape + static_cast<int64_t>(row) * C + c;   // slot k at tp[k * E]
+    if (a.ror == 1) {
+      float y = f[c];
+      for (int i = 1; i <= M; ++i) {
+        tp[(i - 1) * E] = y;
+        y = chain_step(i, y, g1, g2);
+      }
+      const float yM = y;
+      const float r = yM - t[c];
+      s2 += r * r;
+      float yb = cw * r;
+      for (int i = M; i >= 1; --i) {
+        tp[(M + i - 1) * E] = yb;
+        const float yi = i == M ? yM : tp[i * E];
+        chain_step(i, tp[(i - 1) * E], g1, g2);
+        yb *= yi * g1;
+      }
+      bad |= !isfinite(yM) || !isfinite(yb);
+      if (a.dF) static_cast<T*>(a.dF)[orow + c] = to_t<T>(yb);
+    } else {
+      float ad = a.Fd[static_cast<int64_t>(row) * C + c];
+      const float yM = chain_step(M, tp[(M - 1) * E], g1, g2);
+      for (int i = 1; i <= M; ++i) {
+        const float yi = i == M ? yM : tp[i * E];
+        chain_step(i, tp[(i - 1) * E], g1, g2);
+        float* slot = tp + (M + i - 1) * E;
+        *slot = ad * *slot * yi * (g1 * g1 + g2);
+        ad *= yi * g1;
+      }
+      const float r = yM - t[c];
+      s1 += r * ad;
+      float yh = cw * ad;
+      for (int i = M; i >= 1; --i) {
+        const float yi = i == M ? yM : tp[i * E];
+        chain_step(i, tp[(i - 1) * E], g1, g2);
+        yh = tp[(M + i - 1) * E] + yh * yi * g1;
+      }
+      bad |= !isfinite(yh);
+      if (a.dFd) static_cast<T*>(a.dFd)[orow + c] = to_t<T>(yh);
+    }
+  }
+  if (bad && a.status) atomicExch(a.status, DEV_NONFINITE);
+  s2 = warp_sum(s2);
+  s1 = warp_sum(s1);
+  const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) { red[0][wid] = s2; red[1][wid] = s1; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float l = 0.f, ld = 0.f;
+    for (int k = 0; k < static_cast<int>(blockDim.x >> 5); ++k) { l += red[0][k]; ld += red[1][k]; }
+    if (a.ror == 1) {
+      if (a.l) a.l[row] = l * invC;
+    } else {
+      ld *= 2.f * invC;
+      if (a.ld) a.ld[row] = ld;
+      if (a.d_eta && a.eta_w) a.d_eta[row] = sg * (1.f - sg) * ld * a.inv_norm;
+    }
+  }
+}
+
 __global__ void sum_scaled_kernel(const float* __restrict__ x, int n, float scale,
                                   float* __restrict__ out) {
   pdl_entry();
@@ -336,6 +506,14 @@ void fill_cols(const ColFill& f, int rows, cudaStream_t s) {
 template <typename T>
 void loss_seed(const LossArgs& a, cudaStream_t s) {
   if (a.rows <= 0) return;
+  if ((a.loss == 1 && !a.Yi) || (a.loss != 1 && !a.Yf) || !a.F) return;   // no targets: nothing read
+  if (a.loss == 2) {
+    if (a.ror && a.tape && a.chain > 0 && (a.ror == 1 || a.Fd))
+      launch_k(chain_ror_kernel<T>, dim3(a.rows), dim3(256), 0, s, a);
+    else
+      launch_k(chain_loss_kernel<T>, dim3(a.rows), dim3(256), 0, s, a);
+    return;
+  }
   const int warps = 8;
   launch_k(loss_seed_kernel<T>, dim3((a.rows + warps - 1) / warps), dim3(warps * 32), 0, s, a);
 }

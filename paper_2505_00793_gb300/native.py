@@ -18,7 +18,7 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libmixflow.so")
 MF_MAX_LAYERS = 32
 MF_ARCH_MLP, MF_ARCH_DECODER = 0, 1
 ACTS = {"ident": 0, "tanh": 1, "gelu": 2, "silu": 3}
-LOSSES = {"squared": 0, "ce": 1, "next_token_ce": 2}
+LOSSES = {"squared": 0, "ce": 1, "next_token_ce": 2, "chain_mse": 3}
 PRECISIONS = {"fp32": 0, "bf16": 1}
 MF_META_EXAMPLE_WEIGHTS, MF_META_PARAM_LOGLR, MF_META_SCALAR_LOGLR = 1, 2, 4
 MF_HVP_MIXED_FOR, MF_HVP_REV_REV = 0, 1
@@ -38,7 +38,8 @@ class mf_model_desc(C.Structure):
     _fields_ = [("arch", C.c_int), ("n_layers", C.c_int), ("dims", C.c_int * (MF_MAX_LAYERS + 1)),
                 ("act", C.c_int), ("has_bias", C.c_int), ("loss", C.c_int), ("precision", C.c_int),
                 ("d_model", C.c_int), ("n_heads", C.c_int), ("d_ff", C.c_int), ("vocab", C.c_int),
-                ("seq_len", C.c_int), ("rope_base", C.c_float), ("rms_eps", C.c_float)]
+                ("seq_len", C.c_int), ("rope_base", C.c_float), ("rms_eps", C.c_float),
+                ("chain_steps", C.c_int)]
 
 
 class mf_loop_desc(C.Structure):
@@ -132,6 +133,7 @@ def model_desc_for(w) -> mf_model_desc:
     d.has_bias = 1 if w.has_bias else 0
     d.loss = LOSSES[w.loss]
     d.precision = PRECISIONS[w.precision]
+    d.chain_steps = int(w.extra.get("chain_steps", 0))
     return d
 
 
