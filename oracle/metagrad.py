@@ -2,10 +2,14 @@
 
 Test infrastructure only (see ``oracle/__init__.py``).
 
-Inner loop (Eq. 2 with the momentum state as the optimiser state upsilon):
-    m_{t+1}     = mu * m_t + grad L_t(theta_t),      m_0 = 0
-    theta_{t+1} = theta_t - lr (*) m_{t+1}
-with lr = alpha, or exp(eta_lr) per parameter, or exp(eta_s) for a scalar log-lr, and
+Inner loop (Eq. 2; the optimiser state upsilon is the momentum, or Adam's two moments):
+    SGD / heavy ball:  m_{t+1} = mu * m_t + g_t,   theta_{t+1} = theta_t - lr (*) m_{t+1}
+    Adam (Kingma & Ba, with bias correction; the optimiser of Section 5's inner loops):
+        m_{t+1} = b1 m_t + (1 - b1) g_t,   v_{t+1} = b2 v_t + (1 - b2) g_t^2
+        theta_{t+1} = theta_t - lr (*) (m_{t+1} / c1) / (sqrt(v_{t+1} / c2) + eps),
+        c1 = 1 - b1^(t+1),  c2 = 1 - b2^(t+1)
+with g_t = grad L_t(theta_t), zero initial state, lr = alpha, or exp(eta_lr) per parameter,
+or exp(eta_s) for a scalar log-lr, and
 L_t = (1/B) sum_b sigmoid(eta_{t,b}) l_b when per-example weight logits are meta-parameters.
 Outer loss V(theta_T) is the unweighted mean loss on the held-out batch.
 
@@ -69,30 +73,55 @@ def example_weights(w, eta: torch.Tensor, t: int):
     return torch.sigmoid(ex[t])
 
 
-def _step(w, theta, m, eta, x, y, t, create_graph):
-    """One inner update Phi(theta_t, m_t, eta, x_t) -> (theta_{t+1}, m_{t+1})."""
+def _safe_sqrt(v):
+    """sqrt(v) whose derivative at v = 0 is taken as 0.  v_{t+1} = 0 only where every
+    gradient so far was exactly 0, and there m_{t+1} = 0 and dv/dg = 2 (1 - b2) g = 0 too, so
+    every path through that derivative is multiplied by 0 (the limit of the product)."""
+    pos = v > 0
+    return torch.where(pos, torch.sqrt(torch.where(pos, v, torch.ones_like(v))),
+                       torch.zeros_like(v))
+
+
+def n_state(w) -> int:
+    """Number of optimiser state tensors: m for SGD / heavy ball, (m, v) for Adam."""
+    return 2 if getattr(w, "optimizer", "sgd") == "adam" else 1
+
+
+def _step(w, theta, state, eta, x, y, t, create_graph):
+    """One inner update Phi(theta_t, upsilon_t, eta, x_t) -> (theta_{t+1}, upsilon_{t+1})."""
     L = model.weighted_inner_loss(w, theta, x, y, example_weights(w, eta, t))
     (g,) = torch.autograd.grad(L, theta, create_graph=create_graph)
+    lr = learning_rate(w, eta)
+    if n_state(w) == 2:
+        m, v = state
+        m_next = w.beta1 * m + (1.0 - w.beta1) * g
+        v_next = w.beta2 * v + (1.0 - w.beta2) * g * g
+        c1 = 1.0 - w.beta1 ** (t + 1)
+        c2 = 1.0 - w.beta2 ** (t + 1)
+        theta_next = theta - lr * (m_next / c1) / (_safe_sqrt(v_next / c2) + w.adam_eps)
+        return theta_next, (m_next, v_next)
+    (m,) = state
     m_next = w.momentum * m + g
-    theta_next = theta - learning_rate(w, eta) * m_next
-    return theta_next, m_next
+    theta_next = theta - lr * m_next
+    return theta_next, (m_next,)
 
 
 def rollout(w, inp, eta=None):
-    """Inner rollout storing every (theta_t, m_t), t = 0..T.  Returns (thetas, ms)."""
+    """Inner rollout storing every (theta_t, upsilon_t), t = 0..T.  Returns (thetas, states)
+    with states[t] a tuple of state tensors."""
     eta = t64(inp.eta if eta is None else eta)
     X, Y = t64(inp.inner_x), t64(inp.inner_y)
     theta = t64(inp.theta0)
-    m = torch.zeros_like(theta)
-    thetas, ms = [theta], [m]
+    state = tuple(torch.zeros_like(theta) for _ in range(n_state(w)))
+    thetas, states = [theta], [state]
     for t in range(w.T):
         th = theta.clone().requires_grad_(True)
         with torch.enable_grad():
-            tn, mn = _step(w, th, m, eta, X[t], Y[t], t, create_graph=False)
-        theta, m = tn.detach(), mn.detach()
+            tn, sn = _step(w, th, state, eta, X[t], Y[t], t, create_graph=False)
+        theta, state = tn.detach(), tuple(v.detach() for v in sn)
         thetas.append(theta)
-        ms.append(m)
-    return thetas, ms
+        states.append(state)
+    return thetas, states
 
 
 def value(w, inp, eta=None) -> float:
@@ -108,24 +137,26 @@ def meta_grad(w, inp, eta=None):
     """
     eta0 = t64(inp.eta if eta is None else eta)
     X, Y = t64(inp.inner_x), t64(inp.inner_y)
-    thetas, ms = rollout(w, inp, eta0)
-    # Outer gradient (Eq. 4): cotangent (dV/d theta_T, 0) on (theta_T, m_T).
+    thetas, states = rollout(w, inp, eta0)
+    # Outer gradient (Eq. 4): cotangent (dV/d theta_T, 0) on (theta_T, upsilon_T).
     thT = thetas[-1].clone().requires_grad_(True)
     with torch.enable_grad():
         V = model.outer_loss(w, thT, t64(inp.outer_x), t64(inp.outer_y))
         (theta_bar,) = torch.autograd.grad(V, thT)
-    m_bar = torch.zeros_like(theta_bar)
+    s_bar = tuple(torch.zeros_like(theta_bar) for _ in range(n_state(w)))
     d_eta = torch.zeros_like(eta0)
     for t in range(w.T - 1, -1, -1):
         th = thetas[t].clone().requires_grad_(True)
-        m = ms[t].clone().requires_grad_(True)
+        st = tuple(v.clone().requires_grad_(True) for v in states[t])
         et = eta0.clone().requires_grad_(True)
         with torch.enable_grad():
-            tn, mn = _step(w, th, m, et, X[t], Y[t], t, create_graph=True)
-            gt, gm, ge = torch.autograd.grad((tn, mn), (th, m, et), (theta_bar, m_bar),
-                                             allow_unused=True)
-        theta_bar = gt
-        m_bar = gm if gm is not None else torch.zeros_like(m_bar)
+            tn, sn = _step(w, th, st, et, X[t], Y[t], t, create_graph=True)
+            grads = torch.autograd.grad((tn, *sn), (th, *st, et), (theta_bar, *s_bar),
+                                        allow_unused=True)
+        theta_bar = grads[0]
+        s_bar = tuple(gs if gs is not None else torch.zeros_like(theta_bar)
+                      for gs in grads[1:-1])
+        ge = grads[-1]
         if ge is not None:
             d_eta = d_eta + ge
     return {"d_eta": d_eta.numpy(), "d_theta0": theta_bar.numpy(), "V": float(V.detach())}

@@ -76,7 +76,11 @@ class Workload:
     T: int
     B_outer: int
     alpha: float = 0.0              # constant lr (when no log-lr meta-parameter)
-    momentum: float = 0.0
+    momentum: float = 0.0           # heavy-ball coefficient (optimizer "sgd")
+    optimizer: str = "sgd"          # sgd (plain or heavy-ball) | adam
+    beta1: float = 0.9              # Adam moment decays and epsilon
+    beta2: float = 0.999
+    adam_eps: float = 1e-8
     meta_kind: int = EXAMPLE_WEIGHTS
     loglr_mean: float = 0.0
     loglr_std: float = 0.0

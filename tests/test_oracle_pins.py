@@ -9,7 +9,9 @@
 * P4  explicit Hessian of a 8->16->1 tanh MLP by finite differences of the gradient, which
       is itself pinned to finite differences of the plain forward loss.
 * P5  special cases: alpha = 0 gives zero weight meta-gradient and dV/dtheta_0 = grad V;
-      T = 1 gives d eta_b = -(alpha/B) sigma'(eta_b) grad l_b(theta_0) . grad V(theta_1).
+      T = 1 gives d eta_b = -(alpha/B) sigma'(eta_b) grad l_b(theta_0) . grad V(theta_1);
+      Adam's first step from zero moments is theta_1 = theta_0 - lr g / (|g| + eps) exactly,
+      so d eta_b = (sigma'(eta_b)/B) grad l_b . (-lr eps / (|g| + eps)^2 (*) grad V(theta_1)).
 * tangent losses dl_b/dtheta . v against finite differences of l_b.
 """
 import math
@@ -48,6 +50,13 @@ SMALL = {
     "ex_slr_tanh_mom": synth.Workload("ex_slr_tanh_mom", [5, 7, 2], "tanh", "squared", "fp32",
                                       B=4, T=3, B_outer=6, momentum=0.5, meta_kind=EX | SLR,
                                       noise_std=0.1, extra={"scalar_loglr": math.log(0.3)}),
+    # Adam inner loops (eps large enough that its derivative terms are not negligible)
+    "adam_ex_gelu": synth.Workload("adam_ex_gelu", [5, 6, 3], "gelu", "ce", "fp32", B=4, T=3,
+                                   B_outer=5, alpha=0.05, optimizer="adam", adam_eps=1e-3),
+    "adam_plr_tanh": synth.Workload("adam_plr_tanh", [4, 5, 2], "tanh", "squared", "fp32", B=5,
+                                    T=3, B_outer=4, meta_kind=PLR, optimizer="adam",
+                                    beta1=0.8, beta2=0.95, adam_eps=1e-2,
+                                    loglr_mean=math.log(0.02), loglr_std=0.1, noise_std=0.1),
 }
 
 
@@ -205,6 +214,27 @@ def test_p5_single_step():
         glb = om.grad(w, inp.theta0, inp.inner_x[0][b:b + 1], inp.inner_y[0][b:b + 1])
         expect.append(-(w.alpha / w.B) * s[b] * (1 - s[b]) * glb @ gV)
     assert _rel(res["d_eta"], expect) < 1e-12
+
+
+def test_p5_adam_single_step():
+    w = synth.Workload("adam1", [4, 6, 2], "tanh", "squared", "fp32", B=5, T=1, B_outer=4,
+                       alpha=0.05, optimizer="adam", adam_eps=1e-2, noise_std=0.1)
+    inp = synth.make_inputs(w)
+    eta = inp.eta.astype(np.float64)
+    s = 1 / (1 + np.exp(-eta))
+    g = om.grad(w, inp.theta0, inp.inner_x[0], inp.inner_y[0], s)
+    theta1 = inp.theta0.astype(np.float64) - w.alpha * g / (np.abs(g) + w.adam_eps)
+    thetas, _ = om.rollout(w, inp)
+    assert _rel(thetas[1].numpy(), theta1) < 1e-14
+    gV = om.grad(w, theta1, inp.outer_x, inp.outer_y)
+    dthdg = -w.alpha * w.adam_eps / (np.abs(g) + w.adam_eps) ** 2
+    expect = []
+    for b in range(w.B):
+        glb = om.grad(w, inp.theta0, inp.inner_x[0][b:b + 1], inp.inner_y[0][b:b + 1])
+        expect.append(s[b] * (1 - s[b]) / w.B * glb @ (dthdg * gV))
+    res = om.meta_grad(w, inp)
+    assert _rel(res["d_eta"], expect) < 1e-12
+    assert np.abs(expect).max() > 1e-6
 
 
 def test_tangent_losses_fd():

@@ -121,12 +121,20 @@ class Unrolled:
             o += P
         if w.meta_kind & SLR:
             lr = [mp.exp(eta[o])] * P
-        th, m = list(theta0), [mp.mpf(0)] * P
+        th, m, v = list(theta0), [mp.mpf(0)] * P, [mp.mpf(0)] * P
         for t in range(w.T):
             c = [1 / (1 + mp.exp(-v)) for v in ex[t * B:(t + 1) * B]] if ex else [mp.mpf(1)] * B
             g = self.grad(*th, *c, *self.x[t], *self.y[t])
-            m = [w.momentum * mi + gi for mi, gi in zip(m, g)]
-            th = [ti - li * mi for ti, li, mi in zip(th, lr, m)]
+            if w.optimizer == "adam":   # Kingma & Ba with bias correction
+                b1, b2 = mp.mpf(w.beta1), mp.mpf(w.beta2)
+                m = [b1 * mi + (1 - b1) * gi for mi, gi in zip(m, g)]
+                v = [b2 * vi + (1 - b2) * gi * gi for vi, gi in zip(v, g)]
+                c1, c2 = 1 - b1 ** (t + 1), 1 - b2 ** (t + 1)
+                th = [ti - li * (mi / c1) / (mp.sqrt(vi / c2) + mp.mpf(w.adam_eps))
+                      for ti, li, mi, vi in zip(th, lr, m, v)]
+            else:
+                m = [w.momentum * mi + gi for mi, gi in zip(m, g)]
+                th = [ti - li * mi for ti, li, mi in zip(th, lr, m)]
         return self.outer(*th, *self.ox, *self.oy)
 
     def meta_grad(self):
@@ -159,6 +167,13 @@ CASES = {
                                   B_outer=2, alpha=0.4, noise_std=0.2, eta_std=1.0),
     # the motivating example of Section 3 (Eq. 8), M = 2, theta_0 the meta-parameter
     "toy_chain": synth.toy("s4", 2, 2, 2, T=2, precision="fp32", init_std=0.7),
+    # Adam inner loops: weight logits with cross-entropy, per-parameter log learning rates
+    "adam_ex_ce": synth.Workload("s5", [3, 3, 3], "tanh", "ce", "fp32", B=3, T=3, B_outer=2,
+                                 alpha=0.05, optimizer="adam", adam_eps=1e-3, eta_std=1.0),
+    "adam_plr": synth.Workload("s6", [2, 3, 2], "silu", "squared", "fp32", B=2, T=2, B_outer=3,
+                               meta_kind=PLR, optimizer="adam", beta1=0.8, beta2=0.95,
+                               adam_eps=1e-2, loglr_mean=math.log(0.03), loglr_std=0.2,
+                               noise_std=0.1),
 }
 
 
