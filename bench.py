@@ -208,12 +208,15 @@ def run_gpu(args):
     w = synth.WORKLOADS[args.workload]
     if args.chain_steps is not None:
         w = w.with_(extra={**w.extra, "chain_steps": args.chain_steps})
+    if args.optimizer == "adam":
+        w = w.with_(optimizer="adam", momentum=0.0, adam_eps=args.adam_eps)
     w = _replica_workload(w, rank)
     inp = synth.make_inputs(w)
     d = native.to_device_inputs(w, inp)
     mf = native.MixFlow.for_workload(w)
     rr = args.hvp_mode == "rr"
-    loop = native.loop_desc_for(w, native.MF_HVP_REV_REV if rr else native.MF_HVP_MIXED_FOR)
+    loop = native.loop_desc_for(w, native.MF_HVP_REV_REV if rr else native.MF_HVP_MIXED_FOR,
+                                ckpt_every=args.ckpt_every)
     d_eta = torch.empty(w.n_eta, device="cuda")
     # the meta-gradient lands in d_eta, or in d theta_0 when theta_0 is the meta-parameter
     d_th = torch.empty(w.n_params, device="cuda") if w.n_eta == 0 else None
@@ -312,7 +315,14 @@ def run_gpu(args):
     # static part (Section 4's accounting): the theta_t store (and m_t store when the learning
     # rate is a meta-parameter), the inputs, eta and d eta; the rest is the sweep's dynamic memory
     lr_meta = bool(w.meta_kind & (synth.PARAM_LOGLR | synth.SCALAR_LOGLR))
-    store = (w.T + 1 + (w.T if lr_meta else 0)) * w.n_params * 4
+    k = min(max(args.ckpt_every, 1), w.T)
+    if w.optimizer == "adam":       # m_t and v_t for every t (their cotangents are dynamic)
+        m_slots = 2 * (w.T // k + k - 1)
+    elif lr_meta:
+        m_slots = w.T // k + k - 1
+    else:
+        m_slots = (w.T // k + 1) if (w.momentum != 0 and k > 1) else 0
+    store = ((w.T // k + k) + m_slots) * w.n_params * 4
     static_gb = (store + inputs_bytes + d_out.numel() * 4) / 1e9
 
     out = None
@@ -332,7 +342,11 @@ def run_gpu(args):
             "config": {"workload": WORKLOAD_DESCS[args.workload]
                        + ("; reverse-over-reverse HVPs" if rr else "")
                        + (f"; M overridden to {args.chain_steps}"
-                          if args.chain_steps is not None else ""),
+                          if args.chain_steps is not None else "")
+                       + (f"; checkpoint store in segments of {args.ckpt_every} steps"
+                          if args.ckpt_every > 1 else "")
+                       + (f"; Adam inner optimiser (b1 0.9, b2 0.999, eps {args.adam_eps:g}) "
+                          "in place of SGD" if args.optimizer == "adam" else ""),
                        "parallelism": f"replicas x{ws}",
                        "l2": "flushed before every timed step (256 MB write outside the step events)"},
             "roofline": {"bound": "tensor", "kernel": "tc_dual_gemm_kernel (tcgen05 dual GEMM)",
@@ -375,6 +389,11 @@ def main():
     ap.add_argument("--chain-steps", type=int, default=None,
                     help="M of the motivating example's recursion (--workload toy)")
     ap.add_argument("--hvp-mode", default="for", choices=["for", "rr"])
+    ap.add_argument("--optimizer", default="sgd", choices=["sgd", "adam"],
+                    help="inner optimiser (adam replaces the workload's SGD / momentum)")
+    ap.add_argument("--adam-eps", type=float, default=1e-8)
+    ap.add_argument("--ckpt-every", type=int, default=1,
+                    help="segment length of the theta_t store (1 = keep every theta_t)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

@@ -75,6 +75,7 @@ enum { MF_LOSS_SQUARED = 0, MF_LOSS_SOFTMAX_CE = 1, MF_LOSS_NEXT_TOKEN_CE = 2,
 enum { MF_PREC_FP32 = 0, MF_PREC_BF16 = 1 };
 enum { MF_META_EXAMPLE_WEIGHTS = 1, MF_META_PARAM_LOGLR = 2, MF_META_SCALAR_LOGLR = 4 };
 enum { MF_HVP_MIXED_FOR = 0, MF_HVP_REV_REV = 1 };
+enum { MF_OPTIM_SGD = 0, MF_OPTIM_ADAM = 1 };
 
 #define MF_MAX_LAYERS 32
 
@@ -119,7 +120,7 @@ typedef struct {
 /* Inner loop (Eq. 2) and meta-parameters.
  *  T          inner steps (>= 1);  B rows per inner batch;  B_outer rows of the outer batch.
  *  alpha      constant learning rate (used when no log-lr meta-parameter is set).
- *  momentum   heavy-ball coefficient mu in [0, 1) (0 = plain SGD).
+ *  momentum   heavy-ball coefficient mu in [0, 1) (0 = plain SGD); must be 0 with Adam.
  *  meta_kind  bit mask of MF_META_*; eta is laid out as [T*B example-weight logits]
  *             [P per-parameter log-lrs][1 scalar log-lr], in that order, for the bits set.
  *             PARAM_LOGLR and SCALAR_LOGLR are mutually exclusive.
@@ -130,13 +131,35 @@ typedef struct {
  *             MLPs keep every layer's dz and da (and the chain loss its tape); the decoder
  *             keeps the residual-stream cotangent at every block output and recomputes the
  *             cotangents inside a block.
- *  ckpt_every 1 = keep every theta_t in the checkpoint store (the only value accepted). */
+ *  ckpt_every k: segment length of the checkpoint store (Section 4).  0 or 1 keeps every
+ *             theta_t (and m_t when needed): T+1 parameter slots.  k > 1 keeps theta_t only
+ *             for t a multiple of k, plus k-1 slots for one segment; the sweep re-runs each
+ *             earlier segment's rollout from its checkpoint before walking it back, with the
+ *             same kernels, so results are bit-identical to k = 1 for one extra rollout's
+ *             work.  theta slots: floor(T/k) + k (k = sqrt(T) minimises them).  m slots:
+ *             floor(T/k) + k - 1 when the learning rate is a meta-parameter (the sweep reads
+ *             every m_t); floor(T/k) + 1 for momentum alone with k > 1 (checkpoints plus one
+ *             running slot, to restart segments); none otherwise.  k > T acts as T.
+ *             Negative values are MF_ERR_INVALID_ARG.
+ *  optimizer  MF_OPTIM_SGD (plain or heavy-ball, the default when the field is 0) or
+ *             MF_OPTIM_ADAM, the inner optimiser of Section 5's language-model tasks
+ *             (Kingma & Ba, with bias correction): m' = b1 m + (1-b1) g, v' = b2 v + (1-b2) g^2,
+ *             theta' = theta - lr (m'/c1) / (sqrt(v'/c2) + eps), c1 = 1 - b1^(t+1),
+ *             c2 = 1 - b2^(t+1), zero initial moments; lr as for SGD (alpha or exp of a
+ *             log-lr meta-parameter).  The sweep reverses each step elementwise: the HVP's
+ *             tangent is the gradient cotangent g-bar_t = (1-b1) M + 2 (1-b2) g_t V, with M, V
+ *             the cotangents of m_{t+1}, v_{t+1}; g_t is recovered as (m_{t+1} - b1 m_t)/(1-b1).
+ *             The store keeps m_t and v_t for every t (segmented like theta) plus two
+ *             cotangent vectors: 2 (floor(T/k) + k - 1) + 2 extra |theta| slots.
+ *  beta1, beta2, adam_eps  Adam's decays in [0, 1) and epsilon (> 0); ignored for SGD. */
 typedef struct {
   int T, B, B_outer;
   float alpha, momentum;
   int meta_kind;
   int hvp_mode;
   int ckpt_every;
+  int optimizer;
+  float beta1, beta2, adam_eps;
 } mf_loop_desc;
 
 /* Create a handle for one inner-model architecture.  *out receives a library-owned handle.

@@ -8,6 +8,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <cmath>
 #include <mutex>
 #include <string>
 #include <utility>
@@ -687,8 +688,15 @@ mf_status validate_loop(mf_ctx* h, const mf_loop_desc* lp) {
   if (lp->hvp_mode != MF_HVP_MIXED_FOR && lp->hvp_mode != MF_HVP_REV_REV)
     return fail(h, MF_ERR_INVALID_ARG, "unknown hvp_mode");
 
-  if (lp->ckpt_every != 1 && lp->ckpt_every != 0)
-    return fail(h, MF_ERR_UNSUPPORTED, "only ckpt_every = 1 is implemented");
+  if (lp->ckpt_every < 0) return fail(h, MF_ERR_INVALID_ARG, "ckpt_every must be >= 0");
+  if (lp->optimizer != MF_OPTIM_SGD && lp->optimizer != MF_OPTIM_ADAM)
+    return fail(h, MF_ERR_INVALID_ARG, "unknown optimizer");
+  if (lp->optimizer == MF_OPTIM_ADAM &&
+      (lp->momentum != 0.f || !(lp->beta1 >= 0.f && lp->beta1 < 1.f) ||
+       !(lp->beta2 >= 0.f && lp->beta2 < 1.f) || !(lp->adam_eps > 0.f) ||
+       !std::isfinite(lp->adam_eps)))
+    return fail(h, MF_ERR_INVALID_ARG,
+                "Adam needs momentum 0, beta1 and beta2 in [0, 1) and a finite adam_eps > 0");
   return MF_OK;
 }
 
@@ -713,6 +721,51 @@ mf_status check_x(mf_ctx* h, const void* x, int rows) {
 size_t y_stride_bytes(const mf_ctx* h, int rows) {
   return h->md.loss == MF_LOSS_SOFTMAX_CE ? static_cast<size_t>(rows) * 4
                                           : static_cast<size_t>(rows) * h->dims[h->L] * 4;
+}
+
+// Checkpoint store of the sweep (Section 4; segment rematerialisation when k > 1).  theta_t
+// lives in checkpoint slot t/k when t is a multiple of k, else in segment slot (t mod k) - 1;
+// the segment slots hold one segment at a time and the sweep refills them from the segment's
+// checkpoint.  m_t (t >= 1) is kept the same way, without a slot for m_0 = 0, when the sweep
+// reads it (a log-learning-rate meta-parameter).  When only a recompute needs it (momentum
+// with k > 1), the checkpoints keep it and one running slot carries it inside a segment.
+struct Store {
+  int k = 1, T = 0, n_ck = 1;
+  bool m_kept = false, m_run_only = false;
+  bool adam = false;   // Adam: v_t kept like m_t after the m slots, then m-bar and v-bar
+  int theta_idx(int t) const { return t % k == 0 ? t / k : n_ck + t % k - 1; }
+  int m_idx(int t) const {
+    return t % k == 0 ? t / k - 1 : (m_run_only ? n_ck - 1 : n_ck - 1 + t % k - 1);
+  }
+  int theta_slots() const { return n_ck + k - 1; }
+  int m_slots() const {
+    const int nm = !m_kept ? 0 : m_run_only ? n_ck : n_ck - 1 + k - 1;
+    return adam ? 2 * nm + 2 : nm;
+  }
+  int v_idx(int t) const { return n_ck - 1 + k - 1 + m_idx(t); }
+  int mbar_idx() const { return 2 * (n_ck - 1 + k - 1); }
+};
+
+Store make_store(const mf_loop_desc* lp) {
+  Store st;
+  st.T = lp->T;
+  st.k = lp->ckpt_every <= 1 ? 1 : std::min(lp->ckpt_every, lp->T);
+  st.n_ck = lp->T / st.k + 1;
+  const bool lr_meta = lp->meta_kind & (MF_META_PARAM_LOGLR | MF_META_SCALAR_LOGLR);
+  st.adam = lp->optimizer == MF_OPTIM_ADAM;
+  st.m_kept = lr_meta || st.adam || (lp->momentum != 0.f && st.k > 1);
+  st.m_run_only = st.m_kept && !lr_meta && !st.adam;
+  return st;
+}
+
+// Adam's hyper-parameters and the bias corrections of inner step j on an update.
+void set_adam(mf::LayerUpdArgs& a, const mf_loop_desc* lp, int j) {
+  a.adam = 1;
+  a.b1 = lp->beta1;
+  a.b2 = lp->beta2;
+  a.eps = lp->adam_eps;
+  a.c1 = static_cast<float>(1.0 - std::pow(static_cast<double>(lp->beta1), j + 1));
+  a.c2 = static_cast<float>(1.0 - std::pow(static_cast<double>(lp->beta2), j + 1));
 }
 
 struct LrSel {
@@ -740,50 +793,75 @@ LrSel lr_select(const mf_ctx* h, const mf_loop_desc* lp, const float* eta) {
   return r;
 }
 
-// Inner rollout (Eq. 2).  With store_all, theta slot t holds theta_t and m slot j holds
-// m_{j+1} when the learning rate is a meta-parameter; otherwise two theta slots ping-pong.
-// Each step's update (K4) also casts theta_{t+1} into the GEMM operand copies.  X is the
-// model executor (MLP or decoder).
+// One inner step (Eq. 2): forward, loss and backward at theta, then K4 writes theta' (and m'
+// when m_out is set) and casts theta' into the GEMM operand copies.  m = null reads m_t = 0.
 template <typename X>
-void rollout(X& ex, const mf_loop_desc* lp, const float* eta, const void* inner_x,
-             const void* inner_y, const LrSel& lr, bool store_all, float** theta_T) {
+void inner_step(X& ex, const mf_loop_desc* lp, const float* eta, const void* inner_x,
+                const void* inner_y, const LrSel& lr, int t, const float* theta, const float* m,
+                float* theta_out, float* m_out, const float* v = nullptr,
+                float* v_out = nullptr) {
   mf_ctx* h = ex.h;
   const int B = lp->B;
-  const size_t xs = ex.x_step_bytes(B);
-  const size_t ys = ex.y_step_bytes(B);
-  float* m_run = (lp->momentum != 0.f && !lr.lr_meta) ? ex.u_buf() : nullptr;
-  if (m_run) { mf::fill(m_run, h->P, 0.f, ex.s); ex.launched(); }
-  const float* m_prev = nullptr;
-  ex.cast_params(ex.theta_slot(0), false);
-  for (int t = 0; t < lp->T; ++t) {
-    float* th = ex.theta_slot(store_all ? t : (t & 1));
-    float* th_next = ex.theta_slot(store_all ? t + 1 : ((t + 1) & 1));
-    const void* x = static_cast<const char*>(inner_x) + xs * t;
-    const void* y = static_cast<const char*>(inner_y) + ys * t;
-    ex.forward(B, x, th, nullptr, false);
-    const float* ew = (lp->meta_kind & MF_META_EXAMPLE_WEIGHTS) ? eta + static_cast<int64_t>(t) * B : nullptr;
-    ex.loss(B, false, y, ew, nullptr, nullptr, nullptr, nullptr);
-    float* g = ex.g_buf();
-    ex.backward(B, false, nullptr, g);
-    float* m_out = nullptr;
-    if (lr.lr_meta && store_all) m_out = ex.m_slot(t);
-    else if (lr.lr_meta) m_out = ex.m_slot(0);
-    else if (m_run) m_out = m_run;
-    mf::LayerUpdArgs a;
-    a.mode = mf::LU_ROLLOUT;
-    a.theta = th;
-    a.m = lr.lr_meta ? m_prev : m_run;
-    a.g = g;
-    a.theta_out = th_next;
-    a.m_out = m_out;
-    a.mu = lp->momentum;
-    a.lr = lr.lr;
-    a.status = h->d_status;
-    ex.update(a);
-    m_prev = m_out;
+  const void* x = static_cast<const char*>(inner_x) + ex.x_step_bytes(B) * t;
+  const void* y = static_cast<const char*>(inner_y) + ex.y_step_bytes(B) * t;
+  ex.forward(B, x, theta, nullptr, false);
+  const float* ew = (lp->meta_kind & MF_META_EXAMPLE_WEIGHTS) ? eta + static_cast<int64_t>(t) * B : nullptr;
+  ex.loss(B, false, y, ew, nullptr, nullptr, nullptr, nullptr);
+  float* g = ex.g_buf();
+  ex.backward(B, false, nullptr, g);
+  mf::LayerUpdArgs a;
+  a.mode = mf::LU_ROLLOUT;
+  a.theta = theta;
+  a.m = m;
+  a.g = g;
+  a.theta_out = theta_out;
+  a.m_out = m_out;
+  a.mu = lp->momentum;
+  a.lr = lr.lr;
+  a.status = h->d_status;
+  if (lp->optimizer == MF_OPTIM_ADAM) {
+    set_adam(a, lp, t);
+    a.v = v;
+    a.v_out = v_out;
+  }
+  ex.update(a);
+}
+
+// Inner rollout over steps [t0, t1) into the checkpoint store: theta_{t+1} (and m_{t+1} when
+// kept) go to their slots.  Without kept momentum slots a running m lives in the u buffer
+// (only on the first pass, before the sweep uses u).  Expects theta_{t0} cast already.
+template <typename X>
+void rollout_store(X& ex, const mf_loop_desc* lp, const Store& st, const float* eta,
+                   const void* inner_x, const void* inner_y, const LrSel& lr, int t0, int t1) {
+  float* m_run = (lp->momentum != 0.f && !st.m_kept) ? ex.u_buf() : nullptr;
+  for (int t = t0; t < t1; ++t) {
+    const float* m_in = m_run ? (t > t0 ? m_run : nullptr)
+                              : (st.m_kept && t > 0 ? ex.m_slot(st.m_idx(t)) : nullptr);
+    float* m_out = m_run ? m_run : (st.m_kept ? ex.m_slot(st.m_idx(t + 1)) : nullptr);
+    const float* v_in = st.adam && t > 0 ? ex.m_slot(st.v_idx(t)) : nullptr;
+    float* v_out = st.adam ? ex.m_slot(st.v_idx(t + 1)) : nullptr;
+    inner_step(ex, lp, eta, inner_x, inner_y, lr, t, ex.theta_slot(st.theta_idx(t)), m_in,
+               ex.theta_slot(st.theta_idx(t + 1)), m_out, v_in, v_out);
     if (ex.st != MF_OK) return;
   }
-  *theta_T = ex.theta_slot(store_all ? lp->T : (lp->T & 1));
+}
+
+// Inner rollout without a store (mf_inner_rollout): two theta slots ping-pong; m runs in the
+// u buffer, or in m slot 0 when the learning rate is a meta-parameter.
+template <typename X>
+void rollout_plain(X& ex, const mf_loop_desc* lp, const float* eta, const void* inner_x,
+                   const void* inner_y, const LrSel& lr, float** theta_T) {
+  const bool adam = lp->optimizer == MF_OPTIM_ADAM;
+  float* m_run = adam || lr.lr_meta ? ex.m_slot(0) : lp->momentum != 0.f ? ex.u_buf() : nullptr;
+  float* v_run = adam ? ex.m_slot(1) : nullptr;
+  ex.cast_params(ex.theta_slot(0), false);
+  for (int t = 0; t < lp->T; ++t) {
+    inner_step(ex, lp, eta, inner_x, inner_y, lr, t, ex.theta_slot(t & 1),
+               t > 0 ? m_run : nullptr, ex.theta_slot((t + 1) & 1), m_run,
+               t > 0 ? v_run : nullptr, v_run);
+    if (ex.st != MF_OK) return;
+  }
+  *theta_T = ex.theta_slot(lp->T & 1);
 }
 
 // Algorithm 2 once the workspace is in place: rollout, outer gradient (Eq. 4), then the
@@ -796,16 +874,21 @@ mf_status meta_grad_run(X& ex, const mf_loop_desc* lp, const float* theta0, cons
   cudaStream_t s = ex.s;
   const int T = lp->T, B = lp->B, Bo = lp->B_outer;
   const LrSel lr = lr_select(h, lp, eta);
+  const Store st = make_store(lp);
+  const int k = st.k;
+  auto theta_at = [&](int t) { return ex.theta_slot(st.theta_idx(t)); };
+  auto m_at = [&](int t) { return ex.m_slot(st.m_idx(t)); };   // m_t, t >= 1
   const bool scalar_lr = lp->meta_kind & MF_META_SCALAR_LOGLR;
-  MF_CUDA(h, cudaMemcpyAsync(ex.theta_slot(0), theta0, h->P * 4, cudaMemcpyDeviceToDevice, s));
+  MF_CUDA(h, cudaMemcpyAsync(theta_at(0), theta0, h->P * 4, cudaMemcpyDeviceToDevice, s));
   const int64_t ne = n_eta_of(h, lp);
   if (ne > 0) MF_CUDA(h, cudaMemsetAsync(d_eta, 0, ne * 4, s));
   ex.prepare();
 
-  // 1. rollout with the theta_t store
-  float* thT = nullptr;
-  rollout(ex, lp, eta, inner_x, inner_y, lr, true, &thT);
+  // 1. rollout into the checkpoint store; the last segment stays in the segment slots
+  ex.cast_params(theta_at(0), false);
+  rollout_store(ex, lp, st, eta, inner_x, inner_y, lr, 0, T);
   if (ex.st != MF_OK) return ex.st;
+  float* thT = theta_at(T);
 
   // 2. outer gradient theta_bar_T = grad V(theta_T)  (Eq. 4); theta_T is already cast
   float* tbar = ex.tbar_buf();
@@ -821,16 +904,31 @@ mf_status meta_grad_run(X& ex, const mf_loop_desc* lp, const float* theta0, cons
     ex.launched();
   }
   float* d_plr = lr.off_plr >= 0 ? d_eta + lr.off_plr : nullptr;
+  // Adam: reverse of inner step j from its stored outputs; u = g-bar_j, and the cotangents of
+  // m_j, v_j replace those of m_{j+1}, v_{j+1} in place
+  auto adam_pre = [&](mf::LayerUpdArgs& a, int j, bool bar_in) {
+    set_adam(a, lp, j);
+    a.adam_pre = true;
+    a.bar_in = bar_in;
+    a.m_adj = m_at(j + 1);
+    a.v_adj = ex.m_slot(st.v_idx(j + 1));
+    a.m_prev = j > 0 ? m_at(j) : nullptr;
+    a.mbar = ex.m_slot(st.mbar_idx());
+    a.vbar = ex.m_slot(st.mbar_idx() + 1);
+    a.u_out = u;
+  };
   // u_{T-1} = -lr theta_bar_T ;  d eta_lr += -lr m_T theta_bar_T ; cast theta_{T-1}, u_{T-1}
+  // (Adam: u_{T-1} = g-bar_{T-1} from theta_bar_T and zero moment cotangents)
   {
     mf::LayerUpdArgs a;
     a.mode = mf::LU_ADJOINT;
     a.theta_bar = tbar;
-    a.m_adj = lr.lr_meta ? ex.m_slot(T - 1) : nullptr;
+    a.m_adj = lr.lr_meta ? m_at(T) : nullptr;
     a.u_out = u;
+    if (st.adam) adam_pre(a, T - 1, false);
     a.d_plr = d_plr;
     a.partials = scalar_lr ? part + static_cast<int64_t>(T - 1) * nb : nullptr;
-    a.cast_src = ex.theta_slot(T - 1);
+    a.cast_src = theta_at(T - 1);
     a.mu = lp->momentum;
     a.lr = lr.lr;
     a.status = h->d_status;
@@ -841,8 +939,30 @@ mf_status meta_grad_run(X& ex, const mf_loop_desc* lp, const float* theta0, cons
   const size_t xs = ex.x_step_bytes(B);
   const size_t ys = ex.y_step_bytes(B);
   const bool exw = lp->meta_kind & MF_META_EXAMPLE_WEIGHTS;
+  bool adam_pending = false;   // Adam's reverse of step t waits for its segment's recompute
   for (int t = T - 1; t >= 0; --t) {
-    const float* th = ex.theta_slot(t);
+    // entering an earlier segment [t+1-k, t+1): rebuild theta and m of its steps from the
+    // segment's checkpoint (the rollout's own kernels, so bit-identical); this leaves
+    // theta_t cast for the forward below
+    if (t + 1 < T && (t + 1) % k == 0 && k > 1) {
+      const int a0 = t + 1 - k;
+      ex.cast_params(theta_at(a0), false);
+      rollout_store(ex, lp, st, eta, inner_x, inner_y, lr, a0, t);
+      if (ex.st != MF_OK) return ex.st;
+    }
+    if (adam_pending) {
+      mf::LayerUpdArgs a;
+      a.mode = mf::LU_ADJOINT;
+      a.theta_bar = tbar;
+      adam_pre(a, t, true);
+      a.d_plr = d_plr;
+      a.partials = scalar_lr ? part + static_cast<int64_t>(t) * nb : nullptr;
+      a.lr = lr.lr;
+      a.status = h->d_status;
+      ex.update(a);
+      adam_pending = false;
+    }
+    const float* th = theta_at(t);
     const void* x = static_cast<const char*>(inner_x) + xs * t;
     const void* y = static_cast<const char*>(inner_y) + ys * t;
     const float* ew = exw ? eta + static_cast<int64_t>(t) * B : nullptr;
@@ -860,13 +980,20 @@ mf_status meta_grad_run(X& ex, const mf_loop_desc* lp, const float* theta0, cons
     a.mode = mf::LU_ADJOINT;
     a.theta_bar = tbar;
     a.Hu = Hu;
-    if (t > 0) {
-      a.m_adj = lr.lr_meta ? ex.m_slot(t - 1) : nullptr;
+    const bool in_store = t % k != 0 || k == 1;   // theta_{t-1}, m_{t-1} in the store now
+    if (t > 0 && st.adam && !in_store) {
+      a.adam = 1;            // theta_bar only; the reverse of step t-1 follows the recompute
+      adam_pending = true;
+    } else if (t > 0) {
+      a.m_adj = lr.lr_meta ? m_at(t) : nullptr;
       a.u_in = u;
       a.u_out = u;
+      if (st.adam) adam_pre(a, t - 1, true);
       a.d_plr = d_plr;
       a.partials = scalar_lr ? part + static_cast<int64_t>(t - 1) * nb : nullptr;
-      a.cast_src = ex.theta_slot(t - 1);
+      // theta_{t-1} is in the store only within this segment or at a checkpoint; otherwise
+      // the recompute of its segment casts it
+      if (in_store) a.cast_src = theta_at(t - 1);
     }
     a.mu = lp->momentum;
     a.lr = lr.lr;
@@ -891,7 +1018,7 @@ mf_status rollout_run(X& ex, const mf_loop_desc* lp, const float* theta0, const 
   MF_CUDA(h, cudaMemcpyAsync(ex.theta_slot(0), theta0, h->P * 4, cudaMemcpyDeviceToDevice, ex.s));
   ex.prepare();
   float* thT = nullptr;
-  rollout(ex, lp, eta, inner_x, inner_y, lr, false, &thT);
+  rollout_plain(ex, lp, eta, inner_x, inner_y, lr, &thT);
   if (ex.st != MF_OK) return ex.st;
   MF_CUDA(h, cudaMemcpyAsync(thetaT, thT, h->P * 4, cudaMemcpyDeviceToDevice, ex.s));
   return MF_OK;
@@ -939,9 +1066,10 @@ mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
                          const float* eta, const void* inner_x, const void* inner_y,
                          const void* outer_x, const void* outer_y, float* d_eta,
                          float* d_theta0, float* outer_loss, cudaStream_t s) {
-  const bool lr_meta = lp->meta_kind & (MF_META_PARAM_LOGLR | MF_META_SCALAR_LOGLR);
-  return with_exec<E>(h, std::max(lp->B, lp->B_outer), lp->T, lp->T + 1, lr_meta ? lp->T : 0,
-                      lp->meta_kind & MF_META_SCALAR_LOGLR, lp->hvp_mode == MF_HVP_REV_REV, s,
+  const Store store = make_store(lp);
+  return with_exec<E>(h, std::max(lp->B, lp->B_outer), lp->T, store.theta_slots(),
+                      store.m_slots(), lp->meta_kind & MF_META_SCALAR_LOGLR,
+                      lp->hvp_mode == MF_HVP_REV_REV, s,
                       [&](auto& ex) {
                         return meta_grad_run(ex, lp, theta0, eta, inner_x, inner_y, outer_x,
                                              outer_y, d_eta, d_theta0, outer_loss);
@@ -952,7 +1080,8 @@ template <typename E>
 mf_status rollout_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0, const float* eta,
                        const void* inner_x, const void* inner_y, float* thetaT, cudaStream_t s) {
   const bool lr_meta = lp->meta_kind & (MF_META_PARAM_LOGLR | MF_META_SCALAR_LOGLR);
-  return with_exec<E>(h, lp->B, lp->T, 2, lr_meta ? 1 : 0, false, false, s, [&](auto& ex) {
+  const int m_slots = lp->optimizer == MF_OPTIM_ADAM ? 2 : lr_meta ? 1 : 0;
+  return with_exec<E>(h, lp->B, lp->T, 2, m_slots, false, false, s, [&](auto& ex) {
     return rollout_run(ex, lp, theta0, eta, inner_x, inner_y, thetaT);
   });
 }
@@ -1097,15 +1226,16 @@ mf_status mf_workspace_bytes(mf_handle h, const mf_loop_desc* lp, size_t* bytes)
   if (!h || !bytes) return MF_ERR_INVALID_ARG;
   mf_status st = validate_loop(h, lp);
   if (st != MF_OK) return st;
-  const bool lr_meta = lp->meta_kind & (MF_META_PARAM_LOGLR | MF_META_SCALAR_LOGLR);
+  const Store store = make_store(lp);
   if (h->decoder) {
-    *bytes = make_dec_plan(h, h->Ly, std::max(lp->B, lp->B_outer), lp->T, lp->T + 1,
-                           lr_meta ? lp->T : 0, lp->meta_kind & MF_META_SCALAR_LOGLR,
+    *bytes = make_dec_plan(h, h->Ly, std::max(lp->B, lp->B_outer), lp->T, store.theta_slots(),
+                           store.m_slots(), lp->meta_kind & MF_META_SCALAR_LOGLR,
                            lp->hvp_mode == MF_HVP_REV_REV).bytes;
     return MF_OK;
   }
-  *bytes = make_plan(h, std::max(lp->B, lp->B_outer), lp->T, lp->T + 1, lr_meta ? lp->T : 0,
-                     lp->meta_kind & MF_META_SCALAR_LOGLR, lp->hvp_mode == MF_HVP_REV_REV).bytes;
+  *bytes = make_plan(h, std::max(lp->B, lp->B_outer), lp->T, store.theta_slots(),
+                     store.m_slots(), lp->meta_kind & MF_META_SCALAR_LOGLR,
+                     lp->hvp_mode == MF_HVP_REV_REV).bytes;
   return MF_OK;
 }
 
@@ -1131,6 +1261,10 @@ mf_status mf_inner_rollout(mf_handle h, const mf_loop_desc* lp, const float* the
                      static_cast<uint64_t>(lp->meta_kind),
                      static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->alpha)),
                      static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->momentum)),
+                     static_cast<uint64_t>(lp->optimizer),
+                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->beta1)),
+                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->beta2)),
+                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->adam_eps)),
                      reinterpret_cast<uint64_t>(theta0), reinterpret_cast<uint64_t>(eta),
                      reinterpret_cast<uint64_t>(inner_x), reinterpret_cast<uint64_t>(inner_y),
                      reinterpret_cast<uint64_t>(thetaT)})
@@ -1190,6 +1324,11 @@ mf_status mf_meta_grad(mf_handle h, const mf_loop_desc* lp, const float* theta0,
   for (uint64_t v : {static_cast<uint64_t>(lp->T), static_cast<uint64_t>(lp->B),
                      static_cast<uint64_t>(lp->B_outer), static_cast<uint64_t>(lp->meta_kind),
                      static_cast<uint64_t>(lp->hvp_mode),
+                     static_cast<uint64_t>(make_store(lp).k),
+                     static_cast<uint64_t>(lp->optimizer),
+                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->beta1)),
+                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->beta2)),
+                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->adam_eps)),
                      static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->alpha)),
                      static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->momentum)),
                      reinterpret_cast<uint64_t>(theta0), reinterpret_cast<uint64_t>(eta),

@@ -155,6 +155,20 @@ struct LayerUpdArgs {
   float mu = 0.f;
   LrArgs lr;
   int* status = nullptr;
+  // Adam (adam = 1), for the step whose bias corrections are c1 = 1 - b1^(j+1), c2 = 1 - b2^(j+1):
+  //  LU_ROLLOUT: m' = b1 m + (1-b1) g, v' = b2 v + (1-b2) g^2, theta' = theta - lr (m'/c1) /
+  //              (sqrt(v'/c2) + eps); v (nullable = 0) in, v_out out.
+  //  LU_ADJOINT with adam_pre: the reverse of step j from its outputs (m_adj = m_{j+1},
+  //              v_adj = v_{j+1}) and input momentum m_prev = m_j (nullable = 0), with the
+  //              cotangents theta_bar (after += Hu), mbar, vbar of theta_{j+1}, m_{j+1}, v_{j+1}
+  //              (read only when bar_in): writes u_out = g-bar_j and mbar, vbar <- those of
+  //              m_j, v_j; d eta_lr gets -lr theta_bar (m_{j+1}/c1) / (sqrt(v_{j+1}/c2) + eps).
+  int adam = 0;
+  bool adam_pre = false, bar_in = false;
+  float b1 = 0.f, b2 = 0.f, eps = 0.f, c1 = 1.f, c2 = 1.f;
+  const float* v = nullptr; float* v_out = nullptr;
+  const float* v_adj = nullptr; const float* m_prev = nullptr;
+  float* mbar = nullptr; float* vbar = nullptr;
 };
 template <typename T>
 void layer_update(const LayerTable& tab, const LayerUpdArgs& a, cudaStream_t s);

@@ -354,13 +354,49 @@ __global__ void __launch_bounds__(TILE * TROWS) layer_update_kernel(const LayerT
     float vw = 0.f, vu = 0.f;
     if (r < rows && c < dout) {
       const int64_t k = tab.off[l] + static_cast<int64_t>(r) * dout + c;
-      if (a.mode == LU_ROLLOUT) {
+      if (a.mode == LU_ROLLOUT && a.adam) {
+        const float g = a.g[k];
+        const float mn = (a.m ? a.b1 * a.m[k] : 0.f) + (1.f - a.b1) * g;
+        const float vn = (a.v ? a.b2 * a.v[k] : 0.f) + (1.f - a.b2) * g * g;
+        const float tn = a.theta[k] - lr_at(a.lr, k) * (mn / a.c1) / (sqrtf(vn / a.c2) + a.eps);
+        a.theta_out[k] = tn;
+        if (a.m_out) a.m_out[k] = mn;
+        if (a.v_out) a.v_out[k] = vn;
+        bad |= !isfinite(tn);
+        vw = tn;
+      } else if (a.mode == LU_ROLLOUT) {
         const float mn = (a.m ? a.mu * a.m[k] : 0.f) + a.g[k];
         const float tn = a.theta[k] - lr_at(a.lr, k) * mn;
         a.theta_out[k] = tn;
         if (a.m_out) a.m_out[k] = mn;
         bad |= !isfinite(tn);
         vw = tn;
+      } else if (a.mode == LU_ADJOINT && a.adam) {
+        const float tb = a.theta_bar[k] + (a.Hu ? a.Hu[k] : 0.f);
+        a.theta_bar[k] = tb;
+        bad |= !isfinite(tb);
+        if (a.adam_pre) {
+          // theta_{j+1} = theta_j - lr (m/c1) / (s + eps), s = sqrt(v/c2), m = m_{j+1}, v = v_{j+1}
+          const float lr = lr_at(a.lr, k);
+          const float m1 = a.m_adj[k], v1 = a.v_adj[k];
+          const float s = sqrtf(v1 / a.c2);
+          const float den = s + a.eps;
+          const float q = -lr * tb;
+          // cotangents of m_{j+1} and v_{j+1} (at v = 0, where m = g = 0, the sqrt term is 0)
+          const float Mb = (a.bar_in ? a.mbar[k] : 0.f) + q / (a.c1 * den);
+          const float Vb = (a.bar_in ? a.vbar[k] : 0.f) -
+                           (s > 0.f ? q * m1 / (a.c1 * den * den * 2.f * s * a.c2) : 0.f);
+          const float g = (m1 - (a.m_prev ? a.b1 * a.m_prev[k] : 0.f)) / (1.f - a.b1);
+          vu = (1.f - a.b1) * Mb + 2.f * (1.f - a.b2) * g * Vb;
+          a.u_out[k] = vu;
+          a.mbar[k] = a.b1 * Mb;
+          a.vbar[k] = a.b2 * Vb;
+          const float contrib = -lr * (m1 / a.c1) / den * tb;
+          if (a.d_plr) a.d_plr[k] += contrib;
+          else acc += contrib;
+          bad |= !isfinite(vu);
+        }
+        if (a.cast_src) vw = a.cast_src[k];
       } else if (a.mode == LU_ADJOINT) {
         const float tb = a.theta_bar[k] + (a.Hu ? a.Hu[k] : 0.f);
         a.theta_bar[k] = tb;

@@ -20,6 +20,7 @@ MF_ARCH_MLP, MF_ARCH_DECODER = 0, 1
 ACTS = {"ident": 0, "tanh": 1, "gelu": 2, "silu": 3}
 LOSSES = {"squared": 0, "ce": 1, "next_token_ce": 2, "chain_mse": 3}
 PRECISIONS = {"fp32": 0, "bf16": 1}
+OPTIMIZERS = {"sgd": 0, "adam": 1}
 MF_META_EXAMPLE_WEIGHTS, MF_META_PARAM_LOGLR, MF_META_SCALAR_LOGLR = 1, 2, 4
 MF_HVP_MIXED_FOR, MF_HVP_REV_REV = 0, 1
 MF_OPT_CUDA_GRAPHS, MF_OPT_PDL, MF_OPT_CONCURRENT, MF_OPT_GEMM_2SM = 1, 2, 3, 4
@@ -45,7 +46,8 @@ class mf_model_desc(C.Structure):
 class mf_loop_desc(C.Structure):
     _fields_ = [("T", C.c_int), ("B", C.c_int), ("B_outer", C.c_int), ("alpha", C.c_float),
                 ("momentum", C.c_float), ("meta_kind", C.c_int), ("hvp_mode", C.c_int),
-                ("ckpt_every", C.c_int)]
+                ("ckpt_every", C.c_int), ("optimizer", C.c_int), ("beta1", C.c_float),
+                ("beta2", C.c_float), ("adam_eps", C.c_float)]
 
 
 class MixflowError(RuntimeError):
@@ -137,13 +139,15 @@ def model_desc_for(w) -> mf_model_desc:
     return d
 
 
-def loop_desc_for(w, hvp_mode: int = MF_HVP_MIXED_FOR) -> mf_loop_desc:
+def loop_desc_for(w, hvp_mode: int = MF_HVP_MIXED_FOR, ckpt_every: int = 1) -> mf_loop_desc:
     l = mf_loop_desc()
     l.T, l.B, l.B_outer = w.T, w.B, w.B_outer
     l.alpha, l.momentum = w.alpha, w.momentum
     l.meta_kind = w.meta_kind
     l.hvp_mode = hvp_mode
-    l.ckpt_every = 1
+    l.ckpt_every = ckpt_every
+    l.optimizer = OPTIMIZERS[getattr(w, "optimizer", "sgd")]
+    l.beta1, l.beta2, l.adam_eps = w.beta1, w.beta2, w.adam_eps
     return l
 
 
