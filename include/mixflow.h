@@ -248,8 +248,14 @@ mf_status mf_kernel_time(mf_handle h, double* ms, uint64_t* launches, double* fl
  * MF_OPT_GEMM_2SM (process-wide): 1 (default) computes a bf16 GEMM with 256-row tiles on
  * CTA pairs (tcgen05 cta_group::2) when its grid of pairs fills the GPU, 0 never, 2 for
  * every GEMM with more than 128 rows (for tests).  Results are identical up to the
- * summation order within a tile, which both forms share. */
-enum { MF_OPT_CUDA_GRAPHS = 1, MF_OPT_PDL = 2, MF_OPT_CONCURRENT = 3, MF_OPT_GEMM_2SM = 4 };
+ * summation order within a tile, which both forms share.
+ * MF_OPT_FLASH_ATTN (default 1): the decoder's dual attention runs fused, without the
+ * S x S probabilities and their tangent in memory (bf16 decoders with d_model/n_heads = 64
+ * and seq_len a multiple of 64; others always use the materialised form).  0 materialises
+ * them (per block, for the backward).  Setting it drops the handle's captured graphs and
+ * changes the workspace size. */
+enum { MF_OPT_CUDA_GRAPHS = 1, MF_OPT_PDL = 2, MF_OPT_CONCURRENT = 3, MF_OPT_GEMM_2SM = 4,
+       MF_OPT_FLASH_ATTN = 5 };
 mf_status mf_set_option(mf_handle h, int option, int value);
 
 /* Host-side fault injection for tests: kind 1 = the next workspace allocation fails;

@@ -78,6 +78,7 @@ struct mf_ctx {
   cudaStream_t sstream = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   bool concurrent = true;
+  bool flash = true;          // fused dual attention where supported (MF_OPT_FLASH_ATTN)
 };
 
 namespace {
@@ -117,7 +118,7 @@ int n_update_tiles(const mf_ctx* h) {
   int tiles = 0;
   for (int l = 0; l < h->L; ++l) {
     const int rows = h->dims[l] + (h->md.has_bias ? 1 : 0);
-    tiles += ((rows + 31) / 32) * ((h->dims[l + 1] + 31) / 32);
+    tiles += mf::update_blocks(rows, h->dims[l + 1]);
   }
   return tiles;
 }
@@ -342,7 +343,7 @@ struct Exec {
       tab.dout[l] = dout;
       tab.off[l] = h->woff[l];
       tab.tile0[l] = tiles;
-      tiles += ((tab.rows[l] + 31) / 32) * ((dout + 31) / 32);
+      tiles += mf::update_blocks(tab.rows[l], dout);
       tab.ldw[l] = ld8(dout);
       tab.ldwt[l] = 0;
       tab.W[l] = at<T>(p.o_Wb[l]);
@@ -1432,6 +1433,11 @@ mf_status mf_set_option(mf_handle h, int option, int value) {
   }
   if (option == MF_OPT_CONCURRENT) {
     h->concurrent = value != 0;
+    drop_graphs(h);
+    return MF_OK;
+  }
+  if (option == MF_OPT_FLASH_ATTN) {
+    h->flash = value != 0;
     drop_graphs(h);
     return MF_OK;
   }

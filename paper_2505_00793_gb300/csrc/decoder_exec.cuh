@@ -58,6 +58,11 @@ struct DecPlan {
   // every block (the stored reverse graph, at block granularity)
   bool ror = false;
   std::vector<size_t> dxs;
+  // fused dual attention: per block the row statistics (lse, then rbar) instead of P and P';
+  // D and D' of the block being differentiated
+  bool flash = false;
+  std::vector<size_t> fst;
+  size_t fD = 0;
 };
 
 DecPlan make_dec_plan(const mf_ctx* h, const DecLayout& Ly, int rows, int T, int n_theta_slots,
@@ -80,7 +85,7 @@ DecPlan make_dec_plan(const mf_ctx* h, const DecLayout& Ly, int rows, int T, int
   p.o_u = take(P4);
   const auto tens = dec_tensors(Ly);
   int tiles = 0;
-  for (const auto& t : tens) tiles += ((t.rows + 31) / 32) * ((t.cols + 31) / 32);
+  for (const auto& t : tens) tiles += mf::update_blocks(t.rows, t.cols);
   p.nb = tiles;
   p.o_part = take(with_partials ? static_cast<size_t>(p.nb) * (T > 0 ? T : 1) * 4 : 4);
   p.o_l = take(static_cast<size_t>(rows) * 4);
@@ -100,7 +105,9 @@ DecPlan make_dec_plan(const mf_ctx* h, const DecLayout& Ly, int rows, int T, int
   }
   const size_t Nd4 = N * d * 4, NdT = N * d * es;
   const size_t head = static_cast<size_t>(BH) * S * Ly.dh * es;
-  const size_t SS = static_cast<size_t>(BH) * S * S;
+  p.flash = h->flash && h->bf16 && mf::flash_supported(static_cast<int>(S), Ly.dh);
+  const size_t SS = p.flash ? 0 : static_cast<size_t>(BH) * S * S;
+  const size_t stat = static_cast<size_t>(BH) * S * 4;
   for (int l = 0; l < Ly.L; ++l) {
     p.x1.push_back(take(Nd4)); p.x1d.push_back(take(Nd4));
     p.r1.push_back(take(N * 4)); p.r1d.push_back(take(N * 4));
@@ -112,6 +119,7 @@ DecPlan make_dec_plan(const mf_ctx* h, const DecLayout& Ly, int rows, int T, int
     p.K.push_back(take(head)); p.Kd.push_back(take(head));
     p.Vv.push_back(take(head)); p.Vd.push_back(take(head));
     p.P.push_back(take(SS * es)); p.Pd.push_back(take(SS * es));
+    if (p.flash) p.fst.push_back(take(2 * stat));
     p.Om.push_back(take(NdT)); p.Omd.push_back(take(NdT));
     p.z1.push_back(take(N * F * 4)); p.z1d.push_back(take(N * F * 4));
     p.a1.push_back(take(N * F * es)); p.a1d.push_back(take(N * F * es));
@@ -131,6 +139,7 @@ DecPlan make_dec_plan(const mf_ctx* h, const DecLayout& Ly, int rows, int T, int
   p.dOh = take(head); p.dOhd = take(head);
   p.dP = take(SS * 4); p.dPd = take(SS * 4);
   p.dS = take(SS * es); p.dSd = take(SS * es);
+  if (p.flash) p.fD = take(2 * stat);
   const size_t head4 = static_cast<size_t>(BH) * S * Ly.dh * 4;
   p.dQ = take(head4); p.dQd = take(head4); p.dK = take(head4); p.dKd = take(head4);
   p.dV = take(head4); p.dVd = take(head4);
@@ -173,7 +182,7 @@ struct DecExec {
       tab.dout[i] = t.cols;
       tab.off[i] = t.off;
       tab.tile0[i] = tiles;
-      tiles += ((t.rows + 31) / 32) * ((t.cols + 31) / 32);
+      tiles += mf::update_blocks(t.rows, t.cols);
       tab.ldw[i] = ld8(t.cols);
       tab.ldwt[i] = 0;
       tab.W[i] = t.cast ? at<T>(p.o_W[i]) : nullptr;   // read K- or MN-major, never transposed
@@ -248,6 +257,19 @@ struct DecExec {
   }
 
   // C = X Y^T style linear product; dual adds X' Y^T + X Y'^T (or the weight-tangent sum).
+  // Operands of the fused attention of block l: its heads and row statistics.
+  mf::FlashArgs flash_args(int l, int BH) const {
+    auto hb = [&](size_t o) { return reinterpret_cast<const __nv_bfloat16*>(at<T>(o)); };
+    mf::FlashArgs fa;
+    fa.BH = BH;
+    fa.S = Ly.S;
+    fa.Q = hb(p.Q[l]); fa.K = hb(p.K[l]); fa.V = hb(p.Vv[l]);
+    fa.Qd = hb(p.Qd[l]); fa.Kd = hb(p.Kd[l]); fa.Vd = hb(p.Vd[l]);
+    fa.lse = at<float>(p.fst[l]);
+    fa.rbar = fa.lse + static_cast<int64_t>(BH) * Ly.S;
+    return fa;
+  }
+
   GemmArgs lin(int M, int N, int K, const void* A0, const void* A1, int lda, const void* B0,
                const void* B1, int ldb, bool dual) const {
     GemmArgs g;
@@ -324,6 +346,14 @@ struct DecExec {
         launched();
       }
 
+      if (p.flash) {
+        // fused causal attention and its tangent: O, O' and the row statistics
+        mf::FlashArgs fa = flash_args(l, BH);
+        fa.O = at<float>(p.O);
+        fa.Od = dual ? at<float>(p.Od) : nullptr;
+        mf::flash_fwd(fa, dual, s);
+        launched();
+      } else {
       // scores S = Q K^T (dual: Q' K^T + Q K'^T), batch over B*H
       {
         GemmArgs g = lin(S, S, dh, at<T>(p.Q[l]), at<T>(p.Qd[l]), dh, at<T>(p.K[l]), at<T>(p.Kd[l]),
@@ -345,6 +375,7 @@ struct DecExec {
         g.C0 = at<float>(p.O); g.ldc0 = dh;
         g.C1 = at<float>(p.Od); g.ldc1 = dh;
         gemm(g);
+      }
       }
       mf::dec_head_merge<T>(N, S, H, dh, at<float>(p.O), at<T>(p.Om[l]), d, s);
       launched();
@@ -548,6 +579,23 @@ struct DecExec {
         mf::dec_head_split<T>(N, S, H, dh, at<float>(p.dhd), at<T>(p.dOhd), s);
         launched();
       }
+      if (p.flash) {
+        // fused backward of the attention and its tangent, from D = rowsum(dO O) (and D')
+        float* D = at<float>(p.fD);
+        float* Dd = D + static_cast<int64_t>(BH) * S;
+        mf::flash_prep(N, S, H, at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr,
+                       at<T>(p.Om[l]), dual ? at<T>(p.Omd[l]) : nullptr, d, D,
+                       dual ? Dd : nullptr, s);
+        mf::FlashArgs fa = flash_args(l, BH);
+        fa.dO = reinterpret_cast<const __nv_bfloat16*>(at<T>(p.dOh));
+        fa.dOd = dual ? reinterpret_cast<const __nv_bfloat16*>(at<T>(p.dOhd)) : nullptr;
+        fa.D = D;
+        fa.Dd = dual ? Dd : nullptr;
+        fa.dQ = at<float>(p.dQ); fa.dK = at<float>(p.dK); fa.dV = at<float>(p.dV);
+        if (dual) { fa.dQd = at<float>(p.dQd); fa.dKd = at<float>(p.dKd); fa.dVd = at<float>(p.dVd); }
+        mf::flash_bwd(fa, dual, s);
+        launched(3);
+      } else {
       // dP = dO V^T (dual: dO' V^T + dO V'^T)
       {
         GemmArgs g = lin(S, S, dh, at<T>(p.dOh), at<T>(p.dOhd), dh, at<T>(p.Vv[l]), at<T>(p.Vd[l]), dh, dual);
@@ -585,6 +633,7 @@ struct DecExec {
         g.C0 = at<float>(p.dK); g.ldc0 = dh;
         g.C1 = at<float>(p.dKd); g.ldc1 = dh;
         gemm(g);
+      }
       }
       const float qscale = 1.f / sqrtf(static_cast<float>(dh));
       mf::dec_rope_merge<T>(N, S, H, dh, Ly.base, qscale, at<float>(p.dQ), at<float>(p.dK),

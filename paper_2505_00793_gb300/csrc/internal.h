@@ -130,6 +130,14 @@ struct LrArgs {
 // its first din[l] rows are cast to the GEMM operand copies W (row-major [din][ldw]) and
 // WT (transposed [dout][ldwt]), or U / UT for the tangent.
 constexpr int kMaxLayers = 96;
+// Fused update kernel geometry: UPD_THREADS threads of four parameters each per block;
+// update_blocks is the block count of one layer (and the number of scalar-lr partials).
+constexpr int UPD_THREADS = 256;
+constexpr int UPD_ELEMS = UPD_THREADS * 4;
+inline int update_blocks(int rows, int cols) {
+  return static_cast<int>((static_cast<int64_t>(rows) * cols + UPD_ELEMS - 1) / UPD_ELEMS);
+}
+
 struct LayerTable {
   int n = 0;
   int rows[kMaxLayers], din[kMaxLayers], dout[kMaxLayers];
@@ -169,6 +177,7 @@ struct LayerUpdArgs {
   const float* v = nullptr; float* v_out = nullptr;
   const float* v_adj = nullptr; const float* m_prev = nullptr;
   float* mbar = nullptr; float* vbar = nullptr;
+  bool vec_ok = false;   // set by layer_update: every vector above is 16-byte aligned
 };
 template <typename T>
 void layer_update(const LayerTable& tab, const LayerUpdArgs& a, cudaStream_t s);
@@ -183,6 +192,28 @@ void ror_fwd_elem(int act, const float* dzbar, const float* Z, const float* dA, 
 template <typename T>
 void ror_bwd_elem(int act, const float* zpart, const float* abar, const float* Z, int rows,
                   int cols, T* zb, int ld, T* zbT, int ldT, cudaStream_t s);
+
+// ---- fused dual attention (flash_attn.cu) -------------------------------------------------
+// Heads [BH][S][64] bf16 (q pre-scaled by 1/sqrt(64)), causal.  Forward: O (and O') float32
+// [BH][S][64], per-row lse and rbar [BH][S].  Backward: from dO (and dO') bf16 heads and
+// D, D' [BH][S] (flash_prep), writes dQ, dK, dV (and tangents) float32 [BH][S][64].
+struct FlashArgs {
+  int BH = 0, S = 0;
+  const __nv_bfloat16 *Q = nullptr, *K = nullptr, *V = nullptr;
+  const __nv_bfloat16 *Qd = nullptr, *Kd = nullptr, *Vd = nullptr;
+  const __nv_bfloat16 *dO = nullptr, *dOd = nullptr;
+  float *O = nullptr, *Od = nullptr, *lse = nullptr, *rbar = nullptr;
+  const float *D = nullptr, *Dd = nullptr;
+  float *dQ = nullptr, *dQd = nullptr, *dK = nullptr, *dKd = nullptr, *dV = nullptr,
+        *dVd = nullptr;
+};
+bool flash_supported(int S, int dh);
+void flash_fwd(const FlashArgs& a, bool dual, cudaStream_t s);
+void flash_bwd(const FlashArgs& a, bool dual, cudaStream_t s);
+// D = rowsum(dO (*) O), D' = rowsum(dO' (*) O + dO (*) O') per (token, head) from float32
+// merged gradients [N][ld] and bf16 merged outputs; Dd / dOd / Od may be null (primal).
+void flash_prep(int N, int S, int H, const float* dO, const float* dOd, const void* O,
+                const void* Od, int ld, float* D, float* Dd, cudaStream_t s);
 
 // ---- decoder-only transformer kernels (decoder_kernels.cu) ------------------------------
 void dec_embed_fwd(int N, int S, int d, int V, const int* ids, const float* E, const float* UE,

@@ -329,123 +329,200 @@ __device__ __forceinline__ float lr_at(const LrArgs& lr, int64_t i) {
   return lr.alpha;
 }
 
-// One 32 x 32 tile of one layer's [rows][dout] slice of the flat parameter vector per block.
+// Four consecutive parameters per thread, UPD_ELEMS per block, blocks assigned to layers by
+// tab.tile0.  A layer whose offset and width are multiples of 4 moves them as float4 (and
+// its operand copies as four-element stores in one row); others go element by element.
+__device__ __forceinline__ void ld4(float (&x)[4], const float* p, int64_t k, bool vec, int cnt) {
+  if (vec) {
+    const float4 t = *reinterpret_cast<const float4*>(p + k);
+    x[0] = t.x; x[1] = t.y; x[2] = t.z; x[3] = t.w;
+  } else {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) x[j] = j < cnt ? p[k + j] : 0.f;
+  }
+}
+
+__device__ __forceinline__ void st4(float* p, int64_t k, const float (&x)[4], bool vec, int cnt) {
+  if (vec) {
+    *reinterpret_cast<float4*>(p + k) = make_float4(x[0], x[1], x[2], x[3]);
+  } else {
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (j < cnt) p[k + j] = x[j];
+  }
+}
+
 template <typename T>
-__global__ void __launch_bounds__(TILE * TROWS) layer_update_kernel(const LayerTable tab,
-                                                                    const LayerUpdArgs a) {
+__device__ __forceinline__ void st_copy(T* W, int64_t e0, int dout, int din, int ldw,
+                                        const float (&x)[4], bool vec, int cnt) {
+  if (vec) {   // four elements of one row
+    const int r = static_cast<int>(e0 / dout), c = static_cast<int>(e0 % dout);
+    if (r >= din) return;
+    T* q = W + static_cast<int64_t>(r) * ldw + c;
+    if constexpr (sizeof(T) == 2) {
+      __nv_bfloat162 lo = __floats2bfloat162_rn(x[0], x[1]);
+      __nv_bfloat162 hi = __floats2bfloat162_rn(x[2], x[3]);
+      uint2 v;
+      v.x = *reinterpret_cast<uint32_t*>(&lo);
+      v.y = *reinterpret_cast<uint32_t*>(&hi);
+      *reinterpret_cast<uint2*>(q) = v;
+    } else {
+      *reinterpret_cast<float4*>(q) = make_float4(x[0], x[1], x[2], x[3]);
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if (j >= cnt) break;
+      const int64_t e = e0 + j;
+      const int r = static_cast<int>(e / dout), c = static_cast<int>(e % dout);
+      if (r < din) W[static_cast<int64_t>(r) * ldw + c] = to_t<T>(x[j]);
+    }
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(UPD_THREADS) layer_update_kernel(const LayerTable tab,
+                                                                   const LayerUpdArgs a) {
   pdl_entry();
-  __shared__ float tw[TILE][TILE + 1];   // values cast into W / WT
-  __shared__ float tu[TILE][TILE + 1];   // values cast into U / UT
-  __shared__ float red[TILE * TROWS / 32];
+  __shared__ float red[UPD_THREADS / 32];
   int l = 0;
   while (l + 1 < tab.n && static_cast<int>(blockIdx.x) >= tab.tile0[l + 1]) ++l;
-  const int t = blockIdx.x - tab.tile0[l];
-  const int dout = tab.dout[l], rows = tab.rows[l], din = tab.din[l];
-  const int tiles_c = (dout + TILE - 1) / TILE;
-  const int r0 = (t / tiles_c) * TILE, c0 = (t % tiles_c) * TILE;
-  const int tx = threadIdx.x, ty = threadIdx.y;
+  const int dout = tab.dout[l], din = tab.din[l];
+  const int64_t n = static_cast<int64_t>(tab.rows[l]) * dout;
+  const int64_t e0 = (static_cast<int64_t>(blockIdx.x - tab.tile0[l]) * UPD_THREADS + threadIdx.x) * 4;
   const bool cast_w = (a.mode == LU_ROLLOUT) || (a.mode == LU_CAST && !a.cast_src_to_u) ||
                       (a.mode == LU_ADJOINT && a.cast_src);
   const bool cast_u = (a.mode == LU_CAST && a.cast_src_to_u) || (a.mode == LU_ADJOINT && a.u_out);
   bool bad = false;
   float acc = 0.f;
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int r = r0 + i, c = c0 + tx;
-    float vw = 0.f, vu = 0.f;
-    if (r < rows && c < dout) {
-      const int64_t k = tab.off[l] + static_cast<int64_t>(r) * dout + c;
-      if (a.mode == LU_ROLLOUT && a.adam) {
-        const float g = a.g[k];
-        const float mn = (a.m ? a.b1 * a.m[k] : 0.f) + (1.f - a.b1) * g;
-        const float vn = (a.v ? a.b2 * a.v[k] : 0.f) + (1.f - a.b2) * g * g;
-        const float tn = a.theta[k] - lr_at(a.lr, k) * (mn / a.c1) / (sqrtf(vn / a.c2) + a.eps);
-        a.theta_out[k] = tn;
-        if (a.m_out) a.m_out[k] = mn;
-        if (a.v_out) a.v_out[k] = vn;
-        bad |= !isfinite(tn);
-        vw = tn;
-      } else if (a.mode == LU_ROLLOUT) {
-        const float mn = (a.m ? a.mu * a.m[k] : 0.f) + a.g[k];
-        const float tn = a.theta[k] - lr_at(a.lr, k) * mn;
-        a.theta_out[k] = tn;
-        if (a.m_out) a.m_out[k] = mn;
-        bad |= !isfinite(tn);
-        vw = tn;
-      } else if (a.mode == LU_ADJOINT && a.adam) {
-        const float tb = a.theta_bar[k] + (a.Hu ? a.Hu[k] : 0.f);
-        a.theta_bar[k] = tb;
-        bad |= !isfinite(tb);
-        if (a.adam_pre) {
-          // theta_{j+1} = theta_j - lr (m/c1) / (s + eps), s = sqrt(v/c2), m = m_{j+1}, v = v_{j+1}
-          const float lr = lr_at(a.lr, k);
-          const float m1 = a.m_adj[k], v1 = a.v_adj[k];
-          const float s = sqrtf(v1 / a.c2);
-          const float den = s + a.eps;
-          const float q = -lr * tb;
-          // cotangents of m_{j+1} and v_{j+1} (at v = 0, where m = g = 0, the sqrt term is 0)
-          const float Mb = (a.bar_in ? a.mbar[k] : 0.f) + q / (a.c1 * den);
-          const float Vb = (a.bar_in ? a.vbar[k] : 0.f) -
-                           (s > 0.f ? q * m1 / (a.c1 * den * den * 2.f * s * a.c2) : 0.f);
-          const float g = (m1 - (a.m_prev ? a.b1 * a.m_prev[k] : 0.f)) / (1.f - a.b1);
-          vu = (1.f - a.b1) * Mb + 2.f * (1.f - a.b2) * g * Vb;
-          a.u_out[k] = vu;
-          a.mbar[k] = a.b1 * Mb;
-          a.vbar[k] = a.b2 * Vb;
-          const float contrib = -lr * (m1 / a.c1) / den * tb;
-          if (a.d_plr) a.d_plr[k] += contrib;
-          else acc += contrib;
-          bad |= !isfinite(vu);
+  if (e0 < n) {
+    const int cnt = static_cast<int>(n - e0 < 4 ? n - e0 : 4);
+    const bool vec = a.vec_ok && cnt == 4 && (tab.off[l] & 3) == 0 && (dout & 3) == 0;
+    const int64_t k = tab.off[l] + e0;
+    float vw[4] = {0.f, 0.f, 0.f, 0.f}, vu[4] = {0.f, 0.f, 0.f, 0.f};
+    float lr[4];
+    const bool need_lr = a.mode == LU_ROLLOUT ||
+                         (a.mode == LU_ADJOINT && (a.adam_pre || a.m_adj || a.u_out));
+    if (a.lr.plr && need_lr) {
+      ld4(lr, a.lr.plr, k, vec, cnt);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) lr[j] = expf(lr[j]);
+    } else {
+      const float l0 = a.lr.slr ? expf(a.lr.slr[0]) : a.lr.alpha;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) lr[j] = l0;
+    }
+    if (a.mode == LU_ROLLOUT) {
+      float th[4], g[4], m[4] = {0.f, 0.f, 0.f, 0.f}, v[4] = {0.f, 0.f, 0.f, 0.f};
+      ld4(th, a.theta, k, vec, cnt);
+      ld4(g, a.g, k, vec, cnt);
+      if (a.m) ld4(m, a.m, k, vec, cnt);
+      if (a.adam && a.v) ld4(v, a.v, k, vec, cnt);
+      float mn[4], vn[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        if (a.adam) {
+          mn[j] = a.b1 * m[j] + (1.f - a.b1) * g[j];
+          vn[j] = a.b2 * v[j] + (1.f - a.b2) * g[j] * g[j];
+          vw[j] = th[j] - lr[j] * (mn[j] / a.c1) / (sqrtf(vn[j] / a.c2) + a.eps);
+        } else {
+          mn[j] = a.mu * m[j] + g[j];
+          vn[j] = 0.f;
+          vw[j] = th[j] - lr[j] * mn[j];
         }
-        if (a.cast_src) vw = a.cast_src[k];
-      } else if (a.mode == LU_ADJOINT) {
-        const float tb = a.theta_bar[k] + (a.Hu ? a.Hu[k] : 0.f);
-        a.theta_bar[k] = tb;
-        bad |= !isfinite(tb);
-        const float lr = lr_at(a.lr, k);
+        bad |= j < cnt && !isfinite(vw[j]);
+      }
+      st4(a.theta_out, k, vw, vec, cnt);
+      if (a.m_out) st4(a.m_out, k, mn, vec, cnt);
+      if (a.adam && a.v_out) st4(a.v_out, k, vn, vec, cnt);
+    } else if (a.mode == LU_ADJOINT) {
+      float tb[4], hu[4] = {0.f, 0.f, 0.f, 0.f};
+      ld4(tb, a.theta_bar, k, vec, cnt);
+      if (a.Hu) ld4(hu, a.Hu, k, vec, cnt);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        tb[j] += hu[j];
+        bad |= j < cnt && !isfinite(tb[j]);
+      }
+      st4(a.theta_bar, k, tb, vec, cnt);
+      float contrib[4] = {0.f, 0.f, 0.f, 0.f};
+      bool have_contrib = false;
+      if (a.adam && a.adam_pre) {
+        // reverse of Adam step j from its outputs m1 = m_{j+1}, v1 = v_{j+1} (see LayerUpdArgs)
+        float m1[4], v1[4], mp[4] = {0.f, 0.f, 0.f, 0.f};
+        float mb[4] = {0.f, 0.f, 0.f, 0.f}, vb[4] = {0.f, 0.f, 0.f, 0.f};
+        ld4(m1, a.m_adj, k, vec, cnt);
+        ld4(v1, a.v_adj, k, vec, cnt);
+        if (a.m_prev) ld4(mp, a.m_prev, k, vec, cnt);
+        if (a.bar_in) {
+          ld4(mb, a.mbar, k, vec, cnt);
+          ld4(vb, a.vbar, k, vec, cnt);
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float sq = sqrtf(v1[j] / a.c2);
+          const float den = sq + a.eps;
+          const float q = -lr[j] * tb[j];
+          // at v = 0 (where m = g = 0) the sqrt term is 0
+          const float Mb = mb[j] + q / (a.c1 * den);
+          const float Vb = vb[j] - (sq > 0.f ? q * m1[j] / (a.c1 * den * den * 2.f * sq * a.c2) : 0.f);
+          const float g = (m1[j] - a.b1 * mp[j]) / (1.f - a.b1);
+          vu[j] = (1.f - a.b1) * Mb + 2.f * (1.f - a.b2) * g * Vb;
+          mb[j] = a.b1 * Mb;
+          vb[j] = a.b2 * Vb;
+          contrib[j] = -lr[j] * (m1[j] / a.c1) / den * tb[j];
+          bad |= j < cnt && !isfinite(vu[j]);
+        }
+        st4(a.u_out, k, vu, vec, cnt);
+        st4(a.mbar, k, mb, vec, cnt);
+        st4(a.vbar, k, vb, vec, cnt);
+        have_contrib = true;
+      } else if (!a.adam) {
         if (a.m_adj) {
-          const float contrib = -lr * a.m_adj[k] * tb;
-          if (a.d_plr) a.d_plr[k] += contrib;
-          else acc += contrib;
+          float ma[4];
+          ld4(ma, a.m_adj, k, vec, cnt);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) contrib[j] = -lr[j] * ma[j] * tb[j];
+          have_contrib = true;
         }
         if (a.u_out) {
-          vu = (a.u_in ? a.mu * a.u_in[k] : 0.f) - lr * tb;
-          a.u_out[k] = vu;
+          float ui[4] = {0.f, 0.f, 0.f, 0.f};
+          if (a.u_in) ld4(ui, a.u_in, k, vec, cnt);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) vu[j] = a.mu * ui[j] - lr[j] * tb[j];
+          st4(a.u_out, k, vu, vec, cnt);
         }
-        if (a.cast_src) vw = a.cast_src[k];
-      } else {
-        const float v = a.cast_src[k];
-        vw = v;
-        vu = v;
       }
+      if (have_contrib) {
+        if (a.d_plr) {
+          float dp[4];
+          ld4(dp, a.d_plr, k, vec, cnt);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) dp[j] += contrib[j];
+          st4(a.d_plr, k, dp, vec, cnt);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) acc += j < cnt ? contrib[j] : 0.f;
+        }
+      }
+      if (a.cast_src) ld4(vw, a.cast_src, k, vec, cnt);
+    } else {
+      ld4(vw, a.cast_src, k, vec, cnt);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) vu[j] = vw[j];
     }
-    tw[i][tx] = vw;
-    tu[i][tx] = vu;
-    // row-major operand copies (only the din weight rows; the bias row stays float32)
-    if (r < din && c < dout) {
-      const int64_t o = static_cast<int64_t>(r) * tab.ldw[l] + c;
-      if (cast_w) static_cast<T*>(tab.W[l])[o] = to_t<T>(vw);
-      if (cast_u) static_cast<T*>(tab.U[l])[o] = to_t<T>(vu);
-    }
+    if (cast_w && tab.W[l]) st_copy<T>(static_cast<T*>(tab.W[l]), e0, dout, din, tab.ldw[l], vw, vec, cnt);
+    if (cast_u && tab.U[l]) st_copy<T>(static_cast<T*>(tab.U[l]), e0, dout, din, tab.ldw[l], vu, vec, cnt);
   }
   if (bad && a.status) atomicExch(a.status, DEV_NONFINITE);
-  if (a.partials) {
+  if (a.partials) {   // one deterministic partial sum per block (scalar log-lr)
     acc = warp_sum(acc);
-    const int lin = ty * TILE + tx;
-    if ((lin & 31) == 0) red[lin >> 5] = acc;
-  }
-  __syncthreads();
-  if (a.partials && ty == 0) {
-    float v = tx < (TILE * TROWS / 32) ? red[tx] : 0.f;
-    v = warp_sum(v);
-    if (tx == 0) a.partials[blockIdx.x] = v;
-  }
-  // transposed operand copies [dout][ldwt]
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int c = c0 + i, r = r0 + tx;
-    if (c < dout && r < din) {
-      const int64_t o = static_cast<int64_t>(c) * tab.ldwt[l] + r;
-      if (cast_w && tab.WT[l]) static_cast<T*>(tab.WT[l])[o] = to_t<T>(tw[tx][i]);
-      if (cast_u && tab.UT[l]) static_cast<T*>(tab.UT[l])[o] = to_t<T>(tu[tx][i]);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+      float v = threadIdx.x < UPD_THREADS / 32 ? red[threadIdx.x] : 0.f;
+      v = warp_sum(v);
+      if (threadIdx.x == 0) a.partials[blockIdx.x] = v;
     }
   }
 }
@@ -559,10 +636,26 @@ void sum_scaled(const float* x, int n, float scale, float* out, cudaStream_t s) 
 }
 
 template <typename T>
-void layer_update(const LayerTable& tab, const LayerUpdArgs& a, cudaStream_t s) {
+void layer_update(const LayerTable& tab, const LayerUpdArgs& args, cudaStream_t s) {
   const int blocks = tab.tile0[tab.n];
   if (blocks <= 0) return;
-  launch_k(layer_update_kernel<T>, dim3(blocks), dim3(TILE, TROWS), 0, s, tab, a);
+  // float4 access only when every vector the call touches is 16-byte aligned (caller
+  // pointers such as theta or eta + offset need not be)
+  LayerUpdArgs a = args;
+  uintptr_t any = 0;
+  for (const void* p : {static_cast<const void*>(a.cast_src), static_cast<const void*>(a.theta),
+                        static_cast<const void*>(a.m), static_cast<const void*>(a.g),
+                        static_cast<const void*>(a.theta_out), static_cast<const void*>(a.m_out),
+                        static_cast<const void*>(a.theta_bar), static_cast<const void*>(a.Hu),
+                        static_cast<const void*>(a.m_adj), static_cast<const void*>(a.u_in),
+                        static_cast<const void*>(a.u_out), static_cast<const void*>(a.d_plr),
+                        static_cast<const void*>(a.lr.plr), static_cast<const void*>(a.v),
+                        static_cast<const void*>(a.v_out), static_cast<const void*>(a.v_adj),
+                        static_cast<const void*>(a.m_prev), static_cast<const void*>(a.mbar),
+                        static_cast<const void*>(a.vbar)})
+    any |= reinterpret_cast<uintptr_t>(p);
+  a.vec_ok = (any & 15) == 0;
+  launch_k(layer_update_kernel<T>, dim3(blocks), dim3(UPD_THREADS), 0, s, tab, a);
 }
 
 template <typename T>

@@ -1,0 +1,67 @@
+"""Run mf_meta_grad a few times on a named case, for capturing kernels under ncu.
+
+``python -m paper_2505_00793_gb300.profile_run --case NAME [--calls N]`` prints the kernel
+launches of one call (from mf_stats) and runs N eager calls (CUDA graphs off, so every launch
+is visible).  The cases keep the device footprint at a few GB while the HBM-bound kernels
+still move far more than the 129 MB L2 per launch:
+
+* deep_4k       two 4096 x 4096 SiLU layers (33.6M parameters), B = 512, T = 2, momentum 0.9,
+                per-parameter log learning rates: the fused update kernels (K4/K5)
+* deep_4k_adam  the same with the Adam inner optimiser
+* decoder_small the bench's 6 x d512 decoder (row kernels: RMSNorm, RoPE, softmax, CE)
+* toy           the motivating example, M = 8 (chain loss kernels), either HVP mode
+"""
+from __future__ import annotations
+
+import argparse
+import math
+
+
+def case(name: str):
+    from paper_2505_00793_gb300 import synth
+    if name == "deep_4k":
+        return synth.Workload("deep_4k", [4096] * 3, "silu", "squared", "bf16", B=512, T=2,
+                              B_outer=512, momentum=0.9, meta_kind=synth.PARAM_LOGLR,
+                              loglr_mean=math.log(1e-2), loglr_std=0.1)
+    if name == "deep_4k_adam":
+        return case("deep_4k").with_(name="deep_4k_adam", momentum=0.0, optimizer="adam",
+                                     loglr_mean=math.log(1e-4))
+    if name in ("decoder_small", "toy"):
+        return synth.WORKLOADS[name]
+    raise ValueError(name)
+
+
+def main() -> None:
+    import torch
+    from paper_2505_00793_gb300 import native, synth
+
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--case", required=True,
+                    choices=["deep_4k", "deep_4k_adam", "decoder_small", "toy"])
+    ap.add_argument("--calls", type=int, default=3)
+    ap.add_argument("--hvp-mode", type=int, default=0)
+    args = ap.parse_args()
+    torch.cuda.set_device(0)
+    w = case(args.case)
+    inp = synth.make_inputs(w)
+    d = native.to_device_inputs(w, inp)
+    mf = native.MixFlow.for_workload(w)
+    mf.set_option(native.MF_OPT_CUDA_GRAPHS, 0)
+    loop = native.loop_desc_for(w, args.hvp_mode)
+    d_eta = torch.empty(w.n_eta, device="cuda")
+    d_th = torch.empty(w.n_params, device="cuda")
+    V = torch.empty(1, device="cuda")
+    n0, _ = mf.stats()
+    for i in range(args.calls):
+        mf.meta_grad(loop, d["theta0"], d["eta"], d["inner_x"], d["inner_y"], d["outer_x"],
+                     d["outer_y"], d_eta, d_th, V)
+        mf.sync()
+        if i == 0:
+            n1, peak = mf.stats()
+            print(f"{args.case}: {n1 - n0} launches per call, workspace {peak / 1e9:.2f} GB",
+                  flush=True)
+    mf.close()
+
+
+if __name__ == "__main__":
+    main()
