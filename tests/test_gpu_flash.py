@@ -112,3 +112,29 @@ def test_flash_workspace_saving():
     ss = BH * S * S
     saved = (2 * L + 2) * ss * 2 + 4 * ss * 4 - (L + 1) * 2 * BH * S * 4
     assert abs((ws_m - ws_f) - saved) <= 256 * (4 * L + 16), (ws_m - ws_f, saved)
+
+
+@pytest.mark.gpu
+def test_decoder_large_full_size_hvp_symmetry():
+    """The 218M-parameter decoder (12 blocks, d 1024, 16 heads, S = 1024, fused attention)
+    at full size: u^T (H v) = v^T (H u) through mf_hvp (Eqs. 6-7), and H is linear in its
+    direction.  Directions are scaled like the weights (0.02)."""
+    torch, native = need_gpu()
+    w = synth.WORKLOADS["decoder_large"]
+    w1 = w.with_(T=1)
+    inp = synth.make_inputs(w1)
+    d = native.to_device_inputs(w1, inp)
+    mf = native.MixFlow.for_workload(w)
+    u = torch.from_numpy(synth.random_direction(w.n_params, 4, 1)).cuda() * 0.02
+    v = torch.from_numpy(synth.random_direction(w.n_params, 4, 2)).cuda() * 0.02
+    Hu, Hv, Hs = torch.empty_like(u), torch.empty_like(v), torch.empty_like(u)
+    for vec, out in ((u, Hu), (v, Hv), (u + v, Hs)):
+        mf.hvp(w.B, d["theta0"], d["inner_x"][0], d["inner_y"][0], vec, out)
+    mf.sync()
+    mf.close()
+    a = float(torch.dot(u.double(), Hv.double()))
+    b = float(torch.dot(v.double(), Hu.double()))
+    assert np.isfinite(a) and np.isfinite(b)
+    scale = float(u.double().norm() * Hv.double().norm())
+    assert abs(a - b) <= 2e-2 * scale, (a, b, scale)
+    assert rel_l2(Hs.cpu().numpy(), (Hu + Hv).cpu().numpy()) < 2e-2
