@@ -345,11 +345,8 @@ struct Exec {
       tab.tile0[l] = tiles;
       tiles += mf::update_blocks(tab.rows[l], dout);
       tab.ldw[l] = ld8(dout);
-      tab.ldwt[l] = 0;
       tab.W[l] = at<T>(p.o_Wb[l]);
-      tab.WT[l] = nullptr;         // every product reads W row-major (K- or MN-major)
       tab.U[l] = at<T>(p.o_Ub[l]);
-      tab.UT[l] = nullptr;
     }
     tab.tile0[h->L] = tiles;
   }
@@ -614,7 +611,7 @@ struct Exec {
       if (l + 1 < L) {
         mf::ror_fwd_elem<T>(h->md.act, at<float>(p.o_DZB), at<float>(p.o_Z[l]),
                             at<float>(p.o_SA[l + 1]), rows, dout, at<T>(p.o_DAB[l]), p.lda[l + 1],
-                            nullptr, 0, at<float>(p.o_ZP[l]), s);
+                            at<float>(p.o_ZP[l]), s);
         launched();
       } else {
         // loss Hessian along dzbar (this is the forward tangent of the logits): zbar_{L-1},
@@ -646,7 +643,7 @@ struct Exec {
       const int din = h->dims[l], dout = h->dims[l + 1];
       if (l + 1 < L) {
         mf::ror_bwd_elem<T>(h->md.act, at<float>(p.o_ZP[l]), at<float>(p.o_AB), at<float>(p.o_Z[l]),
-                            rows, dout, at<T>(p.o_ZB), ld8(dout), nullptr, 0, s);
+                            rows, dout, at<T>(p.o_ZB), ld8(dout), s);
         launched();
       }
       // (H v)_{W_l, b_l} = [a_{l-1}^T; 1] zbar_l + [dabar_{l-1}^T; 0] dz_l

@@ -63,6 +63,7 @@ struct DecPlan {
   bool flash = false;
   std::vector<size_t> fst;
   size_t fD = 0;
+  size_t rope = 0;   // RoPE (cos, sin) table [S][dh/2]
 };
 
 DecPlan make_dec_plan(const mf_ctx* h, const DecLayout& Ly, int rows, int T, int n_theta_slots,
@@ -140,6 +141,7 @@ DecPlan make_dec_plan(const mf_ctx* h, const DecLayout& Ly, int rows, int T, int
   p.dP = take(SS * 4); p.dPd = take(SS * 4);
   p.dS = take(SS * es); p.dSd = take(SS * es);
   if (p.flash) p.fD = take(2 * stat);
+  p.rope = take(static_cast<size_t>(S) * (Ly.dh / 2) * 2 * 4);
   const size_t head4 = static_cast<size_t>(BH) * S * Ly.dh * 4;
   p.dQ = take(head4); p.dQd = take(head4); p.dK = take(head4); p.dKd = take(head4);
   p.dV = take(head4); p.dVd = take(head4);
@@ -184,11 +186,8 @@ struct DecExec {
       tab.tile0[i] = tiles;
       tiles += mf::update_blocks(t.rows, t.cols);
       tab.ldw[i] = ld8(t.cols);
-      tab.ldwt[i] = 0;
       tab.W[i] = t.cast ? at<T>(p.o_W[i]) : nullptr;   // read K- or MN-major, never transposed
-      tab.WT[i] = nullptr;
       tab.U[i] = t.cast ? at<T>(p.o_U[i]) : nullptr;
-      tab.UT[i] = nullptr;
     }
     tab.tile0[tab.n] = tiles;
   }
@@ -287,7 +286,10 @@ struct DecExec {
     g.bsC0 = g.bsC1 = bsC;
   }
 
-  void prepare() {}
+  void prepare() {
+    mf::dec_rope_table(Ly.S, Ly.dh, Ly.base, at<float>(p.rope), s);
+    launched();
+  }
 
   void update(const mf::LayerUpdArgs& a) {
     mf::layer_update<T>(tab, a, s);
@@ -337,11 +339,11 @@ struct DecExec {
         gemm(g);
       }
       const float qscale = 1.f / sqrtf(static_cast<float>(dh));
-      mf::dec_rope_split<T>(N, S, H, dh, Ly.base, qscale, at<float>(p.qkv), at<T>(p.Q[l]),
+      mf::dec_rope_split<T>(N, S, H, dh, at<float>(p.rope), qscale, at<float>(p.qkv), at<T>(p.Q[l]),
                             at<T>(p.K[l]), at<T>(p.Vv[l]), s);
       launched();
       if (dual) {
-        mf::dec_rope_split<T>(N, S, H, dh, Ly.base, qscale, at<float>(p.qkvd), at<T>(p.Qd[l]),
+        mf::dec_rope_split<T>(N, S, H, dh, at<float>(p.rope), qscale, at<float>(p.qkvd), at<T>(p.Qd[l]),
                               at<T>(p.Kd[l]), at<T>(p.Vd[l]), s);
         launched();
       }
@@ -486,7 +488,10 @@ struct DecExec {
   }
 
   // residual gradient (float32) -> operand-type seed
-  void seed_from(const float* X, const float* Xd, bool dual) {
+  // bf16 seeds dy (dy') of the next products from the residual-stream gradient dx (dx');
+  // skipped when the RMSNorm backward that produced dx already wrote them (fresh)
+  void seed_from(const float* X, const float* Xd, bool dual, bool fresh = false) {
+    if (fresh) return;
     const int N = rows_cur * Ly.S, d = Ly.d;
     mf::cast_rows<T>(X, N, d, at<T>(p.dy), d, s);
     launched();
@@ -518,7 +523,8 @@ struct DecExec {
     if (dual) cudaMemsetAsync(at<float>(p.dxd), 0, static_cast<size_t>(N) * d * 4, s);
     mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.xf), at<float>(p.xfd), at<float>(p.rf), at<float>(p.rfd),
                            theta_cur + Ly.gf, dual ? u + Ly.gf : nullptr, at<float>(p.dh),
-                           dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx), at<float>(p.dxd), s);
+                           dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx), at<float>(p.dxd), s,
+                           at<T>(p.dy), dual ? at<T>(p.dyd) : nullptr);
     mf::dec_gain_grad(N, d, at<float>(p.xf), at<float>(p.xfd), at<float>(p.rf), at<float>(p.rfd),
                       at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr, G(Ly.gf), Hh(Ly.gf),
                       at<float>(p.gpart), s);
@@ -531,8 +537,8 @@ struct DecExec {
         cudaMemcpyAsync(at<float>(p.dx), at<float>(p.dxs[l]), static_cast<size_t>(N) * d * 4,
                         cudaMemcpyDeviceToDevice, s);
       }
-      // ---- MLP branch: seed = dx -------------------------------------------------------
-      seed_from(at<float>(p.dx), at<float>(p.dxd), dual);
+      // ---- MLP branch: seed = dx (already in bf16 unless dx was just restored) ---------
+      seed_from(at<float>(p.dx), at<float>(p.dxd), dual, ror_mode != 2);
       wprod(F, d, at<T>(p.a1[l]), at<T>(p.a1d[l]), at<T>(p.dy), at<T>(p.dyd), dual, G(Ly.W2[l]),
             Hh(Ly.W2[l]));
       {
@@ -561,10 +567,10 @@ struct DecExec {
       mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.x2[l]), at<float>(p.x2d[l]), at<float>(p.r2[l]),
                              at<float>(p.r2d[l]), theta_cur + Ly.g2[l], dual ? u + Ly.g2[l] : nullptr,
                              at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx),
-                             at<float>(p.dxd), s);
+                             at<float>(p.dxd), s, at<T>(p.dy), dual ? at<T>(p.dyd) : nullptr);
       launched(2);
-      // ---- attention branch: seed = dx --------------------------------------------------
-      seed_from(at<float>(p.dx), at<float>(p.dxd), dual);
+      // ---- attention branch: seed = dx (written in bf16 by the norm backward above) -----
+      seed_from(at<float>(p.dx), at<float>(p.dxd), dual, true);
       wprod(d, d, at<T>(p.Om[l]), at<T>(p.Omd[l]), at<T>(p.dy), at<T>(p.dyd), dual, G(Ly.Wo[l]),
             Hh(Ly.Wo[l]));
       {
@@ -636,11 +642,11 @@ struct DecExec {
       }
       }
       const float qscale = 1.f / sqrtf(static_cast<float>(dh));
-      mf::dec_rope_merge<T>(N, S, H, dh, Ly.base, qscale, at<float>(p.dQ), at<float>(p.dK),
+      mf::dec_rope_merge<T>(N, S, H, dh, at<float>(p.rope), qscale, at<float>(p.dQ), at<float>(p.dK),
                             at<float>(p.dV), at<T>(p.dqkv), 3 * d, s);
       launched();
       if (dual) {
-        mf::dec_rope_merge<T>(N, S, H, dh, Ly.base, qscale, at<float>(p.dQd), at<float>(p.dKd),
+        mf::dec_rope_merge<T>(N, S, H, dh, at<float>(p.rope), qscale, at<float>(p.dQd), at<float>(p.dKd),
                               at<float>(p.dVd), at<T>(p.dqkvd), 3 * d, s);
         launched();
       }
@@ -659,7 +665,8 @@ struct DecExec {
       mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.x1[l]), at<float>(p.x1d[l]), at<float>(p.r1[l]),
                              at<float>(p.r1d[l]), theta_cur + Ly.g1[l], dual ? u + Ly.g1[l] : nullptr,
                              at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx),
-                             at<float>(p.dxd), s);
+                             at<float>(p.dxd), s, l > 0 ? at<T>(p.dy) : nullptr,
+                             l > 0 && dual ? at<T>(p.dyd) : nullptr);
       launched(2);
     }
     mf::dec_embed_bwd(V, d, at<int>(p.o_start), at<int>(p.o_order), at<float>(p.dx),

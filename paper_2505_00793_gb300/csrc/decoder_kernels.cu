@@ -126,7 +126,8 @@ __global__ void rmsnorm_bwd_kernel(int d, const float* __restrict__ x, const flo
                                    const float* __restrict__ rr, const float* __restrict__ rrd,
                                    const float* __restrict__ g, const float* __restrict__ gd,
                                    const float* __restrict__ dy, const float* __restrict__ dyd,
-                                   float* __restrict__ dx, float* __restrict__ dxd) {
+                                   float* __restrict__ dx, float* __restrict__ dxd,
+                                   T* __restrict__ dxb, T* __restrict__ dxdb) {
   pdl_entry();
   const int r = blockIdx.x;
   const int64_t o = static_cast<int64_t>(r) * d;
@@ -150,11 +151,15 @@ __global__ void rmsnorm_bwd_kernel(int d, const float* __restrict__ x, const flo
   for (int j = threadIdx.x; j < d; j += blockDim.x) {
     const float n = x[o + j] * rs;
     const float dn = dy[o + j] * g[j];
-    dx[o + j] += rs * (dn - n * c);
+    const float v = dx[o + j] + rs * (dn - n * c);
+    dx[o + j] = v;
+    if (dxb) dxb[o + j] = to_t<T>(v);
     if (dual) {
       const float nd = xd[o + j] * rs + x[o + j] * rsd;
       const float dnd = dyd[o + j] * g[j] + dy[o + j] * gd[j];
-      dxd[o + j] += rsd * (dn - n * c) + rs * (dnd - nd * c - n * cd);
+      const float vd = dxd[o + j] + rsd * (dn - n * c) + rs * (dnd - nd * c - n * cd);
+      dxd[o + j] = vd;
+      if (dxdb) dxdb[o + j] = to_t<T>(vd);
     }
   }
 }
@@ -215,11 +220,23 @@ __global__ void gain_grad_final_kernel(int nchunk, int d, const float* __restric
   if (partd && dgd) dgd[j] = td;
 }
 
+// RoPE angle table: (cos, sin) of s * base^(-2 j / dh) for positions s < S and pairs
+// j < dh/2, interleaved, computed once per call in double precision.
+__global__ void rope_table_kernel(int S, int half, int dh, double base, float* __restrict__ tab) {
+  pdl_entry();
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= S * half) return;
+  const int s = i / half, j = i % half;
+  const double ang = static_cast<double>(s) * pow(base, -2.0 * j / dh);
+  tab[2 * i] = static_cast<float>(cos(ang));
+  tab[2 * i + 1] = static_cast<float>(sin(ang));
+}
+
 // RoPE (rotate-half) on q and k, q scaled by 1/sqrt(dh), head split.  qkv [N][3d] float32
-// (token-major) -> Q, K, V [B*H][S][dh] in T.  Angle of pair j at position s:
-// s * base^(-2 j / dh).
+// (token-major) -> Q, K, V [B*H][S][dh] in T.  cos / sin of the angle of pair j at position
+// s come from the table of rope_table_kernel.
 template <typename T>
-__global__ void rope_split_kernel(int S, int H, int dh, float base, float qscale,
+__global__ void rope_split_kernel(int S, int H, int dh, const float* __restrict__ rtab, float qscale,
                                   const float* __restrict__ qkv, T* __restrict__ Q,
                                   T* __restrict__ K, T* __restrict__ Vv) {
   pdl_entry();
@@ -230,9 +247,8 @@ __global__ void rope_split_kernel(int S, int H, int dh, float base, float qscale
   for (int c = threadIdx.x; c < d; c += blockDim.x) {
     const int h = c / dh, e = c % dh;
     const int j = e < half ? e : e - half;
-    const float ang = static_cast<float>(s) * powf(base, -2.f * static_cast<float>(j) / static_cast<float>(dh));
-    float sn, cs;
-    sincosf(ang, &sn, &cs);
+    const float2 cs_sn = reinterpret_cast<const float2*>(rtab)[s * half + j];
+    const float cs = cs_sn.x, sn = cs_sn.y;
     const float q = row[c], k = row[d + c];
     const float qo = e < half ? -row[c + half] : row[c - half];
     const float ko = e < half ? -row[d + c + half] : row[d + c - half];
@@ -247,7 +263,7 @@ __global__ void rope_split_kernel(int S, int H, int dh, float base, float qscale
 // dqkv [N][3d] row-major (T):  dq = R^T(dQ) qscale, dk = R^T(dK), dv = dV, with
 // R^T(y) = y cos + [y2, -y1] sin.
 template <typename T>
-__global__ void rope_merge_kernel(int S, int H, int dh, float base, float qscale,
+__global__ void rope_merge_kernel(int S, int H, int dh, const float* __restrict__ rtab, float qscale,
                                   const float* __restrict__ dQ, const float* __restrict__ dK,
                                   const float* __restrict__ dV, T* __restrict__ out, int ldo) {
   pdl_entry();
@@ -257,9 +273,8 @@ __global__ void rope_merge_kernel(int S, int H, int dh, float base, float qscale
   for (int c = threadIdx.x; c < d; c += blockDim.x) {
     const int h = c / dh, e = c % dh;
     const int j = e < half ? e : e - half;
-    const float ang = static_cast<float>(s) * powf(base, -2.f * static_cast<float>(j) / static_cast<float>(dh));
-    float sn, cs;
-    sincosf(ang, &sn, &cs);
+    const float2 cs_sn = reinterpret_cast<const float2*>(rtab)[s * half + j];
+    const float cs = cs_sn.x, sn = cs_sn.y;
     const int64_t o = ((static_cast<int64_t>(b) * H + h) * S + s) * dh;
     const float q = dQ[o + e], k = dK[o + e];
     const float qo = e < half ? dQ[o + e + half] : -dQ[o + e - half];
@@ -547,47 +562,81 @@ __global__ void token_order_kernel(const int* __restrict__ start, const int* __r
 }
 
 // dE[v] = sum over tokens with id v (in position order) of dx[token]; one block per id.
-__global__ void embed_bwd_kernel(int d, const int* __restrict__ start,
-                                 const int* __restrict__ order, const float* __restrict__ dx,
-                                 const float* __restrict__ dxd, float* __restrict__ dE,
-                                 float* __restrict__ dEd) {
+// Embedding gradient: row v of dE is the sum of dx over the tokens with id v, in token order
+// (start/order from the counting sort).  Eight warps split a segment into contiguous parts
+// (Zipf-distributed ids give a few very long segments).  A warp sums every column of a row
+// at once (up to 1024 columns: eight float4 loads per lane in flight), then the warps'
+// partial sums are added in warp order, so the result is deterministic.
+__global__ void __launch_bounds__(256) embed_bwd_kernel(int d, const int* __restrict__ start,
+                                                        const int* __restrict__ order,
+                                                        const float* __restrict__ dx,
+                                                        const float* __restrict__ dxd,
+                                                        float* __restrict__ dE,
+                                                        float* __restrict__ dEd, bool vec_out) {
   pdl_entry();
+  constexpr int NC = 8;                 // 128-column chunks per pass
+  __shared__ float4 part[2][8][32];
   const int v = blockIdx.x;
-  const int a = start[v], e = start[v + 1];
-  for (int j = threadIdx.x; j < d; j += blockDim.x) {
-    float s = 0.f, sd = 0.f;
-    for (int k = a; k < e; ++k) {
-      const int64_t o = static_cast<int64_t>(order[k]) * d + j;
-      s += dx[o];
-      if (dxd) sd += dxd[o];
+  const int a = start[v], cnt = start[v + 1] - a;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r0 = a + (w * cnt) / 8, r1 = a + ((w + 1) * cnt) / 8;
+  const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int g0 = 0; g0 < d; g0 += NC * 128) {
+    float4 acc[NC], dacc[NC];
+#pragma unroll
+    for (int q = 0; q < NC; ++q) { acc[q] = zero; dacc[q] = zero; }
+    // the row indices of 32 rows at a time, one per lane, broadcast by shuffles, so a row's
+    // loads do not wait on its index load
+    for (int kb = r0; kb < r1; kb += 32) {
+      const int mine = kb + lane < r1 ? order[kb + lane] : 0;
+      const int nb = r1 - kb < 32 ? r1 - kb : 32;
+#pragma unroll 2
+      for (int t = 0; t < nb; ++t) {
+        const int64_t ro = static_cast<int64_t>(__shfl_sync(0xffffffffu, mine, t)) * d;
+#pragma unroll
+        for (int q = 0; q < NC; ++q) {
+          const int c = g0 + q * 128 + lane * 4;
+          if (c < d) {
+            const float4 x = *reinterpret_cast<const float4*>(dx + ro + c);
+            acc[q].x += x.x; acc[q].y += x.y; acc[q].z += x.z; acc[q].w += x.w;
+            if (dxd) {
+              const float4 y = *reinterpret_cast<const float4*>(dxd + ro + c);
+              dacc[q].x += y.x; dacc[q].y += y.y; dacc[q].z += y.z; dacc[q].w += y.w;
+            }
+          }
+        }
+      }
     }
-    if (dE) dE[static_cast<int64_t>(v) * d + j] = s;
-    if (dEd) dEd[static_cast<int64_t>(v) * d + j] = sd;
+#pragma unroll
+    for (int q = 0; q < NC; ++q) {
+      const int c0 = g0 + q * 128;
+      if (c0 >= d) break;          // uniform across the block
+      part[0][w][lane] = acc[q];
+      part[1][w][lane] = dacc[q];
+      __syncthreads();
+      if (threadIdx.x < 64) {
+        const int which = threadIdx.x >> 5, l = threadIdx.x & 31, cc = c0 + l * 4;
+        float4 t = part[which][0][l];
+        for (int r = 1; r < 8; ++r) {
+          const float4 u = part[which][r][l];
+          t.x += u.x; t.y += u.y; t.z += u.z; t.w += u.w;
+        }
+        float* out = which == 0 ? dE : dEd;
+        if (out && cc < d) {
+          float* dst = out + static_cast<int64_t>(v) * d + cc;
+          if (vec_out) {
+            *reinterpret_cast<float4*>(dst) = t;
+          } else {   // the caller's gradient buffer need not be 16-byte aligned
+            dst[0] = t.x; dst[1] = t.y; dst[2] = t.z; dst[3] = t.w;
+          }
+        }
+      }
+      __syncthreads();
+    }
   }
 }
 
 constexpr int TILE = 32, TROWS = 8;
-
-// Batched transpose: X [batch][rows][ld] -> XT [batch][cols][ldT].
-template <typename TI, typename TO>
-__global__ void transpose_b_kernel(const TI* __restrict__ X, int rows, int cols, int ld,
-                                   int64_t bsX, TO* __restrict__ XT, int ldT, int64_t bsT) {
-  pdl_entry();
-  __shared__ float tile[TILE][TILE + 1];
-  const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
-  X += blockIdx.z * bsX;
-  XT += blockIdx.z * bsT;
-  const int tx = threadIdx.x, ty = threadIdx.y;
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int r = r0 + i, c = c0 + tx;
-    if (r < rows && c < cols) tile[i][tx] = ld_t(X, static_cast<int64_t>(r) * ld + c);
-  }
-  __syncthreads();
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int c = c0 + i, r = r0 + tx;
-    if (c < cols && r < rows) XT[static_cast<int64_t>(c) * ldT + r] = to_t<TO>(tile[tx][i]);
-  }
-}
 
 // Row-major cast (with a leading dimension) float32 -> T.
 template <typename T>
@@ -627,8 +676,9 @@ void dec_rmsnorm_fwd(int N, int d, float eps, const float* x_in, const float* y,
 template <typename T>
 void dec_rmsnorm_bwd(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
                      const float* g, const float* gd, const float* dy, const float* dyd, float* dx,
-                     float* dxd, cudaStream_t s) {
-  launch_k(rmsnorm_bwd_kernel<T>, dim3(N), dim3(256), 0, s, d, x, xd, r, rd, g, gd, dy, dyd, dx, dxd);
+                     float* dxd, cudaStream_t s, T* dxb, T* dxdb) {
+  launch_k(rmsnorm_bwd_kernel<T>, dim3(N), dim3(256), 0, s, d, x, xd, r, rd, g, gd, dy, dyd, dx, dxd,
+           dxb, dxdb);
 }
 
 int dec_gain_chunks(int N) { return (N + GG_ROWS - 1) / GG_ROWS; }
@@ -645,16 +695,22 @@ void dec_gain_grad(int N, int d, const float* x, const float* xd, const float* r
            dg, dgd);
 }
 
-template <typename T>
-void dec_rope_split(int N, int S, int H, int dh, float base, float qscale, const float* qkv, T* Q,
-                    T* K, T* V, cudaStream_t s) {
-  launch_k(rope_split_kernel<T>, dim3(N), dim3(256), 0, s, S, H, dh, base, qscale, qkv, Q, K, V);
+void dec_rope_table(int S, int dh, float base, float* tab, cudaStream_t s) {
+  const int n = S * (dh / 2);
+  launch_k(rope_table_kernel, dim3((n + 255) / 256), dim3(256), 0, s, S, dh / 2, dh,
+           static_cast<double>(base), tab);
 }
 
 template <typename T>
-void dec_rope_merge(int N, int S, int H, int dh, float base, float qscale, const float* dQ,
+void dec_rope_split(int N, int S, int H, int dh, const float* rtab, float qscale, const float* qkv,
+                    T* Q, T* K, T* V, cudaStream_t s) {
+  launch_k(rope_split_kernel<T>, dim3(N), dim3(256), 0, s, S, H, dh, rtab, qscale, qkv, Q, K, V);
+}
+
+template <typename T>
+void dec_rope_merge(int N, int S, int H, int dh, const float* rtab, float qscale, const float* dQ,
                     const float* dK, const float* dV, T* out, int ldo, cudaStream_t s) {
-  launch_k(rope_merge_kernel<T>, dim3(N), dim3(256), 0, s, S, H, dh, base, qscale, dQ, dK, dV, out, ldo);
+  launch_k(rope_merge_kernel<T>, dim3(N), dim3(256), 0, s, S, H, dh, rtab, qscale, dQ, dK, dV, out, ldo);
 }
 
 template <typename T>
@@ -710,15 +766,8 @@ void dec_token_csr(int N, int S, int V, const int* ids, int* count, int* start, 
 
 void dec_embed_bwd(int V, int d, const int* start, const int* order, const float* dx,
                    const float* dxd, float* dE, float* dEd, cudaStream_t s) {
-  launch_k(embed_bwd_kernel, dim3(V), dim3(256), 0, s, d, start, order, dx, dxd, dE, dEd);
-}
-
-template <typename TI, typename TO>
-void transpose_batched(const TI* X, int rows, int cols, int ld, int64_t bsX, TO* XT, int ldT,
-                       int64_t bsT, int batch, cudaStream_t s) {
-  if (rows <= 0 || cols <= 0 || batch <= 0) return;
-  dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE, batch);
-  launch_k(transpose_b_kernel<TI, TO>, dim3(grid), dim3(TILE, TROWS), 0, s, X, rows, cols, ld, bsX, XT, ldT, bsT);
+  const bool vec_out = ((reinterpret_cast<uintptr_t>(dE) | reinterpret_cast<uintptr_t>(dEd)) & 15) == 0;
+  launch_k(embed_bwd_kernel, dim3(V), dim3(256), 0, s, d, start, order, dx, dxd, dE, dEd, vec_out);
 }
 
 template <typename T>
@@ -732,10 +781,10 @@ void cast_rows(const float* X, int rows, int cols, T* Y, int ldy, cudaStream_t s
                                    float*, float*, T*, T*, int, cudaStream_t);                     \
   template void dec_rmsnorm_bwd<T>(int, int, const float*, const float*, const float*,             \
                                    const float*, const float*, const float*, const float*,         \
-                                   const float*, float*, float*, cudaStream_t);                    \
-  template void dec_rope_split<T>(int, int, int, int, float, float, const float*, T*, T*, T*,      \
+                                   const float*, float*, float*, cudaStream_t, T*, T*);            \
+  template void dec_rope_split<T>(int, int, int, int, const float*, float, const float*, T*, T*, T*,      \
                                   cudaStream_t);                                                   \
-  template void dec_rope_merge<T>(int, int, int, int, float, float, const float*, const float*,    \
+  template void dec_rope_merge<T>(int, int, int, int, const float*, float, const float*, const float*,    \
                                   const float*, T*, int, cudaStream_t);                            \
   template void dec_head_merge<T>(int, int, int, int, const float*, T*, int, cudaStream_t);       \
   template void dec_head_split<T>(int, int, int, int, const float*, T*, cudaStream_t);            \
@@ -749,13 +798,5 @@ void cast_rows(const float* X, int rows, int cols, T* Y, int ldy, cudaStream_t s
 MF_DEC_INST(float)
 MF_DEC_INST(__nv_bfloat16)
 #undef MF_DEC_INST
-template void transpose_batched<float, float>(const float*, int, int, int, int64_t, float*, int,
-                                              int64_t, int, cudaStream_t);
-template void transpose_batched<__nv_bfloat16, __nv_bfloat16>(const __nv_bfloat16*, int, int, int,
-                                                              int64_t, __nv_bfloat16*, int, int64_t,
-                                                              int, cudaStream_t);
-template void transpose_batched<float, __nv_bfloat16>(const float*, int, int, int, int64_t,
-                                                      __nv_bfloat16*, int, int64_t, int,
-                                                      cudaStream_t);
 
 }  // namespace mf

@@ -67,20 +67,6 @@ extern int g_pair_mode;
 cudaError_t simt_gemm(const GemmArgs& a, cudaStream_t s);
 
 // ---- elementwise / row kernels (kernels.cu); T is float or __nv_bfloat16 -------------
-// X [rows][ld] (T) -> XT [cols][ldT] (T)
-template <typename T>
-void transpose(const T* X, int rows, int cols, int ld, T* XT, int ldT, cudaStream_t s);
-// Set one row (columns 0..cols-1) of each listed matrix to a value: the bias row of the
-// augmented transposed activations [a^T; 1] and [a'^T; 0] of the weight products.
-struct RowFill {
-  int n = 0;
-  void* dst[64];
-  int row[64];
-  int ld[64];
-  float value[64];
-};
-template <typename T>
-void fill_rows(const RowFill& f, int cols, cudaStream_t s);
 
 // Column fills: dst[n][r * ld[n] + col[n]] = value[n] for r < rows.
 struct ColFill {
@@ -127,8 +113,8 @@ struct LrArgs {
 
 // Per-layer view of the flat parameter vector for the fused update/cast kernel.  Layer l
 // occupies rows[l] x dout[l] floats at off[l] (W_l rows, then the bias row when present);
-// its first din[l] rows are cast to the GEMM operand copies W (row-major [din][ldw]) and
-// WT (transposed [dout][ldwt]), or U / UT for the tangent.
+// its first din[l] rows are cast to the GEMM operand copy W (row-major [din][ldw]), or U for
+// the tangent.
 constexpr int kMaxLayers = 96;
 // Fused update kernel geometry: UPD_THREADS threads of four parameters each per block;
 // update_blocks is the block count of one layer (and the number of scalar-lr partials).
@@ -143,20 +129,20 @@ struct LayerTable {
   int rows[kMaxLayers], din[kMaxLayers], dout[kMaxLayers];
   int64_t off[kMaxLayers];
   int tile0[kMaxLayers + 1];
-  int ldw[kMaxLayers], ldwt[kMaxLayers];
-  void* W[kMaxLayers]; void* WT[kMaxLayers]; void* U[kMaxLayers]; void* UT[kMaxLayers];
+  int ldw[kMaxLayers];
+  void* W[kMaxLayers]; void* U[kMaxLayers];
 };
 
 enum LuMode : int { LU_CAST = 0, LU_ROLLOUT = 1, LU_ADJOINT = 2 };
 struct LayerUpdArgs {
   int mode = LU_CAST;
-  const float* cast_src = nullptr;  // parameters to cast into W/WT (nullable)
-  bool cast_src_to_u = false;       // LU_CAST: write into U/UT instead of W/WT
-  // LU_ROLLOUT (K4):  m' = mu m + g ; theta' = theta - lr m' ; cast theta' into W/WT
+  const float* cast_src = nullptr;  // parameters to cast into W (nullable)
+  bool cast_src_to_u = false;       // LU_CAST: write into U instead of W
+  // LU_ROLLOUT (K4):  m' = mu m + g ; theta' = theta - lr m' ; cast theta' into W
   const float* theta = nullptr; const float* m = nullptr; const float* g = nullptr;
   float* theta_out = nullptr; float* m_out = nullptr;
   // LU_ADJOINT (K5):  theta_bar += Hu ; d eta_lr from m_adj ; u' = mu u - lr theta_bar ;
-  //                   cast u' into U/UT
+  //                   cast u' into U
   float* theta_bar = nullptr; const float* Hu = nullptr; const float* m_adj = nullptr;
   const float* u_in = nullptr; float* u_out = nullptr; float* d_plr = nullptr;
   float* partials = nullptr;       // scalar log-lr: one partial per block (tile)
@@ -185,13 +171,13 @@ void layer_update(const LayerTable& tab, const LayerUpdArgs& a, cudaStream_t s);
 void fill(float* p, int64_t n, float v, cudaStream_t s);
 
 // Reverse-over-reverse element kernels (MLP): dabar = dzbar phi'(z), zpart = dzbar phi''(z) da;
-// zbar = zpart + abar phi'(z).  T outputs row-major and transposed.
+// zbar = zpart + abar phi'(z).  T outputs row-major [rows][ld].
 template <typename T>
 void ror_fwd_elem(int act, const float* dzbar, const float* Z, const float* dA, int rows, int cols,
-                  T* dab, int ld, T* dabT, int ldT, float* zpart, cudaStream_t s);
+                  T* dab, int ld, float* zpart, cudaStream_t s);
 template <typename T>
 void ror_bwd_elem(int act, const float* zpart, const float* abar, const float* Z, int rows,
-                  int cols, T* zb, int ld, T* zbT, int ldT, cudaStream_t s);
+                  int cols, T* zb, int ld, cudaStream_t s);
 
 // ---- fused dual attention (flash_attn.cu) -------------------------------------------------
 // Heads [BH][S][64] bf16 (q pre-scaled by 1/sqrt(64)), causal.  Forward: O (and O') float32
@@ -222,20 +208,24 @@ template <typename T>
 void dec_rmsnorm_fwd(int N, int d, float eps, const float* x_in, const float* y, const float* xd_in,
                      const float* yd, const float* g, const float* gd, float* x_out, float* xd_out,
                      float* r, float* rd, T* h, T* hd, int ldh, cudaStream_t s);
+// dx (+=) the RMSNorm backward; when dxb / dxdb are given the updated dx / dx' are also
+// written in T (the next GEMM seeds), row-major [N][d].
 template <typename T>
 void dec_rmsnorm_bwd(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
                      const float* g, const float* gd, const float* dy, const float* dyd, float* dx,
-                     float* dxd, cudaStream_t s);
+                     float* dxd, cudaStream_t s, T* dxb = nullptr, T* dxdb = nullptr);
 int dec_gain_chunks(int N);
 // part: scratch of 2 * dec_gain_chunks(N) * d floats
 void dec_gain_grad(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
                    const float* dy, const float* dyd, float* dg, float* dgd, float* part,
                    cudaStream_t s);
+// RoPE table [S][dh/2] of (cos, sin) pairs, float32, from double-precision angles.
+void dec_rope_table(int S, int dh, float base, float* tab, cudaStream_t s);
 template <typename T>
-void dec_rope_split(int N, int S, int H, int dh, float base, float qscale, const float* qkv, T* Q,
-                    T* K, T* V, cudaStream_t s);
+void dec_rope_split(int N, int S, int H, int dh, const float* rtab, float qscale, const float* qkv,
+                    T* Q, T* K, T* V, cudaStream_t s);
 template <typename T>
-void dec_rope_merge(int N, int S, int H, int dh, float base, float qscale, const float* dQ,
+void dec_rope_merge(int N, int S, int H, int dh, const float* rtab, float qscale, const float* dQ,
                     const float* dK, const float* dV, T* out, int ldo, cudaStream_t s);
 template <typename T>
 void dec_head_merge(int N, int S, int H, int dh, const float* O, T* out, int ldo, cudaStream_t s);
@@ -260,9 +250,6 @@ void dec_token_csr(int N, int S, int V, const int* ids, int* count, int* start, 
                    int* tmp, cudaStream_t s);
 void dec_embed_bwd(int V, int d, const int* start, const int* order, const float* dx,
                    const float* dxd, float* dE, float* dEd, cudaStream_t s);
-template <typename TI, typename TO>
-void transpose_batched(const TI* X, int rows, int cols, int ld, int64_t bsX, TO* XT, int ldT,
-                       int64_t bsT, int batch, cudaStream_t s);
 template <typename T>
 void cast_rows(const float* X, int rows, int cols, T* Y, int ldy, cudaStream_t s);
 

@@ -2,11 +2,13 @@
 //
 //  * per-example loss seeds with the tangent per-example loss (the mixed term of Eq. 7 for
 //    per-example weights) and d eta_{t,b} = sigmoid'(eta_{t,b}) * l'_b / B;
-//  * the fused per-layer update kernel: the inner-step update of Eq. 2 (rollout) or the
-//    adjoint update of the reverse sweep (Eq. 5 with the Hessian product supplied by the
-//    forward-over-reverse pass), each fused with the cast of the next step's parameters /
-//    tangent into the row-major and transposed GEMM operand copies;
-//  * transposes, row fills and a deterministic sum.
+//  * the fused per-layer update kernel: the inner-step update of Eq. 2 (rollout, SGD,
+//    heavy ball or Adam) or the adjoint update of the reverse sweep (Eq. 5 with the Hessian
+//    product supplied by the forward-over-reverse pass, and the elementwise reverse of the
+//    optimiser step), each fused with the cast of the next step's parameters / tangent into
+//    the bf16 GEMM operand copies;
+//  * the chain loss of the motivating example, in both HVP modes;
+//  * the reverse-over-reverse element kernels, column fills and a deterministic sum.
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <math.h>
@@ -22,34 +24,6 @@ int g_pdl = 1;
 namespace {
 
 constexpr int TILE = 32, TROWS = 8;
-
-template <typename T>
-__global__ void transpose_kernel(const T* __restrict__ X, int rows, int cols, int ld,
-                                 T* __restrict__ XT, int ldT) {
-  pdl_entry();
-  __shared__ T tile[TILE][TILE + 1];
-  const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
-  const int tx = threadIdx.x, ty = threadIdx.y;
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int r = r0 + i, c = c0 + tx;
-    if (r < rows && c < cols) tile[i][tx] = X[static_cast<int64_t>(r) * ld + c];
-  }
-  __syncthreads();
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int c = c0 + i, r = r0 + tx;
-    if (c < cols && r < rows) XT[static_cast<int64_t>(c) * ldT + r] = tile[tx][i];
-  }
-}
-
-template <typename T>
-__global__ void fill_rows_kernel(const RowFill f, int cols) {
-  pdl_entry();
-  const int k = blockIdx.y;
-  const int c = blockIdx.x * blockDim.x + threadIdx.x;
-  if (k >= f.n || c >= cols) return;
-  T* dst = static_cast<T*>(f.dst[k]);
-  dst[static_cast<int64_t>(f.row[k]) * f.ld[k] + c] = to_t<T>(f.value[k]);
-}
 
 template <typename T>
 __global__ void fill_cols_kernel(const ColFill f, int rows) {
@@ -528,62 +502,41 @@ __global__ void __launch_bounds__(UPD_THREADS) layer_update_kernel(const LayerTa
 }
 
 // Reverse-over-reverse, forward layer order: from dzbar (the adjoint of the backward's dz):
-//   dabar = dzbar phi'(z)  (T, row-major and transposed),  zpart = dzbar phi''(z) da.
+//   dabar = dzbar phi'(z)  (T, row-major [rows][ld]),  zpart = dzbar phi''(z) da.
 template <typename T>
 __global__ void ror_fwd_elem_kernel(int act, const float* __restrict__ dzbar,
                                     const float* __restrict__ Z, const float* __restrict__ dA,
                                     int rows, int cols, T* __restrict__ dab, int ld,
-                                    T* __restrict__ dabT, int ldT, float* __restrict__ zpart) {
+                                    float* __restrict__ zpart) {
   pdl_entry();
-  __shared__ float tile[TILE][TILE + 1];
-  const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
-  const int tx = threadIdx.x, ty = threadIdx.y;
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int r = r0 + i, c = c0 + tx;
-    float v = 0.f;
+  const int c = blockIdx.x * TILE + threadIdx.x;
+  for (int i = threadIdx.y; i < TILE; i += TROWS) {
+    const int r = blockIdx.y * TILE + i;
     if (r < rows && c < cols) {
       const int64_t o = static_cast<int64_t>(r) * cols + c;
       float f, d1, d2;
       act_eval(act, Z[o], f, d1, d2);
-      v = dzbar[o] * d1;
       zpart[o] = dzbar[o] * d2 * dA[o];
-      dab[static_cast<int64_t>(r) * ld + c] = to_t<T>(v);
+      dab[static_cast<int64_t>(r) * ld + c] = to_t<T>(dzbar[o] * d1);
     }
-    tile[i][tx] = v;
-  }
-  __syncthreads();
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int c = c0 + i, r = r0 + tx;
-    if (dabT && c < cols && r < rows) dabT[static_cast<int64_t>(c) * ldT + r] = to_t<T>(tile[tx][i]);
   }
 }
 
-// Reverse-over-reverse, reverse layer order:  zbar = zpart + abar phi'(z)  (T, both layouts).
+// Reverse-over-reverse, reverse layer order:  zbar = zpart + abar phi'(z)  (T, [rows][ld]).
 template <typename T>
 __global__ void ror_bwd_elem_kernel(int act, const float* __restrict__ zpart,
                                     const float* __restrict__ abar, const float* __restrict__ Z,
-                                    int rows, int cols, T* __restrict__ zb, int ld,
-                                    T* __restrict__ zbT, int ldT) {
+                                    int rows, int cols, T* __restrict__ zb, int ld) {
   pdl_entry();
-  __shared__ float tile[TILE][TILE + 1];
-  const int c0 = blockIdx.x * TILE, r0 = blockIdx.y * TILE;
-  const int tx = threadIdx.x, ty = threadIdx.y;
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int r = r0 + i, c = c0 + tx;
-    float v = 0.f;
+  const int c = blockIdx.x * TILE + threadIdx.x;
+  for (int i = threadIdx.y; i < TILE; i += TROWS) {
+    const int r = blockIdx.y * TILE + i;
     if (r < rows && c < cols) {
       const int64_t o = static_cast<int64_t>(r) * cols + c;
       float f, d1, d2;
       act_eval(act, Z[o], f, d1, d2);
-      v = zpart[o] + abar[o] * d1;
-      zb[static_cast<int64_t>(r) * ld + c] = to_t<T>(v);
+      zb[static_cast<int64_t>(r) * ld + c] = to_t<T>(zpart[o] + abar[o] * d1);
     }
-    tile[i][tx] = v;
-  }
-  __syncthreads();
-  for (int i = ty; i < TILE; i += TROWS) {
-    const int c = c0 + i, r = r0 + tx;
-    if (zbT && c < cols && r < rows) zbT[static_cast<int64_t>(c) * ldT + r] = to_t<T>(tile[tx][i]);
   }
 }
 
@@ -595,20 +548,6 @@ __global__ void fill_kernel(float* p, int64_t n, float v) {
 }
 
 }  // namespace
-
-template <typename T>
-void transpose(const T* X, int rows, int cols, int ld, T* XT, int ldT, cudaStream_t s) {
-  if (rows <= 0 || cols <= 0) return;
-  dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE);
-  launch_k(transpose_kernel<T>, dim3(grid), dim3(TILE, TROWS), 0, s, X, rows, cols, ld, XT, ldT);
-}
-
-template <typename T>
-void fill_rows(const RowFill& f, int cols, cudaStream_t s) {
-  if (f.n <= 0 || cols <= 0) return;
-  dim3 grid((cols + 255) / 256, f.n);
-  launch_k(fill_rows_kernel<T>, dim3(grid), dim3(256), 0, s, f, cols);
-}
 
 template <typename T>
 void fill_cols(const ColFill& f, int rows, cudaStream_t s) {
@@ -660,20 +599,20 @@ void layer_update(const LayerTable& tab, const LayerUpdArgs& args, cudaStream_t 
 
 template <typename T>
 void ror_fwd_elem(int act, const float* dzbar, const float* Z, const float* dA, int rows, int cols,
-                  T* dab, int ld, T* dabT, int ldT, float* zpart, cudaStream_t s) {
+                  T* dab, int ld, float* zpart, cudaStream_t s) {
   if (rows <= 0 || cols <= 0) return;
   dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE);
-  launch_k(ror_fwd_elem_kernel<T>, dim3(grid), dim3(TILE, TROWS), 0, s, act, dzbar, Z, dA, rows, cols, dab, ld,
-                                                             dabT, ldT, zpart);
+  launch_k(ror_fwd_elem_kernel<T>, dim3(grid), dim3(TILE, TROWS), 0, s, act, dzbar, Z, dA, rows,
+           cols, dab, ld, zpart);
 }
 
 template <typename T>
 void ror_bwd_elem(int act, const float* zpart, const float* abar, const float* Z, int rows,
-                  int cols, T* zb, int ld, T* zbT, int ldT, cudaStream_t s) {
+                  int cols, T* zb, int ld, cudaStream_t s) {
   if (rows <= 0 || cols <= 0) return;
   dim3 grid((cols + TILE - 1) / TILE, (rows + TILE - 1) / TILE);
-  launch_k(ror_bwd_elem_kernel<T>, dim3(grid), dim3(TILE, TROWS), 0, s, act, zpart, abar, Z, rows, cols, zb, ld,
-                                                             zbT, ldT);
+  launch_k(ror_bwd_elem_kernel<T>, dim3(grid), dim3(TILE, TROWS), 0, s, act, zpart, abar, Z, rows,
+           cols, zb, ld);
 }
 
 void fill(float* p, int64_t n, float v, cudaStream_t s) {
@@ -684,15 +623,13 @@ void fill(float* p, int64_t n, float v, cudaStream_t s) {
 }
 
 #define MF_INST(T)                                                                 \
-  template void transpose<T>(const T*, int, int, int, T*, int, cudaStream_t);     \
-  template void fill_rows<T>(const RowFill&, int, cudaStream_t);                  \
   template void fill_cols<T>(const ColFill&, int, cudaStream_t);                  \
   template void loss_seed<T>(const LossArgs&, cudaStream_t);                      \
   template void layer_update<T>(const LayerTable&, const LayerUpdArgs&, cudaStream_t);        \
   template void ror_fwd_elem<T>(int, const float*, const float*, const float*, int, int, T*, int, \
-                                T*, int, float*, cudaStream_t);                                   \
+                                float*, cudaStream_t);                                            \
   template void ror_bwd_elem<T>(int, const float*, const float*, const float*, int, int, T*, int,  \
-                                T*, int, cudaStream_t);
+                                cudaStream_t);
 MF_INST(float)
 MF_INST(__nv_bfloat16)
 #undef MF_INST

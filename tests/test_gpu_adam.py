@@ -33,6 +33,9 @@ FP32 = {
                                   B_outer=6, meta_kind=EX | SLR, optimizer="adam",
                                   adam_eps=1e-6, noise_std=0.1,
                                   extra={"scalar_loglr": math.log(0.01)}),
+    "ex_plr": synth.Workload("a_explr", [5, 7, 3], "tanh", "squared", "fp32", B=5, T=3,
+                             B_outer=4, meta_kind=EX | PLR, optimizer="adam", adam_eps=1e-3,
+                             loglr_mean=math.log(0.01), loglr_std=0.1, noise_std=0.1),
     "multi_tile": synth.Workload("a_mt", [40, 136, 70, 3], "tanh", "squared", "fp32", B=90, T=3,
                                  B_outer=70, alpha=0.005, optimizer="adam", adam_eps=1e-3,
                                  noise_std=0.1),

@@ -28,6 +28,11 @@ FP32_CASES = {
                                       noise_std=0.1, extra={"scalar_loglr": math.log(0.3)}),
     "fp32_multi_tile": synth.Workload("fp32_multi_tile", [40, 136, 70, 3], "tanh", "squared",
                                       "fp32", B=90, T=3, B_outer=70, alpha=0.2, noise_std=0.1),
+    # weight logits and per-parameter log-lrs together: d eta_lr starts T*B = 15 floats into
+    # eta, so the fused update takes its element-wise (unaligned) path
+    "tiny_ex_plr_mom": synth.Workload("tiny_ex_plr_mom", [5, 7, 3], "tanh", "squared", "fp32",
+                                      B=5, T=3, B_outer=4, momentum=0.5, meta_kind=EX | PLR,
+                                      loglr_mean=math.log(0.1), loglr_std=0.1, noise_std=0.1),
 }
 
 BF16_CASES = {
