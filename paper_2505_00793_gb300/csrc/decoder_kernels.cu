@@ -385,6 +385,21 @@ __global__ void softmax_bwd_kernel(int S, int rows, const T* __restrict__ P,
 
 // Next-token cross-entropy row statistics, one block per token row r = b S + s, target
 // ids[b][s+1]:  lse, l = lse - f_y, l' = p.f' - f'_y (with p = softmax(f)).
+// Running softmax statistics (max m, sum of exp(f - m), sum of exp(f - m) f'), merged
+// exactly: rescale both sums to the larger max.
+struct SoftStat {
+  float m, s, t;
+};
+__device__ __forceinline__ SoftStat soft_merge(SoftStat a, SoftStat b) {
+  const float M = fmaxf(a.m, b.m);
+  if (M == -INFINITY) return a;
+  const float ea = expf(a.m - M), eb = expf(b.m - M);
+  return {M, a.s * ea + b.s * eb, a.t * ea + b.t * eb};
+}
+
+// Next-token CE statistics of one token row in one pass over the logits (and their
+// tangent): lse = m + log s, pf = sum_c p_c f'_c = t / s, then l = lse - f_y and
+// l' = pf - f'_y.  Fixed reduction order (lanes, then warps), so results are deterministic.
 __global__ void ce_stats_kernel(int S, int V, const int* __restrict__ ids,
                                 const float* __restrict__ F, const float* __restrict__ Fd,
                                 float* __restrict__ lse, float* __restrict__ l,
@@ -398,37 +413,46 @@ __global__ void ce_stats_kernel(int S, int V, const int* __restrict__ ids,
     y = 0;
   }
   const float* f = F + static_cast<int64_t>(r) * V;
-  __shared__ float red[32];
-  float mx = -INFINITY;
-  for (int c = threadIdx.x; c < V; c += blockDim.x) mx = fmaxf(mx, f[c]);
-  mx = warp_max(mx);
+  const float* fd = Fd ? Fd + static_cast<int64_t>(r) * V : nullptr;
+  SoftStat st{-INFINITY, 0.f, 0.f};
+  auto add = [&](float x, float xd) {
+    if (x > st.m) {
+      const float sc = expf(st.m - x);
+      st.s *= sc;
+      st.t *= sc;
+      st.m = x;
+    }
+    const float e = expf(x - st.m);
+    st.s += e;
+    st.t += e * xd;
+  };
+  // rows are V floats with V a multiple of 8 (validated), so float4 loads stay aligned
+  for (int c = threadIdx.x * 4; c < V; c += blockDim.x * 4) {
+    const float4 x = *reinterpret_cast<const float4*>(f + c);
+    float4 xd = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (fd) xd = *reinterpret_cast<const float4*>(fd + c);
+    add(x.x, xd.x); add(x.y, xd.y); add(x.z, xd.z); add(x.w, xd.w);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const SoftStat q{__shfl_xor_sync(0xffffffffu, st.m, o), __shfl_xor_sync(0xffffffffu, st.s, o),
+                     __shfl_xor_sync(0xffffffffu, st.t, o)};
+    st = soft_merge(st, q);
+  }
+  __shared__ SoftStat red[32];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
-  if (lane == 0) red[w] = mx;
+  if (lane == 0) red[w] = st;
   __syncthreads();
-  if (w == 0) {
-    float v = lane < nw ? red[lane] : -INFINITY;
-    v = warp_max(v);
-    if (lane == 0) red[0] = v;
-  }
-  __syncthreads();
-  mx = red[0];
-  __syncthreads();
-  float se = 0.f;
-  for (int c = threadIdx.x; c < V; c += blockDim.x) se += expf(f[c] - mx);
-  const float2 a = block_sum2(se, 0.f);
-  const float lz = mx + logf(a.x);
-  float pfd = 0.f;
-  if (Fd) {
-    const float* fd = Fd + static_cast<int64_t>(r) * V;
-    for (int c = threadIdx.x; c < V; c += blockDim.x) pfd += expf(f[c] - lz) * fd[c];
-  }
-  const float2 bsum = block_sum2(pfd, 0.f);
   if (threadIdx.x == 0) {
+    SoftStat tot = red[0];
+    for (int k = 1; k < nw; ++k) tot = soft_merge(tot, red[k]);
+    const float lz = tot.m + logf(tot.s);
     lse[r] = lz;
     l[r] = lz - f[y];
-    if (Fd) {
-      pf[r] = bsum.x;
-      ld[r] = bsum.x - Fd[static_cast<int64_t>(r) * V + y];
+    if (fd) {
+      const float p_f = tot.t / tot.s;
+      pf[r] = p_f;
+      ld[r] = p_f - fd[y];
     }
   }
 }
@@ -581,6 +605,18 @@ __global__ void __launch_bounds__(256) embed_bwd_kernel(int d, const int* __rest
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r0 = a + (w * cnt) / 8, r1 = a + ((w + 1) * cnt) / 8;
   const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (cnt == 0) {   // an id absent from the batch (most of a large vocabulary): zero rows
+    for (int c = threadIdx.x * 4; c < d; c += 256 * 4) {
+      for (int which = 0; which < 2; ++which) {
+        float* out = which == 0 ? dE : dEd;
+        if (!out) continue;
+        float* dst = out + static_cast<int64_t>(v) * d + c;
+        if (vec_out) *reinterpret_cast<float4*>(dst) = zero;
+        else { dst[0] = 0.f; dst[1] = 0.f; dst[2] = 0.f; dst[3] = 0.f; }
+      }
+    }
+    return;
+  }
   for (int g0 = 0; g0 < d; g0 += NC * 128) {
     float4 acc[NC], dacc[NC];
 #pragma unroll

@@ -10,6 +10,8 @@ still move far more than the 129 MB L2 per launch:
 * deep_4k_adam  the same with the Adam inner optimiser
 * decoder_small the bench's 6 x d512 decoder (row kernels: RMSNorm, RoPE, softmax, CE)
 * toy           the motivating example, M = 8 (chain loss kernels), either HVP mode
+* decoder_s1024 two blocks of the larger decoder (d 1024, 16 heads, S = 1024), two
+                sequences: the fused attention at the larger decoder's sequence length
 """
 from __future__ import annotations
 
@@ -28,6 +30,9 @@ def case(name: str):
                                      loglr_mean=math.log(1e-4))
     if name in ("decoder_small", "toy"):
         return synth.WORKLOADS[name]
+    if name == "decoder_s1024":
+        return synth.decoder("decoder_s1024", 1024, 16, 4096, 2, 32768, 1024, B=2, T=2,
+                             B_outer=2, alpha=1e-3)
     raise ValueError(name)
 
 
@@ -37,7 +42,8 @@ def main() -> None:
 
     ap = argparse.ArgumentParser()
     ap.add_argument("--case", required=True,
-                    choices=["deep_4k", "deep_4k_adam", "decoder_small", "toy"])
+                    choices=["deep_4k", "deep_4k_adam", "decoder_small", "toy",
+                             "decoder_s1024"])
     ap.add_argument("--calls", type=int, default=3)
     ap.add_argument("--hvp-mode", type=int, default=0)
     args = ap.parse_args()
