@@ -76,8 +76,11 @@ cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why) {
       pair = 1;
       if (bn == 0) bn = a.N > 128 ? 256 : 128;
     } else if (g_pair_mode == 1 && bn == 0 && a.M >= 256) {
-      if (pairs_m * ((a.N + 255) / 256) >= 76) { pair = 1; bn = 256; }
-      else if (pairs_m * ((a.N + 127) / 128) >= 60) { pair = 1; bn = 128; }
+      // 256-wide pairs when they fill a wave of 76 pairs, or when 128-wide pairs would spill
+      // into a second wave while the 256-wide grid still holds 40 or more pairs
+      const int p256 = pairs_m * ((a.N + 255) / 256), p128 = pairs_m * ((a.N + 127) / 128);
+      if (p256 >= 76 || (p128 > 76 && p256 >= 40)) { pair = 1; bn = 256; }
+      else if (p128 >= 60) { pair = 1; bn = 128; }
     }
   }
   if (bn == 0) {
@@ -85,8 +88,12 @@ cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why) {
     // would leave most SMs idle (small-batch layers), else 128 (dual) or 256 columns.
     const bool dual = a.terms & (T_C1_A1B0 | T_C1_A0B1);
     const int tiles_m = ((a.M + 127) / 128) * nbatch;
+    const int nkb = (a.K + 63) / 64;
     if (a.N <= 16) bn = 16;
     else if (a.N <= 32) bn = 32;
+    // Long K (weight products over thousands of tokens): 128-wide tiles stage twice the
+    // MMA work per byte of 64-wide ones, and the cluster K split fills the GPU instead.
+    else if (a.N > 64 && nkb >= 32) bn = 128;
     else if (a.N <= 64 || tiles_m * ((a.N + 127) / 128) < 76) bn = 64;
     else if (dual || tiles_m * ((a.N + 255) / 256) < 152) bn = 128;
     else bn = 256;
