@@ -121,6 +121,154 @@ __global__ void rmsnorm_fwd_kernel(int d, float eps, const float* __restrict__ x
 // Dual RMSNorm backward, accumulated into the residual gradient:
 //   dx += r (dn - n c),  c = mean(dn n),  dn = dy g
 //   dx' += r' (dn - n c) + r (dn' - n' c - n c'),  dn' = dy' g + dy g',  c' = mean(dn' n + dn n')
+// Warp-per-row versions of the RMSNorm forward and backward (eight rows per block, float4
+// access, shuffle reductions), used when every vector is 16-byte aligned and d is a multiple
+// of 4; same arithmetic as the block-per-row kernels above and below.
+__device__ __forceinline__ float warp_sum_all(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+template <typename T>
+__device__ __forceinline__ void st_t4(T* p, float a, float b, float c, float d) {
+  if constexpr (sizeof(T) == 2) {
+    __nv_bfloat162 lo = __floats2bfloat162_rn(a, b), hi = __floats2bfloat162_rn(c, d);
+    uint2 v;
+    v.x = *reinterpret_cast<uint32_t*>(&lo);
+    v.y = *reinterpret_cast<uint32_t*>(&hi);
+    *reinterpret_cast<uint2*>(p) = v;
+  } else {
+    *reinterpret_cast<float4*>(p) = make_float4(a, b, c, d);
+  }
+}
+
+__device__ __forceinline__ float4 ld4f(const float* p) { return *reinterpret_cast<const float4*>(p); }
+
+template <typename T>
+__global__ void __launch_bounds__(256) rmsnorm_fwd_warp_kernel(
+    int N, int d, float eps, const float* __restrict__ x_in, const float* __restrict__ y,
+    const float* __restrict__ xd_in, const float* __restrict__ yd, const float* __restrict__ g,
+    const float* __restrict__ gd, float* __restrict__ x_out, float* __restrict__ xd_out,
+    float* __restrict__ rr, float* __restrict__ rrd, T* __restrict__ h, T* __restrict__ hd,
+    int ldh) {
+  pdl_entry();
+  const int r = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (r >= N) return;
+  const int64_t o = static_cast<int64_t>(r) * d;
+  const bool dual = xd_in != nullptr;
+  float s2 = 0.f, s1 = 0.f;
+  for (int c = lane * 4; c < d; c += 128) {
+    float4 v = ld4f(x_in + o + c);
+    if (y) { const float4 t = ld4f(y + o + c); v.x += t.x; v.y += t.y; v.z += t.z; v.w += t.w; }
+    *reinterpret_cast<float4*>(x_out + o + c) = v;
+    s2 += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+    if (dual) {
+      float4 vd = ld4f(xd_in + o + c);
+      if (yd) { const float4 t = ld4f(yd + o + c); vd.x += t.x; vd.y += t.y; vd.z += t.z; vd.w += t.w; }
+      *reinterpret_cast<float4*>(xd_out + o + c) = vd;
+      s1 += v.x * vd.x + v.y * vd.y + v.z * vd.z + v.w * vd.w;
+    }
+  }
+  s2 = warp_sum_all(s2);
+  s1 = warp_sum_all(s1);
+  const float inv_d = 1.f / static_cast<float>(d);
+  const float rs = rsqrtf(s2 * inv_d + eps);
+  const float rsd = -rs * rs * rs * s1 * inv_d;
+  if (lane == 0) {
+    rr[r] = rs;
+    if (dual) rrd[r] = rsd;
+  }
+  const int64_t oh = static_cast<int64_t>(r) * ldh;
+  for (int c = lane * 4; c < d; c += 128) {
+    const float4 v = ld4f(x_out + o + c), gg = ld4f(g + c);
+    const float n0 = v.x * rs, n1 = v.y * rs, n2 = v.z * rs, n3 = v.w * rs;
+    st_t4<T>(h + oh + c, gg.x * n0, gg.y * n1, gg.z * n2, gg.w * n3);
+    if (dual) {
+      const float4 vd = ld4f(xd_out + o + c), ggd = ld4f(gd + c);
+      const float m0 = vd.x * rs + v.x * rsd, m1 = vd.y * rs + v.y * rsd;
+      const float m2 = vd.z * rs + v.z * rsd, m3 = vd.w * rs + v.w * rsd;
+      st_t4<T>(hd + oh + c, ggd.x * n0 + gg.x * m0, ggd.y * n1 + gg.y * m1,
+               ggd.z * n2 + gg.z * m2, ggd.w * n3 + gg.w * m3);
+    }
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) rmsnorm_bwd_warp_kernel(
+    int N, int d, const float* __restrict__ x, const float* __restrict__ xd,
+    const float* __restrict__ rr, const float* __restrict__ rrd, const float* __restrict__ g,
+    const float* __restrict__ gd, const float* __restrict__ dy, const float* __restrict__ dyd,
+    float* __restrict__ dx, float* __restrict__ dxd, T* __restrict__ dxb, T* __restrict__ dxdb) {
+  pdl_entry();
+  const int r = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (r >= N) return;
+  const int64_t o = static_cast<int64_t>(r) * d;
+  const bool dual = dyd != nullptr;
+  const float rs = rr[r];
+  const float rsd = dual ? rrd[r] : 0.f;
+  float sc = 0.f, scd = 0.f;
+  for (int c = lane * 4; c < d; c += 128) {
+    const float4 xv = ld4f(x + o + c), dv = ld4f(dy + o + c), gg = ld4f(g + c);
+    const float xs[4] = {xv.x, xv.y, xv.z, xv.w}, ds[4] = {dv.x, dv.y, dv.z, dv.w};
+    const float gs[4] = {gg.x, gg.y, gg.z, gg.w};
+    float xds[4] = {0.f, 0.f, 0.f, 0.f}, dds[4] = {0.f, 0.f, 0.f, 0.f}, gds[4] = {0.f, 0.f, 0.f, 0.f};
+    if (dual) {
+      const float4 a = ld4f(xd + o + c), b = ld4f(dyd + o + c), e = ld4f(gd + c);
+      xds[0] = a.x; xds[1] = a.y; xds[2] = a.z; xds[3] = a.w;
+      dds[0] = b.x; dds[1] = b.y; dds[2] = b.z; dds[3] = b.w;
+      gds[0] = e.x; gds[1] = e.y; gds[2] = e.z; gds[3] = e.w;
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float n = xs[j] * rs;
+      const float dn = ds[j] * gs[j];
+      sc += dn * n;
+      if (dual) {
+        const float nd = xds[j] * rs + xs[j] * rsd;
+        const float dnd = dds[j] * gs[j] + ds[j] * gds[j];
+        scd += dnd * n + dn * nd;
+      }
+    }
+  }
+  sc = warp_sum_all(sc);
+  scd = warp_sum_all(scd);
+  const float inv_d = 1.f / static_cast<float>(d);
+  const float cc = sc * inv_d, ccd = scd * inv_d;
+  for (int c = lane * 4; c < d; c += 128) {
+    const float4 xv = ld4f(x + o + c), dv = ld4f(dy + o + c), gg = ld4f(g + c), ov = ld4f(dx + o + c);
+    const float xs[4] = {xv.x, xv.y, xv.z, xv.w}, ds[4] = {dv.x, dv.y, dv.z, dv.w};
+    const float gs[4] = {gg.x, gg.y, gg.z, gg.w}, os[4] = {ov.x, ov.y, ov.z, ov.w};
+    float out[4], outd[4] = {0.f, 0.f, 0.f, 0.f};
+    float xds[4] = {0.f, 0.f, 0.f, 0.f}, dds[4] = {0.f, 0.f, 0.f, 0.f}, gds[4] = {0.f, 0.f, 0.f, 0.f};
+    float ods[4] = {0.f, 0.f, 0.f, 0.f};
+    if (dual) {
+      const float4 a = ld4f(xd + o + c), b = ld4f(dyd + o + c), e = ld4f(gd + c), f = ld4f(dxd + o + c);
+      xds[0] = a.x; xds[1] = a.y; xds[2] = a.z; xds[3] = a.w;
+      dds[0] = b.x; dds[1] = b.y; dds[2] = b.z; dds[3] = b.w;
+      gds[0] = e.x; gds[1] = e.y; gds[2] = e.z; gds[3] = e.w;
+      ods[0] = f.x; ods[1] = f.y; ods[2] = f.z; ods[3] = f.w;
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float n = xs[j] * rs;
+      const float dn = ds[j] * gs[j];
+      out[j] = os[j] + rs * (dn - n * cc);
+      if (dual) {
+        const float nd = xds[j] * rs + xs[j] * rsd;
+        const float dnd = dds[j] * gs[j] + ds[j] * gds[j];
+        outd[j] = ods[j] + rsd * (dn - n * cc) + rs * (dnd - nd * cc - n * ccd);
+      }
+    }
+    *reinterpret_cast<float4*>(dx + o + c) = make_float4(out[0], out[1], out[2], out[3]);
+    if (dxb) st_t4<T>(dxb + o + c, out[0], out[1], out[2], out[3]);
+    if (dual) {
+      *reinterpret_cast<float4*>(dxd + o + c) = make_float4(outd[0], outd[1], outd[2], outd[3]);
+      if (dxdb) st_t4<T>(dxdb + o + c, outd[0], outd[1], outd[2], outd[3]);
+    }
+  }
+}
+
 template <typename T>
 __global__ void rmsnorm_bwd_kernel(int d, const float* __restrict__ x, const float* __restrict__ xd,
                                    const float* __restrict__ rr, const float* __restrict__ rrd,
@@ -705,6 +853,16 @@ template <typename T>
 void dec_rmsnorm_fwd(int N, int d, float eps, const float* x_in, const float* y, const float* xd_in,
                      const float* yd, const float* g, const float* gd, float* x_out, float* xd_out,
                      float* r, float* rd, T* h, T* hd, int ldh, cudaStream_t s) {
+  uintptr_t any = reinterpret_cast<uintptr_t>(x_in) | reinterpret_cast<uintptr_t>(y) |
+                  reinterpret_cast<uintptr_t>(xd_in) | reinterpret_cast<uintptr_t>(yd) |
+                  reinterpret_cast<uintptr_t>(g) | reinterpret_cast<uintptr_t>(gd) |
+                  reinterpret_cast<uintptr_t>(x_out) | reinterpret_cast<uintptr_t>(xd_out) |
+                  reinterpret_cast<uintptr_t>(h) | reinterpret_cast<uintptr_t>(hd);
+  if ((any & 15) == 0 && (d & 3) == 0 && (ldh & 7) == 0) {
+    launch_k(rmsnorm_fwd_warp_kernel<T>, dim3((N + 7) / 8), dim3(256), 0, s, N, d, eps, x_in, y,
+             xd_in, yd, g, gd, x_out, xd_out, r, rd, h, hd, ldh);
+    return;
+  }
   launch_k(rmsnorm_fwd_kernel<T>, dim3(N), dim3(256), 0, s, d, eps, x_in, y, xd_in, yd, g, gd, x_out, xd_out, r, rd,
                                           h, hd, ldh);
 }
@@ -713,6 +871,16 @@ template <typename T>
 void dec_rmsnorm_bwd(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
                      const float* g, const float* gd, const float* dy, const float* dyd, float* dx,
                      float* dxd, cudaStream_t s, T* dxb, T* dxdb) {
+  uintptr_t any = reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(xd) |
+                  reinterpret_cast<uintptr_t>(g) | reinterpret_cast<uintptr_t>(gd) |
+                  reinterpret_cast<uintptr_t>(dy) | reinterpret_cast<uintptr_t>(dyd) |
+                  reinterpret_cast<uintptr_t>(dx) | reinterpret_cast<uintptr_t>(dxd) |
+                  reinterpret_cast<uintptr_t>(dxb) | reinterpret_cast<uintptr_t>(dxdb);
+  if ((any & 15) == 0 && (d & 3) == 0) {
+    launch_k(rmsnorm_bwd_warp_kernel<T>, dim3((N + 7) / 8), dim3(256), 0, s, N, d, x, xd, r, rd, g,
+             gd, dy, dyd, dx, dxd, dxb, dxdb);
+    return;
+  }
   launch_k(rmsnorm_bwd_kernel<T>, dim3(N), dim3(256), 0, s, d, x, xd, r, rd, g, gd, dy, dyd, dx, dxd,
            dxb, dxdb);
 }
