@@ -357,3 +357,24 @@ def test_toy_zero_steps_is_linear_closed_form():
         tb = tb - w.alpha * H @ tb
     res = om.meta_grad(w, inp)
     assert _rel(res["d_theta0"], tb) < 1e-12
+
+
+def test_oracle_matches_its_golden_values():
+    """The oracle reproduces the values tests/golden/make_oracle_golden.py wrote with it (a
+    regression anchor for its own arithmetic; the paper prints no worked values)."""
+    import json
+    import os
+    import sys
+    here = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+    sys.path.insert(0, here)
+    import make_oracle_golden as g
+    with open(os.path.join(here, "oracle_golden.json")) as f:
+        gold = json.load(f)
+    assert set(gold) == set(g.CASES)
+    for name, w in g.CASES.items():
+        r = om.meta_grad(w, synth.make_inputs(w))
+        assert abs(r["V"] - gold[name]["V"]) <= 1e-12 * abs(gold[name]["V"])
+        for key in ("d_eta", "d_theta0"):
+            ref = np.array(gold[name][key])
+            if ref.size:
+                assert _rel(r[key], ref) < 1e-12, (name, key)
