@@ -47,12 +47,12 @@ __device__ __forceinline__ void act_eval(int act, float z, float& f, float& d1, 
 // Per-element epilogue of a dual GEMM (shared by the tensor-core and SIMT kernels).
 //  EPI_STORE:   C0 = acc0 + bias0, C1 = acc1 + bias1.
 //  EPI_ACT_FWD: z = acc0 + bias0, z' = acc1 + bias1 -> C0 = z, C1 = z' (float32),
-//               a = phi(z), a' = phi'(z) z'  -> A, Ad (row-major) and AT, AdT (transposed).
+//               a = phi(z), a' = phi'(z) z'  -> A, Ad (row-major).
 //  EPI_ACT_BWD: da = acc0, da' = acc1, z, z' read from Z, Zd ->
-//               dz = phi'(z) da, dz' = phi''(z) z' da + phi'(z) da'  -> A, Ad, AT, AdT.
+//               dz = phi'(z) da, dz' = phi''(z) z' da + phi'(z) da'  -> A, Ad.
 struct EpiOut {
   float c0, c1;     // float32 outputs for C0 / C1
-  float o0, o1;     // values for A / Ad (and their transposes)
+  float o0, o1;     // values for A / Ad
 };
 
 __device__ __forceinline__ EpiOut epi_eval(const EpiParams& e, int m, int n, float acc0,

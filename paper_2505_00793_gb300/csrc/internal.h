@@ -24,12 +24,12 @@ enum EpiMode : int { EPI_STORE = 0, EPI_ACT_FWD = 1, EPI_ACT_BWD = 2 };
 
 // Fused epilogue of a dual GEMM (see device_math.cuh for the element rules).  The A family
 // outputs have the operand element type of the GEMM backend (bf16 for tensor cores, float
-// for the SIMT path): A/Ad row-major [M][lda], AT/AdT transposed [N][ldt]; each nullable.
+// for the SIMT path): A/Ad row-major [M][lda], each nullable.  The next GEMM reads them in
+// place (K- or MN-major), so no transposed copy is written.
 struct EpiParams {
   int mode = EPI_STORE;
   int act = ACT_IDENT;
   void* A = nullptr; void* Ad = nullptr; int lda = 0;
-  void* AT = nullptr; void* AdT = nullptr; int ldt = 0;
   const float* Z = nullptr; const float* Zd = nullptr; int ldz = 0;   // EPI_ACT_BWD inputs
 };
 

@@ -87,8 +87,6 @@ __global__ void __launch_bounds__(256) simt_dual_gemm_kernel(SimtParams p) {
   const EpiParams& e = p.epi;
   float* A = static_cast<float*>(e.A);
   float* Ad = static_cast<float*>(e.Ad);
-  float* AT = static_cast<float*>(e.AT);
-  float* AdT = static_cast<float*>(e.AdT);
   for (int i = 0; i < 4; ++i) {
     const int gm = m0 + ty * 4 + i;
     if (gm >= p.M) continue;
@@ -100,11 +98,7 @@ __global__ void __launch_bounds__(256) simt_dual_gemm_kernel(SimtParams p) {
       if (p.C[1] && dual) p.C[1][static_cast<int64_t>(gm) * p.ldc[1] + gn] = o.c1;
       if (e.mode != EPI_STORE) {
         if (A) A[static_cast<int64_t>(gm) * e.lda + gn] = o.o0;
-        if (AT) AT[static_cast<int64_t>(gn) * e.ldt + gm] = o.o0;
-        if (dual) {
-          if (Ad) Ad[static_cast<int64_t>(gm) * e.lda + gn] = o.o1;
-          if (AdT) AdT[static_cast<int64_t>(gn) * e.ldt + gm] = o.o1;
-        }
+        if (dual && Ad) Ad[static_cast<int64_t>(gm) * e.lda + gn] = o.o1;
       }
     }
   }

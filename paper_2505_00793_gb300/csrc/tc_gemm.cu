@@ -7,16 +7,19 @@
 // which gives the primal-only layer, the input layer (A' = 0) and the weight-tangent
 // product [a'; a]^T [dz; dz'] from the same kernel.
 //
-// CTA = 6 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues tcgen05.mma from
-// one thread, warps 2..5 drain the accumulators (tcgen05.ld) and run the fused epilogue
-// (bias, activation and its derivatives, bf16 operand stores for the next GEMM in both
-// row-major and transposed layouts).  Tile 128 x BN x (64 KA) (bf16, 128-byte swizzle, KA
-// swizzle atoms per pipeline stage), multi-stage mbarrier pipeline.  Row-major outputs are
-// staged in swizzled shared memory and written by per-warp TMA stores (coalesced); the
-// transposed operand copies are written directly (consecutive lanes = consecutive rows).  GEMMs with few output tiles split K across a thread-block
-// cluster of S CTAs; the partial accumulators meet in distributed shared memory and each
-// CTA reduces 128/S rows in a fixed order (deterministic).  Every mbarrier wait is bounded;
-// on expiry the CTA records DEV_TIMEOUT and carries on to the end without further waits.
+// One-SM tiles: a CTA of 18 warps. Warp 0 issues the TMA loads, warp 1 owns TMEM and issues
+// tcgen05.mma from one thread, and sixteen epilogue warps drain the accumulators
+// (tcgen05.ld) and run the fused epilogue: bias, activation and its derivatives, and the
+// bf16 operand stores that the next GEMM reads in place. Warps sharing a TMEM lane quadrant
+// split its columns. Tile 128 x BN x (64 KA) (bf16, 128-byte swizzle, KA swizzle atoms per
+// pipeline stage) with a multi-stage mbarrier pipeline. Operands are K-major or MN-major
+// (64-row boxes), so no operand is ever stored transposed. Each product term (MMA) rotates over
+// up to four TMEM accumulator blocks so that dependent MMAs do not serialise. CTA-pair tiles
+// (cta_group::2, 256 rows) serve GEMMs whose pair grid fills the GPU. GEMMs with few output
+// tiles split K across a thread-block cluster of S CTAs: the partial accumulators meet in
+// distributed shared memory, and each CTA reduces 128/S rows in a fixed order, so results are
+// deterministic. Every mbarrier wait is bounded; on expiry the CTA records DEV_TIMEOUT and
+// carries on to the end without further waits.
 #include "tc_gemm_impl.cuh"
 
 namespace mf {
@@ -56,13 +59,13 @@ cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why) {
       }
   }
   if (a.epi.mode != EPI_STORE) {
-    const void* outs[4] = {a.epi.A, a.epi.Ad, a.epi.AT, a.epi.AdT};
-    for (int i = 0; i < 4; ++i)
+    const void* outs[2] = {a.epi.A, a.epi.Ad};
+    for (int i = 0; i < 2; ++i)
       if (outs[i] && (reinterpret_cast<uintptr_t>(outs[i]) & 15)) {
         *why = "epilogue outputs must be 16-byte aligned";
         return cudaErrorInvalidValue;
       }
-    if ((a.epi.lda & 7) || (a.epi.ldt & 7)) {
+    if (a.epi.lda & 7) {
       *why = "epilogue leading dimensions must be multiples of 8";
       return cudaErrorInvalidValue;
     }

@@ -7,16 +7,19 @@
 // which gives the primal-only layer, the input layer (A' = 0) and the weight-tangent
 // product [a'; a]^T [dz; dz'] from the same kernel.
 //
-// CTA = 6 warps: warp 0 issues TMA loads, warp 1 owns TMEM and issues tcgen05.mma from
-// one thread, warps 2..5 drain the accumulators (tcgen05.ld) and run the fused epilogue
-// (bias, activation and its derivatives, bf16 operand stores for the next GEMM in both
-// row-major and transposed layouts).  Tile 128 x BN x (64 KA) (bf16, 128-byte swizzle, KA
-// swizzle atoms per pipeline stage), multi-stage mbarrier pipeline.  Row-major outputs are
-// staged in swizzled shared memory and written by per-warp TMA stores (coalesced); the
-// transposed operand copies are written directly (consecutive lanes = consecutive rows).  GEMMs with few output tiles split K across a thread-block
-// cluster of S CTAs; the partial accumulators meet in distributed shared memory and each
-// CTA reduces 128/S rows in a fixed order (deterministic).  Every mbarrier wait is bounded;
-// on expiry the CTA records DEV_TIMEOUT and carries on to the end without further waits.
+// One-SM tiles: a CTA of 18 warps. Warp 0 issues the TMA loads, warp 1 owns TMEM and issues
+// tcgen05.mma from one thread, and sixteen epilogue warps drain the accumulators
+// (tcgen05.ld) and run the fused epilogue: bias, activation and its derivatives, and the
+// bf16 operand stores that the next GEMM reads in place. Warps sharing a TMEM lane quadrant
+// split its columns. Tile 128 x BN x (64 KA) (bf16, 128-byte swizzle, KA swizzle atoms per
+// pipeline stage) with a multi-stage mbarrier pipeline. Operands are K-major or MN-major
+// (64-row boxes), so no operand is ever stored transposed. Each product term (MMA) rotates over
+// up to four TMEM accumulator blocks so that dependent MMAs do not serialise. CTA-pair tiles
+// (cta_group::2, 256 rows) serve GEMMs whose pair grid fills the GPU. GEMMs with few output
+// tiles split K across a thread-block cluster of S CTAs: the partial accumulators meet in
+// distributed shared memory, and each CTA reduces 128/S rows in a fixed order, so results are
+// deterministic. Every mbarrier wait is bounded; on expiry the CTA records DEV_TIMEOUT and
+// carries on to the end without further waits.
 // Implementation of the tcgen05 dual GEMM, included by tc_gemm.cu (plain stores) and by
 // tc_gemm_act.cu (activation epilogues).  The epilogue mode and the activation are template
 // parameters so that each kernel instance carries only its own per-element code.
@@ -245,8 +248,8 @@ __device__ __forceinline__ void epi_bar() {   // the epilogue warps only
   asm volatile("bar.sync 1, %0;" ::"n"(EPI_THREADS) : "memory");
 }
 
-// Row-per-thread epilogue for 16 consecutive columns (no split): float32 outputs, the
-// row-major bf16 operand rows and the transposed bf16 operand columns.
+// Row-per-thread epilogue for 16 consecutive columns (no split): float32 outputs and the
+// row-major bf16 operand rows.
 template <int MODE, int ACT>
 __device__ __forceinline__ void epilogue16(const TcParams& p, int row, int col0,
                                            const float (&v0)[16], const float (&v1)[16],
@@ -308,19 +311,6 @@ __device__ __forceinline__ void epilogue16(const TcParams& p, int row, int col0,
       }
     }
   }
-  // transposed operand copies: for each column, the 32 lanes of the warp write 32
-  // consecutive rows (coalesced)
-  __nv_bfloat16* AT = static_cast<__nv_bfloat16*>(e.AT);
-  __nv_bfloat16* AdT = static_cast<__nv_bfloat16*>(e.AdT);
-  if (rowok) {
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      const int n = col0 + j;
-      if (n >= p.N) break;
-      if (AT) AT[static_cast<int64_t>(n) * e.ldt + row] = __float2bfloat16_rn(o0[j]);
-      if (AdT && dual) AdT[static_cast<int64_t>(n) * e.ldt + row] = __float2bfloat16_rn(o1[j]);
-    }
-  }
 }
 
 __device__ __forceinline__ void fence_proxy_async() {
@@ -363,8 +353,6 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
   uint8_t* sA = stg + 4 * STG_F32_BOX;
   uint8_t* sAd = sA + STG_BF16_BOX;
   const int sw = lane & 7;
-  __nv_bfloat16* AT = static_cast<__nv_bfloat16*>(e.AT);
-  __nv_bfloat16* AdT = static_cast<__nv_bfloat16*>(e.AdT);
   for (int c = c_begin; c < c_end; c += 64) {
     if (c > c_begin) {
       if (lane == 0) bulk_wait_read();
@@ -414,16 +402,6 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
           *reinterpret_cast<uint4*>(sAd + lane * 128 + pos) =
               make_uint4(pack_bf16x2(o1[8 * k], o1[8 * k + 1]), pack_bf16x2(o1[8 * k + 2], o1[8 * k + 3]),
                          pack_bf16x2(o1[8 * k + 4], o1[8 * k + 5]), pack_bf16x2(o1[8 * k + 6], o1[8 * k + 7]));
-      }
-      // transposed operand copies, coalesced across the warp's rows
-      if (MODE != EPI_STORE && rowok) {
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const int n = n0 + cc + j;
-          if (n >= p.N) break;
-          if (AT) AT[static_cast<int64_t>(n) * e.ldt + row] = __float2bfloat16_rn(o0[j]);
-          if (AdT && dual) AdT[static_cast<int64_t>(n) * e.ldt + row] = __float2bfloat16_rn(o1[j]);
-        }
       }
     }
     fence_proxy_async();
@@ -793,27 +771,22 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
       }
       epi_bar();
-      // Phase B: fused epilogue, one column per thread, 8-row chunks (the transposed bf16
-      // operand gets one 16-byte store per chunk; row-major stores are coalesced across
-      // consecutive columns)
+      // Phase B: fused epilogue, one column per thread, 8-row chunks (row-major stores are
+      // coalesced across consecutive columns)
       constexpr int CW = BN < EPI_THREADS ? BN : EPI_THREADS;
       const int tpc = EPI_THREADS / CW;          // threads per column
       const EpiParams ep = p.epi;
-      __nv_bfloat16* AT = static_cast<__nv_bfloat16*>(ep.AT);
-      __nv_bfloat16* AdT = static_cast<__nv_bfloat16*>(ep.AdT);
       __nv_bfloat16* A = static_cast<__nv_bfloat16*>(ep.A);
       __nv_bfloat16* Ad = static_cast<__nv_bfloat16*>(ep.Ad);
       for (int col = e % BN; col < BN; col += EPI_THREADS) {
         const int n = n0 + col;
         for (int ch = e / CW; ch * 8 < rows_per; ch += tpc) {
-          float t0[8], t1[8];
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             const int rr = ch * 8 + j;
             const float v0 = R[rr * LDP + col];
             const float v1 = dual ? R[(rows_per + rr) * LDP + col] : 0.f;
             const int m = m0 + r_begin + rr;
-            t0[j] = t1[j] = 0.f;
             if (m < p.M && n < p.N) {
               const EpiOut o = epi_eval_t<MODE, ACT>(ep, m, n, v0, v1, p.bias0, p.bias1, dual);
               if (p.C0) p.C0[static_cast<int64_t>(m) * p.ldc0 + n] = o.c0;
@@ -821,24 +794,6 @@ __global__ void __launch_bounds__(THREADS, 1)
               if (MODE != EPI_STORE) {
                 if (A) A[static_cast<int64_t>(m) * ep.lda + n] = __float2bfloat16_rn(o.o0);
                 if (Ad && dual) Ad[static_cast<int64_t>(m) * ep.lda + n] = __float2bfloat16_rn(o.o1);
-              }
-              t0[j] = o.o0;
-              t1[j] = o.o1;
-            }
-          }
-          if (MODE != EPI_STORE && n < p.N) {
-            const int mb = m0 + r_begin + ch * 8;
-            for (int w = 0; w < 2; ++w) {
-              __nv_bfloat16* X = w == 0 ? AT : AdT;
-              const float* t = w == 0 ? t0 : t1;
-              if (!X || (w == 1 && !dual)) continue;
-              __nv_bfloat16* dst = X + static_cast<int64_t>(n) * ep.ldt + mb;
-              if (mb + 8 <= p.M) {
-                *reinterpret_cast<uint4*>(dst) =
-                    make_uint4(pack_bf16x2(t[0], t[1]), pack_bf16x2(t[2], t[3]),
-                               pack_bf16x2(t[4], t[5]), pack_bf16x2(t[6], t[7]));
-              } else {
-                for (int j = 0; j < 8; ++j) if (mb + j < p.M) dst[j] = __float2bfloat16_rn(t[j]);
               }
             }
           }
