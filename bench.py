@@ -10,9 +10,11 @@ Prints one JSON line (rank 0).  ``--impl reference`` times the CPU float64 oracl
 Multi-GPU runs are independent replicas (weak scaling), one process per GPU under torchrun.
 
 ``--workload`` measures another configuration the same way (deep MLP, the two decoder-only
-transformers, the motivating example of Section 3 with ``--chain-steps M``); ``--hvp-mode rr`` runs the reverse-over-reverse sweep instead of the
-mixed-mode one (MLPs), for the memory comparison.  Those lines skip the CPU baseline unless
-``--cpu-baseline`` is given.
+transformers, the motivating example of Section 3 with ``--chain-steps M``).
+``--hvp-mode rr`` runs the reverse-over-reverse sweep instead of the mixed-mode one, for the
+memory comparison. ``--ckpt-every k`` keeps the theta_t store in segments of k steps, and
+``--optimizer adam`` replaces the workload's SGD / momentum by Adam. Those lines skip the
+CPU baseline unless ``--cpu-baseline`` is given.
 """
 from __future__ import annotations
 
