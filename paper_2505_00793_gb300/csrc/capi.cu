@@ -26,6 +26,11 @@ namespace {
 constexpr size_t ALIGN = 256;
 inline size_t align_up(size_t x, size_t a = ALIGN) { return (x + a - 1) / a * a; }
 inline int ld8(int x) { return (x + 7) / 8 * 8; }
+inline uint32_t float_bits(float f) {
+  uint32_t u;
+  memcpy(&u, &f, sizeof(u));
+  return u;
+}
 
 }  // namespace
 
@@ -1257,12 +1262,12 @@ mf_status mf_inner_rollout(mf_handle h, const mf_loop_desc* lp, const float* the
   uint64_t key = 0x726f6c6cULL;
   for (uint64_t v : {static_cast<uint64_t>(lp->T), static_cast<uint64_t>(lp->B),
                      static_cast<uint64_t>(lp->meta_kind),
-                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->alpha)),
-                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->momentum)),
+                     static_cast<uint64_t>(float_bits(lp->alpha)),
+                     static_cast<uint64_t>(float_bits(lp->momentum)),
                      static_cast<uint64_t>(lp->optimizer),
-                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->beta1)),
-                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->beta2)),
-                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->adam_eps)),
+                     static_cast<uint64_t>(float_bits(lp->beta1)),
+                     static_cast<uint64_t>(float_bits(lp->beta2)),
+                     static_cast<uint64_t>(float_bits(lp->adam_eps)),
                      reinterpret_cast<uint64_t>(theta0), reinterpret_cast<uint64_t>(eta),
                      reinterpret_cast<uint64_t>(inner_x), reinterpret_cast<uint64_t>(inner_y),
                      reinterpret_cast<uint64_t>(thetaT)})
@@ -1324,11 +1329,11 @@ mf_status mf_meta_grad(mf_handle h, const mf_loop_desc* lp, const float* theta0,
                      static_cast<uint64_t>(lp->hvp_mode),
                      static_cast<uint64_t>(make_store(lp).k),
                      static_cast<uint64_t>(lp->optimizer),
-                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->beta1)),
-                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->beta2)),
-                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->adam_eps)),
-                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->alpha)),
-                     static_cast<uint64_t>(*reinterpret_cast<const uint32_t*>(&lp->momentum)),
+                     static_cast<uint64_t>(float_bits(lp->beta1)),
+                     static_cast<uint64_t>(float_bits(lp->beta2)),
+                     static_cast<uint64_t>(float_bits(lp->adam_eps)),
+                     static_cast<uint64_t>(float_bits(lp->alpha)),
+                     static_cast<uint64_t>(float_bits(lp->momentum)),
                      reinterpret_cast<uint64_t>(theta0), reinterpret_cast<uint64_t>(eta),
                      reinterpret_cast<uint64_t>(inner_x), reinterpret_cast<uint64_t>(inner_y),
                      reinterpret_cast<uint64_t>(outer_x), reinterpret_cast<uint64_t>(outer_y),

@@ -820,8 +820,6 @@ __global__ void __launch_bounds__(256) embed_bwd_kernel(int d, const int* __rest
   }
 }
 
-constexpr int TILE = 32, TROWS = 8;
-
 // Row-major cast (with a leading dimension) float32 -> T.
 template <typename T>
 __global__ void cast_rows_kernel(const float* __restrict__ X, int rows, int cols, T* __restrict__ Y,

@@ -297,12 +297,6 @@ __global__ void sum_scaled_kernel(const float* __restrict__ x, int n, float scal
   }
 }
 
-__device__ __forceinline__ float lr_at(const LrArgs& lr, int64_t i) {
-  if (lr.plr) return expf(lr.plr[i]);
-  if (lr.slr) return expf(lr.slr[0]);
-  return lr.alpha;
-}
-
 // Four consecutive parameters per thread, UPD_ELEMS per block, blocks assigned to layers by
 // tab.tile0.  A layer whose offset and width are multiples of 4 moves them as float4 (and
 // its operand copies as four-element stores in one row); others go element by element.
