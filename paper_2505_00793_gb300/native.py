@@ -2,8 +2,10 @@
 
 Argument marshalling only: every step of the meta-gradient runs in the library's CUDA
 kernels.  Functions keep the C names; ``MixFlow`` wraps a handle and takes torch tensors
-(device memory and streams come from PyTorch).  Importing this module raises if the
-library has not been built - there is no fallback implementation.
+(device memory and streams come from PyTorch).  Creating a handle (or any call) raises if
+the library has not been built - there is no fallback implementation.  Tensor arguments are
+checked before the call: a CUDA tensor, contiguous, of the dtype the ABI states; the library
+itself only sees pointers and cannot tell a host pointer or a wrong element type.
 """
 from __future__ import annotations
 
@@ -103,10 +105,33 @@ def lib() -> C.CDLL:
     return _lib
 
 
-def _ptr(t):
+def _dev(t, name, dtype, rows=False):
+    """Device pointer of tensor argument ``name`` (None -> NULL) after checking its dtype,
+    layout (contiguous; with ``rows``, only unit stride along the last axis, the leading
+    dimension being passed separately) and that it lives on a CUDA device."""
     if t is None:
         return None
+    if t.dtype != dtype:
+        raise ValueError(f"{name}: dtype {t.dtype}, expected {dtype}")
+    if rows:
+        if t.dim() != 2 or (t.shape[1] > 1 and t.stride(1) != 1):
+            raise ValueError(f"{name}: expected a 2-D tensor with unit stride along its rows")
+    elif not t.is_contiguous():
+        raise ValueError(f"{name}: expected a contiguous tensor")
+    if not t.is_cuda:
+        raise ValueError(f"{name}: expected a CUDA tensor, got one on {t.device}")
     return C.c_void_p(t.data_ptr())
+
+
+def io_dtypes(desc: mf_model_desc):
+    """torch dtypes of (x, y) for a model: token ids for decoders; for MLPs bf16 or float32
+    inputs (the model's precision) and int32 class labels (cross-entropy) or float32 targets."""
+    import torch
+    if desc.arch == MF_ARCH_DECODER:
+        return torch.int32, torch.int32
+    x = torch.bfloat16 if desc.precision == PRECISIONS["bf16"] else torch.float32
+    y = torch.int32 if desc.loss == LOSSES["ce"] else torch.float32
+    return x, y
 
 
 def _stream(stream):
@@ -154,10 +179,15 @@ def loop_desc_for(w, hvp_mode: int = MF_HVP_MIXED_FOR, ckpt_every: int = 1) -> m
 def mf_dual_gemm_bf16(M, N, K, A0, A1, B0, B1, C0, C1, terms, bias0=None, bias1=None,
                       stream=None):
     """C0/C1 (float32) = selected products of bf16 K-major operands (see mixflow.h)."""
+    import torch
+    bf, f32 = torch.bfloat16, torch.float32
     ld = lambda t: (t.stride(0) if t is not None else 0)
-    st = lib().mf_dual_gemm_bf16(M, N, K, _ptr(A0), ld(A0), _ptr(A1), ld(A1), _ptr(B0), ld(B0),
-                                 _ptr(B1), ld(B1), _ptr(C0), ld(C0), _ptr(bias0), _ptr(C1),
-                                 ld(C1), _ptr(bias1), terms, _stream(stream))
+    st = lib().mf_dual_gemm_bf16(M, N, K, _dev(A0, "A0", bf, True), ld(A0),
+                                 _dev(A1, "A1", bf, True), ld(A1), _dev(B0, "B0", bf, True),
+                                 ld(B0), _dev(B1, "B1", bf, True), ld(B1),
+                                 _dev(C0, "C0", f32, True), ld(C0), _dev(bias0, "bias0", f32),
+                                 _dev(C1, "C1", f32, True), ld(C1), _dev(bias1, "bias1", f32),
+                                 terms, _stream(stream))
     if st != 0:
         raise MixflowError(st, "mf_dual_gemm_bf16")
 
@@ -173,6 +203,7 @@ class MixFlow:
         if st != 0:
             raise MixflowError(st, "mf_create")
         self.h = h
+        self.x_dtype, self.y_dtype = io_dtypes(desc)
 
     @classmethod
     def for_workload(cls, w):
@@ -210,20 +241,35 @@ class MixFlow:
 
     def meta_grad(self, loop, theta0, eta, inner_x, inner_y, outer_x, outer_y, d_eta,
                   d_theta0=None, outer_loss=None, stream=None):
-        st = self._lib.mf_meta_grad(self.h, C.byref(loop), _ptr(theta0), _ptr(eta), _ptr(inner_x),
-                                    _ptr(inner_y), _ptr(outer_x), _ptr(outer_y), _ptr(d_eta),
-                                    _ptr(d_theta0), _ptr(outer_loss), _stream(stream))
+        import torch
+        f32, xd, yd = torch.float32, self.x_dtype, self.y_dtype
+        st = self._lib.mf_meta_grad(self.h, C.byref(loop), _dev(theta0, "theta0", f32),
+                                    _dev(eta, "eta", f32), _dev(inner_x, "inner_x", xd),
+                                    _dev(inner_y, "inner_y", yd), _dev(outer_x, "outer_x", xd),
+                                    _dev(outer_y, "outer_y", yd), _dev(d_eta, "d_eta", f32),
+                                    _dev(d_theta0, "d_theta0", f32),
+                                    _dev(outer_loss, "outer_loss", f32), _stream(stream))
         self._check(st, "mf_meta_grad")
 
     def inner_rollout(self, loop, theta0, eta, inner_x, inner_y, thetaT, stream=None):
-        st = self._lib.mf_inner_rollout(self.h, C.byref(loop), _ptr(theta0), _ptr(eta),
-                                        _ptr(inner_x), _ptr(inner_y), _ptr(thetaT), _stream(stream))
+        import torch
+        f32 = torch.float32
+        st = self._lib.mf_inner_rollout(self.h, C.byref(loop), _dev(theta0, "theta0", f32),
+                                        _dev(eta, "eta", f32),
+                                        _dev(inner_x, "inner_x", self.x_dtype),
+                                        _dev(inner_y, "inner_y", self.y_dtype),
+                                        _dev(thetaT, "thetaT", f32), _stream(stream))
         self._check(st, "mf_inner_rollout")
 
     def hvp(self, B, theta, x, y, v, Hv, ex_w=None, tangent_losses=None, grad=None,
             hvp_mode=MF_HVP_MIXED_FOR, stream=None):
-        st = self._lib.mf_hvp(self.h, B, _ptr(theta), _ptr(x), _ptr(y), _ptr(ex_w), _ptr(v),
-                              _ptr(Hv), _ptr(tangent_losses), _ptr(grad), hvp_mode, _stream(stream))
+        import torch
+        f32 = torch.float32
+        st = self._lib.mf_hvp(self.h, B, _dev(theta, "theta", f32), _dev(x, "x", self.x_dtype),
+                              _dev(y, "y", self.y_dtype), _dev(ex_w, "ex_w", f32),
+                              _dev(v, "v", f32), _dev(Hv, "Hv", f32),
+                              _dev(tangent_losses, "tangent_losses", f32),
+                              _dev(grad, "grad", f32), hvp_mode, _stream(stream))
         self._check(st, "mf_hvp")
 
     def sync(self):
