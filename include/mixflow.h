@@ -187,16 +187,20 @@ mf_status mf_workspace_bytes(mf_handle h, const mf_loop_desc* loop, size_t* byte
 /* Free the cached workspace now (the next call allocates it again). */
 mf_status mf_release_workspace(mf_handle h);
 
-/* Inner rollout only (Eq. 2, Algorithm 2's loop): theta0 [P] float32, eta as above,
- * inner_x [T][B][d_in] (bf16 for MF_PREC_BF16, float32 for MF_PREC_FP32), inner_y
- * [T][B] int32 labels or [T][B][d_out] float32 targets.  Writes thetaT [P]. */
+/* Inner rollout only (Eq. 2, Algorithm 2's loop): theta0 [P] float32, eta [n_eta] float32
+ * (NULL allowed when n_eta = 0), inner_x [T][B][d_in] (bf16 for MF_PREC_BF16, float32 for
+ * MF_PREC_FP32), inner_y [T][B] int32 labels (MF_LOSS_SOFTMAX_CE) or [T][B][d_out] float32
+ * targets.  Decoders: inner_x = inner_y = int32 token ids [T][B][seq_len+1].  Writes
+ * thetaT [P].  bf16 inputs must start on a 16-byte boundary with d_in a multiple of 8.
+ * Errors: MF_ERR_INVALID_ARG (descriptor, NULL or misaligned tensor), MF_ERR_OOM (workspace),
+ * MF_ERR_CUDA; device-side errors come from mf_sync(). */
 mf_status mf_inner_rollout(mf_handle h, const mf_loop_desc* loop, const float* theta0,
                            const float* eta, const void* inner_x, const void* inner_y,
                            float* thetaT, void* stream);
 
 /* One fwdrev_grad backward step (Section 3.1): at parameters theta [P], on the batch
- * x [B][d_in] / y [B] or [B][d_out] with per-example loss weights ex_w [B] (NULL = all 1),
- * for L = (1/B) sum_b ex_w_b l_b:
+ * x [B][d_in] / y [B] or [B][d_out] (decoders: x = y = token ids [B][seq_len+1]) with
+ * per-example loss weights ex_w [B] (NULL = all 1), for L = (1/B) sum_b ex_w_b l_b:
  *   Hv [P]             = (d^2 L / d theta^2) v        (forward-over-reverse)
  *   tangent_losses [B] = grad l_b(theta) . v           (nullable; the mixed term per example)
  *   grad [P]           = grad L(theta)                 (nullable)
@@ -206,11 +210,15 @@ mf_status mf_hvp(mf_handle h, int B, const float* theta, const void* x, const vo
                  float* grad, int hvp_mode, void* stream);
 
 /* The meta-gradient (Algorithm 2): rollout storing theta_t (and m_t when lr is a
- * meta-parameter), outer gradient (Eq. 4), then the mixed-mode reverse sweep t = T-1..0.
- *   d_eta [n_eta]      dV/d eta (same layout as eta).
- *   d_theta0 [P]       dV/d theta_0 (nullable).
- *   outer_loss [1]     V (nullable, device float).
- * outer_x [B_outer][d_in], outer_y [B_outer] int32 or [B_outer][d_out] float32. */
+ * meta-parameter; m_t and v_t with Adam), outer gradient (Eq. 4), then the reverse sweep
+ * t = T-1..0 with the loop's hvp_mode.  Inputs as for mf_inner_rollout, plus
+ * outer_x [B_outer][d_in], outer_y [B_outer] int32 or [B_outer][d_out] float32 (decoders:
+ * outer_x = outer_y = token ids [B_outer][seq_len+1]).  Outputs (float32, device):
+ *   d_eta [n_eta]      dV/d eta (same layout as eta; NULL allowed when n_eta = 0).
+ *   d_theta0 [P]       dV/d theta_0 (nullable; required when n_eta = 0).
+ *   outer_loss [1]     V (nullable).
+ * Errors: as for mf_inner_rollout; device-side MF_ERR_NONFINITE (a NaN or Inf in theta_t or
+ * an adjoint) and MF_ERR_TIMEOUT come from mf_sync(), after which the handle stays usable. */
 mf_status mf_meta_grad(mf_handle h, const mf_loop_desc* loop, const float* theta0,
                        const float* eta, const void* inner_x, const void* inner_y,
                        const void* outer_x, const void* outer_y, float* d_eta,
