@@ -216,6 +216,8 @@ def run_gpu(args):
     inp = synth.make_inputs(w)
     d = native.to_device_inputs(w, inp)
     mf = native.MixFlow.for_workload(w)
+    if args.gemm_persistent:
+        mf.set_option(native.MF_OPT_GEMM_PERSISTENT, 1)
     rr = args.hvp_mode == "rr"
     loop = native.loop_desc_for(w, native.MF_HVP_REV_REV if rr else native.MF_HVP_MIXED_FOR,
                                 ckpt_every=args.ckpt_every)
@@ -348,7 +350,9 @@ def run_gpu(args):
                        + (f"; checkpoint store in segments of {args.ckpt_every} steps"
                           if args.ckpt_every > 1 else "")
                        + (f"; Adam inner optimiser (b1 0.9, b2 0.999, eps {args.adam_eps:g}) "
-                          "in place of SGD" if args.optimizer == "adam" else ""),
+                          "in place of SGD" if args.optimizer == "adam" else "")
+                       + ("; CTA-pair GEMMs as persistent kernels"
+                          if args.gemm_persistent else ""),
                        "parallelism": f"replicas x{ws}",
                        "l2": "flushed before every timed step (256 MB write outside the step events)"},
             "roofline": {"bound": "tensor", "kernel": "tc_dual_gemm_kernel (tcgen05 dual GEMM)",
@@ -396,6 +400,8 @@ def main():
     ap.add_argument("--adam-eps", type=float, default=1e-8)
     ap.add_argument("--ckpt-every", type=int, default=1,
                     help="segment length of the theta_t store (1 = keep every theta_t)")
+    ap.add_argument("--gemm-persistent", action="store_true",
+                    help="run CTA-pair GEMMs as persistent kernels (MF_OPT_GEMM_PERSISTENT)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

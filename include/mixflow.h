@@ -261,9 +261,14 @@ mf_status mf_kernel_time(mf_handle h, double* ms, uint64_t* launches, double* fl
  * S x S probabilities and their tangent in memory (bf16 decoders with d_model/n_heads = 64
  * and seq_len a multiple of 64; others always use the materialised form).  0 materialises
  * them (per block, for the backward).  Setting it drops the handle's captured graphs and
- * changes the workspace size. */
+ * changes the workspace size.
+ * MF_OPT_GEMM_PERSISTENT (process-wide, default 0): 1 runs every GEMM that takes CTA-pair
+ * tiles as a persistent kernel: one pair per SM pair walks a static list of output tiles,
+ * with two TMEM accumulator sets so that a tile's epilogue overlaps the next tile's main loop
+ * (dual products then take 128-wide tiles).  Same products and summation order within a
+ * tile as the one-tile form.  Setting it drops the handle's captured graphs. */
 enum { MF_OPT_CUDA_GRAPHS = 1, MF_OPT_PDL = 2, MF_OPT_CONCURRENT = 3, MF_OPT_GEMM_2SM = 4,
-       MF_OPT_FLASH_ATTN = 5 };
+       MF_OPT_FLASH_ATTN = 5, MF_OPT_GEMM_PERSISTENT = 6 };
 mf_status mf_set_option(mf_handle h, int option, int value);
 
 /* Host-side fault injection for tests: kind 1 = the next workspace allocation fails;

@@ -63,6 +63,10 @@ cudaError_t tc_gemm_act(const GemmArgs& a, cudaStream_t s, const char** why, int
 // Process-wide choice of 2-SM tiles for GEMMs that leave it automatic: 0 never, 1 when the
 // grid fills the GPU (default), 2 whenever M > 128.
 extern int g_pair_mode;
+// Persistent CTA-pair form of the tcgen05 GEMM (tc_gemm_persist.cu): 2-SM tiles go through it
+// when g_gemm_persist is 1 (MF_OPT_GEMM_PERSISTENT; default 0).  bn is 128 or 256.
+cudaError_t tc_gemm_persist(const GemmArgs& a, cudaStream_t s, const char** why, int bn);
+extern int g_gemm_persist;
 // SIMT float32 GEMM with the same semantics (simt_gemm.cu).
 cudaError_t simt_gemm(const GemmArgs& a, cudaStream_t s);
 

@@ -102,6 +102,7 @@ cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why) {
     else bn = 256;
   }
   if (a.b_mn && bn < 64) bn = 64;   // MN-major B is staged in 64-row boxes
+  if (pair && g_gemm_persist) return tc_gemm_persist(a, s, why, bn);
   if (a.epi.mode == EPI_STORE) return launch_bn<EPI_STORE, ACT_IDENT>(a, s, why, bn, pair);
   return tc_gemm_act(a, s, why, bn, pair);
 }

@@ -31,8 +31,15 @@ def main() -> None:
 
     ap = argparse.ArgumentParser()
     ap.add_argument("--only", default="", help="substring of the shape names to run")
+    ap.add_argument("--persistent", action="store_true",
+                    help="CTA-pair tiles as persistent kernels (MF_OPT_GEMM_PERSISTENT)")
     args = ap.parse_args()
     torch.cuda.set_device(0)
+    if args.persistent:   # a process-wide option, set through any handle
+        from paper_2505_00793_gb300 import synth
+        h = native.MixFlow.for_workload(synth.WORKLOADS["tiny"])
+        h.set_option(native.MF_OPT_GEMM_PERSISTENT, 1)
+        h.close()
     s = torch.cuda.current_stream()
     for name, M, N, K, t in SHAPES:
         if args.only and args.only not in name:
@@ -62,7 +69,8 @@ def main() -> None:
         e1.record(s)
         torch.cuda.synchronize()
         cb = e0.elapsed_time(e1) / n
-        print(json.dumps({"name": name, "M": M, "N": N, "K": K, "terms": t, "us": ms * 1e3,
+        print(json.dumps({"name": name, "M": M, "N": N, "K": K, "terms": t,
+                          "persistent": args.persistent, "us": ms * 1e3,
                           "tflops": 2.0 * M * N * K * terms / ms / 1e9,
                           "cublas_one_product_tflops": 2.0 * M * N * K / cb / 1e9}), flush=True)
         del A0, A1, B0, B1, C0, C1
