@@ -218,6 +218,8 @@ def run_gpu(args):
     mf = native.MixFlow.for_workload(w)
     if args.gemm_persistent:
         mf.set_option(native.MF_OPT_GEMM_PERSISTENT, 1)
+    if args.fused_head:
+        mf.set_option(native.MF_OPT_FUSED_HEAD, 1)
     rr = args.hvp_mode == "rr"
     loop = native.loop_desc_for(w, native.MF_HVP_REV_REV if rr else native.MF_HVP_MIXED_FOR,
                                 ckpt_every=args.ckpt_every)
@@ -352,7 +354,9 @@ def run_gpu(args):
                        + (f"; Adam inner optimiser (b1 0.9, b2 0.999, eps {args.adam_eps:g}) "
                           "in place of SGD" if args.optimizer == "adam" else "")
                        + ("; CTA-pair GEMMs as persistent kernels"
-                          if args.gemm_persistent else ""),
+                          if args.gemm_persistent else "")
+                       + ("; output layer, loss and data product fused"
+                          if args.fused_head else ""),
                        "parallelism": f"replicas x{ws}",
                        "l2": "flushed before every timed step (256 MB write outside the step events)"},
             "roofline": {"bound": "tensor", "kernel": "tc_dual_gemm_kernel (tcgen05 dual GEMM)",
@@ -402,6 +406,8 @@ def main():
                     help="segment length of the theta_t store (1 = keep every theta_t)")
     ap.add_argument("--gemm-persistent", action="store_true",
                     help="run CTA-pair GEMMs as persistent kernels (MF_OPT_GEMM_PERSISTENT)")
+    ap.add_argument("--fused-head", action="store_true",
+                    help="output layer, loss and data product in one kernel (MF_OPT_FUSED_HEAD)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

@@ -266,9 +266,15 @@ mf_status mf_kernel_time(mf_handle h, double* ms, uint64_t* launches, double* fl
  * tiles as a persistent kernel: one pair per SM pair walks a static list of output tiles,
  * with two TMEM accumulator sets so that a tile's epilogue overlaps the next tile's main loop
  * (dual products then take 128-wide tiles).  Same products and summation order within a
- * tile as the one-tile form.  Setting it drops the handle's captured graphs. */
+ * tile as the one-tile form.  Setting it drops the handle's captured graphs.
+ * MF_OPT_FUSED_HEAD (process-wide, default 0): 1 computes the output layer of an MLP with at
+ * most 16 outputs and a squared or softmax cross-entropy loss in one kernel per pass: the
+ * layer's forward product, the loss with its seeds and tangent losses, and its data product
+ * into the layer below (one block per example row, float32 accumulation; the weight product
+ * stays a GEMM).  The reverse-over-reverse sweep and the chain loss keep the separate
+ * launches.  Setting it drops the handle's captured graphs. */
 enum { MF_OPT_CUDA_GRAPHS = 1, MF_OPT_PDL = 2, MF_OPT_CONCURRENT = 3, MF_OPT_GEMM_2SM = 4,
-       MF_OPT_FLASH_ATTN = 5, MF_OPT_GEMM_PERSISTENT = 6 };
+       MF_OPT_FLASH_ATTN = 5, MF_OPT_GEMM_PERSISTENT = 6, MF_OPT_FUSED_HEAD = 7 };
 mf_status mf_set_option(mf_handle h, int option, int value);
 
 /* Host-side fault injection for tests: kind 1 = the next workspace allocation fails;

@@ -19,7 +19,7 @@ OUT_DIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(OUT_DIR, "libmixflow.so")
 BUILD_DIR = os.path.join(ROOT, "_build")
 SOURCES = ["tc_gemm.cu", "tc_gemm_act.cu", "tc_gemm_persist.cu", "simt_gemm.cu", "kernels.cu",
-           "decoder_kernels.cu", "flash_attn.cu", "capi.cu"]
+           "head_fused.cu", "decoder_kernels.cu", "flash_attn.cu", "capi.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "-I" + os.path.join(ROOT, "include")]

@@ -336,6 +336,16 @@ struct Exec {
   int loss_kind() const {
     return h->md.loss == MF_LOSS_SOFTMAX_CE ? 1 : h->md.loss == MF_LOSS_CHAIN_MSE ? 2 : 0;
   }
+  // The output layer's forward product, loss and data product as one kernel
+  // (MF_OPT_FUSED_HEAD); never inside the reverse-over-reverse HVP, whose adjoint passes
+  // read the logits and the stored reverse graph.
+  bool no_fuse = false;
+  const float* fwd_theta = nullptr;   // parameters and tangent of the last forward pass
+  const float* fwd_u = nullptr;
+  bool fused_head() const {
+    return mf::g_fused_head && !no_fuse && !ror_store && loss_kind() != 2 &&
+           h->dims[h->L] <= mf::kHeadMaxOut;
+  }
 
   Exec(mf_ctx* h_, const Plan& p_, cudaStream_t s_)
       : h(h_), p(p_), s(s_), base(static_cast<char*>(h_->ws)) {
@@ -457,6 +467,8 @@ struct Exec {
   // Forward pass of `rows` examples: primal (z) or dual (z, z_dot along u).  Hidden layers
   // fuse bias, activation and its tangent into the GEMM epilogue.
   void forward(int rows, const void* xv, const float* theta, const float* u, bool dual) {
+    fwd_theta = theta;
+    fwd_u = u;
     const int din0 = h->dims[0];
     const size_t es = sizeof(T);
     // inputs into the augmented layer-0 activations (the bias column is already set)
@@ -466,6 +478,7 @@ struct Exec {
       h->err = "input copy failed";
     }
     for (int l = 0; l < h->L; ++l) {
+      if (l == h->L - 1 && fused_head()) break;   // the output layer runs in loss()
       const int din = h->dims[l], dout = h->dims[l + 1];
       GemmArgs g;
       g.M = rows; g.N = dout; g.K = din;
@@ -517,7 +530,43 @@ struct Exec {
       a.tape = at<float>(p.o_CH);
       a.ror = 1;
     }
+    if (fused_head()) {
+      head(rows, dual, a, fwd_theta, fwd_u);
+      return;
+    }
     mf::loss_seed<T>(a, s);
+    launched();
+  }
+
+  // Fused output layer (see fused_head): forward product of layer L-1 from the activations
+  // the forward pass left, the loss `a`, and the data product into layer L-2's seeds.
+  void head(int rows, bool dual, const mf::LossArgs& a, const float* theta, const float* u) {
+    if (st != MF_OK) return;
+    const int L = h->L, l = L - 1, din = h->dims[l], dout = h->dims[L];
+    mf::HeadArgs ha;
+    ha.rows = rows; ha.D = din; ha.C = dout; ha.dual = dual;
+    ha.act = h->md.act;
+    ha.A = at<T>(p.o_A[l]);
+    ha.Ad = dual && l > 0 ? at<T>(p.o_Ad[l]) : nullptr;
+    ha.lda = p.lda[l];
+    ha.W = at<T>(p.o_Wb[l]); ha.U = at<T>(p.o_Ub[l]); ha.ldw = ld8(dout);
+    ha.bias = h->md.has_bias ? theta + h->boff[l] : nullptr;
+    ha.ubias = dual && h->md.has_bias ? u + h->boff[l] : nullptr;
+    ha.loss = a;
+    if (l > 0) {
+      ha.Z = at<float>(p.o_Z[l - 1]);
+      ha.Zd = dual ? at<float>(p.o_Zd[l - 1]) : nullptr;
+      ha.ldz = din;
+      ha.dz_prev = dz_buf(l - 1);
+      ha.dzd_prev = dual ? at<T>(p.o_dZd[(l - 1) & 1]) : nullptr;
+      ha.ld_prev = ld8(din);
+    }
+    const cudaError_t e = mf::head_fused<T>(ha, s);
+    if (e != cudaSuccess) {
+      st = MF_ERR_CUDA;
+      h->err = std::string("fused head launch failed: ") + cudaGetErrorString(e);
+      return;
+    }
     launched();
   }
 
@@ -552,6 +601,12 @@ struct Exec {
       if (l == 0) {
         if (wgemm) gemm(g);
         break;
+      }
+      if (l == h->L - 1 && fused_head()) {
+        // the fused head kernel has written layer l-1's seeds already; layer l-1's data
+        // product overwrites the seed set this weight product reads, so it runs in order
+        if (wgemm) gemm(g);
+        continue;
       }
       // data product: da = dz W^T ; da' = dz' W^T + dz U^T ; epilogue -> dz, dz' of layer l-1
       GemmArgs d;
@@ -593,6 +648,7 @@ struct Exec {
                const float* eta_w, const float* ex_w, float* Hv, float* grad, float* ld_out,
                float* d_eta) {
     const int L = h->L, hb = h->md.has_bias ? 1 : 0;
+    no_fuse = true;
     forward(rows, x, theta, nullptr, false);
     ror_store = true;
     loss(rows, false, y, eta_w, ex_w, nullptr, nullptr, nullptr);
@@ -674,6 +730,7 @@ struct Exec {
       d.C0 = at<float>(p.o_AB); d.ldc0 = din;
       gemm(d);
     }
+    no_fuse = false;
   }
 };
 
@@ -1436,6 +1493,12 @@ mf_status mf_set_option(mf_handle h, int option, int value) {
   if (option == MF_OPT_GEMM_PERSISTENT) {
     if (value < 0 || value > 1) return fail(h, MF_ERR_INVALID_ARG, "MF_OPT_GEMM_PERSISTENT takes 0 or 1");
     mf::g_gemm_persist = value;
+    drop_graphs(h);
+    return MF_OK;
+  }
+  if (option == MF_OPT_FUSED_HEAD) {
+    if (value < 0 || value > 1) return fail(h, MF_ERR_INVALID_ARG, "MF_OPT_FUSED_HEAD takes 0 or 1");
+    mf::g_fused_head = value;
     drop_graphs(h);
     return MF_OK;
   }

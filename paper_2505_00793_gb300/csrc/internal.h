@@ -106,6 +106,27 @@ struct LossArgs {
 template <typename T>
 void loss_seed(const LossArgs& a, cudaStream_t s);
 
+// Fused narrow head (head_fused.cu): the output layer's forward product, the loss of
+// loss_seed (squared or softmax CE) and the output layer's data product with the activation
+// backward of the layer below, one block per example row.  Used for outputs of at most
+// kHeadMaxOut units when g_fused_head is 1 (MF_OPT_FUSED_HEAD; default 0).
+constexpr int kHeadMaxOut = 16;
+struct HeadArgs {
+  int rows = 0, D = 0, C = 0;      // example rows, head input width, head outputs
+  bool dual = false;               // tangent pass along u
+  int act = ACT_IDENT;             // activation of the layer below the head
+  const void* A = nullptr; const void* Ad = nullptr; int lda = 0;   // head inputs [rows][lda] (T)
+  const void* W = nullptr; const void* U = nullptr; int ldw = 0;    // [D][ldw] operand copies (T)
+  const float* bias = nullptr; const float* ubias = nullptr;        // nullable
+  LossArgs loss;                   // targets, weights, outputs and the head seeds (dF, dFd, ldo)
+  const float* Z = nullptr; const float* Zd = nullptr; int ldz = 0;      // layer below: z, z'
+  void* dz_prev = nullptr; void* dzd_prev = nullptr; int ld_prev = 0;    // its seeds (T); null:
+                                                                         // no data product
+};
+template <typename T>
+cudaError_t head_fused(const HeadArgs& a, cudaStream_t s);
+extern int g_fused_head;
+
 // out[0] = scale * sum_i x[i] (deterministic, one block)
 void sum_scaled(const float* x, int n, float scale, float* out, cudaStream_t s);
 
