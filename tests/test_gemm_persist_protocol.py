@@ -1,0 +1,179 @@
+"""Barrier protocol of the persistent CTA-pair GEMM (csrc/tc_gemm_persist.cu), model-checked
+on the CPU.
+
+The kernel's three roles are modelled as coroutines over mbarriers with PTX phase semantics
+(a barrier completes a phase when its pending arrivals and transaction bytes reach zero;
+`try_wait.parity P` succeeds once the phase of parity P has completed).  Asynchronous
+completions (TMA bytes, tcgen05.commit arrivals, which keep their issue order) are queued
+events.  Random interleavings must finish without deadlock, every MMA must read the stage
+data of its own tile and K block, no stage may be refilled before the MMA consumed it, and
+no accumulator set may be overwritten before every epilogue warp of both CTAs read it.
+The parity and count formulas are the kernel's:
+  producer   stage s = g % S, waits empty[s] parity ((g / S) & 1) ^ 1
+  MMA        tile j uses set j & 1 (two sets) for the (j >> 1)-th time: waits acc_empty[set]
+             parity (use & 1) ^ 1, then full[s] parity (g / S) & 1 per K block
+  epilogue   waits acc_full[set] parity use & 1, then arrives on the even CTA's acc_empty[set]
+             (count 2 x EPI_WARPS)."""
+import random
+
+import pytest
+
+
+class Bar:
+    def __init__(self, count):
+        self.count, self.pending, self.tx, self.k = count, count, 0, 0
+
+    def _check(self):
+        if self.pending == 0 and self.tx == 0:
+            self.k += 1
+            self.pending = self.count
+
+    def arrive(self):
+        self.pending -= 1
+        assert self.pending >= 0, "more arrivals than the barrier's count"
+        self._check()
+
+    def arrive_expect_tx(self, nbytes):
+        self.tx += nbytes
+        self.arrive()
+
+    def complete_tx(self, nbytes):
+        self.tx -= nbytes
+        self._check()
+
+    def try_wait(self, parity):
+        return (self.k & 1) != parity
+
+
+class Deadlock(Exception):
+    pass
+
+
+def run_pair(ntiles, pair, npairs, nk, stages, nsets, epi_warps, seed,
+             acc_empty_count=None, mma_parity_flip=0):
+    """One CTA pair of the persistent kernel; returns the number of tiles it drained."""
+    rnd = random.Random(seed)
+    full0 = [Bar(1) for _ in range(stages)]                       # even CTA only
+    empty = [[Bar(1) for _ in range(stages)] for _ in range(2)]   # both CTAs
+    acc_full = [[Bar(1) for _ in range(2)] for _ in range(2)]
+    acc_empty0 = [Bar(acc_empty_count or 2 * epi_warps) for _ in range(2)]
+    stage_data = [[None] * stages for _ in range(2)]
+    consumed, reads, acc = set(), {}, [None, None]
+    events = []
+    tiles = list(range(pair, ntiles, npairs))
+
+    def set_use(j):
+        return (j & 1, j >> 1) if nsets == 2 else (0, j)
+
+    def producer(rank):
+        g = 0
+        for t in tiles:
+            for i in range(nk):
+                s, ph = g % stages, (g // stages) & 1
+                while not empty[rank][s].try_wait(ph ^ 1):
+                    yield
+                assert g < stages or (g - stages) in consumed, "stage refilled before consumed"
+                if rank == 0:
+                    full0[s].arrive_expect_tx(2)
+                stage_data[rank][s] = (t, i)
+                events.append(("tx", s))
+                g += 1
+                yield
+
+    def mma():
+        for j, t in enumerate(tiles):
+            st, use = set_use(j)
+            while not acc_empty0[st].try_wait((use & 1) ^ 1 ^ mma_parity_flip):
+                yield
+            assert use == 0 or reads.get((st, use - 1), 0) == 2 * epi_warps, \
+                "accumulator set overwritten before the epilogue read it"
+            acc[st] = [t, []]
+            for i in range(nk):
+                g = j * nk + i
+                s, ph = g % stages, (g // stages) & 1
+                while not full0[s].try_wait(ph):
+                    yield
+                assert stage_data[0][s] == (t, i) and stage_data[1][s] == (t, i), "stage data"
+                acc[st][1].append(i)
+                events.append(("commit_stage", s, g))
+                yield
+            events.append(("commit_acc", st))
+            yield
+
+    def epilogue(rank):
+        for j, t in enumerate(tiles):
+            st, use = set_use(j)
+            while not acc_full[rank][st].try_wait(use & 1):
+                yield
+            assert acc[st] == [t, list(range(nk))], "epilogue read an unfinished tile"
+            yield
+            reads[(st, use)] = reads.get((st, use), 0) + 1
+            acc_empty0[st].arrive()
+            yield
+
+    actors = [producer(0), producer(1), mma()]
+    actors += [epilogue(r) for r in (0, 1) for _ in range(epi_warps)]
+    steps = 0
+    while actors or events:
+        c = rnd.randrange(len(actors) + (1 if events else 0))
+        if c == len(actors):
+            commits = [k for k, e in enumerate(events) if e[0] != "tx"]
+            tx = [k for k, e in enumerate(events) if e[0] == "tx"]
+            # TMA bytes land in any order; tcgen05.commit arrivals keep their issue order
+            idx = commits[0] if commits and (not tx or rnd.random() < 0.5) else rnd.choice(tx)
+            ev = events.pop(idx)
+            if ev[0] == "tx":
+                full0[ev[1]].complete_tx(1)
+            elif ev[0] == "commit_stage":
+                consumed.add(ev[2])
+                empty[0][ev[1]].arrive()
+                empty[1][ev[1]].arrive()
+            else:
+                acc_full[0][ev[1]].arrive()
+                acc_full[1][ev[1]].arrive()
+            continue
+        try:
+            next(actors[c])
+        except StopIteration:
+            actors.pop(c)
+        steps += 1
+        if steps > 200000:
+            raise Deadlock()
+    # tiles whose accumulators every epilogue warp of both CTAs read
+    return sum(1 for n in reads.values() if n == 2 * epi_warps)
+
+
+def _configs(n):
+    rnd = random.Random(12345)
+    for seed in range(n):
+        npairs = rnd.randint(1, 4)
+        yield dict(ntiles=rnd.randint(1, 12), pair=rnd.randrange(npairs), npairs=npairs,
+                   nk=rnd.randint(1, 7), stages=rnd.randint(2, 6), nsets=rnd.choice([1, 2]),
+                   epi_warps=rnd.choice([1, 2, 8]), seed=seed)
+
+
+def test_protocol_completes_every_tile():
+    for cfg in _configs(400):
+        expect = len(range(cfg["pair"], cfg["ntiles"], cfg["npairs"]))
+        assert run_pair(**cfg) == expect, cfg
+
+
+@pytest.mark.parametrize("mistake", ["acc_empty_count", "mma_parity"])
+def test_model_catches_planted_mistakes(mistake):
+    """A wrong arrival count or a flipped parity on the accumulator hand-off is caught in
+    (nearly) every configuration where a set is reused."""
+    caught = eligible = 0
+    for cfg in _configs(60):
+        if len(range(cfg["pair"], cfg["ntiles"], cfg["npairs"])) < 3:
+            continue
+        eligible += 1
+        kw = dict(cfg)
+        if mistake == "acc_empty_count":
+            kw["acc_empty_count"] = cfg["epi_warps"] + 1 if cfg["epi_warps"] > 1 else 3
+        else:
+            kw["mma_parity_flip"] = 1
+        try:
+            run_pair(**kw)
+        except (AssertionError, Deadlock):
+            caught += 1
+    assert eligible > 20 and caught >= 0.9 * eligible, (caught, eligible)
