@@ -152,21 +152,26 @@ def _dram_traffic():
         return None
 
 
-def cpu_oracle_time(w, t_sample=None):
+def cpu_oracle_time(w, t_sample=None, min_seconds=0.0):
     """Wall time of the float64 oracle meta-gradient on workload w, run on the first
     ``t_sample`` inner steps (all T when None) and scaled by T / t_sample.  Scaling also
     multiplies the outer-gradient part, so a sampled figure over-states the oracle's time
-    slightly.  Returns (seconds for the full workload, seconds spent, threads)."""
+    slightly.  The oracle runs again until ``min_seconds`` of CPU work are spent; the time is
+    the mean over the runs.  Returns (seconds for the full workload, seconds spent, threads,
+    runs)."""
     import torch
     from paper_2505_00793_gb300 import synth
     from oracle import metagrad as om
     ts = w.T if t_sample is None else min(t_sample, w.T)
     ws = w.with_(T=ts)
     inp = synth.make_inputs(ws)
-    t0 = time.perf_counter()
-    om.meta_grad(ws, inp)
-    spent = time.perf_counter() - t0
-    return spent * w.T / ts, spent, torch.get_num_threads()
+    spent, runs = 0.0, 0
+    while runs == 0 or spent < min_seconds:
+        t0 = time.perf_counter()
+        om.meta_grad(ws, inp)
+        spent += time.perf_counter() - t0
+        runs += 1
+    return spent / runs * w.T / ts, spent, torch.get_num_threads(), runs
 
 
 def run_reference(args):
@@ -179,7 +184,7 @@ def run_reference(args):
         cpu_oracle_time(w, REF_T_SAMPLE)
     est = []
     for _ in range(args.steps):
-        full, spent, cores = cpu_oracle_time(w, REF_T_SAMPLE)
+        full, spent, cores, _ = cpu_oracle_time(w, REF_T_SAMPLE)
         est.append(full)
     ms = 1000.0 * statistics.mean(est)
     value = 1000.0 / ms
@@ -336,10 +341,10 @@ def run_gpu(args):
         cpu = None
         default = args.workload == WORKLOAD and not rr
         if ws == 1 and not args.no_cpu_baseline and (default or args.cpu_baseline):
-            full_s, spent, cores = cpu_oracle_time(w)
+            full_s, spent, cores, runs = cpu_oracle_time(w, min_seconds=10.0)
             cpu = {"value": 1.0 / full_s, "unit": "meta-steps/s", "cores": cores, "kind": "oracle",
-                   "sample": f"one full oracle meta-gradient of the workload (T=16, {spent:.1f} s "
-                             "of CPU work)"}
+                   "sample": f"{runs} full oracle meta-gradients of the workload (T={w.T}), "
+                             f"{spent:.1f} s of CPU work, mean time per meta-gradient"}
         out = {
             "metric": "meta-grad steps/s", "value": value, "unit": "meta-steps/s", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,

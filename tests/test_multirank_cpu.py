@@ -96,3 +96,17 @@ def test_reference_line_contract(monkeypatch):
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["value"] == d["value"]
     assert d["higher_is_better"] is True
+
+
+def test_cpu_baseline_repeats_to_its_minimum_time():
+    """The CPU baseline repeats the oracle until the requested CPU time is spent and reports
+    the mean per meta-gradient."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2505_00793_gb300 import synth
+    w = synth.WORKLOADS["tiny"]
+    full, spent, cores, runs = bench.cpu_oracle_time(w, min_seconds=0.2)
+    assert runs >= 2 and spent >= 0.2 and cores >= 1
+    assert abs(full - spent / runs) <= 1e-12 * spent
+    full1, spent1, _, runs1 = bench.cpu_oracle_time(w)
+    assert runs1 == 1 and full1 == spent1
