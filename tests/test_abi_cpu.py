@@ -92,3 +92,69 @@ def test_binding_checks_tensor_arguments():
             assert d[k].dtype == y_dt and d[k].is_contiguous(), (w.name, k)
         for k in ("theta0", "eta"):
             assert d[k].dtype == torch.float32, (w.name, k)
+
+
+def _header_enums():
+    """Every `NAME = value` of the header's enums (comments stripped)."""
+    txt = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    vals = {}
+    for body in re.findall(r"enum\s*\{(.*?)\}", txt, flags=re.S):
+        for name, v in re.findall(r"\b(MF_[A-Z0-9_]+)\s*=\s*(\d+)", body):
+            vals[name] = int(v)
+    for name, v in re.findall(r"\b(MF_[A-Z_]+)\s*=\s*(\d+)\s*[,}]", txt):
+        vals.setdefault(name, int(v))
+    return vals
+
+
+def test_binding_constants_match_header():
+    """The binding's enum values (options, losses, activations, meta kinds, modes) are the
+    header's."""
+    from paper_2505_00793_gb300 import native
+    h = _header_enums()
+    pairs = {"MF_ARCH_MLP": native.MF_ARCH_MLP, "MF_ARCH_DECODER": native.MF_ARCH_DECODER,
+             "MF_ACT_IDENT": native.ACTS["ident"], "MF_ACT_TANH": native.ACTS["tanh"],
+             "MF_ACT_GELU": native.ACTS["gelu"], "MF_ACT_SILU": native.ACTS["silu"],
+             "MF_LOSS_SQUARED": native.LOSSES["squared"], "MF_LOSS_SOFTMAX_CE": native.LOSSES["ce"],
+             "MF_LOSS_NEXT_TOKEN_CE": native.LOSSES["next_token_ce"],
+             "MF_LOSS_CHAIN_MSE": native.LOSSES["chain_mse"],
+             "MF_PREC_FP32": native.PRECISIONS["fp32"], "MF_PREC_BF16": native.PRECISIONS["bf16"],
+             "MF_OPTIM_SGD": native.OPTIMIZERS["sgd"], "MF_OPTIM_ADAM": native.OPTIMIZERS["adam"],
+             "MF_META_EXAMPLE_WEIGHTS": native.MF_META_EXAMPLE_WEIGHTS,
+             "MF_META_PARAM_LOGLR": native.MF_META_PARAM_LOGLR,
+             "MF_META_SCALAR_LOGLR": native.MF_META_SCALAR_LOGLR,
+             "MF_HVP_MIXED_FOR": native.MF_HVP_MIXED_FOR, "MF_HVP_REV_REV": native.MF_HVP_REV_REV}
+    for name, value in pairs.items():
+        assert h[name] == value, name
+    opts = {k: v for k, v in h.items() if k.startswith("MF_OPT_")}
+    assert opts and all(getattr(native, k) == v for k, v in opts.items())
+    status = {v: k for k, v in h.items() if k == "MF_OK" or k.startswith("MF_ERR_")}
+    assert status == native.STATUS
+
+
+def test_binding_structs_match_header():
+    """ctypes structures have the header's fields, in order, with the header's C types."""
+    from paper_2505_00793_gb300 import native
+    txt = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    ctype = {"int": C.c_int, "float": C.c_float}
+    for name, cls in (("mf_model_desc", native.mf_model_desc),
+                      ("mf_loop_desc", native.mf_loop_desc)):
+        body = re.search(r"typedef struct\s*\{([^{}]*)\}\s*" + name + ";", txt).group(1)
+        fields = []
+        for decl in body.split(";"):
+            decl = decl.strip()
+            if not decl:
+                continue
+            typ, rest = decl.split(None, 1)
+            for item in rest.split(","):
+                item = item.strip()
+                m = re.match(r"(\w+)\s*\[(.*)\]", item)
+                if m:
+                    n = eval(m.group(2).replace("MF_MAX_LAYERS", str(native.MF_MAX_LAYERS)))
+                    fields.append((m.group(1), ctype[typ] * n))
+                else:
+                    fields.append((item, ctype[typ]))
+        got = [(f, t) for f, t in cls._fields_]
+        assert [f for f, _ in got] == [f for f, _ in fields], name
+        for (f, t), (_, u) in zip(got, fields):
+            assert C.sizeof(t) == C.sizeof(u), (name, f)
+            assert getattr(t, "_type_", t) == getattr(u, "_type_", u), (name, f)
