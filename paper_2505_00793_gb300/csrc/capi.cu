@@ -111,6 +111,10 @@ struct Plan {
   std::vector<size_t> o_Wb, o_Ub, o_A, o_Ad, o_Z, o_Zd;
   std::vector<int> lda;  // leading dim of layer l's input activations (room for the bias column)
   size_t o_dZ[2] = {0, 0}, o_dZd[2] = {0, 0};
+  // fused narrow head (MF_OPT_FUSED_HEAD): the output layer's seeds in buffers of their own,
+  // so that its weight product does not hold up the layers below
+  bool head_bufs = false;
+  size_t o_dZh = 0, o_dZdh = 0;
   // reverse-over-reverse: the stored reverse graph (per-layer dz, da) and the adjoints
   bool ror = false;
   std::vector<size_t> o_SZ, o_SA, o_DAB, o_ZP;
@@ -171,6 +175,12 @@ Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slot
   for (int b = 0; b < 2; ++b) {
     p.o_dZ[b] = take(static_cast<size_t>(rows) * ld8(md) * es);
     p.o_dZd[b] = take(static_cast<size_t>(rows) * ld8(md) * es);
+  }
+  if (mf::g_fused_head && !h->decoder && h->dims[L] <= mf::kHeadMaxOut &&
+      h->md.loss != MF_LOSS_CHAIN_MSE) {
+    p.head_bufs = true;
+    p.o_dZh = take(static_cast<size_t>(rows) * ld8(h->dims[L]) * es);
+    p.o_dZdh = take(static_cast<size_t>(rows) * ld8(h->dims[L]) * es);
   }
   if (ror) {
     p.o_SZ.resize(L); p.o_SA.resize(L); p.o_DAB.resize(L); p.o_ZP.resize(L);
@@ -343,7 +353,7 @@ struct Exec {
   const float* fwd_theta = nullptr;   // parameters and tangent of the last forward pass
   const float* fwd_u = nullptr;
   bool fused_head() const {
-    return mf::g_fused_head && !no_fuse && !ror_store && loss_kind() != 2 &&
+    return mf::g_fused_head && p.head_bufs && !no_fuse && !ror_store && loss_kind() != 2 &&
            h->dims[h->L] <= mf::kHeadMaxOut;
   }
 
@@ -531,6 +541,8 @@ struct Exec {
       a.ror = 1;
     }
     if (fused_head()) {
+      a.dF = at<T>(p.o_dZh);
+      a.dFd = dual ? at<T>(p.o_dZdh) : nullptr;
       head(rows, dual, a, fwd_theta, fwd_u);
       return;
     }
@@ -575,16 +587,19 @@ struct Exec {
   // products fuse the activation backward (and its tangent) into the epilogue.
   void backward(int rows, bool dual, float* out_h, float* out_g) {
     const int hb = h->md.has_bias ? 1 : 0;
+    const bool fused = fused_head();
+    bool side_pending = false;   // a weight product on the side stream not joined yet
     for (int l = h->L - 1; l >= 0; --l) {
       const int din = h->dims[l], dout = h->dims[l + 1], b = l & 1;
+      const bool head_seeds = fused && l == h->L - 1;
       // [a 1]^T dz and [a' 0]^T dz + [a 1]^T dz': activations [rows][din+1] and seeds
       // [rows][dout] are read MN-major (K = rows)
       GemmArgs g;
       g.M = din + hb; g.N = dout; g.K = rows;
       g.A0 = at<T>(p.o_A[l]); g.lda0 = p.lda[l];
       g.A1 = at<T>(p.o_Ad[l]); g.lda1 = p.lda[l];
-      g.B0 = dz_buf(l); g.ldb0 = ld8(dout);
-      g.B1 = at<T>(p.o_dZd[b]); g.ldb1 = ld8(dout);
+      g.B0 = head_seeds ? at<T>(p.o_dZh) : dz_buf(l); g.ldb0 = ld8(dout);
+      g.B1 = head_seeds ? at<T>(p.o_dZdh) : at<T>(p.o_dZd[b]); g.ldb1 = ld8(dout);
       g.a_mn = g.b_mn = true;
       if (!dual) {
         g.terms = mf::T_C0_A0B0;
@@ -602,10 +617,17 @@ struct Exec {
         if (wgemm) gemm(g);
         break;
       }
-      if (l == h->L - 1 && fused_head()) {
-        // the fused head kernel has written layer l-1's seeds already; layer l-1's data
-        // product overwrites the seed set this weight product reads, so it runs in order
-        if (wgemm) gemm(g);
+      if (head_seeds) {
+        // the fused head kernel has written layer l-1's seeds already, and this weight
+        // product reads the head's own seed buffers, which nothing below overwrites: it runs
+        // on the side stream next to the layers below, joined with their weight products
+        if (wgemm && can_fork()) {
+          fork();
+          gemm(g, h->sstream);
+          side_pending = true;
+        } else if (wgemm) {
+          gemm(g);
+        }
         continue;
       }
       // data product: da = dz W^T ; da' = dz' W^T + dz U^T ; epilogue -> dz, dz' of layer l-1
@@ -633,11 +655,13 @@ struct Exec {
         gemm(g, h->sstream);
         gemm(d);
         join();
+        side_pending = false;
       } else {
         if (wgemm) gemm(g);
         gemm(d);
       }
     }
+    if (side_pending) join();
   }
 
   // Hessian-vector product by reverse-over-reverse (Algorithm 1's schedule): primal forward,
