@@ -225,6 +225,8 @@ def run_gpu(args):
         mf.set_option(native.MF_OPT_GEMM_PERSISTENT, 1)
     if args.fused_head:
         mf.set_option(native.MF_OPT_FUSED_HEAD, 1)
+    if args.layer_updates:
+        mf.set_option(native.MF_OPT_LAYER_UPDATES, 1)
     rr = args.hvp_mode == "rr"
     loop = native.loop_desc_for(w, native.MF_HVP_REV_REV if rr else native.MF_HVP_MIXED_FOR,
                                 ckpt_every=args.ckpt_every)
@@ -361,7 +363,9 @@ def run_gpu(args):
                        + ("; CTA-pair GEMMs as persistent kernels"
                           if args.gemm_persistent else "")
                        + ("; output layer, loss and data product fused"
-                          if args.fused_head else ""),
+                          if args.fused_head else "")
+                       + ("; per-layer updates overlapping the backward pass"
+                          if args.layer_updates else ""),
                        "parallelism": f"replicas x{ws}",
                        "l2": "flushed before every timed step (256 MB write outside the step events)"},
             "roofline": {"bound": "tensor", "kernel": "tc_dual_gemm_kernel (tcgen05 dual GEMM)",
@@ -413,6 +417,8 @@ def main():
                     help="run CTA-pair GEMMs as persistent kernels (MF_OPT_GEMM_PERSISTENT)")
     ap.add_argument("--fused-head", action="store_true",
                     help="output layer, loss and data product in one kernel (MF_OPT_FUSED_HEAD)")
+    ap.add_argument("--layer-updates", action="store_true",
+                    help="per-layer updates overlapping the backward pass (MF_OPT_LAYER_UPDATES)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

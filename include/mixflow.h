@@ -272,9 +272,15 @@ mf_status mf_kernel_time(mf_handle h, double* ms, uint64_t* launches, double* fl
  * layer's forward product, the loss with its seeds and tangent losses, and its data product
  * into the layer below (one block per example row, float32 accumulation; the weight product
  * stays a GEMM).  The reverse-over-reverse sweep and the chain loss keep the separate
- * launches.  Setting it drops the handle's captured graphs. */
+ * launches.  Setting it drops the handle's captured graphs.
+ * MF_OPT_LAYER_UPDATES (default 0): 1 runs an MLP's inner-step and adjoint updates layer by
+ * layer on a library stream of the handle, each as soon as its layer's products in the
+ * backward pass are done, so that they overlap the layers below instead of following the
+ * whole pass.  Element for element the same update.  Decoders and the reverse-over-reverse
+ * sweep keep the single update.  Setting it drops the handle's captured graphs. */
 enum { MF_OPT_CUDA_GRAPHS = 1, MF_OPT_PDL = 2, MF_OPT_CONCURRENT = 3, MF_OPT_GEMM_2SM = 4,
-       MF_OPT_FLASH_ATTN = 5, MF_OPT_GEMM_PERSISTENT = 6, MF_OPT_FUSED_HEAD = 7 };
+       MF_OPT_FLASH_ATTN = 5, MF_OPT_GEMM_PERSISTENT = 6, MF_OPT_FUSED_HEAD = 7,
+       MF_OPT_LAYER_UPDATES = 8 };
 mf_status mf_set_option(mf_handle h, int option, int value);
 
 /* Host-side fault injection for tests: kind 1 = the next workspace allocation fails;

@@ -84,6 +84,12 @@ struct mf_ctx {
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   bool concurrent = true;
   bool flash = true;          // fused dual attention where supported (MF_OPT_FLASH_ATTN)
+  // Per-layer parameter updates (MF_OPT_LAYER_UPDATES): an update stream that takes each
+  // layer's update as soon as that layer's backward products are done, joined back into the
+  // working stream at the end of the backward pass.
+  bool layer_updates = false;
+  cudaStream_t ustream = nullptr;
+  cudaEvent_t ev_u_in = nullptr, ev_u_out = nullptr;
 };
 
 namespace {
@@ -465,6 +471,48 @@ struct Exec {
     launched();
   }
 
+  // Per-layer updates (MF_OPT_LAYER_UPDATES).  With upd_after set, backward() runs that
+  // update for layer l on the update stream as soon as layer l's weight and data products are
+  // done (the update overwrites the layer's operand copies, which the data product reads),
+  // and joins the update stream back before it returns; the caller then skips its update of
+  // the whole vector.  Every update element reads and writes only its own parameter, so the
+  // layers' updates are independent of each other and of the layers still in the pass.
+  const mf::LayerUpdArgs* upd_after = nullptr;
+  bool layer_updates_ok() const {
+    return h->layer_updates && h->ustream && h->ev_u_in && h->ev_u_out;
+  }
+  void update_layer(const mf::LayerUpdArgs& a, int l) {
+    mf::LayerTable t1;
+    t1.n = 1;
+    t1.rows[0] = tab.rows[l]; t1.din[0] = tab.din[l]; t1.dout[0] = tab.dout[l];
+    t1.off[0] = tab.off[l];
+    t1.tile0[0] = 0;
+    t1.tile0[1] = tab.tile0[l + 1] - tab.tile0[l];
+    t1.ldw[0] = tab.ldw[l];
+    t1.W[0] = tab.W[l]; t1.U[0] = tab.U[l];
+    mf::LayerUpdArgs b = a;
+    if (b.partials) b.partials += tab.tile0[l];   // this layer's blocks' scalar-lr partials
+    mf::layer_update<T>(t1, b, h->ustream);
+    launched();
+  }
+  // Layer l's products are enqueued on `on`: the update stream waits for them, then updates l.
+  void upd_layer_after(int l, cudaStream_t on) {
+    if (!upd_after || st != MF_OK) return;
+    if (cudaEventRecord(h->ev_u_in, on) != cudaSuccess ||
+        cudaStreamWaitEvent(h->ustream, h->ev_u_in, 0) != cudaSuccess) {
+      st = MF_ERR_CUDA; h->err = "update stream fork failed";
+      return;
+    }
+    update_layer(*upd_after, l);
+  }
+  void upd_join() {
+    if (!upd_after) return;
+    if (cudaEventRecord(h->ev_u_out, h->ustream) != cudaSuccess ||
+        cudaStreamWaitEvent(s, h->ev_u_out, 0) != cudaSuccess) {
+      st = MF_ERR_CUDA; h->err = "update stream join failed";
+    }
+  }
+
   // Cast parameters (or the tangent) into the GEMM operand copies.
   void cast_params(const float* theta, bool tangent) {
     mf::LayerUpdArgs a;
@@ -615,6 +663,7 @@ struct Exec {
       const bool wgemm = dual || out_g;
       if (l == 0) {
         if (wgemm) gemm(g);
+        upd_layer_after(0, s);
         break;
       }
       if (head_seeds) {
@@ -625,8 +674,10 @@ struct Exec {
           fork();
           gemm(g, h->sstream);
           side_pending = true;
-        } else if (wgemm) {
-          gemm(g);
+          upd_layer_after(l, h->sstream);
+        } else {
+          if (wgemm) gemm(g);
+          upd_layer_after(l, s);
         }
         continue;
       }
@@ -660,8 +711,10 @@ struct Exec {
         if (wgemm) gemm(g);
         gemm(d);
       }
+      upd_layer_after(l, s);
     }
     if (side_pending) join();
+    upd_join();
   }
 
   // Hessian-vector product by reverse-over-reverse (Algorithm 1's schedule): primal forward,
@@ -759,6 +812,17 @@ struct Exec {
 };
 
 #include "decoder_exec.cuh"
+
+// Per-layer updates run inside the MLP executor's backward pass (Exec::upd_after); the
+// decoder executor updates the whole vector after the pass.
+template <typename X>
+bool per_layer_updates(X&) { return false; }
+template <typename X>
+void set_upd_after(X&, const mf::LayerUpdArgs*) {}
+template <typename T>
+bool per_layer_updates(Exec<T>& ex) { return ex.layer_updates_ok(); }
+template <typename T>
+void set_upd_after(Exec<T>& ex, const mf::LayerUpdArgs* a) { ex.upd_after = a; }
 
 mf_status validate_loop(mf_ctx* h, const mf_loop_desc* lp) {
   if (!lp) return fail(h, MF_ERR_INVALID_ARG, "loop descriptor is NULL");
@@ -892,7 +956,6 @@ void inner_step(X& ex, const mf_loop_desc* lp, const float* eta, const void* inn
   const float* ew = (lp->meta_kind & MF_META_EXAMPLE_WEIGHTS) ? eta + static_cast<int64_t>(t) * B : nullptr;
   ex.loss(B, false, y, ew, nullptr, nullptr, nullptr, nullptr);
   float* g = ex.g_buf();
-  ex.backward(B, false, nullptr, g);
   mf::LayerUpdArgs a;
   a.mode = mf::LU_ROLLOUT;
   a.theta = theta;
@@ -908,7 +971,11 @@ void inner_step(X& ex, const mf_loop_desc* lp, const float* eta, const void* inn
     a.v = v;
     a.v_out = v_out;
   }
-  ex.update(a);
+  const bool per_layer = per_layer_updates(ex);
+  if (per_layer) set_upd_after(ex, &a);
+  ex.backward(B, false, nullptr, g);
+  if (per_layer) set_upd_after(ex, nullptr);
+  else ex.update(a);
 }
 
 // Inner rollout over steps [t0, t1) into the checkpoint store: theta_{t+1} (and m_{t+1} when
@@ -1051,13 +1118,6 @@ mf_status meta_grad_run(X& ex, const mf_loop_desc* lp, const float* theta0, cons
     const void* y = static_cast<const char*>(inner_y) + ys * t;
     const float* ew = exw ? eta + static_cast<int64_t>(t) * B : nullptr;
     float* de = exw ? d_eta + static_cast<int64_t>(t) * B : nullptr;
-    if (lp->hvp_mode == MF_HVP_REV_REV) {
-      ex.ror_hvp(B, x, th, u, y, ew, nullptr, Hu, nullptr, ex.ld_buf(), de);
-    } else {
-      ex.forward(B, x, th, u, true);
-      ex.loss(B, true, y, ew, nullptr, nullptr, ex.ld_buf(), de);
-      ex.backward(B, true, Hu, nullptr);
-    }
     // theta_bar_t = theta_bar_{t+1} + H u ; d eta_lr += -lr m_t theta_bar_t ;
     // u_{t-1} = mu u_t - lr theta_bar_t ; cast theta_{t-1}, u_{t-1}
     mf::LayerUpdArgs a;
@@ -1082,7 +1142,19 @@ mf_status meta_grad_run(X& ex, const mf_loop_desc* lp, const float* theta0, cons
     a.mu = lp->momentum;
     a.lr = lr.lr;
     a.status = h->d_status;
-    ex.update(a);
+    // H u at theta_t; with per-layer updates the backward pass runs the update above layer by
+    // layer, else it runs once over the whole vector afterwards
+    const bool per_layer = lp->hvp_mode != MF_HVP_REV_REV && per_layer_updates(ex);
+    if (lp->hvp_mode == MF_HVP_REV_REV) {
+      ex.ror_hvp(B, x, th, u, y, ew, nullptr, Hu, nullptr, ex.ld_buf(), de);
+    } else {
+      ex.forward(B, x, th, u, true);
+      ex.loss(B, true, y, ew, nullptr, nullptr, ex.ld_buf(), de);
+      if (per_layer) set_upd_after(ex, &a);
+      ex.backward(B, true, Hu, nullptr);
+      if (per_layer) set_upd_after(ex, nullptr);
+    }
+    if (!per_layer) ex.update(a);
     if (ex.st != MF_OK) return ex.st;
   }
   if (scalar_lr) {
@@ -1183,11 +1255,12 @@ void destroy_handle_objects(mf_ctx* h) {
   if (h->d_status) cudaFree(h->d_status);
   if (h->gstream) cudaStreamDestroy(h->gstream);
   if (h->sstream) cudaStreamDestroy(h->sstream);
-  for (cudaEvent_t e : {h->ev_in, h->ev_out, h->ev_fork, h->ev_join})
+  if (h->ustream) cudaStreamDestroy(h->ustream);
+  for (cudaEvent_t e : {h->ev_in, h->ev_out, h->ev_fork, h->ev_join, h->ev_u_in, h->ev_u_out})
     if (e) cudaEventDestroy(e);
   h->d_status = nullptr;
-  h->gstream = h->sstream = nullptr;
-  h->ev_in = h->ev_out = h->ev_fork = h->ev_join = nullptr;
+  h->gstream = h->sstream = h->ustream = nullptr;
+  h->ev_in = h->ev_out = h->ev_fork = h->ev_join = h->ev_u_in = h->ev_u_out = nullptr;
 }
 
 }  // namespace
@@ -1266,7 +1339,10 @@ mf_status mf_create(const mf_model_desc* d, mf_handle* out) {
       cudaEventCreateWithFlags(&h->ev_out, cudaEventDisableTiming) != cudaSuccess ||
       cudaStreamCreateWithFlags(&h->sstream, cudaStreamNonBlocking) != cudaSuccess ||
       cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess) {
+      cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&h->ustream, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_u_in, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_u_out, cudaEventDisableTiming) != cudaSuccess) {
     cudaGetLastError();
     destroy_handle_objects(h);
     delete h;
@@ -1523,6 +1599,11 @@ mf_status mf_set_option(mf_handle h, int option, int value) {
   if (option == MF_OPT_FUSED_HEAD) {
     if (value < 0 || value > 1) return fail(h, MF_ERR_INVALID_ARG, "MF_OPT_FUSED_HEAD takes 0 or 1");
     mf::g_fused_head = value;
+    drop_graphs(h);
+    return MF_OK;
+  }
+  if (option == MF_OPT_LAYER_UPDATES) {
+    h->layer_updates = value != 0;
     drop_graphs(h);
     return MF_OK;
   }

@@ -26,7 +26,7 @@ OPTIMIZERS = {"sgd": 0, "adam": 1}
 MF_META_EXAMPLE_WEIGHTS, MF_META_PARAM_LOGLR, MF_META_SCALAR_LOGLR = 1, 2, 4
 MF_HVP_MIXED_FOR, MF_HVP_REV_REV = 0, 1
 (MF_OPT_CUDA_GRAPHS, MF_OPT_PDL, MF_OPT_CONCURRENT, MF_OPT_GEMM_2SM, MF_OPT_FLASH_ATTN,
- MF_OPT_GEMM_PERSISTENT, MF_OPT_FUSED_HEAD) = 1, 2, 3, 4, 5, 6, 7
+ MF_OPT_GEMM_PERSISTENT, MF_OPT_FUSED_HEAD, MF_OPT_LAYER_UPDATES) = 1, 2, 3, 4, 5, 6, 7, 8
 STATUS = {0: "MF_OK", 1: "MF_ERR_INVALID_ARG", 2: "MF_ERR_UNSUPPORTED", 3: "MF_ERR_OOM",
           4: "MF_ERR_CUDA", 5: "MF_ERR_NONFINITE", 6: "MF_ERR_TIMEOUT"}
 
