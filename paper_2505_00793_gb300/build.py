@@ -1,8 +1,8 @@
 """Build the native library ``_lib/libmixflow.so`` in-tree (nvcc, sm_103a only).
 
 Usage: ``python -m paper_2505_00793_gb300.build`` (or ``__graft_entry__.build()``).
-Translation units compile in parallel; the link step produces one shared library with the
-C ABI of ``include/mixflow.h``.  Objects go to ``_build/`` (git-ignored).
+Translation units compile in parallel, longest first; the link step produces one shared
+library with the C ABI of ``include/mixflow.h``.  Objects go to ``_build/`` (git-ignored).
 """
 from __future__ import annotations
 
@@ -18,8 +18,10 @@ CSRC = os.path.join(PKG, "csrc")
 OUT_DIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(OUT_DIR, "libmixflow.so")
 BUILD_DIR = os.path.join(ROOT, "_build")
-SOURCES = ["tc_gemm.cu", "tc_gemm_act.cu", "tc_gemm_persist.cu", "simt_gemm.cu", "kernels.cu",
-           "head_fused.cu", "decoder_kernels.cu", "flash_attn.cu", "capi.cu"]
+SOURCES = ["tc_gemm_act_gelu.cu", "tc_gemm_act_silu.cu", "tc_gemm_act_tanh.cu",
+           "tc_gemm_act_ident.cu", "tc_gemm_persist.cu", "tc_gemm.cu", "tc_gemm_act.cu",
+           "decoder_kernels.cu", "flash_attn.cu", "kernels.cu", "head_fused.cu", "simt_gemm.cu",
+           "capi.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "-I" + os.path.join(ROOT, "include")]

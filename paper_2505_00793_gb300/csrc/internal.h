@@ -58,8 +58,13 @@ struct GemmArgs {
 // tcgen05 bf16 GEMM (tc_gemm.cu).  Returns cudaSuccess or the launch error; sets *why on a
 // host-side rejection (bad alignment/ld) and returns cudaErrorInvalidValue.
 cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why);
-// Activation-epilogue instances (tc_gemm_act.cu), called by tc_gemm.
+// Activation-epilogue instances (tc_gemm_act.cu dispatches to one translation unit per
+// activation, tc_gemm_act_<activation>.cu), called by tc_gemm.
 cudaError_t tc_gemm_act(const GemmArgs& a, cudaStream_t s, const char** why, int bn, int pair);
+cudaError_t tc_gemm_act_ident(const GemmArgs& a, cudaStream_t s, const char** why, int bn, int pair);
+cudaError_t tc_gemm_act_tanh(const GemmArgs& a, cudaStream_t s, const char** why, int bn, int pair);
+cudaError_t tc_gemm_act_gelu(const GemmArgs& a, cudaStream_t s, const char** why, int bn, int pair);
+cudaError_t tc_gemm_act_silu(const GemmArgs& a, cudaStream_t s, const char** why, int bn, int pair);
 // Process-wide choice of 2-SM tiles for GEMMs that leave it automatic: 0 never, 1 when the
 // grid fills the GPU (default), 2 whenever M > 128.
 extern int g_pair_mode;

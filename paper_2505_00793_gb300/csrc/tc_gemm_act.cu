@@ -1,26 +1,21 @@
 // Activation-epilogue instances of the tcgen05 dual GEMM (forward: bias + phi, phi' z';
-// backward: phi' da, phi'' z' da + phi' da').  Kept in their own translation unit so that the
-// instances compile in parallel with the plain-store ones.
-#include "tc_gemm_impl.cuh"
+// backward: phi' da, phi'' z' da + phi' da').  The instances of each activation live in a
+// translation unit of their own (tc_gemm_act_<activation>.cu) so that they compile in
+// parallel; this file dispatches on the epilogue mode and the activation.
+#include "internal.h"
 
 namespace mf {
 
 cudaError_t tc_gemm_act(const GemmArgs& a, cudaStream_t s, const char** why, int bn, int pair) {
-  const int act = a.epi.act;
-  if (a.epi.mode == EPI_ACT_FWD) {
-    switch (act) {
-      case ACT_IDENT: return launch_bn<EPI_ACT_FWD, ACT_IDENT>(a, s, why, bn, pair);
-      case ACT_TANH: return launch_bn<EPI_ACT_FWD, ACT_TANH>(a, s, why, bn, pair);
-      case ACT_GELU: return launch_bn<EPI_ACT_FWD, ACT_GELU>(a, s, why, bn, pair);
-      case ACT_SILU: return launch_bn<EPI_ACT_FWD, ACT_SILU>(a, s, why, bn, pair);
-    }
-  } else if (a.epi.mode == EPI_ACT_BWD) {
-    switch (act) {
-      case ACT_IDENT: return launch_bn<EPI_ACT_BWD, ACT_IDENT>(a, s, why, bn, pair);
-      case ACT_TANH: return launch_bn<EPI_ACT_BWD, ACT_TANH>(a, s, why, bn, pair);
-      case ACT_GELU: return launch_bn<EPI_ACT_BWD, ACT_GELU>(a, s, why, bn, pair);
-      case ACT_SILU: return launch_bn<EPI_ACT_BWD, ACT_SILU>(a, s, why, bn, pair);
-    }
+  if (a.epi.mode != EPI_ACT_FWD && a.epi.mode != EPI_ACT_BWD) {
+    *why = "unknown epilogue mode or activation";
+    return cudaErrorInvalidValue;
+  }
+  switch (a.epi.act) {
+    case ACT_IDENT: return tc_gemm_act_ident(a, s, why, bn, pair);
+    case ACT_TANH: return tc_gemm_act_tanh(a, s, why, bn, pair);
+    case ACT_GELU: return tc_gemm_act_gelu(a, s, why, bn, pair);
+    case ACT_SILU: return tc_gemm_act_silu(a, s, why, bn, pair);
   }
   *why = "unknown epilogue mode or activation";
   return cudaErrorInvalidValue;
