@@ -16,6 +16,8 @@ The parity and count formulas are the kernel's:
              (count 2 x EPI_WARPS)."""
 import random
 
+import numpy as np
+
 import pytest
 
 
@@ -177,3 +179,77 @@ def test_model_catches_planted_mistakes(mistake):
         except (AssertionError, Deadlock):
             caught += 1
     assert eligible > 20 and caught >= 0.9 * eligible, (caught, eligible)
+
+
+# ---- index arithmetic of the persistent kernel ---------------------------------------------
+EPI_WARPS_P, BM, BK = 8, 128, 64
+
+
+def _persist_coverage(M, N, BN, batch, npairs):
+    """Every output element written by the kernel's epilogue mapping, and the TMA boxes each
+    CTA loads, for one launch (the kernel's formulas restated)."""
+    tiles_n = -(-N // BN)
+    pairs_m = -(-M // (2 * BM))
+    ntiles = tiles_n * pairs_m * batch
+    BH = BN // 2
+    written = np.zeros((batch, M, N), np.int32)
+    a_rows, b_rows = set(), set()
+    CG = BN // (EPI_WARPS_P // 4)
+    for pair in range(npairs):
+        for t in range(pair, ntiles, npairs):
+            tn = t % tiles_n
+            r = t // tiles_n
+            mp, bz = r % pairs_m, r // pairs_m
+            for rank in (0, 1):
+                m0 = mp * 2 * BM + rank * BM
+                a_rows.add((bz, m0))
+                b_rows.add((bz, tn * BN + rank * BH))
+                n0 = tn * BN
+                for warp in range(2, 2 + EPI_WARPS_P):
+                    q = warp & 3
+                    c_begin = ((warp - 2) >> 2) * CG
+                    for lane in range(32):
+                        row = m0 + q * 32 + lane
+                        for c in range(c_begin, c_begin + CG, 16):
+                            if n0 + c >= N or row >= M:
+                                continue
+                            cols = [n0 + c + j for j in range(16) if n0 + c + j < N]
+                            written[bz, row, cols] += 1
+    return written, a_rows, b_rows, pairs_m, tiles_n
+
+
+@pytest.mark.parametrize("M,N,BN,batch,npairs", [
+    (256, 128, 128, 1, 1), (300, 520, 128, 1, 3), (1000, 130, 256, 1, 76),
+    (1025, 1024, 256, 1, 7), (600, 1000, 128, 3, 5), (2048, 1024, 128, 1, 76)])
+def test_persistent_tiles_cover_every_output_once(M, N, BN, batch, npairs):
+    written, a_rows, b_rows, pairs_m, tiles_n = _persist_coverage(M, N, BN, batch, npairs)
+    assert (written == 1).all()
+    # A boxes: 128 rows per CTA from every 256-row block; B boxes: BN/2 rows per CTA
+    assert {m for _, m in a_rows} == {mp * 2 * BM + r * BM for mp in range(pairs_m) for r in (0, 1)}
+    assert {n for _, n in b_rows} == {tn * BN + r * BN // 2 for tn in range(tiles_n) for r in (0, 1)}
+    # TMA x coordinates: K offsets i * 64 (bf16: 128-byte multiples); MN-major boxes start at
+    # row offsets that are multiples of 64 elements
+    assert all(m % 64 == 0 for _, m in a_rows) and all(n % 64 == 0 for _, n in b_rows)
+
+
+def test_persistent_tmem_columns_fit():
+    """Accumulator sets and blocks as the launcher sizes them stay inside the 512 TMEM
+    columns it allocates, for every tile width and product count the kernel takes."""
+    def acc_blocks(nlogical, bn):
+        return 4 if nlogical * 4 * bn <= 512 else 2 if nlogical * 2 * bn <= 512 else 1
+
+    def persist_nsub(nacc, bn):
+        for n in (4, 2, 1):
+            if 2 * nacc * n * bn <= 512:
+                return n
+        return acc_blocks(nacc, bn)
+
+    for bn in (128, 256):
+        for nacc in (1, 2):
+            nsub = persist_nsub(nacc, bn)
+            nsets = 2 if 2 * nacc * nsub * bn <= 512 else 1
+            set_cols = nacc * nsub * bn
+            assert nsets * set_cols <= 512
+            # highest column an MMA writes: set (nsets-1), block nacc*nsub-1, BN columns
+            assert (nsets - 1) * set_cols + (nacc * nsub - 1) * bn + bn <= 512
+            assert nsub & (nsub - 1) == 0   # the rotation masks with nsub - 1
