@@ -12,6 +12,10 @@ still move far more than the 129 MB L2 per launch:
 * toy           the motivating example, M = 8 (chain loss kernels), either HVP mode
 * decoder_s1024 two blocks of the larger decoder (d 1024, 16 heads, S = 1024), two
                 sequences: the fused attention at the larger decoder's sequence length
+* wide_small    the wide workload's shapes at T = 2 (256-row GEMMs, the 10-class head)
+
+``--gemm-persistent``, ``--fused-head`` and ``--layer-updates`` set the opt-in paths, so that
+their kernels can be captured on the same cases.
 """
 from __future__ import annotations
 
@@ -30,6 +34,8 @@ def case(name: str):
                                      loglr_mean=math.log(1e-4))
     if name in ("decoder_small", "toy"):
         return synth.WORKLOADS[name]
+    if name == "wide_small":
+        return synth.WORKLOADS["wide"].with_(name="wide_small", T=2)
     if name == "decoder_s1024":
         return synth.decoder("decoder_s1024", 1024, 16, 4096, 2, 32768, 1024, B=2, T=2,
                              B_outer=2, alpha=1e-3)
@@ -43,9 +49,12 @@ def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--case", required=True,
                     choices=["deep_4k", "deep_4k_adam", "decoder_small", "toy",
-                             "decoder_s1024"])
+                             "decoder_s1024", "wide_small"])
     ap.add_argument("--calls", type=int, default=3)
     ap.add_argument("--hvp-mode", type=int, default=0)
+    ap.add_argument("--gemm-persistent", action="store_true")
+    ap.add_argument("--fused-head", action="store_true")
+    ap.add_argument("--layer-updates", action="store_true")
     args = ap.parse_args()
     torch.cuda.set_device(0)
     w = case(args.case)
@@ -53,6 +62,9 @@ def main() -> None:
     d = native.to_device_inputs(w, inp)
     mf = native.MixFlow.for_workload(w)
     mf.set_option(native.MF_OPT_CUDA_GRAPHS, 0)
+    mf.set_option(native.MF_OPT_GEMM_PERSISTENT, 1 if args.gemm_persistent else 0)
+    mf.set_option(native.MF_OPT_FUSED_HEAD, 1 if args.fused_head else 0)
+    mf.set_option(native.MF_OPT_LAYER_UPDATES, 1 if args.layer_updates else 0)
     loop = native.loop_desc_for(w, args.hvp_mode)
     d_eta = torch.empty(w.n_eta, device="cuda")
     d_th = torch.empty(w.n_params, device="cuda")
