@@ -1,7 +1,7 @@
 """Throughput of the tcgen05 dual GEMM (``mf_dual_gemm_bf16``) on the shapes of the
 workloads, next to cuBLAS on one product of the same shape.
 
-``python -m paper_2505_00793_gb300.gemm_bench`` prints one JSON line per shape.  TF/s counts
+``python gemm_bench.py`` prints one JSON line per shape.  TF/s counts
 2*M*N*K per product term; times are CUDA events over back-to-back launches with warm L2.
 """
 from __future__ import annotations

@@ -237,10 +237,27 @@ const char* mf_last_error(mf_handle h);
  * every launch of the bf16 dual GEMM (inside the captured graph when graphs are in use);
  * mf_kernel_time synchronises and returns the summed milliseconds and launch count of that
  * kernel since the last reset - for graph replays, those of the most recent replay - plus
- * its algorithmic flops (2*M*N*K per accumulated product term), then resets. */
+ * its algorithmic flops (2*M*N*K per accumulated product term), then resets.
+ * mf_set_kernel_timing(h, 2) instead records the next call's GEMM launches for
+ * mf_replay_gemms (below); 0 and 1 leave a pending record in place. */
 mf_status mf_stats(mf_handle h, uint64_t* launches, size_t* peak_workspace_bytes);
 mf_status mf_set_kernel_timing(mf_handle h, int enable);
 mf_status mf_kernel_time(mf_handle h, double* ms, uint64_t* launches, double* flops);
+
+/* Roofline timing of the bf16 dual GEMM without perturbing the call.  After
+ * mf_set_kernel_timing(h, 2), the handle's next mf_meta_grad / mf_inner_rollout / mf_hvp runs
+ * eagerly (no graph replay) and records the argument list of every bf16 dual GEMM it
+ * launches.  mf_replay_gemms then launches that list back to back, in the recorded order, as
+ * one captured CUDA graph on `stream`, `reps` times between two CUDA events, and returns the
+ * milliseconds of one replay, the launches per replay and their algorithmic flops
+ * (2*M*N*K per product term and batch entry).  The replay reads and overwrites the handle's
+ * workspace and the buffers the recorded call was given: those must still be allocated, and
+ * the outputs of the recorded call are not preserved.  The record is dropped with the
+ * workspace (mf_release_workspace, a larger call, mf_set_allocator, mf_destroy) and replaced
+ * by the next record.  Synchronises `stream`.  Errors: MF_ERR_INVALID_ARG (no record,
+ * reps < 1), MF_ERR_CUDA. */
+mf_status mf_replay_gemms(mf_handle h, int reps, void* stream, double* ms, uint64_t* launches,
+                          double* flops);
 
 /* Library options.  MF_OPT_CUDA_GRAPHS (default 1): a call of mf_meta_grad, mf_inner_rollout
  * or mf_hvp repeated with the same shapes and pointers is captured into a CUDA graph on its
@@ -289,14 +306,17 @@ mf_status mf_set_option(mf_handle h, int option, int value);
 mf_status mf_inject_fault(mf_handle h, int kind);
 
 /* mf_hvp without any device allocation.  The paper has no counterpart to this call; it
- * exists for callers that cannot allocate device memory: code that enqueues work inside a
- * CUDA stream capture where allocation is not allowed, embedders whose device memory is
- * entirely reserved by their own allocator, and hosts that only accept pre-registered
- * buffers.  It computes exactly what mf_hvp computes (MF_HVP_MIXED_FOR) for the model
- * described by `desc`, without a handle: inputs and outputs are caller-owned device
- * pointers as in mf_hvp, and all intermediate storage lives in one 32 MiB array in the
- * library's device memory (a file-scope __device__ array that every GPU loading the
- * library holds until the process exits).
+ * exists for callers that cannot allocate device memory: embedders whose device memory is
+ * entirely reserved up front by their own allocator (a serving process that claims the GPU
+ * at start-up and forbids later cudaMalloc, because a late allocation can fail or stall
+ * the device), and hosts that only accept pre-registered buffers.  It computes exactly
+ * what mf_hvp computes (MF_HVP_MIXED_FOR) for the MLP described by `desc`, without a
+ * handle: inputs and outputs are caller-owned device pointers as in mf_hvp, and all
+ * intermediate storage lives in one 32 MiB array in the library's device memory (a
+ * file-scope __device__ array that every GPU loading the library holds until the process
+ * exits).
+ *  - MLP models only (every loss an MLP takes, the chain loss included); a decoder
+ *    descriptor (MF_ARCH_DECODER or MF_LOSS_NEXT_TOKEN_CE) returns MF_ERR_UNSUPPORTED.
  *  - Returns MF_ERR_INVALID_ARG when the workspace for (desc, B) exceeds that array
  *    (about 32 MiB; e.g. a [128, 256, 256, 10] MLP at B = 64 needs well under 1 MiB).
  *  - The first call on a device looks up the array's device address (cudaGetSymbolAddress)

@@ -146,20 +146,28 @@ def meta_grad(w, inp, eta=None):
     s_bar = tuple(torch.zeros_like(theta_bar) for _ in range(n_state(w)))
     d_eta = torch.zeros_like(eta0)
     for t in range(w.T - 1, -1, -1):
-        th = thetas[t].clone().requires_grad_(True)
-        st = tuple(v.clone().requires_grad_(True) for v in states[t])
-        et = eta0.clone().requires_grad_(True)
-        with torch.enable_grad():
-            tn, sn = _step(w, th, st, et, X[t], Y[t], t, create_graph=True)
-            grads = torch.autograd.grad((tn, *sn), (th, *st, et), (theta_bar, *s_bar),
-                                        allow_unused=True)
-        theta_bar = grads[0]
-        s_bar = tuple(gs if gs is not None else torch.zeros_like(theta_bar)
-                      for gs in grads[1:-1])
-        ge = grads[-1]
+        theta_bar, s_bar, ge = reverse_step(w, eta0, X[t], Y[t], t, thetas[t], states[t],
+                                            theta_bar, s_bar)
         if ge is not None:
             d_eta = d_eta + ge
     return {"d_eta": d_eta.numpy(), "d_theta0": theta_bar.numpy(), "V": float(V.detach())}
+
+
+def reverse_step(w, eta, x, y, t, theta_t, state_t, theta_bar, s_bar):
+    """One step of Algorithm 1's backward loop: rebuild inner step t at (theta_t, upsilon_t)
+    on a tape whose inner gradient is itself taped (create_graph), and pull the cotangent
+    (theta_bar_{t+1}, upsilon_bar_{t+1}) back through it.  Returns (theta_bar_t,
+    upsilon_bar_t, this step's contribution to d eta, or None)."""
+    th = theta_t.clone().requires_grad_(True)
+    st = tuple(v.clone().requires_grad_(True) for v in state_t)
+    et = eta.clone().requires_grad_(True)
+    with torch.enable_grad():
+        tn, sn = _step(w, th, st, et, x, y, t, create_graph=True)
+        grads = torch.autograd.grad((tn, *sn), (th, *st, et), (theta_bar, *s_bar),
+                                    allow_unused=True)
+    theta_bar = grads[0]
+    s_bar = tuple(gs if gs is not None else torch.zeros_like(theta_bar) for gs in grads[1:-1])
+    return theta_bar, s_bar, grads[-1]
 
 
 def grad(w, theta, x, y, weights=None):

@@ -61,6 +61,13 @@ struct mf_ctx {
   bool timing = false;
   std::vector<std::pair<cudaEvent_t, cudaEvent_t>> evs;
   double timed_flops = 0.0;
+  // GEMM launch record (mf_set_kernel_timing(h, 2)): the bf16 dual GEMMs of the next call in
+  // launch order, with their algorithmic flops; mf_replay_gemms replays them back to back as
+  // one captured graph.  Dropped with the workspace the recorded pointers refer to.
+  bool record = false;
+  std::vector<mf::GemmArgs> rec;
+  double rec_flops = 0.0;
+  cudaGraphExec_t rec_exec = nullptr;
 
   // CUDA graphs: a call repeated with the same shapes and pointers is captured once (on the
   // second occurrence) and replayed from then on, on the library's own stream.
@@ -209,8 +216,29 @@ Plan make_plan(const mf_ctx* h, int rows, int T, int n_theta_slots, int n_m_slot
 
 void drop_graphs(mf_ctx* h);
 
+void drop_record(mf_ctx* h) {
+  if (h->rec_exec) cudaGraphExecDestroy(h->rec_exec);
+  h->rec_exec = nullptr;
+  h->rec.clear();
+  h->rec_flops = 0.0;
+}
+
+// Algorithmic flops of one GEMM launch: 2 M N K per accumulated product term and batch entry.
+double gemm_flops(const GemmArgs& g) {
+  return 2.0 * g.M * g.N * static_cast<double>(g.K) * mf::term_count(g.terms) *
+         (g.batch > 1 ? g.batch : 1);
+}
+
+// Called by the executors for every tensor-core GEMM they launch.
+void note_gemm(mf_ctx* h, const GemmArgs& g) {
+  if (!h->record) return;
+  h->rec.push_back(g);
+  h->rec_flops += gemm_flops(g);
+}
+
 void release_ws(mf_ctx* h) {
   drop_graphs(h);
+  drop_record(h);
   if (!h->ws) return;
   cudaDeviceSynchronize();
   if (h->ufree) h->ufree(h->ws, h->ws_bytes, nullptr, h->uctx);
@@ -281,6 +309,20 @@ mf_status run_graphed(mf_ctx* h, mf_ctx::GraphCache& g, uint64_t key, cudaStream
   key = mix_key(key, reinterpret_cast<uintptr_t>(h->ws));
   key = mix_key(key, h->ws_bytes);
   key = mix_key(key, h->timing ? 1 : 0);
+  // Process-wide options change which kernels a call launches; another handle may have set
+  // them since this handle captured its graphs, so they are part of every graph's key.
+  key = mix_key(key, static_cast<uint64_t>(mf::g_pdl));
+  key = mix_key(key, static_cast<uint64_t>(mf::g_pair_mode));
+  key = mix_key(key, static_cast<uint64_t>(mf::g_gemm_persist));
+  key = mix_key(key, static_cast<uint64_t>(mf::g_fused_head));
+  if (h->record) {
+    // one eager execution whose GEMM launches are recorded for mf_replay_gemms
+    drop_record(h);
+    h->record = true;
+    const mf_status st = body(user);
+    h->record = false;
+    return st;
+  }
   if (!h->use_graphs || !h->gstream) return body(user);
   if (g.exec && g.key == key) return graph_launch(h, g, user);
   if (g.pending != key) {
@@ -440,10 +482,11 @@ struct Exec {
       return;
     }
     launched();
+    if (tc) note_gemm(h, g);
     if (tc && h->timing) {
       cudaEventRecordWithFlags(e1, s, ev_flags);
       h->evs.emplace_back(e0, e1);
-      h->timed_flops += 2.0 * g.M * g.N * static_cast<double>(g.K) * mf::term_count(g.terms);
+      h->timed_flops += gemm_flops(g);
     }
   }
 
@@ -1532,8 +1575,64 @@ mf_status mf_stats(mf_handle h, uint64_t* launches, size_t* peak) {
 }
 
 mf_status mf_set_kernel_timing(mf_handle h, int enable) {
-  if (!h) return MF_ERR_INVALID_ARG;
+  if (!h || enable < 0 || enable > 2) return MF_ERR_INVALID_ARG;
+  if (enable == 2) {
+    h->record = true;
+    return MF_OK;
+  }
   h->timing = enable != 0;
+  return MF_OK;
+}
+
+mf_status mf_replay_gemms(mf_handle h, int reps, void* stream, double* ms, uint64_t* launches,
+                          double* flops) {
+  if (!h || reps < 1) return MF_ERR_INVALID_ARG;
+  if (h->rec.empty()) return fail(h, MF_ERR_INVALID_ARG, "no recorded GEMM launches");
+  if (!h->gstream) return fail(h, MF_ERR_UNSUPPORTED, "no library stream for the capture");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (!h->rec_exec) {
+    MF_CUDA(h, cudaStreamBeginCapture(h->gstream, cudaStreamCaptureModeThreadLocal));
+    cudaError_t le = cudaSuccess;
+    const char* why = "";
+    for (const GemmArgs& g : h->rec) {
+      le = mf::tc_gemm(g, h->gstream, &why);
+      if (le != cudaSuccess) break;
+    }
+    cudaGraph_t graph = nullptr;
+    const cudaError_t ce = cudaStreamEndCapture(h->gstream, &graph);
+    if (le != cudaSuccess || ce != cudaSuccess || !graph) {
+      if (graph) cudaGraphDestroy(graph);
+      cudaGetLastError();
+      return fail(h, MF_ERR_CUDA, std::string("GEMM replay capture failed: ") +
+                                      cudaGetErrorString(le != cudaSuccess ? le : ce) + " " + why);
+    }
+    const cudaError_t ie = cudaGraphInstantiate(&h->rec_exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (ie != cudaSuccess) {
+      h->rec_exec = nullptr;
+      cudaGetLastError();
+      return fail(h, MF_ERR_CUDA, std::string("GEMM replay instantiate failed: ") + cudaGetErrorString(ie));
+    }
+  }
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  MF_CUDA(h, cudaEventCreate(&e0));
+  if (cudaEventCreate(&e1) != cudaSuccess) {
+    cudaEventDestroy(e0);
+    return fail(h, MF_ERR_CUDA, "event creation failed");
+  }
+  cudaError_t e = cudaEventRecord(e0, s);
+  for (int r = 0; r < reps && e == cudaSuccess; ++r) e = cudaGraphLaunch(h->rec_exec, s);
+  if (e == cudaSuccess) e = cudaEventRecord(e1, s);
+  if (e == cudaSuccess) e = cudaEventSynchronize(e1);
+  float t = 0.f;
+  if (e == cudaSuccess) e = cudaEventElapsedTime(&t, e0, e1);
+  cudaEventDestroy(e0);
+  cudaEventDestroy(e1);
+  if (e != cudaSuccess) return fail(h, MF_ERR_CUDA, std::string("GEMM replay: ") + cudaGetErrorString(e));
+  h->launches += static_cast<uint64_t>(reps) * h->rec.size();
+  if (ms) *ms = static_cast<double>(t) / reps;
+  if (launches) *launches = h->rec.size();
+  if (flops) *flops = h->rec_flops;
   return MF_OK;
 }
 
@@ -1655,10 +1754,10 @@ mf_status mf_dual_gemm_bf16(int M, int N, int K, const void* A0, int lda0, const
 }  // extern "C"
 
 // ================================ no-allocation HVP =======================================
-// Callers that cannot allocate device memory - code running inside a CUDA graph capture
-// that forbids allocation, embedders whose memory is fully pre-reserved by another
-// allocator, or hosts that only hand out pre-registered buffers - use mf_hvp_noalloc.  Its
-// workspace is one file-scope device array; nothing is allocated per call or per handle.
+// Callers that cannot allocate device memory - embedders whose memory is fully reserved up
+// front by their own allocator, or hosts that only hand out pre-registered buffers - use
+// mf_hvp_noalloc.  Its workspace is one file-scope device array; nothing is allocated per
+// call or per handle.
 namespace {
 
 constexpr size_t kNoAllocScratchBytes = static_cast<size_t>(32) << 20;   // 32 MiB

@@ -247,11 +247,11 @@ struct DecExec {
       return;
     }
     launched();
+    if (tc) note_gemm(h, g);
     if (tc && h->timing) {
       cudaEventRecordWithFlags(e1, s, ev_flags);
       h->evs.emplace_back(e0, e1);
-      h->timed_flops += 2.0 * g.M * g.N * static_cast<double>(g.K) * mf::term_count(g.terms) *
-                        (g.batch > 1 ? g.batch : 1);
+      h->timed_flops += gemm_flops(g);
     }
   }
 

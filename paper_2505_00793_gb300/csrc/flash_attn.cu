@@ -608,18 +608,18 @@ constexpr int SMEM_FWD1 = 6 * TILE_ELEMS * 2, SMEM_FWD0 = 3 * TILE_ELEMS * 2;
 constexpr int SMEM_KV1 = 8 * TILE_ELEMS * 2 + 4 * FT * 4, SMEM_KV0 = 4 * TILE_ELEMS * 2 + 4 * FT * 4;
 constexpr int SMEM_Q1 = 8 * TILE_ELEMS * 2, SMEM_Q0 = 4 * TILE_ELEMS * 2;
 
-// Dynamic shared-memory limits of all six kernels, once per process (before any capture:
+// Dynamic shared-memory limits of all six kernels, once per device (before any capture:
 // the first call of a captured sequence runs eagerly).
 void init_attributes() {
-  static std::once_flag once;
-  std::call_once(once, [] {
+  static PerDeviceOnce once;
+  once.run([](int&) {
     const auto a = cudaFuncAttributeMaxDynamicSharedMemorySize;
     cudaFuncSetAttribute(flash_fwd_kernel<true>, a, SMEM_FWD1);
     cudaFuncSetAttribute(flash_fwd_kernel<false>, a, SMEM_FWD0);
     cudaFuncSetAttribute(flash_bwd_kv_kernel<true>, a, SMEM_KV1);
     cudaFuncSetAttribute(flash_bwd_kv_kernel<false>, a, SMEM_KV0);
     cudaFuncSetAttribute(flash_bwd_q_kernel<true>, a, SMEM_Q1);
-    cudaFuncSetAttribute(flash_bwd_q_kernel<false>, a, SMEM_Q0);
+    return cudaFuncSetAttribute(flash_bwd_q_kernel<false>, a, SMEM_Q0);
   });
 }
 

@@ -5,7 +5,39 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include <mutex>
+
 namespace mf {
+
+// Kernel attributes (cudaFuncSetAttribute) and occupancy figures belong to one device: a
+// process that drives several GPUs sets and measures them once per device.  One instance per
+// call site (a function-local static of the launching template), guarded by its own mutex.
+constexpr int kMaxDevices = 64;
+struct PerDeviceOnce {
+  std::mutex mu;
+  bool done[kMaxDevices] = {};
+  int value[kMaxDevices] = {};
+  // Runs f() -> cudaError_t on the current device unless it already succeeded there.
+  template <typename F>
+  cudaError_t run(F&& f) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    if (done[dev]) return cudaSuccess;
+    e = f(value[dev]);
+    if (e == cudaSuccess) done[dev] = true;
+    return e;
+  }
+  // The value that f stored on the current device (0 before the first success).
+  int get() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 0;
+    std::lock_guard<std::mutex> lock(mu);
+    return value[dev];
+  }
+};
 
 // Device status word values (also the mf_status codes they map to).
 enum : int { DEV_OK = 0, DEV_NONFINITE = 5, DEV_TIMEOUT = 6 };

@@ -961,12 +961,13 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
   }
   if (p.tma_store && EPI_WARPS * STG_WARP > need) need = EPI_WARPS * STG_WARP;
   const int smem = need + 1024;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(tc_dual_gemm_kernel<BN, KA, MODE, ACT>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, 225 * 1024);
+  static PerDeviceOnce attr_once;
+  {
+    cudaError_t e = attr_once.run([](int&) {
+      return cudaFuncSetAttribute(tc_dual_gemm_kernel<BN, KA, MODE, ACT>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, 225 * 1024);
+    });
     if (e != cudaSuccess) return e;
-    attr_set = true;
   }
   if (smem > 225 * 1024) { *why = "shared memory budget exceeded"; return cudaErrorInvalidValue; }
   cudaLaunchConfig_t cfg;
@@ -1230,12 +1231,13 @@ cudaError_t launch_cfg2(const GemmArgs& a, cudaStream_t s, const char** why) {
   int need = stages * off;
   if (p.tma_store && EPI_WARPS2 * STG_WARP > need) need = EPI_WARPS2 * STG_WARP;
   const int smem = need + 1024;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(tc2_dual_gemm_kernel<BN, MODE, ACT>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, 225 * 1024);
+  static PerDeviceOnce attr_once;
+  {
+    cudaError_t e = attr_once.run([](int&) {
+      return cudaFuncSetAttribute(tc2_dual_gemm_kernel<BN, MODE, ACT>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, 225 * 1024);
+    });
     if (e != cudaSuccess) return e;
-    attr_set = true;
   }
   if (smem > 225 * 1024) { *why = "shared memory budget exceeded"; return cudaErrorInvalidValue; }
   cudaLaunchConfig_t cfg;

@@ -353,11 +353,10 @@ __global__ void __launch_bounds__(THREADS_P, 1)
   }
 }
 
-// Co-resident CTA pairs of one kernel instance (cluster occupancy), cached per instance.
+// Co-resident CTA pairs of one kernel instance (cluster occupancy), measured once per
+// device and instance.
 template <int BN, int MODE, int ACT>
-int max_pairs(int smem) {
-  static int cached = 0;
-  if (cached > 0) return cached;
+int max_pairs_on_device(int smem) {
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -382,8 +381,18 @@ int max_pairs(int smem) {
   else
     cudaGetLastError();   // clear the query's error; keep the SM-count estimate
   if (pairs < 1) pairs = 1;
-  cached = pairs;
   return pairs;
+}
+
+template <int BN, int MODE, int ACT>
+int max_pairs(int smem) {
+  static PerDeviceOnce once;
+  once.run([smem](int& v) {
+    v = max_pairs_on_device<BN, MODE, ACT>(smem);
+    return cudaSuccess;
+  });
+  const int v = once.get();
+  return v > 0 ? v : 1;
 }
 
 template <int BN, int MODE, int ACT>
@@ -445,12 +454,13 @@ cudaError_t launch_cfg2p(const GemmArgs& a, cudaStream_t s, const char** why) {
   pp.set_cols = nacc * p.nsub * BN;
 
   const int smem = stages * off + 1024;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(tc2p_dual_gemm_kernel<BN, MODE, ACT>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, 225 * 1024);
+  static PerDeviceOnce attr_once;
+  {
+    cudaError_t e = attr_once.run([](int&) {
+      return cudaFuncSetAttribute(tc2p_dual_gemm_kernel<BN, MODE, ACT>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, 225 * 1024);
+    });
     if (e != cudaSuccess) return e;
-    attr_set = true;
   }
   if (smem > 225 * 1024) { *why = "shared memory budget exceeded"; return cudaErrorInvalidValue; }
   int npairs = max_pairs<BN, MODE, ACT>(225 * 1024);

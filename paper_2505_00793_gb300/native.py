@@ -35,7 +35,7 @@ EXPORTS = ["mf_create", "mf_destroy", "mf_set_allocator", "mf_param_count",
            "mf_workspace_bytes", "mf_release_workspace", "mf_inner_rollout", "mf_hvp",
            "mf_meta_grad", "mf_sync", "mf_status_string", "mf_last_error", "mf_stats",
            "mf_set_kernel_timing", "mf_kernel_time", "mf_inject_fault", "mf_dual_gemm_bf16",
-           "mf_hvp_noalloc", "mf_set_option"]
+           "mf_hvp_noalloc", "mf_set_option", "mf_replay_gemms"]
 
 
 class mf_model_desc(C.Structure):
@@ -82,6 +82,7 @@ def load(path: str = LIB_PATH) -> C.CDLL:
         "mf_stats": ([H, u64p, szp], C.c_int),
         "mf_set_kernel_timing": ([H, C.c_int], C.c_int),
         "mf_kernel_time": ([H, dblp, u64p, dblp], C.c_int),
+        "mf_replay_gemms": ([H, C.c_int, vp, dblp, u64p, dblp], C.c_int),
         "mf_inject_fault": ([H, C.c_int], C.c_int),
         "mf_set_option": ([H, C.c_int, C.c_int], C.c_int),
         "mf_hvp_noalloc": ([C.POINTER(mf_model_desc), C.c_int, vp, vp, vp, vp, vp, vp, vp, vp, vp],
@@ -289,6 +290,38 @@ class MixFlow:
         self._check(self._lib.mf_kernel_time(self.h, C.byref(ms), C.byref(n), C.byref(fl)),
                     "mf_kernel_time")
         return ms.value, n.value, fl.value
+
+    def record_gemms(self):
+        """Record the bf16 dual GEMM launches of the next call (mf_set_kernel_timing(h, 2))."""
+        self._check(self._lib.mf_set_kernel_timing(self.h, 2), "mf_set_kernel_timing")
+
+    def replay_gemms(self, reps: int = 1, stream=None):
+        """(ms of one back-to-back replay of the recorded GEMMs, launches, flops)."""
+        ms, n, fl = C.c_double(), C.c_uint64(), C.c_double()
+        self._check(self._lib.mf_replay_gemms(self.h, reps, _stream(stream), C.byref(ms),
+                                              C.byref(n), C.byref(fl)), "mf_replay_gemms")
+        return ms.value, n.value, fl.value
+
+    def set_torch_allocator(self):
+        """Route the handle's workspace through PyTorch's caching allocator (mf_set_allocator),
+        so that torch.cuda.max_memory_allocated() sees it."""
+        import torch
+
+        @C.CFUNCTYPE(C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p)
+        def _alloc(nbytes, stream, ctx):
+            try:
+                return torch.cuda.caching_allocator_alloc(int(nbytes), stream=stream or 0)
+            except Exception:
+                return None
+
+        @C.CFUNCTYPE(None, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p)
+        def _free(ptr, nbytes, stream, ctx):
+            torch.cuda.caching_allocator_delete(ptr)
+
+        self._alloc_cbs = (_alloc, _free)   # kept alive with the handle
+        self._check(self._lib.mf_set_allocator(self.h, C.cast(_alloc, C.c_void_p),
+                                               C.cast(_free, C.c_void_p), None),
+                    "mf_set_allocator")
 
     def set_option(self, option: int, value: int):
         self._check(self._lib.mf_set_option(self.h, option, value), "mf_set_option")

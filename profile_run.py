@@ -1,6 +1,6 @@
 """Run mf_meta_grad a few times on a named case, for capturing kernels under ncu.
 
-``python -m paper_2505_00793_gb300.profile_run --case NAME [--calls N]`` prints the kernel
+``python profile_run.py --case NAME [--calls N]`` prints the kernel
 launches of one call (from mf_stats) and runs N eager calls (CUDA graphs off, so every launch
 is visible).  The cases keep the device footprint at a few GB while the HBM-bound kernels
 still move far more than the 129 MB L2 per launch:

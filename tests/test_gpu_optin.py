@@ -8,12 +8,7 @@
   oracle at the default path's tolerances.
 - MF_OPT_LAYER_UPDATES: per-layer updates on the update stream; the same update element for
   element, so meta-gradients are bit-identical to the single update (eager, captured and
-  replayed calls).
-
-These paths have not yet run on a GPU; the module runs only with MF_TEST_OPT_IN=1 in the
-environment until they have."""
-import os
-
+  replayed calls)."""
 import numpy as np
 import pytest
 
@@ -23,10 +18,6 @@ from oracle import metagrad as om
 import test_gpu_adam as ta
 import test_gpu_gemm as tg
 import test_gpu_parity as tp
-
-pytestmark = pytest.mark.skipif(os.environ.get("MF_TEST_OPT_IN") != "1",
-                                reason="opt-in paths run with MF_TEST_OPT_IN=1")
-
 
 def _set(native, option, value):
     """Process-wide options; any handle can set them."""

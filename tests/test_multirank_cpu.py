@@ -80,33 +80,68 @@ def test_single_rank_needs_no_process_group():
     assert bench._replica_workload(w, 0) is w
 
 
-def test_reference_line_contract(monkeypatch):
+def _ref_args(**kw):
+    a = {"warmup": 0, "steps": 1, "gpus": 1}
+    a.update(kw)
+    return type("A", (), a)()
+
+
+def _tiny_large_decoder():
+    """A tiny decoder under the name of the sampled workload (same code path, seconds)."""
+    from paper_2505_00793_gb300 import synth
+    return synth.decoder("decoder_large", 16, 2, 32, 2, 32, 8, B=2, T=3, B_outer=2,
+                         momentum=0.9, meta_kind=synth.EXAMPLE_WEIGHTS | synth.SCALAR_LOGLR)
+
+
+@pytest.mark.parametrize("sampled", [True, False])
+def test_reference_line_contract(monkeypatch, sampled):
     """``--impl reference`` prints one JSON line with the contract's keys (the oracle timed on
-    a tiny stand-in workload here, to keep the CPU suite short)."""
+    a tiny stand-in workload here, to keep the CPU suite short); its per-step time times the
+    step count is the timed wall time."""
     sys.path.insert(0, ROOT)
     import bench
     from paper_2505_00793_gb300 import synth
-    monkeypatch.setitem(synth.WORKLOADS, bench.WORKLOAD, synth.WORKLOADS["tiny"].with_(T=16))
+    w = _tiny_large_decoder() if sampled else synth.WORKLOADS["tiny"].with_(T=16)
+    monkeypatch.setitem(synth.WORKLOADS, bench.WORKLOAD, w)
     out = io.StringIO()
     with redirect_stdout(out):
-        rc = bench.run_reference(type("A", (), {"warmup": 0, "steps": 1, "gpus": 1})())
+        rc = bench.run_reference(_ref_args(workload=bench.WORKLOAD, steps=4, warmup=1))
     assert rc == 0
     d = json.loads(out.getvalue().strip().splitlines()[-1])
     assert d["impl"] == "reference" and d["unit"] == "meta-steps/s" and d["value"] > 0
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["value"] == d["value"]
-    assert d["higher_is_better"] is True
+    assert d["higher_is_better"] is True and d["steps"] == 4
+    if sampled:
+        assert d["ms_per_step"] * 4 / 1000.0 <= d["timed_wall_s"] * 1.05 + 0.05
 
 
-def test_cpu_baseline_repeats_to_its_minimum_time():
-    """The CPU baseline repeats the oracle until the requested CPU time is spent and reports
-    the mean per meta-gradient."""
+def test_cpu_baseline_whole_oracle_repeats_to_its_minimum_time():
     sys.path.insert(0, ROOT)
     import bench
     from paper_2505_00793_gb300 import synth
-    w = synth.WORKLOADS["tiny"]
-    full, spent, cores, runs = bench.cpu_oracle_time(w, min_seconds=0.2)
-    assert runs >= 2 and spent >= 0.2 and cores >= 1
-    assert abs(full - spent / runs) <= 1e-12 * spent
-    full1, spent1, _, runs1 = bench.cpu_oracle_time(w)
-    assert runs1 == 1 and full1 == spent1
+    c = bench.cpu_baseline(synth.WORKLOADS["tiny"], min_seconds=0.2)
+    assert c["kind"] == "oracle" and c["value"] > 0 and c["cores"] >= 1
+    assert "whole oracle meta-gradients" in c["sample"]
+
+
+def test_cpu_baseline_units_scale_to_a_meta_step(monkeypatch):
+    """The sampled baseline: one unit of each kind, meta-step time B T (rollout + reverse)
+    + B_outer outer."""
+    sys.path.insert(0, ROOT)
+    import bench
+    w = _tiny_large_decoder()
+    calls = []
+
+    def fake_unit(w_, kind):
+        calls.append(kind)
+        return {"rollout": 0.5, "reverse": 1.5, "outer": 0.25}[kind]
+
+    monkeypatch.setattr(bench, "oracle_unit", fake_unit)
+    c = bench.cpu_baseline(w)
+    assert sorted(calls) == sorted(bench.UNIT_KINDS)
+    assert c["value"] == pytest.approx(1.0 / (w.B * w.T * 2.0 + w.B_outer * 0.25))
+    # the real units run on one sequence of one step
+    monkeypatch.undo()
+    for k in bench.UNIT_KINDS:
+        assert bench.oracle_unit(w, k) > 0

@@ -1,7 +1,8 @@
 """mf_hvp_noalloc: the Hessian-vector product for callers that cannot allocate device
-memory (stream captures that forbid allocation, embedders with fully reserved memory).  Its
-outputs must match mf_hvp's on the same inputs, on two calls in a row (the second call
-finds the first call's leftovers in the shared static workspace).
+memory (embedders whose memory is fully reserved up front by their own allocator, hosts that
+only accept pre-registered buffers).  Its outputs must match mf_hvp's on the same inputs, on
+two calls in a row (the second call finds the first call's leftovers in the shared static
+workspace).
 
 Collected last on purpose: if it fails, a run stopping at the first failure has already
 run every other test."""
@@ -15,12 +16,16 @@ from paper_2505_00793_gb300 import synth
 
 
 @pytest.mark.gpu
-@pytest.mark.parametrize("case", ["bf16", "fp32"])
+@pytest.mark.parametrize("case", ["bf16", "fp32", "chain_bf16"])
 def test_hvp_noalloc_matches_hvp(case):
     torch, native = need_gpu()
     if case == "bf16":
         w = synth.Workload("noalloc_bf16", [128, 256, 136, 10], "gelu", "ce", "bf16", B=64, T=1,
                            B_outer=8, alpha=0.05)
+        tol = 2e-2
+    elif case == "chain_bf16":
+        # the motivating example's chain loss (Eq. 8), M = 3, on a 256-wide map
+        w = synth.toy("noalloc_chain", 256, 96, 3, T=1, precision="bf16", init_std=1.0 / 16.0)
         tol = 2e-2
     else:
         w = synth.Workload("noalloc_fp32", [40, 70, 3], "tanh", "squared", "fp32", B=33, T=1,
@@ -67,3 +72,14 @@ def test_hvp_noalloc_rejects_oversize():
     p = C.c_void_p(dummy.data_ptr())
     st = native.lib().mf_hvp_noalloc(C.byref(desc), w.B, p, p, p, None, p, p, None, None, None)
     assert st == 1   # MF_ERR_INVALID_ARG: the workspace would exceed the static array
+
+
+@pytest.mark.gpu
+def test_hvp_noalloc_rejects_decoder():
+    torch, native = need_gpu()
+    w = synth.decoder("dec_noalloc", 64, 1, 128, 1, 200, 64, B=2, T=1, B_outer=2, alpha=1e-2)
+    desc = native.model_desc_for(w)
+    dummy = torch.zeros(16, device="cuda")
+    p = C.c_void_p(dummy.data_ptr())
+    st = native.lib().mf_hvp_noalloc(C.byref(desc), w.B, p, p, p, None, p, p, None, None, None)
+    assert st == 2   # MF_ERR_UNSUPPORTED: decoders need mf_hvp and a handle
