@@ -24,7 +24,8 @@ Multi-GPU runs are independent replicas (weak scaling), one process per GPU unde
 ``--workload`` measures another configuration the same way (wide and deep MLPs, the small
 transformer, the motivating example of Section 3 with ``--chain-steps M``).
 ``--hvp-mode rr`` runs the reverse-over-reverse sweep instead of the mixed-mode one.
-``--ckpt-every k`` keeps the theta_t store in segments of k steps, and ``--optimizer adam``
+``--ckpt-every k`` keeps the theta_t store in segments of k steps, ``--ckpt-slots s`` in the
+binomial schedule with s snapshots, and ``--optimizer adam``
 replaces the workload's SGD / momentum by Adam. Those lines skip the CPU baseline unless
 ``--cpu-baseline`` is given.
 """
@@ -330,11 +331,17 @@ def run_reference(args):
     return 0
 
 
-def _static_bytes(w, ckpt_every, inputs_bytes, out_bytes):
+def _static_bytes(w, ckpt_every, inputs_bytes, out_bytes, ckpt_slots=0):
     """Section 4's static memory: the theta_t store (and the m_t store when the learning rate
-    is a meta-parameter, m_t and v_t with Adam), the inputs, eta and the meta-gradient."""
+    is a meta-parameter, m_t and v_t with Adam), the inputs, eta and the meta-gradient.  With
+    the binomial store: its s + 3 states (theta, m when kept, v with Adam)."""
     from paper_2505_00793_gb300 import synth
     lr_meta = bool(w.meta_kind & (synth.PARAM_LOGLR | synth.SCALAR_LOGLR))
+    if ckpt_slots > 0:
+        n = min(ckpt_slots, max(w.T - 1, 1)) + 3
+        per = 1 + (1 if (lr_meta or w.momentum != 0 or w.optimizer == "adam") else 0) + \
+            (1 if w.optimizer == "adam" else 0)
+        return n * per * w.n_params * 4 + inputs_bytes + out_bytes
     k = min(max(ckpt_every, 1), w.T)
     if w.optimizer == "adam":       # m_t and v_t for every t (their cotangents are dynamic)
         m_slots = 2 * (w.T // k + k - 1)
@@ -373,7 +380,7 @@ def run_gpu(args):
         mf.set_option(native.MF_OPT_LAYER_UPDATES, 1)
     rr = args.hvp_mode == "rr"
     mode = native.MF_HVP_REV_REV if rr else native.MF_HVP_MIXED_FOR
-    loop = native.loop_desc_for(w, mode, ckpt_every=args.ckpt_every)
+    loop = native.loop_desc_for(w, mode, ckpt_every=args.ckpt_every, ckpt_slots=args.ckpt_slots)
     d_eta = torch.empty(w.n_eta, device="cuda")
     # the meta-gradient lands in d_eta, or in d theta_0 when theta_0 is the meta-parameter
     d_th = torch.empty(w.n_params, device="cuda") if w.n_eta == 0 else None
@@ -395,7 +402,8 @@ def run_gpu(args):
     step()
     mf.sync()
     total_b = torch.cuda.max_memory_allocated()
-    static_b = _static_bytes(w, args.ckpt_every, inputs_bytes, d_out.numel() * 4 + 4)
+    static_b = _static_bytes(w, args.ckpt_every, inputs_bytes, d_out.numel() * 4 + 4,
+                             args.ckpt_slots)
 
     flush = torch.empty(256 * 1024 * 1024 // 4, device="cuda")   # > 129 MB L2
     for _ in range(max(args.warmup, 3)):
@@ -476,7 +484,8 @@ def run_gpu(args):
     # reverse-over-reverse sweep (or of the mixed mode, when rr is the benchmarked one) with
     # peak HBM measured the same way, and its meta-gradient next to this one ----------------
     other = native.MF_HVP_MIXED_FOR if rr else native.MF_HVP_REV_REV
-    loop_o = native.loop_desc_for(w, other, ckpt_every=args.ckpt_every)
+    loop_o = native.loop_desc_for(w, other, ckpt_every=args.ckpt_every,
+                                  ckpt_slots=args.ckpt_slots)
     del flush
     mf.release_workspace()
     torch.cuda.synchronize()
@@ -512,6 +521,9 @@ def run_gpu(args):
                           if args.chain_steps is not None else "")
                        + (f"; checkpoint store in segments of {args.ckpt_every} steps"
                           if args.ckpt_every > 1 else "")
+                       + (f"; binomial checkpoint store with {args.ckpt_slots} snapshots "
+                          f"({native.checkpoint_plan(w.T, 1, args.ckpt_slots)[1]} inner steps "
+                          "recomputed)" if args.ckpt_slots > 0 else "")
                        + (f"; Adam inner optimiser (b1 0.9, b2 0.999, eps {args.adam_eps:g}) "
                           "in place of SGD" if args.optimizer == "adam" else "")
                        + ("; CTA-pair GEMMs as persistent kernels"
@@ -574,6 +586,8 @@ def main():
     ap.add_argument("--optimizer", default="sgd", choices=["sgd", "adam"],
                     help="inner optimiser (adam replaces the workload's SGD / momentum)")
     ap.add_argument("--adam-eps", type=float, default=1e-8)
+    ap.add_argument("--ckpt-slots", type=int, default=0,
+                    help="binomial checkpointing with this many snapshots (0 = off)")
     ap.add_argument("--ckpt-every", type=int, default=1,
                     help="segment length of the theta_t store (1 = keep every theta_t)")
     ap.add_argument("--gemm-persistent", action="store_true",

@@ -151,7 +151,17 @@ typedef struct {
  *             the cotangents of m_{t+1}, v_{t+1}; g_t is recovered as (m_{t+1} - b1 m_t)/(1-b1).
  *             The store keeps m_t and v_t for every t (segmented like theta) plus two
  *             cotangent vectors: 2 (floor(T/k) + k - 1) + 2 extra |theta| slots.
- *  beta1, beta2, adam_eps  Adam's decays in [0, 1) and epsilon (> 0); ignored for SGD. */
+ *  beta1, beta2, adam_eps  Adam's decays in [0, 1) and epsilon (> 0); ignored for SGD.
+ *  ckpt_slots s (0 = off; 1..1024, exclusive with ckpt_every > 1; T <= 4096): binomial
+ *             checkpointing (Section 4's "binomial checkpointing", Griewank's revolve).  The
+ *             store keeps s + 3 states (theta_t, plus m_t whenever momentum, a learned
+ *             learning rate or Adam needs it, plus v_t with Adam): S_0, s snapshots and two
+ *             scratch states; the rollout leaves snapshots on its way, and the sweep
+ *             recomputes every other state forward from a snapshot, following the schedule
+ *             that re-runs the fewest inner steps for s snapshots (dynamic programming over
+ *             the split points; mf_checkpoint_plan reports it).  The same kernels recompute
+ *             the same values, so results are bit-identical to ckpt_every = 1.  Adam adds two
+ *             |theta| buffers for a deferred reverse step.  s >= T - 1 stores every state. */
 typedef struct {
   int T, B, B_outer;
   float alpha, momentum;
@@ -160,6 +170,7 @@ typedef struct {
   int ckpt_every;
   int optimizer;
   float beta1, beta2, adam_eps;
+  int ckpt_slots;
 } mf_loop_desc;
 
 /* Create a handle for one inner-model architecture.  *out receives a library-owned handle.
@@ -183,6 +194,16 @@ mf_status mf_param_count(mf_handle h, const mf_loop_desc* loop, int64_t* n_param
 /* Bytes of workspace mf_meta_grad needs for `loop` (checkpoint store + activations; with
  * MF_HVP_REV_REV also the stored inner backward graph). */
 mf_status mf_workspace_bytes(mf_handle h, const mf_loop_desc* loop, size_t* bytes);
+
+/* Checkpoint plan of a reverse sweep over T inner steps, host-only (no handle, no device):
+ * *state_slots receives the number of stored states (theta_t, each with its optimiser state
+ * where kept) and *recompute_steps the inner steps the sweep re-runs forward, for
+ * ckpt_every = k (uniform segments; 0 or 1 = every state) or ckpt_slots = s > 0 (binomial;
+ * then k must be 0 or 1).  State slots: T + 1 for k = 1; floor(T/k) + k for k > 1 (re-runs
+ * about one rollout); s + 3 for the binomial schedule, with the fewest re-runs for s.
+ * Errors: MF_ERR_INVALID_ARG (T < 1, negative or conflicting k and s, T > 4096 with s). */
+mf_status mf_checkpoint_plan(int T, int ckpt_every, int ckpt_slots, int* state_slots,
+                             int64_t* recompute_steps);
 
 /* Free the cached workspace now (the next call allocates it again). */
 mf_status mf_release_workspace(mf_handle h);
@@ -294,10 +315,18 @@ mf_status mf_replay_gemms(mf_handle h, int reps, void* stream, double* ms, uint6
  * layer on a library stream of the handle, each as soon as its layer's products in the
  * backward pass are done, so that they overlap the layers below instead of following the
  * whole pass.  Element for element the same update.  Decoders and the reverse-over-reverse
- * sweep keep the single update.  Setting it drops the handle's captured graphs. */
+ * sweep keep the single update.  Setting it drops the handle's captured graphs.
+ * MF_OPT_WAIT_LIMIT_US (process-wide, default 2000000 = 2 s; 0..60000000): how long the
+ * tensor-core GEMMs' MMA issuer and epilogue wait for a pipeline stage or an accumulator
+ * before giving up (failure detection: a wait that gives up sets the device status word to
+ * MF_ERR_TIMEOUT, reported by mf_sync).  After giving up, a CTA stops issuing MMAs, lets the
+ * loads and MMAs it already issued complete, and ends; its outputs are then undefined.  A
+ * short limit makes waits give up on a healthy GPU, which tests use.  Takes effect at the
+ * next launch; drops every handle's graphs captured under another limit (graph keys include
+ * it). */
 enum { MF_OPT_CUDA_GRAPHS = 1, MF_OPT_PDL = 2, MF_OPT_CONCURRENT = 3, MF_OPT_GEMM_2SM = 4,
        MF_OPT_FLASH_ATTN = 5, MF_OPT_GEMM_PERSISTENT = 6, MF_OPT_FUSED_HEAD = 7,
-       MF_OPT_LAYER_UPDATES = 8 };
+       MF_OPT_LAYER_UPDATES = 8, MF_OPT_WAIT_LIMIT_US = 9 };
 mf_status mf_set_option(mf_handle h, int option, int value);
 
 /* Host-side fault injection for tests: kind 1 = the next workspace allocation fails;

@@ -18,6 +18,7 @@
 #include "decoder_layout.h"
 #include "internal.h"
 #include "launch.cuh"
+#include "revolve.h"
 
 using mf::GemmArgs;
 
@@ -89,6 +90,10 @@ struct mf_ctx {
   // which a stream capture turns into parallel graph branches.
   cudaStream_t sstream = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  // Decoder backward: the weight product of each linear layer runs on the side stream next
+  // to the data product; ev_w[j] marks the end of the latest weight product that reads seed
+  // buffer j, which the working stream waits for before it rewrites that buffer.
+  cudaEvent_t ev_w[4] = {nullptr, nullptr, nullptr, nullptr};
   bool concurrent = true;
   bool flash = true;          // fused dual attention where supported (MF_OPT_FLASH_ATTN)
   // Per-layer parameter updates (MF_OPT_LAYER_UPDATES): an update stream that takes each
@@ -315,6 +320,7 @@ mf_status run_graphed(mf_ctx* h, mf_ctx::GraphCache& g, uint64_t key, cudaStream
   key = mix_key(key, static_cast<uint64_t>(mf::g_pair_mode));
   key = mix_key(key, static_cast<uint64_t>(mf::g_gemm_persist));
   key = mix_key(key, static_cast<uint64_t>(mf::g_fused_head));
+  key = mix_key(key, static_cast<uint64_t>(mf::g_wait_ns));
   if (h->record) {
     // one eager execution whose GEMM launches are recorded for mf_replay_gemms
     drop_record(h);
@@ -880,6 +886,12 @@ mf_status validate_loop(mf_ctx* h, const mf_loop_desc* lp) {
     return fail(h, MF_ERR_INVALID_ARG, "unknown hvp_mode");
 
   if (lp->ckpt_every < 0) return fail(h, MF_ERR_INVALID_ARG, "ckpt_every must be >= 0");
+  if (lp->ckpt_slots < 0 || lp->ckpt_slots > 1024)
+    return fail(h, MF_ERR_INVALID_ARG, "ckpt_slots must be in 0..1024");
+  if (lp->ckpt_slots > 0 && lp->ckpt_every > 1)
+    return fail(h, MF_ERR_INVALID_ARG, "ckpt_slots and ckpt_every > 1 are exclusive");
+  if (lp->ckpt_slots > 0 && lp->T > 4096)
+    return fail(h, MF_ERR_INVALID_ARG, "binomial checkpointing takes T <= 4096");
   if (lp->optimizer != MF_OPTIM_SGD && lp->optimizer != MF_OPTIM_ADAM)
     return fail(h, MF_ERR_INVALID_ARG, "unknown optimizer");
   if (lp->optimizer == MF_OPTIM_ADAM &&
@@ -924,22 +936,39 @@ struct Store {
   int k = 1, T = 0, n_ck = 1;
   bool m_kept = false, m_run_only = false;
   bool adam = false;   // Adam: v_t kept like m_t after the m slots, then m-bar and v-bar
+  // Binomial schedule (ckpt_slots = s > 0): s + 3 state slots (S_0, s snapshots, two
+  // scratch), each theta plus, when kept, m (and v with Adam); see revolve.h.
+  int bin = 0;
   int theta_idx(int t) const { return t % k == 0 ? t / k : n_ck + t % k - 1; }
   int m_idx(int t) const {
     return t % k == 0 ? t / k - 1 : (m_run_only ? n_ck - 1 : n_ck - 1 + t % k - 1);
   }
-  int theta_slots() const { return n_ck + k - 1; }
+  int theta_slots() const { return bin ? bin + 3 : n_ck + k - 1; }
   int m_slots() const {
+    if (bin) return !m_kept ? 0 : adam ? 2 * (bin + 3) + 4 : bin + 3;
     const int nm = !m_kept ? 0 : m_run_only ? n_ck : n_ck - 1 + k - 1;
     return adam ? 2 * nm + 2 : nm;
   }
   int v_idx(int t) const { return n_ck - 1 + k - 1 + m_idx(t); }
   int mbar_idx() const { return 2 * (n_ck - 1 + k - 1); }
+  // binomial slot j: m at m slot j, v at m slot n + j; then m-bar, v-bar and the two
+  // buffers that keep m_{t+1}, v_{t+1} of a deferred Adam reverse step
+  int bin_v(int j) const { return bin + 3 + j; }
+  int bin_mbar() const { return 2 * (bin + 3); }
+  int bin_pend() const { return 2 * (bin + 3) + 2; }
 };
 
 Store make_store(const mf_loop_desc* lp) {
   Store st;
   st.T = lp->T;
+  if (lp->ckpt_slots > 0) {
+    st.bin = std::min(lp->ckpt_slots, std::max(lp->T - 1, 1));
+    st.adam = lp->optimizer == MF_OPTIM_ADAM;
+    const bool lr_meta = lp->meta_kind & (MF_META_PARAM_LOGLR | MF_META_SCALAR_LOGLR);
+    // recomputation restarts from snapshots, so every kept state carries its momentum
+    st.m_kept = lr_meta || st.adam || lp->momentum != 0.f;
+    return st;
+  }
   st.k = lp->ckpt_every <= 1 ? 1 : std::min(lp->ckpt_every, lp->T);
   st.n_ck = lp->T / st.k + 1;
   const bool lr_meta = lp->meta_kind & (MF_META_PARAM_LOGLR | MF_META_SCALAR_LOGLR);
@@ -1209,6 +1238,224 @@ mf_status meta_grad_run(X& ex, const mf_loop_desc* lp, const float* theta0, cons
   return ex.st;
 }
 
+// ---- binomial checkpointing (ckpt_slots > 0; the schedule of revolve.h) ------------------
+// State slot j: theta in theta slot j; m (when kept) in m slot j, v (Adam) in m slot n + j.
+struct BinSlots {
+  const Store* st;
+  template <typename X> float* theta(X& ex, int j) const { return ex.theta_slot(j); }
+  template <typename X> float* m(X& ex, int j) const { return st->m_kept ? ex.m_slot(j) : nullptr; }
+  template <typename X> float* v(X& ex, int j) const { return st->adam ? ex.m_slot(st->bin_v(j)) : nullptr; }
+};
+
+// S_t0 in slot src -> S_t1 in slot dst by inner steps t0..t1-1.  The intermediate states
+// alternate between dst and the scratch slot that is not dst, so that the last lands in dst;
+// src is never written.  Each step casts the parameters it produces, so theta_t1 is cast at
+// the end.
+template <typename X>
+void bin_advance(X& ex, const mf_loop_desc* lp, const mf::RevolveSchedule& rs, const BinSlots& sl,
+                 const float* eta, const void* inner_x, const void* inner_y, const LrSel& lr,
+                 int t0, int t1, int src, int dst) {
+  const int other = dst == rs.scratch(0) ? rs.scratch(1) : rs.scratch(0);
+  ex.cast_params(sl.theta(ex, src), false);
+  int cur = src;
+  const int n = t1 - t0;
+  for (int k = 0; k < n && ex.st == MF_OK; ++k) {
+    const int t = t0 + k;
+    const int out = (n - 1 - k) % 2 == 0 ? dst : other;
+    inner_step(ex, lp, eta, inner_x, inner_y, lr, t, sl.theta(ex, cur),
+               t > 0 ? sl.m(ex, cur) : nullptr, sl.theta(ex, out), sl.m(ex, out),
+               t > 0 ? sl.v(ex, cur) : nullptr, sl.v(ex, out));
+    cur = out;
+  }
+}
+
+// Algorithm 2 with the binomial store: the rollout leaves the schedule's snapshots on its
+// way and S_T in a scratch slot; the sweep runs the schedule's actions, recomputing states
+// before it reverses them.  The reverse step itself is meta_grad_run's.  The cast of
+// theta_{t-1} (and, with Adam, the reverse of step t-1's moments) fuses into step t's update
+// only when S_{t-1} sits in a slot and the next action reverses it; otherwise the recompute
+// casts theta_{t-1}, and Adam's reverse of step t-1 waits for it, with m_t and v_t copied
+// aside because the recompute may overwrite their slot.
+template <typename X>
+mf_status meta_grad_run_binomial(X& ex, const mf_loop_desc* lp, const float* theta0,
+                                 const float* eta, const void* inner_x, const void* inner_y,
+                                 const void* outer_x, const void* outer_y, float* d_eta,
+                                 float* d_theta0, float* outer_loss) {
+  mf_ctx* h = ex.h;
+  cudaStream_t s = ex.s;
+  const int T = lp->T, B = lp->B, Bo = lp->B_outer;
+  const LrSel lr = lr_select(h, lp, eta);
+  const Store st = make_store(lp);
+  const BinSlots sl{&st};
+  const mf::RevolveSchedule rs = mf::revolve_schedule(T, st.bin);
+  const bool scalar_lr = lp->meta_kind & MF_META_SCALAR_LOGLR;
+  MF_CUDA(h, cudaMemcpyAsync(sl.theta(ex, 0), theta0, h->P * 4, cudaMemcpyDeviceToDevice, s));
+  const int64_t ne = n_eta_of(h, lp);
+  if (ne > 0) MF_CUDA(h, cudaMemsetAsync(d_eta, 0, ne * 4, s));
+  ex.prepare();
+
+  // 1. rollout S_0 -> S_T, leaving S_t in slot keep[t] for the schedule's snapshots
+  {
+    int cur = 0, tc = 0;
+    for (int t = 1; t < T && ex.st == MF_OK; ++t) {
+      if (rs.keep[t] < 0) continue;
+      bin_advance(ex, lp, rs, sl, eta, inner_x, inner_y, lr, tc, t, cur, rs.keep[t]);
+      cur = rs.keep[t];
+      tc = t;
+    }
+    if (ex.st == MF_OK)
+      bin_advance(ex, lp, rs, sl, eta, inner_x, inner_y, lr, tc, T, cur, rs.slot_T);
+  }
+  if (ex.st != MF_OK) return ex.st;
+  const int sT = rs.slot_T;
+
+  // 2. outer gradient at theta_T (cast by the rollout's last step)
+  float* tbar = ex.tbar_buf();
+  float* u = ex.u_buf();
+  float* Hu = ex.g_buf();
+  float* part = ex.part_buf();
+  const int nb = ex.nb();
+  ex.forward(Bo, outer_x, sl.theta(ex, sT), nullptr, false);
+  ex.loss(Bo, false, outer_y, nullptr, nullptr, ex.l_buf(), nullptr, nullptr);
+  ex.backward(Bo, false, nullptr, tbar);
+  if (outer_loss) {
+    mf::sum_scaled(ex.l_buf(), Bo, 1.f / Bo, outer_loss, s);
+    ex.launched();
+  }
+  float* d_plr = lr.off_plr >= 0 ? d_eta + lr.off_plr : nullptr;
+  float* pend_m = st.adam ? ex.m_slot(st.bin_pend()) : nullptr;
+  float* pend_v = st.adam ? ex.m_slot(st.bin_pend() + 1) : nullptr;
+  // Adam's reverse of inner step j: m_{j+1}, v_{j+1} from (mj1, vj1), m_j from slot prev
+  auto adam_pre = [&](mf::LayerUpdArgs& a, int j, bool bar_in, float* mj1, float* vj1,
+                      int prev) {
+    set_adam(a, lp, j);
+    a.adam_pre = true;
+    a.bar_in = bar_in;
+    a.m_adj = mj1;
+    a.v_adj = vj1;
+    a.m_prev = j > 0 ? sl.m(ex, prev) : nullptr;
+    a.mbar = ex.m_slot(st.bin_mbar());
+    a.vbar = ex.m_slot(st.bin_mbar() + 1);
+    a.u_out = u;
+  };
+  size_t ai = 0;    // next action of the schedule
+  // slot of S_{t-1} if the next action reverses step t-1 at once, else -1
+  auto next_rev = [&](int t) {
+    return ai < rs.acts.size() && rs.acts[ai].kind == mf::RevolveAct::REV &&
+                   rs.acts[ai].t0 == t - 1
+               ? rs.acts[ai].src
+               : -1;
+  };
+  bool adam_pending = false, pend_bar_in = false;
+  auto defer_adam = [&](int slot, bool bar_in) {
+    MF_CUDA(h, cudaMemcpyAsync(pend_m, sl.m(ex, slot), h->P * 4, cudaMemcpyDeviceToDevice, s));
+    MF_CUDA(h, cudaMemcpyAsync(pend_v, sl.v(ex, slot), h->P * 4, cudaMemcpyDeviceToDevice, s));
+    adam_pending = true;
+    pend_bar_in = bar_in;
+    return MF_OK;
+  };
+  // u_{T-1} = -lr theta_bar_T ; d eta_lr += -lr m_T theta_bar_T ; cast theta_{T-1}, u_{T-1}
+  {
+    const int prev = next_rev(T);
+    if (st.adam && prev < 0) {
+      const mf_status e = defer_adam(sT, false);
+      if (e != MF_OK) return e;
+    } else {
+      mf::LayerUpdArgs a;
+      a.mode = mf::LU_ADJOINT;
+      a.theta_bar = tbar;
+      a.m_adj = lr.lr_meta ? sl.m(ex, sT) : nullptr;
+      a.u_out = u;
+      if (st.adam) adam_pre(a, T - 1, false, sl.m(ex, sT), sl.v(ex, sT), prev);
+      a.d_plr = d_plr;
+      a.partials = scalar_lr ? part + static_cast<int64_t>(T - 1) * nb : nullptr;
+      a.cast_src = prev >= 0 ? sl.theta(ex, prev) : nullptr;
+      a.mu = lp->momentum;
+      a.lr = lr.lr;
+      a.status = h->d_status;
+      ex.update(a);
+    }
+  }
+
+  // 3. reverse sweep along the schedule
+  const size_t xs = ex.x_step_bytes(B);
+  const size_t ys = ex.y_step_bytes(B);
+  const bool exw = lp->meta_kind & MF_META_EXAMPLE_WEIGHTS;
+  for (int t = T - 1; t >= 0; --t) {
+    while (ai < rs.acts.size() && rs.acts[ai].kind == mf::RevolveAct::ADV) {
+      const mf::RevolveAct& c = rs.acts[ai++];
+      bin_advance(ex, lp, rs, sl, eta, inner_x, inner_y, lr, c.t0, c.t1, c.src, c.dst);
+      if (ex.st != MF_OK) return ex.st;
+    }
+    if (ai >= rs.acts.size() || rs.acts[ai].kind != mf::RevolveAct::REV || rs.acts[ai].t0 != t)
+      return fail(h, MF_ERR_CUDA, "binomial schedule out of order");
+    const int cs = rs.acts[ai++].src;      // slot of S_t
+    if (adam_pending) {   // the reverse of step t's moments, now that m_t is in slot cs
+      mf::LayerUpdArgs a;
+      a.mode = mf::LU_ADJOINT;
+      a.theta_bar = tbar;
+      adam_pre(a, t, pend_bar_in, pend_m, pend_v, cs);
+      a.d_plr = d_plr;
+      a.partials = scalar_lr ? part + static_cast<int64_t>(t) * nb : nullptr;
+      a.lr = lr.lr;
+      a.status = h->d_status;
+      ex.update(a);
+      adam_pending = false;
+    }
+    const float* th = sl.theta(ex, cs);
+    const void* x = static_cast<const char*>(inner_x) + xs * t;
+    const void* y = static_cast<const char*>(inner_y) + ys * t;
+    const float* ew = exw ? eta + static_cast<int64_t>(t) * B : nullptr;
+    float* de = exw ? d_eta + static_cast<int64_t>(t) * B : nullptr;
+    // theta_bar_t = theta_bar_{t+1} + H u ; d eta_lr += -lr m_t theta_bar_t ;
+    // u_{t-1} = mu u_t - lr theta_bar_t ; cast theta_{t-1} (when in a slot), u_{t-1}
+    mf::LayerUpdArgs a;
+    a.mode = mf::LU_ADJOINT;
+    a.theta_bar = tbar;
+    a.Hu = Hu;
+    const int prev = t > 0 ? next_rev(t) : -1;
+    bool defer = false;
+    if (t > 0 && st.adam && prev < 0) {
+      a.adam = 1;            // theta_bar only; the reverse of step t-1 follows the recompute
+      defer = true;
+    } else if (t > 0) {
+      a.m_adj = lr.lr_meta ? sl.m(ex, cs) : nullptr;
+      a.u_in = u;
+      a.u_out = u;
+      if (st.adam) adam_pre(a, t - 1, true, sl.m(ex, cs), sl.v(ex, cs), prev);
+      a.d_plr = d_plr;
+      a.partials = scalar_lr ? part + static_cast<int64_t>(t - 1) * nb : nullptr;
+      if (prev >= 0) a.cast_src = sl.theta(ex, prev);
+    }
+    a.mu = lp->momentum;
+    a.lr = lr.lr;
+    a.status = h->d_status;
+    const bool per_layer = lp->hvp_mode != MF_HVP_REV_REV && per_layer_updates(ex);
+    if (lp->hvp_mode == MF_HVP_REV_REV) {
+      ex.ror_hvp(B, x, th, u, y, ew, nullptr, Hu, nullptr, ex.ld_buf(), de);
+    } else {
+      ex.forward(B, x, th, u, true);
+      ex.loss(B, true, y, ew, nullptr, nullptr, ex.ld_buf(), de);
+      if (per_layer) set_upd_after(ex, &a);
+      ex.backward(B, true, Hu, nullptr);
+      if (per_layer) set_upd_after(ex, nullptr);
+    }
+    if (!per_layer) ex.update(a);
+    if (ex.st != MF_OK) return ex.st;
+    if (defer) {
+      const mf_status e = defer_adam(cs, true);
+      if (e != MF_OK) return e;
+    }
+  }
+  if (scalar_lr) {
+    mf::sum_scaled(part, T * nb, 1.f, d_eta + lr.off_slr, s);
+    ex.launched();
+  }
+  if (d_theta0) MF_CUDA(h, cudaMemcpyAsync(d_theta0, tbar, h->P * 4, cudaMemcpyDeviceToDevice, s));
+  MF_CUDA(h, cudaGetLastError());
+  return ex.st;
+}
+
 template <typename X>
 mf_status rollout_run(X& ex, const mf_loop_desc* lp, const float* theta0, const float* eta,
                       const void* inner_x, const void* inner_y, float* thetaT) {
@@ -1270,6 +1517,10 @@ mf_status meta_grad_impl(mf_ctx* h, const mf_loop_desc* lp, const float* theta0,
                       store.m_slots(), lp->meta_kind & MF_META_SCALAR_LOGLR,
                       lp->hvp_mode == MF_HVP_REV_REV, s,
                       [&](auto& ex) {
+                        if (store.bin)
+                          return meta_grad_run_binomial(ex, lp, theta0, eta, inner_x, inner_y,
+                                                        outer_x, outer_y, d_eta, d_theta0,
+                                                        outer_loss);
                         return meta_grad_run(ex, lp, theta0, eta, inner_x, inner_y, outer_x,
                                              outer_y, d_eta, d_theta0, outer_loss);
                       });
@@ -1299,8 +1550,10 @@ void destroy_handle_objects(mf_ctx* h) {
   if (h->gstream) cudaStreamDestroy(h->gstream);
   if (h->sstream) cudaStreamDestroy(h->sstream);
   if (h->ustream) cudaStreamDestroy(h->ustream);
-  for (cudaEvent_t e : {h->ev_in, h->ev_out, h->ev_fork, h->ev_join, h->ev_u_in, h->ev_u_out})
+  for (cudaEvent_t e : {h->ev_in, h->ev_out, h->ev_fork, h->ev_join, h->ev_u_in, h->ev_u_out,
+                        h->ev_w[0], h->ev_w[1], h->ev_w[2], h->ev_w[3]})
     if (e) cudaEventDestroy(e);
+  for (cudaEvent_t& e : h->ev_w) e = nullptr;
   h->d_status = nullptr;
   h->gstream = h->sstream = h->ustream = nullptr;
   h->ev_in = h->ev_out = h->ev_fork = h->ev_join = h->ev_u_in = h->ev_u_out = nullptr;
@@ -1385,7 +1638,11 @@ mf_status mf_create(const mf_model_desc* d, mf_handle* out) {
       cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess ||
       cudaStreamCreateWithFlags(&h->ustream, cudaStreamNonBlocking) != cudaSuccess ||
       cudaEventCreateWithFlags(&h->ev_u_in, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_u_out, cudaEventDisableTiming) != cudaSuccess) {
+      cudaEventCreateWithFlags(&h->ev_u_out, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_w[0], cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_w[1], cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_w[2], cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_w[3], cudaEventDisableTiming) != cudaSuccess) {
     cudaGetLastError();
     destroy_handle_objects(h);
     delete h;
@@ -1439,6 +1696,29 @@ mf_status mf_workspace_bytes(mf_handle h, const mf_loop_desc* lp, size_t* bytes)
   *bytes = make_plan(h, std::max(lp->B, lp->B_outer), lp->T, store.theta_slots(),
                      store.m_slots(), lp->meta_kind & MF_META_SCALAR_LOGLR,
                      lp->hvp_mode == MF_HVP_REV_REV).bytes;
+  return MF_OK;
+}
+
+mf_status mf_checkpoint_plan(int T, int ckpt_every, int ckpt_slots, int* state_slots,
+                             int64_t* recompute_steps) {
+  if (T < 1 || ckpt_every < 0 || ckpt_slots < 0 || ckpt_slots > 1024 ||
+      (ckpt_slots > 0 && (ckpt_every > 1 || T > 4096)))
+    return MF_ERR_INVALID_ARG;
+  mf_loop_desc lp;
+  memset(&lp, 0, sizeof(lp));
+  lp.T = T;
+  lp.ckpt_every = ckpt_every;
+  lp.ckpt_slots = ckpt_slots;
+  const Store st = make_store(&lp);
+  int64_t re = 0;
+  if (st.bin) {
+    re = mf::revolve_schedule(T, st.bin).recompute;
+  } else if (st.k > 1) {
+    // every segment but the last is re-run from its checkpoint: k - 1 steps each
+    re = static_cast<int64_t>((T - 1) / st.k) * (st.k - 1);
+  }
+  if (state_slots) *state_slots = st.theta_slots();
+  if (recompute_steps) *recompute_steps = re;
   return MF_OK;
 }
 
@@ -1528,6 +1808,7 @@ mf_status mf_meta_grad(mf_handle h, const mf_loop_desc* lp, const float* theta0,
                      static_cast<uint64_t>(lp->B_outer), static_cast<uint64_t>(lp->meta_kind),
                      static_cast<uint64_t>(lp->hvp_mode),
                      static_cast<uint64_t>(make_store(lp).k),
+                     static_cast<uint64_t>(make_store(lp).bin),
                      static_cast<uint64_t>(lp->optimizer),
                      static_cast<uint64_t>(float_bits(lp->beta1)),
                      static_cast<uint64_t>(float_bits(lp->beta2)),
@@ -1698,6 +1979,13 @@ mf_status mf_set_option(mf_handle h, int option, int value) {
   if (option == MF_OPT_FUSED_HEAD) {
     if (value < 0 || value > 1) return fail(h, MF_ERR_INVALID_ARG, "MF_OPT_FUSED_HEAD takes 0 or 1");
     mf::g_fused_head = value;
+    drop_graphs(h);
+    return MF_OK;
+  }
+  if (option == MF_OPT_WAIT_LIMIT_US) {
+    if (value < 0 || value > 60000000)
+      return fail(h, MF_ERR_INVALID_ARG, "MF_OPT_WAIT_LIMIT_US takes 0..60000000");
+    mf::g_wait_ns = static_cast<long long>(value) * 1000LL;
     drop_graphs(h);
     return MF_OK;
   }

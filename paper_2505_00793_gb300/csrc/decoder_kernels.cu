@@ -64,7 +64,7 @@ __global__ void embed_fwd_kernel(const int* __restrict__ ids, int S, int d, int 
   const int b = r / S, s = r % S;
   int id = ids[static_cast<int64_t>(b) * (S + 1) + s];
   if (id < 0 || id >= V) {
-    if (threadIdx.x == 0 && status) atomicExch(status, 1);
+    if (threadIdx.x == 0 && status) atomicMax(status, 1);
     id = 0;
   }
   for (int j = threadIdx.x; j < d; j += blockDim.x) {
@@ -557,7 +557,7 @@ __global__ void ce_stats_kernel(int S, int V, const int* __restrict__ ids,
   const int b = r / S, s = r % S;
   int y = ids[static_cast<int64_t>(b) * (S + 1) + s + 1];
   if (y < 0 || y >= V) {
-    if (threadIdx.x == 0 && status) atomicExch(status, 1);
+    if (threadIdx.x == 0 && status) atomicMax(status, 1);
     y = 0;
   }
   const float* f = F + static_cast<int64_t>(r) * V;

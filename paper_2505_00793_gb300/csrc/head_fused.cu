@@ -145,7 +145,7 @@ __global__ void __launch_bounds__(HEAD_THREADS) head_fused_kernel(const HeadArgs
     if (bad) {
       if (lane == 0) {
         skip = 1;
-        if (L.status) atomicExch(L.status, 1);
+        if (L.status) atomicMax(L.status, 1);
       }
     } else {
       if (on) {

@@ -40,6 +40,9 @@ struct PerDeviceOnce {
 };
 
 // Device status word values (also the mf_status codes they map to).
+// Kernels raise the word with atomicMax, so the most severe condition of a call survives:
+// a timed-out wait (whose skipped work leaves garbage behind) over a non-finite value over
+// an out-of-range label (1).
 enum : int { DEV_OK = 0, DEV_NONFINITE = 5, DEV_TIMEOUT = 6 };
 
 // GEMM product terms (same bit meaning as mf_dual_gemm_bf16's `terms`).
@@ -100,6 +103,9 @@ cudaError_t tc_gemm_act_silu(const GemmArgs& a, cudaStream_t s, const char** why
 // Process-wide choice of 2-SM tiles for GEMMs that leave it automatic: 0 never, 1 when the
 // grid fills the GPU (default), 2 whenever M > 128.
 extern int g_pair_mode;
+// Limit of the tensor-core GEMMs' MMA-issuer and epilogue waits, in nanoseconds
+// (MF_OPT_WAIT_LIMIT_US; default 2 s).  Process-wide, read at launch.
+extern long long g_wait_ns;
 // Persistent CTA-pair form of the tcgen05 GEMM (tc_gemm_persist.cu): 2-SM tiles go through it
 // when g_gemm_persist is 1 (MF_OPT_GEMM_PERSISTENT; default 0).  bn is 128 or 256.
 cudaError_t tc_gemm_persist(const GemmArgs& a, cudaStream_t s, const char** why, int bn);

@@ -81,7 +81,7 @@ __global__ void loss_seed_kernel(const LossArgs a) {
   } else {
     const int y = a.Yi[row];
     if (y < 0 || y >= C) {
-      if (lane == 0 && a.status) atomicExch(a.status, 1);
+      if (lane == 0 && a.status) atomicMax(a.status, 1);
       return;
     }
     float mx = -INFINITY;
@@ -165,7 +165,7 @@ __global__ void chain_loss_kernel(const LossArgs a) {
       if (dFd) dFd[orow + c] = to_t<T>(scale * 2.f * invC * (d1 * ad + r * d2 * fd[c]));
     }
   }
-  if (bad && a.status) atomicExch(a.status, DEV_NONFINITE);
+  if (bad && a.status) atomicMax(a.status, DEV_NONFINITE);
   s2 = warp_sum(s2);
   s1 = warp_sum(s1);
   const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -262,7 +262,7 @@ __global__ void chain_ror_kernel(const LossArgs a) {
       if (a.dFd) static_cast<T*>(a.dFd)[orow + c] = to_t<T>(yh);
     }
   }
-  if (bad && a.status) atomicExch(a.status, DEV_NONFINITE);
+  if (bad && a.status) atomicMax(a.status, DEV_NONFINITE);
   s2 = warp_sum(s2);
   s1 = warp_sum(s1);
   const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -482,7 +482,7 @@ __global__ void __launch_bounds__(UPD_THREADS) layer_update_kernel(const LayerTa
     if (cast_w && tab.W[l]) st_copy<T>(static_cast<T*>(tab.W[l]), e0, dout, din, tab.ldw[l], vw, vec, cnt);
     if (cast_u && tab.U[l]) st_copy<T>(static_cast<T*>(tab.U[l]), e0, dout, din, tab.ldw[l], vu, vec, cnt);
   }
-  if (bad && a.status) atomicExch(a.status, DEV_NONFINITE);
+  if (bad && a.status) atomicMax(a.status, DEV_NONFINITE);
   if (a.partials) {   // one deterministic partial sum per block (scalar log-lr)
     acc = warp_sum(acc);
     if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;

@@ -18,13 +18,14 @@
 // (cta_group::2, 256 rows) serve GEMMs whose pair grid fills the GPU. GEMMs with few output
 // tiles split K across a thread-block cluster of S CTAs: the partial accumulators meet in
 // distributed shared memory, and each CTA reduces 128/S rows in a fixed order, so results are
-// deterministic. Every mbarrier wait is bounded; on expiry the CTA records DEV_TIMEOUT and
-// carries on to the end without further waits.
+// deterministic. Every mbarrier wait is bounded; on expiry the CTA records DEV_TIMEOUT, stops
+// issuing MMAs and drains the loads and MMAs it has issued before it releases its memory.
 #include "tc_gemm_impl.cuh"
 
 namespace mf {
 
 int g_pair_mode = 1;
+long long g_wait_ns = 2000000000LL;
 
 cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why) {
   static const char* dummy;

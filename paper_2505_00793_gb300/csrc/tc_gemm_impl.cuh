@@ -18,8 +18,8 @@
 // (cta_group::2, 256 rows) serve GEMMs whose pair grid fills the GPU. GEMMs with few output
 // tiles split K across a thread-block cluster of S CTAs: the partial accumulators meet in
 // distributed shared memory, and each CTA reduces 128/S rows in a fixed order, so results are
-// deterministic. Every mbarrier wait is bounded; on expiry the CTA records DEV_TIMEOUT and
-// carries on to the end without further waits.
+// deterministic. Every mbarrier wait is bounded; on expiry the CTA records DEV_TIMEOUT, stops
+// issuing MMAs and drains the loads and MMAs it has issued before it releases its memory.
 // Implementation of the tcgen05 dual GEMM, included by tc_gemm.cu (plain stores) and by
 // tc_gemm_act.cu (activation epilogues).  The epilogue mode and the activation are template
 // parameters so that each kernel instance carries only its own per-element code.
@@ -53,7 +53,25 @@ constexpr int EPI_WARPS2 = 8;
 constexpr int EPI_GROUPS2 = EPI_WARPS2 / 4;
 constexpr bool EPI_TMA2 = true;
 constexpr int THREADS2 = 64 + 32 * EPI_WARPS2;
-constexpr long long WAIT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
+// Bounded waits.  Every mbarrier wait gives up after a limit and records DEV_TIMEOUT.  The
+// MMA issuer's and the epilogue's waits use the run-time limit g_wait_ns (TcParams::wait_ns,
+// MF_OPT_WAIT_LIMIT_US; default 2 s).  The TMA producer's waits, and every wait that drains
+// work already issued after a timeout, use the fixed DRAIN_NS, so that a CTA never releases
+// shared memory or TMEM while a TMA load or an MMA it issued is still in flight:
+//  - after a timeout the MMA issuer stops issuing MMAs but keeps consuming the pipeline
+//    (waits for each stage's data, DRAIN_NS, and releases it), so the producer issues and
+//    sees the end of every load of its schedule;
+//  - the MMA issuer then commits and waits for its own last commit (all MMAs complete);
+//  - the producer waits for the last phase it issued on every stage before the CTA's final
+//    barrier (in a CTA pair, the even CTA, whose full barriers count both CTAs' bytes).
+// Only a wait that a healthy GPU never exceeds can run past DRAIN_NS.
+constexpr long long DRAIN_NS = 2000000000LL;
+
+__device__ __forceinline__ long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+  return static_cast<long long>(t);
+}
 
 struct TcParams {
   int M, N, K;
@@ -71,6 +89,7 @@ struct TcParams {
   float* C1; int ldc1; const float* bias1;
   EpiParams epi;
   int* status;
+  long long wait_ns;      // limit of the MMA issuer's and the epilogue's waits
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -99,17 +118,27 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Bounded wait: returns false (and flags the status word) if the phase never completes.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* status) {
+// Bounded wait: returns false (and flags the status word) if the phase has not completed
+// within limit_ns nanoseconds.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* status,
+                                          long long limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
-  long long t0 = clock64();
+  const long long t0 = global_ns();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
-    if (clock64() - t0 > WAIT_CYCLES) {
-      if (status) atomicExch(status, DEV_TIMEOUT);
+    if (global_ns() - t0 > limit_ns) {
+      if (status) atomicMax(status, DEV_TIMEOUT);
       return false;
     }
   }
+}
+
+// The producer's drain: wait for the last phase issued on every stage (issued = number of K
+// blocks whose loads were issued, in ring order).
+__device__ __forceinline__ void drain_loads(uint64_t* full_bar, int issued, int stages,
+                                            int* status) {
+  for (int j = issued - stages > 0 ? issued - stages : 0; j < issued; ++j)
+    if (!mbar_wait(&full_bar[j % stages], (j / stages) & 1, status, DRAIN_NS)) return;
 }
 
 // Every operand map is 3-D {K, rows, batch}; non-batched GEMMs have batch extent 1.
@@ -453,6 +482,7 @@ struct MmaLoop {
   uint64_t* full_bar;
   uint64_t* empty_bar;
   int* status;
+  long long wait_ns;
 };
 
 // The MMA issuer's loop over K blocks.  TERMS != 0 fixes the product mask at compile time
@@ -473,12 +503,17 @@ __device__ __forceinline__ void mma_loop(const MmaLoop& L, unsigned terms_rt, in
   // products into C0 / C1 per K slice
   const uint32_t p0 = __popc(terms & (T_C0_A0B0 | T_C0_A1B0 | T_C0_A0B1 | T_C0_A1B1));
   const uint32_t p1 = __popc(terms & (T_C1_A1B0 | T_C1_A0B1));
+  bool live = true;   // false after a timed-out wait: consume the stages without MMAs
   for (int i = 0; i < L.nk; ++i) {
     const int s = i % L.stages;
     const uint32_t ph = (i / L.stages) & 1;
-    if (!mbar_wait(&L.full_bar[s], ph, L.status)) break;
+    if (!live || !mbar_wait(&L.full_bar[s], ph, L.status, L.wait_ns)) {
+      live = false;
+      if (!mbar_wait(&L.full_bar[s], ph, L.status, DRAIN_NS)) break;
+    }
     tc_fence_after();
     const uint32_t st = L.sbase + s * L.stage_bytes;
+    if (live) {
 #pragma unroll
     for (int a = 0; a < KA; ++a) {
       auto descA = [&](int off) {
@@ -515,6 +550,7 @@ __device__ __forceinline__ void mma_loop(const MmaLoop& L, unsigned terms_rt, in
         if (terms & T_C0_A0B1) mma(0, a0 + advA, b1 + advB);
         if (terms & T_C0_A1B1) mma(0, a1 + advA, b1 + advB);
       }
+    }
     }
     if constexpr (PAIR) mma_commit_pair(&L.empty_bar[s]);
     else mma_commit(&L.empty_bar[s]);
@@ -622,10 +658,11 @@ __global__ void __launch_bounds__(THREADS, 1)
       const int stages = p.stages, stage_bytes = p.stage_bytes, tx_bytes = p.tx_bytes;
       const int a0_off = p.a0_off, a1_off = p.a1_off, b0_off = p.b0_off, b1_off = p.b1_off;
       int* const status = p.status;
-      for (int i = 0; i < nk; ++i) {
+      int issued = 0;
+      for (int i = 0; i < nk; ++i, ++issued) {
         const int s = i % stages;
         const uint32_t ph = (i / stages) & 1;
-        if (!mbar_wait(&empty_bar[s], ph ^ 1, status)) break;
+        if (!mbar_wait(&empty_bar[s], ph ^ 1, status, DRAIN_NS)) break;
         uint8_t* st = smem + s * stage_bytes;
         mbar_expect_tx(&full_bar[s], tx_bytes);
         const int k = (kb0 + i) * SK;
@@ -652,6 +689,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
         }
       }
+      drain_loads(full_bar, issued, stages, status);
     }
     __syncwarp();
   } else if (warp == 1) {
@@ -663,8 +701,10 @@ __global__ void __launch_bounds__(THREADS, 1)
       L.sbase = smem_u32(smem); L.tbase = tbase;
       L.a_mn = p.a_mn; L.b_mn = p.b_mn;
       L.full_bar = full_bar; L.empty_bar = empty_bar; L.status = p.status;
+      L.wait_ns = p.wait_ns;
       mma_dispatch<BN, KA, MODE, false>(L, terms, p.nsub);
       mma_commit(&acc_bar);
+      mbar_wait(&acc_bar, 0, p.status, DRAIN_NS);   // every MMA issued here has completed
     }
     __syncwarp();
   } else {
@@ -680,7 +720,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     constexpr int CG = BN / EPI_GROUPS >= GW ? BN / EPI_GROUPS : BN;
     const int c_begin = CG < BN ? grp * CG : 0;
     const int c_end = CG < BN ? c_begin + CG : (grp == 0 ? BN : 0);
-    const bool ok = nk > 0 && mbar_wait(&acc_bar, 0, p.status);
+    const bool ok = nk > 0 && mbar_wait(&acc_bar, 0, p.status, p.wait_ns);
     tc_fence_after();
     if (S == 1) {
       if (ok) {
@@ -903,6 +943,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s, const char** why) {
   p.C1 = dual ? a.C1 : nullptr; p.ldc1 = a.ldc1; p.bias1 = a.bias1;
   p.epi = a.epi;
   p.status = a.status;
+  p.wait_ns = g_wait_ns;
 
   const int tiles_n = (a.N + BN - 1) / BN, tiles_m = (a.M + BM - 1) / BM;
   const int nkb = (a.K + BK * KA - 1) / (BK * KA);
@@ -1077,10 +1118,11 @@ __global__ void __launch_bounds__(THREADS2, 1)
       int* const status = p.status;
       const uint32_t full0 = dsmem_addr(smem_u32(&full_bar[0]), 0);   // even CTA's barriers
       const int nb0 = n0 + static_cast<int>(rank) * BH;
-      for (int i = 0; i < nk; ++i) {
+      int issued = 0;
+      for (int i = 0; i < nk; ++i, ++issued) {
         const int s = i % stages;
         const uint32_t ph = (i / stages) & 1;
-        if (!mbar_wait(&empty_bar[s], ph ^ 1, status)) break;
+        if (!mbar_wait(&empty_bar[s], ph ^ 1, status, DRAIN_NS)) break;
         if (rank == 0) mbar_expect_tx(&full_bar[s], 2 * stage_bytes);
         const uint32_t bar = full0 + static_cast<uint32_t>(s) * 8u;
         uint8_t* st = smem + s * stage_bytes;
@@ -1104,6 +1146,9 @@ __global__ void __launch_bounds__(THREADS2, 1)
           if (b1_off >= 0) tma_load_3d_pair(st + b1_off, &tmB1, bar, k, nb0, bz);
         }
       }
+      // both CTAs' loads signal the even CTA's full barriers; the odd CTA's producer sees
+      // the same commits and stops at the same stage, and waits at the final cluster barrier
+      if (rank == 0) drain_loads(full_bar, issued, stages, status);
     }
     __syncwarp();
   } else if (warp == 1) {
@@ -1114,8 +1159,10 @@ __global__ void __launch_bounds__(THREADS2, 1)
       L.sbase = smem_u32(smem); L.tbase = tbase;
       L.a_mn = p.a_mn; L.b_mn = p.b_mn;
       L.full_bar = full_bar; L.empty_bar = empty_bar; L.status = p.status;
+      L.wait_ns = p.wait_ns;
       mma_dispatch<BN, 1, MODE, true>(L, terms, p.nsub);
       mma_commit_pair(&acc_bar);
+      mbar_wait(&acc_bar, 0, p.status, DRAIN_NS);   // every MMA of the pair has completed
     }
     __syncwarp();
   } else {
@@ -1126,7 +1173,7 @@ __global__ void __launch_bounds__(THREADS2, 1)
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     constexpr int CG = BN / EPI_GROUPS2;
     const int c_begin = ((warp - 2) >> 2) * CG, c_end = c_begin + CG;
-    const bool ok = mbar_wait(&acc_bar, 0, p.status);
+    const bool ok = mbar_wait(&acc_bar, 0, p.status, p.wait_ns);
     tc_fence_after();
     if (ok) {
       if (p.tma_store) {
@@ -1187,6 +1234,7 @@ cudaError_t launch_cfg2(const GemmArgs& a, cudaStream_t s, const char** why) {
   p.C1 = dual ? a.C1 : nullptr; p.ldc1 = a.ldc1; p.bias1 = a.bias1;
   p.epi = a.epi;
   p.status = a.status;
+  p.wait_ns = g_wait_ns;
   const int nb = a.batch < 1 ? 1 : a.batch;
   const int pairs_m = (a.M + 2 * BM - 1) / (2 * BM), tiles_n = (a.N + BN - 1) / BN;
 

@@ -71,35 +71,49 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
                : "memory");
 }
 
-// Bounded wait that gives up at once when another role of this CTA has timed out already.
-// CLUSTER selects cluster-scope acquire (arrivals from the peer CTA).
+// Bounded wait of the MMA issuer and the epilogue warps (limit_ns = TcParams::wait_ns) that
+// gives up at once when another of these roles in this CTA has timed out already.  CLUSTER
+// selects cluster-scope acquire (arrivals from the peer CTA).  The TMA producer never looks
+// at the abort flag: it waits with DRAIN_NS only, so both CTAs' producers see the same MMA
+// commits and stop at the same stage (see tc_gemm_impl.cuh).
 template <bool CLUSTER>
 __device__ __forceinline__ bool pwait(uint64_t* bar, uint32_t parity, int* status,
-                                      volatile int* abort) {
+                                      volatile int* abort, long long limit_ns) {
   auto probe = [&]() {
     return CLUSTER ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity);
   };
   if (*abort) return false;
   if (probe()) return true;
-  const long long t0 = clock64();
+  const long long t0 = global_ns();
   while (true) {
     if (probe()) return true;
     if (*abort) return false;
-    if (clock64() - t0 > WAIT_CYCLES) {
-      if (status) atomicExch(status, DEV_TIMEOUT);
+    if (global_ns() - t0 > limit_ns) {
+      if (status) atomicMax(status, DEV_TIMEOUT);
       *abort = 1;
       return false;
     }
   }
 }
 
+// Commit of the MMA issuer's earlier tcgen05 work to a barrier of the even CTA only.
+__device__ __forceinline__ void mma_commit_even(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(static_cast<uint16_t>(1))
+      : "memory");
+}
+
 // The MMA issuer's loop over the K blocks of one tile, with the issue order and the
 // accumulator-block rotation of mma_loop (KA = 1, pair form).  The stage ring position
 // continues from g0, the K blocks issued for this pair's earlier tiles; the tile's
-// accumulators start at TMEM address tset.  Returns false if a wait gave up.
+// accumulators start at TMEM address tset.  Once `live` is false (a wait gave up) the
+// stages are consumed without MMAs.  Returns false if even a drain wait gave up.
 template <int BN, unsigned TERMS, int NSUB>
 __device__ __forceinline__ bool mma_tile(const MmaLoop& L, int g0, uint32_t tset,
-                                         unsigned terms_rt, int nsub_rt, volatile int* abort) {
+                                         unsigned terms_rt, int nsub_rt, volatile int* abort,
+                                         bool& live) {
   const uint32_t idesc = idesc_bf16(2 * BM, BN) | (static_cast<uint32_t>(L.a_mn) << 15) |
                          (static_cast<uint32_t>(L.b_mn) << 16);
   const uint64_t stepA = L.a_mn ? 128u : 2u, stepB = L.b_mn ? 128u : 2u;
@@ -111,7 +125,12 @@ __device__ __forceinline__ bool mma_tile(const MmaLoop& L, int g0, uint32_t tset
     const int g = g0 + i;
     const int s = g % L.stages;
     const uint32_t ph = (g / L.stages) & 1;
-    if (!pwait<false>(&L.full_bar[s], ph, L.status, abort)) return false;
+    if (!live || !pwait<false>(&L.full_bar[s], ph, L.status, abort, L.wait_ns)) {
+      live = false;
+      if (!mbar_wait(&L.full_bar[s], ph, L.status, DRAIN_NS)) return false;
+      mma_commit_pair(&L.empty_bar[s]);
+      continue;
+    }
     tc_fence_after();
     const uint32_t st = L.sbase + s * L.stage_bytes;
     auto descA = [&](int off) { return L.a_mn ? sdesc_mn_sw128(st + off) : sdesc_sw128(st + off); };
@@ -148,27 +167,28 @@ __device__ __forceinline__ bool mma_tile(const MmaLoop& L, int g0, uint32_t tset
 // Product masks the library issues get straight-line MMA sequences (as mma_dispatch).
 template <int BN, int MODE>
 __device__ __forceinline__ bool mma_tile_dispatch(const MmaLoop& L, int g0, uint32_t tset,
-                                                  unsigned terms, int nsub, volatile int* abort) {
+                                                  unsigned terms, int nsub, volatile int* abort,
+                                                  bool& live) {
   constexpr int N1 = persist_nsub(1, BN), N2 = persist_nsub(2, BN);
   switch (terms) {
-    case T_C0_A0B0: return mma_tile<BN, T_C0_A0B0, N1>(L, g0, tset, terms, nsub, abort);
+    case T_C0_A0B0: return mma_tile<BN, T_C0_A0B0, N1>(L, g0, tset, terms, nsub, abort, live);
     case T_C0_A0B0 | T_C1_A1B0 | T_C1_A0B1:
-      return mma_tile<BN, T_C0_A0B0 | T_C1_A1B0 | T_C1_A0B1, N2>(L, g0, tset, terms, nsub, abort);
+      return mma_tile<BN, T_C0_A0B0 | T_C1_A1B0 | T_C1_A0B1, N2>(L, g0, tset, terms, nsub, abort, live);
     case T_C0_A0B0 | T_C1_A0B1:
-      return mma_tile<BN, T_C0_A0B0 | T_C1_A0B1, N2>(L, g0, tset, terms, nsub, abort);
+      return mma_tile<BN, T_C0_A0B0 | T_C1_A0B1, N2>(L, g0, tset, terms, nsub, abort, live);
     default: break;
   }
   if constexpr (MODE == EPI_STORE) {
     switch (terms) {
-      case T_C0_A0B1: return mma_tile<BN, T_C0_A0B1, N1>(L, g0, tset, terms, nsub, abort);
+      case T_C0_A0B1: return mma_tile<BN, T_C0_A0B1, N1>(L, g0, tset, terms, nsub, abort, live);
       case T_C0_A1B0 | T_C0_A0B1:
-        return mma_tile<BN, T_C0_A1B0 | T_C0_A0B1, N1>(L, g0, tset, terms, nsub, abort);
+        return mma_tile<BN, T_C0_A1B0 | T_C0_A0B1, N1>(L, g0, tset, terms, nsub, abort, live);
       case T_C0_A0B0 | T_C0_A1B1:
-        return mma_tile<BN, T_C0_A0B0 | T_C0_A1B1, N1>(L, g0, tset, terms, nsub, abort);
+        return mma_tile<BN, T_C0_A0B0 | T_C0_A1B1, N1>(L, g0, tset, terms, nsub, abort, live);
       default: break;
     }
   }
-  return mma_tile<BN, 0, 0>(L, g0, tset, terms, nsub, abort);
+  return mma_tile<BN, 0, 0>(L, g0, tset, terms, nsub, abort, live);
 }
 
 template <int BN, int MODE, int ACT>
@@ -186,6 +206,7 @@ __global__ void __launch_bounds__(THREADS_P, 1)
   __shared__ __align__(8) uint64_t empty_bar[MAX_STAGES];
   __shared__ __align__(8) uint64_t acc_full[2];
   __shared__ __align__(8) uint64_t acc_empty[2];
+  __shared__ __align__(8) uint64_t drain_bar;
   __shared__ uint32_t tmem_slot;
   __shared__ int abort_flag;
 
@@ -211,6 +232,7 @@ __global__ void __launch_bounds__(THREADS_P, 1)
       mbar_init(&acc_full[b], 1);
       mbar_init(&acc_empty[b], 2 * EPI_WARPS_P);
     }
+    mbar_init(&drain_bar, 1);
     abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     if (p.a0_off >= 0) prefetch_tmap(&tmA0);
@@ -246,7 +268,7 @@ __global__ void __launch_bounds__(THREADS_P, 1)
       const int a0_off = p.a0_off, a1_off = p.a1_off, b0_off = p.b0_off, b1_off = p.b1_off;
       int* const status = p.status;
       const uint32_t full0 = dsmem_addr(smem_u32(&full_bar[0]), 0);   // even CTA's barriers
-      int g = 0;
+      int g = 0;   // K blocks issued so far (ring position)
       bool live = true;
       for (int t = pair; t < pp.ntiles && live; t += npairs) {
         int bz, mp, tn;
@@ -256,7 +278,7 @@ __global__ void __launch_bounds__(THREADS_P, 1)
         for (int i = 0; i < nk; ++i, ++g) {
           const int s = g % stages;
           const uint32_t ph = (g / stages) & 1;
-          if (!pwait<false>(&empty_bar[s], ph ^ 1, status, abort)) { live = false; break; }
+          if (!mbar_wait(&empty_bar[s], ph ^ 1, status, DRAIN_NS)) { live = false; break; }
           if (rank == 0) mbar_expect_tx(&full_bar[s], 2 * stage_bytes);
           const uint32_t bar = full0 + static_cast<uint32_t>(s) * 8u;
           uint8_t* st = smem + s * stage_bytes;
@@ -281,6 +303,7 @@ __global__ void __launch_bounds__(THREADS_P, 1)
           }
         }
       }
+      if (rank == 0) drain_loads(full_bar, g, stages, status);
     }
     __syncwarp();
   } else if (warp == 1) {
@@ -292,17 +315,22 @@ __global__ void __launch_bounds__(THREADS_P, 1)
       L.sbase = smem_u32(smem); L.tbase = tbase;
       L.a_mn = p.a_mn; L.b_mn = p.b_mn;
       L.full_bar = full_bar; L.empty_bar = empty_bar; L.status = p.status;
+      L.wait_ns = p.wait_ns;
+      bool live = true;   // false once a wait gave up: the ring is consumed without MMAs
       int j = 0;
       for (int t = pair; t < pp.ntiles; t += npairs, ++j) {
         const int set = pp.nsets == 2 ? (j & 1) : 0;
         const int use = pp.nsets == 2 ? (j >> 1) : j;
         // the epilogue warps of both CTAs have read this set's previous tile
-        if (!pwait<true>(&acc_empty[set], (use & 1) ^ 1, p.status, abort)) break;
+        if (live && !pwait<true>(&acc_empty[set], (use & 1) ^ 1, p.status, abort, p.wait_ns))
+          live = false;
         tc_fence_after();
         const uint32_t tset = tbase + static_cast<uint32_t>(set * pp.set_cols);
-        if (!mma_tile_dispatch<BN, MODE>(L, j * nk, tset, terms, p.nsub, abort)) break;
-        mma_commit_pair(&acc_full[set]);
+        if (!mma_tile_dispatch<BN, MODE>(L, j * nk, tset, terms, p.nsub, abort, live)) break;
+        if (live) mma_commit_pair(&acc_full[set]);
       }
+      mma_commit_even(&drain_bar);
+      mbar_wait(&drain_bar, 0, p.status, DRAIN_NS);   // every MMA of the pair has completed
     }
     __syncwarp();
   } else {
@@ -317,7 +345,7 @@ __global__ void __launch_bounds__(THREADS_P, 1)
     for (int t = pair; t < pp.ntiles; t += npairs, ++j) {
       const int set = pp.nsets == 2 ? (j & 1) : 0;
       const int use = pp.nsets == 2 ? (j >> 1) : j;
-      if (!pwait<false>(&acc_full[set], use & 1, p.status, abort)) break;
+      if (!pwait<false>(&acc_full[set], use & 1, p.status, abort, p.wait_ns)) break;
       tc_fence_after();
       int bz, mp, tn;
       coords(t, bz, mp, tn);
@@ -426,6 +454,7 @@ cudaError_t launch_cfg2p(const GemmArgs& a, cudaStream_t s, const char** why) {
   p.C1 = dual ? a.C1 : nullptr; p.ldc1 = a.ldc1; p.bias1 = a.bias1;
   p.epi = a.epi;
   p.status = a.status;
+  p.wait_ns = g_wait_ns;
   p.tma_store = 0;
   const int nb = a.batch < 1 ? 1 : a.batch;
 

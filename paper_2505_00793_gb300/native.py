@@ -26,7 +26,8 @@ OPTIMIZERS = {"sgd": 0, "adam": 1}
 MF_META_EXAMPLE_WEIGHTS, MF_META_PARAM_LOGLR, MF_META_SCALAR_LOGLR = 1, 2, 4
 MF_HVP_MIXED_FOR, MF_HVP_REV_REV = 0, 1
 (MF_OPT_CUDA_GRAPHS, MF_OPT_PDL, MF_OPT_CONCURRENT, MF_OPT_GEMM_2SM, MF_OPT_FLASH_ATTN,
- MF_OPT_GEMM_PERSISTENT, MF_OPT_FUSED_HEAD, MF_OPT_LAYER_UPDATES) = 1, 2, 3, 4, 5, 6, 7, 8
+ MF_OPT_GEMM_PERSISTENT, MF_OPT_FUSED_HEAD, MF_OPT_LAYER_UPDATES,
+ MF_OPT_WAIT_LIMIT_US) = 1, 2, 3, 4, 5, 6, 7, 8, 9
 STATUS = {0: "MF_OK", 1: "MF_ERR_INVALID_ARG", 2: "MF_ERR_UNSUPPORTED", 3: "MF_ERR_OOM",
           4: "MF_ERR_CUDA", 5: "MF_ERR_NONFINITE", 6: "MF_ERR_TIMEOUT"}
 
@@ -35,7 +36,7 @@ EXPORTS = ["mf_create", "mf_destroy", "mf_set_allocator", "mf_param_count",
            "mf_workspace_bytes", "mf_release_workspace", "mf_inner_rollout", "mf_hvp",
            "mf_meta_grad", "mf_sync", "mf_status_string", "mf_last_error", "mf_stats",
            "mf_set_kernel_timing", "mf_kernel_time", "mf_inject_fault", "mf_dual_gemm_bf16",
-           "mf_hvp_noalloc", "mf_set_option", "mf_replay_gemms"]
+           "mf_hvp_noalloc", "mf_set_option", "mf_replay_gemms", "mf_checkpoint_plan"]
 
 
 class mf_model_desc(C.Structure):
@@ -50,7 +51,7 @@ class mf_loop_desc(C.Structure):
     _fields_ = [("T", C.c_int), ("B", C.c_int), ("B_outer", C.c_int), ("alpha", C.c_float),
                 ("momentum", C.c_float), ("meta_kind", C.c_int), ("hvp_mode", C.c_int),
                 ("ckpt_every", C.c_int), ("optimizer", C.c_int), ("beta1", C.c_float),
-                ("beta2", C.c_float), ("adam_eps", C.c_float)]
+                ("beta2", C.c_float), ("adam_eps", C.c_float), ("ckpt_slots", C.c_int)]
 
 
 class MixflowError(RuntimeError):
@@ -83,6 +84,7 @@ def load(path: str = LIB_PATH) -> C.CDLL:
         "mf_set_kernel_timing": ([H, C.c_int], C.c_int),
         "mf_kernel_time": ([H, dblp, u64p, dblp], C.c_int),
         "mf_replay_gemms": ([H, C.c_int, vp, dblp, u64p, dblp], C.c_int),
+        "mf_checkpoint_plan": ([C.c_int, C.c_int, C.c_int, C.POINTER(C.c_int), i64p], C.c_int),
         "mf_inject_fault": ([H, C.c_int], C.c_int),
         "mf_set_option": ([H, C.c_int, C.c_int], C.c_int),
         "mf_hvp_noalloc": ([C.POINTER(mf_model_desc), C.c_int, vp, vp, vp, vp, vp, vp, vp, vp, vp],
@@ -166,13 +168,24 @@ def model_desc_for(w) -> mf_model_desc:
     return d
 
 
-def loop_desc_for(w, hvp_mode: int = MF_HVP_MIXED_FOR, ckpt_every: int = 1) -> mf_loop_desc:
+def checkpoint_plan(T: int, ckpt_every: int = 1, ckpt_slots: int = 0):
+    """(stored states, inner steps re-run) of a sweep's checkpoint plan (mf_checkpoint_plan)."""
+    n, r = C.c_int(), C.c_int64()
+    st = lib().mf_checkpoint_plan(T, ckpt_every, ckpt_slots, C.byref(n), C.byref(r))
+    if st != 0:
+        raise MixflowError(st, "mf_checkpoint_plan")
+    return n.value, r.value
+
+
+def loop_desc_for(w, hvp_mode: int = MF_HVP_MIXED_FOR, ckpt_every: int = 1,
+                  ckpt_slots: int = 0) -> mf_loop_desc:
     l = mf_loop_desc()
     l.T, l.B, l.B_outer = w.T, w.B, w.B_outer
     l.alpha, l.momentum = w.alpha, w.momentum
     l.meta_kind = w.meta_kind
     l.hvp_mode = hvp_mode
     l.ckpt_every = ckpt_every
+    l.ckpt_slots = ckpt_slots
     l.optimizer = OPTIMIZERS[getattr(w, "optimizer", "sgd")]
     l.beta1, l.beta2, l.adam_eps = w.beta1, w.beta2, w.adam_eps
     return l

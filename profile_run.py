@@ -13,6 +13,8 @@ still move far more than the 129 MB L2 per launch:
 * decoder_s1024 two blocks of the larger decoder (d 1024, 16 heads, S = 1024), two
                 sequences: the fused attention at the larger decoder's sequence length
 * wide_small    the wide workload's shapes at T = 2 (256-row GEMMs, the 10-class head)
+* decoder_large_T2  the bench workload (12 x d1024, 16 heads, S = 1024, B = 8, heavy ball,
+                weights + scalar log-lr) at T = 2: every kernel of a step at full size
 
 ``--gemm-persistent``, ``--fused-head`` and ``--layer-updates`` set the opt-in paths, so that
 their kernels can be captured on the same cases.
@@ -36,6 +38,8 @@ def case(name: str):
         return synth.WORKLOADS[name]
     if name == "wide_small":
         return synth.WORKLOADS["wide"].with_(name="wide_small", T=2)
+    if name == "decoder_large_T2":
+        return synth.WORKLOADS["decoder_large"].with_(name="decoder_large_T2", T=2)
     if name == "decoder_s1024":
         return synth.decoder("decoder_s1024", 1024, 16, 4096, 2, 32768, 1024, B=2, T=2,
                              B_outer=2, alpha=1e-3)
@@ -49,7 +53,7 @@ def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--case", required=True,
                     choices=["deep_4k", "deep_4k_adam", "decoder_small", "toy",
-                             "decoder_s1024", "wide_small"])
+                             "decoder_s1024", "wide_small", "decoder_large_T2"])
     ap.add_argument("--calls", type=int, default=3)
     ap.add_argument("--hvp-mode", type=int, default=0)
     ap.add_argument("--gemm-persistent", action="store_true")

@@ -2,7 +2,7 @@
 
 Failures are made on the host or through inputs the kernels check themselves: invalid loop
 descriptors, the host-side fault injector (a failed workspace allocation, a device wait
-reported as expired), a NaN in theta_0 (caught by the update kernel's finiteness check),
+reported as expired), device waits that really expire under a zero wait limit, a NaN in theta_0 (caught by the update kernel's finiteness check),
 and out-of-range class labels and token ids (bounds-checked, clamped and reported by the
 loss and embedding kernels).  After every error the handle stays usable and the next call
 gives the same result as a fresh handle.  Degenerate sizes (one example, one inner step,
@@ -90,6 +90,41 @@ def test_injected_timeout_then_recovery():
     with pytest.raises(native.MixflowError) as e:
         mf.sync()
     assert e.value.status == TIMEOUT
+    out = _call(mf, native, w, d, bufs)
+    mf.close()
+    assert np.array_equal(out[0], ref[0]) and np.array_equal(out[1], ref[1])
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("persistent", [False, True])
+def test_device_wait_expiry_then_recovery(persistent):
+    """A real device-side timeout, no injection: with MF_OPT_WAIT_LIMIT_US = 0 the
+    tensor-core GEMMs' MMA issuer and epilogue give up at their first wait that does not
+    complete at once, record the timeout, let the loads and MMAs they issued complete and
+    end.  mf_sync reports MF_ERR_TIMEOUT (no trap; the context stays usable), and with the
+    default limit back the same handle reproduces a fresh handle's meta-gradient bit for bit.
+    The persistent variant sends every GEMM of more than 128 rows (the weight products here)
+    through the persistent CTA-pair kernel."""
+    torch, native = need_gpu()
+    w = synth.Workload("wait_bf16", [128, 256, 136, 10], "gelu", "ce", "bf16", B=64, T=2,
+                       B_outer=64, alpha=0.05)
+    inp = synth.make_inputs(w)
+    ref = _fresh(w, inp)
+    mf = native.MixFlow.for_workload(w)
+    d = native.to_device_inputs(w, inp)
+    bufs = _buffers(torch, w)
+    try:
+        mf.set_option(native.MF_OPT_WAIT_LIMIT_US, 0)
+        if persistent:
+            mf.set_option(native.MF_OPT_GEMM_2SM, 2)
+            mf.set_option(native.MF_OPT_GEMM_PERSISTENT, 1)
+        with pytest.raises(native.MixflowError) as e:
+            _call(mf, native, w, d, bufs)
+        assert e.value.status == TIMEOUT
+    finally:
+        mf.set_option(native.MF_OPT_WAIT_LIMIT_US, 2000000)
+        mf.set_option(native.MF_OPT_GEMM_PERSISTENT, 0)
+        mf.set_option(native.MF_OPT_GEMM_2SM, 1)
     out = _call(mf, native, w, d, bufs)
     mf.close()
     assert np.array_equal(out[0], ref[0]) and np.array_equal(out[1], ref[1])
