@@ -225,8 +225,9 @@ struct DecExec {
   T* Uw(int64_t off) const { return at<T>(p.o_U[tidx(off)]); }
 
 
-  void gemm(GemmArgs g) {
+  void gemm(GemmArgs g, cudaStream_t on = nullptr) {
     if (st != MF_OK) return;
+    const cudaStream_t s = on ? on : this->s;
     g.status = h->d_status;
     cudaEvent_t e0 = nullptr, e1 = nullptr;
     unsigned ev_flags = cudaEventRecordDefault;
@@ -463,10 +464,44 @@ struct DecExec {
     chk("decoder loss");
   }
 
+  // Weight products on the side stream (MF_OPT_CONCURRENT): each runs next to the data
+  // product of its layer, after the seeds it reads are written on the working stream.
+  // Seed buffers: 0 = dy (read by the W2 and Wo products), 1 = dz1 (W1), 2 = dqkv (Wqkv).
+  enum { WS_W2 = 0, WS_WO = 1, WS_W1 = 2, WS_QKV = 3, WS_NONE = -1 };
+  bool w_rec[4] = {false, false, false, false};
+  bool side_used = false;
+  bool conc() const {
+    return h->concurrent && h->sstream && h->ev_fork && h->ev_join && h->ev_w[0] &&
+           h->ev_w[1] && h->ev_w[2] && h->ev_w[3];
+  }
+  void chk_cuda(cudaError_t e, const char* what) {
+    if (e != cudaSuccess && st == MF_OK) {
+      st = MF_ERR_CUDA;
+      h->err = std::string(what) + ": " + cudaGetErrorString(e);
+    }
+  }
+  // the working stream waits until every weight product reading seed buffer `buf` is done
+  void wait_seed_readers(int buf) {
+    const int slots[2][2] = {{WS_W2, WS_WO}, {WS_W1, WS_NONE}};
+    const int* sl = buf == 0 ? slots[0] : buf == 1 ? slots[1] : nullptr;
+    auto wait1 = [&](int j) {
+      if (j >= 0 && w_rec[j]) chk_cuda(cudaStreamWaitEvent(s, h->ev_w[j], 0), "seed wait");
+    };
+    if (sl) { wait1(sl[0]); wait1(sl[1]); }
+    else wait1(WS_QKV);
+  }
+  void side_join() {
+    if (!side_used) return;
+    chk_cuda(cudaEventRecord(h->ev_join, h->sstream), "side join");
+    chk_cuda(cudaStreamWaitEvent(s, h->ev_join, 0), "side join");
+    side_used = false;
+    for (bool& r : w_rec) r = false;
+  }
+
   // weight product into out (grad) / outh (tangent): A^T seed with K = tokens; the
   // activations A [tokens][M] and the seeds [tokens][Nn] are read MN-major
   void wprod(int M, int Nn, const T* A_, const T* Ad_, const T* S_, const T* Sd_, bool dual,
-             float* outg, float* outh) {
+             float* outg, float* outh, int slot = WS_NONE) {
     if (!dual && !outg) return;   // primal backward kept only for its cotangents
     GemmArgs g;
     g.M = M; g.N = Nn; g.K = rows_cur * Ly.S;
@@ -484,7 +519,18 @@ struct DecExec {
       g.terms = mf::T_C0_A1B0 | mf::T_C0_A0B1;
       g.C0 = outh; g.ldc0 = Nn;
     }
-    gemm(g);
+    if (!conc()) {
+      gemm(g);
+      return;
+    }
+    chk_cuda(cudaEventRecord(h->ev_fork, s), "side fork");
+    chk_cuda(cudaStreamWaitEvent(h->sstream, h->ev_fork, 0), "side fork");
+    gemm(g, h->sstream);
+    side_used = true;
+    if (slot >= 0) {
+      chk_cuda(cudaEventRecord(h->ev_w[slot], h->sstream), "side event");
+      w_rec[slot] = true;
+    }
   }
 
   // residual gradient (float32) -> operand-type seed
@@ -492,6 +538,7 @@ struct DecExec {
   // skipped when the RMSNorm backward that produced dx already wrote them (fresh)
   void seed_from(const float* X, const float* Xd, bool dual, bool fresh = false) {
     if (fresh) return;
+    wait_seed_readers(0);
     const int N = rows_cur * Ly.S, d = Ly.d;
     mf::cast_rows<T>(X, N, d, at<T>(p.dy), d, s);
     launched();
@@ -521,6 +568,7 @@ struct DecExec {
     }
     cudaMemsetAsync(at<float>(p.dx), 0, static_cast<size_t>(N) * d * 4, s);
     if (dual) cudaMemsetAsync(at<float>(p.dxd), 0, static_cast<size_t>(N) * d * 4, s);
+    wait_seed_readers(0);
     mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.xf), at<float>(p.xfd), at<float>(p.rf), at<float>(p.rfd),
                            theta_cur + Ly.gf, dual ? u + Ly.gf : nullptr, at<float>(p.dh),
                            dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx), at<float>(p.dxd), s,
@@ -540,7 +588,8 @@ struct DecExec {
       // ---- MLP branch: seed = dx (already in bf16 unless dx was just restored) ---------
       seed_from(at<float>(p.dx), at<float>(p.dxd), dual, ror_mode != 2);
       wprod(F, d, at<T>(p.a1[l]), at<T>(p.a1d[l]), at<T>(p.dy), at<T>(p.dyd), dual, G(Ly.W2[l]),
-            Hh(Ly.W2[l]));
+            Hh(Ly.W2[l]), WS_W2);
+      wait_seed_readers(1);   // the data product's epilogue rewrites dz1
       {
         GemmArgs g = lin(N, F, d, at<T>(p.dy), at<T>(p.dyd), d, W(Ly.W2[l]), Uw(Ly.W2[l]), ld8(d), dual);
         g.epi.mode = mf::EPI_ACT_BWD;
@@ -554,7 +603,7 @@ struct DecExec {
         gemm(g);
       }
       wprod(d, F, at<T>(p.h2[l]), at<T>(p.h2d[l]), at<T>(p.dz1), at<T>(p.dz1d), dual, G(Ly.W1[l]),
-            Hh(Ly.W1[l]));
+            Hh(Ly.W1[l]), WS_W1);
       {
         GemmArgs g = lin(N, d, F, at<T>(p.dz1), at<T>(p.dz1d), F, W(Ly.W1[l]), Uw(Ly.W1[l]), ld8(F), dual);
         g.C0 = at<float>(p.dh); g.ldc0 = d;
@@ -564,6 +613,7 @@ struct DecExec {
       mf::dec_gain_grad(N, d, at<float>(p.x2[l]), at<float>(p.x2d[l]), at<float>(p.r2[l]),
                         at<float>(p.r2d[l]), at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr,
                         G(Ly.g2[l]), Hh(Ly.g2[l]), at<float>(p.gpart), s);
+      wait_seed_readers(0);
       mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.x2[l]), at<float>(p.x2d[l]), at<float>(p.r2[l]),
                              at<float>(p.r2d[l]), theta_cur + Ly.g2[l], dual ? u + Ly.g2[l] : nullptr,
                              at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx),
@@ -572,7 +622,7 @@ struct DecExec {
       // ---- attention branch: seed = dx (written in bf16 by the norm backward above) -----
       seed_from(at<float>(p.dx), at<float>(p.dxd), dual, true);
       wprod(d, d, at<T>(p.Om[l]), at<T>(p.Omd[l]), at<T>(p.dy), at<T>(p.dyd), dual, G(Ly.Wo[l]),
-            Hh(Ly.Wo[l]));
+            Hh(Ly.Wo[l]), WS_WO);
       {
         GemmArgs g = lin(N, d, d, at<T>(p.dy), at<T>(p.dyd), d, W(Ly.Wo[l]), Uw(Ly.Wo[l]), ld8(d), dual);
         g.C0 = at<float>(p.dh); g.ldc0 = d;
@@ -642,6 +692,7 @@ struct DecExec {
       }
       }
       const float qscale = 1.f / sqrtf(static_cast<float>(dh));
+      wait_seed_readers(2);
       mf::dec_rope_merge<T>(N, S, H, dh, at<float>(p.rope), qscale, at<float>(p.dQ), at<float>(p.dK),
                             at<float>(p.dV), at<T>(p.dqkv), 3 * d, s);
       launched();
@@ -651,7 +702,7 @@ struct DecExec {
         launched();
       }
       wprod(d, 3 * d, at<T>(p.h1[l]), at<T>(p.h1d[l]), at<T>(p.dqkv), at<T>(p.dqkvd), dual,
-            G(Ly.Wqkv[l]), Hh(Ly.Wqkv[l]));
+            G(Ly.Wqkv[l]), Hh(Ly.Wqkv[l]), WS_QKV);
       {
         GemmArgs g = lin(N, d, 3 * d, at<T>(p.dqkv), at<T>(p.dqkvd), 3 * d, W(Ly.Wqkv[l]),
                          Uw(Ly.Wqkv[l]), ld8(3 * d), dual);
@@ -662,6 +713,7 @@ struct DecExec {
       mf::dec_gain_grad(N, d, at<float>(p.x1[l]), at<float>(p.x1d[l]), at<float>(p.r1[l]),
                         at<float>(p.r1d[l]), at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr,
                         G(Ly.g1[l]), Hh(Ly.g1[l]), at<float>(p.gpart), s);
+      if (l > 0) wait_seed_readers(0);
       mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.x1[l]), at<float>(p.x1d[l]), at<float>(p.r1[l]),
                              at<float>(p.r1d[l]), theta_cur + Ly.g1[l], dual ? u + Ly.g1[l] : nullptr,
                              at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx),
@@ -672,6 +724,7 @@ struct DecExec {
     mf::dec_embed_bwd(V, d, at<int>(p.o_start), at<int>(p.o_order), at<float>(p.dx),
                       dual ? at<float>(p.dxd) : nullptr, G(Ly.E), Hh(Ly.E), s);
     launched();
+    side_join();
     chk("decoder backward");
   }
 
