@@ -372,8 +372,8 @@ def run_gpu(args):
     d = native.to_device_inputs(w, inp)
     mf = native.MixFlow.for_workload(w)
     mf.set_torch_allocator()        # the workspace shows in torch's memory statistics
-    if args.gemm_persistent:
-        mf.set_option(native.MF_OPT_GEMM_PERSISTENT, 1)
+    if args.gemm_persistent is not None:
+        mf.set_option(native.MF_OPT_GEMM_PERSISTENT, args.gemm_persistent)
     if args.fused_head:
         mf.set_option(native.MF_OPT_FUSED_HEAD, 1)
     if args.layer_updates:
@@ -509,7 +509,7 @@ def run_gpu(args):
         if ws == 1 and not args.no_cpu_baseline and (default or args.cpu_baseline):
             cpu = cpu_baseline(w)
         traffic = _dram_traffic(args.workload) if default and not (
-            args.gemm_persistent or args.fused_head or args.layer_updates) else None
+            args.gemm_persistent is not None or args.fused_head or args.layer_updates) else None
         out = {
             "metric": "meta-grad steps/s", "value": value, "unit": "meta-steps/s", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
@@ -526,8 +526,8 @@ def run_gpu(args):
                           "recomputed)" if args.ckpt_slots > 0 else "")
                        + (f"; Adam inner optimiser (b1 0.9, b2 0.999, eps {args.adam_eps:g}) "
                           "in place of SGD" if args.optimizer == "adam" else "")
-                       + ("; CTA-pair GEMMs as persistent kernels"
-                          if args.gemm_persistent else "")
+                       + (f"; persistent CTA-pair GEMM mode {args.gemm_persistent}"
+                          if args.gemm_persistent is not None else "")
                        + ("; output layer, loss and data product fused"
                           if args.fused_head else "")
                        + ("; per-layer updates overlapping the backward pass"
@@ -590,8 +590,9 @@ def main():
                     help="binomial checkpointing with this many snapshots (0 = off)")
     ap.add_argument("--ckpt-every", type=int, default=1,
                     help="segment length of the theta_t store (1 = keep every theta_t)")
-    ap.add_argument("--gemm-persistent", action="store_true",
-                    help="run CTA-pair GEMMs as persistent kernels (MF_OPT_GEMM_PERSISTENT)")
+    ap.add_argument("--gemm-persistent", type=int, nargs="?", const=1, default=None,
+                    help="MF_OPT_GEMM_PERSISTENT mode (0 off; 1 all, duals 128-wide; 2 "
+                         "single-accumulator only, the library default; 3 all, duals 256-wide)")
     ap.add_argument("--fused-head", action="store_true",
                     help="output layer, loss and data product in one kernel (MF_OPT_FUSED_HEAD)")
     ap.add_argument("--layer-updates", action="store_true",

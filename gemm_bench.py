@@ -31,14 +31,14 @@ def main() -> None:
 
     ap = argparse.ArgumentParser()
     ap.add_argument("--only", default="", help="substring of the shape names to run")
-    ap.add_argument("--persistent", action="store_true",
-                    help="CTA-pair tiles as persistent kernels (MF_OPT_GEMM_PERSISTENT)")
+    ap.add_argument("--persistent", type=int, nargs="?", const=1, default=None,
+                    help="MF_OPT_GEMM_PERSISTENT mode (library default when absent)")
     args = ap.parse_args()
     torch.cuda.set_device(0)
-    if args.persistent:   # a process-wide option, set through any handle
+    if args.persistent is not None:   # a process-wide option, set through any handle
         from paper_2505_00793_gb300 import synth
         h = native.MixFlow.for_workload(synth.WORKLOADS["tiny"])
-        h.set_option(native.MF_OPT_GEMM_PERSISTENT, 1)
+        h.set_option(native.MF_OPT_GEMM_PERSISTENT, args.persistent)
         h.close()
     s = torch.cuda.current_stream()
     for name, M, N, K, t in SHAPES:

@@ -300,11 +300,15 @@ mf_status mf_replay_gemms(mf_handle h, int reps, void* stream, double* ms, uint6
  * and seq_len a multiple of 64; others always use the materialised form).  0 materialises
  * them (per block, for the backward).  Setting it drops the handle's captured graphs and
  * changes the workspace size.
- * MF_OPT_GEMM_PERSISTENT (process-wide, default 0): 1 runs every GEMM that takes CTA-pair
- * tiles as a persistent kernel: one pair per SM pair walks a static list of output tiles,
- * with two TMEM accumulator sets so that a tile's epilogue overlaps the next tile's main loop
- * (dual products then take 128-wide tiles).  Same products and summation order within a
- * tile as the one-tile form.  Setting it drops the handle's captured graphs.
+ * MF_OPT_GEMM_PERSISTENT (process-wide, default 2): GEMMs that take CTA-pair tiles run as a
+ * persistent kernel: one pair per SM pair walks a static list of output tiles (grouped so
+ * that the pairs running together share row blocks of A and a band of B), with two TMEM
+ * accumulator sets when they fit so that a tile's epilogue overlaps the next tile's main
+ * loop.  0 never; 1 every pair GEMM, dual products at 128-wide tiles (two sets of their two
+ * accumulators fit); 2 single-accumulator products only (dual products keep the one-tile
+ * kernel, which was faster for them on the larger transformer's shapes); 3 every pair GEMM,
+ * dual products at 256-wide tiles with one accumulator set.  Same products and summation
+ * order within a tile as the one-tile form.  Setting it drops the handle's captured graphs.
  * MF_OPT_FUSED_HEAD (process-wide, default 0): 1 computes the output layer of an MLP with at
  * most 16 outputs and a squared or softmax cross-entropy loss in one kernel per pass: the
  * layer's forward product, the loss with its seeds and tangent losses, and its data product

@@ -1971,7 +1971,7 @@ mf_status mf_set_option(mf_handle h, int option, int value) {
     return MF_OK;
   }
   if (option == MF_OPT_GEMM_PERSISTENT) {
-    if (value < 0 || value > 1) return fail(h, MF_ERR_INVALID_ARG, "MF_OPT_GEMM_PERSISTENT takes 0 or 1");
+    if (value < 0 || value > 3) return fail(h, MF_ERR_INVALID_ARG, "MF_OPT_GEMM_PERSISTENT takes 0..3");
     mf::g_gemm_persist = value;
     drop_graphs(h);
     return MF_OK;

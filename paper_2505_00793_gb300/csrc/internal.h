@@ -106,8 +106,10 @@ extern int g_pair_mode;
 // Limit of the tensor-core GEMMs' MMA-issuer and epilogue waits, in nanoseconds
 // (MF_OPT_WAIT_LIMIT_US; default 2 s).  Process-wide, read at launch.
 extern long long g_wait_ns;
-// Persistent CTA-pair form of the tcgen05 GEMM (tc_gemm_persist.cu): 2-SM tiles go through it
-// when g_gemm_persist is 1 (MF_OPT_GEMM_PERSISTENT; default 0).  bn is 128 or 256.
+// Persistent CTA-pair form of the tcgen05 GEMM (tc_gemm_persist.cu), MF_OPT_GEMM_PERSISTENT:
+// g_gemm_persist 0 = off; 1 = every 2-SM GEMM, dual products at 128-wide tiles with two
+// TMEM accumulator sets; 2 (default) = single-accumulator 2-SM GEMMs only; 3 = every 2-SM
+// GEMM, dual products at their 256-wide tiles with one accumulator set.  bn is 128 or 256.
 cudaError_t tc_gemm_persist(const GemmArgs& a, cudaStream_t s, const char** why, int bn);
 extern int g_gemm_persist;
 // SIMT float32 GEMM with the same semantics (simt_gemm.cu).

@@ -27,7 +27,7 @@
 
 namespace mf {
 
-int g_gemm_persist = 0;
+int g_gemm_persist = 2;
 
 namespace {
 
@@ -47,8 +47,11 @@ __host__ __device__ constexpr int persist_sets(int nacc, int bn) {
   return 2 * nacc * persist_nsub(nacc, bn) * bn <= 512 ? 2 : 1;
 }
 
+// Tile list order (L2 reuse): per batch entry, groups of `group` 256-row blocks; inside a
+// group the row blocks vary fastest, then the n tile; groups follow each other.  The pairs
+// running at one time then share a few row blocks of A and a band of n tiles of B.
 struct PersistParams {
-  int tiles_n, pairs_m, ntiles;   // tile list order: n fastest, then 256-row blocks, then batch
+  int tiles_n, pairs_m, ntiles, group;
   int nsets;                      // accumulator sets in TMEM (1 or 2)
   int set_cols;                   // TMEM columns of one set
 };
@@ -253,12 +256,16 @@ __global__ void __launch_bounds__(THREADS_P, 1)
   volatile int* abort = &abort_flag;
   pdl_entry();
 
-  // Tile t of the list: n tile fastest, then the 256-row block, then the batch index.
+  // Tile t of the list (grouped order, see PersistParams).
   auto coords = [&](int t, int& bz, int& mp, int& tn) {
-    tn = t % pp.tiles_n;
-    const int r = t / pp.tiles_n;
-    mp = r % pp.pairs_m;
-    bz = r / pp.pairs_m;
+    const int per_batch = pp.tiles_n * pp.pairs_m;
+    bz = t / per_batch;
+    const int r = t % per_batch;
+    const int gsz = pp.group * pp.tiles_n;
+    const int g = r / gsz, w = r % gsz;
+    const int rows = min(pp.group, pp.pairs_m - g * pp.group);
+    mp = g * pp.group + w % rows;
+    tn = w / rows;
   };
 
   if (warp == 0) {
@@ -479,6 +486,7 @@ cudaError_t launch_cfg2p(const GemmArgs& a, cudaStream_t s, const char** why) {
   const int64_t ntiles = static_cast<int64_t>(pp.tiles_n) * pp.pairs_m * nb;
   if (ntiles > (1 << 30)) { *why = "too many tiles"; return cudaErrorInvalidValue; }
   pp.ntiles = static_cast<int>(ntiles);
+  pp.group = pp.pairs_m < 8 ? pp.pairs_m : 8;
   pp.nsets = persist_sets(nacc, BN);
   pp.set_cols = nacc * p.nsub * BN;
 
@@ -525,9 +533,11 @@ cudaError_t launch_bn_p(const GemmArgs& a, cudaStream_t s, const char** why, int
 
 cudaError_t tc_gemm_persist(const GemmArgs& a, cudaStream_t s, const char** why, int bn) {
   const int act = a.epi.act;
-  // Dual products take 128-wide tiles unless the caller fixed the width: two sets of their
-  // two accumulators then fit TMEM, so epilogues overlap main loops.
-  if (bn == 256 && a.bn == 0 && (a.terms & (T_C1_A1B0 | T_C1_A0B1))) bn = 128;
+  // Dual products take 128-wide tiles unless the caller fixed the width or mode 3 keeps
+  // them at 256: two sets of their two accumulators then fit TMEM, so epilogues overlap main
+  // loops.
+  if (bn == 256 && a.bn == 0 && g_gemm_persist != 3 && (a.terms & (T_C1_A1B0 | T_C1_A0B1)))
+    bn = 128;
   if (a.epi.mode == EPI_STORE) return launch_bn_p<EPI_STORE, ACT_IDENT>(a, s, why, bn);
   if (a.epi.mode == EPI_ACT_FWD) {
     switch (act) {

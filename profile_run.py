@@ -56,7 +56,8 @@ def main() -> None:
                              "decoder_s1024", "wide_small", "decoder_large_T2"])
     ap.add_argument("--calls", type=int, default=3)
     ap.add_argument("--hvp-mode", type=int, default=0)
-    ap.add_argument("--gemm-persistent", action="store_true")
+    ap.add_argument("--gemm-persistent", type=int, nargs="?", const=1, default=None,
+                    help="MF_OPT_GEMM_PERSISTENT mode (library default when absent)")
     ap.add_argument("--fused-head", action="store_true")
     ap.add_argument("--layer-updates", action="store_true")
     args = ap.parse_args()
@@ -66,7 +67,8 @@ def main() -> None:
     d = native.to_device_inputs(w, inp)
     mf = native.MixFlow.for_workload(w)
     mf.set_option(native.MF_OPT_CUDA_GRAPHS, 0)
-    mf.set_option(native.MF_OPT_GEMM_PERSISTENT, 1 if args.gemm_persistent else 0)
+    if args.gemm_persistent is not None:
+        mf.set_option(native.MF_OPT_GEMM_PERSISTENT, args.gemm_persistent)
     mf.set_option(native.MF_OPT_FUSED_HEAD, 1 if args.fused_head else 0)
     mf.set_option(native.MF_OPT_LAYER_UPDATES, 1 if args.layer_updates else 0)
     loop = native.loop_desc_for(w, args.hvp_mode)

@@ -197,9 +197,12 @@ def _persist_coverage(M, N, BN, batch, npairs):
     CG = BN // (EPI_WARPS_P // 4)
     for pair in range(npairs):
         for t in range(pair, ntiles, npairs):
-            tn = t % tiles_n
-            r = t // tiles_n
-            mp, bz = r % pairs_m, r // pairs_m
+            # grouped order of the kernel: groups of up to 8 row blocks, rows fastest
+            group = min(pairs_m, 8)
+            bz, r = divmod(t, tiles_n * pairs_m)
+            g, w = divmod(r, group * tiles_n)
+            rows = min(group, pairs_m - g * group)
+            mp, tn = g * group + w % rows, w // rows
             for rank in (0, 1):
                 m0 = mp * 2 * BM + rank * BM
                 a_rows.add((bz, m0))
@@ -220,7 +223,8 @@ def _persist_coverage(M, N, BN, batch, npairs):
 
 @pytest.mark.parametrize("M,N,BN,batch,npairs", [
     (256, 128, 128, 1, 1), (300, 520, 128, 1, 3), (1000, 130, 256, 1, 76),
-    (1025, 1024, 256, 1, 7), (600, 1000, 128, 3, 5), (2048, 1024, 128, 1, 76)])
+    (1025, 1024, 256, 1, 7), (600, 1000, 128, 3, 5), (2048, 1024, 128, 1, 76),
+    (2900, 520, 128, 2, 9)])
 def test_persistent_tiles_cover_every_output_once(M, N, BN, batch, npairs):
     written, a_rows, b_rows, pairs_m, tiles_n = _persist_coverage(M, N, BN, batch, npairs)
     assert (written == 1).all()

@@ -123,7 +123,7 @@ def test_device_wait_expiry_then_recovery(persistent):
         assert e.value.status == TIMEOUT
     finally:
         mf.set_option(native.MF_OPT_WAIT_LIMIT_US, 2000000)
-        mf.set_option(native.MF_OPT_GEMM_PERSISTENT, 0)
+        mf.set_option(native.MF_OPT_GEMM_PERSISTENT, 2)   # the default
         mf.set_option(native.MF_OPT_GEMM_2SM, 1)
     out = _call(mf, native, w, d, bufs)
     mf.close()

@@ -34,7 +34,7 @@ def persistent():
     _set(native, native.MF_OPT_GEMM_2SM, 2)
     _set(native, native.MF_OPT_GEMM_PERSISTENT, 1)
     yield
-    _set(native, native.MF_OPT_GEMM_PERSISTENT, 0)
+    _set(native, native.MF_OPT_GEMM_PERSISTENT, 2)   # the default
     _set(native, native.MF_OPT_GEMM_2SM, 1)
 
 
