@@ -20,7 +20,7 @@ LIB = os.path.join(OUT_DIR, "libmixflow.so")
 BUILD_DIR = os.path.join(ROOT, "_build")
 SOURCES = ["tc_gemm_act_gelu.cu", "tc_gemm_act_silu.cu", "tc_gemm_act_tanh.cu",
            "tc_gemm_act_ident.cu", "tc_gemm_persist.cu", "tc_gemm.cu", "tc_gemm_act.cu",
-           "decoder_kernels.cu", "flash_attn.cu", "kernels.cu", "head_fused.cu", "simt_gemm.cu",
+           "decoder_kernels.cu", "flash_tc.cu", "flash_attn.cu", "kernels.cu", "head_fused.cu", "simt_gemm.cu",
            "capi.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",

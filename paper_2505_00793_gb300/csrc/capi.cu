@@ -95,7 +95,7 @@ struct mf_ctx {
   // buffer j, which the working stream waits for before it rewrites that buffer.
   cudaEvent_t ev_w[4] = {nullptr, nullptr, nullptr, nullptr};
   bool concurrent = true;
-  bool flash = true;          // fused dual attention where supported (MF_OPT_FLASH_ATTN)
+  int flash = 1;              // fused dual attention where supported (MF_OPT_FLASH_ATTN)
   // Per-layer parameter updates (MF_OPT_LAYER_UPDATES): an update stream that takes each
   // layer's update as soon as that layer's backward products are done, joined back into the
   // working stream at the end of the backward pass.
@@ -2000,7 +2000,8 @@ mf_status mf_set_option(mf_handle h, int option, int value) {
     return MF_OK;
   }
   if (option == MF_OPT_FLASH_ATTN) {
-    h->flash = value != 0;
+    if (value < 0 || value > 3) return fail(h, MF_ERR_INVALID_ARG, "MF_OPT_FLASH_ATTN takes 0..3");
+    h->flash = value;
     drop_graphs(h);
     return MF_OK;
   }

@@ -628,6 +628,12 @@ void init_attributes() {
 bool flash_supported(int S, int dh) { return dh == FDH && S > 0 && S % FT == 0; }
 
 void flash_fwd(const FlashArgs& a, bool dual, cudaStream_t s) {
+  // tcgen05 forward: the dual kernel at tc >= 1, the primal one too at tc = 2 (launch errors
+  // surface at the caller's check)
+  if (a.tc >= (dual ? 1 : 2) && flash_tc_supported(a.S, FDH)) {
+    flash_tc_fwd(a, dual, s);
+    return;
+  }
   init_attributes();
   const dim3 grid(a.S / FT, a.BH);
   if (dual)

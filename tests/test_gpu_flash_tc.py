@@ -1,0 +1,88 @@
+"""Fused dual attention on tcgen05 tensor cores (sequences of whole 128-token tiles) against
+the float64 oracle and against the warp-level fused kernels of the same library.
+
+MF_OPT_FLASH_ATTN 3 runs both forward kernels (S, S' into TMEM, P and P (*) S' through
+shared memory into the O and tangent products) on tcgen05, 1 (the default) the dual one; 2
+keeps the warp-level kernels.  Cases span one to
+three 128-query tiles per head (the causal diagonal and off-diagonal key tiles), one to four
+heads, momentum with the scalar log-lr, both HVP modes, and attention scores spread far
+beyond the running-maximum bound (weights of scale 0.3), so that rows rescale their
+accumulators in TMEM."""
+import math
+
+import numpy as np
+import pytest
+
+from gpu_util import need_gpu, rel_l2
+from paper_2505_00793_gb300 import synth
+from oracle import metagrad as om
+
+EX, SLR = synth.EXAMPLE_WEIGHTS, synth.SCALAR_LOGLR
+
+CASES = {
+    # d, H, F, L, V, S
+    "one_tile": synth.decoder("t1", 128, 2, 256, 1, 256, 128, B=3, T=2, B_outer=2, alpha=1e-2),
+    "two_tiles_4h": synth.decoder("t2", 256, 4, 512, 2, 304, 256, B=2, T=2, B_outer=2,
+                                  alpha=1e-2),
+    "three_tiles_mom": synth.decoder("t3", 64, 1, 128, 1, 200, 384, B=2, T=3, B_outer=2,
+                                     momentum=0.9, meta_kind=EX | SLR,
+                                     extra={"scalar_loglr": math.log(1e-2)}),
+}
+# Scores of standard deviation 12 (maximum 51): nearly one-hot rows whose running maximum
+# moves by more than the bound between key tiles.  bf16 operands move such scores by about
+# 0.2 and the probabilities by e^0.2, so this case is compared with the warp-level kernels on
+# the same inputs rather than with the float64 oracle.
+SHARP = synth.decoder("t4", 128, 2, 256, 1, 256, 384, B=2, T=1, B_outer=2,
+                      alpha=1e-4).with_(init_std=0.3)
+
+
+def _run(w, inp, flash, mode=0):
+    torch, native = need_gpu()
+    mf = native.MixFlow.for_workload(w)
+    mf.set_option(native.MF_OPT_FLASH_ATTN, flash)
+    loop = native.loop_desc_for(w, mode)
+    d = native.to_device_inputs(w, inp)
+    d_eta = torch.full((w.n_eta,), float("nan"), device="cuda")
+    d_th = torch.full((w.n_params,), float("nan"), device="cuda")
+    V = torch.full((1,), float("nan"), device="cuda")
+    outs = []
+    for _ in range(3):   # eager, capture, replay
+        mf.meta_grad(loop, d["theta0"], d["eta"], d["inner_x"], d["inner_y"], d["outer_x"],
+                     d["outer_y"], d_eta, d_th, V)
+        mf.sync()
+        outs.append((d_eta.cpu().numpy().copy(), d_th.cpu().numpy().copy(), float(V.cpu())))
+    mf.close()
+    for o in outs[1:]:
+        assert np.array_equal(o[0], outs[0][0]) and np.array_equal(o[1], outs[0][1])
+    return outs[0]
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("mode", [0, 1])
+@pytest.mark.parametrize("name", list(CASES))
+def test_flash_tc_meta_grad(name, mode):
+    w = CASES[name]
+    inp = synth.make_inputs(w)
+    ref = om.meta_grad(w, inp)
+    de_t, dt_t, V_t = _run(w, inp, 3, mode)
+    de_d, dt_d, V_d = _run(w, inp, 1, mode)
+    de_w, dt_w, V_w = _run(w, inp, 2, mode)
+    for de, dt, V in ((de_t, dt_t, V_t), (de_d, dt_d, V_d), (de_w, dt_w, V_w)):
+        assert np.isfinite(de).all() and np.isfinite(dt).all()
+        assert rel_l2(de, ref["d_eta"]) < 2e-2, (name, rel_l2(de, ref["d_eta"]))
+        assert rel_l2(dt, ref["d_theta0"]) < 2e-2, (name, rel_l2(dt, ref["d_theta0"]))
+        assert abs(V - ref["V"]) <= 2e-2 * abs(ref["V"])
+    # the two kernels differ only in summation order and bf16 rounding points
+    assert rel_l2(dt_t, dt_w) < 1e-2, (name, rel_l2(dt_t, dt_w))
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("mode", [0, 1])
+def test_flash_tc_rescaling_rows(mode):
+    inp = synth.make_inputs(SHARP)
+    de_t, dt_t, V_t = _run(SHARP, inp, 3, mode)
+    de_w, dt_w, V_w = _run(SHARP, inp, 2, mode)
+    assert np.isfinite(de_t).all() and np.isfinite(dt_t).all()
+    assert rel_l2(dt_t, dt_w) < 1e-2, rel_l2(dt_t, dt_w)
+    assert rel_l2(de_t, de_w) < 1e-2, rel_l2(de_t, de_w)
+    assert abs(V_t - V_w) <= 1e-3 * abs(V_w)
