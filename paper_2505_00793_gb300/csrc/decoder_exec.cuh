@@ -133,7 +133,9 @@ DecPlan make_dec_plan(const mf_ctx* h, const DecLayout& Ly, int rows, int T, int
   p.dF = take(N * V * es); p.dFd = take(N * V * es);
   p.qkv = take(N * 3 * d * 4); p.qkvd = take(N * 3 * d * 4);
   p.Sc = take(SS * 4); p.Scd = take(SS * 4);
-  p.O = take(static_cast<size_t>(BH) * S * Ly.dh * 4); p.Od = take(static_cast<size_t>(BH) * S * Ly.dh * 4);
+  // per-head float32 attention outputs (the fused attention writes them head-merged instead)
+  const size_t osz = p.flash ? 0 : static_cast<size_t>(BH) * S * Ly.dh * 4;
+  p.O = take(osz); p.Od = take(osz);
   p.y = take(Nd4); p.yd = take(Nd4);
   p.dx = take(Nd4); p.dxd = take(Nd4); p.dh = take(Nd4); p.dhd = take(Nd4);
   p.dy = take(NdT); p.dyd = take(NdT);
@@ -353,9 +355,12 @@ struct DecExec {
 
       if (p.flash) {
         // fused causal attention and its tangent: O, O' and the row statistics
+        // fused causal attention and its tangent, written head-merged as the Wo operands
         mf::FlashArgs fa = flash_args(l, BH);
-        fa.O = at<float>(p.O);
-        fa.Od = dual ? at<float>(p.Od) : nullptr;
+        fa.H = H;
+        fa.ldo = d;
+        fa.Om = reinterpret_cast<__nv_bfloat16*>(at<T>(p.Om[l]));
+        fa.Omd = dual ? reinterpret_cast<__nv_bfloat16*>(at<T>(p.Omd[l])) : nullptr;
         mf::flash_fwd(fa, dual, s);
         launched();
       } else {
@@ -381,12 +386,12 @@ struct DecExec {
         g.C1 = at<float>(p.Od); g.ldc1 = dh;
         gemm(g);
       }
-      }
       mf::dec_head_merge<T>(N, S, H, dh, at<float>(p.O), at<T>(p.Om[l]), d, s);
       launched();
       if (dual) {
         mf::dec_head_merge<T>(N, S, H, dh, at<float>(p.Od), at<T>(p.Omd[l]), d, s);
         launched();
+      }
       }
       // y = O Wo
       {
@@ -631,19 +636,22 @@ struct DecExec {
         g.C1 = at<float>(p.dhd); g.ldc1 = d;
         gemm(g);
       }
-      mf::dec_head_split<T>(N, S, H, dh, at<float>(p.dh), at<T>(p.dOh), s);
-      launched();
-      if (dual) {
-        mf::dec_head_split<T>(N, S, H, dh, at<float>(p.dhd), at<T>(p.dOhd), s);
+      if (!p.flash) {
+        mf::dec_head_split<T>(N, S, H, dh, at<float>(p.dh), at<T>(p.dOh), s);
         launched();
+        if (dual) {
+          mf::dec_head_split<T>(N, S, H, dh, at<float>(p.dhd), at<T>(p.dOhd), s);
+          launched();
+        }
       }
       if (p.flash) {
         // fused backward of the attention and its tangent, from D = rowsum(dO O) (and D')
         float* D = at<float>(p.fD);
         float* Dd = D + static_cast<int64_t>(BH) * S;
+        // D, D' and the per-head bf16 copies of dO, dO' in one pass over dO
         mf::flash_prep(N, S, H, at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr,
                        at<T>(p.Om[l]), dual ? at<T>(p.Omd[l]) : nullptr, d, D,
-                       dual ? Dd : nullptr, s);
+                       dual ? Dd : nullptr, at<T>(p.dOh), dual ? at<T>(p.dOhd) : nullptr, s);
         mf::FlashArgs fa = flash_args(l, BH);
         fa.dO = reinterpret_cast<const __nv_bfloat16*>(at<T>(p.dOh));
         fa.dOd = dual ? reinterpret_cast<const __nv_bfloat16*>(at<T>(p.dOhd)) : nullptr;

@@ -383,6 +383,26 @@ __global__ void rope_table_kernel(int S, int half, int dh, double base, float* _
 // RoPE (rotate-half) on q and k, q scaled by 1/sqrt(dh), head split.  qkv [N][3d] float32
 // (token-major) -> Q, K, V [B*H][S][dh] in T.  cos / sin of the angle of pair j at position
 // s come from the table of rope_table_kernel.
+// Four consecutive values stored as T (one 16-byte or 8-byte store).
+template <typename T>
+__device__ __forceinline__ void store4(T* p, float a, float b, float c, float d);
+template <>
+__device__ __forceinline__ void store4<float>(float* p, float a, float b, float c, float d) {
+  *reinterpret_cast<float4*>(p) = make_float4(a, b, c, d);
+}
+template <>
+__device__ __forceinline__ void store4<__nv_bfloat16>(__nv_bfloat16* p, float a, float b, float c,
+                                                      float d) {
+  const __nv_bfloat162 lo = __floats2bfloat162_rn(a, b), hi = __floats2bfloat162_rn(c, d);
+  uint2 v;
+  v.x = *reinterpret_cast<const uint32_t*>(&lo);
+  v.y = *reinterpret_cast<const uint32_t*>(&hi);
+  *reinterpret_cast<uint2*>(p) = v;
+}
+
+// Each thread takes four consecutive dimensions e..e+3 of one head (dh a multiple of 8, so
+// the rotate-half partners e +- dh/2 are four consecutive values too): 16-byte loads of q, k,
+// v, their partners and two (cos, sin) pairs of the table; 8-byte (bf16) stores.
 template <typename T>
 __global__ void rope_split_kernel(int S, int H, int dh, const float* __restrict__ rtab, float qscale,
                                   const float* __restrict__ qkv, T* __restrict__ Q,
@@ -392,24 +412,38 @@ __global__ void rope_split_kernel(int S, int H, int dh, const float* __restrict_
   const int b = r / S, s = r % S;
   const int d = H * dh, half = dh / 2;
   const float* row = qkv + static_cast<int64_t>(r) * 3 * d;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+  for (int c = 4 * threadIdx.x; c < d; c += 4 * blockDim.x) {
     const int h = c / dh, e = c % dh;
-    const int j = e < half ? e : e - half;
-    const float2 cs_sn = reinterpret_cast<const float2*>(rtab)[s * half + j];
-    const float cs = cs_sn.x, sn = cs_sn.y;
-    const float q = row[c], k = row[d + c];
-    const float qo = e < half ? -row[c + half] : row[c - half];
-    const float ko = e < half ? -row[d + c + half] : row[d + c - half];
+    const bool lo = e < half;
+    const int j = lo ? e : e - half;
+    const int po = lo ? c + half : c - half;            // partner columns
+    const float sg = lo ? -1.f : 1.f;                   // rot(x) = [-x2, x1]
+    const float4 t01 = *reinterpret_cast<const float4*>(rtab + 2 * (s * half + j));
+    const float4 t23 = *reinterpret_cast<const float4*>(rtab + 2 * (s * half + j + 2));
+    const float cs[4] = {t01.x, t01.z, t23.x, t23.z}, sn[4] = {t01.y, t01.w, t23.y, t23.w};
+    const float4 q = *reinterpret_cast<const float4*>(row + c);
+    const float4 qp = *reinterpret_cast<const float4*>(row + po);
+    const float4 k = *reinterpret_cast<const float4*>(row + d + c);
+    const float4 kp = *reinterpret_cast<const float4*>(row + d + po);
+    const float4 v = *reinterpret_cast<const float4*>(row + 2 * d + c);
+    const float qa[4] = {q.x, q.y, q.z, q.w}, qb[4] = {qp.x, qp.y, qp.z, qp.w};
+    const float ka[4] = {k.x, k.y, k.z, k.w}, kb[4] = {kp.x, kp.y, kp.z, kp.w};
+    float qo[4], ko[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      qo[i] = (qa[i] * cs[i] + sg * qb[i] * sn[i]) * qscale;
+      ko[i] = ka[i] * cs[i] + sg * kb[i] * sn[i];
+    }
     const int64_t o = ((static_cast<int64_t>(b) * H + h) * S + s) * dh + e;
-    Q[o] = to_t<T>((q * cs + qo * sn) * qscale);
-    K[o] = to_t<T>(k * cs + ko * sn);
-    Vv[o] = to_t<T>(row[2 * d + c]);
+    store4<T>(Q + o, qo[0], qo[1], qo[2], qo[3]);
+    store4<T>(K + o, ko[0], ko[1], ko[2], ko[3]);
+    store4<T>(Vv + o, v.x, v.y, v.z, v.w);
   }
 }
 
 // Transpose of the RoPE/split map for the backward: dQ, dK, dV [B*H][S][dh] (float32) ->
 // dqkv [N][3d] row-major (T):  dq = R^T(dQ) qscale, dk = R^T(dK), dv = dV, with
-// R^T(y) = y cos + [y2, -y1] sin.
+// R^T(y) = y cos + [y2, -y1] sin.  Four consecutive dimensions per thread, as above.
 template <typename T>
 __global__ void rope_merge_kernel(int S, int H, int dh, const float* __restrict__ rtab, float qscale,
                                   const float* __restrict__ dQ, const float* __restrict__ dK,
@@ -418,19 +452,33 @@ __global__ void rope_merge_kernel(int S, int H, int dh, const float* __restrict_
   const int r = blockIdx.x;
   const int b = r / S, s = r % S;
   const int d = H * dh, half = dh / 2;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+  T* row = out + static_cast<int64_t>(r) * ldo;
+  for (int c = 4 * threadIdx.x; c < d; c += 4 * blockDim.x) {
     const int h = c / dh, e = c % dh;
-    const int j = e < half ? e : e - half;
-    const float2 cs_sn = reinterpret_cast<const float2*>(rtab)[s * half + j];
-    const float cs = cs_sn.x, sn = cs_sn.y;
+    const bool lo = e < half;
+    const int j = lo ? e : e - half;
+    const int pe = lo ? e + half : e - half;
+    const float sg = lo ? 1.f : -1.f;                   // R^T: [y2, -y1]
+    const float4 t01 = *reinterpret_cast<const float4*>(rtab + 2 * (s * half + j));
+    const float4 t23 = *reinterpret_cast<const float4*>(rtab + 2 * (s * half + j + 2));
+    const float cs[4] = {t01.x, t01.z, t23.x, t23.z}, sn[4] = {t01.y, t01.w, t23.y, t23.w};
     const int64_t o = ((static_cast<int64_t>(b) * H + h) * S + s) * dh;
-    const float q = dQ[o + e], k = dK[o + e];
-    const float qo = e < half ? dQ[o + e + half] : -dQ[o + e - half];
-    const float ko = e < half ? dK[o + e + half] : -dK[o + e - half];
-    T* row = out + static_cast<int64_t>(r) * ldo;
-    row[c] = to_t<T>((q * cs + qo * sn) * qscale);
-    row[d + c] = to_t<T>(k * cs + ko * sn);
-    row[2 * d + c] = to_t<T>(dV[o + e]);
+    const float4 q = *reinterpret_cast<const float4*>(dQ + o + e);
+    const float4 qp = *reinterpret_cast<const float4*>(dQ + o + pe);
+    const float4 k = *reinterpret_cast<const float4*>(dK + o + e);
+    const float4 kp = *reinterpret_cast<const float4*>(dK + o + pe);
+    const float4 v = *reinterpret_cast<const float4*>(dV + o + e);
+    const float qa[4] = {q.x, q.y, q.z, q.w}, qb[4] = {qp.x, qp.y, qp.z, qp.w};
+    const float ka[4] = {k.x, k.y, k.z, k.w}, kb[4] = {kp.x, kp.y, kp.z, kp.w};
+    float qo[4], ko[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      qo[i] = (qa[i] * cs[i] + sg * qb[i] * sn[i]) * qscale;
+      ko[i] = ka[i] * cs[i] + sg * kb[i] * sn[i];
+    }
+    store4<T>(row + c, qo[0], qo[1], qo[2], qo[3]);
+    store4<T>(row + d + c, ko[0], ko[1], ko[2], ko[3]);
+    store4<T>(row + 2 * d + c, v.x, v.y, v.z, v.w);
   }
 }
 

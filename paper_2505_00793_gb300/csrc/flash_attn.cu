@@ -263,17 +263,23 @@ __global__ void __launch_bounds__(FTHREADS) flash_fwd_kernel(const FlashArgs a) 
     inv[h] = 1.f / lsum[h];
     rb[h] = DUAL ? rsum[h] * inv[h] : 0.f;
   }
+  // head-merged bf16 rows: token b*S + q, column hh*64 + e (see FlashArgs::Om)
+  const int hb = a.H > 0 ? bh / a.H : 0, hh = a.H > 0 ? bh % a.H : 0;
 #pragma unroll
   for (int n = 0; n < 8; ++n)
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      const int64_t off = hoff + static_cast<int64_t>(qrow0 + h * 8) * FDH + n * 8 + (lane & 3) * 2;
+      const int col = n * 8 + (lane & 3) * 2;
+      const int64_t off = hoff + static_cast<int64_t>(qrow0 + h * 8) * FDH + col;
+      const int64_t moff = (static_cast<int64_t>(hb) * a.S + qrow0 + h * 8) * a.ldo + hh * FDH + col;
       const float o0 = o[n][2 * h] * inv[h], o1 = o[n][2 * h + 1] * inv[h];
-      *reinterpret_cast<float2*>(a.O + off) = make_float2(o0, o1);
+      if (a.Om) *reinterpret_cast<uint32_t*>(a.Om + moff) = pack(o0, o1);
+      else *reinterpret_cast<float2*>(a.O + off) = make_float2(o0, o1);
       if (DUAL) {
         const float d0 = (oa[n][2 * h] + ob[n][2 * h]) * inv[h] - rb[h] * o0;
         const float d1 = (oa[n][2 * h + 1] + ob[n][2 * h + 1]) * inv[h] - rb[h] * o1;
-        *reinterpret_cast<float2*>(a.Od + off) = make_float2(d0, d1);
+        if (a.Om) *reinterpret_cast<uint32_t*>(a.Omd + moff) = pack(d0, d1);
+        else *reinterpret_cast<float2*>(a.Od + off) = make_float2(d0, d1);
       }
     }
   if ((lane & 3) == 0) {
@@ -574,22 +580,30 @@ __global__ void __launch_bounds__(FTHREADS) flash_bwd_q_kernel(const FlashArgs a
 }
 
 // D = rowsum(dO (*) O) and D' = rowsum(dO' (*) O + dO (*) O') per (token, head), from the
-// float32 head-merged output gradients [N][ld] and the bf16 merged attention outputs.
+// float32 head-merged output gradients [N][ld] and the bf16 merged attention outputs; the
+// same pass writes dO (dO') as bf16 per head ([B*H][S][64]) for the backward kernels.  One
+// warp per (token, head), two adjacent columns per lane (8-byte loads, 4-byte stores).
 __global__ void flash_prep_kernel(int N, int S, int H, const float* __restrict__ dO,
                                   const float* __restrict__ dOd, const bf16* __restrict__ O,
                                   const bf16* __restrict__ Od, int ld, float* __restrict__ D,
-                                  float* __restrict__ Dd) {
+                                  float* __restrict__ Dd, bf16* __restrict__ dOh,
+                                  bf16* __restrict__ dOhd) {
   pdl_entry();
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (warp >= N * H) return;
   const int n = warp / H, hh = warp % H;
-  const int64_t base = static_cast<int64_t>(n) * ld + hh * FDH;
-  float d = 0.f, dd = 0.f;
-  for (int c = lane; c < FDH; c += 32) {
-    const float o = __bfloat162float(O[base + c]);
-    const float g = dO[base + c];
-    d += g * o;
-    if (Dd) dd += dOd[base + c] * o + g * __bfloat162float(Od[base + c]);
+  const int64_t base = static_cast<int64_t>(n) * ld + hh * FDH + 2 * lane;
+  const int b = n / S, sidx = n % S;
+  const int64_t i = (static_cast<int64_t>(b) * H + hh) * S + sidx;
+  const float2 g = *reinterpret_cast<const float2*>(dO + base);
+  const float2 o = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(O + base));
+  float d = g.x * o.x + g.y * o.y, dd = 0.f;
+  if (dOh) *reinterpret_cast<uint32_t*>(dOh + i * FDH + 2 * lane) = pack(g.x, g.y);
+  if (Dd) {
+    const float2 gd = *reinterpret_cast<const float2*>(dOd + base);
+    const float2 od = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(Od + base));
+    dd = gd.x * o.x + gd.y * o.y + g.x * od.x + g.y * od.y;
+    if (dOhd) *reinterpret_cast<uint32_t*>(dOhd + i * FDH + 2 * lane) = pack(gd.x, gd.y);
   }
 #pragma unroll
   for (int s = 16; s > 0; s >>= 1) {
@@ -597,8 +611,6 @@ __global__ void flash_prep_kernel(int N, int S, int H, const float* __restrict__
     dd += __shfl_xor_sync(0xffffffffu, dd, s);
   }
   if (lane == 0) {
-    const int b = n / S, sidx = n % S;
-    const int64_t i = (static_cast<int64_t>(b) * H + hh) * S + sidx;
     D[i] = d;
     if (Dd) Dd[i] = dd;
   }
@@ -655,12 +667,14 @@ void flash_bwd(const FlashArgs& a, bool dual, cudaStream_t s) {
 }
 
 void flash_prep(int N, int S, int H, const float* dO, const float* dOd, const void* O,
-                const void* Od, int ld, float* D, float* Dd, cudaStream_t s) {
+                const void* Od, int ld, float* D, float* Dd, void* dOh, void* dOhd,
+                cudaStream_t s) {
   const int warps = N * H;
   const int threads = 256;
   const int blocks = (warps * 32 + threads - 1) / threads;
   launch_k(flash_prep_kernel, dim3(blocks), dim3(threads), 0, s, N, S, H, dO, dOd,
-           static_cast<const bf16*>(O), static_cast<const bf16*>(Od), ld, D, Dd);
+           static_cast<const bf16*>(O), static_cast<const bf16*>(Od), ld, D, Dd,
+           static_cast<bf16*>(dOh), static_cast<bf16*>(dOhd));
 }
 
 }  // namespace mf

@@ -58,6 +58,8 @@ struct FtcCfg {
 struct FtcParams {
   int BH, S;
   float *O, *Od, *lse, *rbar;
+  int H, ldo;                        // head-merged bf16 outputs when Om is set
+  __nv_bfloat16 *Om, *Omd;
   int* status;
 };
 
@@ -370,26 +372,46 @@ __global__ void __launch_bounds__(FTC_THREADS, FtcCfg<DUAL>::CTAS)
       const float inv = 1.f / l;
       const float rb = DUAL ? rs * inv : 0.f;
       const int64_t grow = static_cast<int64_t>(row0) + qt * TQ + r;
-      float* orow = p.O + grow * HD;
+      // head-merged bf16 row: token b*S + q, columns hh*64 .. hh*64 + 63
+      const int hb = p.H > 0 ? bh / p.H : 0, hh = p.H > 0 ? bh % p.H : 0;
+      const int64_t mrow = (static_cast<int64_t>(hb) * p.S + qt * TQ + r) * p.ldo + hh * HD;
 #pragma unroll 1
       for (int c0 = 0; c0 < HD; c0 += 16) {
         float o[16];
         tmem_ld16(tb + lo + C::C_O + c0, o);
 #pragma unroll
         for (int i = 0; i < 16; ++i) o[i] *= inv;
+        if (p.Om) {
+          uint4* dst = reinterpret_cast<uint4*>(p.Om + mrow + c0);
+          dst[0] = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]),
+                              pack_bf16x2(o[4], o[5]), pack_bf16x2(o[6], o[7]));
+          dst[1] = make_uint4(pack_bf16x2(o[8], o[9]), pack_bf16x2(o[10], o[11]),
+                              pack_bf16x2(o[12], o[13]), pack_bf16x2(o[14], o[15]));
+        } else {
+          float* orow = p.O + grow * HD;
 #pragma unroll
-        for (int i = 0; i < 16; i += 4)
-          *reinterpret_cast<float4*>(orow + c0 + i) = make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]);
+          for (int i = 0; i < 16; i += 4)
+            *reinterpret_cast<float4*>(orow + c0 + i) =
+                make_float4(o[i], o[i + 1], o[i + 2], o[i + 3]);
+        }
         if (DUAL) {
           float t[16];
           tmem_ld16(tb + lo + C::C_T + c0, t);
-          float* drow = p.Od + grow * HD;
 #pragma unroll
           for (int i = 0; i < 16; ++i) t[i] = t[i] * inv - rb * o[i];
+          if (p.Om) {
+            uint4* dst = reinterpret_cast<uint4*>(p.Omd + mrow + c0);
+            dst[0] = make_uint4(pack_bf16x2(t[0], t[1]), pack_bf16x2(t[2], t[3]),
+                                pack_bf16x2(t[4], t[5]), pack_bf16x2(t[6], t[7]));
+            dst[1] = make_uint4(pack_bf16x2(t[8], t[9]), pack_bf16x2(t[10], t[11]),
+                                pack_bf16x2(t[12], t[13]), pack_bf16x2(t[14], t[15]));
+          } else {
+            float* drow = p.Od + grow * HD;
 #pragma unroll
-          for (int i = 0; i < 16; i += 4)
-            *reinterpret_cast<float4*>(drow + c0 + i) =
-                make_float4(t[i], t[i + 1], t[i + 2], t[i + 3]);
+            for (int i = 0; i < 16; i += 4)
+              *reinterpret_cast<float4*>(drow + c0 + i) =
+                  make_float4(t[i], t[i + 1], t[i + 2], t[i + 3]);
+          }
         }
       }
       p.lse[grow] = m + __logf(l);
@@ -430,6 +452,10 @@ cudaError_t launch_ftc_fwd(const FlashArgs& a, cudaStream_t s) {
   p.Od = a.Od;
   p.lse = a.lse;
   p.rbar = a.rbar;
+  p.H = a.H;
+  p.ldo = a.ldo;
+  p.Om = a.Om;
+  p.Omd = a.Omd;
   p.status = a.status;
   return launch_k(flash_tc_fwd_kernel<DUAL>, dim3(a.S / TQ, a.BH), dim3(FTC_THREADS),
                   C::SMEM, s, mQ, mK, mV, mQd, mKd, mVd, p);

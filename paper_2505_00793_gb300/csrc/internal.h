@@ -262,6 +262,10 @@ struct FlashArgs {
   const float *D = nullptr, *Dd = nullptr;
   float *dQ = nullptr, *dQd = nullptr, *dK = nullptr, *dKd = nullptr, *dV = nullptr,
         *dVd = nullptr;
+  // Forward outputs, head-merged: when Om is set the forward writes O (and O') as T, token
+  // major [B*S][ldo] at column h*64 + e (H heads), instead of float32 O / Od per head.
+  int H = 0, ldo = 0;
+  __nv_bfloat16 *Om = nullptr, *Omd = nullptr;
   int tc = 1;              // tcgen05 forward where S is a multiple of 128: 0 never,
                            // 1 the dual kernel, 2 the dual and the primal kernels
   int* status = nullptr;   // device status word (bounded waits of the tcgen05 kernels)
@@ -274,8 +278,10 @@ void flash_fwd(const FlashArgs& a, bool dual, cudaStream_t s);
 void flash_bwd(const FlashArgs& a, bool dual, cudaStream_t s);
 // D = rowsum(dO (*) O), D' = rowsum(dO' (*) O + dO (*) O') per (token, head) from float32
 // merged gradients [N][ld] and bf16 merged outputs; Dd / dOd / Od may be null (primal).
+// The same pass writes dO (and dO') as bf16 per head, [B*H][S][64], for the backward kernels.
 void flash_prep(int N, int S, int H, const float* dO, const float* dOd, const void* O,
-                const void* Od, int ld, float* D, float* Dd, cudaStream_t s);
+                const void* Od, int ld, float* D, float* Dd, void* dOh, void* dOhd,
+                cudaStream_t s);
 
 // ---- decoder-only transformer kernels (decoder_kernels.cu) ------------------------------
 void dec_embed_fwd(int N, int S, int d, int V, const int* ids, const float* E, const float* UE,

@@ -353,8 +353,16 @@ __global__ void __launch_bounds__(UPD_THREADS) layer_update_kernel(const LayerTa
                                                                    const LayerUpdArgs a) {
   pdl_entry();
   __shared__ float red[UPD_THREADS / 32];
+  // the layer of this block: the last l with tile0[l] <= blockIdx.x (binary search)
   int l = 0;
-  while (l + 1 < tab.n && static_cast<int>(blockIdx.x) >= tab.tile0[l + 1]) ++l;
+  {
+    int hi = tab.n - 1;
+    while (l < hi) {
+      const int mid = (l + hi + 1) >> 1;
+      if (static_cast<int>(blockIdx.x) >= tab.tile0[mid]) l = mid;
+      else hi = mid - 1;
+    }
+  }
   const int dout = tab.dout[l], din = tab.din[l];
   const int64_t n = static_cast<int64_t>(tab.rows[l]) * dout;
   const int64_t e0 = (static_cast<int64_t>(blockIdx.x - tab.tile0[l]) * UPD_THREADS + threadIdx.x) * 4;
@@ -407,6 +415,15 @@ __global__ void __launch_bounds__(UPD_THREADS) layer_update_kernel(const LayerTa
       float tb[4], hu[4] = {0.f, 0.f, 0.f, 0.f};
       ld4(tb, a.theta_bar, k, vec, cnt);
       if (a.Hu) ld4(hu, a.Hu, k, vec, cnt);
+      // every other input of the plain (non-Adam) adjoint is loaded before the first store,
+      // so that a thread's loads are in flight together (the pointers may alias in place)
+      float ma[4] = {0.f, 0.f, 0.f, 0.f}, ui[4] = {0.f, 0.f, 0.f, 0.f};
+      float dp[4] = {0.f, 0.f, 0.f, 0.f};
+      const bool plain = !a.adam;
+      if (plain && a.m_adj) ld4(ma, a.m_adj, k, vec, cnt);
+      if (plain && a.u_out && a.u_in) ld4(ui, a.u_in, k, vec, cnt);
+      if (plain && a.m_adj && a.d_plr) ld4(dp, a.d_plr, k, vec, cnt);
+      if (plain && a.cast_src) ld4(vw, a.cast_src, k, vec, cnt);
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         tb[j] += hu[j];
@@ -445,17 +462,13 @@ __global__ void __launch_bounds__(UPD_THREADS) layer_update_kernel(const LayerTa
         st4(a.mbar, k, mb, vec, cnt);
         st4(a.vbar, k, vb, vec, cnt);
         have_contrib = true;
-      } else if (!a.adam) {
+      } else if (plain) {
         if (a.m_adj) {
-          float ma[4];
-          ld4(ma, a.m_adj, k, vec, cnt);
 #pragma unroll
           for (int j = 0; j < 4; ++j) contrib[j] = -lr[j] * ma[j] * tb[j];
           have_contrib = true;
         }
         if (a.u_out) {
-          float ui[4] = {0.f, 0.f, 0.f, 0.f};
-          if (a.u_in) ld4(ui, a.u_in, k, vec, cnt);
 #pragma unroll
           for (int j = 0; j < 4; ++j) vu[j] = a.mu * ui[j] - lr[j] * tb[j];
           st4(a.u_out, k, vu, vec, cnt);
@@ -463,8 +476,7 @@ __global__ void __launch_bounds__(UPD_THREADS) layer_update_kernel(const LayerTa
       }
       if (have_contrib) {
         if (a.d_plr) {
-          float dp[4];
-          ld4(dp, a.d_plr, k, vec, cnt);
+          if (!plain) ld4(dp, a.d_plr, k, vec, cnt);
 #pragma unroll
           for (int j = 0; j < 4; ++j) dp[j] += contrib[j];
           st4(a.d_plr, k, dp, vec, cnt);
@@ -473,7 +485,7 @@ __global__ void __launch_bounds__(UPD_THREADS) layer_update_kernel(const LayerTa
           for (int j = 0; j < 4; ++j) acc += j < cnt ? contrib[j] : 0.f;
         }
       }
-      if (a.cast_src) ld4(vw, a.cast_src, k, vec, cnt);
+      if (!plain && a.cast_src) ld4(vw, a.cast_src, k, vec, cnt);
     } else {
       ld4(vw, a.cast_src, k, vec, cnt);
 #pragma unroll

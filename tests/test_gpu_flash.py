@@ -96,8 +96,9 @@ def test_flash_hvp(name):
 def test_flash_workspace_saving():
     """Without P and P' per block and the score scratch: the decoder_small workspace shrinks
     by (2 L + 2) B H S^2 bf16 values (P, P' per block; dS, dS') and 4 B H S^2 float32 values
-    (scores, score gradients and their tangents), less the row statistics (lse and rbar per
-    block, D and D') of 2 (L + 1) B H S float32 values."""
+    (scores, score gradients and their tangents) and the per-head float32 outputs O, O'
+    (2 B H S d_head values; the fused forward writes them head-merged in bf16), less the row
+    statistics (lse and rbar per block, D and D') of 2 (L + 1) B H S float32 values."""
     torch, native = need_gpu()
     w = synth.WORKLOADS["decoder_small"]
     mf = native.MixFlow.for_workload(w)
@@ -110,7 +111,8 @@ def test_flash_workspace_saving():
     S, L = w.seq, w.n_blocks
     BH = max(w.B, w.B_outer) * w.n_heads
     ss = BH * S * S
-    saved = (2 * L + 2) * ss * 2 + 4 * ss * 4 - (L + 1) * 2 * BH * S * 4
+    dh = w.d_model // w.n_heads
+    saved = (2 * L + 2) * ss * 2 + 4 * ss * 4 + 2 * BH * S * dh * 4 - (L + 1) * 2 * BH * S * 4
     assert abs((ws_m - ws_f) - saved) <= 256 * (4 * L + 16), (ws_m - ws_f, saved)
 
 
