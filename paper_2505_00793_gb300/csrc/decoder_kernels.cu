@@ -661,6 +661,7 @@ __global__ void ce_seed_kernel(int S, int V, const int* __restrict__ ids,
                                const float* __restrict__ lse, const float* __restrict__ pf,
                                const float* __restrict__ eta_w, const float* __restrict__ ex_w,
                                float inv_norm, T* __restrict__ dF, T* __restrict__ dFd, int ldo) {
+  // four consecutive logits per thread (V and ldo multiples of 8): 16-byte loads
   pdl_entry();
   const int r = blockIdx.y;
   const int b = r / S, s = r % S;
@@ -671,11 +672,19 @@ __global__ void ce_seed_kernel(int S, int V, const int* __restrict__ ids,
   const float c = w * inv_norm;
   const float lz = lse[r];
   const float pfr = Fd ? pf[r] : 0.f;
-  for (int col = blockIdx.x * blockDim.x + threadIdx.x; col < V; col += gridDim.x * blockDim.x) {
-    const int64_t o = static_cast<int64_t>(r) * V + col;
-    const float p = expf(F[o] - lz);
-    dF[static_cast<int64_t>(r) * ldo + col] = to_t<T>(c * (p - (col == y ? 1.f : 0.f)));
-    if (Fd) dFd[static_cast<int64_t>(r) * ldo + col] = to_t<T>(c * p * (Fd[o] - pfr));
+  const int64_t orow = static_cast<int64_t>(r) * V, drow = static_cast<int64_t>(r) * ldo;
+  for (int col = 4 * (blockIdx.x * blockDim.x + threadIdx.x); col < V;
+       col += 4 * gridDim.x * blockDim.x) {
+    const float4 f = *reinterpret_cast<const float4*>(F + orow + col);
+    const float p0 = expf(f.x - lz), p1 = expf(f.y - lz), p2 = expf(f.z - lz), p3 = expf(f.w - lz);
+    store4<T>(dF + drow + col, c * (p0 - (col == y ? 1.f : 0.f)),
+              c * (p1 - (col + 1 == y ? 1.f : 0.f)), c * (p2 - (col + 2 == y ? 1.f : 0.f)),
+              c * (p3 - (col + 3 == y ? 1.f : 0.f)));
+    if (Fd) {
+      const float4 fd = *reinterpret_cast<const float4*>(Fd + orow + col);
+      store4<T>(dFd + drow + col, c * p0 * (fd.x - pfr), c * p1 * (fd.y - pfr),
+                c * p2 * (fd.z - pfr), c * p3 * (fd.w - pfr));
+    }
   }
 }
 
@@ -994,7 +1003,7 @@ template <typename T>
 void dec_ce_seed(int N, int S, int V, const int* ids, const float* F, const float* Fd,
                  const float* lse, const float* pf, const float* eta_w, const float* ex_w,
                  float inv_norm, T* dF, T* dFd, int ldo, cudaStream_t s) {
-  dim3 grid((V + 255) / 256 > 16 ? 16 : (V + 255) / 256, N);
+  dim3 grid((V + 1023) / 1024 > 8 ? 8 : (V + 1023) / 1024, N);
   launch_k(ce_seed_kernel<T>, dim3(grid), dim3(256), 0, s, S, V, ids, F, Fd, lse, pf, eta_w, ex_w, inv_norm, dF, dFd,
                                          ldo);
 }
