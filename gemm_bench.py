@@ -19,6 +19,7 @@ SHAPES = [
     ("large transformer qkv dual", 8192, 3072, 1024, 25),
     ("large transformer W1 dual", 8192, 4096, 1024, 25),
     ("large transformer W2 dual", 8192, 1024, 4096, 25),
+    ("large transformer Wo dual", 8192, 1024, 1024, 25),
     ("large transformer head dual", 8192, 32768, 1024, 25),
     ("large transformer head weight tangent", 1024, 32768, 8192, 6),
     ("square 8192", 8192, 8192, 8192, 1),
@@ -33,6 +34,9 @@ def main() -> None:
     ap.add_argument("--only", default="", help="substring of the shape names to run")
     ap.add_argument("--persistent", type=int, nargs="?", const=1, default=None,
                     help="MF_OPT_GEMM_PERSISTENT mode (library default when absent)")
+    ap.add_argument("--split", action="store_true",
+                    help="dual products (terms 25) as two single-accumulator launches: "
+                         "C0 = A0 B0^T, then C1 = A1 B0^T + A0 B1^T")
     args = ap.parse_args()
     torch.cuda.set_device(0)
     if args.persistent is not None:   # a process-wide option, set through any handle
@@ -48,14 +52,20 @@ def main() -> None:
         A0, A1, B0, B1 = mk(M), mk(M), mk(N), mk(N)
         C0 = torch.empty(M, N, device="cuda")
         C1 = torch.empty(M, N, device="cuda")
+        def run():
+            if args.split and t == 25:
+                native.mf_dual_gemm_bf16(M, N, K, A0, A1, B0, B1, C0, None, 1, stream=s)
+                native.mf_dual_gemm_bf16(M, N, K, A0, A1, B0, B1, C1, None, 2 | 4, stream=s)
+            else:
+                native.mf_dual_gemm_bf16(M, N, K, A0, A1, B0, B1, C0, C1, t, stream=s)
         for _ in range(3):
-            native.mf_dual_gemm_bf16(M, N, K, A0, A1, B0, B1, C0, C1, t, stream=s)
+            run()
         torch.cuda.synchronize()
         n = 20 if M * N * K < 1e11 else 10
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(s)
         for _ in range(n):
-            native.mf_dual_gemm_bf16(M, N, K, A0, A1, B0, B1, C0, C1, t, stream=s)
+            run()
         e1.record(s)
         torch.cuda.synchronize()
         ms = e0.elapsed_time(e1) / n
@@ -70,7 +80,7 @@ def main() -> None:
         torch.cuda.synchronize()
         cb = e0.elapsed_time(e1) / n
         print(json.dumps({"name": name, "M": M, "N": N, "K": K, "terms": t,
-                          "persistent": args.persistent, "us": ms * 1e3,
+                          "persistent": args.persistent, "split": args.split, "us": ms * 1e3,
                           "tflops": 2.0 * M * N * K * terms / ms / 1e9,
                           "cublas_one_product_tflops": 2.0 * M * N * K / cb / 1e9}), flush=True)
         del A0, A1, B0, B1, C0, C1
