@@ -1712,7 +1712,7 @@ mf_status mf_checkpoint_plan(int T, int ckpt_every, int ckpt_slots, int* state_s
   const Store st = make_store(&lp);
   int64_t re = 0;
   if (st.bin) {
-    re = mf::revolve_schedule(T, st.bin).recompute;
+    re = mf::revolve_recompute_steps(mf::revolve_schedule(T, st.bin));
   } else if (st.k > 1) {
     // every segment but the last is re-run from its checkpoint: k - 1 steps each
     re = static_cast<int64_t>((T - 1) / st.k) * (st.k - 1);

@@ -5,8 +5,8 @@
 // The sweep reverses inner steps t = T-1, ..., 0 and needs the state S_t = (theta_t and the
 // optimiser state m_t, v_t) when it reverses step t.  With s snapshot slots besides S_0, a
 // schedule stores some states and recomputes the others by re-running inner steps forward
-// from a stored one.  This file computes the schedule that re-runs the fewest inner steps,
-// by dynamic programming over the split points of the classical recursion:
+// from a stored one.  This file computes the schedule that re-runs the fewest inner steps.
+// The classical recursion over split points defines the optimum:
 //
 //   F(n, s)  forward steps needed to reverse n consecutive steps [i, i + n) when S_i is
 //            stored and s slots are free:  F(1, s) = 0,  F(n, 0) = n (n - 1) / 2 (every S_t
@@ -18,6 +18,13 @@
 //            segment and can leave S_{i+m} in a slot on its way (no extra forward steps):
 //            G(1, s) = 0,  G(n, 0) = n (n - 1) / 2,
 //            G(n, s) = min(G(n, s - 1), min_{0<m<n} G(n - m, s - 1) + F(m, s)).
+//
+// Both have closed forms through Griewank's minimal count t(l, c) = r l - C(c + r, c + 1) for
+// reversing l steps with c checkpoints (r the least integer with C(c + r, c) >= l, Griewank
+// 1992):  F(n, s) = t(n, s + 1)  and  G(n, s) = t(n + 1, s + 1) - n.  The builder walks the
+// recursion and takes, at each node, the fewest slots and then the smallest split m that
+// reach the closed-form value, so the schedule needs no O(T^2 s) table: building one costs
+// O(T) nodes, each scanning its splits.
 //
 // Slots: 0 holds S_0; 1..s are the snapshot slots; s + 1 and s + 2 are two scratch slots
 // that an advance ping-pongs through, ending in its destination (S_T after the rollout and
@@ -44,54 +51,26 @@ struct RevolveSchedule {
   std::vector<int> keep;            // [T + 1]: slot the rollout leaves S_t in, or -1
   int slot_T = 0;                   // slot of S_T after the rollout
   std::vector<RevolveAct> acts;     // after the rollout and the outer gradient
-  int64_t recompute = 0;            // inner steps re-run by the sweep (G(T, s))
+  int64_t recompute = 0;            // inner steps re-run by the sweep: G(T, s)
   int n_slots() const { return s + 3; }
   int scratch(int j) const { return s + 1 + j; }
 };
 
 namespace revolve_detail {
 
-struct Tables {
-  int T, S;
-  std::vector<int64_t> F, G;      // [(n) * (S + 1) + s]
-  std::vector<int> fm, gm;        // best split (0 = naive or fewer slots, see fs/gs)
-  std::vector<int> fs, gs;        // slots actually used (<= s)
-  int64_t& f(int n, int s) { return F[static_cast<size_t>(n) * (S + 1) + s]; }
-  int64_t& g(int n, int s) { return G[static_cast<size_t>(n) * (S + 1) + s]; }
-  int& fmi(int n, int s) { return fm[static_cast<size_t>(n) * (S + 1) + s]; }
-  int& gmi(int n, int s) { return gm[static_cast<size_t>(n) * (S + 1) + s]; }
-  int& fsi(int n, int s) { return fs[static_cast<size_t>(n) * (S + 1) + s]; }
-  int& gsi(int n, int s) { return gs[static_cast<size_t>(n) * (S + 1) + s]; }
+// Griewank's t(l, c): forward steps to reverse l steps with c >= 1 checkpoints.
+inline int64_t griewank_t(int64_t l, int64_t c) {
+  if (l <= 1) return 0;
+  if (c == 1) return l * (l - 1) / 2;
+  int64_t r = 0, b = 1;                 // b = C(c + r, c)
+  while (b < l) { ++r; b = b * (c + r) / r; }
+  return r * l - b * r / (c + 1);       // C(c + r, c + 1) = C(c + r, c) r / (c + 1)
+}
 
-  Tables(int T_, int S_) : T(T_), S(S_) {
-    const size_t sz = static_cast<size_t>(T + 1) * (S + 1);
-    F.assign(sz, 0); G.assign(sz, 0);
-    fm.assign(sz, 0); gm.assign(sz, 0); fs.assign(sz, 0); gs.assign(sz, 0);
-    for (int n = 1; n <= T; ++n) {
-      for (int s = 0; s <= S; ++s) {
-        const int64_t naive = static_cast<int64_t>(n) * (n - 1) / 2;
-        if (n == 1 || s == 0) {
-          f(n, s) = g(n, s) = n == 1 ? 0 : naive;
-          fmi(n, s) = gmi(n, s) = 0;
-          fsi(n, s) = gsi(n, s) = s;
-          continue;
-        }
-        // fewer slots first (ties keep the smaller slot count)
-        f(n, s) = f(n, s - 1); fmi(n, s) = fmi(n, s - 1); fsi(n, s) = fsi(n, s - 1);
-        g(n, s) = g(n, s - 1); gmi(n, s) = gmi(n, s - 1); gsi(n, s) = gsi(n, s - 1);
-        for (int m = 1; m < n; ++m) {
-          const int64_t cf = m + f(n - m, s - 1) + f(m, s);
-          if (cf < f(n, s)) { f(n, s) = cf; fmi(n, s) = m; fsi(n, s) = s; }
-          const int64_t cg = g(n - m, s - 1) + f(m, s);
-          if (cg < g(n, s)) { g(n, s) = cg; gmi(n, s) = m; gsi(n, s) = s; }
-        }
-      }
-    }
-  }
-};
+inline int64_t F(int n, int s) { return griewank_t(n, static_cast<int64_t>(s) + 1); }
+inline int64_t G(int n, int s) { return griewank_t(n + 1, static_cast<int64_t>(s) + 1) - n; }
 
 struct Builder {
-  Tables& tb;
   RevolveSchedule& out;
   std::vector<int> free_slots;
 
@@ -107,9 +86,27 @@ struct Builder {
     out.acts.push_back({RevolveAct::REV, i, 0, a, 0});
   }
 
+  // fewest slots su <= s that reach the optimum of n steps, then the smallest split m
+  // (0 when su == 0: the naive schedule)
+  template <bool TOP>
+  void choose(int n, int s, int& su, int& m) const {
+    if (s > n) s = n;                     // more slots than steps never help
+    const int64_t v = TOP ? G(n, s) : F(n, s);
+    su = s;
+    while (su > 0 && (TOP ? G(n, su - 1) : F(n, su - 1)) == v) --su;
+    m = 0;
+    if (su == 0) return;
+    for (int k = 1; k < n; ++k) {
+      const int64_t c = TOP ? G(n - k, su - 1) + F(k, su) : k + F(n - k, su - 1) + F(k, su);
+      if (c == v) { m = k; return; }
+    }
+    su = 0;                               // unreachable when the closed forms hold
+  }
+
   void rev_f(int i, int n, int a, int s) {
     if (n == 1) { out.acts.push_back({RevolveAct::REV, i, 0, a, 0}); return; }
-    const int su = tb.fsi(n, s), m = tb.fmi(n, s);
+    int su, m;
+    choose<false>(n, s, su, m);
     if (su == 0 || m == 0) { naive(i, n, a); return; }
     const int b = take();
     out.acts.push_back({RevolveAct::ADV, i, i + m, a, b});
@@ -120,7 +117,8 @@ struct Builder {
 
   void rev_g(int i, int n, int a, int s) {
     if (n == 1) { out.acts.push_back({RevolveAct::REV, i, 0, a, 0}); return; }
-    const int su = tb.gsi(n, s), m = tb.gmi(n, s);
+    int su, m;
+    choose<true>(n, s, su, m);
     if (su == 0 || m == 0) { naive(i, n, a); return; }
     const int b = take();
     out.keep[i + m] = b;              // the rollout leaves S_{i+m} in slot b
@@ -139,11 +137,10 @@ inline RevolveSchedule revolve_schedule(int T, int s) {
   r.s = s;
   r.keep.assign(T + 1, -1);
   r.keep[0] = 0;
-  revolve_detail::Tables tb(T, s);
-  revolve_detail::Builder b{tb, r, {}};
+  revolve_detail::Builder b{r, {}};
   for (int j = s; j >= 1; --j) b.free_slots.push_back(j);
   b.rev_g(0, T, 0, s);
-  r.recompute = tb.g(T, s);
+  r.recompute = revolve_detail::G(T, s);
   r.slot_T = r.scratch(0);
   return r;
 }

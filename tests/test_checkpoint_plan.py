@@ -5,6 +5,10 @@ optimum for reversing l steps with c checkpoints, t(l, c) = r l - C(c + r, c + 1
 repetition number, C(c + r - 1, c) < l <= C(c + r, c): in this library's accounting (the
 reverse of step t re-runs that step's forward inside the Hessian-vector product, and S_0 is
 stored apart from the s snapshot slots) the sweep re-runs t(T + 1, s + 1) - T inner steps."""
+import os
+import shutil
+import subprocess
+from functools import lru_cache
 from math import comb
 
 import pytest
@@ -20,6 +24,22 @@ def _griewank(l, c):
     return r * l - comb(c + r, c + 1)
 
 
+@lru_cache(maxsize=None)
+def _recursion(n, s, top):
+    """The split-point recursion itself, by brute force: F (top=False) reverses n steps
+    from a stored S_i with s free slots, each split paying m steps to advance; G (top=True)
+    splits the rolled-out top level, whose advances are free."""
+    if n == 1:
+        return 0
+    if s == 0:
+        return n * (n - 1) // 2
+    best = _recursion(n, s - 1, top)
+    for m in range(1, n):
+        c = _recursion(n - m, s - 1, top) + _recursion(m, s, False) + (0 if top else m)
+        best = min(best, c)
+    return best
+
+
 def _plan(T, k=1, s=0):
     try:
         return native.checkpoint_plan(T, k, s)
@@ -33,6 +53,41 @@ def test_binomial_recompute_is_griewank_optimum(T):
         slots, re = _plan(T, 1, s)
         assert re == _griewank(T + 1, min(s, max(T - 1, 1)) + 1) - T, (T, s, re)
         assert slots == min(s, max(T - 1, 1)) + 3
+
+
+def test_binomial_recompute_is_recursion_optimum():
+    # the library builds its schedule from closed forms; the recursion they solve, by brute force
+    for T in range(1, 41):
+        for s in range(1, 9):
+            sb = min(s, max(T - 1, 1))
+            assert _plan(T, 1, s)[1] == _recursion(T, sb, True), (T, s)
+
+
+def test_binomial_schedule_replays():
+    """Replays the library's schedules slot by slot on the host (tests/revolve_check.cpp)."""
+    gxx = shutil.which("g++")
+    if gxx is None:
+        pytest.skip("g++ not found")
+    here = os.path.dirname(os.path.abspath(__file__))
+    csrc = os.path.join(os.path.dirname(here), "paper_2505_00793_gb300", "csrc")
+    exe = os.path.join(os.environ.get("TMPDIR", "/tmp"), f"revolve_check_{os.getpid()}")
+    subprocess.run([gxx, "-std=c++17", "-O2", "-I", csrc, os.path.join(here, "revolve_check.cpp"),
+                    "-o", exe], check=True)
+    try:
+        out = subprocess.run([exe], capture_output=True, text=True, timeout=120)
+    finally:
+        if os.path.exists(exe):
+            os.remove(exe)
+    assert out.returncode == 0 and "bad=0" in out.stdout, out.stdout[-2000:]
+
+
+def test_binomial_plan_is_fast_at_the_limits():
+    # the closed forms keep the largest schedule (T = 4096, s = 1024) to milliseconds
+    import time
+    t0 = time.perf_counter()
+    slots, re = _plan(4096, 1, 1024)
+    assert time.perf_counter() - t0 < 5.0
+    assert (slots, re) == (1027, _griewank(4097, 1025) - 4096)
 
 
 def test_binomial_trade_off():
