@@ -20,6 +20,7 @@ SHAPES = [
     ("large transformer W1 dual", 8192, 4096, 1024, 25),
     ("large transformer W2 dual", 8192, 1024, 4096, 25),
     ("large transformer Wo dual", 8192, 1024, 1024, 25),
+    ("large transformer Wqkv data dual", 8192, 1024, 3072, 25),
     ("large transformer head dual", 8192, 32768, 1024, 25),
     ("large transformer head weight tangent", 1024, 32768, 8192, 6),
     ("square 8192", 8192, 8192, 8192, 1),

@@ -102,21 +102,21 @@ __device__ __forceinline__ void act_eval_t(float z, float& f, float& d1, float& 
   }
 }
 
+// The per-element arithmetic of epi_eval_t on values already loaded: z, zd the stored
+// pre-activation and its tangent (EPI_ACT_BWD), b0, b1 the biases (0 when absent).
 template <int MODE, int ACT>
-__device__ __forceinline__ EpiOut epi_eval_t(const EpiParams& e, int m, int n, float acc0,
-                                             float acc1, const float* bias0,
-                                             const float* bias1, bool dual) {
+__device__ __forceinline__ EpiOut epi_core_t(float acc0, float acc1, float z_in, float zd_in,
+                                             float b0, float b1, bool dual) {
   EpiOut r;
   if constexpr (MODE == EPI_ACT_BWD) {
-    const float z = e.Z[static_cast<int64_t>(m) * e.ldz + n];
     float f, d1, d2;
-    act_eval_t<ACT>(z, f, d1, d2);
+    act_eval_t<ACT>(z_in, f, d1, d2);
     r.c0 = acc0; r.c1 = acc1;
     r.o0 = d1 * acc0;
-    r.o1 = dual ? d2 * e.Zd[static_cast<int64_t>(m) * e.ldz + n] * acc0 + d1 * acc1 : 0.f;
+    r.o1 = dual ? d2 * zd_in * acc0 + d1 * acc1 : 0.f;
   } else {
-    const float z = acc0 + (bias0 ? bias0[n] : 0.f);
-    const float zd = acc1 + (bias1 ? bias1[n] : 0.f);
+    const float z = acc0 + b0;
+    const float zd = acc1 + b1;
     r.c0 = z; r.c1 = zd;
     if constexpr (MODE == EPI_ACT_FWD) {
       float f, d1, d2;
@@ -128,6 +128,20 @@ __device__ __forceinline__ EpiOut epi_eval_t(const EpiParams& e, int m, int n, f
     }
   }
   return r;
+}
+
+template <int MODE, int ACT>
+__device__ __forceinline__ EpiOut epi_eval_t(const EpiParams& e, int m, int n, float acc0,
+                                             float acc1, const float* bias0,
+                                             const float* bias1, bool dual) {
+  if constexpr (MODE == EPI_ACT_BWD) {
+    const float z = e.Z[static_cast<int64_t>(m) * e.ldz + n];
+    const float zd = dual ? e.Zd[static_cast<int64_t>(m) * e.ldz + n] : 0.f;
+    return epi_core_t<MODE, ACT>(acc0, acc1, z, zd, 0.f, 0.f, dual);
+  } else {
+    return epi_core_t<MODE, ACT>(acc0, acc1, 0.f, 0.f, bias0 ? bias0[n] : 0.f,
+                                 bias1 ? bias1[n] : 0.f, dual);
+  }
 }
 
 }  // namespace mf

@@ -342,6 +342,149 @@ __device__ __forceinline__ void epilogue16(const TcParams& p, int row, int col0,
   }
 }
 
+// ---- warp-cooperative row blocks through shared memory ---------------------------------
+// The row-per-thread epilogues hold one accumulator row per lane (tcgen05.ld 32x32b), so a
+// warp's direct 16-byte store touches 32 rows, 32 memory lines.  These helpers move a block
+// of 32 rows x 64 bytes through a 2 KB per-warp buffer instead: lane l handles 16-byte quad
+// l % 4 of rows l / 4 + 8 i (i = 0..3), so each warp access covers 8 rows x 64 bytes.  Row r's
+// quad c sits at 128-byte line r >> 1, slot (r & 1) * 4 + (c ^ ((r >> 1) & 3)): both the
+// row-wise and the quad-wise accesses of a warp are free of bank conflicts.
+constexpr int STG_ROWS_BYTES = 32 * 64;
+
+__device__ __forceinline__ int stg_quad(int r, int c) {
+  return (r >> 1) * 128 + ((((r & 1) << 2) | (c ^ ((r >> 1) & 3))) << 4);
+}
+
+// Rows row0 .. row0 + 31 (those below M) of a float32 matrix, 16 columns from col0 (16-byte
+// aligned rows), into this lane's row: out[j] = src[(row0 + lane) * ld + col0 + j].
+__device__ __forceinline__ void warp_load_rows16(uint8_t* stg, int lane, int row0, int M,
+                                                 const float* src, int64_t ld, int col0,
+                                                 float (&out)[16]) {
+  const int rq = lane >> 2, cq = lane & 3;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int r = rq + 8 * i;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (row0 + r < M) v = *reinterpret_cast<const float4*>(src + (row0 + r) * ld + col0 + 4 * cq);
+    *reinterpret_cast<float4*>(stg + stg_quad(r, cq)) = v;
+  }
+  __syncwarp();
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    const float4 v = *reinterpret_cast<const float4*>(stg + stg_quad(lane, c));
+    out[4 * c] = v.x; out[4 * c + 1] = v.y; out[4 * c + 2] = v.z; out[4 * c + 3] = v.w;
+  }
+  __syncwarp();
+}
+
+// This lane's 64-byte row (quads q[0..3]) of a 32-row block, stored by quads: quad c of
+// row r goes to dst(r, c) (nullptr: not stored) when row0 + r < M.
+template <class Dst>
+__device__ __forceinline__ void warp_store_rows(uint8_t* stg, int lane, int row0, int M,
+                                                const uint4 (&q)[4], Dst dst) {
+#pragma unroll
+  for (int c = 0; c < 4; ++c) *reinterpret_cast<uint4*>(stg + stg_quad(lane, c)) = q[c];
+  __syncwarp();
+  const int rq = lane >> 2, cq = lane & 3;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int r = rq + 8 * i;
+    const uint4 v = *reinterpret_cast<const uint4*>(stg + stg_quad(r, cq));
+    void* d = dst(r, cq);
+    if (d && row0 + r < M) *reinterpret_cast<uint4*>(d) = v;
+  }
+  __syncwarp();
+}
+
+__device__ __forceinline__ uint4 quad_f32(const float* v) {
+  return make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]),
+                    __float_as_uint(v[3]));
+}
+__device__ __forceinline__ uint4 quad_bf16(const float* v) {
+  return make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
+                    pack_bf16x2(v[6], v[7]));
+}
+
+// Whether the coalesced row-block epilogue may serve this GEMM: 16-byte aligned rows of
+// every matrix it reads or writes.
+__device__ __forceinline__ bool rows16_ok(const TcParams& p, int mode, bool dual) {
+  auto al = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15) == 0; };
+  bool ok = true;
+  if (p.C0) ok = ok && al(p.C0) && !(p.ldc0 & 3);
+  if (p.C1 && dual) ok = ok && al(p.C1) && !(p.ldc1 & 3);
+  if (mode != EPI_STORE) {
+    if (p.epi.A) ok = ok && al(p.epi.A) && !(p.epi.lda & 7);
+    if (p.epi.Ad && dual) ok = ok && al(p.epi.Ad) && !(p.epi.lda & 7);
+  }
+  if (mode == EPI_ACT_BWD) {
+    ok = ok && al(p.epi.Z) && !(p.epi.ldz & 3);
+    if (dual) ok = ok && al(p.epi.Zd);
+  }
+  return ok;
+}
+
+// epilogue16 for a full chunk (col0 + 16 <= N) of the warp's 32 rows row0 .. row0 + 31, with
+// the stored pre-activations read and the outputs written through the per-warp buffer stg
+// (STG_ROWS_BYTES).  The arithmetic per element is epi_core_t, as in epilogue16.
+template <int MODE, int ACT>
+__device__ __forceinline__ void epilogue16_rows(const TcParams& p, uint8_t* stg, int lane,
+                                                int row0, int col0, const float (&v0)[16],
+                                                const float (&v1)[16], bool dual) {
+  const EpiParams e = p.epi;
+  const int row = row0 + lane;
+  const bool rowok = row < p.M;
+  float z[16], zd[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) z[j] = zd[j] = 0.f;
+  if constexpr (MODE == EPI_ACT_BWD) {
+    warp_load_rows16(stg, lane, row0, p.M, e.Z, e.ldz, col0, z);
+    if (dual) warp_load_rows16(stg, lane, row0, p.M, e.Zd, e.ldz, col0, zd);
+  }
+  float c0[16], c1[16], o0[16], o1[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const int n = col0 + j;
+    EpiOut o;
+    if (rowok) {
+      const float b0 = MODE != EPI_ACT_BWD && p.bias0 ? p.bias0[n] : 0.f;
+      const float b1 = MODE != EPI_ACT_BWD && p.bias1 ? p.bias1[n] : 0.f;
+      o = epi_core_t<MODE, ACT>(v0[j], v1[j], z[j], zd[j], b0, b1, dual);
+    } else {
+      o.c0 = o.c1 = o.o0 = o.o1 = 0.f;
+    }
+    c0[j] = o.c0; c1[j] = o.c1; o0[j] = o.o0; o1[j] = o.o1;
+  }
+  if (p.C0) {
+    const uint4 q[4] = {quad_f32(c0), quad_f32(c0 + 4), quad_f32(c0 + 8), quad_f32(c0 + 12)};
+    float* const C = p.C0;
+    const int64_t ld = p.ldc0;
+    warp_store_rows(stg, lane, row0, p.M, q, [&](int r, int c) -> void* {
+      return C + (row0 + r) * ld + col0 + 4 * c;
+    });
+  }
+  if (p.C1 && dual) {
+    const uint4 q[4] = {quad_f32(c1), quad_f32(c1 + 4), quad_f32(c1 + 8), quad_f32(c1 + 12)};
+    float* const C = p.C1;
+    const int64_t ld = p.ldc1;
+    warp_store_rows(stg, lane, row0, p.M, q, [&](int r, int c) -> void* {
+      return C + (row0 + r) * ld + col0 + 4 * c;
+    });
+  }
+  if constexpr (MODE != EPI_STORE) {
+    // A and Ad rows side by side: quads 0, 1 of A, quads 2, 3 of Ad
+    __nv_bfloat16* const A = static_cast<__nv_bfloat16*>(e.A);
+    __nv_bfloat16* const Ad = dual ? static_cast<__nv_bfloat16*>(e.Ad) : nullptr;
+    if (A || Ad) {
+      const uint4 q[4] = {quad_bf16(o0), quad_bf16(o0 + 8), quad_bf16(o1), quad_bf16(o1 + 8)};
+      const int64_t ld = e.lda;
+      warp_store_rows(stg, lane, row0, p.M, q, [&](int r, int c) -> void* {
+        __nv_bfloat16* X = c < 2 ? A : Ad;
+        return X ? X + (row0 + r) * ld + col0 + 8 * (c & 1) : nullptr;
+      });
+    }
+  }
+}
+
 __device__ __forceinline__ void fence_proxy_async() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -362,10 +505,13 @@ __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wa
 
 // Per-warp staging of a 32-row slab of the tile for TMA stores (128-byte swizzle: the
 // 16-byte chunk j of row r sits at chunk position j ^ (r % 8) of the row's 128 bytes).
-// Layout per warp: C0 [2 boxes of 32x32 f32] | C1 [2 boxes] | A [32x64 bf16] | Ad [32x64].
+// Layout per warp: C0 [2 boxes of 32x32 f32] | C1 [2 boxes] | A [32x64 bf16] | Ad [32x64],
 constexpr int STG_F32_BOX = 32 * 32 * 4;          // 4 KB
 constexpr int STG_BF16_BOX = 32 * 64 * 2;         // 4 KB
-constexpr int STG_WARP = 4 * STG_F32_BOX + 2 * STG_BF16_BOX;   // 24 KB
+// ... followed by the row-block buffer (STG_ROWS_BYTES) through which the backward
+// epilogues read the stored pre-activations.
+constexpr int STG_ZROWS = 4 * STG_F32_BOX + 2 * STG_BF16_BOX;
+constexpr int STG_WARP = STG_ZROWS + STG_ROWS_BYTES;              // 26 KB
 
 // TMA-store epilogue of one warp (32 rows) over the tile's BN columns, 64 at a time.
 template <int BN, int MODE, int ACT>
@@ -381,7 +527,14 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
   uint8_t* sC1 = stg + 2 * STG_F32_BOX;
   uint8_t* sA = stg + 4 * STG_F32_BOX;
   uint8_t* sAd = sA + STG_BF16_BOX;
+  uint8_t* sZ = stg + STG_ZROWS;
   const int sw = lane & 7;
+  // backward epilogues: the stored pre-activations of full chunks through sZ
+  bool zrows_ok = false;
+  if constexpr (MODE == EPI_ACT_BWD) {
+    auto al = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15) == 0; };
+    zrows_ok = al(e.Z) && !(e.ldz & 3) && (!dual || al(e.Zd));
+  }
   for (int c = c_begin; c < c_end; c += 64) {
     if (c > c_begin) {
       if (lane == 0) bulk_wait_read();
@@ -399,12 +552,28 @@ __device__ __forceinline__ void epilogue_tma(const TcParams& p, const CUtensorMa
         for (int j = 0; j < 16; ++j) v1[j] = 0.f;
       }
       float c0[16], c1[16], o0[16], o1[16];
+      float z[16], zd[16];
+      const bool zrows = zrows_ok && n0 + cc + 16 <= p.N;     // warp-uniform
+      if constexpr (MODE == EPI_ACT_BWD) {
+        if (zrows) {
+          warp_load_rows16(sZ, lane, m0 + q * 32, p.M, e.Z, e.ldz, n0 + cc, z);
+          if (dual) warp_load_rows16(sZ, lane, m0 + q * 32, p.M, e.Zd, e.ldz, n0 + cc, zd);
+          else {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) zd[j] = 0.f;
+          }
+        }
+      }
 #pragma unroll
       for (int j = 0; j < 16; ++j) {
         const int n = n0 + cc + j;
         EpiOut o;
-        if (rowok && n < p.N) o = epi_eval_t<MODE, ACT>(e, row, n, v0[j], v1[j], p.bias0, p.bias1, dual);
-        else o.c0 = o.c1 = o.o0 = o.o1 = 0.f;
+        if (rowok && n < p.N) {
+          if (MODE == EPI_ACT_BWD && zrows) o = epi_core_t<MODE, ACT>(v0[j], v1[j], z[j], zd[j], 0.f, 0.f, dual);
+          else o = epi_eval_t<MODE, ACT>(e, row, n, v0[j], v1[j], p.bias0, p.bias1, dual);
+        } else {
+          o.c0 = o.c1 = o.o0 = o.o1 = 0.f;
+        }
         c0[j] = o.c0; c1[j] = o.c1; o0[j] = o.o0; o1[j] = o.o1;
       }
       // float32 slabs: box (sub / 2), chunks (sub % 2) * 4 .. + 3 of the 128-byte row
@@ -475,6 +644,57 @@ __device__ __forceinline__ void mma_commit_pair(uint64_t* bar) {
       : "memory");
 }
 
+// The MMA issuer's barrier operations on precomputed shared-memory addresses (the issue
+// loop keeps its ring position and descriptors in registers: a single thread issues every
+// MMA, and each instruction between two MMAs delays the tensor pipe).
+__device__ __forceinline__ bool mbar_try_wait_addr(uint32_t addr, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(addr), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ bool mbar_wait_addr(uint32_t addr, uint32_t parity, int* status,
+                                               long long limit_ns) {
+  if (mbar_try_wait_addr(addr, parity)) return true;
+  const long long t0 = global_ns();
+  while (true) {
+    if (mbar_try_wait_addr(addr, parity)) return true;
+    if (global_ns() - t0 > limit_ns) {
+      if (status) atomicMax(status, DEV_TIMEOUT);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void mma_commit_addr(uint32_t addr) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   addr)
+               : "memory");
+}
+
+__device__ __forceinline__ void mma_commit_pair_addr(uint32_t addr) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(addr),
+      "h"(static_cast<uint16_t>(3))
+      : "memory");
+}
+
+// Shared-memory descriptors of one operand for stage 0 of the ring.  The descriptor's
+// address field holds (address & 0x3FFFF) >> 4 in its low 14 bits, and every stage, K atom
+// and K slice lies inside the CTA's shared memory, so moving a descriptor by a byte offset
+// is a 64-bit add of offset >> 4 that never carries out of the field.
+__device__ __forceinline__ uint64_t op_desc(uint32_t sbase, int off, int mn) {
+  if (off < 0) return 0;
+  return mn ? sdesc_mn_sw128(sbase + off) : sdesc_sw128(sbase + off);
+}
+
 struct MmaLoop {
   int nk, stages, stage_bytes, a0_off, a1_off, b0_off, b1_off;
   int a_mn, b_mn;
@@ -488,8 +708,10 @@ struct MmaLoop {
 // The MMA issuer's loop over K blocks.  TERMS != 0 fixes the product mask at compile time
 // (TERMS = 0 reads `terms` at run time) so that the issue sequence is straight-line code:
 // a single thread issues every tcgen05.mma, and instructions between MMAs delay the tensor
-// pipe.  Products of K slice kk go to accumulator block kk mod NSUB (see ld_acc16).  PAIR
-// issues the M = 256 form for a CTA pair and multicasts the commits to both CTAs.
+// pipe.  The ring position, the barrier addresses and the operand descriptors advance by
+// additions (no division by the stage count, no descriptor rebuilt per K block).  Products
+// of K slice kk go to accumulator block kk mod NSUB (see ld_acc16).  PAIR issues the M = 256
+// form for a CTA pair and multicasts the commits to both CTAs.
 template <int BN, int KA, unsigned TERMS, int NSUB, bool PAIR>
 __device__ __forceinline__ void mma_loop(const MmaLoop& L, unsigned terms_rt, int nsub_rt) {
   constexpr int A_ATOM = BM * BK * 2, B_ATOM = (PAIR ? BN / 2 : BN) * BK * 2;
@@ -498,34 +720,34 @@ __device__ __forceinline__ void mma_loop(const MmaLoop& L, unsigned terms_rt, in
                          (static_cast<uint32_t>(L.b_mn) << 16);
   // descriptor advance per K=16 slice, in 16-byte units: 32 bytes K-major, 16 rows MN-major
   const uint64_t stepA = L.a_mn ? 128u : 2u, stepB = L.b_mn ? 128u : 2u;
+  // per K atom (KA > 1, K-major operands only)
+  const uint64_t atomA = L.a_mn ? 0u : static_cast<uint64_t>(A_ATOM >> 4);
+  const uint64_t atomB = L.b_mn ? 0u : static_cast<uint64_t>(B_ATOM >> 4);
   const unsigned terms = TERMS ? TERMS : terms_rt;
   const uint32_t nsub = NSUB ? static_cast<uint32_t>(NSUB) : static_cast<uint32_t>(nsub_rt);
   // products into C0 / C1 per K slice
   const uint32_t p0 = __popc(terms & (T_C0_A0B0 | T_C0_A1B0 | T_C0_A0B1 | T_C0_A1B1));
   const uint32_t p1 = __popc(terms & (T_C1_A1B0 | T_C1_A0B1));
+  const uint64_t a0s = op_desc(L.sbase, L.a0_off, L.a_mn), a1s = op_desc(L.sbase, L.a1_off, L.a_mn);
+  const uint64_t b0s = op_desc(L.sbase, L.b0_off, L.b_mn), b1s = op_desc(L.sbase, L.b1_off, L.b_mn);
+  const uint64_t stage_step = static_cast<uint64_t>(L.stage_bytes >> 4);
+  const uint32_t full0 = smem_u32(L.full_bar), empty0 = smem_u32(L.empty_bar);
+  int s = 0;
+  uint32_t ph = 0;
+  uint64_t soff = 0;   // descriptor offset of stage s
   bool live = true;   // false after a timed-out wait: consume the stages without MMAs
   for (int i = 0; i < L.nk; ++i) {
-    const int s = i % L.stages;
-    const uint32_t ph = (i / L.stages) & 1;
-    if (!live || !mbar_wait(&L.full_bar[s], ph, L.status, L.wait_ns)) {
+    const uint32_t fb = full0 + 8u * static_cast<uint32_t>(s);
+    if (!live || !mbar_wait_addr(fb, ph, L.status, L.wait_ns)) {
       live = false;
-      if (!mbar_wait(&L.full_bar[s], ph, L.status, DRAIN_NS)) break;
+      if (!mbar_wait_addr(fb, ph, L.status, DRAIN_NS)) break;
     }
     tc_fence_after();
-    const uint32_t st = L.sbase + s * L.stage_bytes;
     if (live) {
 #pragma unroll
     for (int a = 0; a < KA; ++a) {
-      auto descA = [&](int off) {
-        return L.a_mn ? sdesc_mn_sw128(st + off) : sdesc_sw128(st + off + a * A_ATOM);
-      };
-      auto descB = [&](int off) {
-        return L.b_mn ? sdesc_mn_sw128(st + off) : sdesc_sw128(st + off + a * B_ATOM);
-      };
-      const uint64_t a0 = L.a0_off >= 0 ? descA(L.a0_off) : 0;
-      const uint64_t a1 = L.a1_off >= 0 ? descA(L.a1_off) : 0;
-      const uint64_t b0 = L.b0_off >= 0 ? descB(L.b0_off) : 0;
-      const uint64_t b1 = L.b1_off >= 0 ? descB(L.b1_off) : 0;
+      const uint64_t a0 = a0s + soff + a * atomA, a1 = a1s + soff + a * atomA;
+      const uint64_t b0 = b0s + soff + a * atomB, b1 = b1s + soff + a * atomB;
 #pragma unroll
       for (int kk = 0; kk < BK / 16; ++kk) {
         // The j-th product of K slice kk into accumulator c goes to block
@@ -552,8 +774,16 @@ __device__ __forceinline__ void mma_loop(const MmaLoop& L, unsigned terms_rt, in
       }
     }
     }
-    if constexpr (PAIR) mma_commit_pair(&L.empty_bar[s]);
-    else mma_commit(&L.empty_bar[s]);
+    const uint32_t eb = empty0 + 8u * static_cast<uint32_t>(s);
+    if constexpr (PAIR) mma_commit_pair_addr(eb);
+    else mma_commit_addr(eb);
+    if (++s == L.stages) {
+      s = 0;
+      ph ^= 1u;
+      soff = 0;
+    } else {
+      soff += stage_step;
+    }
   }
 }
 

@@ -1,4 +1,4 @@
-// Persistent CTA-pair form of the tcgen05 dual GEMM (opt-in: MF_OPT_GEMM_PERSISTENT).
+// Persistent CTA-pair form of the tcgen05 dual GEMM (MF_OPT_GEMM_PERSISTENT, on by default).
 //
 // The one-tile kernels of tc_gemm_impl.cuh give every 256 x BN output tile its own CTA pair,
 // so each tile pays the prologue (barrier init, TMEM allocation, tensor-map prefetch) and its
@@ -14,8 +14,9 @@
 // Roles per CTA (as in the one-tile pair kernel): warp 0 issues the TMA loads of this CTA's
 // 128 rows of A and BN/2 rows of B; warp 1 owns TMEM, and in the even CTA one thread issues
 // tcgen05.mma.cta_group::2 (M = 256) for the pair; EPI_WARPS_P warps drain this CTA's 128
-// accumulator rows, one TMEM lane quadrant and one column share per warp, storing straight
-// from registers (no staging buffer, so all of shared memory is pipeline).
+// accumulator rows, one TMEM lane quadrant and one column share per warp; full 16-column
+// chunks are stored through a 2 KB row-block buffer per warp (8 rows x 64 bytes per warp
+// store, see epilogue16_rows), ragged ones straight from registers.
 //
 // Barriers: full[s] / empty[s] per pipeline stage (full in the even CTA, completed by both
 // CTAs' TMA bytes; empty in both, by the MMA commit multicast); per accumulator set,
@@ -75,7 +76,8 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
 }
 
 // Bounded wait of the MMA issuer and the epilogue warps (limit_ns = TcParams::wait_ns) that
-// gives up at once when another of these roles in this CTA has timed out already.  CLUSTER
+// gives up at once, unless the phase has already completed, when another of these roles in
+// this CTA has timed out.  CLUSTER
 // selects cluster-scope acquire (arrivals from the peer CTA).  The TMA producer never looks
 // at the abort flag: it waits with DRAIN_NS only, so both CTAs' producers see the same MMA
 // commits and stop at the same stage (see tc_gemm_impl.cuh).
@@ -85,11 +87,28 @@ __device__ __forceinline__ bool pwait(uint64_t* bar, uint32_t parity, int* statu
   auto probe = [&]() {
     return CLUSTER ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity);
   };
-  if (*abort) return false;
   if (probe()) return true;
+  if (*abort) return false;
   const long long t0 = global_ns();
   while (true) {
     if (probe()) return true;
+    if (*abort) return false;
+    if (global_ns() - t0 > limit_ns) {
+      if (status) atomicMax(status, DEV_TIMEOUT);
+      *abort = 1;
+      return false;
+    }
+  }
+}
+
+// The same wait on a precomputed shared::cta address (this CTA's barrier, CTA-scope acquire).
+__device__ __forceinline__ bool pwait_addr(uint32_t addr, uint32_t parity, int* status,
+                                           volatile int* abort, long long limit_ns) {
+  if (mbar_try_wait_addr(addr, parity)) return true;
+  if (*abort) return false;
+  const long long t0 = global_ns();
+  while (true) {
+    if (mbar_try_wait_addr(addr, parity)) return true;
     if (*abort) return false;
     if (global_ns() - t0 > limit_ns) {
       if (status) atomicMax(status, DEV_TIMEOUT);
@@ -108,13 +127,21 @@ __device__ __forceinline__ void mma_commit_even(uint64_t* bar) {
       : "memory");
 }
 
+// The MMA issuer's ring state, carried across tiles: stage s and its phase, the barrier
+// addresses of stage 0 and the stage-0 operand descriptors (see op_desc).
+struct IssueRing {
+  uint64_t a0s, a1s, b0s, b1s, stage_step, soff;
+  uint32_t full0, empty0, ph;
+  int s;
+};
+
 // The MMA issuer's loop over the K blocks of one tile, with the issue order and the
-// accumulator-block rotation of mma_loop (KA = 1, pair form).  The stage ring position
-// continues from g0, the K blocks issued for this pair's earlier tiles; the tile's
-// accumulators start at TMEM address tset.  Once `live` is false (a wait gave up) the
-// stages are consumed without MMAs.  Returns false if even a drain wait gave up.
+// accumulator-block rotation of mma_loop (KA = 1, pair form); the ring position continues
+// from the pair's earlier tiles.  The tile's accumulators start at TMEM address tset.  Once
+// `live` is false (a wait gave up) the stages are consumed without MMAs.  Returns false if
+// even a drain wait gave up.
 template <int BN, unsigned TERMS, int NSUB>
-__device__ __forceinline__ bool mma_tile(const MmaLoop& L, int g0, uint32_t tset,
+__device__ __forceinline__ bool mma_tile(const MmaLoop& L, IssueRing& R, uint32_t tset,
                                          unsigned terms_rt, int nsub_rt, volatile int* abort,
                                          bool& live) {
   const uint32_t idesc = idesc_bf16(2 * BM, BN) | (static_cast<uint32_t>(L.a_mn) << 15) |
@@ -125,73 +152,74 @@ __device__ __forceinline__ bool mma_tile(const MmaLoop& L, int g0, uint32_t tset
   const uint32_t p0 = __popc(terms & (T_C0_A0B0 | T_C0_A1B0 | T_C0_A0B1 | T_C0_A1B1));
   const uint32_t p1 = __popc(terms & (T_C1_A1B0 | T_C1_A0B1));
   for (int i = 0; i < L.nk; ++i) {
-    const int g = g0 + i;
-    const int s = g % L.stages;
-    const uint32_t ph = (g / L.stages) & 1;
-    if (!live || !pwait<false>(&L.full_bar[s], ph, L.status, abort, L.wait_ns)) {
+    const uint32_t fb = R.full0 + 8u * static_cast<uint32_t>(R.s);
+    const uint32_t eb = R.empty0 + 8u * static_cast<uint32_t>(R.s);
+    if (!live || !pwait_addr(fb, R.ph, L.status, abort, L.wait_ns)) {
       live = false;
-      if (!mbar_wait(&L.full_bar[s], ph, L.status, DRAIN_NS)) return false;
-      mma_commit_pair(&L.empty_bar[s]);
-      continue;
-    }
-    tc_fence_after();
-    const uint32_t st = L.sbase + s * L.stage_bytes;
-    auto descA = [&](int off) { return L.a_mn ? sdesc_mn_sw128(st + off) : sdesc_sw128(st + off); };
-    auto descB = [&](int off) { return L.b_mn ? sdesc_mn_sw128(st + off) : sdesc_sw128(st + off); };
-    const uint64_t a0 = L.a0_off >= 0 ? descA(L.a0_off) : 0;
-    const uint64_t a1 = L.a1_off >= 0 ? descA(L.a1_off) : 0;
-    const uint64_t b0 = L.b0_off >= 0 ? descB(L.b0_off) : 0;
-    const uint64_t b1 = L.b1_off >= 0 ? descB(L.b1_off) : 0;
+      if (!mbar_wait_addr(fb, R.ph, L.status, DRAIN_NS)) return false;
+      mma_commit_pair_addr(eb);
+    } else {
+      tc_fence_after();
+      const uint64_t a0 = R.a0s + R.soff, a1 = R.a1s + R.soff;
+      const uint64_t b0 = R.b0s + R.soff, b1 = R.b1s + R.soff;
 #pragma unroll
-    for (int kk = 0; kk < BK / 16; ++kk) {
-      const uint64_t advA = static_cast<uint64_t>(kk) * stepA;
-      const uint64_t advB = static_cast<uint64_t>(kk) * stepB;
-      const bool first = i == 0;
-      uint32_t q0 = static_cast<uint32_t>(kk) * p0, q1 = static_cast<uint32_t>(kk) * p1;
-      auto mma = [&](uint32_t c, uint64_t ad, uint64_t bd) {
-        uint32_t& q = c ? q1 : q0;
-        const uint32_t blk = c * nsub + (q & (nsub - 1));
-        const uint32_t f = (first && q < nsub) ? 0u : 1u;
-        ++q;
-        mma_bf16_pair(tset + blk * BN, ad, bd, idesc, f);
-      };
-      if (terms & T_C0_A0B0) mma(0, a0 + advA, b0 + advB);
-      if (terms & T_C1_A1B0) mma(1, a1 + advA, b0 + advB);
-      if (terms & T_C0_A1B0) mma(0, a1 + advA, b0 + advB);
-      if (terms & T_C1_A0B1) mma(1, a0 + advA, b1 + advB);
-      if (terms & T_C0_A0B1) mma(0, a0 + advA, b1 + advB);
-      if (terms & T_C0_A1B1) mma(0, a1 + advA, b1 + advB);
+      for (int kk = 0; kk < BK / 16; ++kk) {
+        const uint64_t advA = static_cast<uint64_t>(kk) * stepA;
+        const uint64_t advB = static_cast<uint64_t>(kk) * stepB;
+        const bool first = i == 0;
+        uint32_t q0 = static_cast<uint32_t>(kk) * p0, q1 = static_cast<uint32_t>(kk) * p1;
+        auto mma = [&](uint32_t c, uint64_t ad, uint64_t bd) {
+          uint32_t& q = c ? q1 : q0;
+          const uint32_t blk = c * nsub + (q & (nsub - 1));
+          const uint32_t f = (first && q < nsub) ? 0u : 1u;
+          ++q;
+          mma_bf16_pair(tset + blk * BN, ad, bd, idesc, f);
+        };
+        if (terms & T_C0_A0B0) mma(0, a0 + advA, b0 + advB);
+        if (terms & T_C1_A1B0) mma(1, a1 + advA, b0 + advB);
+        if (terms & T_C0_A1B0) mma(0, a1 + advA, b0 + advB);
+        if (terms & T_C1_A0B1) mma(1, a0 + advA, b1 + advB);
+        if (terms & T_C0_A0B1) mma(0, a0 + advA, b1 + advB);
+        if (terms & T_C0_A1B1) mma(0, a1 + advA, b1 + advB);
+      }
+      mma_commit_pair_addr(eb);
     }
-    mma_commit_pair(&L.empty_bar[s]);
+    if (++R.s == L.stages) {
+      R.s = 0;
+      R.ph ^= 1u;
+      R.soff = 0;
+    } else {
+      R.soff += R.stage_step;
+    }
   }
   return true;
 }
 
 // Product masks the library issues get straight-line MMA sequences (as mma_dispatch).
 template <int BN, int MODE>
-__device__ __forceinline__ bool mma_tile_dispatch(const MmaLoop& L, int g0, uint32_t tset,
+__device__ __forceinline__ bool mma_tile_dispatch(const MmaLoop& L, IssueRing& R, uint32_t tset,
                                                   unsigned terms, int nsub, volatile int* abort,
                                                   bool& live) {
   constexpr int N1 = persist_nsub(1, BN), N2 = persist_nsub(2, BN);
   switch (terms) {
-    case T_C0_A0B0: return mma_tile<BN, T_C0_A0B0, N1>(L, g0, tset, terms, nsub, abort, live);
+    case T_C0_A0B0: return mma_tile<BN, T_C0_A0B0, N1>(L, R, tset, terms, nsub, abort, live);
     case T_C0_A0B0 | T_C1_A1B0 | T_C1_A0B1:
-      return mma_tile<BN, T_C0_A0B0 | T_C1_A1B0 | T_C1_A0B1, N2>(L, g0, tset, terms, nsub, abort, live);
+      return mma_tile<BN, T_C0_A0B0 | T_C1_A1B0 | T_C1_A0B1, N2>(L, R, tset, terms, nsub, abort, live);
     case T_C0_A0B0 | T_C1_A0B1:
-      return mma_tile<BN, T_C0_A0B0 | T_C1_A0B1, N2>(L, g0, tset, terms, nsub, abort, live);
+      return mma_tile<BN, T_C0_A0B0 | T_C1_A0B1, N2>(L, R, tset, terms, nsub, abort, live);
     default: break;
   }
   if constexpr (MODE == EPI_STORE) {
     switch (terms) {
-      case T_C0_A0B1: return mma_tile<BN, T_C0_A0B1, N1>(L, g0, tset, terms, nsub, abort, live);
+      case T_C0_A0B1: return mma_tile<BN, T_C0_A0B1, N1>(L, R, tset, terms, nsub, abort, live);
       case T_C0_A1B0 | T_C0_A0B1:
-        return mma_tile<BN, T_C0_A1B0 | T_C0_A0B1, N1>(L, g0, tset, terms, nsub, abort, live);
+        return mma_tile<BN, T_C0_A1B0 | T_C0_A0B1, N1>(L, R, tset, terms, nsub, abort, live);
       case T_C0_A0B0 | T_C0_A1B1:
-        return mma_tile<BN, T_C0_A0B0 | T_C0_A1B1, N1>(L, g0, tset, terms, nsub, abort, live);
+        return mma_tile<BN, T_C0_A0B0 | T_C0_A1B1, N1>(L, R, tset, terms, nsub, abort, live);
       default: break;
     }
   }
-  return mma_tile<BN, 0, 0>(L, g0, tset, terms, nsub, abort, live);
+  return mma_tile<BN, 0, 0>(L, R, tset, terms, nsub, abort, live);
 }
 
 template <int BN, int MODE, int ACT>
@@ -324,6 +352,17 @@ __global__ void __launch_bounds__(THREADS_P, 1)
       L.full_bar = full_bar; L.empty_bar = empty_bar; L.status = p.status;
       L.wait_ns = p.wait_ns;
       bool live = true;   // false once a wait gave up: the ring is consumed without MMAs
+      IssueRing R;
+      R.a0s = op_desc(L.sbase, L.a0_off, L.a_mn);
+      R.a1s = op_desc(L.sbase, L.a1_off, L.a_mn);
+      R.b0s = op_desc(L.sbase, L.b0_off, L.b_mn);
+      R.b1s = op_desc(L.sbase, L.b1_off, L.b_mn);
+      R.stage_step = static_cast<uint64_t>(L.stage_bytes >> 4);
+      R.soff = 0;
+      R.full0 = smem_u32(full_bar);
+      R.empty0 = smem_u32(empty_bar);
+      R.ph = 0;
+      R.s = 0;
       int j = 0;
       for (int t = pair; t < pp.ntiles; t += npairs, ++j) {
         const int set = pp.nsets == 2 ? (j & 1) : 0;
@@ -333,7 +372,7 @@ __global__ void __launch_bounds__(THREADS_P, 1)
           live = false;
         tc_fence_after();
         const uint32_t tset = tbase + static_cast<uint32_t>(set * pp.set_cols);
-        if (!mma_tile_dispatch<BN, MODE>(L, j * nk, tset, terms, p.nsub, abort, live)) break;
+        if (!mma_tile_dispatch<BN, MODE>(L, R, tset, terms, p.nsub, abort, live)) break;
         if (live) mma_commit_pair(&acc_full[set]);
       }
       mma_commit_even(&drain_bar);
@@ -348,6 +387,10 @@ __global__ void __launch_bounds__(THREADS_P, 1)
     constexpr int CG = BN / EPI_GROUPS_P;
     const int c_begin = ((warp - 2) >> 2) * CG, c_end = c_begin + CG;
     const uint32_t empty0 = dsmem_addr(smem_u32(&acc_empty[0]), 0);   // even CTA's barriers
+    // full chunks go through this warp's row-block buffer behind the pipeline stages
+    uint8_t* const stg = smem + p.stages * p.stage_bytes + (warp - 2) * STG_ROWS_BYTES;
+    const bool rows_ok = rows16_ok(p, MODE, dual) &&
+                         (p.batch <= 1 || (!(p.bsC0 & 3) && !(p.bsC1 & 3)));
     int j = 0;
     for (int t = pair; t < pp.ntiles; t += npairs, ++j) {
       const int set = pp.nsets == 2 ? (j & 1) : 0;
@@ -370,7 +413,10 @@ __global__ void __launch_bounds__(THREADS_P, 1)
 #pragma unroll
           for (int i = 0; i < 16; ++i) v1[i] = 0.f;
         }
-        if (n0 + c < p.N) epilogue16<MODE, ACT>(p, m0 + r, n0 + c, v0, v1, dual);
+        if (rows_ok && n0 + c + 16 <= p.N)
+          epilogue16_rows<MODE, ACT>(p, stg, lane, m0 + q * 32, n0 + c, v0, v1, dual);
+        else if (n0 + c < p.N)
+          epilogue16<MODE, ACT>(p, m0 + r, n0 + c, v0, v1, dual);
       }
       // every lane's TMEM reads of this tile are complete (tcgen05.wait::ld in ld_acc16)
       tc_fence_before();
@@ -452,7 +498,8 @@ cudaError_t launch_cfg2p(const GemmArgs& a, cudaStream_t s, const char** why) {
   p.stage_bytes = off;
   p.tx_bytes = off;
   p.nsub = persist_nsub(nacc, BN);
-  int stages = (220 * 1024) / off;     // no epilogue staging: all of it is pipeline
+  // pipeline stages, then one row-block buffer per epilogue warp
+  int stages = (220 * 1024 - EPI_WARPS_P * STG_ROWS_BYTES) / off;
   if (stages > MAX_STAGES) stages = MAX_STAGES;
   if (stages < 2) { *why = "tile does not fit shared memory"; return cudaErrorInvalidValue; }
   p.stages = stages;
@@ -490,7 +537,7 @@ cudaError_t launch_cfg2p(const GemmArgs& a, cudaStream_t s, const char** why) {
   pp.nsets = persist_sets(nacc, BN);
   pp.set_cols = nacc * p.nsub * BN;
 
-  const int smem = stages * off + 1024;
+  const int smem = stages * off + EPI_WARPS_P * STG_ROWS_BYTES + 1024;
   static PerDeviceOnce attr_once;
   {
     cudaError_t e = attr_once.run([](int&) {
