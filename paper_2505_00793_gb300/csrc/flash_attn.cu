@@ -130,8 +130,10 @@ __global__ void __launch_bounds__(FTHREADS) flash_fwd_kernel(const FlashArgs a) 
   bf16* Kds = Qds + TILE_ELEMS;
   bf16* Vds = Kds + TILE_ELEMS;
   const int nq = a.S / FT;
-  const int qt = nq - 1 - static_cast<int>(blockIdx.x);   // longest rows first
-  const int bh = blockIdx.y;
+  // grid (heads, tiles): blocks dispatch heads fastest, so every head's longest query tile
+  // goes first and the shortest ones fill the tail of the launch
+  const int qt = nq - 1 - static_cast<int>(blockIdx.y);
+  const int bh = blockIdx.x;
   const int64_t hoff = static_cast<int64_t>(bh) * a.S * FDH;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r0 = w * 16;
@@ -311,8 +313,8 @@ __global__ void __launch_bounds__(FTHREADS) flash_bwd_kv_kernel(const FlashArgs 
   float* s_D = st + 2 * FT;
   float* s_Dd = st + 3 * FT;
   const int nt_ = a.S / FT;
-  const int kt = static_cast<int>(blockIdx.x);
-  const int bh = blockIdx.y;
+  const int kt = static_cast<int>(blockIdx.y);     // grid (heads, tiles): longest first
+  const int bh = blockIdx.x;
   const int64_t hoff = static_cast<int64_t>(bh) * a.S * FDH;
   const int64_t soff = static_cast<int64_t>(bh) * a.S;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -460,8 +462,8 @@ __global__ void __launch_bounds__(FTHREADS) flash_bwd_q_kernel(const FlashArgs a
   bf16* Kds = dOds + TILE_ELEMS;
   bf16* Vds = Kds + TILE_ELEMS;
   const int nq = a.S / FT;
-  const int qt = nq - 1 - static_cast<int>(blockIdx.x);
-  const int bh = blockIdx.y;
+  const int qt = nq - 1 - static_cast<int>(blockIdx.y);   // grid (heads, tiles): longest first
+  const int bh = blockIdx.x;
   const int64_t hoff = static_cast<int64_t>(bh) * a.S * FDH;
   const int64_t soff = static_cast<int64_t>(bh) * a.S;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -647,7 +649,7 @@ void flash_fwd(const FlashArgs& a, bool dual, cudaStream_t s) {
     return;
   }
   init_attributes();
-  const dim3 grid(a.S / FT, a.BH);
+  const dim3 grid(a.BH, a.S / FT);
   if (dual)
     launch_k(flash_fwd_kernel<true>, grid, dim3(FTHREADS), SMEM_FWD1, s, a);
   else
@@ -656,7 +658,7 @@ void flash_fwd(const FlashArgs& a, bool dual, cudaStream_t s) {
 
 void flash_bwd(const FlashArgs& a, bool dual, cudaStream_t s) {
   init_attributes();
-  const dim3 grid(a.S / FT, a.BH);
+  const dim3 grid(a.BH, a.S / FT);
   if (dual) {
     launch_k(flash_bwd_kv_kernel<true>, grid, dim3(FTHREADS), SMEM_KV1, s, a);
     launch_k(flash_bwd_q_kernel<true>, grid, dim3(FTHREADS), SMEM_Q1, s, a);

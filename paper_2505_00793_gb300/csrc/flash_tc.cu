@@ -160,8 +160,10 @@ __global__ void __launch_bounds__(FTC_THREADS, FtcCfg<DUAL>::CTAS)
   uint8_t* sKV = smem + C::Q_B;             // stage st: K, V, K', V' (8 KB each)
   uint8_t* sP = sKV + C::STAGES * C::STAGE_B;   // P, then P (*) S' (16 KB each)
   const int nq = p.S / TQ;
-  const int qt = nq - 1 - static_cast<int>(blockIdx.x);   // longest rows first
-  const int bh = static_cast<int>(blockIdx.y);
+  // grid (heads, tiles): heads dispatch fastest, so every head's longest query tile goes
+  // first and the shortest ones fill the tail of the launch
+  const int qt = nq - 1 - static_cast<int>(blockIdx.y);
+  const int bh = static_cast<int>(blockIdx.x);
   const int row0 = bh * p.S;                // the head's first row in the [BH*S][64] maps
   const int nkt = (qt + 1) * (TQ / TK);     // key tiles up to the diagonal
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -457,7 +459,7 @@ cudaError_t launch_ftc_fwd(const FlashArgs& a, cudaStream_t s) {
   p.Om = a.Om;
   p.Omd = a.Omd;
   p.status = a.status;
-  return launch_k(flash_tc_fwd_kernel<DUAL>, dim3(a.S / TQ, a.BH), dim3(FTC_THREADS),
+  return launch_k(flash_tc_fwd_kernel<DUAL>, dim3(a.BH, a.S / TQ), dim3(FTC_THREADS),
                   C::SMEM, s, mQ, mK, mV, mQd, mKd, mVd, p);
 }
 
