@@ -374,6 +374,8 @@ def run_gpu(args):
     mf.set_torch_allocator()        # the workspace shows in torch's memory statistics
     if args.gemm_persistent is not None:
         mf.set_option(native.MF_OPT_GEMM_PERSISTENT, args.gemm_persistent)
+    if args.flash_attn is not None:
+        mf.set_option(native.MF_OPT_FLASH_ATTN, args.flash_attn)
     if args.fused_head:
         mf.set_option(native.MF_OPT_FUSED_HEAD, 1)
     if args.layer_updates:
@@ -510,6 +512,8 @@ def run_gpu(args):
             cpu = cpu_baseline(w)
         traffic = _dram_traffic(args.workload) if default and not (
             args.gemm_persistent is not None or args.fused_head or args.layer_updates) else None
+        flash_desc = {0: "attention materialised per block", 1: "", 2: "warp-level fused attention only",
+                      3: "tcgen05 fused attention forwards", 4: "tcgen05 fused attention backward"}
         out = {
             "metric": "meta-grad steps/s", "value": value, "unit": "meta-steps/s", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
@@ -528,6 +532,8 @@ def run_gpu(args):
                           "in place of SGD" if args.optimizer == "adam" else "")
                        + (f"; persistent CTA-pair GEMM mode {args.gemm_persistent}"
                           if args.gemm_persistent is not None else "")
+                       + (f"; {flash_desc[args.flash_attn]}"
+                          if args.flash_attn not in (None, 1) else "")
                        + ("; output layer, loss and data product fused"
                           if args.fused_head else "")
                        + ("; per-layer updates overlapping the backward pass"
@@ -591,8 +597,11 @@ def main():
     ap.add_argument("--ckpt-every", type=int, default=1,
                     help="segment length of the theta_t store (1 = keep every theta_t)")
     ap.add_argument("--gemm-persistent", type=int, nargs="?", const=1, default=None,
-                    help="MF_OPT_GEMM_PERSISTENT mode (0 off; 1 all, duals 128-wide; 2 "
-                         "single-accumulator only, the library default; 3 all, duals 256-wide)")
+                    help="MF_OPT_GEMM_PERSISTENT mode (0 off; 1 all, duals 128-wide; 2 as 1 "
+                         "but duals with K > 2048 on the one-tile kernel, the library default; "
+                         "3 all, duals 256-wide)")
+    ap.add_argument("--flash-attn", type=int, default=None, choices=[0, 1, 2, 3, 4],
+                    help="MF_OPT_FLASH_ATTN (library default 1)")
     ap.add_argument("--fused-head", action="store_true",
                     help="output layer, loss and data product in one kernel (MF_OPT_FUSED_HEAD)")
     ap.add_argument("--layer-updates", action="store_true",

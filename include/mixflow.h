@@ -300,7 +300,8 @@ mf_status mf_replay_gemms(mf_handle h, int reps, void* stream, double* ms, uint6
  * and seq_len a multiple of 64; others always use the materialised form).  With 1, the
  * dual (tangent-carrying) forward of sequences of whole 128-token tiles runs on tcgen05
  * tensor cores and every other attention kernel on warp-level MMAs; 3 runs the primal
- * forward on tcgen05 as well; 2 uses the warp-level kernels only.  0 materialises them (per
+ * forward on tcgen05 as well; 4 runs the dual forward and both backward kernels (primal
+ * and dual) on tcgen05; 2 uses the warp-level kernels only.  0 materialises them (per
  * block, for the backward).  Setting it drops the handle's captured graphs and changes the
  * workspace size.
  * MF_OPT_GEMM_PERSISTENT (process-wide, default 2): GEMMs that take CTA-pair tiles run as a

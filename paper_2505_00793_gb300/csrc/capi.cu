@@ -2000,7 +2000,7 @@ mf_status mf_set_option(mf_handle h, int option, int value) {
     return MF_OK;
   }
   if (option == MF_OPT_FLASH_ATTN) {
-    if (value < 0 || value > 3) return fail(h, MF_ERR_INVALID_ARG, "MF_OPT_FLASH_ATTN takes 0..3");
+    if (value < 0 || value > 4) return fail(h, MF_ERR_INVALID_ARG, "MF_OPT_FLASH_ATTN takes 0..4");
     h->flash = value;
     drop_graphs(h);
     return MF_OK;

@@ -657,6 +657,11 @@ void flash_fwd(const FlashArgs& a, bool dual, cudaStream_t s) {
 }
 
 void flash_bwd(const FlashArgs& a, bool dual, cudaStream_t s) {
+  // tcgen05 backward (launch errors surface at the caller's check)
+  if (a.tc_bwd && flash_tc_bwd_supported(a, dual)) {
+    flash_tc_bwd(a, dual, s);
+    return;
+  }
   init_attributes();
   const dim3 grid(a.BH, a.S / FT);
   if (dual) {

@@ -41,6 +41,8 @@ constexpr int P_ATOM = TQ * TK * 2;            // 16 KB: P of one key tile, [128
 constexpr int FTC_THREADS = 192;               // producer, MMA, four softmax warps
 constexpr float TAU = 8.f;
 constexpr long long FTC_WAIT_NS = 2000000000LL;
+constexpr int BT_Q = 64;           // backward: queries (key-tile kernel) or keys (query-tile
+                                   // kernel) per streamed tile
 
 template <bool DUAL>
 struct FtcCfg {
@@ -463,6 +465,653 @@ cudaError_t launch_ftc_fwd(const FlashArgs& a, cudaStream_t s) {
                   C::SMEM, s, mQ, mK, mV, mQd, mKd, mVd, p);
 }
 
+// ---- backward on tcgen05 --------------------------------------------------------------
+// Two kernels, as the warp-level backward: one CTA per (head, 128-key tile) for dK, dV and
+// their tangents, one per (head, 128-query tile) for dQ and its tangent, so every sum keeps
+// a fixed order.  The key-tile kernel walks 64-query tiles from the diagonal on:
+//   warp 0      TMA producer: K, V (K', V') once; per query tile Q, dO (Q', dO') and the
+//               row statistics lse, D (rbar, D') into a two-stage ring;
+//   warp 1      one thread issues the MMAs (M 128 keys, N 64, K 64):
+//                 S^T = K Q^T,  S'^T = K' Q^T + K Q'^T,  dP^T = V dO^T,
+//                 dP'^T = V' dO^T + V dO'^T                          (scores, TMEM)
+//                 dV += P^T dO,  dV' += P'^T dO + P^T dO',
+//                 dK += dS^T Q,  dK' += dS'^T Q + dS^T Q'            (Q, dO read MN-major)
+//               and issues the next tile's scores as soon as the elementwise warps have read
+//               this tile's, before this tile's accumulating products, so the tensor pipe
+//               computes them while the elementwise warps work on the next tile;
+//   warps 2..5  thread r owns key row r (TMEM lane r): P^T = exp(S^T - lse) (causal),
+//               dS^T = P^T (*) (dP^T - D), P'^T = P^T (*) (S'^T - rbar),
+//               dS'^T = P'^T (*) (dP^T - D) + P^T (*) (dP'^T - D'), kept as bf16 in
+//               registers, then written to shared memory (the A operands) once the previous
+//               tile's accumulating products have read it.
+// The query-tile kernel is the same with the roles of queries and keys exchanged: Q, dO
+// (Q', dO') stay resident, K, V (K', V') stream per 64-key tile, and dQ += dS K,
+// dQ' += dS' K + dS K' (K read MN-major).
+constexpr int BW_THREADS = 192;
+constexpr int ROWS128_B = 128 * HD * 2;        // 16 KB: [128][64] bf16
+constexpr int ROWS64_B = 64 * HD * 2;          // 8 KB: [64][64] bf16
+constexpr int OPND_B = 128 * 64 * 2;           // 16 KB: [128][64] bf16 A operand
+
+template <bool DUAL>
+struct KvCfg {
+  static constexpr int NRES = DUAL ? 4 : 2;    // K, V (K', V'): 128 rows each
+  static constexpr int NT = DUAL ? 4 : 2;      // Q, dO (Q', dO') per query tile: 64 rows
+  static constexpr int NSTAT = DUAL ? 4 : 2;   // lse, D (rbar, D'): 64 floats each
+  static constexpr int STAGES = 2;
+  static constexpr int STAT_OFF = NT * ROWS64_B;
+  static constexpr int STAGE_B = STAT_OFF + 1024;
+  static constexpr int NOP = DUAL ? 4 : 2;     // P^T, dS^T (P'^T, dS'^T)
+  static constexpr int SMEM = NRES * ROWS128_B + STAGES * STAGE_B + NOP * OPND_B + 1024;
+  static constexpr int CTAS = DUAL ? 1 : 2;
+  static constexpr uint32_t TMEM_COLS = DUAL ? 512 : 256;
+  static constexpr uint32_t C_S = 0, C_SD = 64, C_DP = DUAL ? 128 : 64, C_DPD = 192;
+  static constexpr uint32_t C_DV = DUAL ? 256 : 128, C_DVD = 320, C_DK = DUAL ? 384 : 192,
+                            C_DKD = 448;
+};
+
+template <bool DUAL>
+struct QCfg {
+  static constexpr int NRES = DUAL ? 4 : 2;    // Q, dO (Q', dO'): 128 rows each
+  static constexpr int NT = DUAL ? 4 : 2;      // K, V (K', V') per key tile: 64 rows
+  static constexpr int STAGES = 2;
+  static constexpr int STAGE_B = NT * ROWS64_B;
+  static constexpr int NOP = DUAL ? 2 : 1;     // dS (dS')
+  static constexpr int SMEM = NRES * ROWS128_B + STAGES * STAGE_B + NOP * OPND_B + 1024;
+  static constexpr int CTAS = DUAL ? 1 : 2;
+  static constexpr uint32_t TMEM_COLS = DUAL ? 512 : 256;
+  static constexpr uint32_t C_S = 0, C_SD = 64, C_DP = DUAL ? 128 : 64, C_DPD = 192;
+  static constexpr uint32_t C_DQ = DUAL ? 256 : 128, C_DQD = 320;
+};
+
+struct FtbParams {
+  int BH, S;
+  const float *lse, *rbar, *D, *Dd;
+  float *dQ, *dQd, *dK, *dKd, *dV, *dVd;
+  int* status;
+};
+
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes,
+                                          uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// Four 16-column TMEM loads in flight, then one wait.
+__device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// A 128 x 64 float32 accumulator row (this thread's TMEM lane) to global memory.
+__device__ __forceinline__ void store_acc_row(uint32_t taddr, float* dst) {
+#pragma unroll 1
+  for (int c0 = 0; c0 < HD; c0 += 16) {
+    float v[16];
+    tmem_ld16(taddr + c0, v);
+#pragma unroll
+    for (int i = 0; i < 16; i += 4)
+      *reinterpret_cast<float4*>(dst + c0 + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+  }
+}
+
+template <bool DUAL>
+__global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
+    flash_tc_bwd_kv_kernel(const __grid_constant__ CUtensorMap tmK,
+                           const __grid_constant__ CUtensorMap tmV,
+                           const __grid_constant__ CUtensorMap tmKd,
+                           const __grid_constant__ CUtensorMap tmVd,
+                           const __grid_constant__ CUtensorMap tmQ,
+                           const __grid_constant__ CUtensorMap tmdO,
+                           const __grid_constant__ CUtensorMap tmQd,
+                           const __grid_constant__ CUtensorMap tmdOd, const FtbParams prm) {
+  using C = KvCfg<DUAL>;
+  const FtbParams p = prm;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t res_full, s_full, s_free, p_full, o_done, drain;
+  __shared__ __align__(8) uint64_t st_full[C::STAGES], st_empty[C::STAGES];
+  __shared__ uint32_t tmem_slot;
+  __shared__ int abort_flag;
+
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* sRes = smem;                                  // K, V, K', V'
+  uint8_t* sSt = smem + C::NRES * ROWS128_B;             // stage: Q, dO, Q', dO', statistics
+  uint8_t* sOp = sSt + C::STAGES * C::STAGE_B;           // P^T, dS^T, P'^T, dS'^T
+  // grid (heads, key tiles): heads fastest, and key tile 0 meets the most query tiles
+  const int kt = static_cast<int>(blockIdx.y);
+  const int bh = static_cast<int>(blockIdx.x);
+  const int row0 = bh * p.S;
+  const int key0 = kt * 128;
+  const int j0 = key0 / BT_Q;                            // first query tile on the diagonal
+  const int ntile = p.S / BT_Q - j0;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&res_full, 1);
+    mbar_init(&s_full, 1);
+    mbar_init(&s_free, 4);
+    mbar_init(&p_full, 4);
+    mbar_init(&o_done, 1);
+    mbar_init(&drain, 1);
+    for (int i = 0; i < C::STAGES; ++i) {
+      mbar_init(&st_full[i], 1);
+      mbar_init(&st_empty[i], 1);
+    }
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    prefetch_tmap(&tmK);
+    prefetch_tmap(&tmV);
+    prefetch_tmap(&tmQ);
+    prefetch_tmap(&tmdO);
+    if (DUAL) {
+      prefetch_tmap(&tmKd);
+      prefetch_tmap(&tmVd);
+      prefetch_tmap(&tmQd);
+      prefetch_tmap(&tmdOd);
+    }
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&tmem_slot)),
+                 "r"(C::TMEM_COLS));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tb = tmem_slot;
+  volatile int* abort = &abort_flag;
+  pdl_entry();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---- TMA producer ---------------------------------------------------------------
+      mbar_expect_tx(&res_full, C::NRES * ROWS128_B);
+      tma_load_3d(sRes, &tmK, &res_full, 0, row0 + key0, 0);
+      tma_load_3d(sRes + ROWS128_B, &tmV, &res_full, 0, row0 + key0, 0);
+      if (DUAL) {
+        tma_load_3d(sRes + 2 * ROWS128_B, &tmKd, &res_full, 0, row0 + key0, 0);
+        tma_load_3d(sRes + 3 * ROWS128_B, &tmVd, &res_full, 0, row0 + key0, 0);
+      }
+      int issued = 0;
+      for (int i = 0; i < ntile; ++i, ++issued) {
+        const int st = i % C::STAGES;
+        const uint32_t ph = (i / C::STAGES) & 1;
+        if (!fwait(&st_empty[st], ph ^ 1, p.status, abort)) break;
+        mbar_expect_tx(&st_full[st], C::NT * ROWS64_B + C::NSTAT * BT_Q * 4);
+        uint8_t* b = sSt + st * C::STAGE_B;
+        const int qr = row0 + (j0 + i) * BT_Q;
+        tma_load_3d(b, &tmQ, &st_full[st], 0, qr, 0);
+        tma_load_3d(b + ROWS64_B, &tmdO, &st_full[st], 0, qr, 0);
+        bulk_load(b + C::STAT_OFF, p.lse + qr, BT_Q * 4, &st_full[st]);
+        bulk_load(b + C::STAT_OFF + 256, p.D + qr, BT_Q * 4, &st_full[st]);
+        if (DUAL) {
+          tma_load_3d(b + 2 * ROWS64_B, &tmQd, &st_full[st], 0, qr, 0);
+          tma_load_3d(b + 3 * ROWS64_B, &tmdOd, &st_full[st], 0, qr, 0);
+          bulk_load(b + C::STAT_OFF + 512, p.rbar + qr, BT_Q * 4, &st_full[st]);
+          bulk_load(b + C::STAT_OFF + 768, p.Dd + qr, BT_Q * 4, &st_full[st]);
+        }
+      }
+      // every load issued has landed before the CTA can end
+      mbar_wait(&res_full, 0, p.status, FTC_WAIT_NS);
+      drain_loads(st_full, issued, C::STAGES, p.status);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---- MMA issuer -------------------------------------------------------------------
+      const uint32_t idS = idesc_bf16(128, BT_Q);
+      const uint32_t idA = idesc_bf16(128, HD) | (1u << 16);   // B (Q, dO) read MN-major
+      const uint32_t aK = smem_u32(sRes), aV = aK + ROWS128_B;
+      const uint32_t aKd = aK + 2 * ROWS128_B, aVd = aK + 3 * ROWS128_B;
+      const uint32_t aP = smem_u32(sOp), adS = aP + OPND_B;
+      const uint32_t aPd = aP + 2 * OPND_B, adSd = aP + 3 * OPND_B;
+      // scores of query tile i (waits for its stage)
+      auto scores = [&](int i) -> bool {
+        const int st = i % C::STAGES;
+        if (!fwait(&st_full[st], (i / C::STAGES) & 1, p.status, abort)) return false;
+        tc_fence_after();
+        const uint32_t aQ = smem_u32(sSt + st * C::STAGE_B), adO = aQ + ROWS64_B;
+        const uint32_t aQd = aQ + 2 * ROWS64_B, adOd = aQ + 3 * ROWS64_B;
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk)
+          mma_bf16(tb + C::C_S, sdesc_sw128(aK) + 2 * kk, sdesc_sw128(aQ) + 2 * kk, idS, kk > 0);
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk)
+          mma_bf16(tb + C::C_DP, sdesc_sw128(aV) + 2 * kk, sdesc_sw128(adO) + 2 * kk, idS, kk > 0);
+        if (DUAL) {
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            mma_bf16(tb + C::C_SD, sdesc_sw128(aKd) + 2 * kk, sdesc_sw128(aQ) + 2 * kk, idS, kk > 0);
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            mma_bf16(tb + C::C_SD, sdesc_sw128(aK) + 2 * kk, sdesc_sw128(aQd) + 2 * kk, idS, 1);
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            mma_bf16(tb + C::C_DPD, sdesc_sw128(aVd) + 2 * kk, sdesc_sw128(adO) + 2 * kk, idS, kk > 0);
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            mma_bf16(tb + C::C_DPD, sdesc_sw128(aV) + 2 * kk, sdesc_sw128(adOd) + 2 * kk, idS, 1);
+        }
+        mma_commit(&s_full);
+        return true;
+      };
+      bool ok = fwait(&res_full, 0, p.status, abort) && scores(0);
+      for (int i = 0; ok && i < ntile; ++i) {
+        // the elementwise warps have read the scores of tile i: the next tile's may overwrite
+        if (!fwait(&s_free, i & 1, p.status, abort)) break;
+        if (i + 1 < ntile && !scores(i + 1)) break;
+        if (!fwait(&p_full, i & 1, p.status, abort)) break;
+        tc_fence_after();
+        const int st = i % C::STAGES;
+        const uint32_t aQ = smem_u32(sSt + st * C::STAGE_B), adO = aQ + ROWS64_B;
+        const uint32_t aQd = aQ + 2 * ROWS64_B, adOd = aQ + 3 * ROWS64_B;
+#pragma unroll
+        for (int kk = 0; kk < BT_Q / 16; ++kk) {
+          const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
+          const uint64_t bO = sdesc_mn_sw128(adO) + 128 * kk, bQ = sdesc_mn_sw128(aQ) + 128 * kk;
+          mma_bf16(tb + C::C_DV, sdesc_sw128(aP) + 2 * kk, bO, idA, acc);
+          mma_bf16(tb + C::C_DK, sdesc_sw128(adS) + 2 * kk, bQ, idA, acc);
+          if (DUAL) {
+            const uint64_t bOd = sdesc_mn_sw128(adOd) + 128 * kk;
+            const uint64_t bQd = sdesc_mn_sw128(aQd) + 128 * kk;
+            mma_bf16(tb + C::C_DVD, sdesc_sw128(aPd) + 2 * kk, bO, idA, acc);
+            mma_bf16(tb + C::C_DVD, sdesc_sw128(aP) + 2 * kk, bOd, idA, 1);
+            mma_bf16(tb + C::C_DKD, sdesc_sw128(adSd) + 2 * kk, bQ, idA, acc);
+            mma_bf16(tb + C::C_DKD, sdesc_sw128(adS) + 2 * kk, bQd, idA, 1);
+          }
+        }
+        mma_commit(&st_empty[st]);
+        mma_commit(&o_done);
+      }
+      // every MMA issued here has completed before TMEM is released
+      mma_commit(&drain);
+      mbar_wait(&drain, 0, p.status, FTC_WAIT_NS);
+    }
+    __syncwarp();
+  } else {
+    // ---- elementwise: thread r owns key row r of the tile (TMEM lane r) -----------------
+    const int q4 = warp & 3;
+    const int r = q4 * 32 + lane;
+    const uint32_t lo = static_cast<uint32_t>(q4 * 32) << 16;
+    const int key = key0 + r;
+    bool ok = true;
+    for (int i = 0; i < ntile; ++i) {
+      if (!wwait(&s_full, i & 1, p.status, abort)) { ok = false; break; }
+      tc_fence_after();
+      const float* stat = reinterpret_cast<const float*>(sSt + (i % C::STAGES) * C::STAGE_B + C::STAT_OFF);
+      const int qbase = (j0 + i) * BT_Q;
+      uint32_t pk[BT_Q / 2], dsk[BT_Q / 2], pdk[DUAL ? BT_Q / 2 : 1], dsdk[DUAL ? BT_Q / 2 : 1];
+#pragma unroll
+      for (int c0 = 0; c0 < BT_Q; c0 += 16) {
+        float sv[16], dp[16], sd[16], dpd[16];
+        tmem_ld16_nowait(tb + lo + C::C_S + c0, sv);
+        tmem_ld16_nowait(tb + lo + C::C_DP + c0, dp);
+        if (DUAL) {
+          tmem_ld16_nowait(tb + lo + C::C_SD + c0, sd);
+          tmem_ld16_nowait(tb + lo + C::C_DPD + c0, dpd);
+        }
+        tmem_wait_ld();
+#pragma unroll
+        for (int e = 0; e < 16; e += 2) {
+          float pv[2], dsv[2], pdv[2], dsdv[2];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int c = c0 + e + h;
+            const float pp = qbase + c >= key ? __expf(sv[e + h] - stat[c]) : 0.f;
+            const float dpm = dp[e + h] - stat[64 + c];
+            pv[h] = pp;
+            dsv[h] = pp * dpm;
+            if (DUAL) {
+              const float pd = pp * (sd[e + h] - stat[128 + c]);
+              pdv[h] = pd;
+              dsdv[h] = pd * dpm + pp * (dpd[e + h] - stat[192 + c]);
+            }
+          }
+          pk[(c0 + e) / 2] = pack_bf16x2(pv[0], pv[1]);
+          dsk[(c0 + e) / 2] = pack_bf16x2(dsv[0], dsv[1]);
+          if (DUAL) {
+            pdk[(c0 + e) / 2] = pack_bf16x2(pdv[0], pdv[1]);
+            dsdk[(c0 + e) / 2] = pack_bf16x2(dsdv[0], dsdv[1]);
+          }
+        }
+      }
+      // this tile's scores are read: the next tile's may be computed
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_local(&s_free);
+      // the previous tile's accumulating products have read the A operands
+      if (i > 0 && !wwait(&o_done, (i - 1) & 1, p.status, abort)) { ok = false; break; }
+#pragma unroll
+      for (int ch = 0; ch < BT_Q / 8; ++ch) {
+        *reinterpret_cast<uint4*>(sOp + swz(r, ch)) =
+            make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]);
+        *reinterpret_cast<uint4*>(sOp + OPND_B + swz(r, ch)) =
+            make_uint4(dsk[4 * ch], dsk[4 * ch + 1], dsk[4 * ch + 2], dsk[4 * ch + 3]);
+        if (DUAL) {
+          *reinterpret_cast<uint4*>(sOp + 2 * OPND_B + swz(r, ch)) =
+              make_uint4(pdk[4 * ch], pdk[4 * ch + 1], pdk[4 * ch + 2], pdk[4 * ch + 3]);
+          *reinterpret_cast<uint4*>(sOp + 3 * OPND_B + swz(r, ch)) =
+              make_uint4(dsdk[4 * ch], dsdk[4 * ch + 1], dsdk[4 * ch + 2], dsdk[4 * ch + 3]);
+        }
+      }
+      fence_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_local(&p_full);
+    }
+    // ---- outputs: dV, dK (dV', dK') rows of this key ------------------------------------
+    if (ok && wwait(&o_done, (ntile - 1) & 1, p.status, abort)) {
+      tc_fence_after();
+      const int64_t off = (static_cast<int64_t>(row0) + key) * HD;
+      store_acc_row(tb + lo + C::C_DV, p.dV + off);
+      store_acc_row(tb + lo + C::C_DK, p.dK + off);
+      if (DUAL) {
+        store_acc_row(tb + lo + C::C_DVD, p.dVd + off);
+        store_acc_row(tb + lo + C::C_DKD, p.dKd + off);
+      }
+    }
+    tc_fence_before();
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tb),
+                 "r"(C::TMEM_COLS));
+  }
+}
+
+template <bool DUAL>
+__global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
+    flash_tc_bwd_q_kernel(const __grid_constant__ CUtensorMap tmQ,
+                          const __grid_constant__ CUtensorMap tmdO,
+                          const __grid_constant__ CUtensorMap tmQd,
+                          const __grid_constant__ CUtensorMap tmdOd,
+                          const __grid_constant__ CUtensorMap tmK,
+                          const __grid_constant__ CUtensorMap tmV,
+                          const __grid_constant__ CUtensorMap tmKd,
+                          const __grid_constant__ CUtensorMap tmVd, const FtbParams prm) {
+  using C = QCfg<DUAL>;
+  const FtbParams p = prm;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t res_full, s_full, s_free, p_full, o_done, drain;
+  __shared__ __align__(8) uint64_t st_full[C::STAGES], st_empty[C::STAGES];
+  __shared__ uint32_t tmem_slot;
+  __shared__ int abort_flag;
+
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* sRes = smem;                                  // Q, dO, Q', dO'
+  uint8_t* sSt = smem + C::NRES * ROWS128_B;             // stage: K, V, K', V'
+  uint8_t* sOp = sSt + C::STAGES * C::STAGE_B;           // dS, dS'
+  // grid (heads, query tiles): heads fastest, the last query tile (most key tiles) first
+  const int nq = p.S / 128;
+  const int qt = nq - 1 - static_cast<int>(blockIdx.y);
+  const int bh = static_cast<int>(blockIdx.x);
+  const int row0 = bh * p.S;
+  const int q0 = qt * 128;
+  const int ntile = (q0 + 128) / BT_Q;                   // key tiles up to the diagonal
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&res_full, 1);
+    mbar_init(&s_full, 1);
+    mbar_init(&s_free, 4);
+    mbar_init(&p_full, 4);
+    mbar_init(&o_done, 1);
+    mbar_init(&drain, 1);
+    for (int i = 0; i < C::STAGES; ++i) {
+      mbar_init(&st_full[i], 1);
+      mbar_init(&st_empty[i], 1);
+    }
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    prefetch_tmap(&tmQ);
+    prefetch_tmap(&tmdO);
+    prefetch_tmap(&tmK);
+    prefetch_tmap(&tmV);
+    if (DUAL) {
+      prefetch_tmap(&tmQd);
+      prefetch_tmap(&tmdOd);
+      prefetch_tmap(&tmKd);
+      prefetch_tmap(&tmVd);
+    }
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(&tmem_slot)),
+                 "r"(C::TMEM_COLS));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tb = tmem_slot;
+  volatile int* abort = &abort_flag;
+  pdl_entry();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---- TMA producer ---------------------------------------------------------------
+      mbar_expect_tx(&res_full, C::NRES * ROWS128_B);
+      tma_load_3d(sRes, &tmQ, &res_full, 0, row0 + q0, 0);
+      tma_load_3d(sRes + ROWS128_B, &tmdO, &res_full, 0, row0 + q0, 0);
+      if (DUAL) {
+        tma_load_3d(sRes + 2 * ROWS128_B, &tmQd, &res_full, 0, row0 + q0, 0);
+        tma_load_3d(sRes + 3 * ROWS128_B, &tmdOd, &res_full, 0, row0 + q0, 0);
+      }
+      int issued = 0;
+      for (int i = 0; i < ntile; ++i, ++issued) {
+        const int st = i % C::STAGES;
+        const uint32_t ph = (i / C::STAGES) & 1;
+        if (!fwait(&st_empty[st], ph ^ 1, p.status, abort)) break;
+        mbar_expect_tx(&st_full[st], C::STAGE_B);
+        uint8_t* b = sSt + st * C::STAGE_B;
+        const int kr = row0 + i * BT_Q;
+        tma_load_3d(b, &tmK, &st_full[st], 0, kr, 0);
+        tma_load_3d(b + ROWS64_B, &tmV, &st_full[st], 0, kr, 0);
+        if (DUAL) {
+          tma_load_3d(b + 2 * ROWS64_B, &tmKd, &st_full[st], 0, kr, 0);
+          tma_load_3d(b + 3 * ROWS64_B, &tmVd, &st_full[st], 0, kr, 0);
+        }
+      }
+      mbar_wait(&res_full, 0, p.status, FTC_WAIT_NS);
+      drain_loads(st_full, issued, C::STAGES, p.status);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---- MMA issuer -------------------------------------------------------------------
+      const uint32_t idS = idesc_bf16(128, BT_Q);
+      const uint32_t idA = idesc_bf16(128, HD) | (1u << 16);   // B (K) read MN-major
+      const uint32_t aQ = smem_u32(sRes), adO = aQ + ROWS128_B;
+      const uint32_t aQd = aQ + 2 * ROWS128_B, adOd = aQ + 3 * ROWS128_B;
+      const uint32_t adS = smem_u32(sOp), adSd = adS + OPND_B;
+      auto scores = [&](int i) -> bool {
+        const int st = i % C::STAGES;
+        if (!fwait(&st_full[st], (i / C::STAGES) & 1, p.status, abort)) return false;
+        tc_fence_after();
+        const uint32_t aK = smem_u32(sSt + st * C::STAGE_B), aV = aK + ROWS64_B;
+        const uint32_t aKd = aK + 2 * ROWS64_B, aVd = aK + 3 * ROWS64_B;
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk)
+          mma_bf16(tb + C::C_S, sdesc_sw128(aQ) + 2 * kk, sdesc_sw128(aK) + 2 * kk, idS, kk > 0);
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk)
+          mma_bf16(tb + C::C_DP, sdesc_sw128(adO) + 2 * kk, sdesc_sw128(aV) + 2 * kk, idS, kk > 0);
+        if (DUAL) {
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            mma_bf16(tb + C::C_SD, sdesc_sw128(aQd) + 2 * kk, sdesc_sw128(aK) + 2 * kk, idS, kk > 0);
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            mma_bf16(tb + C::C_SD, sdesc_sw128(aQ) + 2 * kk, sdesc_sw128(aKd) + 2 * kk, idS, 1);
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            mma_bf16(tb + C::C_DPD, sdesc_sw128(adOd) + 2 * kk, sdesc_sw128(aV) + 2 * kk, idS, kk > 0);
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            mma_bf16(tb + C::C_DPD, sdesc_sw128(adO) + 2 * kk, sdesc_sw128(aVd) + 2 * kk, idS, 1);
+        }
+        mma_commit(&s_full);
+        return true;
+      };
+      bool ok = fwait(&res_full, 0, p.status, abort) && scores(0);
+      for (int i = 0; ok && i < ntile; ++i) {
+        if (!fwait(&s_free, i & 1, p.status, abort)) break;
+        if (i + 1 < ntile && !scores(i + 1)) break;
+        if (!fwait(&p_full, i & 1, p.status, abort)) break;
+        tc_fence_after();
+        const int st = i % C::STAGES;
+        const uint32_t aK = smem_u32(sSt + st * C::STAGE_B), aKd = aK + 2 * ROWS64_B;
+#pragma unroll
+        for (int kk = 0; kk < BT_Q / 16; ++kk) {
+          const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
+          const uint64_t bK = sdesc_mn_sw128(aK) + 128 * kk;
+          mma_bf16(tb + C::C_DQ, sdesc_sw128(adS) + 2 * kk, bK, idA, acc);
+          if (DUAL) {
+            mma_bf16(tb + C::C_DQD, sdesc_sw128(adSd) + 2 * kk, bK, idA, acc);
+            mma_bf16(tb + C::C_DQD, sdesc_sw128(adS) + 2 * kk, sdesc_mn_sw128(aKd) + 128 * kk, idA, 1);
+          }
+        }
+        mma_commit(&st_empty[st]);
+        mma_commit(&o_done);
+      }
+      mma_commit(&drain);
+      mbar_wait(&drain, 0, p.status, FTC_WAIT_NS);
+    }
+    __syncwarp();
+  } else {
+    // ---- elementwise: thread r owns query row r of the tile (TMEM lane r) ---------------
+    const int q4 = warp & 3;
+    const int r = q4 * 32 + lane;
+    const uint32_t lo = static_cast<uint32_t>(q4 * 32) << 16;
+    const int q = q0 + r;
+    const int64_t gi = static_cast<int64_t>(row0) + q;
+    const float lse = p.lse[gi], Dv = p.D[gi];
+    const float rb = DUAL ? p.rbar[gi] : 0.f, Ddv = DUAL ? p.Dd[gi] : 0.f;
+    bool ok = true;
+    for (int i = 0; i < ntile; ++i) {
+      if (!wwait(&s_full, i & 1, p.status, abort)) { ok = false; break; }
+      tc_fence_after();
+      const int kbase = i * BT_Q;
+      uint32_t dsk[BT_Q / 2], dsdk[DUAL ? BT_Q / 2 : 1];
+#pragma unroll
+      for (int c0 = 0; c0 < BT_Q; c0 += 16) {
+        float sv[16], dp[16], sd[16], dpd[16];
+        tmem_ld16_nowait(tb + lo + C::C_S + c0, sv);
+        tmem_ld16_nowait(tb + lo + C::C_DP + c0, dp);
+        if (DUAL) {
+          tmem_ld16_nowait(tb + lo + C::C_SD + c0, sd);
+          tmem_ld16_nowait(tb + lo + C::C_DPD + c0, dpd);
+        }
+        tmem_wait_ld();
+#pragma unroll
+        for (int e = 0; e < 16; e += 2) {
+          float dsv[2], dsdv[2];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int key = kbase + c0 + e + h;
+            const float pp = key <= q ? __expf(sv[e + h] - lse) : 0.f;
+            const float dpm = dp[e + h] - Dv;
+            dsv[h] = pp * dpm;
+            if (DUAL) {
+              const float pd = pp * (sd[e + h] - rb);
+              dsdv[h] = pd * dpm + pp * (dpd[e + h] - Ddv);
+            }
+          }
+          dsk[(c0 + e) / 2] = pack_bf16x2(dsv[0], dsv[1]);
+          if (DUAL) dsdk[(c0 + e) / 2] = pack_bf16x2(dsdv[0], dsdv[1]);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_local(&s_free);
+      if (i > 0 && !wwait(&o_done, (i - 1) & 1, p.status, abort)) { ok = false; break; }
+#pragma unroll
+      for (int ch = 0; ch < BT_Q / 8; ++ch) {
+        *reinterpret_cast<uint4*>(sOp + swz(r, ch)) =
+            make_uint4(dsk[4 * ch], dsk[4 * ch + 1], dsk[4 * ch + 2], dsk[4 * ch + 3]);
+        if (DUAL)
+          *reinterpret_cast<uint4*>(sOp + OPND_B + swz(r, ch)) =
+              make_uint4(dsdk[4 * ch], dsdk[4 * ch + 1], dsdk[4 * ch + 2], dsdk[4 * ch + 3]);
+      }
+      fence_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_local(&p_full);
+    }
+    if (ok && wwait(&o_done, (ntile - 1) & 1, p.status, abort)) {
+      tc_fence_after();
+      const int64_t off = gi * HD;
+      store_acc_row(tb + lo + C::C_DQ, p.dQ + off);
+      if (DUAL) store_acc_row(tb + lo + C::C_DQD, p.dQd + off);
+    }
+    tc_fence_before();
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tb),
+                 "r"(C::TMEM_COLS));
+  }
+}
+
+template <bool DUAL>
+cudaError_t launch_ftc_bwd(const FlashArgs& a, cudaStream_t s) {
+  using KC = KvCfg<DUAL>;
+  using QC = QCfg<DUAL>;
+  const int rows = a.BH * a.S;
+  CUtensorMap k128[4], q64[4], q128[4], k64[4];
+  const void* kv[4] = {a.K, a.V, a.Kd, a.Vd};
+  const void* qo[4] = {a.Q, a.dO, a.Qd, a.dOd};
+  for (int i = 0; i < 4; ++i) {
+    memset(&k128[i], 0, sizeof(CUtensorMap)); memset(&q64[i], 0, sizeof(CUtensorMap));
+    memset(&q128[i], 0, sizeof(CUtensorMap)); memset(&k64[i], 0, sizeof(CUtensorMap));
+    if (i >= 2 && !DUAL) continue;
+    if (!make_map(&k128[i], kv[i], HD, rows, HD, 128) || !make_map(&k64[i], kv[i], HD, rows, HD, BT_Q) ||
+        !make_map(&q128[i], qo[i], HD, rows, HD, 128) || !make_map(&q64[i], qo[i], HD, rows, HD, BT_Q))
+      return cudaErrorInvalidValue;
+  }
+  static PerDeviceOnce attr_once;
+  cudaError_t e = attr_once.run([](int&) {
+    cudaError_t r = cudaFuncSetAttribute(flash_tc_bwd_kv_kernel<DUAL>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, KC::SMEM);
+    if (r != cudaSuccess) return r;
+    return cudaFuncSetAttribute(flash_tc_bwd_q_kernel<DUAL>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, QC::SMEM);
+  });
+  if (e != cudaSuccess) return e;
+  FtbParams p;
+  p.BH = a.BH;
+  p.S = a.S;
+  p.lse = a.lse;
+  p.rbar = a.rbar;
+  p.D = a.D;
+  p.Dd = a.Dd;
+  p.dQ = a.dQ; p.dQd = a.dQd;
+  p.dK = a.dK; p.dKd = a.dKd;
+  p.dV = a.dV; p.dVd = a.dVd;
+  p.status = a.status;
+  const dim3 grid(a.BH, a.S / 128);
+  e = launch_k(flash_tc_bwd_kv_kernel<DUAL>, grid, dim3(BW_THREADS), KC::SMEM, s, k128[0],
+               k128[1], k128[2], k128[3], q64[0], q64[1], q64[2], q64[3], p);
+  if (e != cudaSuccess) return e;
+  return launch_k(flash_tc_bwd_q_kernel<DUAL>, grid, dim3(BW_THREADS), QC::SMEM, s, q128[0],
+                  q128[1], q128[2], q128[3], k64[0], k64[1], k64[2], k64[3], p);
+}
+
 }  // namespace
 }  // namespace mf
 
@@ -473,6 +1122,20 @@ bool flash_tc_supported(int S, int dh) { return dh == HD && S > 0 && S % TQ == 0
 cudaError_t flash_tc_fwd(const FlashArgs& a, bool dual, cudaStream_t s) {
   if (!flash_tc_supported(a.S, HD) || a.BH < 1) return cudaErrorInvalidValue;
   return dual ? launch_ftc_fwd<true>(a, s) : launch_ftc_fwd<false>(a, s);
+}
+
+bool flash_tc_bwd_supported(const FlashArgs& a, bool dual) {
+  if (!flash_tc_supported(a.S, HD) || a.BH < 1) return false;
+  // the row statistics stream into shared memory by bulk copies of 64 floats
+  const void* stats[4] = {a.lse, a.D, a.rbar, a.Dd};
+  for (int i = 0; i < (dual ? 4 : 2); ++i)
+    if (!stats[i] || (reinterpret_cast<uintptr_t>(stats[i]) & 15)) return false;
+  return true;
+}
+
+cudaError_t flash_tc_bwd(const FlashArgs& a, bool dual, cudaStream_t s) {
+  if (!flash_tc_bwd_supported(a, dual)) return cudaErrorInvalidValue;
+  return dual ? launch_ftc_bwd<true>(a, s) : launch_ftc_bwd<false>(a, s);
 }
 
 }  // namespace mf

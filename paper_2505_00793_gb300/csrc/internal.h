@@ -269,12 +269,17 @@ struct FlashArgs {
   __nv_bfloat16 *Om = nullptr, *Omd = nullptr;
   int tc = 1;              // tcgen05 forward where S is a multiple of 128: 0 never,
                            // 1 the dual kernel, 2 the dual and the primal kernels
+  int tc_bwd = 0;          // 1: tcgen05 backward (primal and dual) where supported
   int* status = nullptr;   // device status word (bounded waits of the tcgen05 kernels)
 };
 bool flash_supported(int S, int dh);
 // tcgen05 forward (flash_tc.cu): S a multiple of 128, 64-wide heads.
 bool flash_tc_supported(int S, int dh);
 cudaError_t flash_tc_fwd(const FlashArgs& a, bool dual, cudaStream_t s);
+// tcgen05 backward (both kernels): S a multiple of 128, 64-wide heads, 16-byte aligned row
+// statistics.
+bool flash_tc_bwd_supported(const FlashArgs& a, bool dual);
+cudaError_t flash_tc_bwd(const FlashArgs& a, bool dual, cudaStream_t s);
 void flash_fwd(const FlashArgs& a, bool dual, cudaStream_t s);
 void flash_bwd(const FlashArgs& a, bool dual, cudaStream_t s);
 // D = rowsum(dO (*) O), D' = rowsum(dO' (*) O + dO (*) O') per (token, head) from float32

@@ -16,7 +16,8 @@ still move far more than the 129 MB L2 per launch:
 * decoder_large_T2  the bench workload (12 x d1024, 16 heads, S = 1024, B = 8, heavy ball,
                 weights + scalar log-lr) at T = 2: every kernel of a step at full size
 
-``--gemm-persistent``, ``--fused-head`` and ``--layer-updates`` set the opt-in paths, so that
+``--gemm-persistent``, ``--fused-head``, ``--layer-updates`` and ``--flash-attn`` set the
+opt-in paths, so that
 their kernels can be captured on the same cases.
 """
 from __future__ import annotations
@@ -60,6 +61,8 @@ def main() -> None:
                     help="MF_OPT_GEMM_PERSISTENT mode (library default when absent)")
     ap.add_argument("--fused-head", action="store_true")
     ap.add_argument("--layer-updates", action="store_true")
+    ap.add_argument("--flash-attn", type=int, default=None, choices=[0, 1, 2, 3, 4],
+                    help="MF_OPT_FLASH_ATTN (library default when absent)")
     args = ap.parse_args()
     torch.cuda.set_device(0)
     w = case(args.case)
@@ -71,6 +74,8 @@ def main() -> None:
         mf.set_option(native.MF_OPT_GEMM_PERSISTENT, args.gemm_persistent)
     mf.set_option(native.MF_OPT_FUSED_HEAD, 1 if args.fused_head else 0)
     mf.set_option(native.MF_OPT_LAYER_UPDATES, 1 if args.layer_updates else 0)
+    if args.flash_attn is not None:
+        mf.set_option(native.MF_OPT_FLASH_ATTN, args.flash_attn)
     loop = native.loop_desc_for(w, args.hvp_mode)
     d_eta = torch.empty(w.n_eta, device="cuda")
     d_th = torch.empty(w.n_params, device="cuda")

@@ -2,8 +2,10 @@
 the float64 oracle and against the warp-level fused kernels of the same library.
 
 MF_OPT_FLASH_ATTN 3 runs both forward kernels (S, S' into TMEM, P and P (*) S' through
-shared memory into the O and tangent products) on tcgen05, 1 (the default) the dual one; 2
-keeps the warp-level kernels.  Cases span one to
+shared memory into the O and tangent products) on tcgen05, 1 (the default) the dual one; 4
+the dual forward and both backward kernels (scores and their tangents into TMEM, P^T, dS^T
+and tangents through shared memory into the dK, dV, dQ products); 2 keeps the warp-level
+kernels.  Cases span one to
 three 128-query tiles per head (the causal diagonal and off-diagonal key tiles), one to four
 heads, momentum with the scalar log-lr, both HVP modes, and attention scores spread far
 beyond the running-maximum bound (weights of scale 0.3), so that rows rescale their
@@ -67,13 +69,18 @@ def test_flash_tc_meta_grad(name, mode):
     de_t, dt_t, V_t = _run(w, inp, 3, mode)
     de_d, dt_d, V_d = _run(w, inp, 1, mode)
     de_w, dt_w, V_w = _run(w, inp, 2, mode)
-    for de, dt, V in ((de_t, dt_t, V_t), (de_d, dt_d, V_d), (de_w, dt_w, V_w)):
+    de_b, dt_b, V_b = _run(w, inp, 4, mode)
+    for de, dt, V in ((de_t, dt_t, V_t), (de_d, dt_d, V_d), (de_w, dt_w, V_w), (de_b, dt_b, V_b)):
         assert np.isfinite(de).all() and np.isfinite(dt).all()
         assert rel_l2(de, ref["d_eta"]) < 2e-2, (name, rel_l2(de, ref["d_eta"]))
         assert rel_l2(dt, ref["d_theta0"]) < 2e-2, (name, rel_l2(dt, ref["d_theta0"]))
         assert abs(V - ref["V"]) <= 2e-2 * abs(ref["V"])
     # the two kernels differ only in summation order and bf16 rounding points
     assert rel_l2(dt_t, dt_w) < 1e-2, (name, rel_l2(dt_t, dt_w))
+    # 4 and 1 share the forward; their backward kernels differ in summation order only
+    assert V_b == V_d
+    assert rel_l2(dt_b, dt_d) < 2e-3, (name, rel_l2(dt_b, dt_d))
+    assert rel_l2(de_b, de_d) < 2e-3, (name, rel_l2(de_b, de_d))
 
 
 @pytest.mark.gpu
@@ -82,6 +89,10 @@ def test_flash_tc_rescaling_rows(mode):
     inp = synth.make_inputs(SHARP)
     de_t, dt_t, V_t = _run(SHARP, inp, 3, mode)
     de_w, dt_w, V_w = _run(SHARP, inp, 2, mode)
+    de_b, dt_b, V_b = _run(SHARP, inp, 4, mode)
+    assert np.isfinite(de_b).all() and np.isfinite(dt_b).all()
+    assert rel_l2(dt_b, dt_w) < 1e-2, rel_l2(dt_b, dt_w)
+    assert rel_l2(de_b, de_w) < 1e-2, rel_l2(de_b, de_w)
     assert np.isfinite(de_t).all() and np.isfinite(dt_t).all()
     assert rel_l2(dt_t, dt_w) < 1e-2, rel_l2(dt_t, dt_w)
     assert rel_l2(de_t, de_w) < 1e-2, rel_l2(de_t, de_w)
