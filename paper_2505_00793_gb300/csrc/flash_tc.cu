@@ -479,7 +479,8 @@ cudaError_t launch_ftc_fwd(const FlashArgs& a, cudaStream_t s) {
 //               and issues the next tile's scores as soon as the elementwise warps have read
 //               this tile's, before this tile's accumulating products, so the tensor pipe
 //               computes them while the elementwise warps work on the next tile;
-//   warps 2..5  thread r owns key row r (TMEM lane r): P^T = exp(S^T - lse) (causal),
+//   warps 2..9  two threads per key row r (TMEM lane r), each on 32 of the 64 query
+//               columns: P^T = exp(S^T - lse) (causal),
 //               dS^T = P^T (*) (dP^T - D), P'^T = P^T (*) (S'^T - rbar),
 //               dS'^T = P'^T (*) (dP^T - D) + P^T (*) (dP'^T - D'), kept as bf16 in
 //               registers, then written to shared memory (the A operands) once the previous
@@ -487,7 +488,9 @@ cudaError_t launch_ftc_fwd(const FlashArgs& a, cudaStream_t s) {
 // The query-tile kernel is the same with the roles of queries and keys exchanged: Q, dO
 // (Q', dO') stay resident, K, V (K', V') stream per 64-key tile, and dQ += dS K,
 // dQ' += dS' K + dS K' (K read MN-major).
-constexpr int BW_THREADS = 192;
+constexpr int BW_EW = 8;                       // elementwise warps: two per TMEM lane quadrant,
+                                               // each on half of the tile's 64 columns
+constexpr int BW_THREADS = 64 + 32 * BW_EW;
 constexpr int ROWS128_B = 128 * HD * 2;        // 16 KB: [128][64] bf16
 constexpr int ROWS64_B = 64 * HD * 2;          // 8 KB: [64][64] bf16
 constexpr int OPND_B = 128 * 64 * 2;           // 16 KB: [128][64] bf16 A operand
@@ -495,7 +498,8 @@ constexpr int OPND_B = 128 * 64 * 2;           // 16 KB: [128][64] bf16 A operan
 template <bool DUAL>
 struct KvCfg {
   static constexpr int NRES = DUAL ? 4 : 2;    // K, V (K', V'): 128 rows each
-  static constexpr int NT = DUAL ? 4 : 2;      // Q, dO (Q', dO') per query tile: 64 rows
+  static constexpr int NT = DUAL ? 4 : 2;      // Q, (Q',) dO (, dO') per query tile: 64 rows
+  static constexpr int OFF_DO = DUAL ? 2 * ROWS64_B : ROWS64_B;   // Q' right after Q, dO' after dO
   static constexpr int NSTAT = DUAL ? 4 : 2;   // lse, D (rbar, D'): 64 floats each
   static constexpr int STAGES = 2;
   static constexpr int STAT_OFF = NT * ROWS64_B;
@@ -512,7 +516,8 @@ struct KvCfg {
 template <bool DUAL>
 struct QCfg {
   static constexpr int NRES = DUAL ? 4 : 2;    // Q, dO (Q', dO'): 128 rows each
-  static constexpr int NT = DUAL ? 4 : 2;      // K, V (K', V') per key tile: 64 rows
+  static constexpr int NT = DUAL ? 4 : 2;      // K, (K',) V (, V') per key tile: 64 rows
+  static constexpr int OFF_V = DUAL ? 2 * ROWS64_B : ROWS64_B;    // K' right after K, V' after V
   static constexpr int STAGES = 2;
   static constexpr int STAGE_B = NT * ROWS64_B;
   static constexpr int NOP = DUAL ? 2 : 1;     // dS (dS')
@@ -553,10 +558,11 @@ __device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, float (&v)[16])
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// A 128 x 64 float32 accumulator row (this thread's TMEM lane) to global memory.
-__device__ __forceinline__ void store_acc_row(uint32_t taddr, float* dst) {
+// Columns cb .. cb + 31 of a 128 x 64 float32 accumulator row (this thread's TMEM lane) to
+// global memory.
+__device__ __forceinline__ void store_acc_row(uint32_t taddr, float* dst, int cb) {
 #pragma unroll 1
-  for (int c0 = 0; c0 < HD; c0 += 16) {
+  for (int c0 = cb; c0 < cb + 32; c0 += 16) {
     float v[16];
     tmem_ld16(taddr + c0, v);
 #pragma unroll
@@ -600,8 +606,8 @@ __global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
   if (threadIdx.x == 0) {
     mbar_init(&res_full, 1);
     mbar_init(&s_full, 1);
-    mbar_init(&s_free, 4);
-    mbar_init(&p_full, 4);
+    mbar_init(&s_free, BW_EW);
+    mbar_init(&p_full, BW_EW);
     mbar_init(&o_done, 1);
     mbar_init(&drain, 1);
     for (int i = 0; i < C::STAGES; ++i) {
@@ -653,11 +659,11 @@ __global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
         uint8_t* b = sSt + st * C::STAGE_B;
         const int qr = row0 + (j0 + i) * BT_Q;
         tma_load_3d(b, &tmQ, &st_full[st], 0, qr, 0);
-        tma_load_3d(b + ROWS64_B, &tmdO, &st_full[st], 0, qr, 0);
+        tma_load_3d(b + C::OFF_DO, &tmdO, &st_full[st], 0, qr, 0);
         bulk_load(b + C::STAT_OFF, p.lse + qr, BT_Q * 4, &st_full[st]);
         bulk_load(b + C::STAT_OFF + 256, p.D + qr, BT_Q * 4, &st_full[st]);
         if (DUAL) {
-          tma_load_3d(b + 2 * ROWS64_B, &tmQd, &st_full[st], 0, qr, 0);
+          tma_load_3d(b + ROWS64_B, &tmQd, &st_full[st], 0, qr, 0);
           tma_load_3d(b + 3 * ROWS64_B, &tmdOd, &st_full[st], 0, qr, 0);
           bulk_load(b + C::STAT_OFF + 512, p.rbar + qr, BT_Q * 4, &st_full[st]);
           bulk_load(b + C::STAT_OFF + 768, p.Dd + qr, BT_Q * 4, &st_full[st]);
@@ -677,32 +683,36 @@ __global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
       const uint32_t aKd = aK + 2 * ROWS128_B, aVd = aK + 3 * ROWS128_B;
       const uint32_t aP = smem_u32(sOp), adS = aP + OPND_B;
       const uint32_t aPd = aP + 2 * OPND_B, adSd = aP + 3 * OPND_B;
-      // scores of query tile i (waits for its stage)
+      // scores of query tile i (waits for its stage).  Dual: the products that share an A
+      // operand run as one N = 128 MMA over the adjacent B tiles and TMEM accumulators,
+      // K [Q | Q']^T -> [S^T | S'^T] and V [dO | dO']^T -> [dP^T | dP'^T], then the
+      // remaining terms K' Q^T, V' dO^T accumulate into the tangents.
+      const uint32_t idS2 = idesc_bf16(128, 2 * BT_Q);
       auto scores = [&](int i) -> bool {
         const int st = i % C::STAGES;
         if (!fwait(&st_full[st], (i / C::STAGES) & 1, p.status, abort)) return false;
         tc_fence_after();
-        const uint32_t aQ = smem_u32(sSt + st * C::STAGE_B), adO = aQ + ROWS64_B;
-        const uint32_t aQd = aQ + 2 * ROWS64_B, adOd = aQ + 3 * ROWS64_B;
-#pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk)
-          mma_bf16(tb + C::C_S, sdesc_sw128(aK) + 2 * kk, sdesc_sw128(aQ) + 2 * kk, idS, kk > 0);
-#pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk)
-          mma_bf16(tb + C::C_DP, sdesc_sw128(aV) + 2 * kk, sdesc_sw128(adO) + 2 * kk, idS, kk > 0);
+        const uint32_t aQ = smem_u32(sSt + st * C::STAGE_B), adO = aQ + C::OFF_DO;
         if (DUAL) {
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_SD, sdesc_sw128(aKd) + 2 * kk, sdesc_sw128(aQ) + 2 * kk, idS, kk > 0);
+            mma_bf16(tb + C::C_S, sdesc_sw128(aK) + 2 * kk, sdesc_sw128(aQ) + 2 * kk, idS2, kk > 0);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_SD, sdesc_sw128(aK) + 2 * kk, sdesc_sw128(aQd) + 2 * kk, idS, 1);
+            mma_bf16(tb + C::C_DP, sdesc_sw128(aV) + 2 * kk, sdesc_sw128(adO) + 2 * kk, idS2, kk > 0);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_DPD, sdesc_sw128(aVd) + 2 * kk, sdesc_sw128(adO) + 2 * kk, idS, kk > 0);
+            mma_bf16(tb + C::C_SD, sdesc_sw128(aKd) + 2 * kk, sdesc_sw128(aQ) + 2 * kk, idS, 1);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_DPD, sdesc_sw128(aV) + 2 * kk, sdesc_sw128(adOd) + 2 * kk, idS, 1);
+            mma_bf16(tb + C::C_DPD, sdesc_sw128(aVd) + 2 * kk, sdesc_sw128(adO) + 2 * kk, idS, 1);
+        } else {
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            mma_bf16(tb + C::C_S, sdesc_sw128(aK) + 2 * kk, sdesc_sw128(aQ) + 2 * kk, idS, kk > 0);
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            mma_bf16(tb + C::C_DP, sdesc_sw128(aV) + 2 * kk, sdesc_sw128(adO) + 2 * kk, idS, kk > 0);
         }
         mma_commit(&s_full);
         return true;
@@ -715,21 +725,23 @@ __global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
         if (!fwait(&p_full, i & 1, p.status, abort)) break;
         tc_fence_after();
         const int st = i % C::STAGES;
-        const uint32_t aQ = smem_u32(sSt + st * C::STAGE_B), adO = aQ + ROWS64_B;
-        const uint32_t aQd = aQ + 2 * ROWS64_B, adOd = aQ + 3 * ROWS64_B;
+        const uint32_t aQ = smem_u32(sSt + st * C::STAGE_B), adO = aQ + C::OFF_DO;
+        // dual: P^T [dO | dO'] -> [dV | dV'] and dS^T [Q | Q'] -> [dK | dK'] as N = 128
+        // MMAs (the tangent tiles sit one 64-column MN box after the primal ones), then
+        // P'^T dO into dV' and dS'^T Q into dK'
+        const uint32_t idA2 = idesc_bf16(128, 2 * HD) | (1u << 16);
 #pragma unroll
         for (int kk = 0; kk < BT_Q / 16; ++kk) {
           const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
           const uint64_t bO = sdesc_mn_sw128(adO) + 128 * kk, bQ = sdesc_mn_sw128(aQ) + 128 * kk;
-          mma_bf16(tb + C::C_DV, sdesc_sw128(aP) + 2 * kk, bO, idA, acc);
-          mma_bf16(tb + C::C_DK, sdesc_sw128(adS) + 2 * kk, bQ, idA, acc);
           if (DUAL) {
-            const uint64_t bOd = sdesc_mn_sw128(adOd) + 128 * kk;
-            const uint64_t bQd = sdesc_mn_sw128(aQd) + 128 * kk;
-            mma_bf16(tb + C::C_DVD, sdesc_sw128(aPd) + 2 * kk, bO, idA, acc);
-            mma_bf16(tb + C::C_DVD, sdesc_sw128(aP) + 2 * kk, bOd, idA, 1);
-            mma_bf16(tb + C::C_DKD, sdesc_sw128(adSd) + 2 * kk, bQ, idA, acc);
-            mma_bf16(tb + C::C_DKD, sdesc_sw128(adS) + 2 * kk, bQd, idA, 1);
+            mma_bf16(tb + C::C_DV, sdesc_sw128(aP) + 2 * kk, bO, idA2, acc);
+            mma_bf16(tb + C::C_DK, sdesc_sw128(adS) + 2 * kk, bQ, idA2, acc);
+            mma_bf16(tb + C::C_DVD, sdesc_sw128(aPd) + 2 * kk, bO, idA, 1);
+            mma_bf16(tb + C::C_DKD, sdesc_sw128(adSd) + 2 * kk, bQ, idA, 1);
+          } else {
+            mma_bf16(tb + C::C_DV, sdesc_sw128(aP) + 2 * kk, bO, idA, acc);
+            mma_bf16(tb + C::C_DK, sdesc_sw128(adS) + 2 * kk, bQ, idA, acc);
           }
         }
         mma_commit(&st_empty[st]);
@@ -741,20 +753,23 @@ __global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
     }
     __syncwarp();
   } else {
-    // ---- elementwise: thread r owns key row r of the tile (TMEM lane r) -----------------
+    // ---- elementwise: key row r (TMEM lane r), query columns cb .. cb + 31 -----------------
     const int q4 = warp & 3;
     const int r = q4 * 32 + lane;
+    const int cb = ((warp - 2) >> 2) * 32;
     const uint32_t lo = static_cast<uint32_t>(q4 * 32) << 16;
     const int key = key0 + r;
     bool ok = true;
     for (int i = 0; i < ntile; ++i) {
       if (!wwait(&s_full, i & 1, p.status, abort)) { ok = false; break; }
       tc_fence_after();
-      const float* stat = reinterpret_cast<const float*>(sSt + (i % C::STAGES) * C::STAGE_B + C::STAT_OFF);
+      const float4* stat = reinterpret_cast<const float4*>(
+          sSt + (i % C::STAGES) * C::STAGE_B + C::STAT_OFF);   // lse, D, rbar, D' (16 float4 each)
       const int qbase = (j0 + i) * BT_Q;
-      uint32_t pk[BT_Q / 2], dsk[BT_Q / 2], pdk[DUAL ? BT_Q / 2 : 1], dsdk[DUAL ? BT_Q / 2 : 1];
+      uint32_t pk[16], dsk[16], pdk[DUAL ? 16 : 1], dsdk[DUAL ? 16 : 1];
 #pragma unroll
-      for (int c0 = 0; c0 < BT_Q; c0 += 16) {
+      for (int h = 0; h < 2; ++h) {
+        const int c0 = cb + 16 * h;
         float sv[16], dp[16], sd[16], dpd[16];
         tmem_ld16_nowait(tb + lo + C::C_S + c0, sv);
         tmem_ld16_nowait(tb + lo + C::C_DP + c0, dp);
@@ -763,47 +778,59 @@ __global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
           tmem_ld16_nowait(tb + lo + C::C_DPD + c0, dpd);
         }
         tmem_wait_ld();
+        if (h == 1) {
+          // this tile's scores are read: the next tile's may be computed meanwhile
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_local(&s_free);
+        }
 #pragma unroll
-        for (int e = 0; e < 16; e += 2) {
-          float pv[2], dsv[2], pdv[2], dsdv[2];
+        for (int e = 0; e < 16; e += 4) {
+          const int c = c0 + e;
+          const float4 l4 = stat[c / 4], d4 = stat[16 + c / 4];
+          float4 rb4 = make_float4(0.f, 0.f, 0.f, 0.f), dd4 = rb4;
+          if (DUAL) { rb4 = stat[32 + c / 4]; dd4 = stat[48 + c / 4]; }
+          const float lv[4] = {l4.x, l4.y, l4.z, l4.w}, dv[4] = {d4.x, d4.y, d4.z, d4.w};
+          const float rv[4] = {rb4.x, rb4.y, rb4.z, rb4.w}, ddv[4] = {dd4.x, dd4.y, dd4.z, dd4.w};
+          float pv[4], dsv[4], pdv[4], dsdv[4];
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const int c = c0 + e + h;
-            const float pp = qbase + c >= key ? __expf(sv[e + h] - stat[c]) : 0.f;
-            const float dpm = dp[e + h] - stat[64 + c];
-            pv[h] = pp;
-            dsv[h] = pp * dpm;
+          for (int u = 0; u < 4; ++u) {
+            const float pp = qbase + c + u >= key ? __expf(sv[e + u] - lv[u]) : 0.f;
+            const float dpm = dp[e + u] - dv[u];
+            pv[u] = pp;
+            dsv[u] = pp * dpm;
             if (DUAL) {
-              const float pd = pp * (sd[e + h] - stat[128 + c]);
-              pdv[h] = pd;
-              dsdv[h] = pd * dpm + pp * (dpd[e + h] - stat[192 + c]);
+              const float pd = pp * (sd[e + u] - rv[u]);
+              pdv[u] = pd;
+              dsdv[u] = pd * dpm + pp * (dpd[e + u] - ddv[u]);
             }
           }
-          pk[(c0 + e) / 2] = pack_bf16x2(pv[0], pv[1]);
-          dsk[(c0 + e) / 2] = pack_bf16x2(dsv[0], dsv[1]);
+          const int k = (16 * h + e) / 2;
+          pk[k] = pack_bf16x2(pv[0], pv[1]);
+          pk[k + 1] = pack_bf16x2(pv[2], pv[3]);
+          dsk[k] = pack_bf16x2(dsv[0], dsv[1]);
+          dsk[k + 1] = pack_bf16x2(dsv[2], dsv[3]);
           if (DUAL) {
-            pdk[(c0 + e) / 2] = pack_bf16x2(pdv[0], pdv[1]);
-            dsdk[(c0 + e) / 2] = pack_bf16x2(dsdv[0], dsdv[1]);
+            pdk[k] = pack_bf16x2(pdv[0], pdv[1]);
+            pdk[k + 1] = pack_bf16x2(pdv[2], pdv[3]);
+            dsdk[k] = pack_bf16x2(dsdv[0], dsdv[1]);
+            dsdk[k + 1] = pack_bf16x2(dsdv[2], dsdv[3]);
           }
         }
       }
-      // this tile's scores are read: the next tile's may be computed
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_local(&s_free);
       // the previous tile's accumulating products have read the A operands
       if (i > 0 && !wwait(&o_done, (i - 1) & 1, p.status, abort)) { ok = false; break; }
 #pragma unroll
-      for (int ch = 0; ch < BT_Q / 8; ++ch) {
-        *reinterpret_cast<uint4*>(sOp + swz(r, ch)) =
-            make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]);
-        *reinterpret_cast<uint4*>(sOp + OPND_B + swz(r, ch)) =
-            make_uint4(dsk[4 * ch], dsk[4 * ch + 1], dsk[4 * ch + 2], dsk[4 * ch + 3]);
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t o = swz(r, cb / 8 + j);
+        *reinterpret_cast<uint4*>(sOp + o) = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+        *reinterpret_cast<uint4*>(sOp + OPND_B + o) =
+            make_uint4(dsk[4 * j], dsk[4 * j + 1], dsk[4 * j + 2], dsk[4 * j + 3]);
         if (DUAL) {
-          *reinterpret_cast<uint4*>(sOp + 2 * OPND_B + swz(r, ch)) =
-              make_uint4(pdk[4 * ch], pdk[4 * ch + 1], pdk[4 * ch + 2], pdk[4 * ch + 3]);
-          *reinterpret_cast<uint4*>(sOp + 3 * OPND_B + swz(r, ch)) =
-              make_uint4(dsdk[4 * ch], dsdk[4 * ch + 1], dsdk[4 * ch + 2], dsdk[4 * ch + 3]);
+          *reinterpret_cast<uint4*>(sOp + 2 * OPND_B + o) =
+              make_uint4(pdk[4 * j], pdk[4 * j + 1], pdk[4 * j + 2], pdk[4 * j + 3]);
+          *reinterpret_cast<uint4*>(sOp + 3 * OPND_B + o) =
+              make_uint4(dsdk[4 * j], dsdk[4 * j + 1], dsdk[4 * j + 2], dsdk[4 * j + 3]);
         }
       }
       fence_async_smem();
@@ -811,15 +838,15 @@ __global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
       __syncwarp();
       if (lane == 0) mbar_arrive_local(&p_full);
     }
-    // ---- outputs: dV, dK (dV', dK') rows of this key ------------------------------------
+    // ---- outputs: dV, dK (dV', dK') rows of this key, this thread's columns ---------------
     if (ok && wwait(&o_done, (ntile - 1) & 1, p.status, abort)) {
       tc_fence_after();
       const int64_t off = (static_cast<int64_t>(row0) + key) * HD;
-      store_acc_row(tb + lo + C::C_DV, p.dV + off);
-      store_acc_row(tb + lo + C::C_DK, p.dK + off);
+      store_acc_row(tb + lo + C::C_DV, p.dV + off, cb);
+      store_acc_row(tb + lo + C::C_DK, p.dK + off, cb);
       if (DUAL) {
-        store_acc_row(tb + lo + C::C_DVD, p.dVd + off);
-        store_acc_row(tb + lo + C::C_DKD, p.dKd + off);
+        store_acc_row(tb + lo + C::C_DVD, p.dVd + off, cb);
+        store_acc_row(tb + lo + C::C_DKD, p.dKd + off, cb);
       }
     }
     tc_fence_before();
@@ -867,8 +894,8 @@ __global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
   if (threadIdx.x == 0) {
     mbar_init(&res_full, 1);
     mbar_init(&s_full, 1);
-    mbar_init(&s_free, 4);
-    mbar_init(&p_full, 4);
+    mbar_init(&s_free, BW_EW);
+    mbar_init(&p_full, BW_EW);
     mbar_init(&o_done, 1);
     mbar_init(&drain, 1);
     for (int i = 0; i < C::STAGES; ++i) {
@@ -920,9 +947,9 @@ __global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
         uint8_t* b = sSt + st * C::STAGE_B;
         const int kr = row0 + i * BT_Q;
         tma_load_3d(b, &tmK, &st_full[st], 0, kr, 0);
-        tma_load_3d(b + ROWS64_B, &tmV, &st_full[st], 0, kr, 0);
+        tma_load_3d(b + C::OFF_V, &tmV, &st_full[st], 0, kr, 0);
         if (DUAL) {
-          tma_load_3d(b + 2 * ROWS64_B, &tmKd, &st_full[st], 0, kr, 0);
+          tma_load_3d(b + ROWS64_B, &tmKd, &st_full[st], 0, kr, 0);
           tma_load_3d(b + 3 * ROWS64_B, &tmVd, &st_full[st], 0, kr, 0);
         }
       }
@@ -938,31 +965,34 @@ __global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
       const uint32_t aQ = smem_u32(sRes), adO = aQ + ROWS128_B;
       const uint32_t aQd = aQ + 2 * ROWS128_B, adOd = aQ + 3 * ROWS128_B;
       const uint32_t adS = smem_u32(sOp), adSd = adS + OPND_B;
+      // dual: Q [K | K']^T -> [S | S'] and dO [V | V']^T -> [dP | dP'] as N = 128 MMAs,
+      // then Q' K^T and dO' V^T accumulate into the tangents
+      const uint32_t idS2 = idesc_bf16(128, 2 * BT_Q);
       auto scores = [&](int i) -> bool {
         const int st = i % C::STAGES;
         if (!fwait(&st_full[st], (i / C::STAGES) & 1, p.status, abort)) return false;
         tc_fence_after();
-        const uint32_t aK = smem_u32(sSt + st * C::STAGE_B), aV = aK + ROWS64_B;
-        const uint32_t aKd = aK + 2 * ROWS64_B, aVd = aK + 3 * ROWS64_B;
-#pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk)
-          mma_bf16(tb + C::C_S, sdesc_sw128(aQ) + 2 * kk, sdesc_sw128(aK) + 2 * kk, idS, kk > 0);
-#pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk)
-          mma_bf16(tb + C::C_DP, sdesc_sw128(adO) + 2 * kk, sdesc_sw128(aV) + 2 * kk, idS, kk > 0);
+        const uint32_t aK = smem_u32(sSt + st * C::STAGE_B), aV = aK + C::OFF_V;
         if (DUAL) {
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_SD, sdesc_sw128(aQd) + 2 * kk, sdesc_sw128(aK) + 2 * kk, idS, kk > 0);
+            mma_bf16(tb + C::C_S, sdesc_sw128(aQ) + 2 * kk, sdesc_sw128(aK) + 2 * kk, idS2, kk > 0);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_SD, sdesc_sw128(aQ) + 2 * kk, sdesc_sw128(aKd) + 2 * kk, idS, 1);
+            mma_bf16(tb + C::C_DP, sdesc_sw128(adO) + 2 * kk, sdesc_sw128(aV) + 2 * kk, idS2, kk > 0);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_DPD, sdesc_sw128(adOd) + 2 * kk, sdesc_sw128(aV) + 2 * kk, idS, kk > 0);
+            mma_bf16(tb + C::C_SD, sdesc_sw128(aQd) + 2 * kk, sdesc_sw128(aK) + 2 * kk, idS, 1);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_DPD, sdesc_sw128(adO) + 2 * kk, sdesc_sw128(aVd) + 2 * kk, idS, 1);
+            mma_bf16(tb + C::C_DPD, sdesc_sw128(adOd) + 2 * kk, sdesc_sw128(aV) + 2 * kk, idS, 1);
+        } else {
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            mma_bf16(tb + C::C_S, sdesc_sw128(aQ) + 2 * kk, sdesc_sw128(aK) + 2 * kk, idS, kk > 0);
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            mma_bf16(tb + C::C_DP, sdesc_sw128(adO) + 2 * kk, sdesc_sw128(aV) + 2 * kk, idS, kk > 0);
         }
         mma_commit(&s_full);
         return true;
@@ -974,15 +1004,18 @@ __global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
         if (!fwait(&p_full, i & 1, p.status, abort)) break;
         tc_fence_after();
         const int st = i % C::STAGES;
-        const uint32_t aK = smem_u32(sSt + st * C::STAGE_B), aKd = aK + 2 * ROWS64_B;
+        const uint32_t aK = smem_u32(sSt + st * C::STAGE_B);
+        // dual: dS [K | K'] -> [dQ | dQ'] as one N = 128 MMA, then dS' K into dQ'
+        const uint32_t idA2 = idesc_bf16(128, 2 * HD) | (1u << 16);
 #pragma unroll
         for (int kk = 0; kk < BT_Q / 16; ++kk) {
           const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
           const uint64_t bK = sdesc_mn_sw128(aK) + 128 * kk;
-          mma_bf16(tb + C::C_DQ, sdesc_sw128(adS) + 2 * kk, bK, idA, acc);
           if (DUAL) {
-            mma_bf16(tb + C::C_DQD, sdesc_sw128(adSd) + 2 * kk, bK, idA, acc);
-            mma_bf16(tb + C::C_DQD, sdesc_sw128(adS) + 2 * kk, sdesc_mn_sw128(aKd) + 128 * kk, idA, 1);
+            mma_bf16(tb + C::C_DQ, sdesc_sw128(adS) + 2 * kk, bK, idA2, acc);
+            mma_bf16(tb + C::C_DQD, sdesc_sw128(adSd) + 2 * kk, bK, idA, 1);
+          } else {
+            mma_bf16(tb + C::C_DQ, sdesc_sw128(adS) + 2 * kk, bK, idA, acc);
           }
         }
         mma_commit(&st_empty[st]);
@@ -993,9 +1026,10 @@ __global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
     }
     __syncwarp();
   } else {
-    // ---- elementwise: thread r owns query row r of the tile (TMEM lane r) ---------------
+    // ---- elementwise: query row r (TMEM lane r), key columns cb .. cb + 31 -----------------
     const int q4 = warp & 3;
     const int r = q4 * 32 + lane;
+    const int cb = ((warp - 2) >> 2) * 32;
     const uint32_t lo = static_cast<uint32_t>(q4 * 32) << 16;
     const int q = q0 + r;
     const int64_t gi = static_cast<int64_t>(row0) + q;
@@ -1006,9 +1040,10 @@ __global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
       if (!wwait(&s_full, i & 1, p.status, abort)) { ok = false; break; }
       tc_fence_after();
       const int kbase = i * BT_Q;
-      uint32_t dsk[BT_Q / 2], dsdk[DUAL ? BT_Q / 2 : 1];
+      uint32_t dsk[16], dsdk[DUAL ? 16 : 1];
 #pragma unroll
-      for (int c0 = 0; c0 < BT_Q; c0 += 16) {
+      for (int h = 0; h < 2; ++h) {
+        const int c0 = cb + 16 * h;
         float sv[16], dp[16], sd[16], dpd[16];
         tmem_ld16_nowait(tb + lo + C::C_S + c0, sv);
         tmem_ld16_nowait(tb + lo + C::C_DP + c0, dp);
@@ -1017,35 +1052,38 @@ __global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
           tmem_ld16_nowait(tb + lo + C::C_DPD + c0, dpd);
         }
         tmem_wait_ld();
+        if (h == 1) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_local(&s_free);
+        }
 #pragma unroll
         for (int e = 0; e < 16; e += 2) {
           float dsv[2], dsdv[2];
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const int key = kbase + c0 + e + h;
-            const float pp = key <= q ? __expf(sv[e + h] - lse) : 0.f;
-            const float dpm = dp[e + h] - Dv;
-            dsv[h] = pp * dpm;
+          for (int u = 0; u < 2; ++u) {
+            const int key = kbase + c0 + e + u;
+            const float pp = key <= q ? __expf(sv[e + u] - lse) : 0.f;
+            const float dpm = dp[e + u] - Dv;
+            dsv[u] = pp * dpm;
             if (DUAL) {
-              const float pd = pp * (sd[e + h] - rb);
-              dsdv[h] = pd * dpm + pp * (dpd[e + h] - Ddv);
+              const float pd = pp * (sd[e + u] - rb);
+              dsdv[u] = pd * dpm + pp * (dpd[e + u] - Ddv);
             }
           }
-          dsk[(c0 + e) / 2] = pack_bf16x2(dsv[0], dsv[1]);
-          if (DUAL) dsdk[(c0 + e) / 2] = pack_bf16x2(dsdv[0], dsdv[1]);
+          dsk[(16 * h + e) / 2] = pack_bf16x2(dsv[0], dsv[1]);
+          if (DUAL) dsdk[(16 * h + e) / 2] = pack_bf16x2(dsdv[0], dsdv[1]);
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_local(&s_free);
       if (i > 0 && !wwait(&o_done, (i - 1) & 1, p.status, abort)) { ok = false; break; }
 #pragma unroll
-      for (int ch = 0; ch < BT_Q / 8; ++ch) {
-        *reinterpret_cast<uint4*>(sOp + swz(r, ch)) =
-            make_uint4(dsk[4 * ch], dsk[4 * ch + 1], dsk[4 * ch + 2], dsk[4 * ch + 3]);
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t o = swz(r, cb / 8 + j);
+        *reinterpret_cast<uint4*>(sOp + o) =
+            make_uint4(dsk[4 * j], dsk[4 * j + 1], dsk[4 * j + 2], dsk[4 * j + 3]);
         if (DUAL)
-          *reinterpret_cast<uint4*>(sOp + OPND_B + swz(r, ch)) =
-              make_uint4(dsdk[4 * ch], dsdk[4 * ch + 1], dsdk[4 * ch + 2], dsdk[4 * ch + 3]);
+          *reinterpret_cast<uint4*>(sOp + OPND_B + o) =
+              make_uint4(dsdk[4 * j], dsdk[4 * j + 1], dsdk[4 * j + 2], dsdk[4 * j + 3]);
       }
       fence_async_smem();
       tc_fence_before();
@@ -1055,8 +1093,8 @@ __global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
     if (ok && wwait(&o_done, (ntile - 1) & 1, p.status, abort)) {
       tc_fence_after();
       const int64_t off = gi * HD;
-      store_acc_row(tb + lo + C::C_DQ, p.dQ + off);
-      if (DUAL) store_acc_row(tb + lo + C::C_DQD, p.dQd + off);
+      store_acc_row(tb + lo + C::C_DQ, p.dQ + off, cb);
+      if (DUAL) store_acc_row(tb + lo + C::C_DQD, p.dQd + off, cb);
     }
     tc_fence_before();
   }
