@@ -513,7 +513,8 @@ def run_gpu(args):
         traffic = _dram_traffic(args.workload) if default and not (
             args.gemm_persistent is not None or args.fused_head or args.layer_updates) else None
         flash_desc = {0: "attention materialised per block", 1: "", 2: "warp-level fused attention only",
-                      3: "tcgen05 fused attention forwards", 4: "tcgen05 fused attention backward"}
+                      3: "tcgen05 primal attention forward too",
+                      4: "warp-level fused attention backward"}
         out = {
             "metric": "meta-grad steps/s", "value": value, "unit": "meta-steps/s", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,

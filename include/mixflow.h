@@ -297,11 +297,11 @@ mf_status mf_replay_gemms(mf_handle h, int reps, void* stream, double* ms, uint6
  * summation order within a tile, which both forms share.
  * MF_OPT_FLASH_ATTN (default 1): the decoder's dual attention runs fused, without the
  * S x S probabilities and their tangent in memory (bf16 decoders with d_model/n_heads = 64
- * and seq_len a multiple of 64; others always use the materialised form).  With 1, the
- * dual (tangent-carrying) forward of sequences of whole 128-token tiles runs on tcgen05
- * tensor cores and every other attention kernel on warp-level MMAs; 3 runs the primal
- * forward on tcgen05 as well; 4 runs the dual forward and both backward kernels (primal
- * and dual) on tcgen05; 2 uses the warp-level kernels only.  0 materialises them (per
+ * and seq_len a multiple of 64; others always use the materialised form).  With 1, for
+ * sequences of whole 128-token tiles, the dual (tangent-carrying) forward and both backward
+ * kernels (primal and dual) run on tcgen05 tensor cores and the primal forward on
+ * warp-level MMAs; 3 runs the primal forward on tcgen05 as well; 4 keeps the backward on
+ * warp-level MMAs; 2 uses the warp-level kernels only.  0 materialises them (per
  * block, for the backward).  Setting it drops the handle's captured graphs and changes the
  * workspace size.
  * MF_OPT_GEMM_PERSISTENT (process-wide, default 2): GEMMs that take CTA-pair tiles run as a

@@ -266,7 +266,7 @@ struct DecExec {
     fa.BH = BH;
     fa.S = Ly.S;
     fa.tc = h->flash == 1 || h->flash == 4 ? 1 : h->flash == 3 ? 2 : 0;
-    fa.tc_bwd = h->flash == 4 ? 1 : 0;
+    fa.tc_bwd = h->flash == 1 || h->flash == 3 ? 1 : 0;
     fa.status = h->d_status;
     fa.Q = hb(p.Q[l]); fa.K = hb(p.K[l]); fa.V = hb(p.Vv[l]);
     fa.Qd = hb(p.Qd[l]); fa.Kd = hb(p.Kd[l]); fa.Vd = hb(p.Vd[l]);

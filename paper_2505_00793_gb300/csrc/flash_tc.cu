@@ -10,6 +10,8 @@
 //                 S  = Q K^T,  S' = Q' K^T + Q K'^T            (M 128, N 64 keys, K 64)
 //                 O += P V,  T += (P (*) S') V + P V'          (M 128, N 64, K 64 keys; V
 //                                                               and V' read MN-major in place)
+//               with the products that share an A operand as one N = 128 MMA over adjacent
+//               B tiles and accumulators: Q [K | K']^T -> [S | Q K'^T], P [V | V'] -> [O | P V']
 //   warps 2..5  softmax: thread r owns query row r (TMEM lane r).  It reads its row of S
 //               (and S') from TMEM, updates the running maximum, writes P = exp(S - m) and
 //               P (*) S' as bf16 into shared memory (the A operands of the next products) and
@@ -47,7 +49,8 @@ constexpr int BT_Q = 64;           // backward: queries (key-tile kernel) or key
 template <bool DUAL>
 struct FtcCfg {
   static constexpr int STAGES = DUAL ? 1 : 2;
-  static constexpr int STAGE_B = (DUAL ? 4 : 2) * K_TILE_B;  // K, V (K', V')
+  static constexpr int STAGE_B = (DUAL ? 4 : 2) * K_TILE_B;  // K, (K',) V (, V')
+  static constexpr int OFF_V = (DUAL ? 2 : 1) * K_TILE_B;     // K' follows K, V' follows V
   static constexpr int Q_B = (DUAL ? 2 : 1) * Q_TILE_B;      // Q (Q')
   static constexpr int P_B = (DUAL ? 2 : 1) * P_ATOM;        // P (P (*) S')
   static constexpr int SMEM = Q_B + STAGES * STAGE_B + P_B + 1024;
@@ -159,7 +162,7 @@ __global__ void __launch_bounds__(FTC_THREADS, FtcCfg<DUAL>::CTAS)
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint8_t* sQ = smem;                       // Q, then Q'
-  uint8_t* sKV = smem + C::Q_B;             // stage st: K, V, K', V' (8 KB each)
+  uint8_t* sKV = smem + C::Q_B;             // stage st: K, K', V, V' (8 KB each)
   uint8_t* sP = sKV + C::STAGES * C::STAGE_B;   // P, then P (*) S' (16 KB each)
   const int nq = p.S / TQ;
   // grid (heads, tiles): heads dispatch fastest, so every head's longest query tile goes
@@ -220,9 +223,9 @@ __global__ void __launch_bounds__(FTC_THREADS, FtcCfg<DUAL>::CTAS)
         uint8_t* b = sKV + st * C::STAGE_B;
         const int kr = row0 + j * TK;
         tma_load_3d(b, &tmK, &kv_full[st], 0, kr, 0);
-        tma_load_3d(b + K_TILE_B, &tmV, &kv_full[st], 0, kr, 0);
+        tma_load_3d(b + C::OFF_V, &tmV, &kv_full[st], 0, kr, 0);
         if (DUAL) {
-          tma_load_3d(b + 2 * K_TILE_B, &tmKd, &kv_full[st], 0, kr, 0);
+          tma_load_3d(b + K_TILE_B, &tmKd, &kv_full[st], 0, kr, 0);
           tma_load_3d(b + 3 * K_TILE_B, &tmVd, &kv_full[st], 0, kr, 0);
         }
       }
@@ -236,7 +239,13 @@ __global__ void __launch_bounds__(FTC_THREADS, FtcCfg<DUAL>::CTAS)
       // ---- MMA issuer -------------------------------------------------------------------
       const uint32_t idS = idesc_bf16(TQ, TK);
       const uint32_t idO = idesc_bf16(TQ, HD) | (1u << 16);   // B (V) read MN-major
-      const uint32_t aQ = smem_u32(sQ), aP = smem_u32(sP);
+      const uint32_t idS2 = idesc_bf16(TQ, 2 * TK);
+      const uint32_t idO2 = idesc_bf16(TQ, 2 * HD) | (1u << 16);
+      // operand descriptors, built once: a byte offset moves a descriptor by offset >> 4
+      const uint64_t dQ = sdesc_sw128(smem_u32(sQ)), dQd = dQ + (Q_TILE_B >> 4);
+      const uint64_t dP = sdesc_sw128(smem_u32(sP)), dPS = dP + (P_ATOM >> 4);
+      const uint64_t dKV = sdesc_sw128(smem_u32(sKV)), mKV = sdesc_mn_sw128(smem_u32(sKV));
+      constexpr uint64_t ST_STEP = C::STAGE_B >> 4, V_STEP = C::OFF_V >> 4;
       bool ok = fwait(&q_full, 0, p.status, abort);
       for (int j = 0; ok && j < nkt; ++j) {
         const int st = j % C::STAGES;
@@ -244,34 +253,33 @@ __global__ void __launch_bounds__(FTC_THREADS, FtcCfg<DUAL>::CTAS)
         if (!fwait(&kv_full[st], ph, p.status, abort)) break;
         if (j > 0 && !fwait(&s_free, (j - 1) & 1, p.status, abort)) break;
         tc_fence_after();
-        const uint32_t aK = smem_u32(sKV + st * C::STAGE_B);
-        const uint32_t aV = aK + K_TILE_B;
-#pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk)
-          mma_bf16(tb + C::C_S, sdesc_sw128(aQ) + 2 * kk, sdesc_sw128(aK) + 2 * kk, idS, kk > 0);
+        const uint64_t dK = dKV + st * ST_STEP, mV = mKV + st * ST_STEP + V_STEP;
         if (DUAL) {
-          const uint32_t aQd = aQ + Q_TILE_B, aKd = aK + 2 * K_TILE_B;
+          // Q [K | K']^T -> [S | Q K'^T] in one N = 128 MMA (K' follows K), then Q' K^T into S'
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_SD, sdesc_sw128(aQd) + 2 * kk, sdesc_sw128(aK) + 2 * kk, idS, kk > 0);
+            mma_bf16(tb + C::C_S, dQ + 2 * kk, dK + 2 * kk, idS2, kk > 0);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_SD, sdesc_sw128(aQ) + 2 * kk, sdesc_sw128(aKd) + 2 * kk, idS, 1);
+            mma_bf16(tb + C::C_SD, dQd + 2 * kk, dK + 2 * kk, idS, 1);
+        } else {
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            mma_bf16(tb + C::C_S, dQ + 2 * kk, dK + 2 * kk, idS, kk > 0);
         }
         mma_commit(&s_full);
         if (!fwait(&p_full, j & 1, p.status, abort)) break;
         tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < TK / 16; ++kk) {
-          const uint64_t pa = sdesc_sw128(aP) + 2 * kk;
-          const uint64_t vb = sdesc_mn_sw128(aV) + 128 * kk;
+          const uint64_t vb = mV + 128 * kk;
           const uint32_t acc = (j > 0 || kk > 0) ? 1u : 0u;
-          mma_bf16(tb + C::C_O, pa, vb, idO, acc);
           if (DUAL) {
-            const uint64_t psa = sdesc_sw128(aP + P_ATOM) + 2 * kk;
-            const uint64_t vdb = sdesc_mn_sw128(aK + 3 * K_TILE_B) + 128 * kk;
-            mma_bf16(tb + C::C_T, psa, vb, idO, acc);
-            mma_bf16(tb + C::C_T, pa, vdb, idO, 1);
+            // P [V | V'] -> [O | P V'] in one N = 128 MMA (T follows O), then (P (*) S') V into T
+            mma_bf16(tb + C::C_O, dP + 2 * kk, vb, idO2, acc);
+            mma_bf16(tb + C::C_T, dPS + 2 * kk, vb, idO, 1);
+          } else {
+            mma_bf16(tb + C::C_O, dP + 2 * kk, vb, idO, acc);
           }
         }
         mma_commit(&kv_empty[st]);
@@ -683,6 +691,13 @@ __global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
       const uint32_t aKd = aK + 2 * ROWS128_B, aVd = aK + 3 * ROWS128_B;
       const uint32_t aP = smem_u32(sOp), adS = aP + OPND_B;
       const uint32_t aPd = aP + 2 * OPND_B, adSd = aP + 3 * OPND_B;
+      // operand descriptors, built once: a byte offset moves a descriptor by offset >> 4
+      const uint64_t dK = sdesc_sw128(aK), dV = sdesc_sw128(aV);
+      const uint64_t dKd = sdesc_sw128(aKd), dVd = sdesc_sw128(aVd);
+      const uint64_t dP = sdesc_sw128(aP), ddS = sdesc_sw128(adS);
+      const uint64_t dPd = sdesc_sw128(aPd), ddSd = sdesc_sw128(adSd);
+      const uint64_t dSt = sdesc_sw128(smem_u32(sSt)), mSt = sdesc_mn_sw128(smem_u32(sSt));
+      constexpr uint64_t ST_STEP = C::STAGE_B >> 4, DO_STEP = C::OFF_DO >> 4;
       // scores of query tile i (waits for its stage).  Dual: the products that share an A
       // operand run as one N = 128 MMA over the adjacent B tiles and TMEM accumulators,
       // K [Q | Q']^T -> [S^T | S'^T] and V [dO | dO']^T -> [dP^T | dP'^T], then the
@@ -692,27 +707,27 @@ __global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
         const int st = i % C::STAGES;
         if (!fwait(&st_full[st], (i / C::STAGES) & 1, p.status, abort)) return false;
         tc_fence_after();
-        const uint32_t aQ = smem_u32(sSt + st * C::STAGE_B), adO = aQ + C::OFF_DO;
+        const uint64_t dQ = dSt + st * ST_STEP, ddO = dQ + DO_STEP;
         if (DUAL) {
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_S, sdesc_sw128(aK) + 2 * kk, sdesc_sw128(aQ) + 2 * kk, idS2, kk > 0);
+            mma_bf16(tb + C::C_S, dK + 2 * kk, dQ + 2 * kk, idS2, kk > 0);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_DP, sdesc_sw128(aV) + 2 * kk, sdesc_sw128(adO) + 2 * kk, idS2, kk > 0);
+            mma_bf16(tb + C::C_DP, dV + 2 * kk, ddO + 2 * kk, idS2, kk > 0);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_SD, sdesc_sw128(aKd) + 2 * kk, sdesc_sw128(aQ) + 2 * kk, idS, 1);
+            mma_bf16(tb + C::C_SD, dKd + 2 * kk, dQ + 2 * kk, idS, 1);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_DPD, sdesc_sw128(aVd) + 2 * kk, sdesc_sw128(adO) + 2 * kk, idS, 1);
+            mma_bf16(tb + C::C_DPD, dVd + 2 * kk, ddO + 2 * kk, idS, 1);
         } else {
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_S, sdesc_sw128(aK) + 2 * kk, sdesc_sw128(aQ) + 2 * kk, idS, kk > 0);
+            mma_bf16(tb + C::C_S, dK + 2 * kk, dQ + 2 * kk, idS, kk > 0);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_DP, sdesc_sw128(aV) + 2 * kk, sdesc_sw128(adO) + 2 * kk, idS, kk > 0);
+            mma_bf16(tb + C::C_DP, dV + 2 * kk, ddO + 2 * kk, idS, kk > 0);
         }
         mma_commit(&s_full);
         return true;
@@ -725,7 +740,7 @@ __global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
         if (!fwait(&p_full, i & 1, p.status, abort)) break;
         tc_fence_after();
         const int st = i % C::STAGES;
-        const uint32_t aQ = smem_u32(sSt + st * C::STAGE_B), adO = aQ + C::OFF_DO;
+        const uint64_t mQ = mSt + st * ST_STEP, mdO = mQ + DO_STEP;
         // dual: P^T [dO | dO'] -> [dV | dV'] and dS^T [Q | Q'] -> [dK | dK'] as N = 128
         // MMAs (the tangent tiles sit one 64-column MN box after the primal ones), then
         // P'^T dO into dV' and dS'^T Q into dK'
@@ -733,15 +748,15 @@ __global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
 #pragma unroll
         for (int kk = 0; kk < BT_Q / 16; ++kk) {
           const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
-          const uint64_t bO = sdesc_mn_sw128(adO) + 128 * kk, bQ = sdesc_mn_sw128(aQ) + 128 * kk;
+          const uint64_t bO = mdO + 128 * kk, bQ = mQ + 128 * kk;
           if (DUAL) {
-            mma_bf16(tb + C::C_DV, sdesc_sw128(aP) + 2 * kk, bO, idA2, acc);
-            mma_bf16(tb + C::C_DK, sdesc_sw128(adS) + 2 * kk, bQ, idA2, acc);
-            mma_bf16(tb + C::C_DVD, sdesc_sw128(aPd) + 2 * kk, bO, idA, 1);
-            mma_bf16(tb + C::C_DKD, sdesc_sw128(adSd) + 2 * kk, bQ, idA, 1);
+            mma_bf16(tb + C::C_DV, dP + 2 * kk, bO, idA2, acc);
+            mma_bf16(tb + C::C_DK, ddS + 2 * kk, bQ, idA2, acc);
+            mma_bf16(tb + C::C_DVD, dPd + 2 * kk, bO, idA, 1);
+            mma_bf16(tb + C::C_DKD, ddSd + 2 * kk, bQ, idA, 1);
           } else {
-            mma_bf16(tb + C::C_DV, sdesc_sw128(aP) + 2 * kk, bO, idA, acc);
-            mma_bf16(tb + C::C_DK, sdesc_sw128(adS) + 2 * kk, bQ, idA, acc);
+            mma_bf16(tb + C::C_DV, dP + 2 * kk, bO, idA, acc);
+            mma_bf16(tb + C::C_DK, ddS + 2 * kk, bQ, idA, acc);
           }
         }
         mma_commit(&st_empty[st]);
@@ -965,6 +980,12 @@ __global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
       const uint32_t aQ = smem_u32(sRes), adO = aQ + ROWS128_B;
       const uint32_t aQd = aQ + 2 * ROWS128_B, adOd = aQ + 3 * ROWS128_B;
       const uint32_t adS = smem_u32(sOp), adSd = adS + OPND_B;
+      // operand descriptors, built once: a byte offset moves a descriptor by offset >> 4
+      const uint64_t dQ = sdesc_sw128(aQ), ddO = sdesc_sw128(adO);
+      const uint64_t dQd = sdesc_sw128(aQd), ddOd = sdesc_sw128(adOd);
+      const uint64_t ddS = sdesc_sw128(adS), ddSd = sdesc_sw128(adSd);
+      const uint64_t dSt = sdesc_sw128(smem_u32(sSt)), mSt = sdesc_mn_sw128(smem_u32(sSt));
+      constexpr uint64_t ST_STEP = C::STAGE_B >> 4, V_STEP = C::OFF_V >> 4;
       // dual: Q [K | K']^T -> [S | S'] and dO [V | V']^T -> [dP | dP'] as N = 128 MMAs,
       // then Q' K^T and dO' V^T accumulate into the tangents
       const uint32_t idS2 = idesc_bf16(128, 2 * BT_Q);
@@ -972,27 +993,27 @@ __global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
         const int st = i % C::STAGES;
         if (!fwait(&st_full[st], (i / C::STAGES) & 1, p.status, abort)) return false;
         tc_fence_after();
-        const uint32_t aK = smem_u32(sSt + st * C::STAGE_B), aV = aK + C::OFF_V;
+        const uint64_t dK = dSt + st * ST_STEP, dV = dK + V_STEP;
         if (DUAL) {
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_S, sdesc_sw128(aQ) + 2 * kk, sdesc_sw128(aK) + 2 * kk, idS2, kk > 0);
+            mma_bf16(tb + C::C_S, dQ + 2 * kk, dK + 2 * kk, idS2, kk > 0);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_DP, sdesc_sw128(adO) + 2 * kk, sdesc_sw128(aV) + 2 * kk, idS2, kk > 0);
+            mma_bf16(tb + C::C_DP, ddO + 2 * kk, dV + 2 * kk, idS2, kk > 0);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_SD, sdesc_sw128(aQd) + 2 * kk, sdesc_sw128(aK) + 2 * kk, idS, 1);
+            mma_bf16(tb + C::C_SD, dQd + 2 * kk, dK + 2 * kk, idS, 1);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_DPD, sdesc_sw128(adOd) + 2 * kk, sdesc_sw128(aV) + 2 * kk, idS, 1);
+            mma_bf16(tb + C::C_DPD, ddOd + 2 * kk, dV + 2 * kk, idS, 1);
         } else {
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_S, sdesc_sw128(aQ) + 2 * kk, sdesc_sw128(aK) + 2 * kk, idS, kk > 0);
+            mma_bf16(tb + C::C_S, dQ + 2 * kk, dK + 2 * kk, idS, kk > 0);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            mma_bf16(tb + C::C_DP, sdesc_sw128(adO) + 2 * kk, sdesc_sw128(aV) + 2 * kk, idS, kk > 0);
+            mma_bf16(tb + C::C_DP, ddO + 2 * kk, dV + 2 * kk, idS, kk > 0);
         }
         mma_commit(&s_full);
         return true;
@@ -1004,18 +1025,18 @@ __global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
         if (!fwait(&p_full, i & 1, p.status, abort)) break;
         tc_fence_after();
         const int st = i % C::STAGES;
-        const uint32_t aK = smem_u32(sSt + st * C::STAGE_B);
+        const uint64_t mK = mSt + st * ST_STEP;
         // dual: dS [K | K'] -> [dQ | dQ'] as one N = 128 MMA, then dS' K into dQ'
         const uint32_t idA2 = idesc_bf16(128, 2 * HD) | (1u << 16);
 #pragma unroll
         for (int kk = 0; kk < BT_Q / 16; ++kk) {
           const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
-          const uint64_t bK = sdesc_mn_sw128(aK) + 128 * kk;
+          const uint64_t bK = mK + 128 * kk;
           if (DUAL) {
-            mma_bf16(tb + C::C_DQ, sdesc_sw128(adS) + 2 * kk, bK, idA2, acc);
-            mma_bf16(tb + C::C_DQD, sdesc_sw128(adSd) + 2 * kk, bK, idA, 1);
+            mma_bf16(tb + C::C_DQ, ddS + 2 * kk, bK, idA2, acc);
+            mma_bf16(tb + C::C_DQD, ddSd + 2 * kk, bK, idA, 1);
           } else {
-            mma_bf16(tb + C::C_DQ, sdesc_sw128(adS) + 2 * kk, bK, idA, acc);
+            mma_bf16(tb + C::C_DQ, ddS + 2 * kk, bK, idA, acc);
           }
         }
         mma_commit(&st_empty[st]);

@@ -1,11 +1,11 @@
 """Fused dual attention on tcgen05 tensor cores (sequences of whole 128-token tiles) against
 the float64 oracle and against the warp-level fused kernels of the same library.
 
-MF_OPT_FLASH_ATTN 3 runs both forward kernels (S, S' into TMEM, P and P (*) S' through
-shared memory into the O and tangent products) on tcgen05, 1 (the default) the dual one; 4
-the dual forward and both backward kernels (scores and their tangents into TMEM, P^T, dS^T
-and tangents through shared memory into the dK, dV, dQ products); 2 keeps the warp-level
-kernels.  Cases span one to
+MF_OPT_FLASH_ATTN 1 (the default) runs the dual forward (S, S' into TMEM, P and P (*) S'
+through shared memory into the O and tangent products) and both backward kernels (scores
+and their tangents into TMEM, P^T, dS^T and tangents through shared memory into the dK, dV,
+dQ products) on tcgen05; 3 the primal forward as well; 4 the dual forward only; 2 keeps
+the warp-level kernels.  Cases span one to
 three 128-query tiles per head (the causal diagonal and off-diagonal key tiles), one to four
 heads, momentum with the scalar log-lr, both HVP modes, and attention scores spread far
 beyond the running-maximum bound (weights of scale 0.3), so that rows rescale their
@@ -77,7 +77,8 @@ def test_flash_tc_meta_grad(name, mode):
         assert abs(V - ref["V"]) <= 2e-2 * abs(ref["V"])
     # the two kernels differ only in summation order and bf16 rounding points
     assert rel_l2(dt_t, dt_w) < 1e-2, (name, rel_l2(dt_t, dt_w))
-    # 4 and 1 share the forward; their backward kernels differ in summation order only
+    # 4 and 1 share the forward; their backward kernels (warp-level, tcgen05) differ in
+    # summation order only
     assert V_b == V_d
     assert rel_l2(dt_b, dt_d) < 2e-3, (name, rel_l2(dt_b, dt_d))
     assert rel_l2(de_b, de_d) < 2e-3, (name, rel_l2(de_b, de_d))
