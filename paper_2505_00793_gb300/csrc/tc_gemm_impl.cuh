@@ -355,19 +355,32 @@ __device__ __forceinline__ int stg_quad(int r, int c) {
   return (r >> 1) * 128 + ((((r & 1) << 2) | (c ^ ((r >> 1) & 3))) << 4);
 }
 
-// Rows row0 .. row0 + 31 (those below M) of a float32 matrix, 16 columns from col0 (16-byte
-// aligned rows), into this lane's row: out[j] = src[(row0 + lane) * ld + col0 + j].
-__device__ __forceinline__ void warp_load_rows16(uint8_t* stg, int lane, int row0, int M,
-                                                 const float* src, int64_t ld, int col0,
-                                                 float (&out)[16]) {
+// A 32-row x 16-column float32 block read by quads (lane l: quad l % 4 of rows l / 4 + 8 i),
+// in flight until zrows_finish turns it into rows.
+struct ZRows {
+  float4 q[4];
+};
+
+// Issue the loads of rows row0 .. row0 + 31 (those below M) of a float32 matrix, 16 columns
+// from col0 (16-byte aligned rows).
+__device__ __forceinline__ void zrows_issue(ZRows& z, int lane, int row0, int M, const float* src,
+                                            int64_t ld, int col0) {
   const int rq = lane >> 2, cq = lane & 3;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     const int r = rq + 8 * i;
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (row0 + r < M) v = *reinterpret_cast<const float4*>(src + (row0 + r) * ld + col0 + 4 * cq);
-    *reinterpret_cast<float4*>(stg + stg_quad(r, cq)) = v;
+    z.q[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (row0 + r < M) z.q[i] = *reinterpret_cast<const float4*>(src + (row0 + r) * ld + col0 + 4 * cq);
   }
+}
+
+// ... and transpose them through the warp's buffer into this lane's row:
+// out[j] = src[(row0 + lane) * ld + col0 + j].
+__device__ __forceinline__ void zrows_finish(uint8_t* stg, int lane, const ZRows& z,
+                                             float (&out)[16]) {
+  const int rq = lane >> 2, cq = lane & 3;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) *reinterpret_cast<float4*>(stg + stg_quad(rq + 8 * i, cq)) = z.q[i];
   __syncwarp();
 #pragma unroll
   for (int c = 0; c < 4; ++c) {
@@ -375,6 +388,14 @@ __device__ __forceinline__ void warp_load_rows16(uint8_t* stg, int lane, int row
     out[4 * c] = v.x; out[4 * c + 1] = v.y; out[4 * c + 2] = v.z; out[4 * c + 3] = v.w;
   }
   __syncwarp();
+}
+
+__device__ __forceinline__ void warp_load_rows16(uint8_t* stg, int lane, int row0, int M,
+                                                 const float* src, int64_t ld, int col0,
+                                                 float (&out)[16]) {
+  ZRows z;
+  zrows_issue(z, lane, row0, M, src, ld, col0);
+  zrows_finish(stg, lane, z, out);
 }
 
 // This lane's 64-byte row (quads q[0..3]) of a 32-row block, stored by quads: quad c of
@@ -424,12 +445,14 @@ __device__ __forceinline__ bool rows16_ok(const TcParams& p, int mode, bool dual
 }
 
 // epilogue16 for a full chunk (col0 + 16 <= N) of the warp's 32 rows row0 .. row0 + 31, with
-// the stored pre-activations read and the outputs written through the per-warp buffer stg
-// (STG_ROWS_BYTES).  The arithmetic per element is epi_core_t, as in epilogue16.
+// the outputs written through the per-warp buffer stg (STG_ROWS_BYTES).  Backward
+// epilogues take the chunk's stored pre-activations as loads already issued (zq, zdq: see
+// zrows_issue).  The arithmetic per element is epi_core_t, as in epilogue16.
 template <int MODE, int ACT>
 __device__ __forceinline__ void epilogue16_rows(const TcParams& p, uint8_t* stg, int lane,
                                                 int row0, int col0, const float (&v0)[16],
-                                                const float (&v1)[16], bool dual) {
+                                                const float (&v1)[16], bool dual,
+                                                const ZRows& zq, const ZRows& zdq) {
   const EpiParams e = p.epi;
   const int row = row0 + lane;
   const bool rowok = row < p.M;
@@ -437,8 +460,8 @@ __device__ __forceinline__ void epilogue16_rows(const TcParams& p, uint8_t* stg,
 #pragma unroll
   for (int j = 0; j < 16; ++j) z[j] = zd[j] = 0.f;
   if constexpr (MODE == EPI_ACT_BWD) {
-    warp_load_rows16(stg, lane, row0, p.M, e.Z, e.ldz, col0, z);
-    if (dual) warp_load_rows16(stg, lane, row0, p.M, e.Zd, e.ldz, col0, zd);
+    zrows_finish(stg, lane, zq, z);
+    if (dual) zrows_finish(stg, lane, zdq, zd);
   }
   float c0[16], c1[16], o0[16], o1[16];
 #pragma unroll

@@ -404,8 +404,23 @@ __global__ void __launch_bounds__(THREADS_P, 1)
       p.C0 = C0base ? C0base + bz * p.bsC0 : nullptr;
       p.C1 = C1base ? C1base + bz * p.bsC1 : nullptr;
       const uint32_t taddr = tbase + lane_off + static_cast<uint32_t>(set * pp.set_cols);
+      // backward epilogues: the next full chunk's stored pre-activations load while this
+      // chunk is computed
+      ZRows zq, zdq, zq_n, zdq_n;
+      auto zissue = [&](int c, ZRows& a, ZRows& b) {
+        if (rows_ok && n0 + c + 16 <= p.N) {
+          zrows_issue(a, lane, m0 + q * 32, p.M, p.epi.Z, p.epi.ldz, n0 + c);
+          if (dual) zrows_issue(b, lane, m0 + q * 32, p.M, p.epi.Zd, p.epi.ldz, n0 + c);
+        }
+      };
+      if constexpr (MODE == EPI_ACT_BWD) zissue(c_begin, zq_n, zdq_n);
 #pragma unroll 1
       for (int c = c_begin; c < c_end; c += 16) {
+        if constexpr (MODE == EPI_ACT_BWD) {
+          zq = zq_n;
+          zdq = zdq_n;
+          if (c + 16 < c_end) zissue(c + 16, zq_n, zdq_n);
+        }
         float v0[16], v1[16];
         ld_acc16<BN>(taddr, 0, p.nsub, c, v0);
         if (dual) ld_acc16<BN>(taddr, 1, p.nsub, c, v1);
@@ -414,7 +429,7 @@ __global__ void __launch_bounds__(THREADS_P, 1)
           for (int i = 0; i < 16; ++i) v1[i] = 0.f;
         }
         if (rows_ok && n0 + c + 16 <= p.N)
-          epilogue16_rows<MODE, ACT>(p, stg, lane, m0 + q * 32, n0 + c, v0, v1, dual);
+          epilogue16_rows<MODE, ACT>(p, stg, lane, m0 + q * 32, n0 + c, v0, v1, dual, zq, zdq);
         else if (n0 + c < p.N)
           epilogue16<MODE, ACT>(p, m0 + r, n0 + c, v0, v1, dual);
       }
