@@ -448,11 +448,12 @@ __device__ __forceinline__ bool rows16_ok(const TcParams& p, int mode, bool dual
 // the outputs written through the per-warp buffer stg (STG_ROWS_BYTES).  Backward
 // epilogues take the chunk's stored pre-activations as loads already issued (zq, zdq: see
 // zrows_issue).  The arithmetic per element is epi_core_t, as in epilogue16.
-template <int MODE, int ACT>
-__device__ __forceinline__ void epilogue16_rows(const TcParams& p, uint8_t* stg, int lane,
-                                                int row0, int col0, const float (&v0)[16],
-                                                const float (&v1)[16], bool dual,
-                                                const ZRows& zq, const ZRows& zdq) {
+template <int MODE, int ACT, bool DUALE>
+__device__ __forceinline__ void epilogue16_rows_t(const TcParams& p, uint8_t* stg, int lane,
+                                                  int row0, int col0, const float (&v0)[16],
+                                                  const float (&v1)[16], const ZRows& zq,
+                                                  const ZRows& zdq) {
+  constexpr bool dual = DUALE;
   const EpiParams e = p.epi;
   const int row = row0 + lane;
   const bool rowok = row < p.M;
@@ -506,6 +507,17 @@ __device__ __forceinline__ void epilogue16_rows(const TcParams& p, uint8_t* stg,
       });
     }
   }
+}
+
+// The same with the dual flag as a compile-time constant, so that single-accumulator
+// epilogues carry no tangent arithmetic.
+template <int MODE, int ACT>
+__device__ __forceinline__ void epilogue16_rows(const TcParams& p, uint8_t* stg, int lane,
+                                                int row0, int col0, const float (&v0)[16],
+                                                const float (&v1)[16], bool dual,
+                                                const ZRows& zq, const ZRows& zdq) {
+  if (dual) epilogue16_rows_t<MODE, ACT, true>(p, stg, lane, row0, col0, v0, v1, zq, zdq);
+  else epilogue16_rows_t<MODE, ACT, false>(p, stg, lane, row0, col0, v0, v1, zq, zdq);
 }
 
 __device__ __forceinline__ void fence_proxy_async() {
