@@ -447,47 +447,66 @@ __device__ __forceinline__ bool rows16_ok(const TcParams& p, int mode, bool dual
 // epilogue16 for a full chunk (col0 + 16 <= N) of the warp's 32 rows row0 .. row0 + 31, with
 // the outputs written through the per-warp buffer stg (STG_ROWS_BYTES).  Backward
 // epilogues take the chunk's stored pre-activations as loads already issued (zq, zdq: see
-// zrows_issue).  The arithmetic per element is epi_core_t, as in epilogue16.
+// zrows_issue).  The arithmetic per element is epi_core_t's, as in epilogue16, computed in
+// place (v0, v1 become the float32 outputs) with the activation outputs packed to bf16 pairs
+// at once, so that few values stay live.  Rows at or past M are computed but not stored.
 template <int MODE, int ACT, bool DUALE>
 __device__ __forceinline__ void epilogue16_rows_t(const TcParams& p, uint8_t* stg, int lane,
-                                                  int row0, int col0, const float (&v0)[16],
-                                                  const float (&v1)[16], const ZRows& zq,
+                                                  int row0, int col0, float (&v0)[16],
+                                                  float (&v1)[16], const ZRows& zq,
                                                   const ZRows& zdq) {
   constexpr bool dual = DUALE;
   const EpiParams e = p.epi;
-  const int row = row0 + lane;
-  const bool rowok = row < p.M;
-  float z[16], zd[16];
-#pragma unroll
-  for (int j = 0; j < 16; ++j) z[j] = zd[j] = 0.f;
+  uint32_t pa[8], pad[8];       // bf16 pairs of A and Ad
   if constexpr (MODE == EPI_ACT_BWD) {
+    float z[16];
     zrows_finish(stg, lane, zq, z);
-    if (dual) zrows_finish(stg, lane, zdq, zd);
-  }
-  float c0[16], c1[16], o0[16], o1[16];
+    float zd[16];
+    if constexpr (dual) zrows_finish(stg, lane, zdq, zd);
 #pragma unroll
-  for (int j = 0; j < 16; ++j) {
-    const int n = col0 + j;
-    EpiOut o;
-    if (rowok) {
-      const float b0 = MODE != EPI_ACT_BWD && p.bias0 ? p.bias0[n] : 0.f;
-      const float b1 = MODE != EPI_ACT_BWD && p.bias1 ? p.bias1[n] : 0.f;
-      o = epi_core_t<MODE, ACT>(v0[j], v1[j], z[j], zd[j], b0, b1, dual);
-    } else {
-      o.c0 = o.c1 = o.o0 = o.o1 = 0.f;
+    for (int j = 0; j < 16; j += 2) {
+      float o0[2], o1[2];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const EpiOut o = epi_core_t<MODE, ACT>(v0[j + h], v1[j + h], z[j + h],
+                                               dual ? zd[j + h] : 0.f, 0.f, 0.f, dual);
+        o0[h] = o.o0;
+        o1[h] = o.o1;
+      }
+      pa[j / 2] = pack_bf16x2(o0[0], o0[1]);
+      pad[j / 2] = pack_bf16x2(o1[0], o1[1]);
     }
-    c0[j] = o.c0; c1[j] = o.c1; o0[j] = o.o0; o1[j] = o.o1;
+  } else {
+#pragma unroll
+    for (int j = 0; j < 16; j += 2) {
+      float o0[2], o1[2];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int n = col0 + j + h;
+        const float b0 = p.bias0 ? p.bias0[n] : 0.f;
+        const float b1 = p.bias1 ? p.bias1[n] : 0.f;
+        const EpiOut o = epi_core_t<MODE, ACT>(v0[j + h], v1[j + h], 0.f, 0.f, b0, b1, dual);
+        v0[j + h] = o.c0;
+        v1[j + h] = o.c1;
+        o0[h] = o.o0;
+        o1[h] = o.o1;
+      }
+      if constexpr (MODE != EPI_STORE) {
+        pa[j / 2] = pack_bf16x2(o0[0], o0[1]);
+        pad[j / 2] = pack_bf16x2(o1[0], o1[1]);
+      }
+    }
   }
   if (p.C0) {
-    const uint4 q[4] = {quad_f32(c0), quad_f32(c0 + 4), quad_f32(c0 + 8), quad_f32(c0 + 12)};
+    const uint4 q[4] = {quad_f32(v0), quad_f32(v0 + 4), quad_f32(v0 + 8), quad_f32(v0 + 12)};
     float* const C = p.C0;
     const int64_t ld = p.ldc0;
     warp_store_rows(stg, lane, row0, p.M, q, [&](int r, int c) -> void* {
       return C + (row0 + r) * ld + col0 + 4 * c;
     });
   }
-  if (p.C1 && dual) {
-    const uint4 q[4] = {quad_f32(c1), quad_f32(c1 + 4), quad_f32(c1 + 8), quad_f32(c1 + 12)};
+  if (dual && p.C1) {
+    const uint4 q[4] = {quad_f32(v1), quad_f32(v1 + 4), quad_f32(v1 + 8), quad_f32(v1 + 12)};
     float* const C = p.C1;
     const int64_t ld = p.ldc1;
     warp_store_rows(stg, lane, row0, p.M, q, [&](int r, int c) -> void* {
@@ -499,7 +518,10 @@ __device__ __forceinline__ void epilogue16_rows_t(const TcParams& p, uint8_t* st
     __nv_bfloat16* const A = static_cast<__nv_bfloat16*>(e.A);
     __nv_bfloat16* const Ad = dual ? static_cast<__nv_bfloat16*>(e.Ad) : nullptr;
     if (A || Ad) {
-      const uint4 q[4] = {quad_bf16(o0), quad_bf16(o0 + 8), quad_bf16(o1), quad_bf16(o1 + 8)};
+      const uint4 q[4] = {make_uint4(pa[0], pa[1], pa[2], pa[3]),
+                          make_uint4(pa[4], pa[5], pa[6], pa[7]),
+                          make_uint4(pad[0], pad[1], pad[2], pad[3]),
+                          make_uint4(pad[4], pad[5], pad[6], pad[7])};
       const int64_t ld = e.lda;
       warp_store_rows(stg, lane, row0, p.M, q, [&](int r, int c) -> void* {
         __nv_bfloat16* X = c < 2 ? A : Ad;
@@ -513,8 +535,8 @@ __device__ __forceinline__ void epilogue16_rows_t(const TcParams& p, uint8_t* st
 // epilogues carry no tangent arithmetic.
 template <int MODE, int ACT>
 __device__ __forceinline__ void epilogue16_rows(const TcParams& p, uint8_t* stg, int lane,
-                                                int row0, int col0, const float (&v0)[16],
-                                                const float (&v1)[16], bool dual,
+                                                int row0, int col0, float (&v0)[16],
+                                                float (&v1)[16], bool dual,
                                                 const ZRows& zq, const ZRows& zdq) {
   if (dual) epilogue16_rows_t<MODE, ACT, true>(p, stg, lane, row0, col0, v0, v1, zq, zdq);
   else epilogue16_rows_t<MODE, ACT, false>(p, stg, lane, row0, col0, v0, v1, zq, zdq);

@@ -13,7 +13,7 @@
 //
 // Roles per CTA (as in the one-tile pair kernel): warp 0 issues the TMA loads of this CTA's
 // 128 rows of A and BN/2 rows of B; warp 1 owns TMEM, and in the even CTA one thread issues
-// tcgen05.mma.cta_group::2 (M = 256) for the pair; EPI_WARPS_P warps drain this CTA's 128
+// tcgen05.mma.cta_group::2 (M = 256) for the pair; epi_warps_p warps drain this CTA's 128
 // accumulator rows, one TMEM lane quadrant and one column share per warp; full 16-column
 // chunks are stored through a 2 KB row-block buffer per warp (8 rows x 64 bytes per warp
 // store, see epilogue16_rows), ragged ones straight from registers.
@@ -32,9 +32,13 @@ int g_gemm_persist = 2;
 
 namespace {
 
-constexpr int EPI_WARPS_P = 8;
-constexpr int EPI_GROUPS_P = EPI_WARPS_P / 4;
-constexpr int THREADS_P = 64 + 32 * EPI_WARPS_P;
+// Epilogue warps per CTA: twelve (three per TMEM lane quadrant) where the epilogue is the
+// longer role, eight for the backward epilogues, whose prefetched pre-activations need the
+// registers of a 320-thread CTA.
+template <int MODE>
+__host__ __device__ constexpr int epi_warps_p() { return MODE == EPI_ACT_BWD ? 8 : 12; }
+template <int MODE>
+__host__ __device__ constexpr int threads_p() { return 64 + 32 * epi_warps_p<MODE>(); }
 
 // Accumulator blocks per logical accumulator (the rotation of mma_loop) when two sets of
 // `nacc` accumulators must fit TMEM, else the one-set figure of the one-tile kernels.
@@ -223,7 +227,7 @@ __device__ __forceinline__ bool mma_tile_dispatch(const MmaLoop& L, IssueRing& R
 }
 
 template <int BN, int MODE, int ACT>
-__global__ void __launch_bounds__(THREADS_P, 1)
+__global__ void __launch_bounds__(threads_p<MODE>(), 1)
     tc2p_dual_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
                           const __grid_constant__ CUtensorMap tmA1,
                           const __grid_constant__ CUtensorMap tmB0,
@@ -261,7 +265,7 @@ __global__ void __launch_bounds__(THREADS_P, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], 2 * EPI_WARPS_P);
+      mbar_init(&acc_empty[b], 2 * epi_warps_p<MODE>());
     }
     mbar_init(&drain_bar, 1);
     abort_flag = 0;
@@ -384,8 +388,9 @@ __global__ void __launch_bounds__(THREADS_P, 1)
     const int q = warp & 3;
     const int r = q * 32 + lane;
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
-    constexpr int CG = BN / EPI_GROUPS_P;
-    const int c_begin = ((warp - 2) >> 2) * CG, c_end = c_begin + CG;
+    // the quadrant's epi_warps_p / 4 warps take its 16-column chunks in turn
+    constexpr int CSTEP = 16 * (epi_warps_p<MODE>() / 4);
+    const int c_begin = ((warp - 2) >> 2) * 16, c_end = BN;
     const uint32_t empty0 = dsmem_addr(smem_u32(&acc_empty[0]), 0);   // even CTA's barriers
     // full chunks go through this warp's row-block buffer behind the pipeline stages
     uint8_t* const stg = smem + p.stages * p.stage_bytes + (warp - 2) * STG_ROWS_BYTES;
@@ -415,11 +420,11 @@ __global__ void __launch_bounds__(THREADS_P, 1)
       };
       if constexpr (MODE == EPI_ACT_BWD) zissue(c_begin, zq_n, zdq_n);
 #pragma unroll 1
-      for (int c = c_begin; c < c_end; c += 16) {
+      for (int c = c_begin; c < c_end; c += CSTEP) {
         if constexpr (MODE == EPI_ACT_BWD) {
           zq = zq_n;
           zdq = zdq_n;
-          if (c + 16 < c_end) zissue(c + 16, zq_n, zdq_n);
+          if (c + CSTEP < c_end) zissue(c + CSTEP, zq_n, zdq_n);
         }
         float v0[16], v1[16];
         ld_acc16<BN>(taddr, 0, p.nsub, c, v0);
@@ -460,7 +465,7 @@ int max_pairs_on_device(int smem) {
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof(cfg));
   cfg.gridDim = dim3(2 * (pairs > 0 ? pairs : 1), 1, 1);
-  cfg.blockDim = dim3(THREADS_P, 1, 1);
+  cfg.blockDim = dim3(threads_p<MODE>(), 1, 1);
   cfg.dynamicSmemBytes = smem;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -514,7 +519,7 @@ cudaError_t launch_cfg2p(const GemmArgs& a, cudaStream_t s, const char** why) {
   p.tx_bytes = off;
   p.nsub = persist_nsub(nacc, BN);
   // pipeline stages, then one row-block buffer per epilogue warp
-  int stages = (220 * 1024 - EPI_WARPS_P * STG_ROWS_BYTES) / off;
+  int stages = (220 * 1024 - epi_warps_p<MODE>() * STG_ROWS_BYTES) / off;
   if (stages > MAX_STAGES) stages = MAX_STAGES;
   if (stages < 2) { *why = "tile does not fit shared memory"; return cudaErrorInvalidValue; }
   p.stages = stages;
@@ -552,7 +557,7 @@ cudaError_t launch_cfg2p(const GemmArgs& a, cudaStream_t s, const char** why) {
   pp.nsets = persist_sets(nacc, BN);
   pp.set_cols = nacc * p.nsub * BN;
 
-  const int smem = stages * off + EPI_WARPS_P * STG_ROWS_BYTES + 1024;
+  const int smem = stages * off + epi_warps_p<MODE>() * STG_ROWS_BYTES + 1024;
   static PerDeviceOnce attr_once;
   {
     cudaError_t e = attr_once.run([](int&) {
@@ -567,7 +572,7 @@ cudaError_t launch_cfg2p(const GemmArgs& a, cudaStream_t s, const char** why) {
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof(cfg));
   cfg.gridDim = dim3(2 * npairs, 1, 1);
-  cfg.blockDim = dim3(THREADS_P, 1, 1);
+  cfg.blockDim = dim3(threads_p<MODE>(), 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
