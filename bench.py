@@ -599,7 +599,7 @@ def main():
                     help="segment length of the theta_t store (1 = keep every theta_t)")
     ap.add_argument("--gemm-persistent", type=int, nargs="?", const=1, default=None,
                     help="MF_OPT_GEMM_PERSISTENT mode (0 off; 1 all, duals 128-wide; 2 as 1 "
-                         "but duals with K > 2048 on the one-tile kernel, the library default; "
+                         "but duals with K > 2048 256-wide, the library default; "
                          "3 all, duals 256-wide)")
     ap.add_argument("--flash-attn", type=int, default=None, choices=[0, 1, 2, 3, 4],
                     help="MF_OPT_FLASH_ATTN (library default 1)")

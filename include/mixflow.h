@@ -309,10 +309,10 @@ mf_status mf_replay_gemms(mf_handle h, int reps, void* stream, double* ms, uint6
  * that the pairs running together share row blocks of A and a band of B), with two TMEM
  * accumulator sets when they fit so that a tile's epilogue overlaps the next tile's main
  * loop.  0 never; 1 every pair GEMM, dual products at 128-wide tiles (two sets of their two
- * accumulators fit); 2 as 1, except that dual products with K > 2048 keep the one-tile
- * kernel (its 256-wide dual tiles stage half the operand bytes per MMA, and their long main
- * loops hide its epilogue); 3 every pair GEMM, dual products at 256-wide tiles with one
- * accumulator set.  Same products and summation
+ * accumulators fit); 2 as 1, except that dual products with K > 2048 take 256-wide tiles
+ * with one accumulator set (half the operand bytes per MMA; their long main loops hide the
+ * epilogue that one set cannot overlap); 3 every pair GEMM, dual products at 256-wide tiles
+ * with one accumulator set.  Same products and summation
  * order within a tile as the one-tile form.  Setting it drops the handle's captured graphs.
  * MF_OPT_FUSED_HEAD (process-wide, default 0): 1 computes the output layer of an MLP with at
  * most 16 outputs and a squared or softmax cross-entropy loss in one kernel per pass: the

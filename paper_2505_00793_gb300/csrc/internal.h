@@ -108,9 +108,9 @@ extern int g_pair_mode;
 extern long long g_wait_ns;
 // Persistent CTA-pair form of the tcgen05 GEMM (tc_gemm_persist.cu), MF_OPT_GEMM_PERSISTENT:
 // g_gemm_persist 0 = off; 1 = every 2-SM GEMM, dual products at 128-wide tiles with two
-// TMEM accumulator sets; 2 (default) = as 1 except dual products with K > 2048, which keep
-// the one-tile kernel; 3 = every 2-SM GEMM, dual products at their 256-wide tiles with one
-// accumulator set.  bn is 128 or 256.
+// TMEM accumulator sets; 2 (default) = as 1 except dual products with K > 2048, which take
+// 256-wide tiles with one accumulator set; 3 = every 2-SM GEMM, dual products at their
+// 256-wide tiles with one accumulator set.  bn is 128 or 256.
 cudaError_t tc_gemm_persist(const GemmArgs& a, cudaStream_t s, const char** why, int bn);
 extern int g_gemm_persist;
 // SIMT float32 GEMM with the same semantics (simt_gemm.cu).

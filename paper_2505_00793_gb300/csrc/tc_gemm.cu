@@ -103,13 +103,7 @@ cudaError_t tc_gemm(const GemmArgs& a, cudaStream_t s, const char** why) {
     else bn = 256;
   }
   if (a.b_mn && bn < 64) bn = 64;   // MN-major B is staged in 64-row boxes
-  if (pair && g_gemm_persist) {
-    // mode 2 keeps dual products (two accumulators) with K above 2048 on the one-tile
-    // kernel: their 256-wide tiles stage half the operand bytes per MMA of the persistent
-    // form's 128-wide dual tiles, and a long main loop hides the one-tile epilogue
-    const bool dual = a.terms & (T_C1_A1B0 | T_C1_A0B1);
-    if (g_gemm_persist != 2 || !dual || a.K <= 2048) return tc_gemm_persist(a, s, why, bn);
-  }
+  if (pair && g_gemm_persist) return tc_gemm_persist(a, s, why, bn);
   if (a.epi.mode == EPI_STORE) return launch_bn<EPI_STORE, ACT_IDENT>(a, s, why, bn, pair);
   return tc_gemm_act(a, s, why, bn, pair);
 }

@@ -600,11 +600,13 @@ cudaError_t launch_bn_p(const GemmArgs& a, cudaStream_t s, const char** why, int
 
 cudaError_t tc_gemm_persist(const GemmArgs& a, cudaStream_t s, const char** why, int bn) {
   const int act = a.epi.act;
-  // Dual products take 128-wide tiles unless the caller fixed the width or mode 3 keeps
-  // them at 256: two sets of their two accumulators then fit TMEM, so epilogues overlap main
-  // loops.
-  if (bn == 256 && a.bn == 0 && g_gemm_persist != 3 && (a.terms & (T_C1_A1B0 | T_C1_A0B1)))
-    bn = 128;
+  // Dual products take 128-wide tiles, whose two accumulators fit TMEM twice, so that
+  // epilogues overlap main loops; unless the caller fixed the width, mode 3 keeps them at
+  // 256, and so does mode 2 for K > 2048, where the 256-wide tiles' halved operand bytes per
+  // MMA outweigh the epilogue that a single accumulator set cannot overlap.
+  const bool dual = a.terms & (T_C1_A1B0 | T_C1_A0B1);
+  const bool wide = g_gemm_persist == 3 || (g_gemm_persist == 2 && a.K > 2048);
+  if (bn == 256 && a.bn == 0 && dual && !wide) bn = 128;
   if (a.epi.mode == EPI_STORE) return launch_bn_p<EPI_STORE, ACT_IDENT>(a, s, why, bn);
   if (a.epi.mode == EPI_ACT_FWD) {
     switch (act) {
