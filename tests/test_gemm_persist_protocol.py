@@ -151,7 +151,7 @@ def _configs(n):
         npairs = rnd.randint(1, 4)
         yield dict(ntiles=rnd.randint(1, 12), pair=rnd.randrange(npairs), npairs=npairs,
                    nk=rnd.randint(1, 7), stages=rnd.randint(2, 6), nsets=rnd.choice([1, 2]),
-                   epi_warps=rnd.choice([1, 2, 8]), seed=seed)
+                   epi_warps=rnd.choice([1, 2, 8, 12]), seed=seed)
 
 
 def test_protocol_completes_every_tile():
@@ -182,19 +182,21 @@ def test_model_catches_planted_mistakes(mistake):
 
 
 # ---- index arithmetic of the persistent kernel ---------------------------------------------
-EPI_WARPS_P, BM, BK = 8, 128, 64
+BM, BK = 128, 64
 
 
-def _persist_coverage(M, N, BN, batch, npairs):
+def _persist_coverage(M, N, BN, batch, npairs, epi_warps=12):
     """Every output element written by the kernel's epilogue mapping, and the TMA boxes each
-    CTA loads, for one launch (the kernel's formulas restated)."""
+    CTA loads, for one launch (the kernel's formulas restated).  epi_warps epilogue warps
+    (8 for the backward epilogues, 12 otherwise): epi_warps / 4 per TMEM lane quadrant,
+    taking the quadrant's 16-column chunks in turn."""
     tiles_n = -(-N // BN)
     pairs_m = -(-M // (2 * BM))
     ntiles = tiles_n * pairs_m * batch
     BH = BN // 2
     written = np.zeros((batch, M, N), np.int32)
     a_rows, b_rows = set(), set()
-    CG = BN // (EPI_WARPS_P // 4)
+    groups = epi_warps // 4
     for pair in range(npairs):
         for t in range(pair, ntiles, npairs):
             # grouped order of the kernel: groups of up to 8 row blocks, rows fastest
@@ -208,12 +210,12 @@ def _persist_coverage(M, N, BN, batch, npairs):
                 a_rows.add((bz, m0))
                 b_rows.add((bz, tn * BN + rank * BH))
                 n0 = tn * BN
-                for warp in range(2, 2 + EPI_WARPS_P):
+                for warp in range(2, 2 + epi_warps):
                     q = warp & 3
-                    c_begin = ((warp - 2) >> 2) * CG
+                    c_begin = ((warp - 2) >> 2) * 16
                     for lane in range(32):
                         row = m0 + q * 32 + lane
-                        for c in range(c_begin, c_begin + CG, 16):
+                        for c in range(c_begin, BN, 16 * groups):
                             if n0 + c >= N or row >= M:
                                 continue
                             cols = [n0 + c + j for j in range(16) if n0 + c + j < N]
@@ -221,12 +223,14 @@ def _persist_coverage(M, N, BN, batch, npairs):
     return written, a_rows, b_rows, pairs_m, tiles_n
 
 
+@pytest.mark.parametrize("epi_warps", [8, 12])
 @pytest.mark.parametrize("M,N,BN,batch,npairs", [
     (256, 128, 128, 1, 1), (300, 520, 128, 1, 3), (1000, 130, 256, 1, 76),
     (1025, 1024, 256, 1, 7), (600, 1000, 128, 3, 5), (2048, 1024, 128, 1, 76),
     (2900, 520, 128, 2, 9)])
-def test_persistent_tiles_cover_every_output_once(M, N, BN, batch, npairs):
-    written, a_rows, b_rows, pairs_m, tiles_n = _persist_coverage(M, N, BN, batch, npairs)
+def test_persistent_tiles_cover_every_output_once(M, N, BN, batch, npairs, epi_warps):
+    written, a_rows, b_rows, pairs_m, tiles_n = _persist_coverage(M, N, BN, batch, npairs,
+                                                                  epi_warps)
     assert (written == 1).all()
     # A boxes: 128 rows per CTA from every 256-row block; B boxes: BN/2 rows per CTA
     assert {m for _, m in a_rows} == {mp * 2 * BM + r * BM for mp in range(pairs_m) for r in (0, 1)}
