@@ -796,6 +796,8 @@ __global__ void token_order_kernel(const int* __restrict__ start, const int* __r
 // (Zipf-distributed ids give a few very long segments).  A warp sums every column of a row
 // at once (up to 1024 columns: eight float4 loads per lane in flight), then the warps'
 // partial sums are added in warp order, so the result is deterministic.
+constexpr int EB_SLICE = 256;
+
 __global__ void __launch_bounds__(256) embed_bwd_kernel(int d, const int* __restrict__ start,
                                                         const int* __restrict__ order,
                                                         const float* __restrict__ dx,
@@ -803,15 +805,19 @@ __global__ void __launch_bounds__(256) embed_bwd_kernel(int d, const int* __rest
                                                         float* __restrict__ dE,
                                                         float* __restrict__ dEd, bool vec_out) {
   pdl_entry();
-  constexpr int NC = 8;                 // 128-column chunks per pass
+  // blockIdx.y picks a slice of EB_SLICE columns, so that the rows of a frequent token
+  // (Zipf-distributed ids put hundreds of a batch's tokens on one row) are summed by several
+  // blocks at once
+  constexpr int NC = EB_SLICE / 128;    // 128-column chunks per pass
   __shared__ float4 part[2][8][32];
   const int v = blockIdx.x;
+  const int cs0 = blockIdx.y * EB_SLICE, cs1 = min(d, cs0 + EB_SLICE);
   const int a = start[v], cnt = start[v + 1] - a;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r0 = a + (w * cnt) / 8, r1 = a + ((w + 1) * cnt) / 8;
   const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
   if (cnt == 0) {   // an id absent from the batch (most of a large vocabulary): zero rows
-    for (int c = threadIdx.x * 4; c < d; c += 256 * 4) {
+    for (int c = cs0 + threadIdx.x * 4; c < cs1; c += 256 * 4) {
       for (int which = 0; which < 2; ++which) {
         float* out = which == 0 ? dE : dEd;
         if (!out) continue;
@@ -822,7 +828,7 @@ __global__ void __launch_bounds__(256) embed_bwd_kernel(int d, const int* __rest
     }
     return;
   }
-  for (int g0 = 0; g0 < d; g0 += NC * 128) {
+  for (int g0 = cs0; g0 < cs1; g0 += NC * 128) {
     float4 acc[NC], dacc[NC];
 #pragma unroll
     for (int q = 0; q < NC; ++q) { acc[q] = zero; dacc[q] = zero; }
@@ -837,7 +843,7 @@ __global__ void __launch_bounds__(256) embed_bwd_kernel(int d, const int* __rest
 #pragma unroll
         for (int q = 0; q < NC; ++q) {
           const int c = g0 + q * 128 + lane * 4;
-          if (c < d) {
+          if (c < cs1) {
             const float4 x = *reinterpret_cast<const float4*>(dx + ro + c);
             acc[q].x += x.x; acc[q].y += x.y; acc[q].z += x.z; acc[q].w += x.w;
             if (dxd) {
@@ -851,7 +857,7 @@ __global__ void __launch_bounds__(256) embed_bwd_kernel(int d, const int* __rest
 #pragma unroll
     for (int q = 0; q < NC; ++q) {
       const int c0 = g0 + q * 128;
-      if (c0 >= d) break;          // uniform across the block
+      if (c0 >= cs1) break;        // uniform across the block
       part[0][w][lane] = acc[q];
       part[1][w][lane] = dacc[q];
       __syncthreads();
@@ -863,7 +869,7 @@ __global__ void __launch_bounds__(256) embed_bwd_kernel(int d, const int* __rest
           t.x += u.x; t.y += u.y; t.z += u.z; t.w += u.w;
         }
         float* out = which == 0 ? dE : dEd;
-        if (out && cc < d) {
+        if (out && cc < cs1) {
           float* dst = out + static_cast<int64_t>(v) * d + cc;
           if (vec_out) {
             *reinterpret_cast<float4*>(dst) = t;
@@ -1026,7 +1032,8 @@ void dec_token_csr(int N, int S, int V, const int* ids, int* count, int* start, 
 void dec_embed_bwd(int V, int d, const int* start, const int* order, const float* dx,
                    const float* dxd, float* dE, float* dEd, cudaStream_t s) {
   const bool vec_out = ((reinterpret_cast<uintptr_t>(dE) | reinterpret_cast<uintptr_t>(dEd)) & 15) == 0;
-  launch_k(embed_bwd_kernel, dim3(V), dim3(256), 0, s, d, start, order, dx, dxd, dE, dEd, vec_out);
+  launch_k(embed_bwd_kernel, dim3(V, (d + EB_SLICE - 1) / EB_SLICE), dim3(256), 0, s, d, start,
+           order, dx, dxd, dE, dEd, vec_out);
 }
 
 template <typename T>

@@ -583,36 +583,48 @@ __global__ void __launch_bounds__(FTHREADS) flash_bwd_q_kernel(const FlashArgs a
 
 // D = rowsum(dO (*) O) and D' = rowsum(dO' (*) O + dO (*) O') per (token, head), from the
 // float32 head-merged output gradients [N][ld] and the bf16 merged attention outputs; the
-// same pass writes dO (dO') as bf16 per head ([B*H][S][64]) for the backward kernels.  One
-// warp per (token, head), two adjacent columns per lane (8-byte loads, 4-byte stores).
+// same pass writes dO (dO') as bf16 per head ([B*H][S][64]) for the backward kernels.  Two
+// (token, head) rows per warp, four adjacent columns per lane (16-byte loads of dO).
 __global__ void flash_prep_kernel(int N, int S, int H, const float* __restrict__ dO,
                                   const float* __restrict__ dOd, const bf16* __restrict__ O,
                                   const bf16* __restrict__ Od, int ld, float* __restrict__ D,
                                   float* __restrict__ Dd, bf16* __restrict__ dOh,
                                   bf16* __restrict__ dOhd) {
   pdl_entry();
-  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
-  if (warp >= N * H) return;
-  const int n = warp / H, hh = warp % H;
-  const int64_t base = static_cast<int64_t>(n) * ld + hh * FDH + 2 * lane;
+  // two (token, head) rows per warp, 16 lanes of four columns each
+  const int lane = threadIdx.x & 31;
+  const int row = ((blockIdx.x * blockDim.x + threadIdx.x) >> 5) * 2 + (lane >> 4);
+  const int c = (lane & 15) * 4;
+  const bool ok = row < N * H;
+  const int n = ok ? row / H : 0, hh = ok ? row % H : 0;
+  const int64_t base = static_cast<int64_t>(n) * ld + hh * FDH + c;
   const int b = n / S, sidx = n % S;
   const int64_t i = (static_cast<int64_t>(b) * H + hh) * S + sidx;
-  const float2 g = *reinterpret_cast<const float2*>(dO + base);
-  const float2 o = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(O + base));
-  float d = g.x * o.x + g.y * o.y, dd = 0.f;
-  if (dOh) *reinterpret_cast<uint32_t*>(dOh + i * FDH + 2 * lane) = pack(g.x, g.y);
-  if (Dd) {
-    const float2 gd = *reinterpret_cast<const float2*>(dOd + base);
-    const float2 od = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(Od + base));
-    dd = gd.x * o.x + gd.y * o.y + g.x * od.x + g.y * od.y;
-    if (dOhd) *reinterpret_cast<uint32_t*>(dOhd + i * FDH + 2 * lane) = pack(gd.x, gd.y);
+  float d = 0.f, dd = 0.f;
+  if (ok) {
+    const float4 g = *reinterpret_cast<const float4*>(dO + base);
+    const uint2 ob = *reinterpret_cast<const uint2*>(O + base);
+    const float2 o01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ob.x));
+    const float2 o23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&ob.y));
+    d = g.x * o01.x + g.y * o01.y + g.z * o23.x + g.w * o23.y;
+    if (dOh) *reinterpret_cast<uint2*>(dOh + i * FDH + c) = make_uint2(pack(g.x, g.y), pack(g.z, g.w));
+    if (Dd) {
+      const float4 gd = *reinterpret_cast<const float4*>(dOd + base);
+      const uint2 odb = *reinterpret_cast<const uint2*>(Od + base);
+      const float2 od01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&odb.x));
+      const float2 od23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&odb.y));
+      dd = gd.x * o01.x + gd.y * o01.y + gd.z * o23.x + gd.w * o23.y + g.x * od01.x +
+           g.y * od01.y + g.z * od23.x + g.w * od23.y;
+      if (dOhd)
+        *reinterpret_cast<uint2*>(dOhd + i * FDH + c) = make_uint2(pack(gd.x, gd.y), pack(gd.z, gd.w));
+    }
   }
 #pragma unroll
-  for (int s = 16; s > 0; s >>= 1) {
+  for (int s = 8; s > 0; s >>= 1) {
     d += __shfl_xor_sync(0xffffffffu, d, s);
     dd += __shfl_xor_sync(0xffffffffu, dd, s);
   }
-  if (lane == 0) {
+  if (ok && (lane & 15) == 0) {
     D[i] = d;
     if (Dd) Dd[i] = dd;
   }
@@ -676,7 +688,7 @@ void flash_bwd(const FlashArgs& a, bool dual, cudaStream_t s) {
 void flash_prep(int N, int S, int H, const float* dO, const float* dOd, const void* O,
                 const void* Od, int ld, float* D, float* Dd, void* dOh, void* dOhd,
                 cudaStream_t s) {
-  const int warps = N * H;
+  const int warps = (N * H + 1) / 2;
   const int threads = 256;
   const int blocks = (warps * 32 + threads - 1) / threads;
   launch_k(flash_prep_kernel, dim3(blocks), dim3(threads), 0, s, N, S, H, dO, dOd,
