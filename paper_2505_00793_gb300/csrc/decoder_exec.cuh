@@ -645,6 +645,7 @@ struct DecExec {
           launched();
         }
       }
+      bool merged = false;   // the attention backward writes dqkv itself (no RoPE merge)
       if (p.flash) {
         // fused backward of the attention and its tangent, from D = rowsum(dO O) (and D')
         float* D = at<float>(p.fD);
@@ -660,6 +661,19 @@ struct DecExec {
         fa.Dd = dual ? Dd : nullptr;
         fa.dQ = at<float>(p.dQ); fa.dK = at<float>(p.dK); fa.dV = at<float>(p.dV);
         if (dual) { fa.dQd = at<float>(p.dQd); fa.dKd = at<float>(p.dKd); fa.dVd = at<float>(p.dVd); }
+        // the tcgen05 backward writes the merged, RoPE-inverted bf16 rows of dqkv directly
+        fa.H = H;
+        fa.ldq = 3 * d;
+        fa.rope = at<float>(p.rope);
+        fa.qscale = 1.f / sqrtf(static_cast<float>(dh));
+        fa.dqkv = reinterpret_cast<__nv_bfloat16*>(at<T>(p.dqkv));
+        fa.dqkvd = dual ? reinterpret_cast<__nv_bfloat16*>(at<T>(p.dqkvd)) : nullptr;
+        merged = std::is_same<T, __nv_bfloat16>::value && mf::flash_bwd_merges(fa, dual);
+        if (merged) {
+          wait_seed_readers(2);    // dqkv's previous readers (the side stream) are done
+        } else {
+          fa.dqkv = fa.dqkvd = nullptr;
+        }
         mf::flash_bwd(fa, dual, s);
         launched(3);
       } else {
@@ -702,15 +716,17 @@ struct DecExec {
         gemm(g);
       }
       }
-      const float qscale = 1.f / sqrtf(static_cast<float>(dh));
-      wait_seed_readers(2);
-      mf::dec_rope_merge<T>(N, S, H, dh, at<float>(p.rope), qscale, at<float>(p.dQ), at<float>(p.dK),
-                            at<float>(p.dV), at<T>(p.dqkv), 3 * d, s);
-      launched();
-      if (dual) {
-        mf::dec_rope_merge<T>(N, S, H, dh, at<float>(p.rope), qscale, at<float>(p.dQd), at<float>(p.dKd),
-                              at<float>(p.dVd), at<T>(p.dqkvd), 3 * d, s);
+      if (!merged) {
+        const float qscale = 1.f / sqrtf(static_cast<float>(dh));
+        wait_seed_readers(2);
+        mf::dec_rope_merge<T>(N, S, H, dh, at<float>(p.rope), qscale, at<float>(p.dQ), at<float>(p.dK),
+                              at<float>(p.dV), at<T>(p.dqkv), 3 * d, s);
         launched();
+        if (dual) {
+          mf::dec_rope_merge<T>(N, S, H, dh, at<float>(p.rope), qscale, at<float>(p.dQd), at<float>(p.dKd),
+                                at<float>(p.dVd), at<T>(p.dqkvd), 3 * d, s);
+          launched();
+        }
       }
       wprod(d, 3 * d, at<T>(p.h1[l]), at<T>(p.h1d[l]), at<T>(p.dqkv), at<T>(p.dqkvd), dual,
             G(Ly.Wqkv[l]), Hh(Ly.Wqkv[l]), WS_QKV);

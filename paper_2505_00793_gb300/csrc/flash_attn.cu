@@ -668,6 +668,10 @@ void flash_fwd(const FlashArgs& a, bool dual, cudaStream_t s) {
     launch_k(flash_fwd_kernel<false>, grid, dim3(FTHREADS), SMEM_FWD0, s, a);
 }
 
+bool flash_bwd_merges(const FlashArgs& a, bool dual) {
+  return a.tc_bwd && flash_tc_bwd_supported(a, dual);
+}
+
 void flash_bwd(const FlashArgs& a, bool dual, cudaStream_t s) {
   // tcgen05 backward (launch errors surface at the caller's check)
   if (a.tc_bwd && flash_tc_bwd_supported(a, dual)) {

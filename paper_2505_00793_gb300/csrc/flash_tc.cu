@@ -541,6 +541,11 @@ struct FtbParams {
   const float *lse, *rbar, *D, *Dd;
   float *dQ, *dQd, *dK, *dKd, *dV, *dVd;
   int* status;
+  // merged bf16 outputs (FlashArgs::dqkv): heads H, row stride ldq, RoPE table, q scale
+  __nv_bfloat16 *dqkv, *dqkvd;
+  int H, ldq;
+  const float* rope;
+  float qscale;
 };
 
 __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes,
@@ -576,6 +581,38 @@ __device__ __forceinline__ void store_acc_row(uint32_t taddr, float* dst, int cb
 #pragma unroll
     for (int i = 0; i < 16; i += 4)
       *reinterpret_cast<float4*>(dst + c0 + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+  }
+}
+
+// Columns cb .. cb + 31 of a 64-wide accumulator row (this thread's TMEM lane) as bf16 at
+// dst + cb, with the inverse RoPE rotation of position pos when rot is set: the first half's
+// element j becomes (x_j cos_j + x_{j+32} sin_j) scale, the second half's
+// (x_{j+32} cos_j - x_j sin_j) scale (the partner half is read from the same TMEM lane).
+__device__ __forceinline__ void store_merged_row(uint32_t taddr, int cb, bool rot, int pos,
+                                                 const float* rtab, float scale,
+                                                 __nv_bfloat16* dst) {
+  const int pb = cb ^ 32;
+  const float sg = cb == 0 ? 1.f : -1.f;
+#pragma unroll 1
+  for (int c0 = 0; c0 < 32; c0 += 16) {
+    float x[16], y[16];
+    tmem_ld16_nowait(taddr + cb + c0, x);
+    if (rot) tmem_ld16_nowait(taddr + pb + c0, y);
+    tmem_wait_ld();
+    uint32_t pk[8];
+#pragma unroll
+    for (int e = 0; e < 16; e += 2) {
+      float o0 = x[e], o1 = x[e + 1];
+      if (rot) {
+        const float4 t = *reinterpret_cast<const float4*>(rtab + 2 * (pos * 32 + c0 + e));
+        o0 = (x[e] * t.x + sg * y[e] * t.y) * scale;
+        o1 = (x[e + 1] * t.z + sg * y[e + 1] * t.w) * scale;
+      }
+      pk[e / 2] = pack_bf16x2(o0, o1);
+    }
+    uint4* d4 = reinterpret_cast<uint4*>(dst + cb + c0);
+    d4[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    d4[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
   }
 }
 
@@ -856,12 +893,24 @@ __global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
     // ---- outputs: dV, dK (dV', dK') rows of this key, this thread's columns ---------------
     if (ok && wwait(&o_done, (ntile - 1) & 1, p.status, abort)) {
       tc_fence_after();
-      const int64_t off = (static_cast<int64_t>(row0) + key) * HD;
-      store_acc_row(tb + lo + C::C_DV, p.dV + off, cb);
-      store_acc_row(tb + lo + C::C_DK, p.dK + off, cb);
-      if (DUAL) {
-        store_acc_row(tb + lo + C::C_DVD, p.dVd + off, cb);
-        store_acc_row(tb + lo + C::C_DKD, p.dKd + off, cb);
+      if (p.dqkv) {
+        // merged rows: token b*S + key, k part (rotated) and v part of head h
+        const int hh = bh % p.H, bb = bh / p.H, dm = p.H * HD;
+        const int64_t orow = (static_cast<int64_t>(bb) * p.S + key) * p.ldq + hh * HD;
+        store_merged_row(tb + lo + C::C_DK, cb, true, key, p.rope, 1.f, p.dqkv + orow + dm);
+        store_merged_row(tb + lo + C::C_DV, cb, false, key, p.rope, 1.f, p.dqkv + orow + 2 * dm);
+        if (DUAL) {
+          store_merged_row(tb + lo + C::C_DKD, cb, true, key, p.rope, 1.f, p.dqkvd + orow + dm);
+          store_merged_row(tb + lo + C::C_DVD, cb, false, key, p.rope, 1.f, p.dqkvd + orow + 2 * dm);
+        }
+      } else {
+        const int64_t off = (static_cast<int64_t>(row0) + key) * HD;
+        store_acc_row(tb + lo + C::C_DV, p.dV + off, cb);
+        store_acc_row(tb + lo + C::C_DK, p.dK + off, cb);
+        if (DUAL) {
+          store_acc_row(tb + lo + C::C_DVD, p.dVd + off, cb);
+          store_acc_row(tb + lo + C::C_DKD, p.dKd + off, cb);
+        }
       }
     }
     tc_fence_before();
@@ -1113,9 +1162,18 @@ __global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
     }
     if (ok && wwait(&o_done, (ntile - 1) & 1, p.status, abort)) {
       tc_fence_after();
-      const int64_t off = gi * HD;
-      store_acc_row(tb + lo + C::C_DQ, p.dQ + off, cb);
-      if (DUAL) store_acc_row(tb + lo + C::C_DQD, p.dQd + off, cb);
+      if (p.dqkv) {
+        // merged rows: token b*S + q, q part (rotated and scaled) of head h
+        const int hh = bh % p.H, bb = bh / p.H;
+        const int64_t orow = (static_cast<int64_t>(bb) * p.S + q) * p.ldq + hh * HD;
+        store_merged_row(tb + lo + C::C_DQ, cb, true, q, p.rope, p.qscale, p.dqkv + orow);
+        if (DUAL)
+          store_merged_row(tb + lo + C::C_DQD, cb, true, q, p.rope, p.qscale, p.dqkvd + orow);
+      } else {
+        const int64_t off = gi * HD;
+        store_acc_row(tb + lo + C::C_DQ, p.dQ + off, cb);
+        if (DUAL) store_acc_row(tb + lo + C::C_DQD, p.dQd + off, cb);
+      }
     }
     tc_fence_before();
   }
@@ -1163,6 +1221,12 @@ cudaError_t launch_ftc_bwd(const FlashArgs& a, cudaStream_t s) {
   p.dK = a.dK; p.dKd = a.dKd;
   p.dV = a.dV; p.dVd = a.dVd;
   p.status = a.status;
+  p.dqkv = a.dqkv;
+  p.dqkvd = DUAL ? a.dqkvd : nullptr;
+  p.H = a.H;
+  p.ldq = a.ldq;
+  p.rope = a.rope;
+  p.qscale = a.qscale;
   const dim3 grid(a.BH, a.S / 128);
   e = launch_k(flash_tc_bwd_kv_kernel<DUAL>, grid, dim3(BW_THREADS), KC::SMEM, s, k128[0],
                k128[1], k128[2], k128[3], q64[0], q64[1], q64[2], q64[3], p);
@@ -1185,6 +1249,11 @@ cudaError_t flash_tc_fwd(const FlashArgs& a, bool dual, cudaStream_t s) {
 
 bool flash_tc_bwd_supported(const FlashArgs& a, bool dual) {
   if (!flash_tc_supported(a.S, HD) || a.BH < 1) return false;
+  // merged outputs: 16-byte aligned rows, whole heads, a RoPE table
+  if (a.dqkv && (a.H < 1 || a.BH % a.H || !a.rope || (a.ldq & 7) ||
+                 (reinterpret_cast<uintptr_t>(a.dqkv) & 15) ||
+                 (dual && (!a.dqkvd || (reinterpret_cast<uintptr_t>(a.dqkvd) & 15)))))
+    return false;
   // the row statistics stream into shared memory by bulk copies of 64 floats
   const void* stats[4] = {a.lse, a.D, a.rbar, a.Dd};
   for (int i = 0; i < (dual ? 4 : 2); ++i)

@@ -270,6 +270,15 @@ struct FlashArgs {
   int tc = 1;              // tcgen05 forward where S is a multiple of 128: 0 never,
                            // 1 the dual kernel, 2 the dual and the primal kernels
   int tc_bwd = 0;          // 1: tcgen05 backward (primal and dual) where supported
+  // tcgen05 backward only: when dqkv is set, the kernels write the gradient of the fused
+  // q|k|v projection instead of float32 dQ, dK, dV: token-major bf16 rows [B*S][ldq], q at
+  // column h*64 + e (scaled by qscale), k at H*64 + h*64 + e, v at 2*H*64 + h*64 + e, with
+  // the inverse RoPE rotation of table rope ([S][32] (cos, sin) pairs) applied to q and k
+  // (the output of dec_rope_merge); dqkvd likewise for the tangents.
+  __nv_bfloat16 *dqkv = nullptr, *dqkvd = nullptr;
+  int ldq = 0;
+  const float* rope = nullptr;
+  float qscale = 1.f;
   int* status = nullptr;   // device status word (bounded waits of the tcgen05 kernels)
 };
 bool flash_supported(int S, int dh);
@@ -279,6 +288,8 @@ cudaError_t flash_tc_fwd(const FlashArgs& a, bool dual, cudaStream_t s);
 // tcgen05 backward (both kernels): S a multiple of 128, 64-wide heads, 16-byte aligned row
 // statistics.
 bool flash_tc_bwd_supported(const FlashArgs& a, bool dual);
+// Whether flash_bwd runs the tcgen05 backward for these arguments (and so honours dqkv).
+bool flash_bwd_merges(const FlashArgs& a, bool dual);
 cudaError_t flash_tc_bwd(const FlashArgs& a, bool dual, cudaStream_t s);
 void flash_fwd(const FlashArgs& a, bool dual, cudaStream_t s);
 void flash_bwd(const FlashArgs& a, bool dual, cudaStream_t s);
