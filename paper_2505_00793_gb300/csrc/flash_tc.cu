@@ -584,13 +584,14 @@ __device__ __forceinline__ void store_acc_row(uint32_t taddr, float* dst, int cb
   }
 }
 
-// Columns cb .. cb + 31 of a 64-wide accumulator row (this thread's TMEM lane) as bf16 at
-// dst + cb, with the inverse RoPE rotation of position pos when rot is set: the first half's
-// element j becomes (x_j cos_j + x_{j+32} sin_j) scale, the second half's
+// Columns cb .. cb + 31 of a 64-wide accumulator row (this thread's TMEM lane, row r of
+// the tile) as bf16 into a [128][64] staging tile (128-byte rows, 16-byte chunk c of row r at
+// position c ^ (r & 7)), with the inverse RoPE rotation of position pos when rot is set: the
+// first half's element j becomes (x_j cos_j + x_{j+32} sin_j) scale, the second half's
 // (x_{j+32} cos_j - x_j sin_j) scale (the partner half is read from the same TMEM lane).
-__device__ __forceinline__ void store_merged_row(uint32_t taddr, int cb, bool rot, int pos,
-                                                 const float* rtab, float scale,
-                                                 __nv_bfloat16* dst) {
+__device__ __forceinline__ void stage_merged_row(uint32_t taddr, int cb, bool rot, int pos,
+                                                 const float* rtab, float scale, uint8_t* buf,
+                                                 int r) {
   const int pb = cb ^ 32;
   const float sg = cb == 0 ? 1.f : -1.f;
 #pragma unroll 1
@@ -610,9 +611,29 @@ __device__ __forceinline__ void store_merged_row(uint32_t taddr, int cb, bool ro
       }
       pk[e / 2] = pack_bf16x2(o0, o1);
     }
-    uint4* d4 = reinterpret_cast<uint4*>(dst + cb + c0);
-    d4[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-    d4[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+    const int ch = (cb + c0) >> 3;
+    *reinterpret_cast<uint4*>(buf + r * 128 + (((ch) ^ (r & 7)) << 4)) =
+        make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    *reinterpret_cast<uint4*>(buf + r * 128 + (((ch + 1) ^ (r & 7)) << 4)) =
+        make_uint4(pk[4], pk[5], pk[6], pk[7]);
+  }
+}
+
+// The elementwise warps' barrier (named barrier 1, BW_EW warps).
+__device__ __forceinline__ void ew_bar() {
+  asm volatile("bar.sync 1, %0;" ::"n"(BW_EW * 32) : "memory");
+}
+
+// A staged [128][64] bf16 tile to 128 rows of global memory (row i at row_base(i)), by the
+// elementwise threads (et = 0 .. BW_EW*32 - 1): eight consecutive threads write one row's
+// 128 bytes.
+template <class RowBase>
+__device__ __forceinline__ void staged_rows_out(const uint8_t* buf, int et, RowBase row_base) {
+#pragma unroll 1
+  for (int i = et; i < 128 * 8; i += BW_EW * 32) {
+    const int row = i >> 3, c = i & 7;
+    const uint4 v = *reinterpret_cast<const uint4*>(buf + row * 128 + ((c ^ (row & 7)) << 4));
+    *reinterpret_cast<uint4*>(row_base(row) + c * 8) = v;
   }
 }
 
@@ -891,26 +912,44 @@ __global__ void __launch_bounds__(BW_THREADS, KvCfg<DUAL>::CTAS)
       if (lane == 0) mbar_arrive_local(&p_full);
     }
     // ---- outputs: dV, dK (dV', dK') rows of this key, this thread's columns ---------------
-    if (ok && wwait(&o_done, (ntile - 1) & 1, p.status, abort)) {
-      tc_fence_after();
-      if (p.dqkv) {
-        // merged rows: token b*S + key, k part (rotated) and v part of head h
+    const bool have = ok && wwait(&o_done, (ntile - 1) & 1, p.status, abort);
+    if (have) tc_fence_after();
+    if (p.dqkv) {
+      // merged rows: token b*S + key, k part (rotated) and v part of head h, staged in the
+      // A-operand buffers (the last products have read them) and written row by row; every
+      // elementwise thread meets the barrier, with or without a result (a timed-out call
+      // reports its status and its outputs are void)
+      if (have) {
+        stage_merged_row(tb + lo + C::C_DK, cb, true, key, p.rope, 1.f, sOp, r);
+        stage_merged_row(tb + lo + C::C_DV, cb, false, key, p.rope, 1.f, sOp + OPND_B, r);
+        if (DUAL) {
+          stage_merged_row(tb + lo + C::C_DKD, cb, true, key, p.rope, 1.f, sOp + 2 * OPND_B, r);
+          stage_merged_row(tb + lo + C::C_DVD, cb, false, key, p.rope, 1.f, sOp + 3 * OPND_B, r);
+        }
+      }
+      ew_bar();
+      if (have) {
         const int hh = bh % p.H, bb = bh / p.H, dm = p.H * HD;
-        const int64_t orow = (static_cast<int64_t>(bb) * p.S + key) * p.ldq + hh * HD;
-        store_merged_row(tb + lo + C::C_DK, cb, true, key, p.rope, 1.f, p.dqkv + orow + dm);
-        store_merged_row(tb + lo + C::C_DV, cb, false, key, p.rope, 1.f, p.dqkv + orow + 2 * dm);
+        const int et = threadIdx.x - 64;
+        auto base = [&](__nv_bfloat16* out, int part) {
+          return [=](int i) {
+            return out + (static_cast<int64_t>(bb) * p.S + key0 + i) * p.ldq + part * dm + hh * HD;
+          };
+        };
+        staged_rows_out(sOp, et, base(p.dqkv, 1));
+        staged_rows_out(sOp + OPND_B, et, base(p.dqkv, 2));
         if (DUAL) {
-          store_merged_row(tb + lo + C::C_DKD, cb, true, key, p.rope, 1.f, p.dqkvd + orow + dm);
-          store_merged_row(tb + lo + C::C_DVD, cb, false, key, p.rope, 1.f, p.dqkvd + orow + 2 * dm);
+          staged_rows_out(sOp + 2 * OPND_B, et, base(p.dqkvd, 1));
+          staged_rows_out(sOp + 3 * OPND_B, et, base(p.dqkvd, 2));
         }
-      } else {
-        const int64_t off = (static_cast<int64_t>(row0) + key) * HD;
-        store_acc_row(tb + lo + C::C_DV, p.dV + off, cb);
-        store_acc_row(tb + lo + C::C_DK, p.dK + off, cb);
-        if (DUAL) {
-          store_acc_row(tb + lo + C::C_DVD, p.dVd + off, cb);
-          store_acc_row(tb + lo + C::C_DKD, p.dKd + off, cb);
-        }
+      }
+    } else if (have) {
+      const int64_t off = (static_cast<int64_t>(row0) + key) * HD;
+      store_acc_row(tb + lo + C::C_DV, p.dV + off, cb);
+      store_acc_row(tb + lo + C::C_DK, p.dK + off, cb);
+      if (DUAL) {
+        store_acc_row(tb + lo + C::C_DVD, p.dVd + off, cb);
+        store_acc_row(tb + lo + C::C_DKD, p.dKd + off, cb);
       }
     }
     tc_fence_before();
@@ -1160,20 +1199,31 @@ __global__ void __launch_bounds__(BW_THREADS, QCfg<DUAL>::CTAS)
       __syncwarp();
       if (lane == 0) mbar_arrive_local(&p_full);
     }
-    if (ok && wwait(&o_done, (ntile - 1) & 1, p.status, abort)) {
-      tc_fence_after();
-      if (p.dqkv) {
-        // merged rows: token b*S + q, q part (rotated and scaled) of head h
-        const int hh = bh % p.H, bb = bh / p.H;
-        const int64_t orow = (static_cast<int64_t>(bb) * p.S + q) * p.ldq + hh * HD;
-        store_merged_row(tb + lo + C::C_DQ, cb, true, q, p.rope, p.qscale, p.dqkv + orow);
-        if (DUAL)
-          store_merged_row(tb + lo + C::C_DQD, cb, true, q, p.rope, p.qscale, p.dqkvd + orow);
-      } else {
-        const int64_t off = gi * HD;
-        store_acc_row(tb + lo + C::C_DQ, p.dQ + off, cb);
-        if (DUAL) store_acc_row(tb + lo + C::C_DQD, p.dQd + off, cb);
+    const bool have = ok && wwait(&o_done, (ntile - 1) & 1, p.status, abort);
+    if (have) tc_fence_after();
+    if (p.dqkv) {
+      // merged rows: token b*S + q, q part (rotated and scaled) of head h, staged in the
+      // A-operand buffers and written row by row (every elementwise thread meets the barrier)
+      if (have) {
+        stage_merged_row(tb + lo + C::C_DQ, cb, true, q, p.rope, p.qscale, sOp, r);
+        if (DUAL) stage_merged_row(tb + lo + C::C_DQD, cb, true, q, p.rope, p.qscale, sOp + OPND_B, r);
       }
+      ew_bar();
+      if (have) {
+        const int hh = bh % p.H, bb = bh / p.H;
+        const int et = threadIdx.x - 64;
+        auto base = [&](__nv_bfloat16* out) {
+          return [=](int i) {
+            return out + (static_cast<int64_t>(bb) * p.S + q0 + i) * p.ldq + hh * HD;
+          };
+        };
+        staged_rows_out(sOp, et, base(p.dqkv));
+        if (DUAL) staged_rows_out(sOp + OPND_B, et, base(p.dqkvd));
+      }
+    } else if (have) {
+      const int64_t off = gi * HD;
+      store_acc_row(tb + lo + C::C_DQ, p.dQ + off, cb);
+      if (DUAL) store_acc_row(tb + lo + C::C_DQD, p.dQd + off, cb);
     }
     tc_fence_before();
   }
