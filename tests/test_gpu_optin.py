@@ -1,12 +1,13 @@
-"""The three opt-in paths (off by default), each against the default path or the oracle.
+"""Option paths, each against the default path or the oracle.
 
-- MF_OPT_GEMM_PERSISTENT: the persistent CTA-pair GEMM against float64 products of the same
-  bf16 operands, on grids with several tiles per CTA pair (both TMEM accumulator sets and
-  the stage ring reused across tiles), and bf16 meta-gradients against the oracle.
-- MF_OPT_FUSED_HEAD: the narrow output layer, loss and data product in one kernel;
+- MF_OPT_GEMM_PERSISTENT (on by default, mode 2): the persistent CTA-pair GEMM in modes 1
+  and 3 against float64 products of the same bf16 operands, on grids with several tiles per
+  CTA pair (both TMEM accumulator sets and the stage ring reused across tiles), and bf16
+  meta-gradients against the oracle.
+- MF_OPT_FUSED_HEAD (off by default): the narrow output layer, loss and data product in one kernel;
   meta-gradients, HVPs with gradient and tangent losses, and the label check, against the
   oracle at the default path's tolerances.
-- MF_OPT_LAYER_UPDATES: per-layer updates on the update stream; the same update element for
+- MF_OPT_LAYER_UPDATES (off by default): per-layer updates on the update stream; the same update element for
   element, so meta-gradients are bit-identical to the single update (eager, captured and
   replayed calls)."""
 import numpy as np
@@ -28,11 +29,13 @@ def _set(native, option, value):
 
 # ---- persistent CTA-pair GEMM ------------------------------------------------------------
 
-@pytest.fixture
-def persistent():
+@pytest.fixture(params=[1, 3])
+def persistent(request):
+    """Mode 1 (dual products at 128-wide tiles, two TMEM sets) and mode 3 (256-wide dual
+    tiles, one set: the default mode's path for dual products with K > 2048)."""
     torch, native = need_gpu()
     _set(native, native.MF_OPT_GEMM_2SM, 2)
-    _set(native, native.MF_OPT_GEMM_PERSISTENT, 1)
+    _set(native, native.MF_OPT_GEMM_PERSISTENT, request.param)
     yield
     _set(native, native.MF_OPT_GEMM_PERSISTENT, 2)   # the default
     _set(native, native.MF_OPT_GEMM_2SM, 1)
