@@ -565,7 +565,7 @@ struct DecExec {
     auto Hh = [&](int64_t off) { return dual ? out_h + off : nullptr; };
     mf::dec_token_csr(N, S, V, ids_cur, at<int>(p.o_count), at<int>(p.o_start), at<int>(p.o_order),
                       at<int>(p.o_order_tmp), s);
-    launched(3);
+    launched(4);
     // head: dWh = hf^T dF ; dhf = dF Wh^T
     wprod(d, V, at<T>(p.hf), at<T>(p.hfd), at<T>(p.dF), at<T>(p.dFd), dual, G(Ly.Wh), Hh(Ly.Wh));
     {
@@ -577,14 +577,12 @@ struct DecExec {
     cudaMemsetAsync(at<float>(p.dx), 0, static_cast<size_t>(N) * d * 4, s);
     if (dual) cudaMemsetAsync(at<float>(p.dxd), 0, static_cast<size_t>(N) * d * 4, s);
     wait_seed_readers(0);
-    mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.xf), at<float>(p.xfd), at<float>(p.rf), at<float>(p.rfd),
-                           theta_cur + Ly.gf, dual ? u + Ly.gf : nullptr, at<float>(p.dh),
-                           dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx), at<float>(p.dxd), s,
-                           at<T>(p.dy), dual ? at<T>(p.dyd) : nullptr);
-    mf::dec_gain_grad(N, d, at<float>(p.xf), at<float>(p.xfd), at<float>(p.rf), at<float>(p.rfd),
-                      at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr, G(Ly.gf), Hh(Ly.gf),
-                      at<float>(p.gpart), s);
-    launched(2);
+    launched(mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.xf), at<float>(p.xfd), at<float>(p.rf),
+                                    at<float>(p.rfd), theta_cur + Ly.gf, dual ? u + Ly.gf : nullptr,
+                                    at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr,
+                                    at<float>(p.dx), at<float>(p.dxd), G(Ly.gf), Hh(Ly.gf),
+                                    at<float>(p.gpart), s, at<T>(p.dy),
+                                    dual ? at<T>(p.dyd) : nullptr));
     for (int l = Ly.L - 1; l >= 0; --l) {
       if (ror_mode == 1) {
         cudaMemcpyAsync(at<float>(p.dxs[l]), at<float>(p.dx), static_cast<size_t>(N) * d * 4,
@@ -618,15 +616,14 @@ struct DecExec {
         g.C1 = at<float>(p.dhd); g.ldc1 = d;
         gemm(g);
       }
-      mf::dec_gain_grad(N, d, at<float>(p.x2[l]), at<float>(p.x2d[l]), at<float>(p.r2[l]),
-                        at<float>(p.r2d[l]), at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr,
-                        G(Ly.g2[l]), Hh(Ly.g2[l]), at<float>(p.gpart), s);
       wait_seed_readers(0);
-      mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.x2[l]), at<float>(p.x2d[l]), at<float>(p.r2[l]),
-                             at<float>(p.r2d[l]), theta_cur + Ly.g2[l], dual ? u + Ly.g2[l] : nullptr,
-                             at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx),
-                             at<float>(p.dxd), s, at<T>(p.dy), dual ? at<T>(p.dyd) : nullptr);
-      launched(2);
+      launched(mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.x2[l]), at<float>(p.x2d[l]),
+                                      at<float>(p.r2[l]), at<float>(p.r2d[l]), theta_cur + Ly.g2[l],
+                                      dual ? u + Ly.g2[l] : nullptr, at<float>(p.dh),
+                                      dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx),
+                                      at<float>(p.dxd), G(Ly.g2[l]), Hh(Ly.g2[l]),
+                                      at<float>(p.gpart), s, at<T>(p.dy),
+                                      dual ? at<T>(p.dyd) : nullptr));
       // ---- attention branch: seed = dx (written in bf16 by the norm backward above) -----
       seed_from(at<float>(p.dx), at<float>(p.dxd), dual, true);
       wprod(d, d, at<T>(p.Om[l]), at<T>(p.Omd[l]), at<T>(p.dy), at<T>(p.dyd), dual, G(Ly.Wo[l]),
@@ -737,16 +734,14 @@ struct DecExec {
         g.C1 = at<float>(p.dhd); g.ldc1 = d;
         gemm(g);
       }
-      mf::dec_gain_grad(N, d, at<float>(p.x1[l]), at<float>(p.x1d[l]), at<float>(p.r1[l]),
-                        at<float>(p.r1d[l]), at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr,
-                        G(Ly.g1[l]), Hh(Ly.g1[l]), at<float>(p.gpart), s);
       if (l > 0) wait_seed_readers(0);
-      mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.x1[l]), at<float>(p.x1d[l]), at<float>(p.r1[l]),
-                             at<float>(p.r1d[l]), theta_cur + Ly.g1[l], dual ? u + Ly.g1[l] : nullptr,
-                             at<float>(p.dh), dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx),
-                             at<float>(p.dxd), s, l > 0 ? at<T>(p.dy) : nullptr,
-                             l > 0 && dual ? at<T>(p.dyd) : nullptr);
-      launched(2);
+      launched(mf::dec_rmsnorm_bwd<T>(N, d, at<float>(p.x1[l]), at<float>(p.x1d[l]),
+                                      at<float>(p.r1[l]), at<float>(p.r1d[l]), theta_cur + Ly.g1[l],
+                                      dual ? u + Ly.g1[l] : nullptr, at<float>(p.dh),
+                                      dual ? at<float>(p.dhd) : nullptr, at<float>(p.dx),
+                                      at<float>(p.dxd), G(Ly.g1[l]), Hh(Ly.g1[l]),
+                                      at<float>(p.gpart), s, l > 0 ? at<T>(p.dy) : nullptr,
+                                      l > 0 && dual ? at<T>(p.dyd) : nullptr));
     }
     mf::dec_embed_bwd(V, d, at<int>(p.o_start), at<int>(p.o_order), at<float>(p.dx),
                       dual ? at<float>(p.dxd) : nullptr, G(Ly.E), Hh(Ly.E), s);

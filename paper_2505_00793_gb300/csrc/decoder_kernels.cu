@@ -30,6 +30,10 @@ __device__ __forceinline__ float warp_max(float v) {
   return v;
 }
 
+// SMs of a GB300 (152): sets the grid size of the grid-stride row kernels (a performance
+// choice; every kernel is correct for any grid).
+constexpr int ROW_SMS = 152;
+
 // Block-wide sum of two values (fixed reduction order), blockDim.x a multiple of 32, <= 1024.
 __device__ __forceinline__ float2 block_sum2(float a, float b) {
   __shared__ float2 red[32];
@@ -194,15 +198,13 @@ __global__ void __launch_bounds__(256) rmsnorm_fwd_warp_kernel(
   }
 }
 
+// Row r of the warp-per-row RMSNorm backward (this lane's columns lane*4 + 128 k).
 template <typename T>
-__global__ void __launch_bounds__(256) rmsnorm_bwd_warp_kernel(
-    int N, int d, const float* __restrict__ x, const float* __restrict__ xd,
+__device__ __forceinline__ void rmsnorm_bwd_row(
+    int r, int lane, int d, const float* __restrict__ x, const float* __restrict__ xd,
     const float* __restrict__ rr, const float* __restrict__ rrd, const float* __restrict__ g,
     const float* __restrict__ gd, const float* __restrict__ dy, const float* __restrict__ dyd,
     float* __restrict__ dx, float* __restrict__ dxd, T* __restrict__ dxb, T* __restrict__ dxdb) {
-  pdl_entry();
-  const int r = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
-  if (r >= N) return;
   const int64_t o = static_cast<int64_t>(r) * d;
   const bool dual = dyd != nullptr;
   const float rs = rr[r];
@@ -266,6 +268,49 @@ __global__ void __launch_bounds__(256) rmsnorm_bwd_warp_kernel(
       *reinterpret_cast<float4*>(dxd + o + c) = make_float4(outd[0], outd[1], outd[2], outd[3]);
       if (dxdb) st_t4<T>(dxdb + o + c, outd[0], outd[1], outd[2], outd[3]);
     }
+  }
+}
+
+// The warp-per-row RMSNorm backward, and with part set the gain gradient's partial sums over
+// the block's eight rows (data the row passes have just read, so the rows come from L2):
+// warp w takes 128-column chunks w, w + 8, ..., adds the rows in order and writes partial
+// row blockIdx.x of part (and of partd for the tangent).  The formulas per element are those
+// of gain_grad_partial_kernel.
+template <typename T>
+__global__ void __launch_bounds__(256) rmsnorm_bwd_warp_kernel(
+    int N, int d, const float* __restrict__ x, const float* __restrict__ xd,
+    const float* __restrict__ rr, const float* __restrict__ rrd, const float* __restrict__ g,
+    const float* __restrict__ gd, const float* __restrict__ dy, const float* __restrict__ dyd,
+    float* __restrict__ dx, float* __restrict__ dxd, T* __restrict__ dxb, T* __restrict__ dxdb,
+    float* __restrict__ part, float* __restrict__ partd) {
+  pdl_entry();
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * 8 + w;
+  if (r < N) rmsnorm_bwd_row<T>(r, lane, d, x, xd, rr, rrd, g, gd, dy, dyd, dx, dxd, dxb, dxdb);
+  if (!part) return;
+  const bool dual = partd != nullptr;
+  const int q0 = blockIdx.x * 8, q1 = min(N, q0 + 8);
+  for (int c = w * 128 + lane * 4; c < d; c += 1024) {
+    float4 a = make_float4(0.f, 0.f, 0.f, 0.f), ad = a;
+#pragma unroll 4
+    for (int q = q0; q < q1; ++q) {
+      const int64_t o = static_cast<int64_t>(q) * d + c;
+      const float rs = rr[q];
+      const float4 xv = ld4f(x + o), dv = ld4f(dy + o);
+      const float n0 = xv.x * rs, n1 = xv.y * rs, n2 = xv.z * rs, n3 = xv.w * rs;
+      a.x += dv.x * n0; a.y += dv.y * n1; a.z += dv.z * n2; a.w += dv.w * n3;
+      if (dual) {
+        const float rsd = rrd[q];
+        const float4 xdv = ld4f(xd + o), ddv = ld4f(dyd + o);
+        ad.x += ddv.x * n0 + dv.x * (xdv.x * rs + xv.x * rsd);
+        ad.y += ddv.y * n1 + dv.y * (xdv.y * rs + xv.y * rsd);
+        ad.z += ddv.z * n2 + dv.z * (xdv.z * rs + xv.z * rsd);
+        ad.w += ddv.w * n3 + dv.w * (xdv.w * rs + xv.w * rsd);
+      }
+    }
+    const int64_t po = static_cast<int64_t>(blockIdx.x) * d + c;
+    *reinterpret_cast<float4*>(part + po) = a;
+    if (dual) *reinterpret_cast<float4*>(partd + po) = ad;
   }
 }
 
@@ -353,19 +398,39 @@ __global__ void gain_grad_partial_kernel(int N, int d, const float* __restrict__
   }
 }
 
-__global__ void gain_grad_final_kernel(int nchunk, int d, const float* __restrict__ part,
-                                       const float* __restrict__ partd, float* __restrict__ dg,
-                                       float* __restrict__ dgd) {
+// Stage 2: the nchunk partial rows summed per column in a fixed order.  Block (32, 32) owns 32
+// columns; thread (x, y) adds partial rows y, y + 32, ... in order, then the 32 sums of a
+// column are added in y order.
+constexpr int GF_Y = 32;
+
+__global__ void __launch_bounds__(32 * GF_Y) gain_grad_final_kernel(
+    int nchunk, int d, const float* __restrict__ part, const float* __restrict__ partd,
+    float* __restrict__ dg, float* __restrict__ dgd) {
   pdl_entry();
-  const int j = blockIdx.x * blockDim.x + threadIdx.x;
-  if (j >= d) return;
+  __shared__ float sp[GF_Y][33];
+  __shared__ float spd[GF_Y][33];
+  const int j = blockIdx.x * 32 + threadIdx.x;
   float t = 0.f, td = 0.f;
-  for (int c = 0; c < nchunk; ++c) {
-    t += part[static_cast<int64_t>(c) * d + j];
-    if (partd) td += partd[static_cast<int64_t>(c) * d + j];
+  if (j < d) {
+#pragma unroll 8
+    for (int c = threadIdx.y; c < nchunk; c += GF_Y) {
+      t += part[static_cast<int64_t>(c) * d + j];
+      if (partd) td += partd[static_cast<int64_t>(c) * d + j];
+    }
   }
-  if (dg) dg[j] = t;
-  if (partd && dgd) dgd[j] = td;
+  sp[threadIdx.y][threadIdx.x] = t;
+  spd[threadIdx.y][threadIdx.x] = td;
+  __syncthreads();
+  if (threadIdx.y == 0 && j < d) {
+    float u = 0.f, ud = 0.f;
+#pragma unroll
+    for (int k = 0; k < GF_Y; ++k) {
+      u += sp[k][threadIdx.x];
+      ud += spd[k][threadIdx.x];
+    }
+    if (dg) dg[j] = u;
+    if (partd && dgd) dgd[j] = ud;
+  }
 }
 
 // RoPE angle table: (cos, sin) of s * base^(-2 j / dh) for positions s < S and pairs
@@ -727,30 +792,51 @@ __global__ void token_count_kernel(int N, int S, int V, const int* __restrict__ 
   atomicAdd(&count[id], 1);
 }
 
-// Exclusive scan of count[0..V) into start[0..V] (one block).
-__global__ void scan_kernel(int V, const int* __restrict__ count, int* __restrict__ start) {
-  pdl_entry();
-  __shared__ int part[1024];
-  const int per = (V + blockDim.x - 1) / blockDim.x;
-  const int b0 = threadIdx.x * per;
-  int s = 0;
-  for (int i = b0; i < b0 + per && i < V; ++i) s += count[i];
-  part[threadIdx.x] = s;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    int acc = 0;
-    for (int i = 0; i < static_cast<int>(blockDim.x); ++i) {
-      const int v = part[i];
-      part[i] = acc;
-      acc += v;
-    }
-    start[V] = acc;
+// Exclusive scan of count[0..V) into start[0..V] (one block of SCAN_THREADS).  Thread t owns
+// the run [t per, (t + 1) per): it adds the run (eight independent loads at a time), the block
+// scans the run totals with warp shuffles, and the thread writes its run's starts.
+constexpr int SCAN_THREADS = 1024;
+
+__device__ __forceinline__ int warp_incl_scan(int v, int lane) {
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int t = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v += t;
   }
+  return v;
+}
+
+__global__ void __launch_bounds__(SCAN_THREADS) scan_kernel(int V, const int* __restrict__ count,
+                                                            int* __restrict__ start) {
+  pdl_entry();
+  __shared__ int wtot[SCAN_THREADS / 32];
+  const int per = (V + SCAN_THREADS - 1) / SCAN_THREADS;
+  const int b0 = threadIdx.x * per, b1 = min(V, b0 + per);
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  int run = 0;
+  for (int i0 = b0; i0 < b1; i0 += 8) {
+    int v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = i0 + k < b1 ? count[i0 + k] : 0;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) run += v[k];
+  }
+  const int inc = warp_incl_scan(run, lane);
+  if (lane == 31) wtot[w] = inc;
   __syncthreads();
-  int acc = part[threadIdx.x];
-  for (int i = b0; i < b0 + per && i < V; ++i) {
-    start[i] = acc;
-    acc += count[i];
+  if (w == 0) wtot[lane] = warp_incl_scan(wtot[lane], lane);   // 32 warps
+  __syncthreads();
+  int acc = inc - run + (w > 0 ? wtot[w - 1] : 0);
+  if (threadIdx.x == 0) start[V] = wtot[SCAN_THREADS / 32 - 1];
+  for (int i0 = b0; i0 < b1; i0 += 8) {
+    int v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = i0 + k < b1 ? count[i0 + k] : 0;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      if (i0 + k < b1) start[i0 + k] = acc;
+      acc += v[k];
+    }
   }
 }
 
@@ -769,114 +855,188 @@ __global__ void token_scatter_kernel(int N, int S, int V, const int* __restrict_
   tmp[start[id] + slot] = r;
 }
 
-constexpr int SEG_SMEM = 4096;
+// Ids are dealt to blocks with a stride of gridDim.x (block b takes ids b, b + G, b + 2G, ...),
+// so that the most frequent ids (the smallest, under a Zipf law) land in different blocks,
+// and a block stages the segment bounds of ID_BATCH of its ids at a time.
+constexpr int ID_BATCH = 256;
 
-__global__ void token_order_kernel(const int* __restrict__ start, const int* __restrict__ tmp,
-                                   int* __restrict__ order) {
-  pdl_entry();
-  __shared__ int seg[SEG_SMEM];
-  const int v = blockIdx.x;
-  const int a = start[v], L = start[v + 1] - a;
-  if (L == 0) return;
-  const bool staged = L <= SEG_SMEM;
-  if (staged)
-    for (int i = threadIdx.x; i < L; i += blockDim.x) seg[i] = tmp[a + i];
+__device__ __forceinline__ int stage_bounds(const int* __restrict__ start, int b, int G, int k0,
+                                            int nb, int* s_a, int* s_n) {
+  __syncthreads();   // the previous batch's bounds are no longer read
+  if (threadIdx.x < nb) {
+    const int v = b + (k0 + static_cast<int>(threadIdx.x)) * G;
+    const int a = start[v];
+    s_a[threadIdx.x] = a;
+    s_n[threadIdx.x] = start[v + 1] - a;
+  }
   __syncthreads();
-  for (int i = threadIdx.x; i < L; i += blockDim.x) {
-    const int pi = staged ? seg[i] : tmp[a + i];
-    int rank = 0;
-    for (int k = 0; k < L; ++k) rank += (staged ? seg[k] : tmp[a + k]) < pi;
-    order[a + rank] = pi;
+  return nb;
+}
+
+// Each segment of the scattered positions is put in position order: an entry's rank is the
+// number of entries of the segment at earlier positions.  Segments of up to 32 entries take
+// one warp (ranks by shuffles); longer ones the block, through a bitmap of the positions
+// (rank = set bits below the position) when the batch has at most 32 ORD_BM_WORDS tokens, by
+// direct counting otherwise.
+constexpr int ORD_BM_WORDS = 2048;
+
+__global__ void __launch_bounds__(256) token_order_kernel(int V, int N, const int* __restrict__ start,
+                                                          const int* __restrict__ tmp,
+                                                          int* __restrict__ order) {
+  pdl_entry();
+  __shared__ int s_a[ID_BATCH], s_n[ID_BATCH];
+  __shared__ unsigned bm[ORD_BM_WORDS];
+  __shared__ int wpre[ORD_BM_WORDS];
+  __shared__ int wtot[8];
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = gridDim.x, b = blockIdx.x;
+  const int nmine = (V - b + G - 1) / G;
+  const bool use_bm = N <= 32 * ORD_BM_WORDS;
+  const int nw = (N + 31) >> 5;
+  const int per = (nw + 255) / 256;   // bitmap words per thread in the prefix count
+  for (int k0 = 0; k0 < nmine; k0 += ID_BATCH) {
+    const int nb = stage_bounds(start, b, G, k0, min(ID_BATCH, nmine - k0), s_a, s_n);
+    for (int i = w; i < nb; i += 8) {
+      const int L = s_n[i];
+      if (L == 0 || L > 32) continue;
+      const int a = s_a[i];
+      const int pi = lane < L ? tmp[a + lane] : 0;
+      int rank = 0;
+      for (int k = 0; k < L; ++k) rank += __shfl_sync(0xffffffffu, pi, k) < pi ? 1 : 0;
+      if (lane < L) order[a + rank] = pi;
+    }
+    for (int i = 0; i < nb; ++i) {
+      const int L = s_n[i];   // uniform across the block
+      if (L <= 32) continue;
+      const int a = s_a[i];
+      if (!use_bm) {
+        for (int j = threadIdx.x; j < L; j += blockDim.x) {
+          const int pi = tmp[a + j];
+          int rank = 0;
+          for (int k = 0; k < L; ++k) rank += tmp[a + k] < pi ? 1 : 0;
+          order[a + rank] = pi;
+        }
+        continue;
+      }
+      for (int j = threadIdx.x; j < nw; j += blockDim.x) bm[j] = 0u;
+      __syncthreads();
+      for (int j = threadIdx.x; j < L; j += blockDim.x) {
+        const int pi = tmp[a + j];
+        atomicOr(&bm[pi >> 5], 1u << (pi & 31));
+      }
+      __syncthreads();
+      // exclusive prefix of the words' bit counts: thread t owns words [t per, (t + 1) per)
+      const int j0 = threadIdx.x * per, j1 = min(nw, j0 + per);
+      int run = 0;
+      for (int j = j0; j < j1; ++j) run += __popc(bm[j]);
+      const int inc = warp_incl_scan(run, lane);
+      if (lane == 31) wtot[w] = inc;
+      __syncthreads();
+      int acc = inc - run;
+      for (int k = 0; k < w; ++k) acc += wtot[k];
+      for (int j = j0; j < j1; ++j) {
+        wpre[j] = acc;
+        acc += __popc(bm[j]);
+      }
+      __syncthreads();
+      for (int j = threadIdx.x; j < L; j += blockDim.x) {
+        const int pi = tmp[a + j];
+        const int wd = pi >> 5;
+        order[a + wpre[wd] + __popc(bm[wd] & ((1u << (pi & 31)) - 1u))] = pi;
+      }
+      __syncthreads();   // bm, wpre and wtot are reused by the next segment
+    }
   }
 }
 
-// dE[v] = sum over tokens with id v (in position order) of dx[token]; one block per id.
 // Embedding gradient: row v of dE is the sum of dx over the tokens with id v, in token order
-// (start/order from the counting sort).  Eight warps split a segment into contiguous parts
-// (Zipf-distributed ids give a few very long segments).  A warp sums every column of a row
-// at once (up to 1024 columns: eight float4 loads per lane in flight), then the warps'
-// partial sums are added in warp order, so the result is deterministic.
-constexpr int EB_SLICE = 256;
+// (start/order from the counting sort).  blockIdx.y picks a slice of EB_SLICE columns (one
+// float4 per lane); ids are dealt to blocks with a stride (as in token_order_kernel).  A
+// segment of more than EB_WARP tokens is split by the block's eight warps into contiguous
+// parts, each summed in order, and the parts are added in warp order; a shorter segment (and
+// the zero row of an id absent from the batch) takes one warp, which adds its rows in order,
+// the same sums since each of the eight parts would hold at most one row.  Deterministic.
+constexpr int EB_SLICE = 128;
+constexpr int EB_WARP = 8;
 
-__global__ void __launch_bounds__(256) embed_bwd_kernel(int d, const int* __restrict__ start,
+__device__ __forceinline__ void add4(float4& a, const float4& b) {
+  a.x += b.x; a.y += b.y; a.z += b.z; a.w += b.w;
+}
+
+__device__ __forceinline__ void put_row4(float* out, int64_t off, const float4& v, bool vec_out) {
+  if (vec_out) {
+    *reinterpret_cast<float4*>(out + off) = v;
+  } else {   // the caller's gradient buffer need not be 16-byte aligned
+    out[off] = v.x; out[off + 1] = v.y; out[off + 2] = v.z; out[off + 3] = v.w;
+  }
+}
+
+__global__ void __launch_bounds__(256) embed_bwd_kernel(int V, int d, const int* __restrict__ start,
                                                         const int* __restrict__ order,
                                                         const float* __restrict__ dx,
                                                         const float* __restrict__ dxd,
                                                         float* __restrict__ dE,
                                                         float* __restrict__ dEd, bool vec_out) {
   pdl_entry();
-  // blockIdx.y picks a slice of EB_SLICE columns, so that the rows of a frequent token
-  // (Zipf-distributed ids put hundreds of a batch's tokens on one row) are summed by several
-  // blocks at once
-  constexpr int NC = EB_SLICE / 128;    // 128-column chunks per pass
   __shared__ float4 part[2][8][32];
-  const int v = blockIdx.x;
-  const int cs0 = blockIdx.y * EB_SLICE, cs1 = min(d, cs0 + EB_SLICE);
-  const int a = start[v], cnt = start[v + 1] - a;
+  __shared__ int s_a[ID_BATCH], s_n[ID_BATCH];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int r0 = a + (w * cnt) / 8, r1 = a + ((w + 1) * cnt) / 8;
+  const int c = blockIdx.y * EB_SLICE + lane * 4;
+  const bool col = c < d;
+  const int G = gridDim.x, b = blockIdx.x;
+  const int nmine = (V - b + G - 1) / G;
   const float4 zero = make_float4(0.f, 0.f, 0.f, 0.f);
-  if (cnt == 0) {   // an id absent from the batch (most of a large vocabulary): zero rows
-    for (int c = cs0 + threadIdx.x * 4; c < cs1; c += 256 * 4) {
-      for (int which = 0; which < 2; ++which) {
-        float* out = which == 0 ? dE : dEd;
-        if (!out) continue;
-        float* dst = out + static_cast<int64_t>(v) * d + c;
-        if (vec_out) *reinterpret_cast<float4*>(dst) = zero;
-        else { dst[0] = 0.f; dst[1] = 0.f; dst[2] = 0.f; dst[3] = 0.f; }
+  for (int k0 = 0; k0 < nmine; k0 += ID_BATCH) {
+    const int nb = stage_bounds(start, b, G, k0, min(ID_BATCH, nmine - k0), s_a, s_n);
+    for (int i = w; i < nb; i += 8) {
+      const int cnt = s_n[i];
+      if (cnt > EB_WARP) continue;
+      const int a = s_a[i];
+      const int mine = lane < cnt ? order[a + lane] : 0;
+      float4 acc = zero, dacc = zero;
+      for (int t = 0; t < cnt; ++t) {
+        const int64_t ro = static_cast<int64_t>(__shfl_sync(0xffffffffu, mine, t)) * d + c;
+        if (col) {
+          add4(acc, ld4f(dx + ro));
+          if (dxd) add4(dacc, ld4f(dxd + ro));
+        }
+      }
+      if (col) {
+        const int64_t off = static_cast<int64_t>(b + (k0 + i) * G) * d + c;
+        if (dE) put_row4(dE, off, acc, vec_out);
+        if (dEd) put_row4(dEd, off, dacc, vec_out);
       }
     }
-    return;
-  }
-  for (int g0 = cs0; g0 < cs1; g0 += NC * 128) {
-    float4 acc[NC], dacc[NC];
-#pragma unroll
-    for (int q = 0; q < NC; ++q) { acc[q] = zero; dacc[q] = zero; }
-    // the row indices of 32 rows at a time, one per lane, broadcast by shuffles, so a row's
-    // loads do not wait on its index load
-    for (int kb = r0; kb < r1; kb += 32) {
-      const int mine = kb + lane < r1 ? order[kb + lane] : 0;
-      const int nb = r1 - kb < 32 ? r1 - kb : 32;
-#pragma unroll 2
-      for (int t = 0; t < nb; ++t) {
-        const int64_t ro = static_cast<int64_t>(__shfl_sync(0xffffffffu, mine, t)) * d;
-#pragma unroll
-        for (int q = 0; q < NC; ++q) {
-          const int c = g0 + q * 128 + lane * 4;
-          if (c < cs1) {
-            const float4 x = *reinterpret_cast<const float4*>(dx + ro + c);
-            acc[q].x += x.x; acc[q].y += x.y; acc[q].z += x.z; acc[q].w += x.w;
-            if (dxd) {
-              const float4 y = *reinterpret_cast<const float4*>(dxd + ro + c);
-              dacc[q].x += y.x; dacc[q].y += y.y; dacc[q].z += y.z; dacc[q].w += y.w;
-            }
+    for (int i = 0; i < nb; ++i) {
+      const int cnt = s_n[i];   // uniform across the block
+      if (cnt <= EB_WARP) continue;
+      const int a = s_a[i];
+      const int r0 = a + (w * cnt) / 8, r1 = a + ((w + 1) * cnt) / 8;
+      float4 acc = zero, dacc = zero;
+      // the row indices of 32 rows at a time, one per lane, broadcast by shuffles, so a row's
+      // loads do not wait on its index load
+      for (int kb = r0; kb < r1; kb += 32) {
+        const int mine = kb + lane < r1 ? order[kb + lane] : 0;
+        const int nr = r1 - kb < 32 ? r1 - kb : 32;
+#pragma unroll 4
+        for (int t = 0; t < nr; ++t) {
+          const int64_t ro = static_cast<int64_t>(__shfl_sync(0xffffffffu, mine, t)) * d + c;
+          if (col) {
+            add4(acc, ld4f(dx + ro));
+            if (dxd) add4(dacc, ld4f(dxd + ro));
           }
         }
       }
-    }
-#pragma unroll
-    for (int q = 0; q < NC; ++q) {
-      const int c0 = g0 + q * 128;
-      if (c0 >= cs1) break;        // uniform across the block
-      part[0][w][lane] = acc[q];
-      part[1][w][lane] = dacc[q];
+      part[0][w][lane] = acc;
+      part[1][w][lane] = dacc;
       __syncthreads();
       if (threadIdx.x < 64) {
-        const int which = threadIdx.x >> 5, l = threadIdx.x & 31, cc = c0 + l * 4;
+        const int which = threadIdx.x >> 5, l = threadIdx.x & 31;
+        const int cc = blockIdx.y * EB_SLICE + l * 4;
         float4 t = part[which][0][l];
-        for (int r = 1; r < 8; ++r) {
-          const float4 u = part[which][r][l];
-          t.x += u.x; t.y += u.y; t.z += u.z; t.w += u.w;
-        }
+        for (int r = 1; r < 8; ++r) add4(t, part[which][r][l]);
         float* out = which == 0 ? dE : dEd;
-        if (out && cc < cs1) {
-          float* dst = out + static_cast<int64_t>(v) * d + cc;
-          if (vec_out) {
-            *reinterpret_cast<float4*>(dst) = t;
-          } else {   // the caller's gradient buffer need not be 16-byte aligned
-            dst[0] = t.x; dst[1] = t.y; dst[2] = t.z; dst[3] = t.w;
-          }
-        }
+        if (out && cc < d) put_row4(out, static_cast<int64_t>(b + (k0 + i) * G) * d + cc, t, vec_out);
       }
       __syncthreads();
     }
@@ -898,7 +1058,7 @@ __global__ void cast_rows_kernel(const float* __restrict__ X, int rows, int cols
 
 int blocks_for(int64_t n) {
   int64_t b = (n + 255) / 256;
-  if (b > 152 * 16) b = 152 * 16;
+  if (b > ROW_SMS * 16) b = ROW_SMS * 16;
   return static_cast<int>(b < 1 ? 1 : b);
 }
 
@@ -928,36 +1088,45 @@ void dec_rmsnorm_fwd(int N, int d, float eps, const float* x_in, const float* y,
                                           h, hd, ldh);
 }
 
+// RMSNorm backward (dx += ...) and, when dg or dg' is wanted, the gain gradient; returns the
+// number of kernels launched.  The warp-per-row kernel writes the gain's partial sums of
+// eight rows per block itself; the block-per-row fallback takes the separate column pass.
+int dec_gain_chunks(int N) { return (N + 7) / 8; }
+
 template <typename T>
-void dec_rmsnorm_bwd(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
-                     const float* g, const float* gd, const float* dy, const float* dyd, float* dx,
-                     float* dxd, cudaStream_t s, T* dxb, T* dxdb) {
+int dec_rmsnorm_bwd(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
+                    const float* g, const float* gd, const float* dy, const float* dyd, float* dx,
+                    float* dxd, float* dg, float* dgd, float* part, cudaStream_t s, T* dxb,
+                    T* dxdb) {
+  const bool gain = dg || (dyd && dgd);
   uintptr_t any = reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(xd) |
                   reinterpret_cast<uintptr_t>(g) | reinterpret_cast<uintptr_t>(gd) |
                   reinterpret_cast<uintptr_t>(dy) | reinterpret_cast<uintptr_t>(dyd) |
                   reinterpret_cast<uintptr_t>(dx) | reinterpret_cast<uintptr_t>(dxd) |
-                  reinterpret_cast<uintptr_t>(dxb) | reinterpret_cast<uintptr_t>(dxdb);
+                  reinterpret_cast<uintptr_t>(dxb) | reinterpret_cast<uintptr_t>(dxdb) |
+                  reinterpret_cast<uintptr_t>(part);
+  const dim3 fin_grid((d + 31) / 32), fin_block(32, GF_Y);
   if ((any & 15) == 0 && (d & 3) == 0) {
-    launch_k(rmsnorm_bwd_warp_kernel<T>, dim3((N + 7) / 8), dim3(256), 0, s, N, d, x, xd, r, rd, g,
-             gd, dy, dyd, dx, dxd, dxb, dxdb);
-    return;
+    const int nblk = (N + 7) / 8;
+    float* pp = gain ? part : nullptr;
+    float* ppd = gain && dyd ? part + static_cast<int64_t>(nblk) * d : nullptr;
+    launch_k(rmsnorm_bwd_warp_kernel<T>, dim3(nblk), dim3(256), 0, s, N, d, x, xd, r, rd, g, gd,
+             dy, dyd, dx, dxd, dxb, dxdb, pp, ppd);
+    if (!gain) return 1;
+    launch_k(gain_grad_final_kernel, fin_grid, fin_block, 0, s, nblk, d,
+             static_cast<const float*>(pp), static_cast<const float*>(ppd), dg, dgd);
+    return 2;
   }
   launch_k(rmsnorm_bwd_kernel<T>, dim3(N), dim3(256), 0, s, d, x, xd, r, rd, g, gd, dy, dyd, dx, dxd,
            dxb, dxdb);
-}
-
-int dec_gain_chunks(int N) { return (N + GG_ROWS - 1) / GG_ROWS; }
-
-void dec_gain_grad(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
-                   const float* dy, const float* dyd, float* dg, float* dgd, float* part,
-                   cudaStream_t s) {
-  if (!dg && !(dyd && dgd)) return;
-  const int nchunk = dec_gain_chunks(N);
+  if (!gain) return 1;
+  const int nchunk = (N + GG_ROWS - 1) / GG_ROWS;
   float* partd = dyd ? part + static_cast<int64_t>(nchunk) * d : nullptr;
   launch_k(gain_grad_partial_kernel, dim3((d + 31) / 32, nchunk), dim3(32, 8), 0, s, N, d, x, xd,
            r, rd, dy, dyd, part, partd);
-  launch_k(gain_grad_final_kernel, dim3((d + 255) / 256), dim3(256), 0, s, nchunk, d, part, partd,
-           dg, dgd);
+  launch_k(gain_grad_final_kernel, fin_grid, fin_block, 0, s, nchunk, d,
+           static_cast<const float*>(part), static_cast<const float*>(partd), dg, dgd);
+  return 3;
 }
 
 void dec_rope_table(int S, int dh, float base, float* tab, cudaStream_t s) {
@@ -1023,17 +1192,23 @@ void dec_token_csr(int N, int S, int V, const int* ids, int* count, int* start, 
                    int* tmp, cudaStream_t s) {
   cudaMemsetAsync(count, 0, sizeof(int) * V, s);
   launch_k(token_count_kernel, dim3((N + 255) / 256), dim3(256), 0, s, N, S, V, ids, count);
-  launch_k(scan_kernel, dim3(1), dim3(1024), 0, s, V, count, start);
+  launch_k(scan_kernel, dim3(1), dim3(SCAN_THREADS), 0, s, V, count, start);
   launch_k(token_scatter_kernel, dim3((N + 255) / 256), dim3(256), 0, s, N, S, V, ids, start,
            count, tmp);
-  launch_k(token_order_kernel, dim3(V), dim3(256), 0, s, start, tmp, order);
+  // two blocks per SM, each over V / grid ids
+  launch_k(token_order_kernel, dim3(V < 2 * ROW_SMS ? V : 2 * ROW_SMS), dim3(256), 0, s, V, N,
+           start, static_cast<const int*>(tmp), order);
 }
 
 void dec_embed_bwd(int V, int d, const int* start, const int* order, const float* dx,
                    const float* dxd, float* dE, float* dEd, cudaStream_t s) {
   const bool vec_out = ((reinterpret_cast<uintptr_t>(dE) | reinterpret_cast<uintptr_t>(dEd)) & 15) == 0;
-  launch_k(embed_bwd_kernel, dim3(V, (d + EB_SLICE - 1) / EB_SLICE), dim3(256), 0, s, d, start,
-           order, dx, dxd, dE, dEd, vec_out);
+  // about eight blocks per SM over all column slices
+  const int slices = (d + EB_SLICE - 1) / EB_SLICE;
+  int gx = 8 * ROW_SMS / slices;
+  gx = gx < 1 ? 1 : gx > V ? V : gx;
+  launch_k(embed_bwd_kernel, dim3(gx, slices), dim3(256), 0, s, V, d, start, order, dx, dxd, dE,
+           dEd, vec_out);
 }
 
 template <typename T>
@@ -1045,9 +1220,10 @@ void cast_rows(const float* X, int rows, int cols, T* Y, int ldy, cudaStream_t s
   template void dec_rmsnorm_fwd<T>(int, int, float, const float*, const float*, const float*,      \
                                    const float*, const float*, const float*, float*, float*,       \
                                    float*, float*, T*, T*, int, cudaStream_t);                     \
-  template void dec_rmsnorm_bwd<T>(int, int, const float*, const float*, const float*,             \
-                                   const float*, const float*, const float*, const float*,         \
-                                   const float*, float*, float*, cudaStream_t, T*, T*);            \
+  template int dec_rmsnorm_bwd<T>(int, int, const float*, const float*, const float*,              \
+                                  const float*, const float*, const float*, const float*,          \
+                                  const float*, float*, float*, float*, float*, float*,            \
+                                  cudaStream_t, T*, T*);                                           \
   template void dec_rope_split<T>(int, int, int, int, const float*, float, const float*, T*, T*, T*,      \
                                   cudaStream_t);                                                   \
   template void dec_rope_merge<T>(int, int, int, int, const float*, float, const float*, const float*,    \

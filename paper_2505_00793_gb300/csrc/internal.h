@@ -308,16 +308,16 @@ void dec_rmsnorm_fwd(int N, int d, float eps, const float* x_in, const float* y,
                      const float* yd, const float* g, const float* gd, float* x_out, float* xd_out,
                      float* r, float* rd, T* h, T* hd, int ldh, cudaStream_t s);
 // dx (+=) the RMSNorm backward; when dxb / dxdb are given the updated dx / dx' are also
-// written in T (the next GEMM seeds), row-major [N][d].
-template <typename T>
-void dec_rmsnorm_bwd(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
-                     const float* g, const float* gd, const float* dy, const float* dyd, float* dx,
-                     float* dxd, cudaStream_t s, T* dxb = nullptr, T* dxdb = nullptr);
+// written in T (the next GEMM seeds), row-major [N][d].  When dg (or dg' with dyd) is given,
+// the gain gradient dg[j] = sum_r dy[r][j] x[r][j] r_r (and its tangent) is written too, in
+// a fixed summation order.  part: scratch of 2 * dec_gain_chunks(N) * d floats.  Returns the
+// number of kernels launched.
 int dec_gain_chunks(int N);
-// part: scratch of 2 * dec_gain_chunks(N) * d floats
-void dec_gain_grad(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
-                   const float* dy, const float* dyd, float* dg, float* dgd, float* part,
-                   cudaStream_t s);
+template <typename T>
+int dec_rmsnorm_bwd(int N, int d, const float* x, const float* xd, const float* r, const float* rd,
+                    const float* g, const float* gd, const float* dy, const float* dyd, float* dx,
+                    float* dxd, float* dg, float* dgd, float* part, cudaStream_t s,
+                    T* dxb = nullptr, T* dxdb = nullptr);
 // RoPE table [S][dh/2] of (cos, sin) pairs, float32, from double-precision angles.
 void dec_rope_table(int S, int dh, float base, float* tab, cudaStream_t s);
 template <typename T>
