@@ -7,9 +7,13 @@
 // gradient, so the weight products yield H u directly (no stored reverse graph).
 //
 // Linear layers run on the tcgen05 dual GEMM (the W1 GEMM fuses GELU and its derivatives,
-// the W2 data product fuses the GELU backward); attention scores, P V and the four
-// attention backward products run as batched dual GEMMs over batch x heads; RMSNorm,
-// RoPE, softmax and the loss are row kernels (decoder_kernels.cu).
+// the W2 data product fuses the GELU backward).  Attention runs in the fused dual attention
+// kernels (flash_tc.cu on tcgen05 for bf16 sequences of whole 128-token tiles, flash_attn.cu
+// otherwise); where those do not apply (float32 decoders, heads other than 64 wide,
+// sequences that are not whole 64-token tiles), the scores, P V and the four backward
+// products run as batched dual GEMMs over batch x heads with the softmax row kernels between
+// them.  RMSNorm, RoPE, the embedding gradient and the loss are row kernels
+// (decoder_kernels.cu).
 
 // A parameter tensor as seen by the fused update/cast kernel: rows x cols at off; the first
 // `cast` rows (0 or all) get bf16 operand copies.

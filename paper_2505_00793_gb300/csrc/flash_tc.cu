@@ -1,9 +1,9 @@
 // Fused causal attention and its forward tangent on the 5th-generation tensor cores
-// (tcgen05 + TMEM + TMA): the forward kernel of the dual attention for sequences of whole
-// 128-token tiles (flash_attn.cu holds the formulas, the backward and the warp-level kernels
-// used for other lengths).
+// (tcgen05 + TMEM + TMA) for sequences of whole 128-token tiles: the forward kernel of the
+// dual (and primal) attention, and below it the two backward kernels (flash_attn.cu holds
+// the formulas, the D / D' prep and the warp-level kernels used for other lengths).
 //
-// One CTA per (head, 128-query tile), walking 64-key tiles up to the diagonal:
+// Forward: one CTA per (head, 128-query tile), walking 64-key tiles up to the diagonal:
 //   warp 0      TMA producer: Q (and Q') once, then K, V (and K', V') per key tile into a
 //               ring of shared-memory stages (128-byte swizzle, K-major rows of 64 dims);
 //   warp 1      owns TMEM; one thread issues the MMAs:
