@@ -9,6 +9,8 @@ kernels (csrc/decoder_kernels.cu), restated on the CPU.
   longer ones through a bitmap of positions (rank = set bits below the position, with the
   words' bit counts prefix-summed by 256 threads) when the batch has at most 65536 tokens.
   Must equal a stable sort of the token ids.
+- rmsnorm_bwd_warp_kernel + gain_grad_final_kernel: every (row, column) of the gain gradient is
+  added into exactly one partial row, and every partial row read once by the final sums.
 - embed_bwd_kernel: a segment of up to 8 rows is summed by one warp in row order from zero; a
   longer one by eight warps over contiguous parts, the parts added in warp order.  For up to
   8 rows both give the same float32 bits."""
@@ -138,3 +140,31 @@ def test_short_segment_sum_matches_block_partition_bitwise():
         with np.errstate(over="ignore"):
             b, w = _block_sum(rows), _warp_sum(rows)
         assert b.tobytes() == w.tobytes(), (cnt, rows, b, w)
+
+
+@pytest.mark.parametrize("N,d", [(2048, 1024), (13, 64), (64, 1000), (9, 8), (250, 4096)])
+def test_gain_partials_cover_every_row_and_column_once(N, d):
+    """The RMSNorm backward's gain pass: block b (eight rows), warp w, lane l takes columns
+    w*128 + 4l + 1024k .. + 3 and adds rows 8b .. min(N, 8b + 8) into partial row b; the final
+    kernel's thread (x, y) of block g reads partial rows y, y + 32, ... of column 32g + x."""
+    nblk = (N + 7) // 8
+    contrib = np.zeros((N, d), np.int32)
+    written = np.zeros((nblk, d), np.int32)
+    for b in range(nblk):
+        q0, q1 = 8 * b, min(N, 8 * b + 8)
+        for w in range(8):
+            for lane in range(32):
+                for c in range(w * 128 + lane * 4, d, 1024):
+                    written[b, c:c + 4] += 1
+                    contrib[q0:q1, c:c + 4] += 1
+    assert (written == 1).all() and (contrib == 1).all()
+    read = np.zeros((nblk, d), np.int32)
+    for g in range((d + 31) // 32):
+        for x in range(32):
+            j = g * 32 + x
+            if j >= d:
+                continue
+            for y in range(32):
+                for c in range(y, nblk, 32):
+                    read[c, j] += 1
+    assert (read == 1).all()
